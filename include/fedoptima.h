@@ -1,0 +1,233 @@
+/*
+ * fedoptima.h — C ABI of the GB300 server-side hot path of FedOptima
+ * (arxiv 2504.13850).
+ *
+ * The server holds ONE copy of the server-side network M_s (theta_s, its
+ * momentum and a bf16 shadow used as tensor-core operand), a slab of
+ * `omega` activation batch slots in HBM, one FIFO of slot indices per device
+ * (Q^act_k), the consumption counters c_k and the global device-model
+ * version t.  Devices are not processes here: an upload is a call to
+ * fo_enqueue_activations, a model upload is a call to fo_aggregate.
+ *
+ * Conventions shared by every entry point
+ *   - Return value: FO_OK (0) or a positive outcome code (FO_EMPTY,
+ *     FO_FULL, FO_STALE) that leaves the server consistent, or a negative
+ *     error.  After FO_ERR_CUDA the handle may only be destroyed.
+ *   - Pointers named *_host are host memory; pointers documented as
+ *     "host or device" may be either (unified addressing decides the copy
+ *     direction).  The caller owns every buffer it passes; the library never
+ *     keeps a caller pointer beyond the call.
+ *   - All GPU work is enqueued on streams the library owns; only
+ *     fo_read_losses, fo_server_get_*, fo_server_synchronize and
+ *     fo_server_destroy wait for it.
+ *   - A handle is not thread safe: one thread drives one server.
+ *   - fo_last_error() returns a message for the last failing call on the
+ *     calling thread (empty when there is none).
+ */
+#ifndef FEDOPTIMA_H
+#define FEDOPTIMA_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define FO_API __attribute__((visibility("default")))
+#else
+#define FO_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---------------------------------------------------------------- status */
+#define FO_OK 0
+#define FO_EMPTY 1           /* no queued activation batch: nothing ran          */
+#define FO_FULL 2            /* upload refused: cap omega or ring depth reached   */
+#define FO_STALE 3           /* local model older than t - D: not aggregated      */
+#define FO_ERR_ARG (-1)      /* bad argument; nothing changed                      */
+#define FO_ERR_CUDA (-2)     /* CUDA error; the handle is no longer usable         */
+#define FO_ERR_OOM (-3)      /* device or host allocation failed                   */
+#define FO_ERR_TIMEOUT (-4)  /* a bounded device-side wait gave up                 */
+#define FO_ERR_UNSUPPORTED (-5) /* a layer shape this build has no kernel for      */
+
+/* ------------------------------------------------------------ layer spec */
+/* Op kinds of the server-side network M_s (Sec. 3.2: M is split at a layer,
+ * M_s holds the remaining layers).  Tensor 0 is the uploaded activation
+ * batch xi; op i produces tensor i + 1.  Activations are NHWC; a sequence
+ * batch [B, L, d] is carried as H = L, W = 1, C = d.  The last op's output
+ * is the logits [B, num_classes]; the server loss f_s is softmax
+ * cross-entropy averaged over the batch. */
+enum {
+  FO_OP_CONV = 1,      /* k x k (k = 1 or 3), stride 1|2, pad k/2.  params W[cout][k][k][cin], b[cout] if bias */
+  FO_OP_AFFINE = 2,    /* y = x * scale[c] + shift[c] (batch-norm folded).  params scale[c], shift[c]          */
+  FO_OP_RELU = 3,
+  FO_OP_MAXPOOL2 = 4,  /* 2x2 window, stride 2                                                                  */
+  FO_OP_ADD = 5,       /* y = in0 + in1                                                                         */
+  FO_OP_AVGPOOL = 6,   /* global mean over H, W -> [B, C]                                                        */
+  FO_OP_FLATTEN = 7,   /* [B, H, W, C] -> [B, H*W*C] in (h, w, c) order                                         */
+  FO_OP_LINEAR = 8,    /* y = x W^T + b over the last dim.  params W[cout][cin], b[cout] if bias                 */
+  FO_OP_LAYERNORM = 9, /* over the last dim, eps 1e-5, biased variance.  params gamma[c], beta[c]               */
+  FO_OP_GELU = 10,     /* exact GELU x * Phi(x)                                                                 */
+  FO_OP_ATTENTION = 11,/* in0 = [B, L, 3c] packed q|k|v; `heads` heads of c/heads; keys >= length masked          */
+  FO_OP_MEANPOOL = 12  /* mean over the first length[b] tokens: [B, L, c] -> [B, c]                              */
+};
+
+typedef struct fo_op {
+  int32_t kind;    /* FO_OP_*                                                   */
+  int32_t in0;     /* tensor id of the (first) input, 0 <= in0 <= op index     */
+  int32_t in1;     /* second input of FO_OP_ADD, else ignored                  */
+  int32_t cin;     /* conv/linear input channels; channels c of affine,
+                      layernorm and attention                                 */
+  int32_t cout;    /* conv/linear output channels                             */
+  int32_t k;       /* conv kernel size                                         */
+  int32_t stride;  /* conv stride                                              */
+  int32_t bias;    /* conv/linear: 1 if the op has a bias                      */
+  int32_t heads;   /* attention heads                                           */
+} fo_op;
+
+/* Server optimizer: SGD with momentum, v <- mu v + g, theta <- theta - lr v
+ * (Algorithm 4 training branch; v starts at 0). */
+typedef struct fo_optimizer {
+  float lr;
+  float momentum;
+} fo_optimizer;
+
+enum { FO_DTYPE_F32 = 0, FO_DTYPE_BF16 = 1 };
+enum { FO_SCHED_COUNTER = 0, FO_SCHED_FIFO = 1 };
+
+typedef struct fo_server_cfg {
+  int32_t num_devices;  /* K                                                                  */
+  int32_t omega;        /* global cap on buffered batches, sum_k |Q_k| <= omega (Sec. 3.4.1) */
+  int32_t depth;        /* per-device ring depth, |Q_k| <= depth                             */
+  int32_t batch;        /* B                                                                  */
+  int32_t in_h, in_w, in_c; /* per-sample activation shape (NHWC)                              */
+  int32_t num_classes;
+  int32_t dtype;        /* FO_DTYPE_*: uploaded activation type and compute path              */
+  int32_t seq;          /* 1: each batch carries int32 lengths[B] (attention mask, mean-pool) */
+  int32_t max_delay;    /* D of Algorithm 4                                                   */
+  int32_t sched_policy; /* FO_SCHED_COUNTER (Algorithm 3) or FO_SCHED_FIFO (arrival order)    */
+} fo_server_cfg;
+
+typedef struct fo_server fo_server;
+
+/* Create a server (initialisation stage, Sec. 3.2).  Allocates theta_s,
+ * momentum, gradient, bf16 shadow, the omega-slot activation slab (Eq. 3:
+ * memory is mu_model + omega * mu_act, independent of K) and all
+ * intermediate tensors for one batch.  Parameters start at zero: load them
+ * with fo_server_set_params.  Returns FO_ERR_UNSUPPORTED for layer shapes
+ * without a kernel (e.g. bf16 conv channels not a multiple of 64). */
+FO_API int fo_server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt,
+                     const fo_server_cfg* cfg, fo_server** out);
+FO_API int fo_server_destroy(fo_server* s);
+
+/* Number of parameters of M_s (length of the flat vector below). */
+FO_API int64_t fo_server_num_params(const fo_server* s);
+
+/* Flat parameter / momentum vectors, fp32, in op order: conv W[cout][k][k][cin]
+ * then b; linear W[cout][cin] then b; affine scale then shift; layernorm gamma
+ * then beta.  `host` is host memory of n floats; n must equal
+ * fo_server_num_params.  set_* also refreshes the bf16 shadow; get_* waits
+ * for pending steps. */
+FO_API int fo_server_set_params(fo_server* s, const float* host, int64_t n);
+FO_API int fo_server_get_params(fo_server* s, float* host, int64_t n);
+FO_API int fo_server_set_momentum(fo_server* s, const float* host, int64_t n);
+FO_API int fo_server_get_momentum(fo_server* s, float* host, int64_t n);
+
+/* Task Scheduler put() for an activation message (Algorithm 2) plus the
+ * server-side flow control of Sec. 3.4.1.  `acts` (host or device) holds
+ * B*H*W*C elements of the configured dtype, NHWC; `labels` (host or device)
+ * int32[B]; `lengths` (host or device) int32[B] when cfg.seq, else NULL.
+ * The batch is copied into a free slot before the call returns, so the
+ * caller may reuse its buffers.  *sender_on (may be NULL) receives the
+ * device's Sender Status after the call: 1 = "turn-on" was sent.
+ * FO_FULL: the cap omega or the ring depth is reached; the device is turned
+ * off and, if its queue is empty, waits in a FIFO of blocked devices.
+ * FO_ERR_ARG: bad device id or the device has left. */
+FO_API int fo_enqueue_activations(fo_server* s, int device_id, const void* acts,
+                           const int32_t* labels, const int32_t* lengths,
+                           int* sender_on);
+
+/* Task Scheduler get() (Algorithm 3, counter-based: serve argmin_k c_k over
+ * non-empty queues, ties to the lowest k, then c_k += 1) followed by one
+ * training iteration of Algorithm 4: forward of M_s, loss f_s, backward
+ * (no gradient for the uploaded activations), SGD-momentum update of
+ * theta_s.  Asynchronous: returns once the kernels are enqueued.
+ * *device_used / *slot_used (may be NULL) receive k and the slot index.
+ * FO_EMPTY when every queue is empty (nothing changes). */
+FO_API int fo_server_step(fo_server* s, int* device_used, int32_t* slot_used);
+
+/* Copy the losses of steps [first_step, first_step + n) to host memory.
+ * Waits for those steps.  Only the most recent 2^20 steps are kept. */
+FO_API int fo_read_losses(fo_server* s, float* host_out, int64_t first_step, int64_t n);
+
+/* FedAsync aggregation (Algorithm 4, aggregation branch).  `global`
+ * (device, n floats) is theta_d || theta~_d and is updated in place:
+ * global <- alpha * local + (1 - alpha) * global with
+ * alpha = 1 / (t - version + 1), computed as fmaf(alpha, local - global,
+ * global) in fp32; then t <- t + 1 and *new_version = t.  `local` (device,
+ * n floats, read only) is theta_dk || theta~_dk trained from version t_k =
+ * `version`.  FO_STALE when t - version > D (global and t unchanged).
+ * FO_ERR_ARG when version < 0 or version > t.  Runs on the server's compute
+ * stream, ordered after earlier steps. */
+FO_API int fo_aggregate(fo_server* s, float* global, const float* local, int64_t n,
+                 int device_id, int32_t version, int32_t* new_version);
+
+/* Scheduler state. */
+FO_API int fo_get_counters(const fo_server* s, uint64_t* c_host /* K */);
+FO_API int fo_get_sender_status(const fo_server* s, uint8_t* on_host /* K */);
+FO_API int fo_get_version(const fo_server* s, int32_t* t, int32_t* round /* t / K */);
+/* Device leaving (active = 0: further uploads are refused, its queued
+ * batches are still consumed) or (re)joining (active = 1: c_k becomes
+ * max(c_k, min over the other active devices), Sender on) — Sec. 3.4.2. */
+FO_API int fo_set_device_active(fo_server* s, int device_id, int active);
+
+/* Bytes of the activation slab (omega slots, acts + labels + lengths). */
+FO_API int64_t fo_server_activation_bytes(const fo_server* s);
+/* Wait for all work the server has enqueued. */
+FO_API int fo_server_synchronize(fo_server* s);
+/* The compute stream (a cudaStream_t) the step and aggregation kernels run
+ * on, for callers that time them with CUDA events. */
+FO_API void* fo_server_stream(const fo_server* s);
+/* Kernel launches the last fo_server_step enqueued. */
+FO_API int fo_server_last_step_launches(const fo_server* s);
+
+/* Optional per-kernel timing of fo_server_step: when enabled, each launch of
+ * the step is bracketed by CUDA events on the compute stream.
+ * fo_server_kernel_times fills up to `cap` entries with the name (static
+ * string), launch count and summed milliseconds of every kernel class seen
+ * since profiling was enabled (waits for the stream). */
+FO_API int fo_server_profile(fo_server* s, int enable);
+FO_API int fo_server_kernel_times(fo_server* s, const char** names, int64_t* launches,
+                           double* ms, int cap, int* n_out);
+
+FO_API const char* fo_last_error(void);
+
+/* ------------------------------------------------------------------------
+ * Host-only Task Scheduler (Algorithms 2-3 and the flow control of Sec.
+ * 3.4.1) without any GPU state: the same logic fo_server uses, for trace
+ * replay and tests.  put returns the slot the batch would occupy.
+ * ---------------------------------------------------------------------- */
+typedef struct fo_sched fo_sched;
+FO_API int fo_sched_create(int K, int omega, int depth, int policy, fo_sched** out);
+FO_API int fo_sched_destroy(fo_sched* s);
+FO_API int fo_sched_put(fo_sched* s, int k, int32_t* slot, int* sender_on);
+FO_API int fo_sched_get(fo_sched* s, int* k, int32_t* slot);
+FO_API int fo_sched_set_active(fo_sched* s, int k, int active);
+FO_API int fo_sched_counters(const fo_sched* s, uint64_t* c_host);
+FO_API int fo_sched_sender_status(const fo_sched* s, uint8_t* on_host);
+FO_API int fo_sched_queued(const fo_sched* s, int k); /* |Q_k|, or the total when k < 0 */
+
+/* ------------------------------------------------------------------------
+ * Standalone FedAsync update on caller buffers, for bandwidth sweeps:
+ * global <- fmaf(alpha, local - global, global) over n fp32 elements on
+ * `stream` (a cudaStream_t, NULL = default).  global and local are device
+ * pointers; alpha in (0, 1].  No version bookkeeping.
+ * ---------------------------------------------------------------------- */
+FO_API int fo_axpby_async(float* global, const float* local, int64_t n, float alpha,
+                   void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FEDOPTIMA_H */

@@ -1,0 +1,88 @@
+// Host launchers of the library's CUDA kernels (internal interface).
+#pragma once
+#include <cuda_runtime.h>
+#include <cstdint>
+
+namespace fo {
+
+enum DType { kF32 = 0, kBF16 = 1 };
+
+// ---- CUDA-core implicit-GEMM convolution / linear (fp32 accumulate) ----
+// A linear layer over rows is a 1x1 convolution of N = rows 1x1 images.
+struct ConvShape {
+  int N, H, W, Ci, Co, k, stride, pad, Ho, Wo;
+};
+// y = conv(x, w) + bias, optional ReLU.  x NHWC (dtype dx), w fp32
+// [Co][k][k][Ci], bias fp32 or null, y NHWC (dtype dy).
+void conv_fwd_simt(const ConvShape& s, const void* x, int dt_x, const float* w,
+                   const float* bias, void* y, int dt_y, bool relu, cudaStream_t st);
+// dx (+)= conv^T(dy, w).
+void conv_dgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const float* w,
+                     void* dx, int dt_dx, bool accumulate, cudaStream_t st);
+// dw[Co][k][k][Ci] = sum over output pixels of dy (x) x-window (fp32 out).
+void conv_wgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* x,
+                     int dt_x, float* dw, cudaStream_t st);
+
+// ---- elementwise / reductions (templated on the activation dtype) ----
+void relu_fwd(const void* x, void* y, int64_t n, int dt, cudaStream_t st);
+// dx (+)= dy * (x > 0)
+void relu_bwd(const void* x, const void* dy, void* dx, int64_t n, int dt, bool acc,
+              cudaStream_t st);
+void maxpool2_fwd(const void* x, void* y, int N, int H, int W, int C, int dt, cudaStream_t st);
+void maxpool2_bwd(const void* x, const void* dy, void* dx, int N, int H, int W, int C,
+                  int dt, bool acc, cudaStream_t st);
+// Fused backward of relu(x) followed by maxpool2: dx (+)= route(dy) * (x > 0)
+void relu_maxpool2_bwd(const void* x, const void* dy, void* dx, int N, int H, int W, int C,
+                       int dt, bool acc, cudaStream_t st);
+void affine_fwd(const void* x, const float* scale, const float* shift, void* y, int64_t rows,
+                int C, int dt, cudaStream_t st);
+// dx (+)= dy * scale (dx may be null)
+void affine_dx(const void* dy, const float* scale, void* dx, int64_t rows, int C, int dt,
+               bool acc, cudaStream_t st);
+void add_fwd(const void* a, const void* b, void* y, int64_t n, int dt, cudaStream_t st);
+// y (+)= x
+void copy_or_acc(const void* x, void* y, int64_t n, int dt, bool acc, cudaStream_t st);
+void avgpool_fwd(const void* x, void* y, int N, int HW, int C, int dt, cudaStream_t st);
+void avgpool_bwd(const void* dy, void* dx, int N, int HW, int C, int dt, bool acc,
+                 cudaStream_t st);
+void gelu_fwd(const void* x, void* y, int64_t n, int dt, cudaStream_t st);
+void gelu_bwd(const void* x, const void* dy, void* dx, int64_t n, int dt, bool acc,
+              cudaStream_t st);
+void layernorm_fwd(const void* x, const float* gamma, const float* beta, void* y,
+                   float* mean, float* rstd, int64_t rows, int C, int dt, cudaStream_t st);
+// dx (+)= layernorm input gradient (gamma/beta gradients come from colsum / colsum_lnx)
+void layernorm_bwd_dx(const void* x, const float* gamma, const float* mean, const float* rstd,
+                      const void* dy, void* dx, int64_t rows, int C, int dt, bool acc,
+                      cudaStream_t st);
+// out[c] = sum_r a[r][c] * f(r, c) where f = 1, b[r][c], or the layernorm xhat.
+// `partial` is scratch of at least colsum_partial_floats(rows, C) floats.
+int64_t colsum_partial_floats(int64_t rows, int C);
+void colsum(const void* a, const void* b, int64_t rows, int C, int dt, float* partial,
+            float* out, cudaStream_t st);
+void colsum_lnx(const void* dy, const void* x, const float* mean, const float* rstd,
+                int64_t rows, int C, int dt, float* partial, float* out, cudaStream_t st);
+void meanpool_fwd(const void* x, const int32_t* len, void* y, int B, int L, int C, int dt,
+                  cudaStream_t st);
+void meanpool_bwd(const void* dy, const int32_t* len, void* dx, int B, int L, int C, int dt,
+                  bool acc, cudaStream_t st);
+// Attention over packed qkv [B, L, 3C], heads h (C/h <= 64); probs fp32 [B,h,L,L] saved.
+void attention_fwd(const void* qkv, const int32_t* len, void* out, float* probs, int B, int L,
+                   int C, int heads, int dt, cudaStream_t st);
+void attention_bwd(const void* qkv, const int32_t* len, const float* probs, const void* out,
+                   const void* dout, void* dqkv, int B, int L, int C, int heads, int dt, bool acc,
+                   cudaStream_t st);
+
+// Softmax cross-entropy: loss_slot <- mean_b CE; dlogits = (softmax - onehot)/B.
+void softmax_ce(const float* logits, const int32_t* labels, int B, int C, float* loss_slot,
+                void* dlogits, int dt, cudaStream_t st);
+
+// SGD with momentum over a flat vector (n a multiple of 4, 16-byte aligned):
+// v = mu v + g; theta -= lr v; shadow (bf16, may be null) = bf16(theta).
+void sgd_momentum(float* theta, float* v, const float* g, void* shadow, int64_t n, float lr,
+                  float mu, cudaStream_t st);
+void f32_to_bf16(const float* x, void* y, int64_t n, cudaStream_t st);
+
+// FedAsync update: g = fmaf(alpha, l - g, g).
+void axpby(float* g, const float* l, int64_t n, float alpha, cudaStream_t st);
+
+}  // namespace fo

@@ -1,0 +1,868 @@
+// FedOptima server: C-ABI entry points, HBM activation slab, one-copy
+// server model and the step plan (forward, loss, backward, optimizer).
+//
+// Memory (Eq. 3 of the paper): one copy of theta_s (+ momentum, gradient,
+// bf16 shadow) and `omega` activation batch slots, independent of the
+// number of devices K.  Q^act_k are rings of slot indices on the host
+// (fo_sched.hpp); a slot's bytes live in the slab until the step that
+// consumes it has finished reading them (CUDA events order the reuse).
+#include "fo_server_impl.h"
+#include "fo_tc.h"
+
+#include <cstring>
+#include <functional>
+#include <map>
+#include <new>
+#include <string>
+#include <vector>
+
+namespace {
+
+thread_local std::string g_err;
+
+int set_err(int code, const std::string& msg) {
+  g_err = msg;
+  return code;
+}
+
+#define FO_CUDA(call)                                                                   \
+  do {                                                                                  \
+    cudaError_t e_ = (call);                                                            \
+    if (e_ != cudaSuccess)                                                              \
+      return set_err(FO_ERR_CUDA, std::string(#call) + ": " + cudaGetErrorString(e_)); \
+  } while (0)
+
+}  // namespace
+
+namespace {
+
+int64_t pad64(int64_t n) { return (n + 63) / 64 * 64; }
+
+// Shape inference and parameter layout.  Returns FO_OK or an error.
+int infer(fo_server* s) {
+  const fo_server_cfg& c = s->cfg;
+  int nops = int(s->ops.size());
+  s->T.assign(nops + 1, Tensor());
+  Tensor& t0 = s->T[0];
+  t0.N = c.batch;
+  t0.H = c.in_h;
+  t0.W = c.in_w;
+  t0.C = c.in_c;
+  t0.dt = s->dt;
+  t0.root = 0;
+  s->op_segs.assign(nops, {});
+  int64_t off = 0, flat = 0;
+  auto add_seg = [&](int i, int64_t n) {
+    s->op_segs[i].push_back(int(s->segs.size()));
+    s->segs.push_back({i, off, flat, n});
+    off += pad64(n);
+    flat += n;
+  };
+  for (int i = 0; i < nops; ++i) {
+    const fo_op& op = s->ops[i];
+    if (op.in0 < 0 || op.in0 > i) return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": bad in0");
+    const Tensor& a = s->T[op.in0];
+    Tensor o = a;
+    o.act = o.grad = nullptr;
+    o.root = i + 1;
+    o.consumers = 0;
+    o.dt = s->dt;
+    switch (op.kind) {
+      case FO_OP_CONV: {
+        if (a.C != op.cin || (op.k != 1 && op.k != 3) || (op.stride != 1 && op.stride != 2) || op.cout <= 0)
+          return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": bad conv");
+        int pad = op.k / 2;
+        o.H = (a.H + 2 * pad - op.k) / op.stride + 1;
+        o.W = (a.W + 2 * pad - op.k) / op.stride + 1;
+        o.C = op.cout;
+        add_seg(i, int64_t(op.cout) * op.k * op.k * op.cin);
+        if (op.bias) add_seg(i, op.cout);
+        break;
+      }
+      case FO_OP_AFFINE:
+        if (a.C != op.cin) return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": affine channels");
+        add_seg(i, op.cin);
+        add_seg(i, op.cin);
+        break;
+      case FO_OP_RELU:
+      case FO_OP_GELU:
+        break;
+      case FO_OP_MAXPOOL2:
+        if (a.H % 2 || a.W % 2) return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": maxpool odd size");
+        o.H = a.H / 2;
+        o.W = a.W / 2;
+        break;
+      case FO_OP_ADD: {
+        if (op.in1 < 0 || op.in1 > i) return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": bad in1");
+        const Tensor& b = s->T[op.in1];
+        if (b.N != a.N || b.H != a.H || b.W != a.W || b.C != a.C)
+          return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": add shapes differ");
+        break;
+      }
+      case FO_OP_AVGPOOL:
+        o.H = o.W = 1;
+        break;
+      case FO_OP_FLATTEN:
+        o.C = a.H * a.W * a.C;
+        o.H = o.W = 1;
+        o.root = s->T[op.in0].root;
+        break;
+      case FO_OP_LINEAR:
+        if (a.C != op.cin || op.cout <= 0) return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": linear cin");
+        o.C = op.cout;
+        add_seg(i, int64_t(op.cout) * op.cin);
+        if (op.bias) add_seg(i, op.cout);
+        break;
+      case FO_OP_LAYERNORM:
+        if (a.C != op.cin || a.C % 32) return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": layernorm channels");
+        add_seg(i, op.cin);
+        add_seg(i, op.cin);
+        break;
+      case FO_OP_ATTENTION:
+        if (a.C != 3 * op.cin || op.heads <= 0 || op.cin % op.heads || op.cin / op.heads > 64 ||
+            a.H > 128 || a.W != 1 || !c.seq)
+          return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": attention shape");
+        o.C = op.cin;
+        break;
+      case FO_OP_MEANPOOL:
+        if (a.W != 1 || !c.seq) return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": meanpool shape");
+        o.H = 1;
+        break;
+      default:
+        return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": unknown kind");
+    }
+    s->T[i + 1] = o;
+    s->T[op.in0].consumers++;
+    if (op.kind == FO_OP_ADD) s->T[op.in1].consumers++;
+  }
+  const fo_op& last = s->ops.back();
+  const Tensor& lt = s->T.back();
+  if (last.kind != FO_OP_LINEAR || lt.rows() != c.batch || lt.C != c.num_classes)
+    return set_err(FO_ERR_ARG, "the last op must be a linear layer producing [batch, num_classes]");
+  s->T.back().dt = fo::kF32;  // logits
+  s->n_params = flat;
+  s->n_padded = off;
+  return FO_OK;
+}
+
+float* P(fo_server* s, int op, int which) { return s->theta + s->segs[s->op_segs[op][which]].off; }
+float* G(fo_server* s, int op, int which) { return s->grad + s->segs[s->op_segs[op][which]].off; }
+const fo::bf16* SH(fo_server* s, int op, int which) { return s->shadow + s->segs[s->op_segs[op][which]].off; }
+
+fo::ConvShape conv_shape(const fo_server* s, int i) {
+  const fo_op& op = s->ops[i];
+  const Tensor& a = s->T[op.in0];
+  const Tensor& o = s->T[i + 1];
+  if (op.kind == FO_OP_LINEAR)
+    return {int(a.rows()), 1, 1, op.cin, op.cout, 1, 1, 0, 1, 1};
+  return {a.N, a.H, a.W, op.cin, op.cout, op.k, op.stride, op.k / 2, o.H, o.W};
+}
+
+// Build the list of launches of one server step.
+int build_plan(fo_server* s) {
+  const int nops = int(s->ops.size());
+  const int dt = s->dt;
+  auto& plan = s->plan;
+  plan.clear();
+  auto act = [s](int tid) -> const void* { return tid == 0 ? s->cur_in : s->T[tid].act; };
+
+  // ---------------- forward
+  for (int i = 0; i < nops; ++i) {
+    const fo_op op = s->ops[i];
+    const int a = op.in0, o = i + 1;
+    const Tensor& ta = s->T[a];
+    Tensor& to = s->T[o];
+    switch (op.kind) {
+      case FO_OP_CONV:
+      case FO_OP_LINEAR: {
+        fo::ConvShape cs = conv_shape(s, i);
+        const bool bias = op.bias != 0;
+        fo::TcGemm* tg = fo::tc_plan_forward(s->tc, s, i);
+        if (tg) {
+          plan.push_back({fo::tc_name(tg), [=](cudaStream_t st) { fo::tc_run(tg, act(a), st); }});
+        } else {
+          int dto = to.dt;
+          plan.push_back({op.kind == FO_OP_CONV ? "conv_fwd_simt" : "linear_fwd_simt",
+                          [=](cudaStream_t st) {
+                            fo::conv_fwd_simt(cs, act(a), ta.dt, P(s, i, 0), bias ? P(s, i, 1) : nullptr,
+                                              s->T[o].act, dto, false, st);
+                          }});
+        }
+        break;
+      }
+      case FO_OP_AFFINE:
+        plan.push_back({"affine_fwd", [=](cudaStream_t st) {
+                          fo::affine_fwd(act(a), P(s, i, 0), P(s, i, 1), s->T[o].act, s->T[a].rows(),
+                                         s->T[a].C, dt, st);
+                        }});
+        break;
+      case FO_OP_RELU:
+        plan.push_back({"relu_fwd", [=](cudaStream_t st) {
+                          fo::relu_fwd(act(a), s->T[o].act, s->T[a].numel(), dt, st);
+                        }});
+        break;
+      case FO_OP_MAXPOOL2:
+        plan.push_back({"maxpool2_fwd", [=](cudaStream_t st) {
+                          const Tensor& x = s->T[a];
+                          fo::maxpool2_fwd(act(a), s->T[o].act, x.N, x.H, x.W, x.C, dt, st);
+                        }});
+        break;
+      case FO_OP_ADD: {
+        const int b = op.in1;
+        plan.push_back({"add_fwd", [=](cudaStream_t st) {
+                          fo::add_fwd(act(a), act(b), s->T[o].act, s->T[o].numel(), dt, st);
+                        }});
+        break;
+      }
+      case FO_OP_AVGPOOL:
+        plan.push_back({"avgpool_fwd", [=](cudaStream_t st) {
+                          const Tensor& x = s->T[a];
+                          fo::avgpool_fwd(act(a), s->T[o].act, x.N, x.H * x.W, x.C, dt, st);
+                        }});
+        break;
+      case FO_OP_FLATTEN:
+        break;  // a view
+      case FO_OP_LAYERNORM:
+        plan.push_back({"layernorm_fwd", [=](cudaStream_t st) {
+                          fo::layernorm_fwd(act(a), P(s, i, 0), P(s, i, 1), s->T[o].act, s->ln_mean[i],
+                                            s->ln_rstd[i], s->T[a].rows(), s->T[a].C, dt, st);
+                        }});
+        break;
+      case FO_OP_GELU:
+        plan.push_back({"gelu_fwd", [=](cudaStream_t st) {
+                          fo::gelu_fwd(act(a), s->T[o].act, s->T[a].numel(), dt, st);
+                        }});
+        break;
+      case FO_OP_ATTENTION:
+        plan.push_back({"attention_fwd", [=](cudaStream_t st) {
+                          const Tensor& x = s->T[a];
+                          fo::attention_fwd(act(a), s->cur_len, s->T[o].act, s->attn_probs[i], x.N, x.H,
+                                            op.cin, op.heads, dt, st);
+                        }});
+        break;
+      case FO_OP_MEANPOOL:
+        plan.push_back({"meanpool_fwd", [=](cudaStream_t st) {
+                          const Tensor& x = s->T[a];
+                          fo::meanpool_fwd(act(a), s->cur_len, s->T[o].act, x.N, x.H, x.C, dt, st);
+                        }});
+        break;
+    }
+    (void)to;
+  }
+
+  // ---------------- loss (softmax cross-entropy on fp32 logits)
+  {
+    const int lt = nops;
+    plan.push_back({"softmax_ce", [=](cudaStream_t st) {
+                      fo::softmax_ce((const float*)s->T[lt].act, s->cur_labels, s->cfg.batch,
+                                     s->cfg.num_classes, s->losses + (s->steps_done & (s->kLossRing - 1)),
+                                     s->T[lt].grad, fo::kF32, st);
+                    }});
+  }
+
+  // ---------------- backward
+  std::vector<char> written(nops + 1, 0);
+  written[nops] = 1;  // dlogits
+  // Contribution to tensor `tid`'s gradient: returns the accumulate flag
+  // and marks the root written; tensor 0 receives none.
+  auto contrib = [&](int tid) -> int {
+    int r = s->T[tid].root;
+    int accf = written[r] ? 1 : 0;
+    written[r] = 1;
+    return accf;
+  };
+  for (int i = nops - 1; i >= 0; --i) {
+    const fo_op op = s->ops[i];
+    const int a = op.in0, o = i + 1;
+    const int ro = s->T[o].root;
+    if (!written[ro]) {
+      // Nothing downstream produced a gradient: zero this op's parameter grads.
+      for (int si : s->op_segs[i]) {
+        const ParamSeg seg = s->segs[si];
+        plan.push_back({"memset_grad", [=](cudaStream_t st) {
+                          cudaMemsetAsync(s->grad + seg.off, 0, seg.n * sizeof(float), st);
+                        }});
+      }
+      continue;
+    }
+    const bool need_dx = a != 0;
+    switch (op.kind) {
+      case FO_OP_CONV:
+      case FO_OP_LINEAR: {
+        fo::ConvShape cs = conv_shape(s, i);
+        const int dto = s->T[o].dt, dta = s->T[a].dt;
+        const bool bias = op.bias != 0;
+        if (bias) {
+          plan.push_back({"bias_grad", [=](cudaStream_t st) {
+                            fo::colsum(s->T[o].grad, nullptr, s->T[o].rows(), s->T[o].C, dto,
+                                       s->colsum_scratch, G(s, i, 1), st);
+                          }});
+        }
+        if (need_dx) {
+          int accf = contrib(a);
+          fo::TcGemm* tg = fo::tc_plan_dgrad(s->tc, s, i, accf);
+          if (tg) {
+            plan.push_back({fo::tc_name(tg), [=](cudaStream_t st) { fo::tc_run(tg, nullptr, st); }});
+          } else {
+            plan.push_back({op.kind == FO_OP_CONV ? "conv_dgrad_simt" : "linear_dgrad_simt",
+                            [=](cudaStream_t st) {
+                              fo::conv_dgrad_simt(cs, s->T[o].grad, dto, P(s, i, 0), s->T[a].grad, dta,
+                                                  accf != 0, st);
+                            }});
+          }
+        }
+        fo::TcGemm* tw = fo::tc_plan_wgrad(s->tc, s, i);
+        if (tw) {
+          plan.push_back({fo::tc_name(tw), [=](cudaStream_t st) { fo::tc_run(tw, act(a), st); }});
+        } else {
+          plan.push_back({op.kind == FO_OP_CONV ? "conv_wgrad_simt" : "linear_wgrad_simt",
+                          [=](cudaStream_t st) {
+                            fo::conv_wgrad_simt(cs, s->T[o].grad, dto, act(a), dta, G(s, i, 0), st);
+                          }});
+        }
+        break;
+      }
+      case FO_OP_AFFINE:
+        plan.push_back({"affine_pgrad", [=](cudaStream_t st) {
+                          const Tensor& x = s->T[a];
+                          fo::colsum(s->T[o].grad, act(a), x.rows(), x.C, dt, s->colsum_scratch, G(s, i, 0), st);
+                          fo::colsum(s->T[o].grad, nullptr, x.rows(), x.C, dt, s->colsum_scratch, G(s, i, 1), st);
+                        }});
+        if (need_dx) {
+          int accf = contrib(a);
+          plan.push_back({"affine_dx", [=](cudaStream_t st) {
+                            fo::affine_dx(s->T[o].grad, P(s, i, 0), s->T[a].grad, s->T[a].rows(), s->T[a].C,
+                                          dt, accf != 0, st);
+                          }});
+        }
+        break;
+      case FO_OP_RELU:
+        if (need_dx) {
+          int accf = contrib(a);
+          plan.push_back({"relu_bwd", [=](cudaStream_t st) {
+                            fo::relu_bwd(act(a), s->T[o].grad, s->T[a].grad, s->T[a].numel(), dt, accf != 0, st);
+                          }});
+        }
+        break;
+      case FO_OP_MAXPOOL2:
+        if (need_dx) {
+          int accf = contrib(a);
+          plan.push_back({"maxpool2_bwd", [=](cudaStream_t st) {
+                            const Tensor& x = s->T[a];
+                            fo::maxpool2_bwd(act(a), s->T[o].grad, x.grad, x.N, x.H, x.W, x.C, dt, accf != 0, st);
+                          }});
+        }
+        break;
+      case FO_OP_ADD: {
+        const int b = op.in1;
+        for (int src : {a, b}) {
+          if (src == 0) continue;
+          int accf = contrib(src);
+          plan.push_back({"add_bwd", [=](cudaStream_t st) {
+                            fo::copy_or_acc(s->T[o].grad, s->T[src].grad, s->T[o].numel(), dt, accf != 0, st);
+                          }});
+        }
+        break;
+      }
+      case FO_OP_AVGPOOL:
+        if (need_dx) {
+          int accf = contrib(a);
+          plan.push_back({"avgpool_bwd", [=](cudaStream_t st) {
+                            const Tensor& x = s->T[a];
+                            fo::avgpool_bwd(s->T[o].grad, x.grad, x.N, x.H * x.W, x.C, dt, accf != 0, st);
+                          }});
+        }
+        break;
+      case FO_OP_FLATTEN:
+        break;  // shares the input's gradient buffer
+      case FO_OP_LAYERNORM:
+        plan.push_back({"layernorm_pgrad", [=](cudaStream_t st) {
+                          const Tensor& x = s->T[a];
+                          fo::colsum_lnx(s->T[o].grad, act(a), s->ln_mean[i], s->ln_rstd[i], x.rows(), x.C, dt,
+                                         s->colsum_scratch, G(s, i, 0), st);
+                          fo::colsum(s->T[o].grad, nullptr, x.rows(), x.C, dt, s->colsum_scratch, G(s, i, 1), st);
+                        }});
+        if (need_dx) {
+          int accf = contrib(a);
+          plan.push_back({"layernorm_bwd", [=](cudaStream_t st) {
+                            const Tensor& x = s->T[a];
+                            fo::layernorm_bwd_dx(act(a), P(s, i, 0), s->ln_mean[i], s->ln_rstd[i], s->T[o].grad,
+                                                 x.grad, x.rows(), x.C, dt, accf != 0, st);
+                          }});
+        }
+        break;
+      case FO_OP_GELU:
+        if (need_dx) {
+          int accf = contrib(a);
+          plan.push_back({"gelu_bwd", [=](cudaStream_t st) {
+                            fo::gelu_bwd(act(a), s->T[o].grad, s->T[a].grad, s->T[a].numel(), dt, accf != 0, st);
+                          }});
+        }
+        break;
+      case FO_OP_ATTENTION:
+        if (need_dx) {
+          int accf = contrib(a);
+          plan.push_back({"attention_bwd", [=](cudaStream_t st) {
+                            const Tensor& x = s->T[a];
+                            fo::attention_bwd(act(a), s->cur_len, s->attn_probs[i], s->T[o].act, s->T[o].grad,
+                                              x.grad, x.N, x.H, op.cin, op.heads, dt, accf != 0, st);
+                          }});
+        }
+        break;
+      case FO_OP_MEANPOOL:
+        if (need_dx) {
+          int accf = contrib(a);
+          plan.push_back({"meanpool_bwd", [=](cudaStream_t st) {
+                            const Tensor& x = s->T[a];
+                            fo::meanpool_bwd(s->T[o].grad, s->cur_len, x.grad, x.N, x.H, x.C, dt, accf != 0, st);
+                          }});
+        }
+        break;
+    }
+  }
+
+  // ---------------- optimizer (Algorithm 4: theta_s <- theta_s - gamma_s * update)
+  plan.push_back({"sgd_momentum", [=](cudaStream_t st) {
+                    fo::sgd_momentum(s->theta, s->mom, s->grad, s->shadow, s->n_padded, s->opt.lr,
+                                     s->opt.momentum, st);
+                  }});
+  return FO_OK;
+}
+
+int allocate(fo_server* s) {
+  const fo_server_cfg& c = s->cfg;
+  size_t esz = s->dt == fo::kF32 ? 4 : 2;
+  // parameters
+  s->theta = (float*)s->alloc(s->n_padded * 4);
+  s->mom = (float*)s->alloc(s->n_padded * 4);
+  s->grad = (float*)s->alloc(s->n_padded * 4);
+  if (!s->theta || !s->mom || !s->grad) return set_err(FO_ERR_OOM, "parameter allocation");
+  FO_CUDA(cudaMemset(s->theta, 0, s->n_padded * 4));
+  FO_CUDA(cudaMemset(s->mom, 0, s->n_padded * 4));
+  FO_CUDA(cudaMemset(s->grad, 0, s->n_padded * 4));
+  if (s->dt == fo::kBF16) {
+    s->shadow = (fo::bf16*)s->alloc(s->n_padded * 2);
+    if (!s->shadow) return set_err(FO_ERR_OOM, "shadow allocation");
+    FO_CUDA(cudaMemset(s->shadow, 0, s->n_padded * 2));
+  }
+  // activation slab: omega slots (Eq. 3), 256-byte aligned each
+  s->slot_act_bytes = int64_t(c.batch) * c.in_h * c.in_w * c.in_c * esz;
+  s->slot_stride = (s->slot_act_bytes + 255) / 256 * 256;
+  s->slab = (char*)s->alloc(size_t(s->slot_stride) * c.omega);
+  s->slot_labels = (int32_t*)s->alloc(size_t(c.omega) * c.batch * 4);
+  s->slot_lengths = (int32_t*)s->alloc(size_t(c.omega) * c.batch * 4);
+  if (!s->slab || !s->slot_labels || !s->slot_lengths) return set_err(FO_ERR_OOM, "activation slab");
+  s->slot_ready.assign(c.omega, nullptr);
+  s->slot_free.assign(c.omega, nullptr);
+  s->slot_consumed.assign(c.omega, 0);
+  for (int i = 0; i < c.omega; ++i) {
+    FO_CUDA(cudaEventCreateWithFlags(&s->slot_ready[i], cudaEventDisableTiming));
+    FO_CUDA(cudaEventCreateWithFlags(&s->slot_free[i], cudaEventDisableTiming));
+  }
+  // tensors
+  int nops = int(s->ops.size());
+  for (int tid = 1; tid <= nops; ++tid) {
+    Tensor& t = s->T[tid];
+    if (t.root != tid) continue;
+    t.act = s->alloc(t.bytes());
+    t.grad = s->alloc(t.bytes());
+    if (!t.act || !t.grad) return set_err(FO_ERR_OOM, "tensor allocation");
+  }
+  for (int tid = 1; tid <= nops; ++tid) {
+    Tensor& t = s->T[tid];
+    if (t.root != tid) {
+      t.act = s->T[t.root].act;
+      t.grad = s->T[t.root].grad;
+    }
+  }
+  // scratch for deterministic column sums
+  int64_t cs_floats = 1;
+  for (int i = 0; i < nops; ++i) {
+    const Tensor& o = s->T[i + 1];
+    const Tensor& a = s->T[s->ops[i].in0];
+    cs_floats = std::max(cs_floats, fo::colsum_partial_floats(o.rows(), o.C));
+    cs_floats = std::max(cs_floats, fo::colsum_partial_floats(a.rows(), a.C));
+  }
+  s->colsum_scratch = (float*)s->alloc(cs_floats * 4);
+  s->ln_mean.assign(nops, nullptr);
+  s->ln_rstd.assign(nops, nullptr);
+  s->attn_probs.assign(nops, nullptr);
+  for (int i = 0; i < nops; ++i) {
+    const fo_op& op = s->ops[i];
+    const Tensor& a = s->T[op.in0];
+    if (op.kind == FO_OP_LAYERNORM) {
+      s->ln_mean[i] = (float*)s->alloc(a.rows() * 4);
+      s->ln_rstd[i] = (float*)s->alloc(a.rows() * 4);
+    } else if (op.kind == FO_OP_ATTENTION) {
+      s->attn_probs[i] = (float*)s->alloc(size_t(a.N) * op.heads * a.H * a.H * 4);
+    }
+  }
+  s->losses = (float*)s->alloc(size_t(s->kLossRing) * 4);
+  if (!s->colsum_scratch || !s->losses) return set_err(FO_ERR_OOM, "scratch allocation");
+  FO_CUDA(cudaMemset(s->losses, 0, size_t(s->kLossRing) * 4));
+  return FO_OK;
+}
+
+void destroy_impl(fo_server* s) {
+  if (!s) return;
+  if (s->cs) cudaStreamSynchronize(s->cs);
+  if (s->xs) cudaStreamSynchronize(s->xs);
+  fo::tc_destroy(s->tc);
+  for (auto e : s->slot_ready) if (e) cudaEventDestroy(e);
+  for (auto e : s->slot_free) if (e) cudaEventDestroy(e);
+  for (auto& r : s->prof) {
+    cudaEventDestroy(r.a);
+    cudaEventDestroy(r.b);
+  }
+  for (auto e : s->ev_pool) cudaEventDestroy(e);
+  for (void* p : s->allocs) cudaFree(p);
+  if (s->cs) cudaStreamDestroy(s->cs);
+  if (s->xs) cudaStreamDestroy(s->xs);
+  delete s->sched;
+  delete s;
+}
+
+cudaEvent_t pool_event(fo_server* s) {
+  if (!s->ev_pool.empty()) {
+    cudaEvent_t e = s->ev_pool.back();
+    s->ev_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+}  // namespace
+
+// ===================================================================== C ABI
+
+extern "C" {
+
+const char* fo_last_error(void) { return g_err.c_str(); }
+
+int fo_server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt, const fo_server_cfg* cfg,
+                     fo_server** out) {
+  g_err.clear();
+  if (!ops || n_ops <= 0 || !opt || !cfg || !out) return set_err(FO_ERR_ARG, "null argument");
+  *out = nullptr;
+  const fo_server_cfg& c = *cfg;
+  if (c.num_devices <= 0 || c.omega <= 0 || c.depth <= 0 || c.batch <= 0 || c.batch > 1024 ||
+      c.in_h <= 0 || c.in_w <= 0 || c.in_c <= 0 || c.num_classes <= 0 ||
+      (c.dtype != FO_DTYPE_F32 && c.dtype != FO_DTYPE_BF16) || c.max_delay < 0 ||
+      (c.sched_policy != FO_SCHED_COUNTER && c.sched_policy != FO_SCHED_FIFO))
+    return set_err(FO_ERR_ARG, "bad server configuration");
+  fo_server* s = new (std::nothrow) fo_server();
+  if (!s) return set_err(FO_ERR_OOM, "host allocation");
+  s->cfg = c;
+  s->opt = *opt;
+  s->dt = c.dtype == FO_DTYPE_F32 ? fo::kF32 : fo::kBF16;
+  s->ops.assign(ops, ops + n_ops);
+  int rc = infer(s);
+  if (rc != FO_OK) {
+    destroy_impl(s);
+    return rc;
+  }
+  s->sched = new fo::TaskScheduler(c.num_devices, c.omega, c.depth, c.sched_policy);
+  if (cudaStreamCreateWithFlags(&s->cs, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&s->xs, cudaStreamNonBlocking) != cudaSuccess) {
+    destroy_impl(s);
+    return set_err(FO_ERR_CUDA, "stream creation");
+  }
+  rc = allocate(s);
+  if (rc == FO_OK) rc = fo::tc_create(&s->tc, s);
+  if (rc == FO_OK) rc = build_plan(s);
+  if (rc == FO_OK && cudaDeviceSynchronize() != cudaSuccess) rc = set_err(FO_ERR_CUDA, "create sync");
+  if (rc != FO_OK) {
+    destroy_impl(s);
+    return rc;
+  }
+  *out = s;
+  return FO_OK;
+}
+
+int fo_server_destroy(fo_server* s) {
+  destroy_impl(s);
+  return FO_OK;
+}
+
+int64_t fo_server_num_params(const fo_server* s) { return s ? s->n_params : -1; }
+
+static int copy_params(fo_server* s, float* dev, const float* host, float* host_out, int64_t n) {
+  if (!s || n != s->n_params || (!host && !host_out)) return set_err(FO_ERR_ARG, "bad parameter vector");
+  FO_CUDA(cudaStreamSynchronize(s->cs));
+  for (const ParamSeg& g : s->segs) {
+    if (host) FO_CUDA(cudaMemcpy(dev + g.off, host + g.flat, g.n * 4, cudaMemcpyHostToDevice));
+    else FO_CUDA(cudaMemcpy(host_out + g.flat, dev + g.off, g.n * 4, cudaMemcpyDeviceToHost));
+  }
+  return FO_OK;
+}
+
+int fo_server_set_params(fo_server* s, const float* host, int64_t n) {
+  int rc = copy_params(s, s ? s->theta : nullptr, host, nullptr, n);
+  if (rc != FO_OK) return rc;
+  if (s->shadow) {
+    fo::f32_to_bf16(s->theta, s->shadow, s->n_padded, s->cs);
+    FO_CUDA(cudaStreamSynchronize(s->cs));
+  }
+  return FO_OK;
+}
+int fo_server_get_params(fo_server* s, float* host, int64_t n) {
+  return copy_params(s, s ? s->theta : nullptr, nullptr, host, n);
+}
+int fo_server_set_momentum(fo_server* s, const float* host, int64_t n) {
+  return copy_params(s, s ? s->mom : nullptr, host, nullptr, n);
+}
+int fo_server_get_momentum(fo_server* s, float* host, int64_t n) {
+  return copy_params(s, s ? s->mom : nullptr, nullptr, host, n);
+}
+
+int fo_enqueue_activations(fo_server* s, int device_id, const void* acts, const int32_t* labels,
+                           const int32_t* lengths, int* sender_on) {
+  if (!s || !acts || !labels) return set_err(FO_ERR_ARG, "null argument");
+  if (s->cfg.seq && !lengths) return set_err(FO_ERR_ARG, "lengths required for sequence batches");
+  if (device_id < 0 || device_id >= s->cfg.num_devices) return set_err(FO_ERR_ARG, "bad device id");
+  int32_t slot = -1;
+  int rc = s->sched->put(device_id, &slot);
+  if (sender_on) *sender_on = s->sched->sender_on()[device_id];
+  if (rc == -1) return set_err(FO_ERR_ARG, "device has left");
+  if (rc == 2) return FO_FULL;
+  const int B = s->cfg.batch;
+  if (s->slot_consumed[slot]) FO_CUDA(cudaStreamWaitEvent(s->xs, s->slot_free[slot], 0));
+  FO_CUDA(cudaMemcpyAsync(s->slab + size_t(slot) * s->slot_stride, acts, s->slot_act_bytes,
+                          cudaMemcpyDefault, s->xs));
+  FO_CUDA(cudaMemcpyAsync(s->slot_labels + size_t(slot) * B, labels, B * 4, cudaMemcpyDefault, s->xs));
+  if (lengths)
+    FO_CUDA(cudaMemcpyAsync(s->slot_lengths + size_t(slot) * B, lengths, B * 4, cudaMemcpyDefault, s->xs));
+  FO_CUDA(cudaEventRecord(s->slot_ready[slot], s->xs));
+  // The caller may reuse its buffers once the call returns.
+  FO_CUDA(cudaEventSynchronize(s->slot_ready[slot]));
+  return FO_OK;
+}
+
+int fo_server_step(fo_server* s, int* device_used, int32_t* slot_used) {
+  if (!s) return set_err(FO_ERR_ARG, "null server");
+  int k = -1;
+  int32_t slot = -1;
+  if (s->sched->get(&k, &slot) != 0) {
+    if (device_used) *device_used = -1;
+    if (slot_used) *slot_used = -1;
+    s->last_launches = 0;
+    return FO_EMPTY;
+  }
+  if (device_used) *device_used = k;
+  if (slot_used) *slot_used = slot;
+  const int B = s->cfg.batch;
+  s->cur_in = s->slab + size_t(slot) * s->slot_stride;
+  s->cur_labels = s->slot_labels + size_t(slot) * B;
+  s->cur_len = s->slot_lengths + size_t(slot) * B;
+  fo::tc_set_input(s->tc, slot);
+  FO_CUDA(cudaStreamWaitEvent(s->cs, s->slot_ready[slot], 0));
+  int n = 0;
+  for (const Launch& l : s->plan) {
+    if (s->profiling) {
+      ProfRec r;
+      r.a = pool_event(s);
+      r.b = pool_event(s);
+      int id = -1;
+      for (size_t q = 0; q < s->prof_names.size(); ++q)
+        if (s->prof_names[q] == l.name) id = int(q);
+      if (id < 0) {
+        id = int(s->prof_names.size());
+        s->prof_names.push_back(l.name);
+      }
+      r.name_id = id;
+      cudaEventRecord(r.a, s->cs);
+      l.fn(s->cs);
+      cudaEventRecord(r.b, s->cs);
+      s->prof.push_back(r);
+    } else {
+      l.fn(s->cs);
+    }
+    ++n;
+  }
+  FO_CUDA(cudaGetLastError());
+  FO_CUDA(cudaEventRecord(s->slot_free[slot], s->cs));
+  s->slot_consumed[slot] = 1;
+  s->steps_done++;
+  s->last_launches = n;
+  return FO_OK;
+}
+
+int fo_read_losses(fo_server* s, float* host_out, int64_t first_step, int64_t n) {
+  if (!s || !host_out || first_step < 0 || n < 0 || first_step + n > s->steps_done ||
+      s->steps_done - first_step > s->kLossRing)
+    return set_err(FO_ERR_ARG, "loss range");
+  FO_CUDA(cudaStreamSynchronize(s->cs));
+  for (int64_t i = 0; i < n; ++i) {
+    int64_t idx = (first_step + i) & (s->kLossRing - 1);
+    FO_CUDA(cudaMemcpy(host_out + i, s->losses + idx, 4, cudaMemcpyDeviceToHost));
+  }
+  return FO_OK;
+}
+
+int fo_aggregate(fo_server* s, float* global, const float* local, int64_t n, int device_id,
+                 int32_t version, int32_t* new_version) {
+  if (!s || !global || !local || n < 0) return set_err(FO_ERR_ARG, "null argument");
+  if (device_id < 0 || device_id >= s->cfg.num_devices) return set_err(FO_ERR_ARG, "bad device id");
+  if (version < 0 || version > s->t) return set_err(FO_ERR_ARG, "model version out of range");
+  if (int64_t(s->t) - version > s->cfg.max_delay) {
+    if (new_version) *new_version = s->t;
+    return FO_STALE;
+  }
+  float alpha = 1.0f / float(s->t - version + 1);
+  if (s->profiling) {
+    ProfRec r{0, pool_event(s), pool_event(s)};
+    int id = -1;
+    for (size_t q = 0; q < s->prof_names.size(); ++q)
+      if (std::strcmp(s->prof_names[q], "fedasync_axpby") == 0) id = int(q);
+    if (id < 0) {
+      id = int(s->prof_names.size());
+      s->prof_names.push_back("fedasync_axpby");
+    }
+    r.name_id = id;
+    cudaEventRecord(r.a, s->cs);
+    fo::axpby(global, local, n, alpha, s->cs);
+    cudaEventRecord(r.b, s->cs);
+    s->prof.push_back(r);
+  } else {
+    fo::axpby(global, local, n, alpha, s->cs);
+  }
+  FO_CUDA(cudaGetLastError());
+  s->t += 1;
+  if (new_version) *new_version = s->t;
+  return FO_OK;
+}
+
+int fo_get_counters(const fo_server* s, uint64_t* c) {
+  if (!s || !c) return set_err(FO_ERR_ARG, "null argument");
+  const auto& v = s->sched->counters();
+  for (size_t i = 0; i < v.size(); ++i) c[i] = v[i];
+  return FO_OK;
+}
+int fo_get_sender_status(const fo_server* s, uint8_t* on) {
+  if (!s || !on) return set_err(FO_ERR_ARG, "null argument");
+  const auto& v = s->sched->sender_on();
+  for (size_t i = 0; i < v.size(); ++i) on[i] = v[i];
+  return FO_OK;
+}
+int fo_get_version(const fo_server* s, int32_t* t, int32_t* round) {
+  if (!s) return set_err(FO_ERR_ARG, "null server");
+  if (t) *t = s->t;
+  if (round) *round = s->t / s->cfg.num_devices;
+  return FO_OK;
+}
+int fo_set_device_active(fo_server* s, int device_id, int active) {
+  if (!s) return set_err(FO_ERR_ARG, "null server");
+  return s->sched->set_active(device_id, active) == 0 ? FO_OK : set_err(FO_ERR_ARG, "bad device id");
+}
+int64_t fo_server_activation_bytes(const fo_server* s) {
+  if (!s) return -1;
+  return int64_t(s->cfg.omega) * (s->slot_stride + 2 * int64_t(s->cfg.batch) * 4);
+}
+int fo_server_synchronize(fo_server* s) {
+  if (!s) return set_err(FO_ERR_ARG, "null server");
+  FO_CUDA(cudaStreamSynchronize(s->xs));
+  FO_CUDA(cudaStreamSynchronize(s->cs));
+  return FO_OK;
+}
+void* fo_server_stream(const fo_server* s) { return s ? (void*)s->cs : nullptr; }
+int fo_server_last_step_launches(const fo_server* s) { return s ? s->last_launches : -1; }
+
+int fo_server_profile(fo_server* s, int enable) {
+  if (!s) return set_err(FO_ERR_ARG, "null server");
+  s->profiling = enable != 0;
+  return FO_OK;
+}
+
+int fo_server_kernel_times(fo_server* s, const char** names, int64_t* launches, double* ms, int cap,
+                           int* n_out) {
+  if (!s || !n_out) return set_err(FO_ERR_ARG, "null argument");
+  FO_CUDA(cudaStreamSynchronize(s->cs));
+  for (auto& r : s->prof) {
+    float t = 0.f;
+    cudaEventElapsedTime(&t, r.a, r.b);
+    auto& acc = s->prof_acc[s->prof_names[r.name_id]];
+    acc.first += 1;
+    acc.second += t;
+    s->ev_pool.push_back(r.a);
+    s->ev_pool.push_back(r.b);
+  }
+  s->prof.clear();
+  int n = 0;
+  for (auto& kv : s->prof_acc) {
+    if (n < cap) {
+      if (names) names[n] = kv.first;
+      if (launches) launches[n] = kv.second.first;
+      if (ms) ms[n] = kv.second.second;
+    }
+    ++n;
+  }
+  *n_out = n;
+  return FO_OK;
+}
+
+int fo_axpby_async(float* global, const float* local, int64_t n, float alpha, void* stream) {
+  if (!global || !local || n < 0 || !(alpha > 0.f) || alpha > 1.f) return set_err(FO_ERR_ARG, "bad argument");
+  fo::axpby(global, local, n, alpha, (cudaStream_t)stream);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return set_err(FO_ERR_CUDA, cudaGetErrorString(e));
+  return FO_OK;
+}
+
+// ------------------------------------------------------ host-only scheduler
+struct fo_sched {
+  fo::TaskScheduler* s;
+};
+
+int fo_sched_create(int K, int omega, int depth, int policy, fo_sched** out) {
+  if (!out || K <= 0 || omega <= 0 || depth <= 0 || (policy != FO_SCHED_COUNTER && policy != FO_SCHED_FIFO))
+    return set_err(FO_ERR_ARG, "bad scheduler configuration");
+  *out = new fo_sched{new fo::TaskScheduler(K, omega, depth, policy)};
+  return FO_OK;
+}
+int fo_sched_destroy(fo_sched* s) {
+  if (s) {
+    delete s->s;
+    delete s;
+  }
+  return FO_OK;
+}
+int fo_sched_put(fo_sched* s, int k, int32_t* slot, int* sender_on) {
+  if (!s || !slot) return set_err(FO_ERR_ARG, "null argument");
+  *slot = -1;
+  if (k < 0 || k >= s->s->K()) return set_err(FO_ERR_ARG, "bad device id");
+  int rc = s->s->put(k, slot);
+  if (sender_on) *sender_on = s->s->sender_on()[k];
+  return rc == -1 ? set_err(FO_ERR_ARG, "device has left") : (rc == 2 ? FO_FULL : FO_OK);
+}
+int fo_sched_get(fo_sched* s, int* k, int32_t* slot) {
+  if (!s || !k || !slot) return set_err(FO_ERR_ARG, "null argument");
+  *k = -1;
+  *slot = -1;
+  return s->s->get(k, slot) == 0 ? FO_OK : FO_EMPTY;
+}
+int fo_sched_set_active(fo_sched* s, int k, int active) {
+  if (!s) return set_err(FO_ERR_ARG, "null argument");
+  return s->s->set_active(k, active) == 0 ? FO_OK : set_err(FO_ERR_ARG, "bad device id");
+}
+int fo_sched_counters(const fo_sched* s, uint64_t* c) {
+  if (!s || !c) return set_err(FO_ERR_ARG, "null argument");
+  const auto& v = s->s->counters();
+  for (size_t i = 0; i < v.size(); ++i) c[i] = v[i];
+  return FO_OK;
+}
+int fo_sched_sender_status(const fo_sched* s, uint8_t* on) {
+  if (!s || !on) return set_err(FO_ERR_ARG, "null argument");
+  const auto& v = s->s->sender_on();
+  for (size_t i = 0; i < v.size(); ++i) on[i] = v[i];
+  return FO_OK;
+}
+int fo_sched_queued(const fo_sched* s, int k) {
+  if (!s) return -1;
+  if (k < 0) return s->s->queued_total();
+  if (k >= s->s->K()) return -1;
+  return s->s->queued(k);
+}
+
+}  // extern "C"

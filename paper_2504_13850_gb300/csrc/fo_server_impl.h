@@ -1,0 +1,102 @@
+// Internal state of a FedOptima server (shared by the plan builder and the
+// tensor-core planner).
+#pragma once
+#include "fo_common.cuh"
+#include "fo_kernels.h"
+#include "fo_sched.hpp"
+#include "../../include/fedoptima.h"
+
+#include <functional>
+#include <map>
+#include <string>
+#include <vector>
+
+namespace fo {
+struct TcContext;
+}
+
+struct ParamSeg {
+  int op;
+  int64_t off;   // offset in the padded device vector
+  int64_t flat;  // offset in the caller's flat vector
+  int64_t n;
+};
+
+struct Tensor {
+  int N = 0, H = 0, W = 0, C = 0;
+  int dt = fo::kF32;
+  void* act = nullptr;
+  void* grad = nullptr;
+  int root = -1;        // tensor whose buffers this one aliases (flatten), else itself
+  int consumers = 0;
+  int64_t rows() const { return int64_t(N) * H * W; }
+  int64_t numel() const { return rows() * C; }
+  size_t bytes() const { return size_t(numel()) * (dt == fo::kF32 ? 4 : 2); }
+};
+
+struct Launch {
+  const char* name;
+  std::function<void(cudaStream_t)> fn;
+};
+
+struct ProfRec {
+  int name_id;
+  cudaEvent_t a, b;
+};
+
+struct fo_server {
+  fo_server_cfg cfg{};
+  fo_optimizer opt{};
+  std::vector<fo_op> ops;
+  fo::TaskScheduler* sched = nullptr;
+  cudaStream_t cs = nullptr, xs = nullptr;
+  int dt = fo::kF32;
+
+  int64_t n_params = 0, n_padded = 0;
+  std::vector<ParamSeg> segs;
+  std::vector<std::vector<int>> op_segs;  // per op: indices into segs
+  float *theta = nullptr, *mom = nullptr, *grad = nullptr;
+  fo::bf16* shadow = nullptr;
+
+  int64_t slot_act_bytes = 0, slot_stride = 0;
+  char* slab = nullptr;
+  int32_t* slot_labels = nullptr;
+  int32_t* slot_lengths = nullptr;
+  std::vector<cudaEvent_t> slot_ready, slot_free;
+  std::vector<char> slot_consumed;
+
+  std::vector<Tensor> T;
+  float* colsum_scratch = nullptr;
+  std::vector<float*> ln_mean, ln_rstd, attn_probs;
+
+  const void* cur_in = nullptr;
+  const int32_t* cur_labels = nullptr;
+  const int32_t* cur_len = nullptr;
+  float* losses = nullptr;
+  int64_t steps_done = 0;
+  static constexpr int64_t kLossRing = int64_t(1) << 20;
+
+  std::vector<Launch> plan;
+  int last_launches = 0;
+
+  int32_t t = 0;
+
+  bool profiling = false;
+  std::vector<ProfRec> prof;
+  std::vector<cudaEvent_t> ev_pool;
+  std::vector<const char*> prof_names;
+  std::map<const char*, std::pair<int64_t, double>> prof_acc;
+
+  std::vector<void*> allocs;
+  fo::TcContext* tc = nullptr;
+
+  void* alloc(size_t bytes) {
+    void* p = nullptr;
+    if (bytes == 0) bytes = 256;
+    if (cudaMalloc(&p, bytes) != cudaSuccess) return nullptr;
+    allocs.push_back(p);
+    return p;
+  }
+  int op_of_tensor(int tid) const { return tid - 1; }
+};
+

@@ -1,0 +1,25 @@
+// Tensor-core (tcgen05 / TMEM / TMA) GEMM and implicit-GEMM convolution
+// planner for the bf16 compute path.  The plan functions return nullptr for
+// shapes the tensor-core kernels do not take; the caller then uses the
+// CUDA-core kernels.
+#pragma once
+#include <cuda_runtime.h>
+
+struct fo_server;
+
+namespace fo {
+
+struct TcContext;
+struct TcGemm;
+
+int tc_create(TcContext** out, fo_server* s);
+void tc_destroy(TcContext* c);
+// Selects the tensor maps of batch slot `slot` for the first layer.
+void tc_set_input(TcContext* c, int slot);
+TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int op);
+TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int op, int accumulate);
+TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int op);
+void tc_run(TcGemm* g, const void* input, cudaStream_t st);
+const char* tc_name(const TcGemm* g);
+
+}  // namespace fo

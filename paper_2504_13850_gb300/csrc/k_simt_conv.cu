@@ -1,0 +1,190 @@
+// CUDA-core implicit-GEMM convolution (forward, input gradient, weight
+// gradient) with fp32 accumulation.  This is the fp32 compute path of the
+// library (the fp32 tiny workload) and serves layers whose shapes the
+// tensor-core kernels do not take (e.g. a classifier with 10 outputs).
+//
+// All three passes are one tiled GEMM C[M][N] = sum_k A[M][k] B[k][N] whose
+// operands are gathered on the fly from NHWC tensors:
+//   FWD    M = output pixels, N = Co, k = (r, s, ci):  A = x window, B = w
+//   DGRAD  M = input pixels,  N = Ci, k = (r, s, co):  A = dy (strided), B = w
+//   WGRAD  M = Co, N = (r, s, ci), k = output pixel:   A = dy^T, B = x window
+#include "fo_common.cuh"
+#include "fo_kernels.h"
+
+namespace fo {
+
+namespace {
+
+enum Mode { FWD = 0, DGRAD = 1, WGRAD = 2 };
+
+constexpr int BM = 64, BN = 64, BK = 16, NT = 256;
+
+struct Geo {
+  int N, H, W, Ci, Co, k, stride, pad, Ho, Wo;
+  int64_t M, Ncol, K;
+};
+
+template <typename T>
+__device__ __forceinline__ float ld(const T* p, int64_t i) { return to_f(p[i]); }
+
+// A[m][kk]
+template <int MODE, typename TA>
+__device__ __forceinline__ float load_a(const Geo& g, const TA* a, int64_t m, int64_t kk) {
+  if (m >= g.M || kk >= g.K) return 0.f;
+  if (MODE == FWD) {
+    int ci = int(kk % g.Ci);
+    int rs = int(kk / g.Ci);
+    int r = rs / g.k, s = rs % g.k;
+    int wo = int(m % g.Wo);
+    int64_t t = m / g.Wo;
+    int ho = int(t % g.Ho);
+    int n = int(t / g.Ho);
+    int h = ho * g.stride + r - g.pad, w = wo * g.stride + s - g.pad;
+    if (h < 0 || h >= g.H || w < 0 || w >= g.W) return 0.f;
+    return ld(a, ((int64_t(n) * g.H + h) * g.W + w) * g.Ci + ci);
+  } else if (MODE == DGRAD) {
+    int co = int(kk % g.Co);
+    int rs = int(kk / g.Co);
+    int r = rs / g.k, s = rs % g.k;
+    int w = int(m % g.W);
+    int64_t t = m / g.W;
+    int h = int(t % g.H);
+    int n = int(t / g.H);
+    int hh = h + g.pad - r, ww = w + g.pad - s;
+    if (hh < 0 || ww < 0 || hh % g.stride || ww % g.stride) return 0.f;
+    int ho = hh / g.stride, wo = ww / g.stride;
+    if (ho >= g.Ho || wo >= g.Wo) return 0.f;
+    return ld(a, ((int64_t(n) * g.Ho + ho) * g.Wo + wo) * g.Co + co);
+  } else {  // WGRAD: A[co][p] = dy[p][co]
+    return ld(a, kk * g.Co + m);
+  }
+}
+
+// B[kk][ncol]
+template <int MODE, typename TB>
+__device__ __forceinline__ float load_b(const Geo& g, const TB* b, int64_t kk, int64_t nc) {
+  if (kk >= g.K || nc >= g.Ncol) return 0.f;
+  if (MODE == FWD) {
+    return ld(b, nc * g.K + kk);                  // w[co][(r,s,ci)]
+  } else if (MODE == DGRAD) {
+    int co = int(kk % g.Co);
+    int rs = int(kk / g.Co);                      // w[co][r][s][ci]
+    return ld(b, (int64_t(co) * g.k * g.k + rs) * g.Ci + nc);
+  } else {  // WGRAD: B[p][(r,s,ci)] = x window
+    int ci = int(nc % g.Ci);
+    int rs = int(nc / g.Ci);
+    int r = rs / g.k, s = rs % g.k;
+    int wo = int(kk % g.Wo);
+    int64_t t = kk / g.Wo;
+    int ho = int(t % g.Ho);
+    int n = int(t / g.Ho);
+    int h = ho * g.stride + r - g.pad, w = wo * g.stride + s - g.pad;
+    if (h < 0 || h >= g.H || w < 0 || w >= g.W) return 0.f;
+    return ld(b, ((int64_t(n) * g.H + h) * g.W + w) * g.Ci + ci);
+  }
+}
+
+template <int MODE, typename TA, typename TB, typename TC>
+__global__ void __launch_bounds__(NT) simt_conv_kernel(Geo g, const TA* __restrict__ a,
+                                                       const TB* __restrict__ b,
+                                                       const float* __restrict__ bias,
+                                                       TC* __restrict__ c, int relu, int acc) {
+  __shared__ float As[BK][BM + 4];
+  __shared__ float Bs[BK][BN + 4];
+  const int tid = threadIdx.x;
+  const int tx = tid % 16, ty = tid / 16;
+  const int64_t m0 = int64_t(blockIdx.y) * BM, n0 = int64_t(blockIdx.x) * BN;
+  float accum[4][4] = {};
+  for (int64_t k0 = 0; k0 < g.K; k0 += BK) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      int e = tid + i * NT;           // 0..1023
+      int am = e / BK, ak = e % BK;   // A tile 64 x 16
+      As[ak][am] = load_a<MODE>(g, a, m0 + am, k0 + ak);
+      int bk = e / BN, bn = e % BN;   // B tile 16 x 64
+      Bs[bk][bn] = load_b<MODE>(g, b, k0 + bk, n0 + bn);
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < BK; ++kk) {
+      float av[4], bv[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) av[i] = As[kk][ty + 16 * i];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) bv[j] = Bs[kk][tx + 16 * j];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) accum[i][j] = fmaf(av[i], bv[j], accum[i][j]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    int64_t m = m0 + ty + 16 * i;
+    if (m >= g.M) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      int64_t n = n0 + tx + 16 * j;
+      if (n >= g.Ncol) continue;
+      float v = accum[i][j];
+      if (bias) v += bias[n];
+      if (relu) v = fmaxf(v, 0.f);
+      int64_t idx = m * g.Ncol + n;
+      if (acc) v += to_f(c[idx]);
+      c[idx] = from_f<TC>(v);
+    }
+  }
+}
+
+Geo make_geo(const ConvShape& s, int mode) {
+  Geo g{s.N, s.H, s.W, s.Ci, s.Co, s.k, s.stride, s.pad, s.Ho, s.Wo, 0, 0, 0};
+  int64_t pix_out = int64_t(s.N) * s.Ho * s.Wo, pix_in = int64_t(s.N) * s.H * s.W;
+  if (mode == FWD) {
+    g.M = pix_out; g.Ncol = s.Co; g.K = int64_t(s.k) * s.k * s.Ci;
+  } else if (mode == DGRAD) {
+    g.M = pix_in; g.Ncol = s.Ci; g.K = int64_t(s.k) * s.k * s.Co;
+  } else {
+    g.M = s.Co; g.Ncol = int64_t(s.k) * s.k * s.Ci; g.K = pix_out;
+  }
+  return g;
+}
+
+template <int MODE, typename TA, typename TB, typename TC>
+void launch(const Geo& g, const void* a, const void* b, const float* bias, void* c, bool relu,
+            bool acc, cudaStream_t st) {
+  dim3 grid(ceil_div(g.Ncol, BN), ceil_div(g.M, BM));
+  simt_conv_kernel<MODE, TA, TB, TC><<<grid, NT, 0, st>>>(
+      g, (const TA*)a, (const TB*)b, bias, (TC*)c, relu ? 1 : 0, acc ? 1 : 0);
+}
+
+}  // namespace
+
+void conv_fwd_simt(const ConvShape& s, const void* x, int dt_x, const float* w,
+                   const float* bias, void* y, int dt_y, bool relu, cudaStream_t st) {
+  Geo g = make_geo(s, FWD);
+  if (dt_x == kF32 && dt_y == kF32) launch<FWD, float, float, float>(g, x, w, bias, y, relu, false, st);
+  else if (dt_x == kBF16 && dt_y == kBF16) launch<FWD, bf16, float, bf16>(g, x, w, bias, y, relu, false, st);
+  else if (dt_x == kBF16 && dt_y == kF32) launch<FWD, bf16, float, float>(g, x, w, bias, y, relu, false, st);
+  else launch<FWD, float, float, bf16>(g, x, w, bias, y, relu, false, st);
+}
+
+void conv_dgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const float* w, void* dx,
+                     int dt_dx, bool accumulate, cudaStream_t st) {
+  Geo g = make_geo(s, DGRAD);
+  if (dt_dy == kF32 && dt_dx == kF32) launch<DGRAD, float, float, float>(g, dy, w, nullptr, dx, false, accumulate, st);
+  else if (dt_dy == kBF16 && dt_dx == kBF16) launch<DGRAD, bf16, float, bf16>(g, dy, w, nullptr, dx, false, accumulate, st);
+  else if (dt_dy == kF32 && dt_dx == kBF16) launch<DGRAD, float, float, bf16>(g, dy, w, nullptr, dx, false, accumulate, st);
+  else launch<DGRAD, bf16, float, float>(g, dy, w, nullptr, dx, false, accumulate, st);
+}
+
+void conv_wgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* x, int dt_x,
+                     float* dw, cudaStream_t st) {
+  Geo g = make_geo(s, WGRAD);
+  if (dt_dy == kF32 && dt_x == kF32) launch<WGRAD, float, float, float>(g, dy, x, nullptr, dw, false, false, st);
+  else if (dt_dy == kBF16 && dt_x == kBF16) launch<WGRAD, bf16, bf16, float>(g, dy, x, nullptr, dw, false, false, st);
+  else if (dt_dy == kF32 && dt_x == kBF16) launch<WGRAD, float, bf16, float>(g, dy, x, nullptr, dw, false, false, st);
+  else launch<WGRAD, bf16, float, float>(g, dy, x, nullptr, dw, false, false, st);
+}
+
+}  // namespace fo

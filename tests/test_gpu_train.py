@@ -1,0 +1,127 @@
+"""Server training steps on the GPU against the oracle on the same seeded
+traces: scheduler outcomes and slot indices bit-exact, per-step loss within
+1e-2 relative, parameters within 2e-2 normwise relative on the bf16 path and
+1e-4 on the fp32 path (the tolerances of the method's statement of the
+problem), and the parameter update theta_new - theta_old within a tolerance
+derived below.
+
+Update tolerance.  On the bf16 path each layer rounds its output and the
+operands of its products to bf16 (relative error 2^-9 each); a gradient is
+formed from a chain of at most ~12 such roundings plus fp32 sums, which
+bounds its normwise error by roughly 12 * 2^-9 ~ 2.5e-2 in the worst case;
+4e-2 leaves room for maxpool/ReLU decisions that flip under bf16 rounding.
+On the fp32 path the same chain with 2^-24 rounding gives < 1e-5; 1e-4 is
+used.
+"""
+import numpy as np
+import pytest
+
+from harness import normwise, replay_gpu, replay_oracle
+from paper_2504_13850_gb300 import api, build
+from paper_2504_13850_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    build.build()
+    api.lib()
+
+
+def small(kind):
+    """Shrunk bf16 configurations of each architecture family that still span
+    several tensor-core tiles and a ragged tail."""
+    if kind == "vgg":
+        b = W._Builder()
+        t = b.add("conv", 0, cin=64, cout=128, k=3, stride=1, bias=1)
+        t = b.add("relu", t)
+        t = b.add("conv", t, cin=128, cout=128, k=3, stride=1, bias=1)
+        t = b.add("relu", t)
+        t = b.add("maxpool2", t)
+        t = b.add("conv", t, cin=128, cout=256, k=3, stride=1, bias=1)
+        t = b.add("relu", t)
+        t = b.add("maxpool2", t)
+        t = b.add("flatten", t)
+        t = b.add("linear", t, cin=256 * 4 * 4, cout=128, bias=1)
+        t = b.add("relu", t)
+        b.add("linear", t, cin=128, cout=10, bias=1)
+        return W.shrink(W.CONFIGS["vgg"], ops=b.ops, batch=12, in_hwc=(16, 16, 64), K=3,
+                        omega=6, depth=2)
+    if kind == "resnet":
+        b = W._Builder()
+        t = W._basic_block(b, 0, 64, 128, 2)
+        t = W._basic_block(b, t, 128, 128, 1)
+        t = b.add("avgpool", t)
+        b.add("linear", t, cin=128, cout=100, bias=1)
+        return W.shrink(W.CONFIGS["resnet"], ops=b.ops, batch=10, in_hwc=(16, 16, 64), K=3,
+                        omega=6, depth=2)
+    if kind == "transformer":
+        return W.shrink(W.CONFIGS["transformer"],
+                        ops=W.transformer_ops(d=128, heads=2, ffn=256, blocks=2),
+                        batch=6, in_hwc=(128, 1, 128), K=3, omega=6, depth=2)
+    raise ValueError(kind)
+
+
+def prefill_then_steps(cfg, steps):
+    ev = [("enq", k) for _ in range(cfg["depth"]) for k in range(cfg["K"])]
+    return ev + [("step",)] * steps
+
+
+def compare(cfg, events, loss_tol, param_tol, upd_tol):
+    s, glog = replay_gpu(cfg, events)
+    o, olog = replay_oracle(cfg, events)
+    assert glog == olog                           # scheduler outcomes, slots: bit-exact
+    nsteps = sum(1 for e in glog if e[0] == "step" and e[1] == api.OK)
+    losses = s.read_losses(0, nsteps)
+    ol = np.array(o.losses)
+    assert np.all(np.abs(losses - ol) <= loss_tol * np.abs(ol)), (losses, ol)
+    theta = s.get_params()
+    theta0 = W.init_params(cfg).astype(np.float64)
+    assert normwise(theta, o.theta) <= param_tol
+    assert normwise(theta - theta0, o.theta - theta0) <= upd_tol
+    mom = s.get_momentum()
+    assert normwise(mom, o.v) <= upd_tol
+    return s, o
+
+
+def test_tiny_config_fp32_full_trace():
+    cfg = W.CONFIGS["tiny"]
+    events = prefill_then_steps(cfg, 9)           # 8 steps + one on empty queues
+    s, o = compare(cfg, events, loss_tol=1e-4, param_tol=1e-4, upd_tol=1e-4)
+    assert [int(c) for c in s.counters()] == o.sched.c == [2, 2, 2, 2]
+
+
+@pytest.mark.parametrize("kind", ["vgg", "resnet", "transformer"])
+def test_small_bf16_configs(kind):
+    cfg = small(kind)
+    compare(cfg, prefill_then_steps(cfg, 6), loss_tol=1e-2, param_tol=2e-2, upd_tol=4e-2)
+
+
+def test_arrival_trace_with_refusals_matches_oracle():
+    """A Poisson arrival trace over devices of four speed groups, with the
+    global cap reached: refusals, sender flags and served order bit-exact."""
+    cfg = W.shrink(W.CONFIGS["tiny"], K=6, omega=5, depth=2,
+                   rates=W.group_rates(6))
+    ev = W.trace(cfg, n_steps=12, uploads_per_step=2, prefill=False)
+    compare(cfg, ev, loss_tol=1e-4, param_tol=1e-4, upd_tol=1e-4)
+
+
+def test_activation_memory_is_independent_of_devices():
+    """Eq. 3: server activation memory is omega batches, whatever K is."""
+    cfg = W.CONFIGS["tiny"]
+    a = api.Server.from_config(cfg, K=4, omega=8)
+    b = api.Server.from_config(cfg, K=100, omega=8)
+    assert a.activation_bytes() == b.activation_bytes()
+    B, (H, Wd, Ci) = cfg["batch"], cfg["in_hwc"]
+    assert a.activation_bytes() >= 8 * B * H * Wd * Ci * 4
+
+
+def test_empty_and_bad_calls():
+    cfg = W.CONFIGS["tiny"]
+    s = api.Server.from_config(cfg)
+    assert s.server_step()[0] == api.EMPTY
+    x, _, labels, _ = W.device_batch(cfg, 0, 0)
+    assert s.enqueue_activations(7, x, labels)[0] == api.ERR_ARG
+    s.set_device_active(2, False)
+    assert s.enqueue_activations(2, x, labels)[0] == api.ERR_ARG
