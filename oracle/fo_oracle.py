@@ -36,6 +36,14 @@ Readings where the paper is silent (each one is listed in the design notes):
     row-major window order;
   * the first server layer's input gradient is never formed: nothing is sent
     back to devices (gradient-free offloading, Sec. 3.2.2 / Sec. 3.3.1).
+
+Two precisions.  With storage=None every value is fp64 (the definition).
+With storage="bf16" the oracle keeps the same values a bf16 tensor-core
+implementation stores, so that floating point takes every integer decision
+(ReLU mask, max-pool argmax) in the kernel's precision: each op's output
+and each activation gradient is rounded to bf16 (round to nearest even) when
+stored, and the weights of every conv / linear layer except the logits layer
+are rounded to bf16 before use; arithmetic in between stays fp64.
 """
 from __future__ import annotations
 
@@ -46,6 +54,15 @@ from scipy.special import erf
 
 OK, EMPTY, FULL, STALE = 0, 1, 2, 3
 ERR_ARG = -1
+
+
+def to_bf16(x):
+    """Round to the nearest bfloat16 value (ties to even), returned as fp64.
+    Rounds the fp64 value directly, without an intermediate fp32 step."""
+    x = np.asarray(x, np.float64)
+    m, e = np.frexp(x)                       # x = m * 2**e, 0.5 <= |m| < 1
+    # bf16 keeps 8 significant bits: scale the mantissa to an integer grid
+    return np.ldexp(np.round(np.ldexp(m, 8)), e - 8)
 
 
 # ==========================================================================
@@ -414,14 +431,21 @@ def flatten(ops, grads):
     return np.concatenate([grads[(i, name)].ravel() for i, name, _ in param_shapes(ops)])
 
 
-def forward(ops, params, x, lengths):
+def _weights(ops, params, i, storage):
+    w = params.get((i, "W"))
+    if storage == "bf16" and i < len(ops) - 1:
+        w = to_bf16(w)
+    return w
+
+
+def forward(ops, params, x, lengths, storage=None):
     """Forward pass of M_s.  Returns the list of tensors (tensor 0 = x) and
     per-op caches."""
     T = [np.asarray(x, np.float64)]
     caches = [None] * len(ops)
     for i, op in enumerate(ops):
         kd, a = op["kind"], T[op["in0"]]
-        P = lambda n: params.get((i, n))
+        P = lambda n: _weights(ops, params, i, storage) if n == "W" else params.get((i, n))
         if kd == "conv":
             y = conv_fwd(a, P("W"), P("b"), op["stride"], op["k"] // 2)
         elif kd == "affine":
@@ -448,20 +472,24 @@ def forward(ops, params, x, lengths):
             y = meanpool_fwd(a, lengths)
         else:
             raise ValueError(kd)
+        if storage == "bf16" and i < len(ops) - 1:
+            y = to_bf16(y)
         T.append(y)
     return T, caches
 
 
-def backward(ops, params, T, caches, dlogits, lengths):
+def backward(ops, params, T, caches, dlogits, lengths, storage=None):
     """Backward pass of M_s.  The input tensor (tensor 0) receives no
-    gradient: the server never returns gradients to devices."""
+    gradient: the server never returns gradients to devices.  Contributions
+    to a tensor's gradient are added in reverse op order."""
     G = {len(ops): dlogits}
     grads = {}
+    rnd = to_bf16 if storage == "bf16" else (lambda v: v)
 
     def acc(tid, g):
         if tid == 0 or g is None:
             return
-        G[tid] = G[tid] + g if tid in G else g
+        G[tid] = rnd(G[tid] + g) if tid in G else rnd(g)
 
     for i in range(len(ops) - 1, -1, -1):
         op = ops[i]
@@ -470,7 +498,7 @@ def backward(ops, params, T, caches, dlogits, lengths):
         if dy is None:
             dy = np.zeros_like(T[i + 1])
         need = op["in0"] != 0
-        P = lambda n: params.get((i, n))
+        P = lambda n: _weights(ops, params, i, storage) if n == "W" else params.get((i, n))
         if kd == "conv":
             dx, dw, db = conv_bwd(a, P("W"), dy, op["stride"], op["k"] // 2, need)
             grads[(i, "W")] = dw
@@ -513,12 +541,12 @@ def backward(ops, params, T, caches, dlogits, lengths):
     return grads
 
 
-def loss_and_grad(ops, theta, x, labels, lengths=None):
+def loss_and_grad(ops, theta, x, labels, lengths=None, storage=None):
     """f_s(theta_s; xi) and its gradient (flat fp64)."""
     params = unflatten(ops, theta)
-    T, caches = forward(ops, params, x, lengths)
+    T, caches = forward(ops, params, x, lengths, storage)
     loss, dz = softmax_ce(T[-1], np.asarray(labels))
-    grads = backward(ops, params, T, caches, dz, lengths)
+    grads = backward(ops, params, T, caches, dz, lengths, storage)
     return loss, flatten(ops, grads)
 
 
@@ -528,10 +556,10 @@ def sgd_momentum(theta, v, g, lr, mu):
     return theta - lr * v, v
 
 
-def server_step(ops, theta, v, x, labels, lengths, lr, mu):
+def server_step(ops, theta, v, x, labels, lengths, lr, mu, storage=None):
     """One training iteration of Algorithm 4 (forward, loss, backward,
     update).  Returns (loss, theta, v, g)."""
-    loss, g = loss_and_grad(ops, theta, x, labels, lengths)
+    loss, g = loss_and_grad(ops, theta, x, labels, lengths, storage)
     theta, v = sgd_momentum(np.asarray(theta, np.float64), np.asarray(v, np.float64), g, lr, mu)
     return loss, theta, v, g
 
@@ -545,8 +573,9 @@ class Server:
     server model (theta_s, momentum), batch slots and the aggregator."""
 
     def __init__(self, ops, K, omega, depth, theta0, lr, mu, max_delay=2**31 - 1,
-                 policy="counter"):
+                 policy="counter", storage=None):
         self.ops = ops
+        self.storage = storage
         self.sched = TaskScheduler(K, omega, depth, policy)
         self.agg = Aggregator(K, max_delay)
         self.theta = np.asarray(theta0, np.float64).copy()
@@ -568,7 +597,7 @@ class Server:
             return st, -1, -1
         x, y, ln = self.slots.pop(slot)
         loss, self.theta, self.v, _ = server_step(self.ops, self.theta, self.v, x, y, ln,
-                                                  self.lr, self.mu)
+                                                  self.lr, self.mu, self.storage)
         self.losses.append(loss)
         return OK, k, slot
 

@@ -12,12 +12,12 @@ enum DType { kF32 = 0, kBF16 = 1 };
 struct ConvShape {
   int N, H, W, Ci, Co, k, stride, pad, Ho, Wo;
 };
-// y = conv(x, w) + bias, optional ReLU.  x NHWC (dtype dx), w fp32
-// [Co][k][k][Ci], bias fp32 or null, y NHWC (dtype dy).
-void conv_fwd_simt(const ConvShape& s, const void* x, int dt_x, const float* w,
+// y = conv(x, w) + bias, optional ReLU.  x NHWC, w [Co][k][k][Ci], bias fp32
+// or null, y NHWC; each operand's dtype is given (kF32 / kBF16).
+void conv_fwd_simt(const ConvShape& s, const void* x, int dt_x, const void* w, int dt_w,
                    const float* bias, void* y, int dt_y, bool relu, cudaStream_t st);
 // dx (+)= conv^T(dy, w).
-void conv_dgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const float* w,
+void conv_dgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* w, int dt_w,
                      void* dx, int dt_dx, bool accumulate, cudaStream_t st);
 // dw[Co][k][k][Ci] = sum over output pixels of dy (x) x-window (fp32 out).
 void conv_wgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* x,

@@ -181,11 +181,15 @@ int build_plan(fo_server* s) {
         if (tg) {
           plan.push_back({fo::tc_name(tg), [=](cudaStream_t st) { fo::tc_run(tg, act(a), st); }});
         } else {
-          int dto = to.dt;
+          // Hidden layers of the bf16 path multiply bf16 weights (the shadow);
+          // the fp32 path and the fp32 logits layer use the fp32 master.
+          const int dto = to.dt;
+          const bool wbf = dto == fo::kBF16;
           plan.push_back({op.kind == FO_OP_CONV ? "conv_fwd_simt" : "linear_fwd_simt",
                           [=](cudaStream_t st) {
-                            fo::conv_fwd_simt(cs, act(a), ta.dt, P(s, i, 0), bias ? P(s, i, 1) : nullptr,
-                                              s->T[o].act, dto, false, st);
+                            const void* w = wbf ? (const void*)SH(s, i, 0) : (const void*)P(s, i, 0);
+                            fo::conv_fwd_simt(cs, act(a), ta.dt, w, wbf ? fo::kBF16 : fo::kF32,
+                                              bias ? P(s, i, 1) : nullptr, s->T[o].act, dto, false, st);
                           }});
         }
         break;
@@ -304,10 +308,12 @@ int build_plan(fo_server* s) {
           if (tg) {
             plan.push_back({fo::tc_name(tg), [=](cudaStream_t st) { fo::tc_run(tg, nullptr, st); }});
           } else {
+            const bool wbf = dto == fo::kBF16;
             plan.push_back({op.kind == FO_OP_CONV ? "conv_dgrad_simt" : "linear_dgrad_simt",
                             [=](cudaStream_t st) {
-                              fo::conv_dgrad_simt(cs, s->T[o].grad, dto, P(s, i, 0), s->T[a].grad, dta,
-                                                  accf != 0, st);
+                              const void* w = wbf ? (const void*)SH(s, i, 0) : (const void*)P(s, i, 0);
+                              fo::conv_dgrad_simt(cs, s->T[o].grad, dto, w, wbf ? fo::kBF16 : fo::kF32,
+                                                  s->T[a].grad, dta, accf != 0, st);
                             }});
           }
         }
@@ -572,6 +578,7 @@ int fo_server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt, const
   rc = allocate(s);
   if (rc == FO_OK) rc = fo::tc_create(&s->tc, s);
   if (rc == FO_OK) rc = build_plan(s);
+  if (rc == FO_OK) rc = fo::tc_finalize(s->tc);
   if (rc == FO_OK && cudaDeviceSynchronize() != cudaSuccess) rc = set_err(FO_ERR_CUDA, "create sync");
   if (rc != FO_OK) {
     destroy_impl(s);

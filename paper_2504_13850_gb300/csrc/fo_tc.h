@@ -21,5 +21,9 @@ TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int op, int accumulate);
 TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int op);
 void tc_run(TcGemm* g, const void* input, cudaStream_t st);
 const char* tc_name(const TcGemm* g);
+// Allocates the split-K workspace after every plan is known.
+int tc_finalize(TcContext* c);
+// Device word the tensor-core kernels set on a timed-out wait (0 = none).
+int* tc_error_word(TcContext* c);
 
 }  // namespace fo

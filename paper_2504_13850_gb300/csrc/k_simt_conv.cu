@@ -158,33 +158,41 @@ void launch(const Geo& g, const void* a, const void* b, const float* bias, void*
       g, (const TA*)a, (const TB*)b, bias, (TC*)c, relu ? 1 : 0, acc ? 1 : 0);
 }
 
-}  // namespace
-
-void conv_fwd_simt(const ConvShape& s, const void* x, int dt_x, const float* w,
-                   const float* bias, void* y, int dt_y, bool relu, cudaStream_t st) {
-  Geo g = make_geo(s, FWD);
-  if (dt_x == kF32 && dt_y == kF32) launch<FWD, float, float, float>(g, x, w, bias, y, relu, false, st);
-  else if (dt_x == kBF16 && dt_y == kBF16) launch<FWD, bf16, float, bf16>(g, x, w, bias, y, relu, false, st);
-  else if (dt_x == kBF16 && dt_y == kF32) launch<FWD, bf16, float, float>(g, x, w, bias, y, relu, false, st);
-  else launch<FWD, float, float, bf16>(g, x, w, bias, y, relu, false, st);
+// Instantiate every (A, B, C) dtype combination of one pass.
+template <int MODE, typename TA, typename TB>
+void launch_c(const Geo& g, const void* a, const void* b, const float* bias, void* c, int dtc,
+              bool relu, bool acc, cudaStream_t st) {
+  if (dtc == kF32) launch<MODE, TA, TB, float>(g, a, b, bias, c, relu, acc, st);
+  else launch<MODE, TA, TB, bf16>(g, a, b, bias, c, relu, acc, st);
+}
+template <int MODE, typename TA>
+void launch_bc(const Geo& g, const void* a, const void* b, int dtb, const float* bias, void* c,
+               int dtc, bool relu, bool acc, cudaStream_t st) {
+  if (dtb == kF32) launch_c<MODE, TA, float>(g, a, b, bias, c, dtc, relu, acc, st);
+  else launch_c<MODE, TA, bf16>(g, a, b, bias, c, dtc, relu, acc, st);
+}
+template <int MODE>
+void launch_any(const Geo& g, const void* a, int dta, const void* b, int dtb, const float* bias,
+                void* c, int dtc, bool relu, bool acc, cudaStream_t st) {
+  if (dta == kF32) launch_bc<MODE, float>(g, a, b, dtb, bias, c, dtc, relu, acc, st);
+  else launch_bc<MODE, bf16>(g, a, b, dtb, bias, c, dtc, relu, acc, st);
 }
 
-void conv_dgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const float* w, void* dx,
-                     int dt_dx, bool accumulate, cudaStream_t st) {
-  Geo g = make_geo(s, DGRAD);
-  if (dt_dy == kF32 && dt_dx == kF32) launch<DGRAD, float, float, float>(g, dy, w, nullptr, dx, false, accumulate, st);
-  else if (dt_dy == kBF16 && dt_dx == kBF16) launch<DGRAD, bf16, float, bf16>(g, dy, w, nullptr, dx, false, accumulate, st);
-  else if (dt_dy == kF32 && dt_dx == kBF16) launch<DGRAD, float, float, bf16>(g, dy, w, nullptr, dx, false, accumulate, st);
-  else launch<DGRAD, bf16, float, float>(g, dy, w, nullptr, dx, false, accumulate, st);
+}  // namespace
+
+void conv_fwd_simt(const ConvShape& s, const void* x, int dt_x, const void* w, int dt_w,
+                   const float* bias, void* y, int dt_y, bool relu, cudaStream_t st) {
+  launch_any<FWD>(make_geo(s, FWD), x, dt_x, w, dt_w, bias, y, dt_y, relu, false, st);
+}
+
+void conv_dgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* w, int dt_w,
+                     void* dx, int dt_dx, bool accumulate, cudaStream_t st) {
+  launch_any<DGRAD>(make_geo(s, DGRAD), dy, dt_dy, w, dt_w, nullptr, dx, dt_dx, false, accumulate, st);
 }
 
 void conv_wgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* x, int dt_x,
                      float* dw, cudaStream_t st) {
-  Geo g = make_geo(s, WGRAD);
-  if (dt_dy == kF32 && dt_x == kF32) launch<WGRAD, float, float, float>(g, dy, x, nullptr, dw, false, false, st);
-  else if (dt_dy == kBF16 && dt_x == kBF16) launch<WGRAD, bf16, bf16, float>(g, dy, x, nullptr, dw, false, false, st);
-  else if (dt_dy == kF32 && dt_x == kBF16) launch<WGRAD, float, bf16, float>(g, dy, x, nullptr, dw, false, false, st);
-  else launch<WGRAD, bf16, float, float>(g, dy, x, nullptr, dw, false, false, st);
+  launch_any<WGRAD>(make_geo(s, WGRAD), dy, dt_dy, x, dt_x, nullptr, dw, kF32, false, false, st);
 }
 
 }  // namespace fo

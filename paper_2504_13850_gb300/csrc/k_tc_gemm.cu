@@ -1,22 +1,761 @@
-// Tensor-core path (placeholder: no op is routed to tensor cores yet).
+// Tensor-core GEMM / implicit-GEMM convolution for sm_103a: tcgen05.mma
+// (kind::f16, bf16 operands, fp32 accumulator in TMEM) fed by TMA tiles in
+// 128-byte-swizzled shared memory, with a warp-specialised pipeline:
+//   warp 0      TMA producer (one thread)
+//   warp 1      TMEM allocator and MMA issuer (one thread)
+//   warps 2..5  epilogue: tcgen05.ld of the 128 x BN accumulator, then the
+//               bias / ReLU / bf16 or fp32 store (or an fp32 split-K partial)
+// Every mbarrier wait is bounded: on timeout the kernel records an error
+// code in global memory and leaves instead of spinning forever.
+//
+// Problem kinds (D[M][N] = sum_k A[M][k] B[N][k]):
+//   LIN_FWD    Y = X W^T          A = X  [rows][cin] K-major,  B = W [cout][cin] K-major
+//   LIN_DGRAD  dX = dY W          A = dY [rows][cout] K-major, B = W (N = cin contiguous) MN-major
+//   LIN_WGRAD  dW = dY^T X        A = dY (M = cout contiguous) MN-major, B = X MN-major
+//   CONV_FPROP y = conv(x, W)     A = x window (per tap, 4-D TMA with zero fill) K-major,
+//                                 B = W [Co][taps*Ci] K-major
+//   CONV_DGRAD dx = conv^T(dy, W) A = dy window, taps shifted the other way,
+//                                 B = W rows co, columns tap*Ci + ci: MN-major
+//   CONV_WGRAD dW = sum_p dy (x) x-window: A = dy [P][Co] MN-major, B = x window MN-major
 #include "fo_server_impl.h"
 #include "fo_tc.h"
 
+#include <cuda.h>
+#include <algorithm>
+#include <cstring>
+#include <vector>
+
 namespace fo {
 
-struct TcContext {};
-struct TcGemm {};
+namespace {
 
-int tc_create(TcContext** out, fo_server*) {
-  *out = new TcContext();
+enum Kind { LIN_FWD = 0, LIN_DGRAD = 1, LIN_WGRAD = 2, CONV_FPROP = 3, CONV_DGRAD = 4, CONV_WGRAD = 5 };
+
+constexpr int BM = 128;      // UMMA M (cta_group::1)
+constexpr int BK = 64;       // k-block: one 128-byte swizzle row of bf16
+constexpr int UK = 16;       // UMMA K for kind::f16
+constexpr int kThreads = 192;
+constexpr int kSmemBudget = 200 * 1024;
+
+struct TcParams {
+  CUtensorMap tmA;
+  CUtensorMap tmB;
+  int M, N, KB, kper;
+  // window geometry (spatial size of the windowed tensor and its taps)
+  int H, W, ksz, pad, taps;
+  int cblocks;          // 64-channel blocks per tap (contraction channels)
+  int ntap_ch;          // CONV_WGRAD / CONV_DGRAD: channels per tap in the N index (Ci)
+  int win_rows, win_imgs;  // rows/images covered by one window box
+  // epilogue
+  void* out;
+  int ldo;
+  const float* bias;
+  int relu, acc, out_f32;
+  float* ws;            // split-K partials [splits][M][N] (fp32) or null
+  int* err;
+};
+
+// ----------------------------------------------------------------- PTX
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Wait for the phase with the given parity; gives up after ~2 s.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  while (true) {
+    for (int i = 0; i < 64; ++i)
+      if (mbar_try_wait(bar, parity)) return true;
+    if (global_ns() - t0 > 2000000000ull) return false;
+  }
+}
+__device__ __forceinline__ void tma_2d(void* dst, const CUtensorMap* m, uint64_t* bar, int c0, int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];"
+      ::"r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(m)), "r"(smem_u32(bar)), "r"(c0), "r"(c1)
+      : "memory");
+}
+__device__ __forceinline__ void tma_4d(void* dst, const CUtensorMap* m, uint64_t* bar, int c0, int c1, int c2,
+                                       int c3) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, %5, %6}], "
+      "[%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(m)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+      : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Shared-memory matrix descriptor: start, leading / stride byte offsets,
+// descriptor version 1 (bit 46), 128-byte swizzle (layout 2, bits 61-63).
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= uint64_t((addr >> 4) & 0x3FFF);
+  d |= uint64_t((lbo >> 4) & 0x3FFF) << 16;
+  d |= uint64_t((sbo >> 4) & 0x3FFF) << 32;
+  d |= uint64_t(1) << 46;
+  d |= uint64_t(2) << 61;
+  return d;
+}
+// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B,
+// A / B major-ness, N >> 3 at bit 17, M >> 4 at bit 24.
+__host__ __device__ constexpr uint32_t instr_desc(int n, bool a_mn, bool b_mn) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(a_mn) << 15) | (uint32_t(b_mn) << 16) |
+         (uint32_t(n >> 3) << 17) | (uint32_t(BM >> 4) << 24);
+}
+__device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
+          tmem_d),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+template <int KIND>
+struct KindTraits {
+  static constexpr bool a_mn = (KIND == LIN_WGRAD || KIND == CONV_WGRAD);
+  static constexpr bool b_mn = (KIND == LIN_DGRAD || KIND == LIN_WGRAD || KIND == CONV_DGRAD || KIND == CONV_WGRAD);
+};
+
+// Issue the TMA loads of k-block `kb` for output tile (m0, n0).
+template <int KIND, int BN>
+__device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, int n0, char* sa, char* sb,
+                                            uint64_t* bar) {
+  const int HW = p.H * p.W;
+  if (KIND == LIN_FWD || KIND == LIN_DGRAD) {
+    tma_2d(sa, &p.tmA, bar, kb * BK, m0);
+  } else if (KIND == LIN_WGRAD || KIND == CONV_WGRAD) {
+#pragma unroll
+    for (int j = 0; j < BM / 64; ++j) tma_2d(sa + j * BK * 128, &p.tmA, bar, m0 + j * 64, kb * BK);
+  } else {  // CONV_FPROP / CONV_DGRAD: windowed A
+    const int tap = kb / p.cblocks, c0 = (kb % p.cblocks) * 64;
+    const int r = tap / p.ksz, s = tap % p.ksz;
+    const int n_img = m0 / HW, h0 = (m0 % HW) / p.W;
+    const int dh = (KIND == CONV_FPROP) ? r - p.pad : p.pad - r;
+    const int dw = (KIND == CONV_FPROP) ? s - p.pad : p.pad - s;
+    tma_4d(sa, &p.tmA, bar, c0, dw, h0 + dh, n_img);
+  }
+  if (KIND == LIN_FWD) {
+    tma_2d(sb, &p.tmB, bar, kb * BK, n0);
+  } else if (KIND == CONV_FPROP) {
+    const int tap = kb / p.cblocks, c0 = (kb % p.cblocks) * 64;
+    tma_2d(sb, &p.tmB, bar, tap * p.ntap_ch + c0, n0);
+  } else if (KIND == LIN_DGRAD || KIND == LIN_WGRAD) {
+#pragma unroll
+    for (int j = 0; j < BN / 64; ++j) tma_2d(sb + j * BK * 128, &p.tmB, bar, n0 + j * 64, kb * BK);
+  } else if (KIND == CONV_DGRAD) {
+    const int tap = kb / p.cblocks, co0 = (kb % p.cblocks) * 64;
+#pragma unroll
+    for (int j = 0; j < BN / 64; ++j) tma_2d(sb + j * BK * 128, &p.tmB, bar, tap * p.ntap_ch + n0 + j * 64, co0);
+  } else {  // CONV_WGRAD: N index = tap * Ci + ci; K = output pixel
+    const int tap = n0 / p.ntap_ch, ci0 = n0 % p.ntap_ch;
+    const int r = tap / p.ksz, s = tap % p.ksz;
+    const int pix0 = kb * BK;
+    const int n_img = pix0 / HW, h0 = (pix0 % HW) / p.W;
+#pragma unroll
+    for (int j = 0; j < BN / 64; ++j)
+      tma_4d(sb + j * BK * 128, &p.tmB, bar, ci0 + j * 64, s - p.pad, h0 + r - p.pad, n_img);
+  }
+}
+
+template <int KIND, int BN, int STAGES>
+__global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ TcParams p) {
+  extern __shared__ __align__(1024) char smem_raw[];
+  char* smem = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  constexpr int A_BYTES = BM * BK * 2;
+  constexpr int B_BYTES = BN * BK * 2;
+  constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* accum = empty + STAGES;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM;
+  const int kb0 = blockIdx.z * p.kper;
+  const int kb1 = min(p.KB, kb0 + p.kper);
+  const int nk = kb1 - kb0;
+  constexpr uint32_t kCols = BN < 32 ? 32 : BN;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(accum, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmA)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmB)) : "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(kCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int it = 0; it < nk; ++it) {
+        const int s = it % STAGES;
+        if (!mbar_wait(&empty[s], ((it / STAGES) & 1) ^ 1)) {
+          atomicExch(p.err, 1);
+          *abort_flag = 1;
+          break;
+        }
+        if (*abort_flag) break;
+        char* sa = smem + s * STAGE_BYTES;
+        mbar_expect_tx(&full[s], STAGE_BYTES);
+        load_kblock<KIND, BN>(p, kb0 + it, m0, n0, sa, sa + A_BYTES, &full[s]);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = instr_desc(BN, KindTraits<KIND>::a_mn, KindTraits<KIND>::b_mn);
+      bool ok = true;
+      for (int it = 0; it < nk; ++it) {
+        const int s = it % STAGES;
+        if (!mbar_wait(&full[s], (it / STAGES) & 1)) {
+          atomicExch(p.err, 2);
+          *abort_flag = 1;
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a0 = smem_u32(smem + s * STAGE_BYTES);
+        const uint32_t b0 = a0 + A_BYTES;
+#pragma unroll
+        for (int k = 0; k < BK / UK; ++k) {
+          uint64_t ad, bd;
+          if (KindTraits<KIND>::a_mn) ad = smem_desc(a0 + k * UK * 128, BK * 128, 1024);
+          else ad = smem_desc(a0 + k * UK * 2, 16, 1024);
+          if (KindTraits<KIND>::b_mn) bd = smem_desc(b0 + k * UK * 128, BK * 128, 1024);
+          else bd = smem_desc(b0 + k * UK * 2, 16, 1024);
+          mma_f16(tmem, ad, bd, idesc, (it > 0 || k > 0) ? 1u : 0u);
+        }
+        mma_commit(&empty[s]);
+      }
+      if (ok) mma_commit(accum);
+      else mbar_expect_tx(accum, 0);  // release the epilogue without data
+    }
+  } else {
+    // Epilogue: warp (2..5) % 4 owns TMEM lanes 32 * q .. 32 * q + 31.
+    const int q = warp % 4;
+    const bool ready = mbar_wait(accum, 0);
+    tc_fence_after();
+    if (!ready) atomicExch(p.err, 3);
+    const int m = m0 + q * 32 + lane;
+    const bool valid = ready && !*abort_flag && nk > 0;
+    for (int c = 0; c < BN; c += 16) {
+      uint32_t r[16];
+      tmem_ld16(tmem + (uint32_t(q * 32) << 16) + uint32_t(c), r);
+      if (!valid || m >= p.M) continue;
+      float v[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
+      const int n = n0 + c;
+      if (p.ws) {
+        float4* dst = reinterpret_cast<float4*>(p.ws + (size_t(blockIdx.z) * p.M + m) * p.N + n);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+        continue;
+      }
+      if (p.bias) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] += p.bias[n + j];
+      }
+      if (p.relu) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] = fmaxf(v[j], 0.f);
+      }
+      if (p.out_f32) {
+        float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + size_t(m) * p.ldo + n);
+        if (p.acc) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            float4 o = dst[j];
+            v[4 * j] += o.x; v[4 * j + 1] += o.y; v[4 * j + 2] += o.z; v[4 * j + 3] += o.w;
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+      } else {
+        uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(p.out) + size_t(m) * p.ldo + n);
+        if (p.acc) {
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            uint4 o = dst[j];
+            const bf16* ob = reinterpret_cast<const bf16*>(&o);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) v[8 * j + e] += __bfloat162float(ob[e]);
+          }
+        }
+        uint4 pk[2];
+        uint32_t* pw = reinterpret_cast<uint32_t*>(pk);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          __nv_bfloat162 h2 = __floats2bfloat162_rn(v[2 * j], v[2 * j + 1]);
+          pw[j] = *reinterpret_cast<uint32_t*>(&h2);
+        }
+        dst[0] = pk[0];
+        dst[1] = pk[1];
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kCols) : "memory");
+  }
+}
+
+// Deterministic split-K reduction (fixed order over splits) with the
+// epilogue of the unsplit kernel.
+__global__ void splitk_reduce_k(const float* __restrict__ ws, int splits, int M, int N, void* out, int ldo,
+                                const float* __restrict__ bias, int relu, int acc, int out_f32) {
+  const int64_t total4 = int64_t(M) * N / 4;
+  for (int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; i < total4;
+       i += int64_t(gridDim.x) * blockDim.x) {
+    const int64_t e = i * 4;
+    const int m = int(e / N), n = int(e % N);
+    float4 s = reinterpret_cast<const float4*>(ws)[i];
+    for (int z = 1; z < splits; ++z) {
+      const float4 t = reinterpret_cast<const float4*>(ws + size_t(z) * M * N)[i];
+      s.x += t.x; s.y += t.y; s.z += t.z; s.w += t.w;
+    }
+    float v[4] = {s.x, s.y, s.z, s.w};
+    if (bias) for (int j = 0; j < 4; ++j) v[j] += bias[n + j];
+    if (relu) for (int j = 0; j < 4; ++j) v[j] = fmaxf(v[j], 0.f);
+    if (out_f32) {
+      float* d = reinterpret_cast<float*>(out) + size_t(m) * ldo + n;
+      if (acc) for (int j = 0; j < 4; ++j) v[j] += d[j];
+      *reinterpret_cast<float4*>(d) = make_float4(v[0], v[1], v[2], v[3]);
+    } else {
+      bf16* d = reinterpret_cast<bf16*>(out) + size_t(m) * ldo + n;
+      if (acc) for (int j = 0; j < 4; ++j) v[j] += __bfloat162float(d[j]);
+      __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]), b = __floats2bfloat162_rn(v[2], v[3]);
+      uint2 u;
+      u.x = *reinterpret_cast<uint32_t*>(&a);
+      u.y = *reinterpret_cast<uint32_t*>(&b);
+      *reinterpret_cast<uint2*>(d) = u;
+    }
+  }
+}
+
+template <int KIND, int BN>
+constexpr int stages_for() {
+  return kSmemBudget / (BM * BK * 2 + BN * BK * 2) > 8 ? 8 : kSmemBudget / (BM * BK * 2 + BN * BK * 2);
+}
+template <int KIND, int BN>
+constexpr size_t smem_bytes() {
+  return size_t(stages_for<KIND, BN>()) * (BM * BK * 2 + BN * BK * 2) + 1024 + 256;
+}
+
+typedef void (*KernelFn)(const TcParams);
+
+template <int KIND, int BN>
+KernelFn kernel_ptr() {
+  return tc_gemm_kernel<KIND, BN, stages_for<KIND, BN>()>;
+}
+
+KernelFn pick_kernel(int kind, int bn, size_t* smem) {
+#define FO_PICK(K)                                                  \
+  if (kind == K) {                                                  \
+    if (bn == 256) { *smem = smem_bytes<K, 256>(); return kernel_ptr<K, 256>(); } \
+    if (bn == 128) { *smem = smem_bytes<K, 128>(); return kernel_ptr<K, 128>(); } \
+    *smem = smem_bytes<K, 64>();                                    \
+    return kernel_ptr<K, 64>();                                     \
+  }
+  FO_PICK(LIN_FWD)
+  FO_PICK(LIN_DGRAD)
+  FO_PICK(LIN_WGRAD)
+  FO_PICK(CONV_FPROP)
+  FO_PICK(CONV_DGRAD)
+  FO_PICK(CONV_WGRAD)
+#undef FO_PICK
+  return nullptr;
+}
+
+// ------------------------------------------------------------ tensor maps
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// bf16 tensor map, dims innermost first, strides in bytes of dims 1.. .
+bool make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, const uint64_t* strides,
+              const uint32_t* box) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t d[5], st[4];
+  cuuint32_t b[5], es[5];
+  for (int i = 0; i < rank; ++i) {
+    d[i] = dims[i];
+    b[i] = box[i];
+    es[i] = 1;
+    if (i + 1 < rank) st[i] = strides[i];
+  }
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), d, st, b, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+// 2-D [rows][cols] row-major bf16, box (64 cols, box_rows).
+bool map_2d(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int box_rows) {
+  uint64_t dims[2] = {uint64_t(cols), uint64_t(rows)};
+  uint64_t strides[1] = {uint64_t(cols) * 2};
+  uint32_t box[2] = {64, uint32_t(box_rows)};
+  return make_map(m, base, 2, dims, strides, box);
+}
+
+// 4-D NHWC window map: box (64 channels, W, rows, imgs).
+bool map_window(CUtensorMap* m, const void* base, int N, int H, int W, int C, int rows, int imgs) {
+  uint64_t dims[4] = {uint64_t(C), uint64_t(W), uint64_t(H), uint64_t(N)};
+  uint64_t strides[3] = {uint64_t(C) * 2, uint64_t(W) * C * 2, uint64_t(H) * W * C * 2};
+  uint32_t box[4] = {64, uint32_t(W), uint32_t(rows), uint32_t(imgs)};
+  return make_map(m, base, 4, dims, strides, box);
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------ plans
+struct TcGemm {
+  const char* name;
+  int kind, bn, splits;
+  TcParams p;
+  KernelFn fn;
+  size_t smem;
+  dim3 grid;
+  bool input_A;           // operand fed by the uploaded batch (tensor 0)
+  bool input_B;
+  std::vector<CUtensorMap> slot_maps;  // per slot map of that operand
+  TcContext* ctx;
+};
+
+struct TcContext {
+  std::vector<TcGemm*> gemms;
+  int num_sms = 148;
+  int slot = 0;
+  int* err = nullptr;
+  float* ws = nullptr;
+  size_t ws_floats = 0;
+  fo_server* s = nullptr;
+};
+
+namespace {
+
+bool window_ok(int N, int H, int W, int rows_needed, int* rows, int* imgs) {
+  // A box of `rows_needed` pixels made of whole image rows (and whole images
+  // when it spans several).
+  if (W > 256 || rows_needed % W) return false;
+  int r = rows_needed / W;
+  if (r <= H) {
+    if (H % r) return false;
+    *rows = r;
+    *imgs = 1;
+  } else {
+    if (r % H) return false;
+    *rows = H;
+    *imgs = r / H;
+    if (*imgs > 256) return false;
+  }
+  (void)N;
+  return true;
+}
+
+int pick_bn(int N) {
+  if (N % 256 == 0) return 256;
+  if (N % 128 == 0) return 128;
+  if (N % 64 == 0) return 64;
   return 0;
 }
-void tc_destroy(TcContext* c) { delete c; }
-void tc_set_input(TcContext*, int) {}
-TcGemm* tc_plan_forward(TcContext*, fo_server*, int) { return nullptr; }
-TcGemm* tc_plan_dgrad(TcContext*, fo_server*, int, int) { return nullptr; }
-TcGemm* tc_plan_wgrad(TcContext*, fo_server*, int) { return nullptr; }
-void tc_run(TcGemm*, const void*, cudaStream_t) {}
-const char* tc_name(const TcGemm*) { return "tc"; }
+
+void choose_split(TcContext* c, TcGemm* g, int tiles, int KB) {
+  int want = std::max(1, c->num_sms / std::max(1, tiles));
+  want = std::min(want, std::max(1, KB / 4));
+  int kper = (KB + want - 1) / want;
+  g->splits = (KB + kper - 1) / kper;
+  g->p.kper = kper;
+  g->p.KB = KB;
+}
+
+TcGemm* finish(TcContext* c, TcGemm* g, int M, int N) {
+  g->p.M = M;
+  g->p.N = N;
+  g->p.err = c->err;
+  g->fn = pick_kernel(g->kind, g->bn, &g->smem);
+  if (!g->fn) {
+    delete g;
+    return nullptr;
+  }
+  if (cudaFuncSetAttribute(g->fn, cudaFuncAttributeMaxDynamicSharedMemorySize, int(g->smem)) != cudaSuccess) {
+    delete g;
+    return nullptr;
+  }
+  g->grid = dim3(N / g->bn, (M + BM - 1) / BM, g->splits);
+  if (g->splits > 1) {
+    size_t need = size_t(g->splits) * M * N;
+    c->ws_floats = std::max(c->ws_floats, need);
+  }
+  g->ctx = c;
+  c->gemms.push_back(g);
+  return g;
+}
+
+bool bf16_server(const fo_server* s) { return s->dt == kBF16; }
+
+}  // namespace
+
+int tc_create(TcContext** out, fo_server* s) {
+  TcContext* c = new TcContext();
+  c->s = s;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, dev);
+  c->err = (int*)s->alloc(sizeof(int) * 4);
+  if (!c->err) {
+    delete c;
+    return FO_ERR_OOM;
+  }
+  cudaMemset(c->err, 0, sizeof(int) * 4);
+  *out = c;
+  return FO_OK;
+}
+
+void tc_destroy(TcContext* c) {
+  if (!c) return;
+  for (TcGemm* g : c->gemms) delete g;
+  delete c;
+}
+
+void tc_set_input(TcContext* c, int slot) {
+  if (c) c->slot = slot;
+}
+
+int* tc_error_word(TcContext* c) { return c ? c->err : nullptr; }
+
+// Allocate the split-K workspace once every plan is known.
+int tc_finalize(TcContext* c) {
+  if (!c) return FO_OK;
+  if (c->ws_floats) {
+    c->ws = (float*)c->s->alloc(c->ws_floats * sizeof(float));
+    if (!c->ws) return FO_ERR_OOM;
+  }
+  for (TcGemm* g : c->gemms)
+    if (g->splits > 1) g->p.ws = c->ws;
+  return FO_OK;
+}
+
+static const void* tensor_act(fo_server* s, int tid) { return s->T[tid].act; }
+
+TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i) {
+  if (!c || !bf16_server(s) || getenv("FO_NO_TC")) return nullptr;
+  const fo_op& op = s->ops[i];
+  const Tensor& a = s->T[op.in0];
+  const Tensor& o = s->T[i + 1];
+  if (o.dt != kBF16) return nullptr;  // fp32 logits: CUDA-core path
+  TcGemm* g = new TcGemm();
+  g->p.out = o.act;
+  g->p.ldo = o.C;
+  g->p.bias = op.bias ? s->theta + s->segs[s->op_segs[i][1]].off : nullptr;
+  const bf16* w = s->shadow + s->segs[s->op_segs[i][0]].off;
+  if (op.kind == FO_OP_LINEAR) {
+    int bn = pick_bn(op.cout);
+    if (!bn || op.cin % 64) { delete g; return nullptr; }
+    g->kind = LIN_FWD;
+    g->bn = bn;
+    g->name = "tc_linear_fwd";
+    int M = int(a.rows()), KB = op.cin / 64;
+    choose_split(c, g, (M + BM - 1) / BM * (op.cout / bn), KB);
+    g->input_A = (op.in0 == 0);
+    if (g->input_A) {
+      g->slot_maps.resize(s->cfg.omega);
+      for (int sl = 0; sl < s->cfg.omega; ++sl)
+        if (!map_2d(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, M, op.cin, BM)) { delete g; return nullptr; }
+    } else if (!map_2d(&g->p.tmA, tensor_act(s, op.in0), M, op.cin, BM)) { delete g; return nullptr; }
+    if (!map_2d(&g->p.tmB, w, op.cout, op.cin, bn)) { delete g; return nullptr; }
+    return finish(c, g, M, op.cout);
+  }
+  // convolution: 3x3 (or 1x1) stride 1
+  if (op.stride != 1 || op.cin % 64 || op.cout % 64) { delete g; return nullptr; }
+  int rows, imgs;
+  if (!window_ok(a.N, a.H, a.W, BM, &rows, &imgs) || (int64_t(a.N) * a.H * a.W) % BM) { delete g; return nullptr; }
+  int bn = pick_bn(op.cout);
+  g->kind = CONV_FPROP;
+  g->bn = bn;
+  g->name = "tc_conv_fprop";
+  g->p.H = a.H; g->p.W = a.W; g->p.ksz = op.k; g->p.pad = op.k / 2; g->p.taps = op.k * op.k;
+  g->p.cblocks = op.cin / 64;
+  g->p.ntap_ch = op.cin;
+  g->p.win_rows = rows; g->p.win_imgs = imgs;
+  int M = a.N * a.H * a.W, KB = g->p.taps * g->p.cblocks;
+  choose_split(c, g, M / BM * (op.cout / bn), KB);
+  g->input_A = (op.in0 == 0);
+  if (g->input_A) {
+    g->slot_maps.resize(s->cfg.omega);
+    for (int sl = 0; sl < s->cfg.omega; ++sl)
+      if (!map_window(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, a.N, a.H, a.W, a.C, rows, imgs)) { delete g; return nullptr; }
+  } else if (!map_window(&g->p.tmA, tensor_act(s, op.in0), a.N, a.H, a.W, a.C, rows, imgs)) { delete g; return nullptr; }
+  if (!map_2d(&g->p.tmB, w, op.cout, int64_t(g->p.taps) * op.cin, bn)) { delete g; return nullptr; }
+  return finish(c, g, M, op.cout);
+}
+
+TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate) {
+  if (!c || !bf16_server(s) || getenv("FO_NO_TC")) return nullptr;
+  const fo_op& op = s->ops[i];
+  const Tensor& a = s->T[op.in0];
+  const Tensor& o = s->T[i + 1];
+  if (o.dt != kBF16) return nullptr;
+  TcGemm* g = new TcGemm();
+  g->p.out = a.grad;
+  g->p.ldo = a.C;
+  g->p.acc = accumulate;
+  const bf16* w = s->shadow + s->segs[s->op_segs[i][0]].off;
+  if (op.kind == FO_OP_LINEAR) {
+    int bn = pick_bn(op.cin);
+    if (!bn || op.cout % 64) { delete g; return nullptr; }
+    g->kind = LIN_DGRAD;
+    g->bn = bn;
+    g->name = "tc_linear_dgrad";
+    int M = int(a.rows()), KB = op.cout / 64;
+    choose_split(c, g, (M + BM - 1) / BM * (op.cin / bn), KB);
+    if (!map_2d(&g->p.tmA, o.grad, M, op.cout, BM) || !map_2d(&g->p.tmB, w, op.cout, op.cin, BK)) { delete g; return nullptr; }
+    return finish(c, g, M, op.cin);
+  }
+  if (op.stride != 1 || op.cin % 64 || op.cout % 64) { delete g; return nullptr; }
+  int rows, imgs;
+  if (!window_ok(o.N, o.H, o.W, BM, &rows, &imgs) || (int64_t(a.N) * a.H * a.W) % BM) { delete g; return nullptr; }
+  int bn = pick_bn(op.cin);
+  g->kind = CONV_DGRAD;
+  g->bn = bn;
+  g->name = "tc_conv_dgrad";
+  g->p.H = o.H; g->p.W = o.W; g->p.ksz = op.k; g->p.pad = op.k / 2; g->p.taps = op.k * op.k;
+  g->p.cblocks = op.cout / 64;
+  g->p.ntap_ch = op.cin;
+  int M = a.N * a.H * a.W, KB = g->p.taps * g->p.cblocks;
+  choose_split(c, g, M / BM * (op.cin / bn), KB);
+  if (!map_window(&g->p.tmA, o.grad, o.N, o.H, o.W, o.C, rows, imgs) ||
+      !map_2d(&g->p.tmB, w, op.cout, int64_t(g->p.taps) * op.cin, BK)) { delete g; return nullptr; }
+  return finish(c, g, M, op.cin);
+}
+
+TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
+  if (!c || !bf16_server(s) || getenv("FO_NO_TC")) return nullptr;
+  const fo_op& op = s->ops[i];
+  const Tensor& a = s->T[op.in0];
+  const Tensor& o = s->T[i + 1];
+  if (o.dt != kBF16) return nullptr;
+  TcGemm* g = new TcGemm();
+  g->p.out = s->grad + s->segs[s->op_segs[i][0]].off;
+  g->p.out_f32 = 1;
+  if (op.kind == FO_OP_LINEAR) {
+    int bn = pick_bn(op.cin);
+    if (!bn || op.cout % 128) { delete g; return nullptr; }
+    g->kind = LIN_WGRAD;
+    g->bn = bn;
+    g->name = "tc_linear_wgrad";
+    g->p.ldo = op.cin;
+    int rows = int(a.rows()), KB = (rows + BK - 1) / BK;
+    choose_split(c, g, op.cout / BM * (op.cin / bn), KB);
+    g->input_B = (op.in0 == 0);
+    if (!map_2d(&g->p.tmA, o.grad, rows, op.cout, BK)) { delete g; return nullptr; }
+    if (g->input_B) {
+      g->slot_maps.resize(s->cfg.omega);
+      for (int sl = 0; sl < s->cfg.omega; ++sl)
+        if (!map_2d(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, rows, op.cin, BK)) { delete g; return nullptr; }
+    } else if (!map_2d(&g->p.tmB, tensor_act(s, op.in0), rows, op.cin, BK)) { delete g; return nullptr; }
+    return finish(c, g, op.cout, op.cin);
+  }
+  if (op.stride != 1 || op.cin % 64 || op.cout % 128) { delete g; return nullptr; }
+  int rows, imgs;
+  if (!window_ok(a.N, a.H, a.W, BK, &rows, &imgs) || (int64_t(a.N) * a.H * a.W) % BK) { delete g; return nullptr; }
+  int bn = op.cin % 256 == 0 ? 256 : (op.cin % 128 == 0 ? 128 : 64);
+  g->kind = CONV_WGRAD;
+  g->bn = bn;
+  g->name = "tc_conv_wgrad";
+  g->p.ldo = op.k * op.k * op.cin;
+  g->p.H = a.H; g->p.W = a.W; g->p.ksz = op.k; g->p.pad = op.k / 2; g->p.taps = op.k * op.k;
+  g->p.ntap_ch = op.cin;
+  int P = a.N * a.H * a.W, KB = P / BK;
+  int N = g->p.taps * op.cin;
+  choose_split(c, g, op.cout / BM * (N / bn), KB);
+  g->input_B = (op.in0 == 0);
+  if (!map_2d(&g->p.tmA, o.grad, P, op.cout, BK)) { delete g; return nullptr; }
+  if (g->input_B) {
+    g->slot_maps.resize(s->cfg.omega);
+    for (int sl = 0; sl < s->cfg.omega; ++sl)
+      if (!map_window(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, a.N, a.H, a.W, a.C, rows, imgs)) { delete g; return nullptr; }
+  } else if (!map_window(&g->p.tmB, tensor_act(s, op.in0), a.N, a.H, a.W, a.C, rows, imgs)) { delete g; return nullptr; }
+  return finish(c, g, op.cout, N);
+}
+
+void tc_run(TcGemm* g, const void* input, cudaStream_t st) {
+  (void)input;
+  TcContext* c = g->ctx;
+  if (g->input_A) g->p.tmA = g->slot_maps[c->slot];
+  if (g->input_B) g->p.tmB = g->slot_maps[c->slot];
+  g->fn<<<g->grid, kThreads, g->smem, st>>>(g->p);
+  if (g->splits > 1) {
+    TcParams& p = g->p;
+    int64_t n4 = int64_t(p.M) * p.N / 4;
+    splitk_reduce_k<<<elementwise_blocks(n4, 256), 256, 0, st>>>(p.ws, g->splits, p.M, p.N, p.out, p.ldo, p.bias,
+                                                                  p.relu, p.acc, p.out_f32);
+  }
+}
+
+const char* tc_name(const TcGemm* g) { return g->name; }
 
 }  // namespace fo

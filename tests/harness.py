@@ -70,3 +70,73 @@ def normwise(a, b):
     a = np.asarray(a, np.float64)
     b = np.asarray(b, np.float64)
     return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-300))
+
+
+def param_slices(ops):
+    out, off = [], 0
+    for i, name, shape in O.param_shapes(ops):
+        n = int(np.prod(shape))
+        out.append((f"{i}:{ops[i]['kind']}.{name}", slice(off, off + n)))
+        off += n
+    return out
+
+
+def teacher_forced(cfg, events, max_steps=None):
+    """GPU and oracle in lockstep: before every step the oracle takes the
+    GPU's theta and momentum, then both run the same scheduled batch.  Two
+    oracle readings run side by side: the exact fp64 definition, and the
+    bf16-storage reading (the kernel's precision for every stored tensor, so
+    that ReLU / max-pool decisions are taken alike).  Returns per-step records
+    with the loss, parameter and per-tensor gradient errors against each
+    (gradient recovered exactly as g = v_new - mu v_old)."""
+    from paper_2504_13850_gb300 import api
+    s = api.Server.from_config(cfg)
+    theta0 = W.init_params(cfg)
+    s.set_params(theta0)
+    storage = "bf16" if cfg["dtype"] == W.BF16 else None
+    mk = lambda st: O.Server(cfg["ops"], cfg["K"], cfg["omega"], cfg["depth"], theta0, cfg["lr"],
+                             cfg["momentum"], storage=st)
+    o, ob = mk(None), mk(storage)
+    mu = cfg["momentum"]
+    nb, recs, steps = {}, [], 0
+    slices = param_slices(cfg["ops"])
+    for ev in events:
+        if ev[0] == "enq":
+            k = ev[1]
+            j = nb.get(k, 0)
+            nb[k] = j + 1
+            x, up, labels, lengths = batch_for(cfg, k, j)
+            g_out = s.enqueue_activations(k, up, labels, lengths)
+            o_rc, _ = o.enqueue(k, x, labels, lengths)
+            ob.enqueue(k, x, labels, lengths)
+            assert (g_out[0], g_out[1]) == (o_rc, int(o.sched.on[k]))
+            continue
+        if max_steps is not None and steps >= max_steps:
+            break
+        th0 = s.get_params().astype(np.float64)
+        v0 = s.get_momentum().astype(np.float64)
+        for srv in (o, ob):
+            srv.theta, srv.v = th0.copy(), v0.copy()
+        g_rc, gk, gslot = s.server_step()
+        o_rc, ok, oslot = o.step()
+        ob.step()
+        assert (g_rc, gk, gslot) == (o_rc, ok, oslot)
+        if g_rc != api.OK:
+            continue
+        loss = float(s.read_losses(steps, 1)[0])
+        th1 = s.get_params().astype(np.float64)
+        v1 = s.get_momentum().astype(np.float64)
+        g_gpu = v1 - mu * v0
+        rec = {"step": steps, "loss": loss}
+        for tag, srv in (("exact", o), ("stored", ob)):
+            g_ref = srv.v - mu * v0
+            rec[tag] = {
+                "loss": srv.losses[-1],
+                "param_err": normwise(th1, srv.theta),
+                "update_err": normwise(th1 - th0, srv.theta - th0),
+                "grad_err": normwise(g_gpu, g_ref),
+                "tensor_grad_err": {n: normwise(g_gpu[sl], g_ref[sl]) for n, sl in slices},
+            }
+        recs.append(rec)
+        steps += 1
+    return s, o, recs

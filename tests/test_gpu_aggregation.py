@@ -32,23 +32,30 @@ def check(gpu, ref, g_old, l):
 
 
 def test_tiny_config_each_device_once_is_running_mean():
+    """Each device's model once, all trained from version 0: per step the GPU
+    result is checked elementwise against Algorithm 4 applied to the GPU's own
+    previous global (teacher forced), and the whole chain normwise against the
+    oracle's chain and the closed form (running mean of the locals)."""
     cfg = W.CONFIGS["tiny"]
     n = cfg["agg_params"]
     s = tiny_server()
     g0 = W.global_model(n, cfg["seed"])
     gd = torch.tensor(g0, device="cuda")
-    agg = O.Aggregator(cfg["K"], 2**31 - 1)
-    g_ref = g0.astype(np.float64)
+    chain = O.Aggregator(cfg["K"], 2**31 - 1)
+    g_chain = g0.astype(np.float64)
     locs = []
     for k in range(cfg["K"]):
         l = W.device_model(n, cfg["seed"], k, 0)
         locs.append(l)
         g_before = gd.cpu().numpy().astype(np.float64)
+        step = O.Aggregator(cfg["K"], 2**31 - 1)
+        step.t = k
+        _, ref = step.aggregate(g_before, l, 0)
         rc, t = s.aggregate(gd, torch.tensor(l, device="cuda"), k, 0)
         assert rc == api.OK and t == k + 1
-        st, g_ref = agg.aggregate(g_ref, l, 0)
-        check(gd.cpu().numpy(), g_ref, g_before, l)
-        # closed form: the mean of the first k+1 locals
+        check(gd.cpu().numpy(), ref, g_before, l)
+        _, g_chain = chain.aggregate(g_chain, l, 0)
+        assert normwise(gd.cpu().numpy(), g_chain) <= 1e-6
         assert normwise(gd.cpu().numpy(), np.mean(np.array(locs, np.float64), 0)) <= 1e-6
     assert s.version() == (4, 1)
 

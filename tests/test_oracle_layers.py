@@ -291,3 +291,38 @@ def test_sgd_momentum_constant_gradient_closed_form():
     # theta_n = theta_0 - lr * g * sum_{i=1..n} (1 - mu^i)/(1 - mu)
     s = sum((1 - mu ** i) / (1 - mu) for i in range(1, 21))
     assert np.allclose(th, theta0 - lr * g * s, rtol=1e-13)
+
+
+# --------------------------------------------------------------------------
+# bf16 storage reading
+# --------------------------------------------------------------------------
+
+def test_to_bf16_matches_bit_rounding_and_torch():
+    import torch
+    r = rng(20)
+    x = (r.standard_normal(10000) * np.exp(r.uniform(-20, 20, 10000))).astype(np.float32)
+    ref_bits, _ = W.round_to_bf16(x)[0], None
+    assert np.array_equal(O.to_bf16(x.astype(np.float64)), ref_bits.astype(np.float64))
+    t = torch.tensor(x).to(torch.bfloat16).to(torch.float64).numpy()
+    assert np.array_equal(O.to_bf16(x.astype(np.float64)), t)
+
+
+def test_to_bf16_ties_to_even():
+    one = 1.0
+    assert O.to_bf16(np.array([one + 2.0 ** -8]))[0] == 1.0               # tie -> even (1.0)
+    assert O.to_bf16(np.array([one + 3 * 2.0 ** -8]))[0] == 1.0 + 2.0 ** -6  # tie -> even
+    assert O.to_bf16(np.array([one + 2.0 ** -8 + 2.0 ** -30]))[0] == 1.0 + 2.0 ** -7
+    assert O.to_bf16(np.array([0.0, -0.0]))[1] == 0.0
+
+
+def test_bf16_storage_rounds_every_stored_tensor():
+    from test_oracle_network import make_case
+    ops, theta, x, labels, lengths = make_case("vgg")
+    params = O.unflatten(ops, theta)
+    T, _ = O.forward(ops, params, O.to_bf16(x), lengths, storage="bf16")
+    for t in T[1:-1]:
+        assert np.array_equal(O.to_bf16(t), t)
+    assert not np.array_equal(O.to_bf16(T[-1]), T[-1])     # logits stay unrounded
+    T64, _ = O.forward(ops, params, O.to_bf16(x), lengths)
+    rel = np.linalg.norm(T[-1] - T64[-1]) / np.linalg.norm(T64[-1])
+    assert 1e-5 < rel < 3e-2
