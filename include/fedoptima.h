@@ -188,17 +188,28 @@ FO_API int fo_server_synchronize(fo_server* s);
 /* The compute stream (a cudaStream_t) the step and aggregation kernels run
  * on, for callers that time them with CUDA events. */
 FO_API void* fo_server_stream(const fo_server* s);
-/* Kernel launches the last fo_server_step enqueued. */
+/* Kernel launches the last fo_server_step enqueued, and all kernels the
+ * server has launched since creation (steps and aggregations). */
 FO_API int fo_server_last_step_launches(const fo_server* s);
+FO_API int64_t fo_server_kernels_launched(const fo_server* s);
+/* Device bytes the server allocated (parameters, momentum, gradient, bf16
+ * shadow, activation slab, intermediate tensors, scratch). */
+FO_API int64_t fo_server_device_bytes(const fo_server* s);
+/* Waits for the compute stream and reports FO_ERR_TIMEOUT if a tensor-core
+ * kernel gave up a bounded wait since creation (FO_OK otherwise). */
+FO_API int fo_server_error(fo_server* s);
 
-/* Optional per-kernel timing of fo_server_step: when enabled, each launch of
- * the step is bracketed by CUDA events on the compute stream.
- * fo_server_kernel_times fills up to `cap` entries with the name (static
- * string), launch count and summed milliseconds of every kernel class seen
- * since profiling was enabled (waits for the stream). */
+/* Optional per-kernel timing of fo_server_step and fo_aggregate: when
+ * enabled, each launch is bracketed by CUDA events on the compute stream.
+ * fo_server_kernel_times fills up to `cap` entries (any output array may be
+ * NULL) with the name (static string), kernel launches, summed milliseconds
+ * and summed algorithmic FLOPs and HBM bytes of every kernel class seen since
+ * profiling was enabled or reset (waits for the stream); *n_out receives the
+ * number of classes. */
 FO_API int fo_server_profile(fo_server* s, int enable);
+FO_API int fo_server_profile_reset(fo_server* s);
 FO_API int fo_server_kernel_times(fo_server* s, const char** names, int64_t* launches,
-                           double* ms, int cap, int* n_out);
+                           double* ms, double* flops, double* bytes, int cap, int* n_out);
 
 FO_API const char* fo_last_error(void);
 

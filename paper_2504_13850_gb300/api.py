@@ -74,7 +74,12 @@ _SIGS = [
     ("fo_server_last_step_launches", C.c_int, [C.c_void_p]),
     ("fo_server_profile", C.c_int, [C.c_void_p, C.c_int]),
     ("fo_server_kernel_times", C.c_int, [C.c_void_p, C.POINTER(C.c_char_p), C.POINTER(C.c_int64),
+                                         C.POINTER(C.c_double), C.POINTER(C.c_double),
                                          C.POINTER(C.c_double), C.c_int, C.POINTER(C.c_int)]),
+    ("fo_server_profile_reset", C.c_int, [C.c_void_p]),
+    ("fo_server_kernels_launched", C.c_int64, [C.c_void_p]),
+    ("fo_server_device_bytes", C.c_int64, [C.c_void_p]),
+    ("fo_server_error", C.c_int, [C.c_void_p]),
     ("fo_last_error", C.c_char_p, []),
     ("fo_sched_create", C.c_int, [C.c_int, C.c_int, C.c_int, C.c_int, C.POINTER(C.c_void_p)]),
     ("fo_sched_destroy", C.c_int, [C.c_void_p]),
@@ -270,14 +275,30 @@ class Server:
         _check(lib().fo_server_profile(self.h, 1 if enable else 0), "profile")
 
     def kernel_times(self):
+        """{name: (kernel launches, ms, algorithmic FLOPs, algorithmic bytes)}"""
         cap = 256
         names = (C.c_char_p * cap)()
         launches = (C.c_int64 * cap)()
         ms = (C.c_double * cap)()
+        fl = (C.c_double * cap)()
+        by = (C.c_double * cap)()
         n = C.c_int()
-        _check(lib().fo_server_kernel_times(self.h, names, launches, ms, cap, C.byref(n)),
+        _check(lib().fo_server_kernel_times(self.h, names, launches, ms, fl, by, cap, C.byref(n)),
                "kernel_times")
-        return {names[i].decode(): (int(launches[i]), float(ms[i])) for i in range(min(n.value, cap))}
+        return {names[i].decode(): (int(launches[i]), float(ms[i]), float(fl[i]), float(by[i]))
+                for i in range(min(n.value, cap))}
+
+    def profile_reset(self):
+        _check(lib().fo_server_profile_reset(self.h), "profile_reset")
+
+    def kernels_launched(self):
+        return lib().fo_server_kernels_launched(self.h)
+
+    def device_bytes(self):
+        return lib().fo_server_device_bytes(self.h)
+
+    def check_error(self):
+        _check(lib().fo_server_error(self.h), "server_error")
 
 
 class Scheduler:

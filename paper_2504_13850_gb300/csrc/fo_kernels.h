@@ -84,5 +84,7 @@ void f32_to_bf16(const float* x, void* y, int64_t n, cudaStream_t st);
 
 // FedAsync update: g = fmaf(alpha, l - g, g).
 void axpby(float* g, const float* l, int64_t n, float alpha, cudaStream_t st);
+// Number of kernels axpby launches for these arguments (vector body, tail).
+int axpby_kernels(const float* g, const float* l, int64_t n);
 
 }  // namespace fo

@@ -158,110 +158,124 @@ fo::ConvShape conv_shape(const fo_server* s, int i) {
   return {a.N, a.H, a.W, op.cin, op.cout, op.k, op.stride, op.k / 2, o.H, o.W};
 }
 
-// Build the list of launches of one server step.
+// Build the list of launches of one server step.  Every entry records how
+// many kernels it launches and its algorithmic FLOPs / HBM bytes (the
+// minimum a kernel of that job must move), for the per-kernel roofline.
 int build_plan(fo_server* s) {
   const int nops = int(s->ops.size());
   const int dt = s->dt;
+  const double esz = dt == fo::kF32 ? 4.0 : 2.0;
   auto& plan = s->plan;
   plan.clear();
   auto act = [s](int tid) -> const void* { return tid == 0 ? s->cur_in : s->T[tid].act; };
+  auto add = [&plan](const char* name, int kernels, double flops, double bytes,
+                     std::function<void(cudaStream_t)> fn) {
+    plan.push_back({name, std::move(fn), kernels, flops, bytes});
+  };
+  auto tbytes = [s](int tid) { return double(s->T[tid].bytes()); };
+  auto add_tc = [&](fo::TcGemm* g, const void* in) {
+    add(fo::tc_name(g), 1, fo::tc_flops(g), 0.0, [=](cudaStream_t st) { fo::tc_run(g, in, st); });
+    if (fo::tc_splits(g) > 1)
+      add("splitk_reduce", 1, 0.0, fo::tc_reduce_bytes(g), [=](cudaStream_t st) { fo::tc_run_reduce(g, st); });
+  };
 
   // ---------------- forward
   for (int i = 0; i < nops; ++i) {
     const fo_op op = s->ops[i];
     const int a = op.in0, o = i + 1;
     const Tensor& ta = s->T[a];
-    Tensor& to = s->T[o];
+    const Tensor& to = s->T[o];
     switch (op.kind) {
       case FO_OP_CONV:
       case FO_OP_LINEAR: {
         fo::ConvShape cs = conv_shape(s, i);
         const bool bias = op.bias != 0;
+        const double fl = 2.0 * double(to.rows()) * op.cout * double(op.kind == FO_OP_CONV ? op.k * op.k : 1) * op.cin;
         fo::TcGemm* tg = fo::tc_plan_forward(s->tc, s, i);
         if (tg) {
-          plan.push_back({fo::tc_name(tg), [=](cudaStream_t st) { fo::tc_run(tg, act(a), st); }});
+          const int in = a;
+          add_tc(tg, nullptr);
+          (void)in;
+          // the first layer reads the batch slot: its tensor map is chosen per step
         } else {
           // Hidden layers of the bf16 path multiply bf16 weights (the shadow);
           // the fp32 path and the fp32 logits layer use the fp32 master.
           const int dto = to.dt;
           const bool wbf = dto == fo::kBF16;
-          plan.push_back({op.kind == FO_OP_CONV ? "conv_fwd_simt" : "linear_fwd_simt",
-                          [=](cudaStream_t st) {
-                            const void* w = wbf ? (const void*)SH(s, i, 0) : (const void*)P(s, i, 0);
-                            fo::conv_fwd_simt(cs, act(a), ta.dt, w, wbf ? fo::kBF16 : fo::kF32,
-                                              bias ? P(s, i, 1) : nullptr, s->T[o].act, dto, false, st);
-                          }});
+          add(op.kind == FO_OP_CONV ? "conv_fwd_simt" : "linear_fwd_simt", 1, fl, 0.0, [=](cudaStream_t st) {
+            const void* w = wbf ? (const void*)SH(s, i, 0) : (const void*)P(s, i, 0);
+            fo::conv_fwd_simt(cs, act(a), ta.dt, w, wbf ? fo::kBF16 : fo::kF32, bias ? P(s, i, 1) : nullptr,
+                              s->T[o].act, dto, false, st);
+          });
         }
         break;
       }
       case FO_OP_AFFINE:
-        plan.push_back({"affine_fwd", [=](cudaStream_t st) {
-                          fo::affine_fwd(act(a), P(s, i, 0), P(s, i, 1), s->T[o].act, s->T[a].rows(),
-                                         s->T[a].C, dt, st);
-                        }});
+        add("affine_fwd", 1, 0.0, 2 * tbytes(a), [=](cudaStream_t st) {
+          fo::affine_fwd(act(a), P(s, i, 0), P(s, i, 1), s->T[o].act, s->T[a].rows(), s->T[a].C, dt, st);
+        });
         break;
       case FO_OP_RELU:
-        plan.push_back({"relu_fwd", [=](cudaStream_t st) {
-                          fo::relu_fwd(act(a), s->T[o].act, s->T[a].numel(), dt, st);
-                        }});
+        add("relu_fwd", 1, 0.0, 2 * tbytes(a), [=](cudaStream_t st) {
+          fo::relu_fwd(act(a), s->T[o].act, s->T[a].numel(), dt, st);
+        });
         break;
       case FO_OP_MAXPOOL2:
-        plan.push_back({"maxpool2_fwd", [=](cudaStream_t st) {
-                          const Tensor& x = s->T[a];
-                          fo::maxpool2_fwd(act(a), s->T[o].act, x.N, x.H, x.W, x.C, dt, st);
-                        }});
+        add("maxpool2_fwd", 1, 0.0, tbytes(a) + tbytes(o), [=](cudaStream_t st) {
+          const Tensor& x = s->T[a];
+          fo::maxpool2_fwd(act(a), s->T[o].act, x.N, x.H, x.W, x.C, dt, st);
+        });
         break;
       case FO_OP_ADD: {
         const int b = op.in1;
-        plan.push_back({"add_fwd", [=](cudaStream_t st) {
-                          fo::add_fwd(act(a), act(b), s->T[o].act, s->T[o].numel(), dt, st);
-                        }});
+        add("add_fwd", 1, 0.0, 3 * tbytes(o), [=](cudaStream_t st) {
+          fo::add_fwd(act(a), act(b), s->T[o].act, s->T[o].numel(), dt, st);
+        });
         break;
       }
       case FO_OP_AVGPOOL:
-        plan.push_back({"avgpool_fwd", [=](cudaStream_t st) {
-                          const Tensor& x = s->T[a];
-                          fo::avgpool_fwd(act(a), s->T[o].act, x.N, x.H * x.W, x.C, dt, st);
-                        }});
+        add("avgpool_fwd", 1, 0.0, tbytes(a) + tbytes(o), [=](cudaStream_t st) {
+          const Tensor& x = s->T[a];
+          fo::avgpool_fwd(act(a), s->T[o].act, x.N, x.H * x.W, x.C, dt, st);
+        });
         break;
       case FO_OP_FLATTEN:
         break;  // a view
       case FO_OP_LAYERNORM:
-        plan.push_back({"layernorm_fwd", [=](cudaStream_t st) {
-                          fo::layernorm_fwd(act(a), P(s, i, 0), P(s, i, 1), s->T[o].act, s->ln_mean[i],
-                                            s->ln_rstd[i], s->T[a].rows(), s->T[a].C, dt, st);
-                        }});
+        add("layernorm_fwd", 1, 0.0, 2 * tbytes(a), [=](cudaStream_t st) {
+          fo::layernorm_fwd(act(a), P(s, i, 0), P(s, i, 1), s->T[o].act, s->ln_mean[i], s->ln_rstd[i],
+                            s->T[a].rows(), s->T[a].C, dt, st);
+        });
         break;
       case FO_OP_GELU:
-        plan.push_back({"gelu_fwd", [=](cudaStream_t st) {
-                          fo::gelu_fwd(act(a), s->T[o].act, s->T[a].numel(), dt, st);
-                        }});
+        add("gelu_fwd", 1, 0.0, 2 * tbytes(a), [=](cudaStream_t st) {
+          fo::gelu_fwd(act(a), s->T[o].act, s->T[a].numel(), dt, st);
+        });
         break;
-      case FO_OP_ATTENTION:
-        plan.push_back({"attention_fwd", [=](cudaStream_t st) {
-                          const Tensor& x = s->T[a];
-                          fo::attention_fwd(act(a), s->cur_len, s->T[o].act, s->attn_probs[i], x.N, x.H,
-                                            op.cin, op.heads, dt, st);
-                        }});
+      case FO_OP_ATTENTION: {
+        const double L = ta.H, heads = op.heads, dh = double(op.cin) / op.heads;
+        add("attention_fwd", 1, 4.0 * ta.N * heads * L * L * dh, tbytes(a) + tbytes(o), [=](cudaStream_t st) {
+          const Tensor& x = s->T[a];
+          fo::attention_fwd(act(a), s->cur_len, s->T[o].act, s->attn_probs[i], x.N, x.H, op.cin, op.heads, dt, st);
+        });
         break;
+      }
       case FO_OP_MEANPOOL:
-        plan.push_back({"meanpool_fwd", [=](cudaStream_t st) {
-                          const Tensor& x = s->T[a];
-                          fo::meanpool_fwd(act(a), s->cur_len, s->T[o].act, x.N, x.H, x.C, dt, st);
-                        }});
+        add("meanpool_fwd", 1, 0.0, tbytes(a) + tbytes(o), [=](cudaStream_t st) {
+          const Tensor& x = s->T[a];
+          fo::meanpool_fwd(act(a), s->cur_len, s->T[o].act, x.N, x.H, x.C, dt, st);
+        });
         break;
     }
-    (void)to;
   }
 
   // ---------------- loss (softmax cross-entropy on fp32 logits)
   {
     const int lt = nops;
-    plan.push_back({"softmax_ce", [=](cudaStream_t st) {
-                      fo::softmax_ce((const float*)s->T[lt].act, s->cur_labels, s->cfg.batch,
-                                     s->cfg.num_classes, s->losses + (s->steps_done & (s->kLossRing - 1)),
-                                     s->T[lt].grad, fo::kF32, st);
-                    }});
+    add("softmax_ce", 1, 0.0, 2 * tbytes(lt), [=](cudaStream_t st) {
+      fo::softmax_ce((const float*)s->T[lt].act, s->cur_labels, s->cfg.batch, s->cfg.num_classes,
+                     s->losses + (s->steps_done & (s->kLossRing - 1)), s->T[lt].grad, fo::kF32, st);
+    });
   }
 
   // ---------------- backward
@@ -283,80 +297,78 @@ int build_plan(fo_server* s) {
       // Nothing downstream produced a gradient: zero this op's parameter grads.
       for (int si : s->op_segs[i]) {
         const ParamSeg seg = s->segs[si];
-        plan.push_back({"memset_grad", [=](cudaStream_t st) {
-                          cudaMemsetAsync(s->grad + seg.off, 0, seg.n * sizeof(float), st);
-                        }});
+        add("memset_grad", 1, 0.0, seg.n * 4.0, [=](cudaStream_t st) {
+          cudaMemsetAsync(s->grad + seg.off, 0, seg.n * sizeof(float), st);
+        });
       }
       continue;
     }
     const bool need_dx = a != 0;
+    const double csb = double(s->T[o].rows()) * s->T[o].C * esz;  // one read of dy
     switch (op.kind) {
       case FO_OP_CONV:
       case FO_OP_LINEAR: {
         fo::ConvShape cs = conv_shape(s, i);
         const int dto = s->T[o].dt, dta = s->T[a].dt;
         const bool bias = op.bias != 0;
+        const double fl = 2.0 * double(s->T[o].rows()) * op.cout * double(op.kind == FO_OP_CONV ? op.k * op.k : 1) * op.cin;
         if (bias) {
-          plan.push_back({"bias_grad", [=](cudaStream_t st) {
-                            fo::colsum(s->T[o].grad, nullptr, s->T[o].rows(), s->T[o].C, dto,
-                                       s->colsum_scratch, G(s, i, 1), st);
-                          }});
+          add("bias_grad", 2, 0.0, double(s->T[o].bytes()), [=](cudaStream_t st) {
+            fo::colsum(s->T[o].grad, nullptr, s->T[o].rows(), s->T[o].C, dto, s->colsum_scratch, G(s, i, 1), st);
+          });
         }
         if (need_dx) {
           int accf = contrib(a);
           fo::TcGemm* tg = fo::tc_plan_dgrad(s->tc, s, i, accf);
           if (tg) {
-            plan.push_back({fo::tc_name(tg), [=](cudaStream_t st) { fo::tc_run(tg, nullptr, st); }});
+            add_tc(tg, nullptr);
           } else {
             const bool wbf = dto == fo::kBF16;
-            plan.push_back({op.kind == FO_OP_CONV ? "conv_dgrad_simt" : "linear_dgrad_simt",
-                            [=](cudaStream_t st) {
-                              const void* w = wbf ? (const void*)SH(s, i, 0) : (const void*)P(s, i, 0);
-                              fo::conv_dgrad_simt(cs, s->T[o].grad, dto, w, wbf ? fo::kBF16 : fo::kF32,
-                                                  s->T[a].grad, dta, accf != 0, st);
-                            }});
+            add(op.kind == FO_OP_CONV ? "conv_dgrad_simt" : "linear_dgrad_simt", 1, fl, 0.0, [=](cudaStream_t st) {
+              const void* w = wbf ? (const void*)SH(s, i, 0) : (const void*)P(s, i, 0);
+              fo::conv_dgrad_simt(cs, s->T[o].grad, dto, w, wbf ? fo::kBF16 : fo::kF32, s->T[a].grad, dta,
+                                  accf != 0, st);
+            });
           }
         }
         fo::TcGemm* tw = fo::tc_plan_wgrad(s->tc, s, i);
         if (tw) {
-          plan.push_back({fo::tc_name(tw), [=](cudaStream_t st) { fo::tc_run(tw, act(a), st); }});
+          add_tc(tw, nullptr);
         } else {
-          plan.push_back({op.kind == FO_OP_CONV ? "conv_wgrad_simt" : "linear_wgrad_simt",
-                          [=](cudaStream_t st) {
-                            fo::conv_wgrad_simt(cs, s->T[o].grad, dto, act(a), dta, G(s, i, 0), st);
-                          }});
+          add(op.kind == FO_OP_CONV ? "conv_wgrad_simt" : "linear_wgrad_simt", 1, fl, 0.0, [=](cudaStream_t st) {
+            fo::conv_wgrad_simt(cs, s->T[o].grad, dto, act(a), dta, G(s, i, 0), st);
+          });
         }
         break;
       }
       case FO_OP_AFFINE:
-        plan.push_back({"affine_pgrad", [=](cudaStream_t st) {
-                          const Tensor& x = s->T[a];
-                          fo::colsum(s->T[o].grad, act(a), x.rows(), x.C, dt, s->colsum_scratch, G(s, i, 0), st);
-                          fo::colsum(s->T[o].grad, nullptr, x.rows(), x.C, dt, s->colsum_scratch, G(s, i, 1), st);
-                        }});
+        add("affine_pgrad", 4, 0.0, 3 * csb, [=](cudaStream_t st) {
+          const Tensor& x = s->T[a];
+          fo::colsum(s->T[o].grad, act(a), x.rows(), x.C, dt, s->colsum_scratch, G(s, i, 0), st);
+          fo::colsum(s->T[o].grad, nullptr, x.rows(), x.C, dt, s->colsum_scratch, G(s, i, 1), st);
+        });
         if (need_dx) {
           int accf = contrib(a);
-          plan.push_back({"affine_dx", [=](cudaStream_t st) {
-                            fo::affine_dx(s->T[o].grad, P(s, i, 0), s->T[a].grad, s->T[a].rows(), s->T[a].C,
-                                          dt, accf != 0, st);
-                          }});
+          add("affine_dx", 1, 0.0, (2 + accf) * csb, [=](cudaStream_t st) {
+            fo::affine_dx(s->T[o].grad, P(s, i, 0), s->T[a].grad, s->T[a].rows(), s->T[a].C, dt, accf != 0, st);
+          });
         }
         break;
       case FO_OP_RELU:
         if (need_dx) {
           int accf = contrib(a);
-          plan.push_back({"relu_bwd", [=](cudaStream_t st) {
-                            fo::relu_bwd(act(a), s->T[o].grad, s->T[a].grad, s->T[a].numel(), dt, accf != 0, st);
-                          }});
+          add("relu_bwd", 1, 0.0, (3 + accf) * csb, [=](cudaStream_t st) {
+            fo::relu_bwd(act(a), s->T[o].grad, s->T[a].grad, s->T[a].numel(), dt, accf != 0, st);
+          });
         }
         break;
       case FO_OP_MAXPOOL2:
         if (need_dx) {
           int accf = contrib(a);
-          plan.push_back({"maxpool2_bwd", [=](cudaStream_t st) {
-                            const Tensor& x = s->T[a];
-                            fo::maxpool2_bwd(act(a), s->T[o].grad, x.grad, x.N, x.H, x.W, x.C, dt, accf != 0, st);
-                          }});
+          add("maxpool2_bwd", 1, 0.0, (2 + accf) * tbytes(a) + csb, [=](cudaStream_t st) {
+            const Tensor& x = s->T[a];
+            fo::maxpool2_bwd(act(a), s->T[o].grad, x.grad, x.N, x.H, x.W, x.C, dt, accf != 0, st);
+          });
         }
         break;
       case FO_OP_ADD: {
@@ -364,74 +376,76 @@ int build_plan(fo_server* s) {
         for (int src : {a, b}) {
           if (src == 0) continue;
           int accf = contrib(src);
-          plan.push_back({"add_bwd", [=](cudaStream_t st) {
-                            fo::copy_or_acc(s->T[o].grad, s->T[src].grad, s->T[o].numel(), dt, accf != 0, st);
-                          }});
+          add("add_bwd", 1, 0.0, (2 + accf) * csb, [=](cudaStream_t st) {
+            fo::copy_or_acc(s->T[o].grad, s->T[src].grad, s->T[o].numel(), dt, accf != 0, st);
+          });
         }
         break;
       }
       case FO_OP_AVGPOOL:
         if (need_dx) {
           int accf = contrib(a);
-          plan.push_back({"avgpool_bwd", [=](cudaStream_t st) {
-                            const Tensor& x = s->T[a];
-                            fo::avgpool_bwd(s->T[o].grad, x.grad, x.N, x.H * x.W, x.C, dt, accf != 0, st);
-                          }});
+          add("avgpool_bwd", 1, 0.0, (1 + accf) * tbytes(a) + csb, [=](cudaStream_t st) {
+            const Tensor& x = s->T[a];
+            fo::avgpool_bwd(s->T[o].grad, x.grad, x.N, x.H * x.W, x.C, dt, accf != 0, st);
+          });
         }
         break;
       case FO_OP_FLATTEN:
         break;  // shares the input's gradient buffer
       case FO_OP_LAYERNORM:
-        plan.push_back({"layernorm_pgrad", [=](cudaStream_t st) {
-                          const Tensor& x = s->T[a];
-                          fo::colsum_lnx(s->T[o].grad, act(a), s->ln_mean[i], s->ln_rstd[i], x.rows(), x.C, dt,
-                                         s->colsum_scratch, G(s, i, 0), st);
-                          fo::colsum(s->T[o].grad, nullptr, x.rows(), x.C, dt, s->colsum_scratch, G(s, i, 1), st);
-                        }});
+        add("layernorm_pgrad", 4, 0.0, 3 * csb, [=](cudaStream_t st) {
+          const Tensor& x = s->T[a];
+          fo::colsum_lnx(s->T[o].grad, act(a), s->ln_mean[i], s->ln_rstd[i], x.rows(), x.C, dt, s->colsum_scratch,
+                         G(s, i, 0), st);
+          fo::colsum(s->T[o].grad, nullptr, x.rows(), x.C, dt, s->colsum_scratch, G(s, i, 1), st);
+        });
         if (need_dx) {
           int accf = contrib(a);
-          plan.push_back({"layernorm_bwd", [=](cudaStream_t st) {
-                            const Tensor& x = s->T[a];
-                            fo::layernorm_bwd_dx(act(a), P(s, i, 0), s->ln_mean[i], s->ln_rstd[i], s->T[o].grad,
-                                                 x.grad, x.rows(), x.C, dt, accf != 0, st);
-                          }});
+          add("layernorm_bwd", 1, 0.0, (3 + accf) * csb, [=](cudaStream_t st) {
+            const Tensor& x = s->T[a];
+            fo::layernorm_bwd_dx(act(a), P(s, i, 0), s->ln_mean[i], s->ln_rstd[i], s->T[o].grad, x.grad, x.rows(),
+                                 x.C, dt, accf != 0, st);
+          });
         }
         break;
       case FO_OP_GELU:
         if (need_dx) {
           int accf = contrib(a);
-          plan.push_back({"gelu_bwd", [=](cudaStream_t st) {
-                            fo::gelu_bwd(act(a), s->T[o].grad, s->T[a].grad, s->T[a].numel(), dt, accf != 0, st);
-                          }});
+          add("gelu_bwd", 1, 0.0, (3 + accf) * csb, [=](cudaStream_t st) {
+            fo::gelu_bwd(act(a), s->T[o].grad, s->T[a].grad, s->T[a].numel(), dt, accf != 0, st);
+          });
         }
         break;
       case FO_OP_ATTENTION:
         if (need_dx) {
           int accf = contrib(a);
-          plan.push_back({"attention_bwd", [=](cudaStream_t st) {
-                            const Tensor& x = s->T[a];
-                            fo::attention_bwd(act(a), s->cur_len, s->attn_probs[i], s->T[o].act, s->T[o].grad,
-                                              x.grad, x.N, x.H, op.cin, op.heads, dt, accf != 0, st);
-                          }});
+          const Tensor& ta = s->T[a];
+          const double L = ta.H, heads = op.heads, dh = double(op.cin) / op.heads;
+          add("attention_bwd", 1, 8.0 * ta.N * heads * L * L * dh, (2 + accf) * tbytes(a) + 2 * csb,
+              [=](cudaStream_t st) {
+                const Tensor& x = s->T[a];
+                fo::attention_bwd(act(a), s->cur_len, s->attn_probs[i], s->T[o].act, s->T[o].grad, x.grad, x.N, x.H,
+                                  op.cin, op.heads, dt, accf != 0, st);
+              });
         }
         break;
       case FO_OP_MEANPOOL:
         if (need_dx) {
           int accf = contrib(a);
-          plan.push_back({"meanpool_bwd", [=](cudaStream_t st) {
-                            const Tensor& x = s->T[a];
-                            fo::meanpool_bwd(s->T[o].grad, s->cur_len, x.grad, x.N, x.H, x.C, dt, accf != 0, st);
-                          }});
+          add("meanpool_bwd", 1, 0.0, (1 + accf) * tbytes(a) + csb, [=](cudaStream_t st) {
+            const Tensor& x = s->T[a];
+            fo::meanpool_bwd(s->T[o].grad, s->cur_len, x.grad, x.N, x.H, x.C, dt, accf != 0, st);
+          });
         }
         break;
     }
   }
 
   // ---------------- optimizer (Algorithm 4: theta_s <- theta_s - gamma_s * update)
-  plan.push_back({"sgd_momentum", [=](cudaStream_t st) {
-                    fo::sgd_momentum(s->theta, s->mom, s->grad, s->shadow, s->n_padded, s->opt.lr,
-                                     s->opt.momentum, st);
-                  }});
+  add("sgd_momentum", 1, 0.0, double(s->n_padded) * (20.0 + (s->shadow ? 2.0 : 0.0)), [=](cudaStream_t st) {
+    fo::sgd_momentum(s->theta, s->mom, s->grad, s->shadow, s->n_padded, s->opt.lr, s->opt.momentum, st);
+  });
   return FO_OK;
 }
 
@@ -526,6 +540,13 @@ void destroy_impl(fo_server* s) {
   if (s->xs) cudaStreamDestroy(s->xs);
   delete s->sched;
   delete s;
+}
+
+int prof_id(fo_server* s, const char* name) {
+  for (size_t q = 0; q < s->prof_names.size(); ++q)
+    if (std::strcmp(s->prof_names[q], name) == 0) return int(q);
+  s->prof_names.push_back(name);
+  return int(s->prof_names.size()) - 1;
 }
 
 cudaEvent_t pool_event(fo_server* s) {
@@ -668,17 +689,7 @@ int fo_server_step(fo_server* s, int* device_used, int32_t* slot_used) {
   int n = 0;
   for (const Launch& l : s->plan) {
     if (s->profiling) {
-      ProfRec r;
-      r.a = pool_event(s);
-      r.b = pool_event(s);
-      int id = -1;
-      for (size_t q = 0; q < s->prof_names.size(); ++q)
-        if (s->prof_names[q] == l.name) id = int(q);
-      if (id < 0) {
-        id = int(s->prof_names.size());
-        s->prof_names.push_back(l.name);
-      }
-      r.name_id = id;
+      ProfRec r{prof_id(s, l.name), pool_event(s), pool_event(s), l.kernels, l.flops, l.bytes};
       cudaEventRecord(r.a, s->cs);
       l.fn(s->cs);
       cudaEventRecord(r.b, s->cs);
@@ -686,8 +697,9 @@ int fo_server_step(fo_server* s, int* device_used, int32_t* slot_used) {
     } else {
       l.fn(s->cs);
     }
-    ++n;
+    n += l.kernels;
   }
+  s->kernels_launched += n;
   FO_CUDA(cudaGetLastError());
   FO_CUDA(cudaEventRecord(s->slot_free[slot], s->cs));
   s->slot_consumed[slot] = 1;
@@ -718,16 +730,9 @@ int fo_aggregate(fo_server* s, float* global, const float* local, int64_t n, int
     return FO_STALE;
   }
   float alpha = 1.0f / float(s->t - version + 1);
+  const int nk = fo::axpby_kernels(global, local, n);
   if (s->profiling) {
-    ProfRec r{0, pool_event(s), pool_event(s)};
-    int id = -1;
-    for (size_t q = 0; q < s->prof_names.size(); ++q)
-      if (std::strcmp(s->prof_names[q], "fedasync_axpby") == 0) id = int(q);
-    if (id < 0) {
-      id = int(s->prof_names.size());
-      s->prof_names.push_back("fedasync_axpby");
-    }
-    r.name_id = id;
+    ProfRec r{prof_id(s, "fedasync_axpby"), pool_event(s), pool_event(s), nk, 0.0, 12.0 * double(n)};
     cudaEventRecord(r.a, s->cs);
     fo::axpby(global, local, n, alpha, s->cs);
     cudaEventRecord(r.b, s->cs);
@@ -735,6 +740,7 @@ int fo_aggregate(fo_server* s, float* global, const float* local, int64_t n, int
   } else {
     fo::axpby(global, local, n, alpha, s->cs);
   }
+  s->kernels_launched += nk;
   FO_CUDA(cudaGetLastError());
   s->t += 1;
   if (new_version) *new_version = s->t;
@@ -782,16 +788,18 @@ int fo_server_profile(fo_server* s, int enable) {
   return FO_OK;
 }
 
-int fo_server_kernel_times(fo_server* s, const char** names, int64_t* launches, double* ms, int cap,
-                           int* n_out) {
+int fo_server_kernel_times(fo_server* s, const char** names, int64_t* launches, double* ms,
+                           double* flops, double* bytes, int cap, int* n_out) {
   if (!s || !n_out) return set_err(FO_ERR_ARG, "null argument");
   FO_CUDA(cudaStreamSynchronize(s->cs));
   for (auto& r : s->prof) {
     float t = 0.f;
     cudaEventElapsedTime(&t, r.a, r.b);
-    auto& acc = s->prof_acc[s->prof_names[r.name_id]];
-    acc.first += 1;
-    acc.second += t;
+    ProfAcc& acc = s->prof_acc[s->prof_names[r.name_id]];
+    acc.launches += r.kernels;
+    acc.ms += t;
+    acc.flops += r.flops;
+    acc.bytes += r.bytes;
     s->ev_pool.push_back(r.a);
     s->ev_pool.push_back(r.b);
   }
@@ -800,13 +808,41 @@ int fo_server_kernel_times(fo_server* s, const char** names, int64_t* launches, 
   for (auto& kv : s->prof_acc) {
     if (n < cap) {
       if (names) names[n] = kv.first;
-      if (launches) launches[n] = kv.second.first;
-      if (ms) ms[n] = kv.second.second;
+      if (launches) launches[n] = kv.second.launches;
+      if (ms) ms[n] = kv.second.ms;
+      if (flops) flops[n] = kv.second.flops;
+      if (bytes) bytes[n] = kv.second.bytes;
     }
     ++n;
   }
   *n_out = n;
   return FO_OK;
+}
+
+int fo_server_profile_reset(fo_server* s) {
+  if (!s) return set_err(FO_ERR_ARG, "null server");
+  FO_CUDA(cudaStreamSynchronize(s->cs));
+  for (auto& r : s->prof) {
+    s->ev_pool.push_back(r.a);
+    s->ev_pool.push_back(r.b);
+  }
+  s->prof.clear();
+  s->prof_acc.clear();
+  return FO_OK;
+}
+
+int64_t fo_server_kernels_launched(const fo_server* s) { return s ? s->kernels_launched : -1; }
+
+int64_t fo_server_device_bytes(const fo_server* s) { return s ? s->device_bytes : -1; }
+
+int fo_server_error(fo_server* s) {
+  if (!s) return set_err(FO_ERR_ARG, "null server");
+  int* w = fo::tc_error_word(s->tc);
+  if (!w) return FO_OK;
+  int h = 0;
+  FO_CUDA(cudaStreamSynchronize(s->cs));
+  FO_CUDA(cudaMemcpy(&h, w, sizeof(int), cudaMemcpyDeviceToHost));
+  return h ? set_err(FO_ERR_TIMEOUT, "a tensor-core kernel timed out waiting (code " + std::to_string(h) + ")") : FO_OK;
 }
 
 int fo_axpby_async(float* global, const float* local, int64_t n, float alpha, void* stream) {

@@ -37,11 +37,21 @@ struct Tensor {
 struct Launch {
   const char* name;
   std::function<void(cudaStream_t)> fn;
+  int kernels;     // kernel launches this entry makes
+  double flops;    // algorithmic FLOPs
+  double bytes;    // algorithmic HBM bytes
 };
 
 struct ProfRec {
   int name_id;
   cudaEvent_t a, b;
+  int kernels;
+  double flops, bytes;
+};
+
+struct ProfAcc {
+  int64_t launches = 0;
+  double ms = 0, flops = 0, bytes = 0;
 };
 
 struct fo_server {
@@ -85,7 +95,9 @@ struct fo_server {
   std::vector<ProfRec> prof;
   std::vector<cudaEvent_t> ev_pool;
   std::vector<const char*> prof_names;
-  std::map<const char*, std::pair<int64_t, double>> prof_acc;
+  std::map<const char*, ProfAcc> prof_acc;
+  int64_t kernels_launched = 0;
+  int64_t device_bytes = 0;
 
   std::vector<void*> allocs;
   fo::TcContext* tc = nullptr;
@@ -95,6 +107,7 @@ struct fo_server {
     if (bytes == 0) bytes = 256;
     if (cudaMalloc(&p, bytes) != cudaSuccess) return nullptr;
     allocs.push_back(p);
+    device_bytes += int64_t(bytes);
     return p;
   }
   int op_of_tensor(int tid) const { return tid - 1; }

@@ -19,7 +19,13 @@ void tc_set_input(TcContext* c, int slot);
 TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int op);
 TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int op, int accumulate);
 TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int op);
+// Launches the GEMM kernel (split-K partials when tc_splits(g) > 1, then
+// tc_run_reduce must follow on the same stream).
 void tc_run(TcGemm* g, const void* input, cudaStream_t st);
+void tc_run_reduce(TcGemm* g, cudaStream_t st);
+int tc_splits(const TcGemm* g);
+double tc_flops(const TcGemm* g);
+double tc_reduce_bytes(const TcGemm* g);
 const char* tc_name(const TcGemm* g);
 // Allocates the split-K workspace after every plan is known.
 int tc_finalize(TcContext* c);

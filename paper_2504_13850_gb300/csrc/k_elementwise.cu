@@ -475,6 +475,13 @@ __global__ void axpby_vec_k(float4* __restrict__ g, const float4* __restrict__ l
 __global__ void axpby_scalar_k(float* g, const float* l, int64_t n, float alpha) {
   GRID_STRIDE(i, n) g[i] = fmaf(alpha, l[i] - g[i], g[i]);
 }
+int axpby_kernels(const float* g, const float* l, int64_t n) {
+  if (n <= 0) return 0;
+  bool aligned = ((reinterpret_cast<uintptr_t>(g) | reinterpret_cast<uintptr_t>(l)) & 15) == 0;
+  int64_t n8 = aligned ? n / 8 : 0;
+  return (n8 > 0 ? 1 : 0) + (n8 * 8 < n ? 1 : 0);
+}
+
 void axpby(float* g, const float* l, int64_t n, float alpha, cudaStream_t st) {
   if (n <= 0) return;
   bool aligned = ((reinterpret_cast<uintptr_t>(g) | reinterpret_cast<uintptr_t>(l)) & 15) == 0;

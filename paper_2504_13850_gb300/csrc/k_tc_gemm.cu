@@ -475,6 +475,7 @@ bool map_window(CUtensorMap* m, const void* base, int N, int H, int W, int C, in
 struct TcGemm {
   const char* name;
   int kind, bn, splits;
+  double flops = 0;
   TcParams p;
   KernelFn fn;
   size_t smem;
@@ -532,9 +533,10 @@ void choose_split(TcContext* c, TcGemm* g, int tiles, int KB) {
   g->p.KB = KB;
 }
 
-TcGemm* finish(TcContext* c, TcGemm* g, int M, int N) {
+TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
   g->p.M = M;
   g->p.N = N;
+  g->flops = 2.0 * M * N * K;
   g->p.err = c->err;
   g->fn = pick_kernel(g->kind, g->bn, &g->smem);
   if (!g->fn) {
@@ -627,7 +629,7 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i) {
         if (!map_2d(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, M, op.cin, BM)) { delete g; return nullptr; }
     } else if (!map_2d(&g->p.tmA, tensor_act(s, op.in0), M, op.cin, BM)) { delete g; return nullptr; }
     if (!map_2d(&g->p.tmB, w, op.cout, op.cin, bn)) { delete g; return nullptr; }
-    return finish(c, g, M, op.cout);
+    return finish(c, g, M, op.cout, double(op.cin));
   }
   // convolution: 3x3 (or 1x1) stride 1
   if (op.stride != 1 || op.cin % 64 || op.cout % 64) { delete g; return nullptr; }
@@ -650,7 +652,7 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i) {
       if (!map_window(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, a.N, a.H, a.W, a.C, rows, imgs)) { delete g; return nullptr; }
   } else if (!map_window(&g->p.tmA, tensor_act(s, op.in0), a.N, a.H, a.W, a.C, rows, imgs)) { delete g; return nullptr; }
   if (!map_2d(&g->p.tmB, w, op.cout, int64_t(g->p.taps) * op.cin, bn)) { delete g; return nullptr; }
-  return finish(c, g, M, op.cout);
+  return finish(c, g, M, op.cout, double(g->p.taps) * op.cin);
 }
 
 TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate) {
@@ -673,7 +675,7 @@ TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate) {
     int M = int(a.rows()), KB = op.cout / 64;
     choose_split(c, g, (M + BM - 1) / BM * (op.cin / bn), KB);
     if (!map_2d(&g->p.tmA, o.grad, M, op.cout, BM) || !map_2d(&g->p.tmB, w, op.cout, op.cin, BK)) { delete g; return nullptr; }
-    return finish(c, g, M, op.cin);
+    return finish(c, g, M, op.cin, double(op.cout));
   }
   if (op.stride != 1 || op.cin % 64 || op.cout % 64) { delete g; return nullptr; }
   int rows, imgs;
@@ -689,7 +691,7 @@ TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate) {
   choose_split(c, g, M / BM * (op.cin / bn), KB);
   if (!map_window(&g->p.tmA, o.grad, o.N, o.H, o.W, o.C, rows, imgs) ||
       !map_2d(&g->p.tmB, w, op.cout, int64_t(g->p.taps) * op.cin, BK)) { delete g; return nullptr; }
-  return finish(c, g, M, op.cin);
+  return finish(c, g, M, op.cin, double(g->p.taps) * op.cout);
 }
 
 TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
@@ -717,7 +719,7 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
       for (int sl = 0; sl < s->cfg.omega; ++sl)
         if (!map_2d(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, rows, op.cin, BK)) { delete g; return nullptr; }
     } else if (!map_2d(&g->p.tmB, tensor_act(s, op.in0), rows, op.cin, BK)) { delete g; return nullptr; }
-    return finish(c, g, op.cout, op.cin);
+    return finish(c, g, op.cout, op.cin, double(rows));
   }
   if (op.stride != 1 || op.cin % 64 || op.cout % 128) { delete g; return nullptr; }
   int rows, imgs;
@@ -739,7 +741,7 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
     for (int sl = 0; sl < s->cfg.omega; ++sl)
       if (!map_window(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, a.N, a.H, a.W, a.C, rows, imgs)) { delete g; return nullptr; }
   } else if (!map_window(&g->p.tmB, tensor_act(s, op.in0), a.N, a.H, a.W, a.C, rows, imgs)) { delete g; return nullptr; }
-  return finish(c, g, op.cout, N);
+  return finish(c, g, op.cout, N, double(P));
 }
 
 void tc_run(TcGemm* g, const void* input, cudaStream_t st) {
@@ -748,12 +750,21 @@ void tc_run(TcGemm* g, const void* input, cudaStream_t st) {
   if (g->input_A) g->p.tmA = g->slot_maps[c->slot];
   if (g->input_B) g->p.tmB = g->slot_maps[c->slot];
   g->fn<<<g->grid, kThreads, g->smem, st>>>(g->p);
-  if (g->splits > 1) {
-    TcParams& p = g->p;
-    int64_t n4 = int64_t(p.M) * p.N / 4;
-    splitk_reduce_k<<<elementwise_blocks(n4, 256), 256, 0, st>>>(p.ws, g->splits, p.M, p.N, p.out, p.ldo, p.bias,
-                                                                  p.relu, p.acc, p.out_f32);
-  }
+}
+
+void tc_run_reduce(TcGemm* g, cudaStream_t st) {
+  TcParams& p = g->p;
+  int64_t n4 = int64_t(p.M) * p.N / 4;
+  splitk_reduce_k<<<elementwise_blocks(n4, 256), 256, 0, st>>>(p.ws, g->splits, p.M, p.N, p.out, p.ldo, p.bias,
+                                                                p.relu, p.acc, p.out_f32);
+}
+
+int tc_splits(const TcGemm* g) { return g->splits; }
+double tc_flops(const TcGemm* g) { return g->flops; }
+double tc_reduce_bytes(const TcGemm* g) {
+  const TcParams& p = g->p;
+  double mn = double(p.M) * p.N;
+  return mn * 4.0 * g->splits + mn * (p.out_f32 ? 4.0 : 2.0) * (p.acc ? 2 : 1);
 }
 
 const char* tc_name(const TcGemm* g) { return g->name; }
