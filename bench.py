@@ -43,12 +43,13 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--steps", type=int, default=1000)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default=WORKLOAD)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-agg-sweep", action="store_true")
     return p.parse_args()
 
 
@@ -276,12 +277,10 @@ def run_ours(args):
         step()
     srv.synchronize()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    srv.profile(True)
-    srv.profile_reset()
-    barrier(world)
-    torch.cuda.synchronize()
-    k0 = srv.kernels_launched()
     with ClockSampler(local) as clk:
+        barrier(world)
+        torch.cuda.synchronize()
+        k0 = srv.kernels_launched()
         ev0.record(stream)
         w0 = time.perf_counter()
         for _ in range(args.steps):
@@ -289,15 +288,26 @@ def run_ours(args):
         ev1.record(stream)
         torch.cuda.synchronize()
         wall = time.perf_counter() - w0
-    barrier(world)
+        barrier(world)
     srv.check_error()
     ms_dev = ev0.elapsed_time(ev1)
     launches = srv.kernels_launched() - k0
-    ktimes = srv.kernel_times()
-    srv.profile(False)
     ms_max = max_over_ranks(world, ms_dev, dev)
     samples = sum_over_ranks(world, float(args.steps * B), dev)
     value = samples / (ms_max / 1e3)
+
+    # ---------------- per-kernel times: the same steps again, each launch
+    # bracketed by CUDA events on the compute stream (a separate timed region,
+    # so the events do not perturb the value above)
+    n_prof = min(args.steps, 200)
+    srv.profile(True)
+    srv.profile_reset()
+    torch.cuda.synchronize()
+    for _ in range(n_prof):
+        step()
+    ktimes = srv.kernel_times()
+    srv.profile(False)
+    srv.check_error()
 
     # ---------------- end to end through the C ABI from pinned host memory
     e2e = None
@@ -327,7 +337,7 @@ def run_ours(args):
 
     # ---------------- aggregation bandwidth sweep (standalone FedAsync update)
     agg = None
-    if rank == 0:
+    if rank == 0 and not args.no_agg_sweep:
         n = 200_000_000
         try:
             ga = torch.randn(n, device=dev) * 0.05
@@ -368,7 +378,7 @@ def run_ours(args):
         roof = {"kernel": name, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
                 "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": traffic_for(name),
                 "peak_kind": f"{which} copy", "launches": nl, "ms_total": round(ms_k, 3)}
-    step_flops = sum(v[2] for v in ktimes.values()) / args.steps
+    step_flops = sum(v[2] for v in ktimes.values()) / n_prof
     step_ms = ms_dev / args.steps
     tensor_frac = step_flops / (step_ms / 1e3) / 1e12 / pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
     cpu = None
@@ -394,6 +404,7 @@ def run_ours(args):
         "cpu_baseline": cpu,
         "clocks": clk.summary(),
         "host_wall_ms_per_step": round(1e3 * wall / args.steps, 4),
+        "kernels_profiled_steps": n_prof,
         "kernels": {k: {"launches": v[0], "ms": round(v[1], 3),
                         "tflops": round(v[2] / (v[1] / 1e3) / 1e12, 1) if v[2] and v[1] else None,
                         "gbs": round(v[3] / (v[1] / 1e3) / 1e9, 1) if v[3] and v[1] else None}
