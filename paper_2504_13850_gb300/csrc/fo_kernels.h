@@ -16,9 +16,9 @@ struct ConvShape {
 // or null, y NHWC; each operand's dtype is given (kF32 / kBF16).
 void conv_fwd_simt(const ConvShape& s, const void* x, int dt_x, const void* w, int dt_w,
                    const float* bias, void* y, int dt_y, bool relu, cudaStream_t st);
-// dx (+)= conv^T(dy, w).
+// dx (+)= conv^T(dy, w), times (mask > 0) when mask (same layout as dx) is given.
 void conv_dgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* w, int dt_w,
-                     void* dx, int dt_dx, bool accumulate, cudaStream_t st);
+                     void* dx, int dt_dx, bool accumulate, const void* mask, cudaStream_t st);
 // dw[Co][k][k][Ci] = sum over output pixels of dy (x) x-window (fp32 out).
 void conv_wgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* x,
                      int dt_x, float* dw, cudaStream_t st);
@@ -35,11 +35,11 @@ void maxpool2_bwd(const void* x, const void* dy, void* dx, int N, int H, int W, 
 void relu_maxpool2_bwd(const void* x, const void* dy, void* dx, int N, int H, int W, int C,
                        int dt, bool acc, cudaStream_t st);
 void affine_fwd(const void* x, const float* scale, const float* shift, void* y, int64_t rows,
-                int C, int dt, cudaStream_t st);
+                int C, int dt, bool relu, cudaStream_t st);
 // dx (+)= dy * scale (dx may be null)
 void affine_dx(const void* dy, const float* scale, void* dx, int64_t rows, int C, int dt,
                bool acc, cudaStream_t st);
-void add_fwd(const void* a, const void* b, void* y, int64_t n, int dt, cudaStream_t st);
+void add_fwd(const void* a, const void* b, void* y, int64_t n, int dt, bool relu, cudaStream_t st);
 // y (+)= x
 void copy_or_acc(const void* x, void* y, int64_t n, int dt, bool acc, cudaStream_t st);
 void avgpool_fwd(const void* x, void* y, int N, int HW, int C, int dt, cudaStream_t st);
@@ -71,6 +71,14 @@ void attention_fwd(const void* qkv, const int32_t* len, void* out, float* probs,
 void attention_bwd(const void* qkv, const int32_t* len, const float* probs, const void* out,
                    const void* dout, void* dqkv, int B, int L, int C, int heads, int dt, bool acc,
                    cudaStream_t st);
+
+// Classifier head (last linear layer + softmax cross-entropy), fp32 weights.
+void head_forward_loss(const void* x, int dt, const float* W, const float* bias, const int32_t* labels,
+                       int B, int K, int C, float* logits, float* dz, float* row_loss, cudaStream_t st);
+void head_weight_grad(const float* dz, const void* x, int dt, int B, int K, int C, float* dW, float* db,
+                      const float* row_loss, float* loss_out, cudaStream_t st);
+void head_input_grad(const float* dz, const float* W, int B, int K, int C, const void* mask, void* dx,
+                     int dt, bool acc, cudaStream_t st);
 
 // Softmax cross-entropy: loss_slot <- mean_b CE; dlogits = (softmax - onehot)/B.
 void softmax_ce(const float* logits, const int32_t* labels, int B, int C, float* loss_slot,

@@ -158,45 +158,107 @@ fo::ConvShape conv_shape(const fo_server* s, int i) {
   return {a.N, a.H, a.W, op.cin, op.cout, op.k, op.stride, op.k / 2, o.H, o.W};
 }
 
+// Which kernels absorb which neighbouring work (decided once per network).
+struct Fusion {
+  std::vector<int> fwd_relu;   // producer op -> the relu op it applies, or -1
+  std::vector<char> skip_fwd;  // relu op whose forward is done by its producer
+  std::vector<int> bwd_mask;   // consumer op -> relu op whose mask it applies to its dx, or -1
+  std::vector<char> skip_bwd;  // relu op whose backward is done by its consumer
+  bool head = false;           // last linear + loss handled by the head kernels
+};
+
+bool dx_takes_mask(const fo_server* s, int j) {
+  const fo_op& op = s->ops[j];
+  return op.kind == FO_OP_CONV || op.kind == FO_OP_LINEAR || op.kind == FO_OP_MAXPOOL2;
+}
+
+Fusion analyse(const fo_server* s) {
+  const int nops = int(s->ops.size());
+  Fusion f;
+  f.fwd_relu.assign(nops, -1);
+  f.skip_fwd.assign(nops, 0);
+  f.bwd_mask.assign(nops, -1);
+  f.skip_bwd.assign(nops, 0);
+  std::vector<int> sole(nops + 1, -1);  // the only consumer op of a tensor
+  for (int j = 0; j < nops; ++j) {
+    const fo_op& op = s->ops[j];
+    if (s->T[op.in0].consumers == 1) sole[op.in0] = j;
+    if (op.kind == FO_OP_ADD && s->T[op.in1].consumers == 1) sole[op.in1] = j;
+  }
+  const fo_op& last = s->ops.back();
+  f.head = last.kind == FO_OP_LINEAR && s->cfg.num_classes <= 1024;
+  for (int r = 0; r < nops; ++r) {
+    const fo_op& op = s->ops[r];
+    if (op.kind != FO_OP_RELU || op.in0 == 0) continue;
+    const int p = op.in0 - 1;  // producer op of the relu input
+    const int pk = s->ops[p].kind;
+    if (sole[op.in0] == r && (pk == FO_OP_CONV || pk == FO_OP_LINEAR || pk == FO_OP_AFFINE || pk == FO_OP_ADD) &&
+        !(f.head && p == nops - 1)) {
+      f.fwd_relu[p] = r;
+      f.skip_fwd[r] = 1;
+    }
+    const int j = sole[r + 1];
+    if (j >= 0 && s->ops[j].in0 == r + 1 && (dx_takes_mask(s, j) || (f.head && j == nops - 1))) {
+      f.bwd_mask[j] = r;
+      f.skip_bwd[r] = 1;
+    }
+  }
+  return f;
+}
+
 // Build the list of launches of one server step.  Every entry records how
 // many kernels it launches and its algorithmic FLOPs / HBM bytes (the
 // minimum a kernel of that job must move), for the per-kernel roofline.
+// A ReLU is applied by the kernel producing its input (forward) and by the
+// kernel producing its output gradient (backward): the mask y > 0 of the
+// ReLU output equals x > 0 of its input.
 int build_plan(fo_server* s) {
   const int nops = int(s->ops.size());
   const int dt = s->dt;
   const double esz = dt == fo::kF32 ? 4.0 : 2.0;
   auto& plan = s->plan;
   plan.clear();
+  const Fusion fu = analyse(s);
   auto act = [s](int tid) -> const void* { return tid == 0 ? s->cur_in : s->T[tid].act; };
   auto add = [&plan](const char* name, int kernels, double flops, double bytes,
                      std::function<void(cudaStream_t)> fn) {
     plan.push_back({name, std::move(fn), kernels, flops, bytes});
   };
   auto tbytes = [s](int tid) { return double(s->T[tid].bytes()); };
-  auto add_tc = [&](fo::TcGemm* g, const void* in) {
-    add(fo::tc_name(g), 1, fo::tc_flops(g), 0.0, [=](cudaStream_t st) { fo::tc_run(g, in, st); });
+  auto add_tc = [&](fo::TcGemm* g) {
+    add(fo::tc_name(g), 1, fo::tc_flops(g), 0.0, [=](cudaStream_t st) { fo::tc_run(g, nullptr, st); });
     if (fo::tc_splits(g) > 1)
       add("splitk_reduce", 1, 0.0, fo::tc_reduce_bytes(g), [=](cudaStream_t st) { fo::tc_run_reduce(g, st); });
   };
+  const int L = nops - 1;  // the logits layer
 
   // ---------------- forward
   for (int i = 0; i < nops; ++i) {
     const fo_op op = s->ops[i];
-    const int a = op.in0, o = i + 1;
+    if (fu.skip_fwd[i]) continue;
+    const int a = op.in0;
+    // output buffer: a fused relu writes the relu's output tensor
+    const int o = fu.fwd_relu[i] >= 0 ? fu.fwd_relu[i] + 1 : i + 1;
+    const bool relu = fu.fwd_relu[i] >= 0;
     const Tensor& ta = s->T[a];
-    const Tensor& to = s->T[o];
+    const Tensor& to = s->T[i + 1];
+    if (fu.head && i == L) {
+      const int B = s->cfg.batch, K = op.cin, C = op.cout;
+      add("head_fwd_ce", 1, 2.0 * B * K * C, tbytes(a), [=](cudaStream_t st) {
+        fo::head_forward_loss(act(a), s->T[a].dt, P(s, i, 0), op.bias ? P(s, i, 1) : nullptr, s->cur_labels, B,
+                              K, C, (float*)s->T[i + 1].act, (float*)s->T[i + 1].grad, s->row_loss, st);
+      });
+      continue;
+    }
     switch (op.kind) {
       case FO_OP_CONV:
       case FO_OP_LINEAR: {
         fo::ConvShape cs = conv_shape(s, i);
         const bool bias = op.bias != 0;
         const double fl = 2.0 * double(to.rows()) * op.cout * double(op.kind == FO_OP_CONV ? op.k * op.k : 1) * op.cin;
-        fo::TcGemm* tg = fo::tc_plan_forward(s->tc, s, i);
+        fo::TcGemm* tg = fo::tc_plan_forward(s->tc, s, i, s->T[o].act, relu);
         if (tg) {
-          const int in = a;
-          add_tc(tg, nullptr);
-          (void)in;
-          // the first layer reads the batch slot: its tensor map is chosen per step
+          add_tc(tg);
         } else {
           // Hidden layers of the bf16 path multiply bf16 weights (the shadow);
           // the fp32 path and the fp32 logits layer use the fp32 master.
@@ -205,14 +267,14 @@ int build_plan(fo_server* s) {
           add(op.kind == FO_OP_CONV ? "conv_fwd_simt" : "linear_fwd_simt", 1, fl, 0.0, [=](cudaStream_t st) {
             const void* w = wbf ? (const void*)SH(s, i, 0) : (const void*)P(s, i, 0);
             fo::conv_fwd_simt(cs, act(a), ta.dt, w, wbf ? fo::kBF16 : fo::kF32, bias ? P(s, i, 1) : nullptr,
-                              s->T[o].act, dto, false, st);
+                              s->T[o].act, dto, relu, st);
           });
         }
         break;
       }
       case FO_OP_AFFINE:
         add("affine_fwd", 1, 0.0, 2 * tbytes(a), [=](cudaStream_t st) {
-          fo::affine_fwd(act(a), P(s, i, 0), P(s, i, 1), s->T[o].act, s->T[a].rows(), s->T[a].C, dt, st);
+          fo::affine_fwd(act(a), P(s, i, 0), P(s, i, 1), s->T[o].act, s->T[a].rows(), s->T[a].C, dt, relu, st);
         });
         break;
       case FO_OP_RELU:
@@ -228,8 +290,8 @@ int build_plan(fo_server* s) {
         break;
       case FO_OP_ADD: {
         const int b = op.in1;
-        add("add_fwd", 1, 0.0, 3 * tbytes(o), [=](cudaStream_t st) {
-          fo::add_fwd(act(a), act(b), s->T[o].act, s->T[o].numel(), dt, st);
+        add("add_fwd", 1, 0.0, 3 * tbytes(i + 1), [=](cudaStream_t st) {
+          fo::add_fwd(act(a), act(b), s->T[o].act, s->T[o].numel(), dt, relu, st);
         });
         break;
       }
@@ -253,8 +315,8 @@ int build_plan(fo_server* s) {
         });
         break;
       case FO_OP_ATTENTION: {
-        const double L = ta.H, heads = op.heads, dh = double(op.cin) / op.heads;
-        add("attention_fwd", 1, 4.0 * ta.N * heads * L * L * dh, tbytes(a) + tbytes(o), [=](cudaStream_t st) {
+        const double Ls = ta.H, heads = op.heads, dh = double(op.cin) / op.heads;
+        add("attention_fwd", 1, 4.0 * ta.N * heads * Ls * Ls * dh, tbytes(a) + tbytes(o), [=](cudaStream_t st) {
           const Tensor& x = s->T[a];
           fo::attention_fwd(act(a), s->cur_len, s->T[o].act, s->attn_probs[i], x.N, x.H, op.cin, op.heads, dt, st);
         });
@@ -270,7 +332,7 @@ int build_plan(fo_server* s) {
   }
 
   // ---------------- loss (softmax cross-entropy on fp32 logits)
-  {
+  if (!fu.head) {
     const int lt = nops;
     add("softmax_ce", 1, 0.0, 2 * tbytes(lt), [=](cudaStream_t st) {
       fo::softmax_ce((const float*)s->T[lt].act, s->cur_labels, s->cfg.batch, s->cfg.num_classes,
@@ -291,7 +353,11 @@ int build_plan(fo_server* s) {
   };
   for (int i = nops - 1; i >= 0; --i) {
     const fo_op op = s->ops[i];
-    const int a = op.in0, o = i + 1;
+    if (fu.skip_bwd[i]) {
+      written[s->T[i + 1].root] = 1;
+      continue;
+    }
+    const int a0 = op.in0, o = i + 1;
     const int ro = s->T[o].root;
     if (!written[ro]) {
       // Nothing downstream produced a gradient: zero this op's parameter grads.
@@ -303,8 +369,29 @@ int build_plan(fo_server* s) {
       }
       continue;
     }
-    const bool need_dx = a != 0;
+    // A relu between this op's input and its producer: write the producer's
+    // output gradient directly, masked by the relu output.
+    const int mr = fu.bwd_mask[i];
+    const int a = mr >= 0 ? s->ops[mr].in0 : a0;            // gradient destination
+    const void* mask = mr >= 0 ? s->T[mr + 1].act : nullptr;
+    const bool need_dx = a0 != 0;
     const double csb = double(s->T[o].rows()) * s->T[o].C * esz;  // one read of dy
+    if (fu.head && i == L) {
+      const int B = s->cfg.batch, K = op.cin, C = op.cout;
+      add("head_wgrad", 1, 2.0 * B * K * C, tbytes(a0), [=](cudaStream_t st) {
+        fo::head_weight_grad((const float*)s->T[o].grad, act(a0), s->T[a0].dt, B, K, C, G(s, i, 0),
+                             op.bias ? G(s, i, 1) : nullptr, s->row_loss,
+                             s->losses + (s->steps_done & (s->kLossRing - 1)), st);
+      });
+      if (need_dx) {
+        int accf = contrib(a);
+        add("head_dgrad", 1, 2.0 * B * K * C, (2 + accf) * tbytes(a), [=](cudaStream_t st) {
+          fo::head_input_grad((const float*)s->T[o].grad, P(s, i, 0), B, K, C, mask, s->T[a].grad, s->T[a].dt,
+                              accf != 0, st);
+        });
+      }
+      continue;
+    }
     switch (op.kind) {
       case FO_OP_CONV:
       case FO_OP_LINEAR: {
@@ -319,32 +406,32 @@ int build_plan(fo_server* s) {
         }
         if (need_dx) {
           int accf = contrib(a);
-          fo::TcGemm* tg = fo::tc_plan_dgrad(s->tc, s, i, accf);
+          fo::TcGemm* tg = fo::tc_plan_dgrad(s->tc, s, i, accf, s->T[a].grad, mask);
           if (tg) {
-            add_tc(tg, nullptr);
+            add_tc(tg);
           } else {
             const bool wbf = dto == fo::kBF16;
             add(op.kind == FO_OP_CONV ? "conv_dgrad_simt" : "linear_dgrad_simt", 1, fl, 0.0, [=](cudaStream_t st) {
               const void* w = wbf ? (const void*)SH(s, i, 0) : (const void*)P(s, i, 0);
               fo::conv_dgrad_simt(cs, s->T[o].grad, dto, w, wbf ? fo::kBF16 : fo::kF32, s->T[a].grad, dta,
-                                  accf != 0, st);
+                                  accf != 0, mask, st);
             });
           }
         }
         fo::TcGemm* tw = fo::tc_plan_wgrad(s->tc, s, i);
         if (tw) {
-          add_tc(tw, nullptr);
+          add_tc(tw);
         } else {
           add(op.kind == FO_OP_CONV ? "conv_wgrad_simt" : "linear_wgrad_simt", 1, fl, 0.0, [=](cudaStream_t st) {
-            fo::conv_wgrad_simt(cs, s->T[o].grad, dto, act(a), dta, G(s, i, 0), st);
+            fo::conv_wgrad_simt(cs, s->T[o].grad, dto, act(a0), s->T[a0].dt, G(s, i, 0), st);
           });
         }
         break;
       }
       case FO_OP_AFFINE:
         add("affine_pgrad", 4, 0.0, 3 * csb, [=](cudaStream_t st) {
-          const Tensor& x = s->T[a];
-          fo::colsum(s->T[o].grad, act(a), x.rows(), x.C, dt, s->colsum_scratch, G(s, i, 0), st);
+          const Tensor& x = s->T[a0];
+          fo::colsum(s->T[o].grad, act(a0), x.rows(), x.C, dt, s->colsum_scratch, G(s, i, 0), st);
           fo::colsum(s->T[o].grad, nullptr, x.rows(), x.C, dt, s->colsum_scratch, G(s, i, 1), st);
         });
         if (need_dx) {
@@ -357,23 +444,29 @@ int build_plan(fo_server* s) {
       case FO_OP_RELU:
         if (need_dx) {
           int accf = contrib(a);
+          // mask from the relu output: y > 0 exactly where x > 0
           add("relu_bwd", 1, 0.0, (3 + accf) * csb, [=](cudaStream_t st) {
-            fo::relu_bwd(act(a), s->T[o].grad, s->T[a].grad, s->T[a].numel(), dt, accf != 0, st);
+            fo::relu_bwd(s->T[o].act, s->T[o].grad, s->T[a].grad, s->T[a].numel(), dt, accf != 0, st);
           });
         }
         break;
       case FO_OP_MAXPOOL2:
         if (need_dx) {
           int accf = contrib(a);
-          add("maxpool2_bwd", 1, 0.0, (2 + accf) * tbytes(a) + csb, [=](cudaStream_t st) {
-            const Tensor& x = s->T[a];
-            fo::maxpool2_bwd(act(a), s->T[o].grad, x.grad, x.N, x.H, x.W, x.C, dt, accf != 0, st);
-          });
+          const bool masked = mr >= 0;
+          add(masked ? "relu_maxpool2_bwd" : "maxpool2_bwd", 1, 0.0, (2 + accf) * tbytes(a0) + csb,
+              [=](cudaStream_t st) {
+                const Tensor& x = s->T[a0];
+                if (masked)
+                  fo::relu_maxpool2_bwd(act(a0), s->T[o].grad, s->T[a].grad, x.N, x.H, x.W, x.C, dt, accf != 0, st);
+                else
+                  fo::maxpool2_bwd(act(a0), s->T[o].grad, s->T[a].grad, x.N, x.H, x.W, x.C, dt, accf != 0, st);
+              });
         }
         break;
       case FO_OP_ADD: {
         const int b = op.in1;
-        for (int src : {a, b}) {
+        for (int src : {a0, b}) {
           if (src == 0) continue;
           int accf = contrib(src);
           add("add_bwd", 1, 0.0, (2 + accf) * csb, [=](cudaStream_t st) {
@@ -395,8 +488,8 @@ int build_plan(fo_server* s) {
         break;  // shares the input's gradient buffer
       case FO_OP_LAYERNORM:
         add("layernorm_pgrad", 4, 0.0, 3 * csb, [=](cudaStream_t st) {
-          const Tensor& x = s->T[a];
-          fo::colsum_lnx(s->T[o].grad, act(a), s->ln_mean[i], s->ln_rstd[i], x.rows(), x.C, dt, s->colsum_scratch,
+          const Tensor& x = s->T[a0];
+          fo::colsum_lnx(s->T[o].grad, act(a0), s->ln_mean[i], s->ln_rstd[i], x.rows(), x.C, dt, s->colsum_scratch,
                          G(s, i, 0), st);
           fo::colsum(s->T[o].grad, nullptr, x.rows(), x.C, dt, s->colsum_scratch, G(s, i, 1), st);
         });
@@ -421,8 +514,8 @@ int build_plan(fo_server* s) {
         if (need_dx) {
           int accf = contrib(a);
           const Tensor& ta = s->T[a];
-          const double L = ta.H, heads = op.heads, dh = double(op.cin) / op.heads;
-          add("attention_bwd", 1, 8.0 * ta.N * heads * L * L * dh, (2 + accf) * tbytes(a) + 2 * csb,
+          const double Ls = ta.H, heads = op.heads, dh = double(op.cin) / op.heads;
+          add("attention_bwd", 1, 8.0 * ta.N * heads * Ls * Ls * dh, (2 + accf) * tbytes(a) + 2 * csb,
               [=](cudaStream_t st) {
                 const Tensor& x = s->T[a];
                 fo::attention_bwd(act(a), s->cur_len, s->attn_probs[i], s->T[o].act, s->T[o].grad, x.grad, x.N, x.H,
@@ -518,6 +611,7 @@ int allocate(fo_server* s) {
     }
   }
   s->losses = (float*)s->alloc(size_t(s->kLossRing) * 4);
+  s->row_loss = (float*)s->alloc(size_t(s->cfg.batch) * 4);
   if (!s->colsum_scratch || !s->losses) return set_err(FO_ERR_OOM, "scratch allocation");
   FO_CUDA(cudaMemset(s->losses, 0, size_t(s->kLossRing) * 4));
   return FO_OK;

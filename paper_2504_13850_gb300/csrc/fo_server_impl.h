@@ -83,6 +83,7 @@ struct fo_server {
   const int32_t* cur_labels = nullptr;
   const int32_t* cur_len = nullptr;
   float* losses = nullptr;
+  float* row_loss = nullptr;
   int64_t steps_done = 0;
   static constexpr int64_t kLossRing = int64_t(1) << 20;
 

@@ -16,8 +16,12 @@ int tc_create(TcContext** out, fo_server* s);
 void tc_destroy(TcContext* c);
 // Selects the tensor maps of batch slot `slot` for the first layer.
 void tc_set_input(TcContext* c, int slot);
-TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int op);
-TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int op, int accumulate);
+// Forward of conv/linear op `op` into `out` (bf16, the op's output layout),
+// applying a ReLU when `relu`.
+TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int op, void* out, bool relu);
+// Input gradient of op `op` into `dx` (accumulating when `accumulate`),
+// multiplied by (mask > 0) when `mask` (same layout as dx) is given.
+TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int op, int accumulate, void* dx, const void* mask);
 TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int op);
 // Launches the GEMM kernel (split-K partials when tc_splits(g) > 1, then
 // tc_run_reduce must follow on the same stream).

@@ -129,10 +129,11 @@ void relu_maxpool2_bwd(const void* x, const void* dy, void* dx, int N, int H, in
 
 // ---------------------------------------------------------- affine / add
 template <typename T>
-__global__ void affine_fwd_k(const T* x, const float* sc, const float* sh, T* y, int64_t n, int C) {
+__global__ void affine_fwd_k(const T* x, const float* sc, const float* sh, T* y, int64_t n, int C, int relu) {
   GRID_STRIDE(i, n) {
     int c = int(i % C);
-    y[i] = from_f<T>(fmaf(to_f(x[i]), sc[c], sh[c]));
+    float v = fmaf(to_f(x[i]), sc[c], sh[c]);
+    y[i] = from_f<T>(relu ? fmaxf(v, 0.f) : v);
   }
 }
 template <typename T>
@@ -140,25 +141,28 @@ __global__ void affine_dx_k(const T* dy, const float* sc, T* dx, int64_t n, int 
   GRID_STRIDE(i, n) store(dx, i, to_f(dy[i]) * sc[int(i % C)], acc);
 }
 template <typename T>
-__global__ void add_fwd_k(const T* a, const T* b, T* y, int64_t n) {
-  GRID_STRIDE(i, n) y[i] = from_f<T>(to_f(a[i]) + to_f(b[i]));
+__global__ void add_fwd_k(const T* a, const T* b, T* y, int64_t n, int relu) {
+  GRID_STRIDE(i, n) {
+    float v = to_f(a[i]) + to_f(b[i]);
+    y[i] = from_f<T>(relu ? fmaxf(v, 0.f) : v);
+  }
 }
 template <typename T>
 __global__ void copy_acc_k(const T* x, T* y, int64_t n, int acc) {
   GRID_STRIDE(i, n) store(y, i, to_f(x[i]), acc);
 }
 void affine_fwd(const void* x, const float* scale, const float* shift, void* y, int64_t rows,
-                int C, int dt, cudaStream_t st) {
+                int C, int dt, bool relu, cudaStream_t st) {
   int64_t n = rows * C;
-  FO_DISPATCH(dt, T, affine_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, scale, shift, (T*)y, n, C));
+  FO_DISPATCH(dt, T, affine_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, scale, shift, (T*)y, n, C, relu));
 }
 void affine_dx(const void* dy, const float* scale, void* dx, int64_t rows, int C, int dt,
                bool acc, cudaStream_t st) {
   int64_t n = rows * C;
   FO_DISPATCH(dt, T, affine_dx_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)dy, scale, (T*)dx, n, C, acc));
 }
-void add_fwd(const void* a, const void* b, void* y, int64_t n, int dt, cudaStream_t st) {
-  FO_DISPATCH(dt, T, add_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)a, (const T*)b, (T*)y, n));
+void add_fwd(const void* a, const void* b, void* y, int64_t n, int dt, bool relu, cudaStream_t st) {
+  FO_DISPATCH(dt, T, add_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)a, (const T*)b, (T*)y, n, relu));
 }
 void copy_or_acc(const void* x, void* y, int64_t n, int dt, bool acc, cudaStream_t st) {
   FO_DISPATCH(dt, T, copy_acc_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (T*)y, n, acc));
@@ -317,28 +321,74 @@ __global__ void colsum_partial_k(const T* a, const T* b, const float* mean, cons
     partial[int64_t(blockIdx.y) * C + c] = t;
   }
 }
+// Adds the per-chunk partials of each column: 8 row lanes per column sum
+// interleaved chunks, then combine in a fixed order (deterministic).
 __global__ void colsum_finish_k(const float* partial, int chunks, int C, float* out) {
-  int c = blockIdx.x * blockDim.x + threadIdx.x;
-  if (c >= C) return;
+  __shared__ float red[8][33];
+  const int cl = threadIdx.x % 32, rl = threadIdx.x / 32;
+  const int c = blockIdx.x * 32 + cl;
   float s = 0.f;
-  for (int q = 0; q < chunks; ++q) s += partial[int64_t(q) * C + c];
-  out[c] = s;
+  if (c < C)
+    for (int q = rl; q < chunks; q += 8) s += partial[int64_t(q) * C + c];
+  red[rl][cl] = s;
+  __syncthreads();
+  if (rl == 0 && c < C) {
+    float t = 0.f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) t += red[q][cl];
+    out[c] = t;
+  }
 }
+
+// bf16 column sums with 16-byte loads: thread (g, r) adds columns
+// 8g..8g+7 over rows r, r + rl, ... of its chunk; the rl row lanes of a
+// block are combined in shared memory (fixed order).
+__global__ void colsum_bf16x8_k(const bf16* __restrict__ a, int64_t rows, int C, float* __restrict__ partial) {
+  extern __shared__ float red[];  // [rl][C]
+  const int groups = C / 8;
+  const int g = threadIdx.x % groups, r = threadIdx.x / groups, rl = blockDim.x / groups;
+  const int64_t r0 = int64_t(blockIdx.x) * CS_ROWS;
+  float s[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  if (r < rl) {
+    for (int64_t row = r0 + r; row < r0 + CS_ROWS && row < rows; row += rl) {
+      uint4 u = *reinterpret_cast<const uint4*>(a + row * C + 8 * g);
+      const bf16* e = reinterpret_cast<const bf16*>(&u);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) s[j] += __bfloat162float(e[j]);
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) red[r * C + 8 * g + j] = s[j];
+  }
+  __syncthreads();
+  for (int c = threadIdx.x; c < C; c += blockDim.x) {
+    float t = 0.f;
+    for (int q = 0; q < rl; ++q) t += red[q * C + c];
+    partial[int64_t(blockIdx.x) * C + c] = t;
+  }
+}
+
 void colsum(const void* a, const void* b, int64_t rows, int C, int dt, float* partial, float* out,
             cudaStream_t st) {
+  if (!b && dt == kBF16 && C % 8 == 0 && C / 8 <= 256) {
+    const int groups = C / 8;
+    const int rl = 256 / groups;
+    colsum_bf16x8_k<<<colsum_chunks(rows), groups * rl, sizeof(float) * rl * C, st>>>((const bf16*)a, rows, C, partial);
+    colsum_finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, colsum_chunks(rows), C, out);
+    return;
+  }
   dim3 grid(ceil_div(C, 32), colsum_chunks(rows));
   if (b) {
     FO_DISPATCH(dt, T, colsum_partial_k<1, T><<<grid, 256, 0, st>>>((const T*)a, (const T*)b, nullptr, nullptr, rows, C, partial));
   } else {
     FO_DISPATCH(dt, T, colsum_partial_k<0, T><<<grid, 256, 0, st>>>((const T*)a, nullptr, nullptr, nullptr, rows, C, partial));
   }
-  colsum_finish_k<<<ceil_div(C, 256), 256, 0, st>>>(partial, colsum_chunks(rows), C, out);
+  colsum_finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, colsum_chunks(rows), C, out);
 }
 void colsum_lnx(const void* dy, const void* x, const float* mean, const float* rstd, int64_t rows,
                 int C, int dt, float* partial, float* out, cudaStream_t st) {
   dim3 grid(ceil_div(C, 32), colsum_chunks(rows));
   FO_DISPATCH(dt, T, colsum_partial_k<2, T><<<grid, 256, 0, st>>>((const T*)dy, (const T*)x, mean, rstd, rows, C, partial));
-  colsum_finish_k<<<ceil_div(C, 256), 256, 0, st>>>(partial, colsum_chunks(rows), C, out);
+  colsum_finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, colsum_chunks(rows), C, out);
 }
 
 // ------------------------------------------------------------- meanpool

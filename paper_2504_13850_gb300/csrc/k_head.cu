@@ -1,0 +1,136 @@
+// Classifier head of the server network: the last linear layer (few
+// outputs) fused with the server loss f_s (softmax cross-entropy averaged
+// over the batch) and its backward pass.
+//   head_fwd_ce : logits z = x W^T + b, per-row CE, dz = (softmax(z) - onehot)/B
+//   head_wgrad  : dW = dz^T x, db = sum_b dz, loss = mean of the row losses
+//                 (summed in row order, deterministic)
+//   head_dgrad  : dx (+)= dz W, optionally times a ReLU mask (mask > 0)
+// W and b are the fp32 master weights; dz and the gradients are fp32.
+#include "fo_common.cuh"
+#include "fo_kernels.h"
+
+namespace fo {
+
+namespace {
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// One block per batch row; warps split the classes.  smem: x row (K floats)
+// and the logits (C floats).
+template <typename T>
+__global__ void head_fwd_ce_k(const T* __restrict__ x, const float* __restrict__ W,
+                              const float* __restrict__ bias, const int32_t* __restrict__ labels, int B,
+                              int K, int C, float* __restrict__ logits, float* __restrict__ dz,
+                              float* __restrict__ row_loss) {
+  extern __shared__ float sm[];
+  float* xr = sm;
+  float* z = sm + K;
+  const int b = blockIdx.x;
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32, nw = blockDim.x / 32;
+  for (int k = threadIdx.x; k < K; k += blockDim.x) xr[k] = to_f(x[int64_t(b) * K + k]);
+  __syncthreads();
+  for (int c = warp; c < C; c += nw) {
+    const float* w = W + int64_t(c) * K;
+    float s = 0.f;
+    for (int k = lane; k < K; k += 32) s = fmaf(xr[k], w[k], s);
+    s = warp_sum(s);
+    if (lane == 0) z[c] = s + (bias ? bias[c] : 0.f);
+  }
+  __syncthreads();
+  if (warp == 0) {
+    float m = -INFINITY;
+    for (int c = lane; c < C; c += 32) m = fmaxf(m, z[c]);
+    m = warp_max(m);
+    float se = 0.f;
+    for (int c = lane; c < C; c += 32) se += expf(z[c] - m);
+    se = warp_sum(se);
+    const int y = labels[b];
+    for (int c = lane; c < C; c += 32) {
+      const float p = expf(z[c] - m) / se;
+      dz[int64_t(b) * C + c] = (p - (c == y ? 1.f : 0.f)) / float(B);
+      logits[int64_t(b) * C + c] = z[c];
+    }
+    if (lane == 0) row_loss[b] = m + logf(se) - z[y];
+  }
+}
+
+// dW[c][k] = sum_b dz[b][c] x[b][k]; grid (ceil(K/256), C).
+template <typename T>
+__global__ void head_wgrad_k(const float* __restrict__ dz, const T* __restrict__ x, int B, int K, int C,
+                             float* __restrict__ dW, float* __restrict__ db, const float* __restrict__ row_loss,
+                             float* __restrict__ loss_out) {
+  const int c = blockIdx.y;
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k < K) {
+    float s = 0.f;
+    for (int b = 0; b < B; ++b) s = fmaf(dz[int64_t(b) * C + c], to_f(x[int64_t(b) * K + k]), s);
+    dW[int64_t(c) * K + k] = s;
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    if (db) {
+      float s = 0.f;
+      for (int b = 0; b < B; ++b) s += dz[int64_t(b) * C + c];
+      db[c] = s;
+    }
+    if (c == 0) {
+      float t = 0.f;
+      for (int b = 0; b < B; ++b) t += row_loss[b];
+      *loss_out = t / float(B);
+    }
+  }
+}
+
+// dx[b][k] (+)= (sum_c dz[b][c] W[c][k]) * (mask[b][k] > 0); grid (ceil(K/256), B).
+template <typename T>
+__global__ void head_dgrad_k(const float* __restrict__ dz, const float* __restrict__ W, int B, int K, int C,
+                             const T* __restrict__ mask, T* __restrict__ dx, int acc) {
+  const int b = blockIdx.y;
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= K) return;
+  float s = 0.f;
+  for (int c = 0; c < C; ++c) s = fmaf(dz[int64_t(b) * C + c], W[int64_t(c) * K + k], s);
+  const int64_t i = int64_t(b) * K + k;
+  if (mask && !(to_f(mask[i]) > 0.f)) s = 0.f;
+  if (acc) s += to_f(dx[i]);
+  dx[i] = from_f<T>(s);
+}
+
+}  // namespace
+
+void head_forward_loss(const void* x, int dt, const float* W, const float* bias, const int32_t* labels, int B,
+                       int K, int C, float* logits, float* dz, float* row_loss, cudaStream_t st) {
+  size_t sm = sizeof(float) * (K + C);
+  if (dt == kF32)
+    head_fwd_ce_k<float><<<B, 256, sm, st>>>((const float*)x, W, bias, labels, B, K, C, logits, dz, row_loss);
+  else
+    head_fwd_ce_k<bf16><<<B, 256, sm, st>>>((const bf16*)x, W, bias, labels, B, K, C, logits, dz, row_loss);
+}
+
+void head_weight_grad(const float* dz, const void* x, int dt, int B, int K, int C, float* dW, float* db,
+                      const float* row_loss, float* loss_out, cudaStream_t st) {
+  dim3 grid(ceil_div(K, 256), C);
+  if (dt == kF32)
+    head_wgrad_k<float><<<grid, 256, 0, st>>>(dz, (const float*)x, B, K, C, dW, db, row_loss, loss_out);
+  else
+    head_wgrad_k<bf16><<<grid, 256, 0, st>>>(dz, (const bf16*)x, B, K, C, dW, db, row_loss, loss_out);
+}
+
+void head_input_grad(const float* dz, const float* W, int B, int K, int C, const void* mask, void* dx, int dt,
+                     bool acc, cudaStream_t st) {
+  dim3 grid(ceil_div(K, 256), B);
+  if (dt == kF32)
+    head_dgrad_k<float><<<grid, 256, 0, st>>>(dz, W, B, K, C, (const float*)mask, (float*)dx, acc ? 1 : 0);
+  else
+    head_dgrad_k<bf16><<<grid, 256, 0, st>>>(dz, W, B, K, C, (const bf16*)mask, (bf16*)dx, acc ? 1 : 0);
+}
+
+}  // namespace fo

@@ -88,7 +88,8 @@ template <int MODE, typename TA, typename TB, typename TC>
 __global__ void __launch_bounds__(NT) simt_conv_kernel(Geo g, const TA* __restrict__ a,
                                                        const TB* __restrict__ b,
                                                        const float* __restrict__ bias,
-                                                       TC* __restrict__ c, int relu, int acc) {
+                                                       TC* __restrict__ c, int relu, int acc,
+                                                       const TC* __restrict__ mask) {
   __shared__ float As[BK][BM + 4];
   __shared__ float Bs[BK][BN + 4];
   const int tid = threadIdx.x;
@@ -131,6 +132,7 @@ __global__ void __launch_bounds__(NT) simt_conv_kernel(Geo g, const TA* __restri
       if (bias) v += bias[n];
       if (relu) v = fmaxf(v, 0.f);
       int64_t idx = m * g.Ncol + n;
+      if (mask && !(to_f(mask[idx]) > 0.f)) v = 0.f;
       if (acc) v += to_f(c[idx]);
       c[idx] = from_f<TC>(v);
     }
@@ -152,30 +154,30 @@ Geo make_geo(const ConvShape& s, int mode) {
 
 template <int MODE, typename TA, typename TB, typename TC>
 void launch(const Geo& g, const void* a, const void* b, const float* bias, void* c, bool relu,
-            bool acc, cudaStream_t st) {
+            bool acc, cudaStream_t st, const void* mask = nullptr) {
   dim3 grid(ceil_div(g.Ncol, BN), ceil_div(g.M, BM));
   simt_conv_kernel<MODE, TA, TB, TC><<<grid, NT, 0, st>>>(
-      g, (const TA*)a, (const TB*)b, bias, (TC*)c, relu ? 1 : 0, acc ? 1 : 0);
+      g, (const TA*)a, (const TB*)b, bias, (TC*)c, relu ? 1 : 0, acc ? 1 : 0, (const TC*)mask);
 }
 
 // Instantiate every (A, B, C) dtype combination of one pass.
 template <int MODE, typename TA, typename TB>
 void launch_c(const Geo& g, const void* a, const void* b, const float* bias, void* c, int dtc,
-              bool relu, bool acc, cudaStream_t st) {
-  if (dtc == kF32) launch<MODE, TA, TB, float>(g, a, b, bias, c, relu, acc, st);
-  else launch<MODE, TA, TB, bf16>(g, a, b, bias, c, relu, acc, st);
+              bool relu, bool acc, cudaStream_t st, const void* mask) {
+  if (dtc == kF32) launch<MODE, TA, TB, float>(g, a, b, bias, c, relu, acc, st, mask);
+  else launch<MODE, TA, TB, bf16>(g, a, b, bias, c, relu, acc, st, mask);
 }
 template <int MODE, typename TA>
 void launch_bc(const Geo& g, const void* a, const void* b, int dtb, const float* bias, void* c,
-               int dtc, bool relu, bool acc, cudaStream_t st) {
-  if (dtb == kF32) launch_c<MODE, TA, float>(g, a, b, bias, c, dtc, relu, acc, st);
-  else launch_c<MODE, TA, bf16>(g, a, b, bias, c, dtc, relu, acc, st);
+               int dtc, bool relu, bool acc, cudaStream_t st, const void* mask) {
+  if (dtb == kF32) launch_c<MODE, TA, float>(g, a, b, bias, c, dtc, relu, acc, st, mask);
+  else launch_c<MODE, TA, bf16>(g, a, b, bias, c, dtc, relu, acc, st, mask);
 }
 template <int MODE>
 void launch_any(const Geo& g, const void* a, int dta, const void* b, int dtb, const float* bias,
-                void* c, int dtc, bool relu, bool acc, cudaStream_t st) {
-  if (dta == kF32) launch_bc<MODE, float>(g, a, b, dtb, bias, c, dtc, relu, acc, st);
-  else launch_bc<MODE, bf16>(g, a, b, dtb, bias, c, dtc, relu, acc, st);
+                void* c, int dtc, bool relu, bool acc, cudaStream_t st, const void* mask = nullptr) {
+  if (dta == kF32) launch_bc<MODE, float>(g, a, b, dtb, bias, c, dtc, relu, acc, st, mask);
+  else launch_bc<MODE, bf16>(g, a, b, dtb, bias, c, dtc, relu, acc, st, mask);
 }
 
 }  // namespace
@@ -186,8 +188,8 @@ void conv_fwd_simt(const ConvShape& s, const void* x, int dt_x, const void* w, i
 }
 
 void conv_dgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* w, int dt_w,
-                     void* dx, int dt_dx, bool accumulate, cudaStream_t st) {
-  launch_any<DGRAD>(make_geo(s, DGRAD), dy, dt_dy, w, dt_w, nullptr, dx, dt_dx, false, accumulate, st);
+                     void* dx, int dt_dx, bool accumulate, const void* mask, cudaStream_t st) {
+  launch_any<DGRAD>(make_geo(s, DGRAD), dy, dt_dy, w, dt_w, nullptr, dx, dt_dx, false, accumulate, st, mask);
 }
 
 void conv_wgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* x, int dt_x,

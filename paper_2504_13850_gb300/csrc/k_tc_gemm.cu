@@ -50,6 +50,7 @@ struct TcParams {
   void* out;
   int ldo;
   const float* bias;
+  const bf16* mask;     // ReLU mask (same layout as out): keep where mask > 0
   int relu, acc, out_f32;
   float* ws;            // split-K partials [splits][M][N] (fp32) or null
   int* err;
@@ -307,6 +308,17 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 #pragma unroll
         for (int j = 0; j < 16; ++j) v[j] = fmaxf(v[j], 0.f);
       }
+      if (p.mask) {
+        const uint4* mk = reinterpret_cast<const uint4*>(p.mask + size_t(m) * p.ldo + n);
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          uint4 u = mk[j];
+          const bf16* e = reinterpret_cast<const bf16*>(&u);
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            if (!(__bfloat162float(e[q]) > 0.f)) v[8 * j + q] = 0.f;
+        }
+      }
       if (p.out_f32) {
         float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + size_t(m) * p.ldo + n);
         if (p.acc) {
@@ -352,7 +364,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 // Deterministic split-K reduction (fixed order over splits) with the
 // epilogue of the unsplit kernel.
 __global__ void splitk_reduce_k(const float* __restrict__ ws, int splits, int M, int N, void* out, int ldo,
-                                const float* __restrict__ bias, int relu, int acc, int out_f32) {
+                                const float* __restrict__ bias, int relu, int acc, int out_f32,
+                                const bf16* __restrict__ mask) {
   const int64_t total4 = int64_t(M) * N / 4;
   for (int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; i < total4;
        i += int64_t(gridDim.x) * blockDim.x) {
@@ -366,6 +379,9 @@ __global__ void splitk_reduce_k(const float* __restrict__ ws, int splits, int M,
     float v[4] = {s.x, s.y, s.z, s.w};
     if (bias) for (int j = 0; j < 4; ++j) v[j] += bias[n + j];
     if (relu) for (int j = 0; j < 4; ++j) v[j] = fmaxf(v[j], 0.f);
+    if (mask)
+      for (int j = 0; j < 4; ++j)
+        if (!(__bfloat162float(mask[size_t(m) * ldo + n + j]) > 0.f)) v[j] = 0.f;
     if (out_f32) {
       float* d = reinterpret_cast<float*>(out) + size_t(m) * ldo + n;
       if (acc) for (int j = 0; j < 4; ++j) v[j] += d[j];
@@ -603,15 +619,16 @@ int tc_finalize(TcContext* c) {
 
 static const void* tensor_act(fo_server* s, int tid) { return s->T[tid].act; }
 
-TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i) {
+TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i, void* out, bool relu) {
   if (!c || !bf16_server(s) || getenv("FO_NO_TC")) return nullptr;
   const fo_op& op = s->ops[i];
   const Tensor& a = s->T[op.in0];
   const Tensor& o = s->T[i + 1];
   if (o.dt != kBF16) return nullptr;  // fp32 logits: CUDA-core path
   TcGemm* g = new TcGemm();
-  g->p.out = o.act;
+  g->p.out = out;
   g->p.ldo = o.C;
+  g->p.relu = relu ? 1 : 0;
   g->p.bias = op.bias ? s->theta + s->segs[s->op_segs[i][1]].off : nullptr;
   const bf16* w = s->shadow + s->segs[s->op_segs[i][0]].off;
   if (op.kind == FO_OP_LINEAR) {
@@ -655,16 +672,17 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i) {
   return finish(c, g, M, op.cout, double(g->p.taps) * op.cin);
 }
 
-TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate) {
+TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate, void* dx, const void* mask) {
   if (!c || !bf16_server(s) || getenv("FO_NO_TC")) return nullptr;
   const fo_op& op = s->ops[i];
   const Tensor& a = s->T[op.in0];
   const Tensor& o = s->T[i + 1];
   if (o.dt != kBF16) return nullptr;
   TcGemm* g = new TcGemm();
-  g->p.out = a.grad;
+  g->p.out = dx;
   g->p.ldo = a.C;
   g->p.acc = accumulate;
+  g->p.mask = static_cast<const bf16*>(mask);
   const bf16* w = s->shadow + s->segs[s->op_segs[i][0]].off;
   if (op.kind == FO_OP_LINEAR) {
     int bn = pick_bn(op.cin);
@@ -756,7 +774,7 @@ void tc_run_reduce(TcGemm* g, cudaStream_t st) {
   TcParams& p = g->p;
   int64_t n4 = int64_t(p.M) * p.N / 4;
   splitk_reduce_k<<<elementwise_blocks(n4, 256), 256, 0, st>>>(p.ws, g->splits, p.M, p.N, p.out, p.ldo, p.bias,
-                                                                p.relu, p.acc, p.out_f32);
+                                                                p.relu, p.acc, p.out_f32, p.mask);
 }
 
 int tc_splits(const TcGemm* g) { return g->splits; }
