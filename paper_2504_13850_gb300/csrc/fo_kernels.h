@@ -66,6 +66,8 @@ void meanpool_fwd(const void* x, const int32_t* len, void* y, int B, int L, int 
 void meanpool_bwd(const void* dy, const int32_t* len, void* dx, int B, int L, int C, int dt,
                   bool acc, cudaStream_t st);
 // Attention over packed qkv [B, L, 3C], heads h (C/h <= 64); probs fp32 [B,h,L,L] saved.
+// attention_prepare sets the kernels' shared-memory limits (call before use / capture).
+void attention_prepare(int L, int C, int heads);
 void attention_fwd(const void* qkv, const int32_t* len, void* out, float* probs, int B, int L,
                    int C, int heads, int dt, cudaStream_t st);
 void attention_bwd(const void* qkv, const int32_t* len, const float* probs, const void* out,
@@ -75,19 +77,22 @@ void attention_bwd(const void* qkv, const int32_t* len, const float* probs, cons
 // Classifier head (last linear layer + softmax cross-entropy), fp32 weights.
 void head_forward_loss(const void* x, int dt, const float* W, const float* bias, const int32_t* labels,
                        int B, int K, int C, float* logits, float* dz, float* row_loss, cudaStream_t st);
+// The batch loss goes to losses[*step & mask].
 void head_weight_grad(const float* dz, const void* x, int dt, int B, int K, int C, float* dW, float* db,
-                      const float* row_loss, float* loss_out, cudaStream_t st);
+                      const float* row_loss, float* losses, const int64_t* step, int64_t mask,
+                      cudaStream_t st);
 void head_input_grad(const float* dz, const float* W, int B, int K, int C, const void* mask, void* dx,
                      int dt, bool acc, cudaStream_t st);
 
-// Softmax cross-entropy: loss_slot <- mean_b CE; dlogits = (softmax - onehot)/B.
-void softmax_ce(const float* logits, const int32_t* labels, int B, int C, float* loss_slot,
-                void* dlogits, int dt, cudaStream_t st);
+// Softmax cross-entropy: losses[*step & mask] <- mean_b CE; dlogits = (softmax - onehot)/B.
+void softmax_ce(const float* logits, const int32_t* labels, int B, int C, float* losses,
+                const int64_t* step, int64_t mask, void* dlogits, int dt, cudaStream_t st);
 
 // SGD with momentum over a flat vector (n a multiple of 4, 16-byte aligned):
 // v = mu v + g; theta -= lr v; shadow (bf16, may be null) = bf16(theta).
+// The step counter (may be null) is incremented once, after the update.
 void sgd_momentum(float* theta, float* v, const float* g, void* shadow, int64_t n, float lr,
-                  float mu, cudaStream_t st);
+                  float mu, int64_t* step, cudaStream_t st);
 void f32_to_bf16(const float* x, void* y, int64_t n, cudaStream_t st);
 
 // FedAsync update: g = fmaf(alpha, l - g, g).

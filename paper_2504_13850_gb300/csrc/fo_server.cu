@@ -335,8 +335,8 @@ int build_plan(fo_server* s) {
   if (!fu.head) {
     const int lt = nops;
     add("softmax_ce", 1, 0.0, 2 * tbytes(lt), [=](cudaStream_t st) {
-      fo::softmax_ce((const float*)s->T[lt].act, s->cur_labels, s->cfg.batch, s->cfg.num_classes,
-                     s->losses + (s->steps_done & (s->kLossRing - 1)), s->T[lt].grad, fo::kF32, st);
+      fo::softmax_ce((const float*)s->T[lt].act, s->cur_labels, s->cfg.batch, s->cfg.num_classes, s->losses,
+                     s->d_step, s->kLossRing - 1, s->T[lt].grad, fo::kF32, st);
     });
   }
 
@@ -380,8 +380,8 @@ int build_plan(fo_server* s) {
       const int B = s->cfg.batch, K = op.cin, C = op.cout;
       add("head_wgrad", 1, 2.0 * B * K * C, tbytes(a0), [=](cudaStream_t st) {
         fo::head_weight_grad((const float*)s->T[o].grad, act(a0), s->T[a0].dt, B, K, C, G(s, i, 0),
-                             op.bias ? G(s, i, 1) : nullptr, s->row_loss,
-                             s->losses + (s->steps_done & (s->kLossRing - 1)), st);
+                             op.bias ? G(s, i, 1) : nullptr, s->row_loss, s->losses, s->d_step,
+                             s->kLossRing - 1, st);
       });
       if (need_dx) {
         int accf = contrib(a);
@@ -537,8 +537,10 @@ int build_plan(fo_server* s) {
 
   // ---------------- optimizer (Algorithm 4: theta_s <- theta_s - gamma_s * update)
   add("sgd_momentum", 1, 0.0, double(s->n_padded) * (20.0 + (s->shadow ? 2.0 : 0.0)), [=](cudaStream_t st) {
-    fo::sgd_momentum(s->theta, s->mom, s->grad, s->shadow, s->n_padded, s->opt.lr, s->opt.momentum, st);
+    fo::sgd_momentum(s->theta, s->mom, s->grad, s->shadow, s->n_padded, s->opt.lr, s->opt.momentum, s->d_step, st);
   });
+  for (int i = 0; i < nops; ++i)
+    if (s->ops[i].kind == FO_OP_ATTENTION) fo::attention_prepare(s->T[s->ops[i].in0].H, s->ops[i].cin, s->ops[i].heads);
   return FO_OK;
 }
 
@@ -612,6 +614,13 @@ int allocate(fo_server* s) {
   }
   s->losses = (float*)s->alloc(size_t(s->kLossRing) * 4);
   s->row_loss = (float*)s->alloc(size_t(s->cfg.batch) * 4);
+  s->d_step = (int64_t*)s->alloc(sizeof(int64_t));
+  if (!s->row_loss || !s->d_step) return set_err(FO_ERR_OOM, "scratch allocation");
+  FO_CUDA(cudaMemset(s->d_step, 0, sizeof(int64_t)));
+  s->graphs.assign(s->cfg.omega, nullptr);
+  s->prof_graphs.assign(s->cfg.omega, nullptr);
+  s->prof_events.assign(s->cfg.omega, {});
+  s->use_graphs = getenv("FO_NO_GRAPH") == nullptr;
   if (!s->colsum_scratch || !s->losses) return set_err(FO_ERR_OOM, "scratch allocation");
   FO_CUDA(cudaMemset(s->losses, 0, size_t(s->kLossRing) * 4));
   return FO_OK;
@@ -621,6 +630,13 @@ void destroy_impl(fo_server* s) {
   if (!s) return;
   if (s->cs) cudaStreamSynchronize(s->cs);
   if (s->xs) cudaStreamSynchronize(s->xs);
+  for (auto g : s->graphs) if (g) cudaGraphExecDestroy(g);
+  for (auto g : s->prof_graphs) if (g) cudaGraphExecDestroy(g);
+  for (auto& v : s->prof_events)
+    for (auto& r : v) {
+      cudaEventDestroy(r.a);
+      cudaEventDestroy(r.b);
+    }
   fo::tc_destroy(s->tc);
   for (auto e : s->slot_ready) if (e) cudaEventDestroy(e);
   for (auto e : s->slot_free) if (e) cudaEventDestroy(e);
@@ -641,6 +657,23 @@ int prof_id(fo_server* s, const char* name) {
     if (std::strcmp(s->prof_names[q], name) == 0) return int(q);
   s->prof_names.push_back(name);
   return int(s->prof_names.size()) - 1;
+}
+
+// Capture the step plan for batch slot `slot` into an executable graph.
+int capture_slot(fo_server* s, int slot, cudaGraphExec_t* out) {
+  const int B = s->cfg.batch;
+  s->cur_in = s->slab + size_t(slot) * s->slot_stride;
+  s->cur_labels = s->slot_labels + size_t(slot) * B;
+  s->cur_len = s->slot_lengths + size_t(slot) * B;
+  fo::tc_set_input(s->tc, slot);
+  cudaGraph_t g = nullptr;
+  FO_CUDA(cudaStreamBeginCapture(s->cs, cudaStreamCaptureModeRelaxed));
+  for (const Launch& l : s->plan) l.fn(s->cs);
+  FO_CUDA(cudaStreamEndCapture(s->cs, &g));
+  cudaError_t e = cudaGraphInstantiate(out, g, 0);
+  cudaGraphDestroy(g);
+  if (e != cudaSuccess) return set_err(FO_ERR_CUDA, std::string("graph instantiate: ") + cudaGetErrorString(e));
+  return FO_OK;
 }
 
 cudaEvent_t pool_event(fo_server* s) {
@@ -694,6 +727,8 @@ int fo_server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt, const
   if (rc == FO_OK) rc = fo::tc_create(&s->tc, s);
   if (rc == FO_OK) rc = build_plan(s);
   if (rc == FO_OK) rc = fo::tc_finalize(s->tc);
+  // Instantiate the step graph of every batch slot up front.
+  for (int sl = 0; rc == FO_OK && s->use_graphs && sl < c.omega; ++sl) rc = capture_slot(s, sl, &s->graphs[sl]);
   if (rc == FO_OK && cudaDeviceSynchronize() != cudaSuccess) rc = set_err(FO_ERR_CUDA, "create sync");
   if (rc != FO_OK) {
     destroy_impl(s);
@@ -781,17 +816,62 @@ int fo_server_step(fo_server* s, int* device_used, int32_t* slot_used) {
   fo::tc_set_input(s->tc, slot);
   FO_CUDA(cudaStreamWaitEvent(s->cs, s->slot_ready[slot], 0));
   int n = 0;
-  for (const Launch& l : s->plan) {
-    if (s->profiling) {
-      ProfRec r{prof_id(s, l.name), pool_event(s), pool_event(s), l.kernels, l.flops, l.bytes};
-      cudaEventRecord(r.a, s->cs);
-      l.fn(s->cs);
-      cudaEventRecord(r.b, s->cs);
-      s->prof.push_back(r);
-    } else {
-      l.fn(s->cs);
+  for (const Launch& l : s->plan) n += l.kernels;
+  if (!s->use_graphs) {
+    for (const Launch& l : s->plan) {
+      if (s->profiling) {
+        ProfRec r{prof_id(s, l.name), pool_event(s), pool_event(s), l.kernels, l.flops, l.bytes};
+        cudaEventRecord(r.a, s->cs);
+        l.fn(s->cs);
+        cudaEventRecord(r.b, s->cs);
+        s->prof.push_back(r);
+      } else {
+        l.fn(s->cs);
+      }
     }
-    n += l.kernels;
+  } else if (!s->profiling) {
+    // One CUDA graph per batch slot: the slot's address and tensor maps are
+    // the only per-step inputs the kernels take from the host.
+    cudaGraphExec_t& ge = s->graphs[slot];
+    if (!ge) {
+      int rc = capture_slot(s, slot, &ge);
+      if (rc != FO_OK) return rc;
+    }
+    FO_CUDA(cudaGraphLaunch(ge, s->cs));
+  } else {
+    // Profiled graph: event records around every plan entry, read back
+    // after the step (no host launch gaps inside the step).
+    cudaGraphExec_t& ge = s->prof_graphs[slot];
+    std::vector<ProfRec>& evs = s->prof_events[slot];
+    if (!ge) {
+      evs.clear();
+      cudaGraph_t g = nullptr;
+      FO_CUDA(cudaStreamBeginCapture(s->cs, cudaStreamCaptureModeRelaxed));
+      for (const Launch& l : s->plan) {
+        ProfRec r{prof_id(s, l.name), nullptr, nullptr, l.kernels, l.flops, l.bytes};
+        cudaEventCreate(&r.a);
+        cudaEventCreate(&r.b);
+        cudaEventRecord(r.a, s->cs);
+        l.fn(s->cs);
+        cudaEventRecord(r.b, s->cs);
+        evs.push_back(r);
+      }
+      FO_CUDA(cudaStreamEndCapture(s->cs, &g));
+      cudaError_t e = cudaGraphInstantiate(&ge, g, 0);
+      cudaGraphDestroy(g);
+      if (e != cudaSuccess) return set_err(FO_ERR_CUDA, std::string("graph instantiate: ") + cudaGetErrorString(e));
+    }
+    FO_CUDA(cudaGraphLaunch(ge, s->cs));
+    FO_CUDA(cudaStreamSynchronize(s->cs));
+    for (const ProfRec& r : evs) {
+      float t = 0.f;
+      FO_CUDA(cudaEventElapsedTime(&t, r.a, r.b));
+      ProfAcc& acc = s->prof_acc[s->prof_names[r.name_id]];
+      acc.launches += r.kernels;
+      acc.ms += t;
+      acc.flops += r.flops;
+      acc.bytes += r.bytes;
+    }
   }
   s->kernels_launched += n;
   FO_CUDA(cudaGetLastError());

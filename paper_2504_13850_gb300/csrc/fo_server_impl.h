@@ -84,6 +84,10 @@ struct fo_server {
   const int32_t* cur_len = nullptr;
   float* losses = nullptr;
   float* row_loss = nullptr;
+  int64_t* d_step = nullptr;   // device copy of steps_done (indexes the loss ring)
+  bool use_graphs = true;
+  std::vector<cudaGraphExec_t> graphs, prof_graphs;  // per batch slot
+  std::vector<std::vector<struct ProfRec>> prof_events;
   int64_t steps_done = 0;
   static constexpr int64_t kLossRing = int64_t(1) << 20;
 

@@ -168,14 +168,20 @@ size_t bwd_smem(int L, int dh) { return sizeof(float) * (4 * L * (dh + 1) + L * 
 
 }  // namespace
 
+void attention_prepare(int L, int C, int heads) {
+  const int f = int(fwd_smem(L, C / heads)), b = int(bwd_smem(L, C / heads));
+  cudaFuncSetAttribute(attn_fwd_k<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, f);
+  cudaFuncSetAttribute(attn_fwd_k<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, f);
+  cudaFuncSetAttribute(attn_bwd_k<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, b);
+  cudaFuncSetAttribute(attn_bwd_k<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, b);
+}
+
 void attention_fwd(const void* qkv, const int32_t* len, void* out, float* probs, int B, int L,
                    int C, int heads, int dt, cudaStream_t st) {
   size_t sm = fwd_smem(L, C / heads);
   if (dt == kF32) {
-    cudaFuncSetAttribute(attn_fwd_k<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
     attn_fwd_k<float><<<B * heads, 256, sm, st>>>((const float*)qkv, len, (float*)out, probs, L, C, heads);
   } else {
-    cudaFuncSetAttribute(attn_fwd_k<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
     attn_fwd_k<bf16><<<B * heads, 256, sm, st>>>((const bf16*)qkv, len, (bf16*)out, probs, L, C, heads);
   }
 }
@@ -185,12 +191,10 @@ void attention_bwd(const void* qkv, const int32_t* len, const float* probs, cons
                    cudaStream_t st) {
   size_t sm = bwd_smem(L, C / heads);
   if (dt == kF32) {
-    cudaFuncSetAttribute(attn_bwd_k<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
     attn_bwd_k<float><<<B * heads, 256, sm, st>>>((const float*)qkv, probs, (const float*)out,
                                                    (const float*)dout, len, (float*)dqkv, L, C,
                                                    heads, acc ? 1 : 0);
   } else {
-    cudaFuncSetAttribute(attn_bwd_k<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(sm));
     attn_bwd_k<bf16><<<B * heads, 256, sm, st>>>((const bf16*)qkv, probs, (const bf16*)out,
                                                   (const bf16*)dout, len, (bf16*)dqkv, L, C,
                                                   heads, acc ? 1 : 0);

@@ -427,8 +427,8 @@ void meanpool_bwd(const void* dy, const int32_t* len, void* dx, int B, int L, in
 // One block; warp w handles rows w, w + 8, ...  The batch-mean loss is
 // summed in a fixed order.
 template <typename T>
-__global__ void softmax_ce_k(const float* z, const int32_t* labels, int B, int C, float* loss_out,
-                             T* dz) {
+__global__ void softmax_ce_k(const float* z, const int32_t* labels, int B, int C, float* losses,
+                             const int64_t* step, int64_t mask, T* dz) {
   __shared__ float row_loss[1024];
   int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   for (int b = warp; b < B; b += blockDim.x / 32) {
@@ -452,19 +452,20 @@ __global__ void softmax_ce_k(const float* z, const int32_t* labels, int B, int C
   if (threadIdx.x == 0) {
     float t = 0.f;
     for (int b = 0; b < B; ++b) t += row_loss[b];
-    *loss_out = t / float(B);
+    losses[*step & mask] = t / float(B);
   }
 }
-void softmax_ce(const float* logits, const int32_t* labels, int B, int C, float* loss_slot,
-                void* dlogits, int dt, cudaStream_t st) {
-  FO_DISPATCH(dt, T, softmax_ce_k<T><<<1, 256, 0, st>>>(logits, labels, B, C, loss_slot, (T*)dlogits));
+void softmax_ce(const float* logits, const int32_t* labels, int B, int C, float* losses,
+                const int64_t* step, int64_t mask, void* dlogits, int dt, cudaStream_t st) {
+  FO_DISPATCH(dt, T, softmax_ce_k<T><<<1, 256, 0, st>>>(logits, labels, B, C, losses, step, mask, (T*)dlogits));
 }
 
 // ------------------------------------------------------ SGD with momentum
 // 16-byte vector loads/stores; n is a multiple of 4.
 __global__ void sgd_momentum_k(float4* __restrict__ theta, float4* __restrict__ v,
                                const float4* __restrict__ g, uint2* __restrict__ shadow,
-                               int64_t n4, float lr, float mu) {
+                               int64_t n4, float lr, float mu, int64_t* step) {
+  if (step && blockIdx.x == 0 && threadIdx.x == 0) *step += 1;
   GRID_STRIDE(i, n4) {
     float4 t = theta[i], m = v[i];
     const float4 gr = g[i];
@@ -488,10 +489,10 @@ __global__ void sgd_momentum_k(float4* __restrict__ theta, float4* __restrict__ 
   }
 }
 void sgd_momentum(float* theta, float* v, const float* g, void* shadow, int64_t n, float lr,
-                  float mu, cudaStream_t st) {
+                  float mu, int64_t* step, cudaStream_t st) {
   int64_t n4 = n / 4;
   sgd_momentum_k<<<elementwise_blocks(n4, 256), 256, 0, st>>>(
-      (float4*)theta, (float4*)v, (const float4*)g, (uint2*)shadow, n4, lr, mu);
+      (float4*)theta, (float4*)v, (const float4*)g, (uint2*)shadow, n4, lr, mu, step);
 }
 __global__ void f32_to_bf16_k(const float* x, bf16* y, int64_t n) {
   GRID_STRIDE(i, n) y[i] = __float2bfloat16_rn(x[i]);

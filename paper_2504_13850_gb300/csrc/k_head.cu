@@ -67,7 +67,7 @@ __global__ void head_fwd_ce_k(const T* __restrict__ x, const float* __restrict__
 template <typename T>
 __global__ void head_wgrad_k(const float* __restrict__ dz, const T* __restrict__ x, int B, int K, int C,
                              float* __restrict__ dW, float* __restrict__ db, const float* __restrict__ row_loss,
-                             float* __restrict__ loss_out) {
+                             float* __restrict__ losses, const int64_t* __restrict__ step, int64_t mask) {
   const int c = blockIdx.y;
   const int k = blockIdx.x * blockDim.x + threadIdx.x;
   if (k < K) {
@@ -84,7 +84,7 @@ __global__ void head_wgrad_k(const float* __restrict__ dz, const T* __restrict__
     if (c == 0) {
       float t = 0.f;
       for (int b = 0; b < B; ++b) t += row_loss[b];
-      *loss_out = t / float(B);
+      losses[*step & mask] = t / float(B);
     }
   }
 }
@@ -116,12 +116,13 @@ void head_forward_loss(const void* x, int dt, const float* W, const float* bias,
 }
 
 void head_weight_grad(const float* dz, const void* x, int dt, int B, int K, int C, float* dW, float* db,
-                      const float* row_loss, float* loss_out, cudaStream_t st) {
+                      const float* row_loss, float* losses, const int64_t* step, int64_t mask,
+                      cudaStream_t st) {
   dim3 grid(ceil_div(K, 256), C);
   if (dt == kF32)
-    head_wgrad_k<float><<<grid, 256, 0, st>>>(dz, (const float*)x, B, K, C, dW, db, row_loss, loss_out);
+    head_wgrad_k<float><<<grid, 256, 0, st>>>(dz, (const float*)x, B, K, C, dW, db, row_loss, losses, step, mask);
   else
-    head_wgrad_k<bf16><<<grid, 256, 0, st>>>(dz, (const bf16*)x, B, K, C, dW, db, row_loss, loss_out);
+    head_wgrad_k<bf16><<<grid, 256, 0, st>>>(dz, (const bf16*)x, B, K, C, dW, db, row_loss, losses, step, mask);
 }
 
 void head_input_grad(const float* dz, const float* W, int B, int K, int C, const void* mask, void* dx, int dt,
