@@ -851,9 +851,10 @@ int fo_server_step(fo_server* s, int* device_used, int32_t* slot_used) {
         ProfRec r{prof_id(s, l.name), nullptr, nullptr, l.kernels, l.flops, l.bytes};
         cudaEventCreate(&r.a);
         cudaEventCreate(&r.b);
-        cudaEventRecord(r.a, s->cs);
+        // External records become event nodes of the graph (timing events).
+        FO_CUDA(cudaEventRecordWithFlags(r.a, s->cs, cudaEventRecordExternal));
         l.fn(s->cs);
-        cudaEventRecord(r.b, s->cs);
+        FO_CUDA(cudaEventRecordWithFlags(r.b, s->cs, cudaEventRecordExternal));
         evs.push_back(r);
       }
       FO_CUDA(cudaStreamEndCapture(s->cs, &g));
