@@ -227,8 +227,6 @@ int build_plan(fo_server* s) {
   auto tbytes = [s](int tid) { return double(s->T[tid].bytes()); };
   auto add_tc = [&](fo::TcGemm* g) {
     add(fo::tc_name(g), 1, fo::tc_flops(g), 0.0, [=](cudaStream_t st) { fo::tc_run(g, nullptr, st); });
-    if (fo::tc_splits(g) > 1)
-      add("splitk_reduce", 1, 0.0, fo::tc_reduce_bytes(g), [=](cudaStream_t st) { fo::tc_run_reduce(g, st); });
   };
   const int L = nops - 1;  // the logits layer
 

@@ -23,13 +23,11 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int op, void* out, bool relu
 // multiplied by (mask > 0) when `mask` (same layout as dx) is given.
 TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int op, int accumulate, void* dx, const void* mask);
 TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int op);
-// Launches the GEMM kernel (split-K partials when tc_splits(g) > 1, then
-// tc_run_reduce must follow on the same stream).
+// Launches the GEMM kernel; a split-K plan runs as clusters of tc_splits(g)
+// CTAs that reduce their partial tiles through distributed shared memory.
 void tc_run(TcGemm* g, const void* input, cudaStream_t st);
-void tc_run_reduce(TcGemm* g, cudaStream_t st);
 int tc_splits(const TcGemm* g);
 double tc_flops(const TcGemm* g);
-double tc_reduce_bytes(const TcGemm* g);
 const char* tc_name(const TcGemm* g);
 // Allocates the split-K workspace after every plan is known.
 int tc_finalize(TcContext* c);

@@ -112,18 +112,111 @@ __global__ void maxpool2_bwd_k(const T* x, const T* dy, T* dx, int N, int H, int
     for (int q = 0; q < 4; ++q) store(dx, off[q], q == arg ? g : 0.f, acc);
   }
 }
+// 8 channels per thread with 16-byte loads (bf16, C % 8 == 0).
+__global__ void maxpool2_fwd_x8_k(const bf16* __restrict__ x, bf16* __restrict__ y, int N, int H, int W, int C) {
+  const int Ho = H / 2, Wo = W / 2, C8 = C / 8;
+  const int64_t n_out = int64_t(N) * Ho * Wo * C8;
+  GRID_STRIDE(o, n_out) {
+    const int c8 = int(o % C8);
+    int64_t t = o / C8;
+    const int j = int(t % Wo);
+    t /= Wo;
+    const int i = int(t % Ho);
+    const int n = int(t / Ho);
+    const int64_t b0 = ((int64_t(n) * H + 2 * i) * W + 2 * j) * C + 8 * c8;
+    const int64_t offs[4] = {b0, b0 + C, b0 + int64_t(W) * C, b0 + int64_t(W) * C + C};
+    uint4 u[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) u[q] = *reinterpret_cast<const uint4*>(x + offs[q]);
+    uint4 r;
+    bf16* rb = reinterpret_cast<bf16*>(&r);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      float m = __bfloat162float(reinterpret_cast<const bf16*>(&u[0])[e]);
+#pragma unroll
+      for (int q = 1; q < 4; ++q) m = fmaxf(m, __bfloat162float(reinterpret_cast<const bf16*>(&u[q])[e]));
+      rb[e] = __float2bfloat16_rn(m);
+    }
+    *reinterpret_cast<uint4*>(y + o * 8) = r;
+  }
+}
+
+// Backward of the above (optionally fused with the ReLU mask of x): the
+// window's gradient goes to its first maximum in row-major order.
+__global__ void maxpool2_bwd_x8_k(const bf16* __restrict__ x, const bf16* __restrict__ dy, bf16* __restrict__ dx,
+                                  int N, int H, int W, int C, int acc, int relu_mask) {
+  const int Ho = H / 2, Wo = W / 2, C8 = C / 8;
+  const int64_t n_out = int64_t(N) * Ho * Wo * C8;
+  GRID_STRIDE(o, n_out) {
+    const int c8 = int(o % C8);
+    int64_t t = o / C8;
+    const int j = int(t % Wo);
+    t /= Wo;
+    const int i = int(t % Ho);
+    const int n = int(t / Ho);
+    const int64_t b0 = ((int64_t(n) * H + 2 * i) * W + 2 * j) * C + 8 * c8;
+    const int64_t offs[4] = {b0, b0 + C, b0 + int64_t(W) * C, b0 + int64_t(W) * C + C};
+    uint4 u[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) u[q] = *reinterpret_cast<const uint4*>(x + offs[q]);
+    const uint4 g4 = *reinterpret_cast<const uint4*>(dy + o * 8);
+    const bf16* gb = reinterpret_cast<const bf16*>(&g4);
+    float out[4][8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      float best = __bfloat162float(reinterpret_cast<const bf16*>(&u[0])[e]);
+      int arg = 0;
+#pragma unroll
+      for (int q = 1; q < 4; ++q) {
+        const float v = __bfloat162float(reinterpret_cast<const bf16*>(&u[q])[e]);
+        if (v > best) { best = v; arg = q; }
+      }
+      float g = __bfloat162float(gb[e]);
+      if (relu_mask && !(best > 0.f)) g = 0.f;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) out[q][e] = q == arg ? g : 0.f;
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      uint4* d = reinterpret_cast<uint4*>(dx + offs[q]);
+      if (acc) {
+        const uint4 old = *d;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) out[q][e] += __bfloat162float(reinterpret_cast<const bf16*>(&old)[e]);
+      }
+      uint4 r;
+      bf16* rb = reinterpret_cast<bf16*>(&r);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) rb[e] = __float2bfloat16_rn(out[q][e]);
+      *d = r;
+    }
+  }
+}
+
 void maxpool2_fwd(const void* x, void* y, int N, int H, int W, int C, int dt, cudaStream_t st) {
   int64_t n = int64_t(N) * (H / 2) * (W / 2) * C;
+  if (dt == kBF16 && C % 8 == 0) {
+    maxpool2_fwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, (bf16*)y, N, H, W, C);
+    return;
+  }
   FO_DISPATCH(dt, T, maxpool2_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (T*)y, N, H, W, C));
 }
 void maxpool2_bwd(const void* x, const void* dy, void* dx, int N, int H, int W, int C, int dt,
                   bool acc, cudaStream_t st) {
   int64_t n = int64_t(N) * (H / 2) * (W / 2) * C;
+  if (dt == kBF16 && C % 8 == 0) {
+    maxpool2_bwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, (const bf16*)dy, (bf16*)dx, N, H, W, C, acc, 0);
+    return;
+  }
   FO_DISPATCH(dt, T, maxpool2_bwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (const T*)dy, (T*)dx, N, H, W, C, acc, 0));
 }
 void relu_maxpool2_bwd(const void* x, const void* dy, void* dx, int N, int H, int W, int C,
                        int dt, bool acc, cudaStream_t st) {
   int64_t n = int64_t(N) * (H / 2) * (W / 2) * C;
+  if (dt == kBF16 && C % 8 == 0) {
+    maxpool2_bwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, (const bf16*)dy, (bf16*)dx, N, H, W, C, acc, 1);
+    return;
+  }
   FO_DISPATCH(dt, T, maxpool2_bwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (const T*)dy, (T*)dx, N, H, W, C, acc, 1));
 }
 
@@ -291,9 +384,11 @@ void layernorm_bwd_dx(const void* x, const float* gamma, const float* mean, cons
 // ---------------------------------------------------- column reductions
 // Deterministic two-pass column sums: pass 1 writes one partial per
 // (row chunk, column), pass 2 adds the chunks in order.
-constexpr int CS_ROWS = 128;   // rows per chunk
+constexpr int CS_ROWS = 128;   // rows per chunk (generic kernel)
+constexpr int CS8_ROWS = 32;   // rows per chunk (16-byte bf16 kernel)
 static int colsum_chunks(int64_t rows) { return ceil_div(rows, CS_ROWS); }
-int64_t colsum_partial_floats(int64_t rows, int C) { return int64_t(colsum_chunks(rows)) * C; }
+static int colsum8_chunks(int64_t rows) { return ceil_div(rows, CS8_ROWS); }
+int64_t colsum_partial_floats(int64_t rows, int C) { return int64_t(colsum8_chunks(rows)) * C; }
 
 // MODE 0: a;  1: a * b;  2: a * (b - mean[r]) * rstd[r]
 template <int MODE, typename T>
@@ -341,18 +436,33 @@ __global__ void colsum_finish_k(const float* partial, int chunks, int C, float* 
 }
 
 // bf16 column sums with 16-byte loads: thread (g, r) adds columns
-// 8g..8g+7 over rows r, r + rl, ... of its chunk; the rl row lanes of a
-// block are combined in shared memory (fixed order).
+// 8g..8g+7 over rows r, r + rl, ... of its 32-row chunk (loads issued
+// before the adds); the rl row lanes of a block are combined in shared
+// memory in a fixed order.
 __global__ void colsum_bf16x8_k(const bf16* __restrict__ a, int64_t rows, int C, float* __restrict__ partial) {
   extern __shared__ float red[];  // [rl][C]
   const int groups = C / 8;
   const int g = threadIdx.x % groups, r = threadIdx.x / groups, rl = blockDim.x / groups;
-  const int64_t r0 = int64_t(blockIdx.x) * CS_ROWS;
+  const int64_t r0 = int64_t(blockIdx.x) * CS8_ROWS;
   float s[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
   if (r < rl) {
-    for (int64_t row = r0 + r; row < r0 + CS_ROWS && row < rows; row += rl) {
-      uint4 u = *reinterpret_cast<const uint4*>(a + row * C + 8 * g);
-      const bf16* e = reinterpret_cast<const bf16*>(&u);
+    constexpr int kMax = CS8_ROWS;  // rl >= 1
+    uint4 u[8];
+    int n = 0;
+    for (int64_t row = r0 + r; row < r0 + CS8_ROWS && row < rows && n < kMax; row += rl) {
+      if (n == 8) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const bf16* e = reinterpret_cast<const bf16*>(&u[q]);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) s[j] += __bfloat162float(e[j]);
+        }
+        n = 0;
+      }
+      u[n++] = *reinterpret_cast<const uint4*>(a + row * C + 8 * g);
+    }
+    for (int q = 0; q < n; ++q) {
+      const bf16* e = reinterpret_cast<const bf16*>(&u[q]);
 #pragma unroll
       for (int j = 0; j < 8; ++j) s[j] += __bfloat162float(e[j]);
     }
@@ -372,8 +482,8 @@ void colsum(const void* a, const void* b, int64_t rows, int C, int dt, float* pa
   if (!b && dt == kBF16 && C % 8 == 0 && C / 8 <= 256) {
     const int groups = C / 8;
     const int rl = 256 / groups;
-    colsum_bf16x8_k<<<colsum_chunks(rows), groups * rl, sizeof(float) * rl * C, st>>>((const bf16*)a, rows, C, partial);
-    colsum_finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, colsum_chunks(rows), C, out);
+    colsum_bf16x8_k<<<colsum8_chunks(rows), groups * rl, sizeof(float) * rl * C, st>>>((const bf16*)a, rows, C, partial);
+    colsum_finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, colsum8_chunks(rows), C, out);
     return;
   }
   dim3 grid(ceil_div(C, 32), colsum_chunks(rows));

@@ -63,19 +63,35 @@ __global__ void head_fwd_ce_k(const T* __restrict__ x, const float* __restrict__
   }
 }
 
-// dW[c][k] = sum_b dz[b][c] x[b][k]; grid (ceil(K/256), C).
+// dW[c][k] = sum_b dz[b][c] x[b][k]: block = 32 columns k x 8 classes c,
+// rows staged through shared memory 64 at a time; grid (ceil(K/32),
+// ceil(C/8)).  Block (0, y) also writes db for its classes; block (0, 0)
+// the batch-mean loss (row order).
 template <typename T>
 __global__ void head_wgrad_k(const float* __restrict__ dz, const T* __restrict__ x, int B, int K, int C,
                              float* __restrict__ dW, float* __restrict__ db, const float* __restrict__ row_loss,
                              float* __restrict__ losses, const int64_t* __restrict__ step, int64_t mask) {
-  const int c = blockIdx.y;
-  const int k = blockIdx.x * blockDim.x + threadIdx.x;
-  if (k < K) {
-    float s = 0.f;
-    for (int b = 0; b < B; ++b) s = fmaf(dz[int64_t(b) * C + c], to_f(x[int64_t(b) * K + k]), s);
-    dW[int64_t(c) * K + k] = s;
+  __shared__ float xs[64][33];
+  __shared__ float ds[64][8];
+  const int kk = threadIdx.x % 32, cc = threadIdx.x / 32;
+  const int k = blockIdx.x * 32 + kk, c = blockIdx.y * 8 + cc;
+  float acc = 0.f;
+  for (int b0 = 0; b0 < B; b0 += 64) {
+    for (int e = threadIdx.x; e < 64 * 32; e += blockDim.x) {
+      const int b = b0 + e / 32, kx = blockIdx.x * 32 + e % 32;
+      xs[e / 32][e % 32] = (b < B && kx < K) ? to_f(x[int64_t(b) * K + kx]) : 0.f;
+    }
+    for (int e = threadIdx.x; e < 64 * 8; e += blockDim.x) {
+      const int b = b0 + e / 8, cx = blockIdx.y * 8 + e % 8;
+      ds[e / 8][e % 8] = (b < B && cx < C) ? dz[int64_t(b) * C + cx] : 0.f;
+    }
+    __syncthreads();
+#pragma unroll 8
+    for (int b = 0; b < 64; ++b) acc = fmaf(ds[b][cc], xs[b][kk], acc);
+    __syncthreads();
   }
-  if (blockIdx.x == 0 && threadIdx.x == 0) {
+  if (k < K && c < C) dW[int64_t(c) * K + k] = acc;
+  if (blockIdx.x == 0 && kk == 0 && c < C) {
     if (db) {
       float s = 0.f;
       for (int b = 0; b < B; ++b) s += dz[int64_t(b) * C + c];
@@ -118,7 +134,7 @@ void head_forward_loss(const void* x, int dt, const float* W, const float* bias,
 void head_weight_grad(const float* dz, const void* x, int dt, int B, int K, int C, float* dW, float* db,
                       const float* row_loss, float* losses, const int64_t* step, int64_t mask,
                       cudaStream_t st) {
-  dim3 grid(ceil_div(K, 256), C);
+  dim3 grid(ceil_div(K, 32), ceil_div(C, 8));
   if (dt == kF32)
     head_wgrad_k<float><<<grid, 256, 0, st>>>(dz, (const float*)x, B, K, C, dW, db, row_loss, losses, step, mask);
   else

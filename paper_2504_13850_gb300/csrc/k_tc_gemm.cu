@@ -52,7 +52,6 @@ struct TcParams {
   const float* bias;
   const bf16* mask;     // ReLU mask (same layout as out): keep where mask > 0
   int relu, acc, out_f32;
-  float* ws;            // split-K partials [splits][M][N] (fp32) or null
   int* err;
 };
 
@@ -145,6 +144,63 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t map_to_cta(uint32_t smem_addr, uint32_t cta) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr), "r"(cta));
+  return r;
+}
+__device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
+
+// Epilogue of 4 consecutive outputs (m, n..n+3): bias, ReLU, ReLU mask,
+// accumulate, store as fp32 or bf16.
+__device__ __forceinline__ void store4(const TcParams& p, int m, int n, float4 a) {
+  float v[4] = {a.x, a.y, a.z, a.w};
+  if (p.bias)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) v[j] += p.bias[n + j];
+  if (p.relu)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) v[j] = fmaxf(v[j], 0.f);
+  if (p.mask) {
+    uint2 u = *reinterpret_cast<const uint2*>(p.mask + size_t(m) * p.ldo + n);
+    const bf16* e = reinterpret_cast<const bf16*>(&u);
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (!(__bfloat162float(e[j]) > 0.f)) v[j] = 0.f;
+  }
+  if (p.out_f32) {
+    float4* d = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + size_t(m) * p.ldo + n);
+    if (p.acc) {
+      float4 o = *d;
+      v[0] += o.x; v[1] += o.y; v[2] += o.z; v[3] += o.w;
+    }
+    *d = make_float4(v[0], v[1], v[2], v[3]);
+  } else {
+    uint2* d = reinterpret_cast<uint2*>(reinterpret_cast<bf16*>(p.out) + size_t(m) * p.ldo + n);
+    if (p.acc) {
+      uint2 o = *d;
+      const bf16* e = reinterpret_cast<const bf16*>(&o);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) v[j] += __bfloat162float(e[j]);
+    }
+    __nv_bfloat162 lo = __floats2bfloat162_rn(v[0], v[1]), hi = __floats2bfloat162_rn(v[2], v[3]);
+    uint2 u;
+    u.x = *reinterpret_cast<uint32_t*>(&lo);
+    u.y = *reinterpret_cast<uint32_t*>(&hi);
+    *d = u;
+  }
+}
+
 template <int KIND>
 struct KindTraits {
   static constexpr bool a_mn = (KIND == LIN_WGRAD || KIND == CONV_WGRAD);
@@ -192,7 +248,10 @@ __device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, i
   }
 }
 
-template <int KIND, int BN, int STAGES>
+// CLUSTER: the gridDim.z CTAs of a cluster split K; each stages its fp32
+// partial tile in shared memory and reduces a slice of rows over all the
+// cluster's partials (distributed shared memory, fixed order).
+template <int KIND, int BN, int STAGES, bool CLUSTER>
 __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ TcParams p) {
   extern __shared__ __align__(1024) char smem_raw[];
   char* smem = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -284,8 +343,23 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     const bool ready = mbar_wait(accum, 0);
     tc_fence_after();
     if (!ready) atomicExch(p.err, 3);
-    const int m = m0 + q * 32 + lane;
+    const int row = q * 32 + lane;
+    const int m = m0 + row;
     const bool valid = ready && !*abort_flag && nk > 0;
+    if (CLUSTER) {
+      // own partial tile -> shared memory (the pipeline buffers are idle now)
+      float* red = reinterpret_cast<float*>(smem);
+      for (int c = 0; c < BN; c += 16) {
+        uint32_t r[16];
+        tmem_ld16(tmem + (uint32_t(q * 32) << 16) + uint32_t(c), r);
+        float4* dst = reinterpret_cast<float4*>(red + row * (BN + 4) + c);
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          dst[j] = valid ? make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                                       __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]))
+                         : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+    } else {
     for (int c = 0; c < BN; c += 16) {
       uint32_t r[16];
       tmem_ld16(tmem + (uint32_t(q * 32) << 16) + uint32_t(c), r);
@@ -294,12 +368,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 #pragma unroll
       for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
       const int n = n0 + c;
-      if (p.ws) {
-        float4* dst = reinterpret_cast<float4*>(p.ws + (size_t(blockIdx.z) * p.M + m) * p.N + n);
-#pragma unroll
-        for (int j = 0; j < 4; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-        continue;
-      }
       if (p.bias) {
 #pragma unroll
         for (int j = 0; j < 16; ++j) v[j] += p.bias[n + j];
@@ -352,49 +420,36 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         dst[1] = pk[1];
       }
     }
+    }
+  }
+  if (CLUSTER) {
+    cluster_sync_all();
+    if (warp >= 2) {
+      const int S = gridDim.z, rank = blockIdx.z;
+      const int r0 = rank * BM / S, r1 = (rank + 1) * BM / S;
+      constexpr int n4 = BN / 4;
+      const int t = threadIdx.x - 64;
+      const uint32_t base = smem_u32(smem);
+      for (int e = t; e < (r1 - r0) * n4; e += 128) {
+        const int row = r0 + e / n4, c = (e % n4) * 4;
+        const int m = m0 + row;
+        if (m >= p.M) continue;
+        const uint32_t off = base + uint32_t((row * (BN + 4) + c) * 4);
+        float4 acc = ld_cluster_f4(map_to_cta(off, 0));
+        for (int z = 1; z < S; ++z) {
+          const float4 v = ld_cluster_f4(map_to_cta(off, uint32_t(z)));
+          acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+        }
+        store4(p, m, n0 + c, acc);
+      }
+    }
+    cluster_sync_all();
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kCols) : "memory");
-  }
-}
-
-// Deterministic split-K reduction (fixed order over splits) with the
-// epilogue of the unsplit kernel.
-__global__ void splitk_reduce_k(const float* __restrict__ ws, int splits, int M, int N, void* out, int ldo,
-                                const float* __restrict__ bias, int relu, int acc, int out_f32,
-                                const bf16* __restrict__ mask) {
-  const int64_t total4 = int64_t(M) * N / 4;
-  for (int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; i < total4;
-       i += int64_t(gridDim.x) * blockDim.x) {
-    const int64_t e = i * 4;
-    const int m = int(e / N), n = int(e % N);
-    float4 s = reinterpret_cast<const float4*>(ws)[i];
-    for (int z = 1; z < splits; ++z) {
-      const float4 t = reinterpret_cast<const float4*>(ws + size_t(z) * M * N)[i];
-      s.x += t.x; s.y += t.y; s.z += t.z; s.w += t.w;
-    }
-    float v[4] = {s.x, s.y, s.z, s.w};
-    if (bias) for (int j = 0; j < 4; ++j) v[j] += bias[n + j];
-    if (relu) for (int j = 0; j < 4; ++j) v[j] = fmaxf(v[j], 0.f);
-    if (mask)
-      for (int j = 0; j < 4; ++j)
-        if (!(__bfloat162float(mask[size_t(m) * ldo + n + j]) > 0.f)) v[j] = 0.f;
-    if (out_f32) {
-      float* d = reinterpret_cast<float*>(out) + size_t(m) * ldo + n;
-      if (acc) for (int j = 0; j < 4; ++j) v[j] += d[j];
-      *reinterpret_cast<float4*>(d) = make_float4(v[0], v[1], v[2], v[3]);
-    } else {
-      bf16* d = reinterpret_cast<bf16*>(out) + size_t(m) * ldo + n;
-      if (acc) for (int j = 0; j < 4; ++j) v[j] += __bfloat162float(d[j]);
-      __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]), b = __floats2bfloat162_rn(v[2], v[3]);
-      uint2 u;
-      u.x = *reinterpret_cast<uint32_t*>(&a);
-      u.y = *reinterpret_cast<uint32_t*>(&b);
-      *reinterpret_cast<uint2*>(d) = u;
-    }
   }
 }
 
@@ -410,17 +465,18 @@ constexpr size_t smem_bytes() {
 typedef void (*KernelFn)(const TcParams);
 
 template <int KIND, int BN>
-KernelFn kernel_ptr() {
-  return tc_gemm_kernel<KIND, BN, stages_for<KIND, BN>()>;
+KernelFn kernel_ptr(bool cluster) {
+  if (cluster) return tc_gemm_kernel<KIND, BN, stages_for<KIND, BN>(), true>;
+  return tc_gemm_kernel<KIND, BN, stages_for<KIND, BN>(), false>;
 }
 
-KernelFn pick_kernel(int kind, int bn, size_t* smem) {
+KernelFn pick_kernel(int kind, int bn, bool cluster, size_t* smem) {
 #define FO_PICK(K)                                                  \
   if (kind == K) {                                                  \
-    if (bn == 256) { *smem = smem_bytes<K, 256>(); return kernel_ptr<K, 256>(); } \
-    if (bn == 128) { *smem = smem_bytes<K, 128>(); return kernel_ptr<K, 128>(); } \
+    if (bn == 256) { *smem = smem_bytes<K, 256>(); return kernel_ptr<K, 256>(cluster); } \
+    if (bn == 128) { *smem = smem_bytes<K, 128>(); return kernel_ptr<K, 128>(cluster); } \
     *smem = smem_bytes<K, 64>();                                    \
-    return kernel_ptr<K, 64>();                                     \
+    return kernel_ptr<K, 64>(cluster);                              \
   }
   FO_PICK(LIN_FWD)
   FO_PICK(LIN_DGRAD)
@@ -507,8 +563,6 @@ struct TcContext {
   int num_sms = 148;
   int slot = 0;
   int* err = nullptr;
-  float* ws = nullptr;
-  size_t ws_floats = 0;
   fo_server* s = nullptr;
 };
 
@@ -540,9 +594,12 @@ int pick_bn(int N) {
   return 0;
 }
 
+// Split K over a cluster of up to 8 CTAs (portable cluster size) when the
+// output tiles alone leave SMs idle; each split keeps >= 4 k-blocks.
 void choose_split(TcContext* c, TcGemm* g, int tiles, int KB) {
   int want = std::max(1, c->num_sms / std::max(1, tiles));
   want = std::min(want, std::max(1, KB / 4));
+  want = std::min(want, 8);
   int kper = (KB + want - 1) / want;
   g->splits = (KB + kper - 1) / kper;
   g->p.kper = kper;
@@ -554,7 +611,7 @@ TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
   g->p.N = N;
   g->flops = 2.0 * M * N * K;
   g->p.err = c->err;
-  g->fn = pick_kernel(g->kind, g->bn, &g->smem);
+  g->fn = pick_kernel(g->kind, g->bn, g->splits > 1, &g->smem);
   if (!g->fn) {
     delete g;
     return nullptr;
@@ -564,10 +621,6 @@ TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
     return nullptr;
   }
   g->grid = dim3(N / g->bn, (M + BM - 1) / BM, g->splits);
-  if (g->splits > 1) {
-    size_t need = size_t(g->splits) * M * N;
-    c->ws_floats = std::max(c->ws_floats, need);
-  }
   g->ctx = c;
   c->gemms.push_back(g);
   return g;
@@ -607,13 +660,7 @@ int* tc_error_word(TcContext* c) { return c ? c->err : nullptr; }
 
 // Allocate the split-K workspace once every plan is known.
 int tc_finalize(TcContext* c) {
-  if (!c) return FO_OK;
-  if (c->ws_floats) {
-    c->ws = (float*)c->s->alloc(c->ws_floats * sizeof(float));
-    if (!c->ws) return FO_ERR_OOM;
-  }
-  for (TcGemm* g : c->gemms)
-    if (g->splits > 1) g->p.ws = c->ws;
+  (void)c;
   return FO_OK;
 }
 
@@ -767,23 +814,27 @@ void tc_run(TcGemm* g, const void* input, cudaStream_t st) {
   TcContext* c = g->ctx;
   if (g->input_A) g->p.tmA = g->slot_maps[c->slot];
   if (g->input_B) g->p.tmB = g->slot_maps[c->slot];
-  g->fn<<<g->grid, kThreads, g->smem, st>>>(g->p);
-}
-
-void tc_run_reduce(TcGemm* g, cudaStream_t st) {
-  TcParams& p = g->p;
-  int64_t n4 = int64_t(p.M) * p.N / 4;
-  splitk_reduce_k<<<elementwise_blocks(n4, 256), 256, 0, st>>>(p.ws, g->splits, p.M, p.N, p.out, p.ldo, p.bias,
-                                                                p.relu, p.acc, p.out_f32, p.mask);
+  if (g->splits == 1) {
+    g->fn<<<g->grid, kThreads, g->smem, st>>>(g->p);
+    return;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = g->grid;
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = g->smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 1;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = g->splits;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaLaunchKernelEx(&cfg, g->fn, g->p);
 }
 
 int tc_splits(const TcGemm* g) { return g->splits; }
 double tc_flops(const TcGemm* g) { return g->flops; }
-double tc_reduce_bytes(const TcGemm* g) {
-  const TcParams& p = g->p;
-  double mn = double(p.M) * p.N;
-  return mn * 4.0 * g->splits + mn * (p.out_f32 ? 4.0 : 2.0) * (p.acc ? 2 : 1);
-}
 
 const char* tc_name(const TcGemm* g) { return g->name; }
 
