@@ -152,12 +152,13 @@ __device__ __forceinline__ uint32_t map_to_cta(uint32_t smem_addr, uint32_t cta)
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr), "r"(cta));
   return r;
 }
+// Read of another CTA's shared memory; ordered by the cluster barriers
+// around the reduction (no memory clobber, so loads can overlap).
 __device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr) {
   float4 v;
   asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
                : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "r"(addr)
-               : "memory");
+               : "r"(addr));
   return v;
 }
 
@@ -198,6 +199,40 @@ __device__ __forceinline__ void store4(const TcParams& p, int m, int n, float4 a
     u.x = *reinterpret_cast<uint32_t*>(&lo);
     u.y = *reinterpret_cast<uint32_t*>(&hi);
     *d = u;
+  }
+}
+
+// Sum of the S partial tiles at G elements per batch, all S*G remote loads
+// issued before the adds (fixed order over z).
+template <int BN, int S, int G>
+__device__ __forceinline__ void cluster_reduce_rows(const TcParams& p, uint32_t base, int r0, int r1, int m0,
+                                                    int n0, int t) {
+  constexpr int n4 = BN / 4;
+  const int total = (r1 - r0) * n4;
+  for (int e0 = t; e0 < total; e0 += 128 * G) {
+    float4 v[G][S];
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const int e = e0 + g * 128;
+      const int row = r0 + (e < total ? e : 0) / n4, c = ((e < total ? e : 0) % n4) * 4;
+      const uint32_t off = base + uint32_t((row * (BN + 4) + c) * 4);
+#pragma unroll
+      for (int z = 0; z < S; ++z) v[g][z] = ld_cluster_f4(map_to_cta(off, uint32_t(z)));
+    }
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const int e = e0 + g * 128;
+      if (e >= total) continue;
+      const int row = r0 + e / n4, c = (e % n4) * 4;
+      const int m = m0 + row;
+      if (m >= p.M) continue;
+      float4 acc = v[g][0];
+#pragma unroll
+      for (int z = 1; z < S; ++z) {
+        acc.x += v[g][z].x; acc.y += v[g][z].y; acc.z += v[g][z].z; acc.w += v[g][z].w;
+      }
+      store4(p, m, n0 + c, acc);
+    }
   }
 }
 
@@ -427,21 +462,16 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     if (warp >= 2) {
       const int S = gridDim.z, rank = blockIdx.z;
       const int r0 = rank * BM / S, r1 = (rank + 1) * BM / S;
-      constexpr int n4 = BN / 4;
       const int t = threadIdx.x - 64;
       const uint32_t base = smem_u32(smem);
-      for (int e = t; e < (r1 - r0) * n4; e += 128) {
-        const int row = r0 + e / n4, c = (e % n4) * 4;
-        const int m = m0 + row;
-        if (m >= p.M) continue;
-        const uint32_t off = base + uint32_t((row * (BN + 4) + c) * 4);
-        float4 acc = ld_cluster_f4(map_to_cta(off, 0));
-        for (int z = 1; z < S; ++z) {
-          const float4 v = ld_cluster_f4(map_to_cta(off, uint32_t(z)));
-          acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
-        }
-        store4(p, m, n0 + c, acc);
-      }
+      if (S == 2) cluster_reduce_rows<BN, 2, 8>(p, base, r0, r1, m0, n0, t);
+      else if (S == 3) cluster_reduce_rows<BN, 3, 4>(p, base, r0, r1, m0, n0, t);
+      else if (S == 4) cluster_reduce_rows<BN, 4, 4>(p, base, r0, r1, m0, n0, t);
+      else if (S <= 6) {
+        if (S == 5) cluster_reduce_rows<BN, 5, 2>(p, base, r0, r1, m0, n0, t);
+        else cluster_reduce_rows<BN, 6, 2>(p, base, r0, r1, m0, n0, t);
+      } else if (S == 7) cluster_reduce_rows<BN, 7, 2>(p, base, r0, r1, m0, n0, t);
+      else cluster_reduce_rows<BN, 8, 2>(p, base, r0, r1, m0, n0, t);
     }
     cluster_sync_all();
   }
@@ -587,23 +617,42 @@ bool window_ok(int N, int H, int W, int rows_needed, int* rows, int* imgs) {
   return true;
 }
 
-int pick_bn(int N) {
-  if (N % 256 == 0) return 256;
-  if (N % 128 == 0) return 128;
-  if (N % 64 == 0) return 64;
-  return 0;
-}
 
-// Split K over a cluster of up to 8 CTAs (portable cluster size) when the
-// output tiles alone leave SMs idle; each split keeps >= 4 k-blocks.
-void choose_split(TcContext* c, TcGemm* g, int tiles, int KB) {
-  int want = std::max(1, c->num_sms / std::max(1, tiles));
-  want = std::min(want, std::max(1, KB / 4));
-  want = std::min(want, 8);
-  int kper = (KB + want - 1) / want;
-  g->splits = (KB + kper - 1) / kper;
-  g->p.kper = kper;
+// Tile width and K split from a small cost model.  One CTA per SM; a CTA
+// costs its k-blocks (a 128-wide k-block runs at ~0.55 of a 256-wide one)
+// plus its epilogue, plus the cluster reduction when K is split; a split
+// cluster holds <= 8 CTAs (portable size) and clusters above 4 pay for
+// their poorer packing into GPCs.  Minimises waves x cost per CTA.
+// Candidate widths divide `ndiv` (N, or the channels of one tap for the
+// weight gradient, whose N index runs over taps x channels).
+void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv) {
+  double best = 1e30;
+  int best_bn = 0, best_s = 1;
+  for (int bn : {256, 128, 64}) {
+    if (ndiv % bn || N % bn) continue;
+    const int tiles = ((M + BM - 1) / BM) * (N / bn);
+    const double per_kb = bn == 256 ? 1.0 : (bn == 128 ? 0.55 : 0.4);
+    const double epi = bn / 64.0;
+    for (int sp = 1; sp <= 8; ++sp) {
+      if (sp > 1 && KB / sp < 4) break;
+      const int kper = (KB + sp - 1) / sp;
+      const int splits = (KB + kper - 1) / kper;
+      if (splits != sp) continue;
+      const int ctas = tiles * splits;
+      const double waves = double((ctas + c->num_sms - 1) / c->num_sms);
+      double cost = waves * (kper * per_kb + epi + (splits > 1 ? 2.0 : 0.0));
+      if (splits > 4) cost *= 1.2;
+      if (cost < best - 1e-9) {
+        best = cost;
+        best_bn = bn;
+        best_s = splits;
+      }
+    }
+  }
+  g->bn = best_bn;
   g->p.KB = KB;
+  g->p.kper = (KB + best_s - 1) / best_s;
+  g->splits = best_s;
 }
 
 TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
@@ -621,6 +670,9 @@ TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
     return nullptr;
   }
   g->grid = dim3(N / g->bn, (M + BM - 1) / BM, g->splits);
+  if (getenv("FO_DEBUG_PLAN"))
+    fprintf(stderr, "[plan] %-16s M=%d N=%d KB=%d BN=%d splits=%d grid=(%u,%u,%u)\n", g->name, M, N, g->p.KB,
+            g->bn, g->splits, g->grid.x, g->grid.y, g->grid.z);
   g->ctx = c;
   c->gemms.push_back(g);
   return g;
@@ -679,13 +731,12 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i, void* out, bool relu)
   g->p.bias = op.bias ? s->theta + s->segs[s->op_segs[i][1]].off : nullptr;
   const bf16* w = s->shadow + s->segs[s->op_segs[i][0]].off;
   if (op.kind == FO_OP_LINEAR) {
-    int bn = pick_bn(op.cout);
-    if (!bn || op.cin % 64) { delete g; return nullptr; }
+    if (op.cout % 64 || op.cin % 64) { delete g; return nullptr; }
     g->kind = LIN_FWD;
-    g->bn = bn;
     g->name = "tc_linear_fwd";
     int M = int(a.rows()), KB = op.cin / 64;
-    choose_split(c, g, (M + BM - 1) / BM * (op.cout / bn), KB);
+    choose_tiles(c, g, M, op.cout, KB, op.cout);
+    const int bn = g->bn;
     g->input_A = (op.in0 == 0);
     if (g->input_A) {
       g->slot_maps.resize(s->cfg.omega);
@@ -699,16 +750,15 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i, void* out, bool relu)
   if (op.stride != 1 || op.cin % 64 || op.cout % 64) { delete g; return nullptr; }
   int rows, imgs;
   if (!window_ok(a.N, a.H, a.W, BM, &rows, &imgs) || (int64_t(a.N) * a.H * a.W) % BM) { delete g; return nullptr; }
-  int bn = pick_bn(op.cout);
   g->kind = CONV_FPROP;
-  g->bn = bn;
   g->name = "tc_conv_fprop";
   g->p.H = a.H; g->p.W = a.W; g->p.ksz = op.k; g->p.pad = op.k / 2; g->p.taps = op.k * op.k;
   g->p.cblocks = op.cin / 64;
   g->p.ntap_ch = op.cin;
   g->p.win_rows = rows; g->p.win_imgs = imgs;
   int M = a.N * a.H * a.W, KB = g->p.taps * g->p.cblocks;
-  choose_split(c, g, M / BM * (op.cout / bn), KB);
+  choose_tiles(c, g, M, op.cout, KB, op.cout);
+  const int bn = g->bn;
   g->input_A = (op.in0 == 0);
   if (g->input_A) {
     g->slot_maps.resize(s->cfg.omega);
@@ -732,28 +782,24 @@ TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate, void* d
   g->p.mask = static_cast<const bf16*>(mask);
   const bf16* w = s->shadow + s->segs[s->op_segs[i][0]].off;
   if (op.kind == FO_OP_LINEAR) {
-    int bn = pick_bn(op.cin);
-    if (!bn || op.cout % 64) { delete g; return nullptr; }
+    if (op.cin % 64 || op.cout % 64) { delete g; return nullptr; }
     g->kind = LIN_DGRAD;
-    g->bn = bn;
     g->name = "tc_linear_dgrad";
     int M = int(a.rows()), KB = op.cout / 64;
-    choose_split(c, g, (M + BM - 1) / BM * (op.cin / bn), KB);
+    choose_tiles(c, g, M, op.cin, KB, op.cin);
     if (!map_2d(&g->p.tmA, o.grad, M, op.cout, BM) || !map_2d(&g->p.tmB, w, op.cout, op.cin, BK)) { delete g; return nullptr; }
     return finish(c, g, M, op.cin, double(op.cout));
   }
   if (op.stride != 1 || op.cin % 64 || op.cout % 64) { delete g; return nullptr; }
   int rows, imgs;
   if (!window_ok(o.N, o.H, o.W, BM, &rows, &imgs) || (int64_t(a.N) * a.H * a.W) % BM) { delete g; return nullptr; }
-  int bn = pick_bn(op.cin);
   g->kind = CONV_DGRAD;
-  g->bn = bn;
   g->name = "tc_conv_dgrad";
   g->p.H = o.H; g->p.W = o.W; g->p.ksz = op.k; g->p.pad = op.k / 2; g->p.taps = op.k * op.k;
   g->p.cblocks = op.cout / 64;
   g->p.ntap_ch = op.cin;
   int M = a.N * a.H * a.W, KB = g->p.taps * g->p.cblocks;
-  choose_split(c, g, M / BM * (op.cin / bn), KB);
+  choose_tiles(c, g, M, op.cin, KB, op.cin);
   if (!map_window(&g->p.tmA, o.grad, o.N, o.H, o.W, o.C, rows, imgs) ||
       !map_2d(&g->p.tmB, w, op.cout, int64_t(g->p.taps) * op.cin, BK)) { delete g; return nullptr; }
   return finish(c, g, M, op.cin, double(g->p.taps) * op.cout);
@@ -769,14 +815,12 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
   g->p.out = s->grad + s->segs[s->op_segs[i][0]].off;
   g->p.out_f32 = 1;
   if (op.kind == FO_OP_LINEAR) {
-    int bn = pick_bn(op.cin);
-    if (!bn || op.cout % 128) { delete g; return nullptr; }
+    if (op.cin % 64 || op.cout % 128) { delete g; return nullptr; }
     g->kind = LIN_WGRAD;
-    g->bn = bn;
     g->name = "tc_linear_wgrad";
     g->p.ldo = op.cin;
     int rows = int(a.rows()), KB = (rows + BK - 1) / BK;
-    choose_split(c, g, op.cout / BM * (op.cin / bn), KB);
+    choose_tiles(c, g, op.cout, op.cin, KB, op.cin);
     g->input_B = (op.in0 == 0);
     if (!map_2d(&g->p.tmA, o.grad, rows, op.cout, BK)) { delete g; return nullptr; }
     if (g->input_B) {
@@ -789,16 +833,14 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
   if (op.stride != 1 || op.cin % 64 || op.cout % 128) { delete g; return nullptr; }
   int rows, imgs;
   if (!window_ok(a.N, a.H, a.W, BK, &rows, &imgs) || (int64_t(a.N) * a.H * a.W) % BK) { delete g; return nullptr; }
-  int bn = op.cin % 256 == 0 ? 256 : (op.cin % 128 == 0 ? 128 : 64);
   g->kind = CONV_WGRAD;
-  g->bn = bn;
   g->name = "tc_conv_wgrad";
   g->p.ldo = op.k * op.k * op.cin;
   g->p.H = a.H; g->p.W = a.W; g->p.ksz = op.k; g->p.pad = op.k / 2; g->p.taps = op.k * op.k;
   g->p.ntap_ch = op.cin;
   int P = a.N * a.H * a.W, KB = P / BK;
   int N = g->p.taps * op.cin;
-  choose_split(c, g, op.cout / BM * (N / bn), KB);
+  choose_tiles(c, g, op.cout, N, KB, op.cin);
   g->input_B = (op.in0 == 0);
   if (!map_2d(&g->p.tmA, o.grad, P, op.cout, BK)) { delete g; return nullptr; }
   if (g->input_B) {
