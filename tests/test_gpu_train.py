@@ -90,24 +90,27 @@ def test_tiny_config_fp32_full_trace():
     assert [int(c) for c in s.counters()] == o.sched.c == [2, 2, 2, 2]
 
 
-def check_teacher_forced(recs, loss_tol=1e-2, param_tol=2e-2, kernel_loss_tol=2e-3,
-                         kernel_grad_tol=1e-2, flip_tol=8e-2):
+def check_teacher_forced(recs, loss_tol=1e-2, param_tol=2e-2, kernel_loss_tol=2e-3, clean_tol=3e-2,
+                         flip_tol=8e-2, decisions=True):
     """Gates of each step.
 
     Against the exact oracle (the stated tolerances): loss within 1e-2
     relative, parameters within 2e-2 normwise.
 
     Against the bf16-storage reading (same stored values, so ReLU / max-pool
-    decisions are taken alike): loss within 2e-3, and the gradient of every
-    parameter tensor within 1e-2 normwise on most steps.  What is left after
-    the shared rounding is fp32 accumulation order (~1e-6) and one-ulp
-    rounding differences of rare elements, a few 1e-3 over a backward chain.
-    A value that lands within accumulation error of a decision (a ReLU input
-    at 0, a max-pool near-tie) can still be decided the other way; one such
-    flip in a layer of B*U decision elements moves that layer's gradient,
-    and everything upstream of it, by about 1/sqrt(B*U_active) -- 3.6% for
-    the small configurations here (B = 12, U_active ~ 64).  So every step must
-    stay within 8e-2 and at least two thirds of the steps within 1e-2."""
+    decisions are taken on the same bf16 numbers): loss within 2e-3 and the
+    gradient of every parameter tensor normwise.  Without decisions (conv /
+    linear / layernorm / attention / GELU chains) what is left is fp32
+    accumulation order (~1e-6) and one-ulp bf16 rounding differences of rare
+    elements, a few 1e-3 over a backward chain: every tensor within 1e-2 on
+    every step.  With decisions, a stored value that lands one bf16 ulp
+    apart can still decide a ReLU at 0 or a max-pool tie (ties are common in
+    bf16) the other way; each such flip re-routes one gradient element and
+    moves the weight gradient of its layer, and everything upstream, by
+    about 1/sqrt(#gradient elements of that layer) -- up to 3.6% for the
+    small FC layer here, ~0.6% per max-pool flip with a few flips per step.
+    So there every tensor stays within 8e-2 on every step and within 3e-2
+    on at least half of the steps."""
     clean = 0
     for r in recs:
         ex, st = r["exact"], r["stored"]
@@ -115,9 +118,11 @@ def check_teacher_forced(recs, loss_tol=1e-2, param_tol=2e-2, kernel_loss_tol=2e
         assert ex["param_err"] <= param_tol, r
         assert abs(r["loss"] - st["loss"]) <= kernel_loss_tol * abs(st["loss"]), r
         worst = max(st["tensor_grad_err"].values())
+        if not decisions:
+            assert worst <= 1e-2, (r["step"], st["tensor_grad_err"])
         assert worst <= flip_tol, (r["step"], st["tensor_grad_err"])
-        clean += worst <= kernel_grad_tol
-    assert 3 * clean >= 2 * len(recs), [max(r["stored"]["tensor_grad_err"].values()) for r in recs]
+        clean += worst <= clean_tol
+    assert 2 * clean >= len(recs), [max(r["stored"]["tensor_grad_err"].values()) for r in recs]
 
 
 @pytest.mark.parametrize("kind", ["vgg", "resnet", "transformer"])
@@ -127,7 +132,40 @@ def test_small_bf16_configs_teacher_forced(kind):
     cfg = small(kind)
     _, _, recs = teacher_forced(cfg, prefill_then_steps(cfg, 6))
     assert len(recs) == 6
-    check_teacher_forced(recs)
+    check_teacher_forced(recs, decisions=kind != "transformer")
+
+
+def decision_free(kind):
+    """Conv / linear stacks without ReLU or max-pool: the tensor-core
+    forward, input-gradient and weight-gradient kernels (tile widths 64-256,
+    K split over clusters) checked without decision flips."""
+    b = W._Builder()
+    if kind == "conv16":
+        t = b.add("conv", 0, cin=64, cout=128, k=3, stride=1, bias=1)
+        t = b.add("conv", t, cin=128, cout=128, k=3, stride=1, bias=1)
+        t = b.add("flatten", t)
+        t = b.add("linear", t, cin=16 * 16 * 128, cout=128, bias=1)
+        b.add("linear", t, cin=128, cout=10, bias=1)
+        return W.shrink(W.CONFIGS["vgg"], ops=b.ops, batch=12, in_hwc=(16, 16, 64), K=3, omega=6, depth=2,
+                        lr=1e-3)
+    if kind == "conv8":
+        t = b.add("conv", 0, cin=128, cout=256, k=3, stride=1, bias=1)
+        t = b.add("conv", t, cin=256, cout=512, k=3, stride=1, bias=1)
+        t = b.add("conv", t, cin=512, cout=256, k=3, stride=1, bias=1)
+        t = b.add("flatten", t)
+        t = b.add("linear", t, cin=8 * 8 * 256, cout=256, bias=1)
+        b.add("linear", t, cin=256, cout=10, bias=1)
+        return W.shrink(W.CONFIGS["vgg"], ops=b.ops, batch=20, in_hwc=(8, 8, 128), K=3, omega=6, depth=2,
+                        lr=1e-3)
+    raise ValueError(kind)
+
+
+@pytest.mark.parametrize("kind", ["conv16", "conv8"])
+def test_decision_free_teacher_forced(kind):
+    cfg = decision_free(kind)
+    _, _, recs = teacher_forced(cfg, prefill_then_steps(cfg, 4))
+    assert len(recs) == 4
+    check_teacher_forced(recs, decisions=False)
 
 
 @pytest.mark.parametrize("kind", ["vgg", "resnet", "transformer"])
