@@ -237,6 +237,19 @@ FO_API int fo_sched_queued(const fo_sched* s, int k); /* |Q_k|, or the total whe
 FO_API int fo_axpby_async(float* global, const float* local, int64_t n, float alpha,
                    void* stream);
 
+/* ------------------------------------------------------------------------
+ * Deterministic column sums out[c] = sum_r x[r][c] of a row-major
+ * [rows][cols] matrix: the reduction the server uses for bias gradients
+ * (the sum over all positions of a layer's output gradient).  x is a device
+ * pointer to fp32 (dtype FO_DTYPE_F32) or bf16 (FO_DTYPE_BF16) values, out a
+ * device pointer to `cols` floats; partial sums over 32-row chunks are added
+ * in a fixed order, so results are bitwise reproducible.  The partial sums
+ * live in scratch this call allocates and frees stream-ordered on `stream`
+ * (a cudaStream_t, NULL = default stream).  FO_ERR_ARG for rows < 1,
+ * cols < 1 or an unknown dtype.
+ * ---------------------------------------------------------------------- */
+FO_API int fo_column_sums(const void* x, int dtype, int64_t rows, int cols, float* out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

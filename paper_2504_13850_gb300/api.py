@@ -90,6 +90,7 @@ _SIGS = [
     ("fo_sched_sender_status", C.c_int, [C.c_void_p, C.c_void_p]),
     ("fo_sched_queued", C.c_int, [C.c_void_p, C.c_int]),
     ("fo_axpby_async", C.c_int, [C.c_void_p, C.c_void_p, C.c_int64, C.c_float, C.c_void_p]),
+    ("fo_column_sums", C.c_int, [C.c_void_p, C.c_int, C.c_int64, C.c_int, C.c_void_p, C.c_void_p]),
 ]
 
 
@@ -339,6 +340,13 @@ class Scheduler:
 
     def queued(self, k=-1):
         return lib().fo_sched_queued(self.h, k)
+
+
+def column_sums(x, out, stream=None):
+    """out[c] = sum_r x[r][c] for a 2-D fp32 / bf16 device tensor x."""
+    import torch
+    dt = DTYPE_BF16 if x.dtype == torch.bfloat16 else DTYPE_F32
+    return lib().fo_column_sums(_ptr(x), dt, x.shape[0], x.shape[1], _ptr(out), stream)
 
 
 def axpby_async(global_, local, alpha, stream=None):

@@ -1018,6 +1018,19 @@ int fo_server_error(fo_server* s) {
   return h ? set_err(FO_ERR_TIMEOUT, "a tensor-core kernel timed out waiting (code " + std::to_string(h) + ")") : FO_OK;
 }
 
+int fo_column_sums(const void* x, int dtype, int64_t rows, int cols, float* out, void* stream) {
+  if (!x || !out || rows < 1 || cols < 1 || (dtype != FO_DTYPE_F32 && dtype != FO_DTYPE_BF16))
+    return set_err(FO_ERR_ARG, "bad column-sum arguments");
+  cudaStream_t st = (cudaStream_t)stream;
+  float* ws = nullptr;
+  FO_CUDA(cudaMallocAsync((void**)&ws, fo::colsum_partial_floats(rows, cols) * sizeof(float), st));
+  fo::colsum(x, nullptr, rows, cols, dtype == FO_DTYPE_F32 ? fo::kF32 : fo::kBF16, ws, out, st);
+  cudaError_t e = cudaGetLastError();
+  cudaFreeAsync(ws, st);
+  if (e != cudaSuccess) return set_err(FO_ERR_CUDA, cudaGetErrorString(e));
+  return FO_OK;
+}
+
 int fo_axpby_async(float* global, const float* local, int64_t n, float alpha, void* stream) {
   if (!global || !local || n < 0 || !(alpha > 0.f) || alpha > 1.f) return set_err(FO_ERR_ARG, "bad argument");
   fo::axpby(global, local, n, alpha, (cudaStream_t)stream);
