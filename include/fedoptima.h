@@ -250,6 +250,28 @@ FO_API int fo_axpby_async(float* global, const float* local, int64_t n, float al
  * ---------------------------------------------------------------------- */
 FO_API int fo_column_sums(const void* x, int dtype, int64_t rows, int cols, float* out, void* stream);
 
+/* ------------------------------------------------------------------------
+ * fo_column_sums without any allocation.  The paper has no counterpart: it
+ * is an interface for callers that cannot allocate device memory when they
+ * need the reduction -- code running while its stream is captured into a
+ * CUDA graph, processes whose device memory belongs to an outside allocator
+ * (a framework's caching allocator or a fixed arena), and loops that must
+ * not allocate after start-up.
+ *
+ * Same arguments, result and determinism as fo_column_sums; the partial
+ * sums go to one fixed device array of 262,144 floats (1 MiB) that the
+ * library holds on every GPU it is loaded on until the process exits.
+ * Limit: ceil(rows / 32) * cols <= 262,144 (e.g. 16,384 rows x 512 columns);
+ * larger inputs return FO_ERR_ARG with the reason in fo_last_error().
+ * The first call on a device looks up the array's device address (once per
+ * device, with that device current); make that first call before any stream
+ * capture.  All calls share the array, and it keeps the last call's
+ * contents: calls that can overlap on the GPU (different streams, no
+ * ordering between them) race on it, so order them on one stream or with
+ * events.  Nothing in the array needs to start at zero.
+ * ---------------------------------------------------------------------- */
+FO_API int fo_column_sums_noalloc(const void* x, int dtype, int64_t rows, int cols, float* out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

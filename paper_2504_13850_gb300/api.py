@@ -91,6 +91,7 @@ _SIGS = [
     ("fo_sched_queued", C.c_int, [C.c_void_p, C.c_int]),
     ("fo_axpby_async", C.c_int, [C.c_void_p, C.c_void_p, C.c_int64, C.c_float, C.c_void_p]),
     ("fo_column_sums", C.c_int, [C.c_void_p, C.c_int, C.c_int64, C.c_int, C.c_void_p, C.c_void_p]),
+    ("fo_column_sums_noalloc", C.c_int, [C.c_void_p, C.c_int, C.c_int64, C.c_int, C.c_void_p, C.c_void_p]),
 ]
 
 
@@ -347,6 +348,14 @@ def column_sums(x, out, stream=None):
     import torch
     dt = DTYPE_BF16 if x.dtype == torch.bfloat16 else DTYPE_F32
     return lib().fo_column_sums(_ptr(x), dt, x.shape[0], x.shape[1], _ptr(out), stream)
+
+
+def column_sums_noalloc(x, out, stream=None):
+    """column_sums with the partial sums in the library's fixed device array
+    (no allocation); see fo_column_sums_noalloc for the size limit."""
+    import torch
+    dt = DTYPE_BF16 if x.dtype == torch.bfloat16 else DTYPE_F32
+    return lib().fo_column_sums_noalloc(_ptr(x), dt, x.shape[0], x.shape[1], _ptr(out), stream)
 
 
 def axpby_async(global_, local, alpha, stream=None):

@@ -34,6 +34,11 @@ int set_err(int code, const std::string& msg) {
 
 }  // namespace
 
+namespace fo {
+// Records `msg` as the calling thread's fo_last_error() and returns `code`.
+int report_error(int code, const std::string& msg) { return set_err(code, msg); }
+}  // namespace fo
+
 namespace {
 
 int64_t pad64(int64_t n) { return (n + 63) / 64 * 64; }
