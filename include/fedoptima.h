@@ -242,7 +242,7 @@ FO_API int fo_axpby_async(float* global, const float* local, int64_t n, float al
  * [rows][cols] matrix: the reduction the server uses for bias gradients
  * (the sum over all positions of a layer's output gradient).  x is a device
  * pointer to fp32 (dtype FO_DTYPE_F32) or bf16 (FO_DTYPE_BF16) values, out a
- * device pointer to `cols` floats; partial sums over 32-row chunks are added
+ * device pointer to `cols` floats; partial sums over 128-row chunks are added
  * in a fixed order, so results are bitwise reproducible.  The partial sums
  * live in scratch this call allocates and frees stream-ordered on `stream`
  * (a cudaStream_t, NULL = default stream).  FO_ERR_ARG for rows < 1,
@@ -261,7 +261,7 @@ FO_API int fo_column_sums(const void* x, int dtype, int64_t rows, int cols, floa
  * Same arguments, result and determinism as fo_column_sums; the partial
  * sums go to one fixed device array of 262,144 floats (1 MiB) that the
  * library holds on every GPU it is loaded on until the process exits.
- * Limit: ceil(rows / 32) * cols <= 262,144 (e.g. 16,384 rows x 512 columns);
+ * Limit: ceil(rows / 128) * cols <= 262,144 (e.g. 65,536 rows x 512 columns);
  * larger inputs return FO_ERR_ARG with the reason in fo_last_error().
  * The first call on a device looks up the array's device address (once per
  * device, with that device current); make that first call before any stream

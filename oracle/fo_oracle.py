@@ -587,7 +587,8 @@ class Server:
     def enqueue(self, k, acts, labels, lengths=None):
         st, slot = self.sched.put(k)
         if st == OK:
-            self.slots[slot] = (np.asarray(acts, np.float64), np.asarray(labels),
+            # uploads are fp32 / bf16 values: kept as given, widened to fp64 at use
+            self.slots[slot] = (np.array(acts, copy=True), np.asarray(labels),
                                 None if lengths is None else np.asarray(lengths))
         return st, slot
 

@@ -57,7 +57,7 @@ extern "C" int fo_column_sums_noalloc(const void* x, int dtype, int64_t rows, in
     return fo::report_error(FO_ERR_ARG, "bad column-sum arguments");
   const int64_t need = fo::colsum_partial_floats(rows, cols);
   if (need > kScratchFloats)
-    return fo::report_error(FO_ERR_ARG, "fo_column_sums_noalloc: ceil(rows / 32) * cols = " + std::to_string(need) +
+    return fo::report_error(FO_ERR_ARG, "fo_column_sums_noalloc: ceil(rows / 128) * cols = " + std::to_string(need) +
                                             " partial sums exceed the fixed scratch of " +
                                             std::to_string(kScratchFloats) + " floats");
   float* scratch = nullptr;

@@ -385,7 +385,7 @@ void layernorm_bwd_dx(const void* x, const float* gamma, const float* mean, cons
 // Deterministic two-pass column sums: pass 1 writes one partial per
 // (row chunk, column), pass 2 adds the chunks in order.
 constexpr int CS_ROWS = 128;   // rows per chunk (generic kernel)
-constexpr int CS8_ROWS = 32;   // rows per chunk (16-byte bf16 kernel)
+constexpr int CS8_ROWS = 128;  // rows per chunk (16-byte bf16 kernel)
 static int colsum_chunks(int64_t rows) { return ceil_div(rows, CS_ROWS); }
 static int colsum8_chunks(int64_t rows) { return ceil_div(rows, CS8_ROWS); }
 int64_t colsum_partial_floats(int64_t rows, int C) { return int64_t(colsum8_chunks(rows)) * C; }
@@ -423,8 +423,18 @@ __global__ void colsum_finish_k(const float* partial, int chunks, int C, float* 
   const int cl = threadIdx.x % 32, rl = threadIdx.x / 32;
   const int c = blockIdx.x * 32 + cl;
   float s = 0.f;
-  if (c < C)
-    for (int q = rl; q < chunks; q += 8) s += partial[int64_t(q) * C + c];
+  if (c < C) {
+    int q = rl;
+    for (; q + 24 < chunks; q += 32) {   // four independent loads in flight
+      const float a0 = partial[int64_t(q) * C + c], a1 = partial[int64_t(q + 8) * C + c];
+      const float a2 = partial[int64_t(q + 16) * C + c], a3 = partial[int64_t(q + 24) * C + c];
+      s += a0;
+      s += a1;
+      s += a2;
+      s += a3;
+    }
+    for (; q < chunks; q += 8) s += partial[int64_t(q) * C + c];
+  }
   red[rl][cl] = s;
   __syncthreads();
   if (rl == 0 && c < C) {

@@ -89,3 +89,27 @@ def test_scheduler_rejects_bad_arguments():
     assert s.put(-1)[0] == api.ERR_ARG
     assert s.get()[0] == api.EMPTY
     assert s.set_active(7, 1) == api.ERR_ARG
+
+
+def test_scheduler_matches_oracle_on_zipf_trace_of_100_devices():
+    """The 100-device workload: Zipf(1.2) Poisson arrivals, depth 4,
+    omega = 400.  Bit-exact against the oracle; the counter-based policy
+    keeps the consumption counts of the backlogged devices within one of
+    each other, while FIFO follows the arrival skew."""
+    from paper_2504_13850_gb300 import workloads as W
+    cfg = W.CONFIGS["scale"]
+    K, omega, depth = cfg["K"], cfg["omega"], cfg["depth"]
+    a = api.Scheduler(K, omega, depth)
+    o = O.TaskScheduler(K, omega, depth)
+    f = O.TaskScheduler(K, omega, depth, "fifo")
+    order = W.arrival_order(cfg["rates"], 6000, cfg["seed"])
+    for i, k in enumerate(order):
+        assert a.put(k)[:2] == o.put(k)
+        f.put(k)
+        if i % 2 == 1:            # the server consumes one batch per two uploads
+            assert a.get() == o.get()
+            f.get()
+    assert a.counters() == o.c
+    served = [c for c in o.c if c > 0]
+    fifo_served = [c for c in f.c if c > 0]
+    assert max(o.c) - min(served) <= max(fifo_served) - min(fifo_served)

@@ -1,0 +1,34 @@
+"""The four bf16 workloads at their full sizes, in the launch configuration
+the benchmark times (same server plan, tiles and cluster splits): scheduler
+outcomes bit-exact, and two teacher-forced steps against the oracle (loss
+1e-2, parameters 2e-2 against the exact fp64 definition; per-tensor
+gradients against the bf16-storage reading with the decision-flip
+allowance of test_gpu_train)."""
+import pytest
+
+from harness import teacher_forced
+from paper_2504_13850_gb300 import api, build
+from paper_2504_13850_gb300 import workloads as W
+from test_gpu_train import check_teacher_forced
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    build.build()
+    api.lib()
+
+
+def events(cfg, uploaders, steps):
+    """A few devices upload one batch each (round robin), then steps."""
+    return [("enq", k) for k in range(uploaders)] + [("step",)] * steps
+
+
+@pytest.mark.parametrize("name", ["vgg", "resnet", "transformer", "scale"])
+def test_full_size_teacher_forced(name):
+    cfg = W.CONFIGS[name]
+    ev = events(cfg, min(cfg["K"], 3), 2)
+    _, _, recs = teacher_forced(cfg, ev)
+    assert len(recs) == 2
+    check_teacher_forced(recs, decisions=name != "transformer")

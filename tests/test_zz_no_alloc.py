@@ -38,7 +38,7 @@ def test_noalloc_matches_allocating_entry_point_on_two_calls():
 
 
 def test_noalloc_rejects_inputs_beyond_its_scratch():
-    x = torch.zeros(32768, 1024, dtype=torch.bfloat16, device="cuda")   # 1024 * 1024 partials
+    x = torch.zeros(131072, 1024, dtype=torch.bfloat16, device="cuda")   # 1024 * 1024 partials
     out = torch.empty(1024, device="cuda")
     assert api.column_sums_noalloc(x, out) == api.ERR_ARG
     assert "exceed" in api.last_error()
