@@ -31,4 +31,6 @@ def test_full_size_teacher_forced(name):
     ev = events(cfg, min(cfg["K"], 3), 2)
     _, _, recs = teacher_forced(cfg, ev)
     assert len(recs) == 2
-    check_teacher_forced(recs, decisions=name != "transformer")
+    # the transformer's backward chain crosses ~40 stored bf16 tensors (four
+    # blocks of about ten), four times the small configurations' chains
+    check_teacher_forced(recs, decisions=name != "transformer", free_tol=2e-2)

@@ -91,7 +91,7 @@ def test_tiny_config_fp32_full_trace():
 
 
 def check_teacher_forced(recs, loss_tol=1e-2, param_tol=2e-2, kernel_loss_tol=2e-3, clean_tol=3e-2,
-                         flip_tol=8e-2, decisions=True):
+                         flip_tol=8e-2, decisions=True, free_tol=1e-2):
     """Gates of each step.
 
     Against the exact oracle (the stated tolerances): loss within 1e-2
@@ -102,8 +102,10 @@ def check_teacher_forced(recs, loss_tol=1e-2, param_tol=2e-2, kernel_loss_tol=2e
     gradient of every parameter tensor normwise.  Without decisions (conv /
     linear / layernorm / attention / GELU chains) what is left is fp32
     accumulation order (~1e-6) and one-ulp bf16 rounding differences of rare
-    elements, a few 1e-3 over a backward chain: every tensor within 1e-2 on
-    every step.  With decisions, a stored value that lands one bf16 ulp
+    elements, a few 1e-3 over a backward chain of ~10 stored tensors: every
+    tensor within free_tol = 1e-2 on every step (the noise grows like the
+    square root of the chain length, so a chain four times longer gets
+    2e-2).  With decisions, a stored value that lands one bf16 ulp
     apart can still decide a ReLU at 0 or a max-pool tie (ties are common in
     bf16) the other way; each such flip re-routes one gradient element and
     moves the weight gradient of its layer, and everything upstream, by
@@ -119,7 +121,7 @@ def check_teacher_forced(recs, loss_tol=1e-2, param_tol=2e-2, kernel_loss_tol=2e
         assert abs(r["loss"] - st["loss"]) <= kernel_loss_tol * abs(st["loss"]), r
         worst = max(st["tensor_grad_err"].values())
         if not decisions:
-            assert worst <= 1e-2, (r["step"], st["tensor_grad_err"])
+            assert worst <= free_tol, (r["step"], st["tensor_grad_err"])
         assert worst <= flip_tol, (r["step"], st["tensor_grad_err"])
         clean += worst <= clean_tol
     assert 2 * clean >= len(recs), [max(r["stored"]["tensor_grad_err"].values()) for r in recs]
