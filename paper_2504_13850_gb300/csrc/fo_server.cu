@@ -409,9 +409,16 @@ int build_plan(fo_server* s) {
         }
         if (need_dx) {
           int accf = contrib(a);
-          fo::TcGemm* tg = fo::tc_plan_dgrad(s->tc, s, i, accf, s->T[a].grad, mask);
-          if (tg) {
-            add_tc(tg);
+          std::vector<fo::TcGemm*> tgs;
+          bool zero_first = false;
+          if (fo::tc_plan_dgrad(s->tc, s, i, accf, s->T[a].grad, mask, &tgs, &zero_first)) {
+            if (zero_first) {
+              const int ta = a;
+              add("memset_dx", 1, 0.0, tbytes(ta), [=](cudaStream_t st) {
+                cudaMemsetAsync(s->T[ta].grad, 0, s->T[ta].bytes(), st);
+              });
+            }
+            for (fo::TcGemm* tg : tgs) add_tc(tg);
           } else {
             const bool wbf = dto == fo::kBF16;
             add(op.kind == FO_OP_CONV ? "conv_dgrad_simt" : "linear_dgrad_simt", 1, fl, 0.0, [=](cudaStream_t st) {

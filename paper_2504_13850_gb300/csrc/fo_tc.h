@@ -5,6 +5,8 @@
 #pragma once
 #include <cuda_runtime.h>
 
+#include <vector>
+
 struct fo_server;
 
 namespace fo {
@@ -20,8 +22,13 @@ void tc_set_input(TcContext* c, int slot);
 // applying a ReLU when `relu`.
 TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int op, void* out, bool relu);
 // Input gradient of op `op` into `dx` (accumulating when `accumulate`),
-// multiplied by (mask > 0) when `mask` (same layout as dx) is given.
-TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int op, int accumulate, void* dx, const void* mask);
+// multiplied by (mask > 0) when `mask` (same layout as dx) is given.  A
+// strided convolution gives one GEMM per output-parity class; when some
+// class has no taps and this is the first contribution, *zero_first asks
+// the caller to clear dx before the GEMMs (which then accumulate).
+// Returns false when the tensor cores do not take the shape.
+bool tc_plan_dgrad(TcContext* c, fo_server* s, int op, int accumulate, void* dx, const void* mask,
+                   std::vector<TcGemm*>* out, bool* zero_first);
 TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int op);
 // Launches the GEMM kernel; a split-K plan runs as clusters of tc_splits(g)
 // CTAs that reduce their partial tiles through distributed shared memory.

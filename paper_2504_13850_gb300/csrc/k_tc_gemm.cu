@@ -43,9 +43,18 @@ struct TcParams {
   int M, N, KB, kper;
   // window geometry (spatial size of the windowed tensor and its taps)
   int H, W, ksz, pad, taps;
+  int stride;           // CONV_FPROP / CONV_WGRAD: stride of the windowed input
   int cblocks;          // 64-channel blocks per tap (contraction channels)
   int ntap_ch;          // CONV_WGRAD / CONV_DGRAD: channels per tap in the N index (Ci)
   int win_rows, win_imgs;  // rows/images covered by one window box
+  // CONV_DGRAD: the taps of this output-parity class, as (tap index r*k+s,
+  // row shift, column shift) of the gradient window
+  int ntap;
+  int tap_rs[9], tap_dh[9], tap_dw[9];
+  // output rows: GEMM row m = (n, i, j) over an Hq x Wq grid is written to
+  // row (n*oH + ostride*i + py)*oW + ostride*j + px of `out` (identity when
+  // ostride == 0)
+  int ostride, py, px, Hq, Wq, oH, oW;
   // epilogue
   void* out;
   int ldo;
@@ -162,9 +171,17 @@ __device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr) {
   return v;
 }
 
+__device__ __forceinline__ size_t out_row(const TcParams& p, int m) {
+  if (!p.ostride) return size_t(m);
+  const int hw = p.Hq * p.Wq;
+  const int n = m / hw, rem = m % hw, i = rem / p.Wq, j = rem % p.Wq;
+  return (size_t(n) * p.oH + p.ostride * i + p.py) * p.oW + p.ostride * j + p.px;
+}
+
 // Epilogue of 4 consecutive outputs (m, n..n+3): bias, ReLU, ReLU mask,
 // accumulate, store as fp32 or bf16.
-__device__ __forceinline__ void store4(const TcParams& p, int m, int n, float4 a) {
+__device__ __forceinline__ void store4(const TcParams& p, int m_gemm, int n, float4 a) {
+  const size_t m = out_row(p, m_gemm);
   float v[4] = {a.x, a.y, a.z, a.w};
   if (p.bias)
 #pragma unroll
@@ -252,13 +269,15 @@ __device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, i
   } else if (KIND == LIN_WGRAD || KIND == CONV_WGRAD) {
 #pragma unroll
     for (int j = 0; j < BM / 64; ++j) tma_2d(sa + j * BK * 128, &p.tmA, bar, m0 + j * 64, kb * BK);
-  } else {  // CONV_FPROP / CONV_DGRAD: windowed A
+  } else if (KIND == CONV_FPROP) {  // windowed A over the (strided) input
     const int tap = kb / p.cblocks, c0 = (kb % p.cblocks) * 64;
     const int r = tap / p.ksz, s = tap % p.ksz;
-    const int n_img = m0 / HW, h0 = (m0 % HW) / p.W;
-    const int dh = (KIND == CONV_FPROP) ? r - p.pad : p.pad - r;
-    const int dw = (KIND == CONV_FPROP) ? s - p.pad : p.pad - s;
-    tma_4d(sa, &p.tmA, bar, c0, dw, h0 + dh, n_img);
+    const int n_img = m0 / HW, h0 = (m0 % HW) / p.W;   // H, W: output grid
+    tma_4d(sa, &p.tmA, bar, c0, s - p.pad, h0 * p.stride + r - p.pad, n_img);
+  } else {  // CONV_DGRAD: window over the output gradient, shifted per tap
+    const int t = kb / p.cblocks, c0 = (kb % p.cblocks) * 64;
+    const int n_img = m0 / HW, h0 = (m0 % HW) / p.W;   // H, W: the class grid (= gradient grid)
+    tma_4d(sa, &p.tmA, bar, c0, p.tap_dw[t], h0 + p.tap_dh[t], n_img);
   }
   if (KIND == LIN_FWD) {
     tma_2d(sb, &p.tmB, bar, kb * BK, n0);
@@ -269,17 +288,18 @@ __device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, i
 #pragma unroll
     for (int j = 0; j < BN / 64; ++j) tma_2d(sb + j * BK * 128, &p.tmB, bar, n0 + j * 64, kb * BK);
   } else if (KIND == CONV_DGRAD) {
-    const int tap = kb / p.cblocks, co0 = (kb % p.cblocks) * 64;
+    const int t = kb / p.cblocks, co0 = (kb % p.cblocks) * 64;
+    const int tap = p.tap_rs[t];
 #pragma unroll
     for (int j = 0; j < BN / 64; ++j) tma_2d(sb + j * BK * 128, &p.tmB, bar, tap * p.ntap_ch + n0 + j * 64, co0);
   } else {  // CONV_WGRAD: N index = tap * Ci + ci; K = output pixel
     const int tap = n0 / p.ntap_ch, ci0 = n0 % p.ntap_ch;
     const int r = tap / p.ksz, s = tap % p.ksz;
     const int pix0 = kb * BK;
-    const int n_img = pix0 / HW, h0 = (pix0 % HW) / p.W;
+    const int n_img = pix0 / HW, h0 = (pix0 % HW) / p.W;   // H, W: output grid
 #pragma unroll
     for (int j = 0; j < BN / 64; ++j)
-      tma_4d(sb + j * BK * 128, &p.tmB, bar, ci0 + j * 64, s - p.pad, h0 + r - p.pad, n_img);
+      tma_4d(sb + j * BK * 128, &p.tmB, bar, ci0 + j * 64, s - p.pad, h0 * p.stride + r - p.pad, n_img);
   }
 }
 
@@ -403,6 +423,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 #pragma unroll
       for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
       const int n = n0 + c;
+      const size_t mo = out_row(p, m);
       if (p.bias) {
 #pragma unroll
         for (int j = 0; j < 16; ++j) v[j] += p.bias[n + j];
@@ -412,7 +433,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         for (int j = 0; j < 16; ++j) v[j] = fmaxf(v[j], 0.f);
       }
       if (p.mask) {
-        const uint4* mk = reinterpret_cast<const uint4*>(p.mask + size_t(m) * p.ldo + n);
+        const uint4* mk = reinterpret_cast<const uint4*>(p.mask + mo * p.ldo + n);
 #pragma unroll
         for (int j = 0; j < 2; ++j) {
           uint4 u = mk[j];
@@ -423,7 +444,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         }
       }
       if (p.out_f32) {
-        float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + size_t(m) * p.ldo + n);
+        float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + mo * p.ldo + n);
         if (p.acc) {
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
@@ -434,7 +455,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 #pragma unroll
         for (int j = 0; j < 4; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
       } else {
-        uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(p.out) + size_t(m) * p.ldo + n);
+        uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(p.out) + mo * p.ldo + n);
         if (p.acc) {
 #pragma unroll
           for (int j = 0; j < 2; ++j) {
@@ -537,8 +558,10 @@ EncodeTiledFn encode_fn() {
 }
 
 // bf16 tensor map, dims innermost first, strides in bytes of dims 1.. .
+// elem (may be null): traversal step per dimension (the box then spans
+// box[i] elements and loads box[i] / elem[i] of them).
 bool make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, const uint64_t* strides,
-              const uint32_t* box) {
+              const uint32_t* box, const uint32_t* elem = nullptr) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t d[5], st[4];
@@ -546,7 +569,7 @@ bool make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, 
   for (int i = 0; i < rank; ++i) {
     d[i] = dims[i];
     b[i] = box[i];
-    es[i] = 1;
+    es[i] = elem ? elem[i] : 1;
     if (i + 1 < rank) st[i] = strides[i];
   }
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), d, st, b, es,
@@ -563,18 +586,23 @@ bool map_2d(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int bo
   return make_map(m, base, 2, dims, strides, box);
 }
 
-// 4-D NHWC window map: box (64 channels, W, rows, imgs).
-bool map_window(CUtensorMap* m, const void* base, int N, int H, int W, int C, int rows, int imgs) {
+// 4-D NHWC window map over an N x H x W x C tensor that loads, per box,
+// 64 channels x ow columns x rows x imgs, stepping `stride` pixels in H and W
+// (the box spans ow*stride columns and rows*stride rows of the tensor).
+bool map_window(CUtensorMap* m, const void* base, int N, int H, int W, int C, int ow, int rows, int imgs,
+                int stride = 1) {
   uint64_t dims[4] = {uint64_t(C), uint64_t(W), uint64_t(H), uint64_t(N)};
   uint64_t strides[3] = {uint64_t(C) * 2, uint64_t(W) * C * 2, uint64_t(H) * W * C * 2};
-  uint32_t box[4] = {64, uint32_t(W), uint32_t(rows), uint32_t(imgs)};
-  return make_map(m, base, 4, dims, strides, box);
+  uint32_t box[4] = {64, uint32_t(ow * stride), uint32_t(rows * stride), uint32_t(imgs)};
+  uint32_t elem[4] = {1, uint32_t(stride), uint32_t(stride), 1};
+  return make_map(m, base, 4, dims, strides, box, elem);
 }
 
 }  // namespace
 
 // ------------------------------------------------------------------ plans
 struct TcGemm {
+  TcGemm() { p.stride = 1; }
   const char* name;
   int kind, bn, splits;
   double flops = 0;
@@ -746,63 +774,122 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i, void* out, bool relu)
     if (!map_2d(&g->p.tmB, w, op.cout, op.cin, bn)) { delete g; return nullptr; }
     return finish(c, g, M, op.cout, double(op.cin));
   }
-  // convolution: 3x3 (or 1x1) stride 1
-  if (op.stride != 1 || op.cin % 64 || op.cout % 64) { delete g; return nullptr; }
+  // convolution: k in {1, 3}, stride in {1, 2}; tiles of 128 output pixels
+  const int st = op.stride, Ho = o.H, Wo = o.W;
+  if (op.cin % 64 || op.cout % 64 || (st == 2 && (a.H != 2 * Ho || a.W != 2 * Wo))) { delete g; return nullptr; }
   int rows, imgs;
-  if (!window_ok(a.N, a.H, a.W, BM, &rows, &imgs) || (int64_t(a.N) * a.H * a.W) % BM) { delete g; return nullptr; }
+  if (!window_ok(a.N, Ho, Wo, BM, &rows, &imgs) || (int64_t(a.N) * Ho * Wo) % BM) { delete g; return nullptr; }
   g->kind = CONV_FPROP;
   g->name = "tc_conv_fprop";
-  g->p.H = a.H; g->p.W = a.W; g->p.ksz = op.k; g->p.pad = op.k / 2; g->p.taps = op.k * op.k;
+  g->p.H = Ho; g->p.W = Wo; g->p.ksz = op.k; g->p.pad = op.k / 2; g->p.taps = op.k * op.k; g->p.stride = st;
   g->p.cblocks = op.cin / 64;
   g->p.ntap_ch = op.cin;
   g->p.win_rows = rows; g->p.win_imgs = imgs;
-  int M = a.N * a.H * a.W, KB = g->p.taps * g->p.cblocks;
+  int M = a.N * Ho * Wo, KB = g->p.taps * g->p.cblocks;
   choose_tiles(c, g, M, op.cout, KB, op.cout);
   const int bn = g->bn;
   g->input_A = (op.in0 == 0);
   if (g->input_A) {
     g->slot_maps.resize(s->cfg.omega);
     for (int sl = 0; sl < s->cfg.omega; ++sl)
-      if (!map_window(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, a.N, a.H, a.W, a.C, rows, imgs)) { delete g; return nullptr; }
-  } else if (!map_window(&g->p.tmA, tensor_act(s, op.in0), a.N, a.H, a.W, a.C, rows, imgs)) { delete g; return nullptr; }
+      if (!map_window(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, a.N, a.H, a.W, a.C, Wo, rows, imgs, st)) { delete g; return nullptr; }
+  } else if (!map_window(&g->p.tmA, tensor_act(s, op.in0), a.N, a.H, a.W, a.C, Wo, rows, imgs, st)) { delete g; return nullptr; }
   if (!map_2d(&g->p.tmB, w, op.cout, int64_t(g->p.taps) * op.cin, bn)) { delete g; return nullptr; }
   return finish(c, g, M, op.cout, double(g->p.taps) * op.cin);
 }
 
-TcGemm* tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate, void* dx, const void* mask) {
-  if (!c || !bf16_server(s) || getenv("FO_NO_TC")) return nullptr;
+bool tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate, void* dx, const void* mask,
+                   std::vector<TcGemm*>* out, bool* zero_first) {
+  out->clear();
+  *zero_first = false;
+  if (!c || !bf16_server(s) || getenv("FO_NO_TC")) return false;
   const fo_op& op = s->ops[i];
   const Tensor& a = s->T[op.in0];
   const Tensor& o = s->T[i + 1];
-  if (o.dt != kBF16) return nullptr;
-  TcGemm* g = new TcGemm();
-  g->p.out = dx;
-  g->p.ldo = a.C;
-  g->p.acc = accumulate;
-  g->p.mask = static_cast<const bf16*>(mask);
+  if (o.dt != kBF16) return false;
   const bf16* w = s->shadow + s->segs[s->op_segs[i][0]].off;
+  auto base = [&]() {
+    TcGemm* g = new TcGemm();
+    g->p.out = dx;
+    g->p.ldo = a.C;
+    g->p.acc = accumulate;
+    g->p.mask = static_cast<const bf16*>(mask);
+    return g;
+  };
   if (op.kind == FO_OP_LINEAR) {
-    if (op.cin % 64 || op.cout % 64) { delete g; return nullptr; }
+    if (op.cin % 64 || op.cout % 64) return false;
+    TcGemm* g = base();
     g->kind = LIN_DGRAD;
     g->name = "tc_linear_dgrad";
     int M = int(a.rows()), KB = op.cout / 64;
     choose_tiles(c, g, M, op.cin, KB, op.cin);
-    if (!map_2d(&g->p.tmA, o.grad, M, op.cout, BM) || !map_2d(&g->p.tmB, w, op.cout, op.cin, BK)) { delete g; return nullptr; }
-    return finish(c, g, M, op.cin, double(op.cout));
+    if (!map_2d(&g->p.tmA, o.grad, M, op.cout, BM) || !map_2d(&g->p.tmB, w, op.cout, op.cin, BK)) { delete g; return false; }
+    if (!finish(c, g, M, op.cin, double(op.cout))) return false;
+    out->push_back(g);
+    return true;
   }
-  if (op.stride != 1 || op.cin % 64 || op.cout % 64) { delete g; return nullptr; }
+  // Convolution input gradient, split by output parity (py, px) for stride 2:
+  // input row y = st*i + py receives output row p = i + dh from tap r when
+  // st*dh = py + pad - r.  Each class is an implicit GEMM over its own taps.
+  const int st = op.stride, pad = op.k / 2, Ho = o.H, Wo = o.W;
+  if (op.cin % 64 || op.cout % 64 || (st == 2 && (a.H != 2 * Ho || a.W != 2 * Wo))) return false;
   int rows, imgs;
-  if (!window_ok(o.N, o.H, o.W, BM, &rows, &imgs) || (int64_t(a.N) * a.H * a.W) % BM) { delete g; return nullptr; }
-  g->kind = CONV_DGRAD;
-  g->name = "tc_conv_dgrad";
-  g->p.H = o.H; g->p.W = o.W; g->p.ksz = op.k; g->p.pad = op.k / 2; g->p.taps = op.k * op.k;
-  g->p.cblocks = op.cout / 64;
-  g->p.ntap_ch = op.cin;
-  int M = a.N * a.H * a.W, KB = g->p.taps * g->p.cblocks;
-  choose_tiles(c, g, M, op.cin, KB, op.cin);
-  if (!map_window(&g->p.tmA, o.grad, o.N, o.H, o.W, o.C, rows, imgs) ||
-      !map_2d(&g->p.tmB, w, op.cout, int64_t(g->p.taps) * op.cin, BK)) { delete g; return nullptr; }
-  return finish(c, g, M, op.cin, double(g->p.taps) * op.cout);
+  if (!window_ok(o.N, Ho, Wo, BM, &rows, &imgs) || (int64_t(o.N) * Ho * Wo) % BM) return false;
+  const int nclass = st * st;
+  bool any_empty = false;
+  struct Cls { int n; int rs[9], dh[9], dw[9]; } cls[4];
+  for (int q = 0; q < nclass; ++q) {
+    const int py = q / st, px = q % st;
+    cls[q].n = 0;
+    for (int r = 0; r < op.k; ++r)
+      for (int sx = 0; sx < op.k; ++sx) {
+        const int vh = py + pad - r, vw = px + pad - sx;
+        if (vh % st || vw % st) continue;
+        int& n = cls[q].n;
+        cls[q].rs[n] = r * op.k + sx;
+        cls[q].dh[n] = vh / st;
+        cls[q].dw[n] = vw / st;
+        ++n;
+      }
+    if (cls[q].n == 0) any_empty = true;
+  }
+  const int eff_acc = any_empty && !accumulate ? 1 : accumulate;
+  *zero_first = any_empty && !accumulate;
+  for (int q = 0; q < nclass; ++q) {
+    if (cls[q].n == 0) continue;
+    TcGemm* g = base();
+    g->p.acc = eff_acc;
+    g->kind = CONV_DGRAD;
+    g->name = "tc_conv_dgrad";
+    g->p.H = Ho; g->p.W = Wo; g->p.ksz = op.k; g->p.pad = pad; g->p.taps = op.k * op.k;
+    g->p.cblocks = op.cout / 64;
+    g->p.ntap_ch = op.cin;
+    g->p.ntap = cls[q].n;
+    for (int t = 0; t < cls[q].n; ++t) {
+      g->p.tap_rs[t] = cls[q].rs[t];
+      g->p.tap_dh[t] = cls[q].dh[t];
+      g->p.tap_dw[t] = cls[q].dw[t];
+    }
+    if (st == 2) {
+      g->p.ostride = 2; g->p.py = q / 2; g->p.px = q % 2;
+      g->p.Hq = Ho; g->p.Wq = Wo; g->p.oH = a.H; g->p.oW = a.W;
+    }
+    const int M = o.N * Ho * Wo, KB = cls[q].n * g->p.cblocks;
+    choose_tiles(c, g, M, op.cin, KB, op.cin);
+    if (!map_window(&g->p.tmA, o.grad, o.N, Ho, Wo, o.C, Wo, rows, imgs) ||
+        !map_2d(&g->p.tmB, w, op.cout, int64_t(g->p.taps) * op.cin, BK)) {
+      delete g;
+      for (TcGemm* x : *out) (void)x;
+      out->clear();
+      return false;
+    }
+    if (!finish(c, g, M, op.cin, double(cls[q].n) * op.cout)) {
+      out->clear();
+      return false;
+    }
+    out->push_back(g);
+  }
+  return true;
 }
 
 TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
@@ -830,15 +917,16 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
     } else if (!map_2d(&g->p.tmB, tensor_act(s, op.in0), rows, op.cin, BK)) { delete g; return nullptr; }
     return finish(c, g, op.cout, op.cin, double(rows));
   }
-  if (op.stride != 1 || op.cin % 64 || op.cout % 128) { delete g; return nullptr; }
+  const int st = op.stride, Ho = o.H, Wo = o.W;
+  if (op.cin % 64 || op.cout % 128 || (st == 2 && (a.H != 2 * Ho || a.W != 2 * Wo))) { delete g; return nullptr; }
   int rows, imgs;
-  if (!window_ok(a.N, a.H, a.W, BK, &rows, &imgs) || (int64_t(a.N) * a.H * a.W) % BK) { delete g; return nullptr; }
+  if (!window_ok(a.N, Ho, Wo, BK, &rows, &imgs) || (int64_t(a.N) * Ho * Wo) % BK) { delete g; return nullptr; }
   g->kind = CONV_WGRAD;
   g->name = "tc_conv_wgrad";
   g->p.ldo = op.k * op.k * op.cin;
-  g->p.H = a.H; g->p.W = a.W; g->p.ksz = op.k; g->p.pad = op.k / 2; g->p.taps = op.k * op.k;
+  g->p.H = Ho; g->p.W = Wo; g->p.ksz = op.k; g->p.pad = op.k / 2; g->p.taps = op.k * op.k; g->p.stride = st;
   g->p.ntap_ch = op.cin;
-  int P = a.N * a.H * a.W, KB = P / BK;
+  int P = a.N * Ho * Wo, KB = P / BK;
   int N = g->p.taps * op.cin;
   choose_tiles(c, g, op.cout, N, KB, op.cin);
   g->input_B = (op.in0 == 0);
@@ -846,8 +934,8 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
   if (g->input_B) {
     g->slot_maps.resize(s->cfg.omega);
     for (int sl = 0; sl < s->cfg.omega; ++sl)
-      if (!map_window(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, a.N, a.H, a.W, a.C, rows, imgs)) { delete g; return nullptr; }
-  } else if (!map_window(&g->p.tmB, tensor_act(s, op.in0), a.N, a.H, a.W, a.C, rows, imgs)) { delete g; return nullptr; }
+      if (!map_window(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, a.N, a.H, a.W, a.C, Wo, rows, imgs, st)) { delete g; return nullptr; }
+  } else if (!map_window(&g->p.tmB, tensor_act(s, op.in0), a.N, a.H, a.W, a.C, Wo, rows, imgs, st)) { delete g; return nullptr; }
   return finish(c, g, op.cout, N, double(P));
 }
 

@@ -159,10 +159,31 @@ def decision_free(kind):
         b.add("linear", t, cin=256, cout=10, bias=1)
         return W.shrink(W.CONFIGS["vgg"], ops=b.ops, batch=20, in_hwc=(8, 8, 128), K=3, omega=6, depth=2,
                         lr=1e-3)
+    if kind == "strided":
+        t = b.add("conv", 0, cin=64, cout=128, k=3, stride=2, bias=1)      # 16x16 -> 8x8
+        t = b.add("conv", t, cin=128, cout=128, k=1, stride=1, bias=1)
+        t = b.add("conv", t, cin=128, cout=256, k=3, stride=2, bias=1)     # 8x8 -> 4x4
+        t = b.add("flatten", t)
+        t = b.add("linear", t, cin=4 * 4 * 256, cout=128, bias=1)
+        b.add("linear", t, cin=128, cout=10, bias=1)
+        return W.shrink(W.CONFIGS["resnet"], ops=b.ops, batch=16, in_hwc=(16, 16, 64), K=3, omega=6, depth=2,
+                        lr=1e-3, classes=10)
+    if kind == "resblock":
+        t1 = b.add("conv", 0, cin=64, cout=64, k=3, stride=1, bias=0)
+        t2 = b.add("conv", t1, cin=64, cout=128, k=3, stride=2, bias=0)
+        t3 = b.add("affine", t2, c=128)
+        t4 = b.add("conv", t1, cin=64, cout=128, k=1, stride=2, bias=0)    # first into t1's gradient
+        t5 = b.add("add", t3, in1=t4)
+        t6 = b.add("conv", t5, cin=128, cout=128, k=3, stride=1, bias=0)
+        t = b.add("flatten", t6)
+        t = b.add("linear", t, cin=8 * 8 * 128, cout=64, bias=1)
+        b.add("linear", t, cin=64, cout=10, bias=1)
+        return W.shrink(W.CONFIGS["resnet"], ops=b.ops, batch=8, in_hwc=(16, 16, 64), K=3, omega=6, depth=2,
+                        lr=1e-3, classes=10)
     raise ValueError(kind)
 
 
-@pytest.mark.parametrize("kind", ["conv16", "conv8"])
+@pytest.mark.parametrize("kind", ["conv16", "conv8", "strided", "resblock"])
 def test_decision_free_teacher_forced(kind):
     cfg = decision_free(kind)
     _, _, recs = teacher_forced(cfg, prefill_then_steps(cfg, 4))
