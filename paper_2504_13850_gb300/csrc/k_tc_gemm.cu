@@ -602,18 +602,20 @@ bool map_window(CUtensorMap* m, const void* base, int N, int H, int W, int C, in
 
 // ------------------------------------------------------------------ plans
 struct TcGemm {
-  TcGemm() { p.stride = 1; }
-  const char* name;
-  int kind, bn, splits;
+  // Every field starts at zero / null (the kernel parameters included);
+  // only the window stride defaults to 1.
+  TcGemm() : p{} { p.stride = 1; }
+  const char* name = nullptr;
+  int kind = 0, bn = 0, splits = 1;
   double flops = 0;
   TcParams p;
-  KernelFn fn;
-  size_t smem;
+  KernelFn fn = nullptr;
+  size_t smem = 0;
   dim3 grid;
-  bool input_A;           // operand fed by the uploaded batch (tensor 0)
-  bool input_B;
+  bool input_A = false;   // operand fed by the uploaded batch (tensor 0)
+  bool input_B = false;
   std::vector<CUtensorMap> slot_maps;  // per slot map of that operand
-  TcContext* ctx;
+  TcContext* ctx = nullptr;
 };
 
 struct TcContext {
