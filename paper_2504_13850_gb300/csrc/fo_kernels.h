@@ -95,6 +95,29 @@ void sgd_momentum(float* theta, float* v, const float* g, void* shadow, int64_t 
                   float mu, int64_t* step, cudaStream_t st);
 void f32_to_bf16(const float* x, void* y, int64_t n, cudaStream_t st);
 
+// ---- vectorised bf16 kernels (k_vec.cu): 8 elements per 16-byte access ----
+bool vec8_ok(int dt, int64_t n);
+void relu_bwd_x8(const void* y, const void* dy, void* dx, int64_t n, bool acc, cudaStream_t st);
+void add_x8(const void* a, const void* b, void* y, int64_t n, bool relu, cudaStream_t st);
+void copy_acc_x8(const void* x, void* y, int64_t n, bool acc, cudaStream_t st);
+void affine_fwd_x8(const void* x, const float* sc, const float* sh, void* y, int64_t n, int C, bool relu,
+                   cudaStream_t st);
+void gelu_fwd_x8(const void* x, void* y, int64_t n, cudaStream_t st);
+void gelu_bwd_x8(const void* x, const void* dy, void* dx, int64_t n, bool acc, cudaStream_t st);
+// Column sums (C % 8 == 0) with a (column block, row chunk) grid.
+int64_t colsum8_partial_floats(int64_t rows, int C);
+void colsum8(const void* a, int64_t rows, int C, float* partial, float* out, cudaStream_t st);
+// Affine backward in one pass: dscale = sum dy*x, dshift = sum dy, dx (+)= dy*scale
+// (dx may be null); partial holds 2 * colsum8_partial_floats floats.
+void affine_bwd8(const void* dy, const void* x, const float* scale, void* dx, bool acc, int64_t rows, int C,
+                 float* partial, float* dscale, float* dshift, cudaStream_t st);
+// Layernorm backward fused with dgamma / dbeta (C % 256 == 0, C <= 512).
+bool layernorm_bwd8_ok(int dt, int C);
+int64_t layernorm_bwd8_partial_floats(int64_t rows, int C);
+void layernorm_bwd8(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
+                    void* dx, int64_t rows, int C, bool acc, float* partial, float* dgamma, float* dbeta,
+                    cudaStream_t st);
+
 // FedAsync update: g = fmaf(alpha, l - g, g).
 void axpby(float* g, const float* l, int64_t n, float alpha, cudaStream_t st);
 // Number of kernels axpby launches for these arguments (vector body, tail).

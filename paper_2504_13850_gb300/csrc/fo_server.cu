@@ -439,6 +439,16 @@ int build_plan(fo_server* s) {
         break;
       }
       case FO_OP_AFFINE:
+        if (fo::vec8_ok(dt, s->T[a0].numel()) && s->T[a0].C % 8 == 0) {
+          // one pass: dscale, dshift and dx (+)= dy * scale
+          const int accf = need_dx ? contrib(a) : 0;
+          add("affine_bwd", 4, 0.0, (need_dx ? 3 + accf : 2) * csb, [=](cudaStream_t st) {
+            const Tensor& x = s->T[a0];
+            fo::affine_bwd8(s->T[o].grad, act(a0), P(s, i, 0), need_dx ? s->T[a].grad : nullptr, accf != 0,
+                            x.rows(), x.C, s->colsum_scratch, G(s, i, 0), G(s, i, 1), st);
+          });
+          break;
+        }
         add("affine_pgrad", 4, 0.0, 3 * csb, [=](cudaStream_t st) {
           const Tensor& x = s->T[a0];
           fo::colsum(s->T[o].grad, act(a0), x.rows(), x.C, dt, s->colsum_scratch, G(s, i, 0), st);
@@ -497,6 +507,16 @@ int build_plan(fo_server* s) {
       case FO_OP_FLATTEN:
         break;  // shares the input's gradient buffer
       case FO_OP_LAYERNORM:
+        if (fo::layernorm_bwd8_ok(dt, s->T[a0].C)) {
+          const int accf = need_dx ? contrib(a) : 0;
+          add("layernorm_bwd", 3, 0.0, (need_dx ? 3 + accf : 2) * csb, [=](cudaStream_t st) {
+            const Tensor& x = s->T[a0];
+            fo::layernorm_bwd8(act(a0), P(s, i, 0), s->ln_mean[i], s->ln_rstd[i], s->T[o].grad,
+                               need_dx ? s->T[a].grad : nullptr, x.rows(), x.C, accf != 0, s->colsum_scratch,
+                               G(s, i, 0), G(s, i, 1), st);
+          });
+          break;
+        }
         add("layernorm_pgrad", 4, 0.0, 3 * csb, [=](cudaStream_t st) {
           const Tensor& x = s->T[a0];
           fo::colsum_lnx(s->T[o].grad, act(a0), s->ln_mean[i], s->ln_rstd[i], x.rows(), x.C, dt, s->colsum_scratch,
@@ -605,8 +625,9 @@ int allocate(fo_server* s) {
   for (int i = 0; i < nops; ++i) {
     const Tensor& o = s->T[i + 1];
     const Tensor& a = s->T[s->ops[i].in0];
-    cs_floats = std::max(cs_floats, fo::colsum_partial_floats(o.rows(), o.C));
-    cs_floats = std::max(cs_floats, fo::colsum_partial_floats(a.rows(), a.C));
+    // two partial arrays (affine / layernorm backward), 64- or 128-row chunks
+    cs_floats = std::max(cs_floats, 4 * fo::colsum_partial_floats(o.rows(), o.C));
+    cs_floats = std::max(cs_floats, 4 * fo::colsum_partial_floats(a.rows(), a.C));
   }
   s->colsum_scratch = (float*)s->alloc(cs_floats * 4);
   s->ln_mean.assign(nops, nullptr);

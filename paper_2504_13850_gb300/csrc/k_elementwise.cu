@@ -57,6 +57,7 @@ void relu_fwd(const void* x, void* y, int64_t n, int dt, cudaStream_t st) {
   FO_DISPATCH(dt, T, relu_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (T*)y, n));
 }
 void relu_bwd(const void* x, const void* dy, void* dx, int64_t n, int dt, bool acc, cudaStream_t st) {
+  if (vec8_ok(dt, n)) return relu_bwd_x8(x, dy, dx, n, acc, st);
   FO_DISPATCH(dt, T, relu_bwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (const T*)dy, (T*)dx, n, acc));
 }
 
@@ -247,6 +248,7 @@ __global__ void copy_acc_k(const T* x, T* y, int64_t n, int acc) {
 void affine_fwd(const void* x, const float* scale, const float* shift, void* y, int64_t rows,
                 int C, int dt, bool relu, cudaStream_t st) {
   int64_t n = rows * C;
+  if (vec8_ok(dt, n) && C % 8 == 0) return affine_fwd_x8(x, scale, shift, y, n, C, relu, st);
   FO_DISPATCH(dt, T, affine_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, scale, shift, (T*)y, n, C, relu));
 }
 void affine_dx(const void* dy, const float* scale, void* dx, int64_t rows, int C, int dt,
@@ -255,9 +257,11 @@ void affine_dx(const void* dy, const float* scale, void* dx, int64_t rows, int C
   FO_DISPATCH(dt, T, affine_dx_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)dy, scale, (T*)dx, n, C, acc));
 }
 void add_fwd(const void* a, const void* b, void* y, int64_t n, int dt, bool relu, cudaStream_t st) {
+  if (vec8_ok(dt, n)) return add_x8(a, b, y, n, relu, st);
   FO_DISPATCH(dt, T, add_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)a, (const T*)b, (T*)y, n, relu));
 }
 void copy_or_acc(const void* x, void* y, int64_t n, int dt, bool acc, cudaStream_t st) {
+  if (vec8_ok(dt, n)) return copy_acc_x8(x, y, n, acc, st);
   FO_DISPATCH(dt, T, copy_acc_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (T*)y, n, acc));
 }
 
@@ -305,9 +309,11 @@ __global__ void gelu_bwd_k(const T* x, const T* dy, T* dx, int64_t n, int acc) {
   }
 }
 void gelu_fwd(const void* x, void* y, int64_t n, int dt, cudaStream_t st) {
+  if (vec8_ok(dt, n)) return gelu_fwd_x8(x, y, n, st);
   FO_DISPATCH(dt, T, gelu_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (T*)y, n));
 }
 void gelu_bwd(const void* x, const void* dy, void* dx, int64_t n, int dt, bool acc, cudaStream_t st) {
+  if (vec8_ok(dt, n)) return gelu_bwd_x8(x, dy, dx, n, acc, st);
   FO_DISPATCH(dt, T, gelu_bwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (const T*)dy, (T*)dx, n, acc));
 }
 
@@ -385,10 +391,8 @@ void layernorm_bwd_dx(const void* x, const float* gamma, const float* mean, cons
 // Deterministic two-pass column sums: pass 1 writes one partial per
 // (row chunk, column), pass 2 adds the chunks in order.
 constexpr int CS_ROWS = 128;   // rows per chunk (generic kernel)
-constexpr int CS8_ROWS = 128;  // rows per chunk (16-byte bf16 kernel)
 static int colsum_chunks(int64_t rows) { return ceil_div(rows, CS_ROWS); }
-static int colsum8_chunks(int64_t rows) { return ceil_div(rows, CS8_ROWS); }
-int64_t colsum_partial_floats(int64_t rows, int C) { return int64_t(colsum8_chunks(rows)) * C; }
+int64_t colsum_partial_floats(int64_t rows, int C) { return int64_t(colsum_chunks(rows)) * C; }
 
 // MODE 0: a;  1: a * b;  2: a * (b - mean[r]) * rstd[r]
 template <int MODE, typename T>
@@ -445,57 +449,9 @@ __global__ void colsum_finish_k(const float* partial, int chunks, int C, float* 
   }
 }
 
-// bf16 column sums with 16-byte loads: thread (g, r) adds columns
-// 8g..8g+7 over rows r, r + rl, ... of its 32-row chunk (loads issued
-// before the adds); the rl row lanes of a block are combined in shared
-// memory in a fixed order.
-__global__ void colsum_bf16x8_k(const bf16* __restrict__ a, int64_t rows, int C, float* __restrict__ partial) {
-  extern __shared__ float red[];  // [rl][C]
-  const int groups = C / 8;
-  const int g = threadIdx.x % groups, r = threadIdx.x / groups, rl = blockDim.x / groups;
-  const int64_t r0 = int64_t(blockIdx.x) * CS8_ROWS;
-  float s[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-  if (r < rl) {
-    constexpr int kMax = CS8_ROWS;  // rl >= 1
-    uint4 u[8];
-    int n = 0;
-    for (int64_t row = r0 + r; row < r0 + CS8_ROWS && row < rows && n < kMax; row += rl) {
-      if (n == 8) {
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          const bf16* e = reinterpret_cast<const bf16*>(&u[q]);
-#pragma unroll
-          for (int j = 0; j < 8; ++j) s[j] += __bfloat162float(e[j]);
-        }
-        n = 0;
-      }
-      u[n++] = *reinterpret_cast<const uint4*>(a + row * C + 8 * g);
-    }
-    for (int q = 0; q < n; ++q) {
-      const bf16* e = reinterpret_cast<const bf16*>(&u[q]);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) s[j] += __bfloat162float(e[j]);
-    }
-#pragma unroll
-    for (int j = 0; j < 8; ++j) red[r * C + 8 * g + j] = s[j];
-  }
-  __syncthreads();
-  for (int c = threadIdx.x; c < C; c += blockDim.x) {
-    float t = 0.f;
-    for (int q = 0; q < rl; ++q) t += red[q * C + c];
-    partial[int64_t(blockIdx.x) * C + c] = t;
-  }
-}
-
 void colsum(const void* a, const void* b, int64_t rows, int C, int dt, float* partial, float* out,
             cudaStream_t st) {
-  if (!b && dt == kBF16 && C % 8 == 0 && C / 8 <= 256) {
-    const int groups = C / 8;
-    const int rl = 256 / groups;
-    colsum_bf16x8_k<<<colsum8_chunks(rows), groups * rl, sizeof(float) * rl * C, st>>>((const bf16*)a, rows, C, partial);
-    colsum_finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, colsum8_chunks(rows), C, out);
-    return;
-  }
+  if (!b && dt == kBF16 && C % 8 == 0) return colsum8(a, rows, C, partial, out, st);
   dim3 grid(ceil_div(C, 32), colsum_chunks(rows));
   if (b) {
     FO_DISPATCH(dt, T, colsum_partial_k<1, T><<<grid, 256, 0, st>>>((const T*)a, (const T*)b, nullptr, nullptr, rows, C, partial));

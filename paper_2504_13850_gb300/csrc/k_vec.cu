@@ -1,0 +1,368 @@
+// Vectorised bf16 elementwise and reduction kernels: 8 elements (16 bytes)
+// per thread and per access.  Used when the tensor is bf16 and its element
+// count (and, where channels matter, its channel count) is a multiple of 8;
+// the scalar kernels of k_elementwise.cu cover the rest.  Column sums are
+// taken per (row chunk, 256-column block) and finished in a fixed order, so
+// every result is deterministic.
+#include "fo_common.cuh"
+#include "fo_kernels.h"
+
+namespace fo {
+
+namespace {
+
+constexpr int kChunk = 128;  // rows per column-sum chunk (as the scalar kernels)
+
+struct V8 {
+  float v[8];
+};
+
+__device__ __forceinline__ V8 ld8(const bf16* p) {
+  const uint4 u = *reinterpret_cast<const uint4*>(p);
+  const bf16* e = reinterpret_cast<const bf16*>(&u);
+  V8 r;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) r.v[j] = __bfloat162float(e[j]);
+  return r;
+}
+__device__ __forceinline__ void st8(bf16* p, const V8& r) {
+  uint4 u;
+  bf16* e = reinterpret_cast<bf16*>(&u);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) e[j] = __float2bfloat16_rn(r.v[j]);
+  *reinterpret_cast<uint4*>(p) = u;
+}
+
+#define GRID_STRIDE8(i, n8) \
+  for (int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; i < (n8); i += int64_t(gridDim.x) * blockDim.x)
+
+__global__ void relu_bwd_x8_k(const bf16* __restrict__ y, const bf16* __restrict__ dy, bf16* __restrict__ dx,
+                              int64_t n8, int acc) {
+  GRID_STRIDE8(i, n8) {
+    const V8 m = ld8(y + 8 * i), g = ld8(dy + 8 * i);
+    V8 o;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) o.v[j] = m.v[j] > 0.f ? g.v[j] : 0.f;
+    if (acc) {
+      const V8 p = ld8(dx + 8 * i);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) o.v[j] += p.v[j];
+    }
+    st8(dx + 8 * i, o);
+  }
+}
+
+__global__ void add_x8_k(const bf16* __restrict__ a, const bf16* __restrict__ b, bf16* __restrict__ y, int64_t n8,
+                         int relu) {
+  GRID_STRIDE8(i, n8) {
+    const V8 p = ld8(a + 8 * i), q = ld8(b + 8 * i);
+    V8 o;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) o.v[j] = relu ? fmaxf(p.v[j] + q.v[j], 0.f) : p.v[j] + q.v[j];
+    st8(y + 8 * i, o);
+  }
+}
+
+__global__ void copy_acc_x8_k(const bf16* __restrict__ x, bf16* __restrict__ y, int64_t n8, int acc) {
+  GRID_STRIDE8(i, n8) {
+    if (!acc) {
+      *reinterpret_cast<uint4*>(y + 8 * i) = *reinterpret_cast<const uint4*>(x + 8 * i);
+    } else {
+      const V8 p = ld8(x + 8 * i), q = ld8(y + 8 * i);
+      V8 o;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) o.v[j] = p.v[j] + q.v[j];
+      st8(y + 8 * i, o);
+    }
+  }
+}
+
+__global__ void affine_fwd_x8_k(const bf16* __restrict__ x, const float* __restrict__ sc,
+                                const float* __restrict__ sh, bf16* __restrict__ y, int64_t n8, int C, int relu) {
+  GRID_STRIDE8(i, n8) {
+    const int c = int((8 * i) % C);
+    const V8 p = ld8(x + 8 * i);
+    V8 o;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float v = fmaf(p.v[j], sc[c + j], sh[c + j]);
+      o.v[j] = relu ? fmaxf(v, 0.f) : v;
+    }
+    st8(y + 8 * i, o);
+  }
+}
+
+__device__ __forceinline__ float gelu_cdf(float x) { return 0.5f * (1.f + erff(x * 0.70710678118654752f)); }
+
+__global__ void gelu_fwd_x8_k(const bf16* __restrict__ x, bf16* __restrict__ y, int64_t n8) {
+  GRID_STRIDE8(i, n8) {
+    const V8 p = ld8(x + 8 * i);
+    V8 o;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) o.v[j] = p.v[j] * gelu_cdf(p.v[j]);
+    st8(y + 8 * i, o);
+  }
+}
+
+__global__ void gelu_bwd_x8_k(const bf16* __restrict__ x, const bf16* __restrict__ dy, bf16* __restrict__ dx,
+                              int64_t n8, int acc) {
+  GRID_STRIDE8(i, n8) {
+    const V8 p = ld8(x + 8 * i), g = ld8(dy + 8 * i);
+    V8 o;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float v = p.v[j];
+      const float pdf = 0.39894228040143268f * expf(-0.5f * v * v);
+      o.v[j] = g.v[j] * (gelu_cdf(v) + v * pdf);
+    }
+    if (acc) {
+      const V8 q = ld8(dx + 8 * i);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) o.v[j] += q.v[j];
+    }
+    st8(dx + 8 * i, o);
+  }
+}
+
+// Column partial sums over a (128-row chunk, 256-column block): thread
+// (g, r) owns columns c0 + 8g .. +7 and rows r, r + 8, ...; the 8 row lanes
+// are combined in shared memory in a fixed order.  MODE 0: sums of a;
+// MODE 1: affine backward (sums of dy * x and dy, and dx (+)= dy * scale).
+template <int MODE>
+__global__ void __launch_bounds__(256) colsum8_k(const bf16* __restrict__ a, const bf16* __restrict__ x,
+                                                 const float* __restrict__ scale, bf16* __restrict__ dx, int acc,
+                                                 int64_t rows, int C, float* __restrict__ p0, float* __restrict__ p1) {
+  __shared__ float red0[8][257];
+  __shared__ float red1[MODE == 1 ? 8 : 1][257];
+  const int g = threadIdx.x % 32, r = threadIdx.x / 32;
+  const int c = blockIdx.x * 256 + 8 * g;
+  const int64_t r0 = int64_t(blockIdx.y) * kChunk;
+  float s0[8] = {0, 0, 0, 0, 0, 0, 0, 0}, s1[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  if (c < C) {
+    float sc[8];
+    if (MODE == 1)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) sc[j] = scale[c + j];
+    for (int64_t row = r0 + r; row < r0 + kChunk && row < rows; row += 8) {
+      const V8 d = ld8(a + row * C + c);
+      if (MODE == 0) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) s0[j] += d.v[j];
+      } else {
+        const V8 xv = ld8(x + row * C + c);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          s0[j] = fmaf(d.v[j], xv.v[j], s0[j]);
+          s1[j] += d.v[j];
+        }
+        if (dx) {
+          V8 o;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) o.v[j] = d.v[j] * sc[j];
+          if (acc) {
+            const V8 q = ld8(dx + row * C + c);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) o.v[j] += q.v[j];
+          }
+          st8(dx + row * C + c, o);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    red0[r][8 * g + j] = s0[j];
+    if (MODE == 1) red1[r][8 * g + j] = s1[j];
+  }
+  __syncthreads();
+  const int cc = blockIdx.x * 256 + threadIdx.x;
+  if (cc < C) {
+    float t0 = 0.f, t1 = 0.f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      t0 += red0[q][threadIdx.x];
+      if (MODE == 1) t1 += red1[q][threadIdx.x];
+    }
+    p0[int64_t(blockIdx.y) * C + cc] = t0;
+    if (MODE == 1) p1[int64_t(blockIdx.y) * C + cc] = t1;
+  }
+}
+
+// Layernorm backward fused with its parameter gradients: one warp per row
+// (dx), and per block of 8 warps x 8 rows the column partials of
+// dy * xhat (gamma) and dy (beta).  C <= 512, C % 256 == 0; dx may be null
+// (a layernorm of the uploaded batch has no input gradient).
+__global__ void __launch_bounds__(256) layernorm_bwd_fused_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
+                                                             const float* __restrict__ mean, const float* __restrict__ rstd,
+                                                             const bf16* __restrict__ dy, bf16* __restrict__ dx,
+                                                             int64_t rows, int C, int acc, float* __restrict__ pg,
+                                                             float* __restrict__ pb) {
+  constexpr int kMaxV = 2;  // up to 2 x 8 x 32 = 512 columns per row
+  __shared__ float redg[8][512];
+  __shared__ float redb[8][512];
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int nv = C / 256;  // 8-wide vectors per lane
+  float sg[kMaxV][8], sb[kMaxV][8];
+#pragma unroll
+  for (int v = 0; v < kMaxV; ++v)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) sg[v][j] = sb[v][j] = 0.f;
+  const int64_t row0 = int64_t(blockIdx.x) * 64;
+  for (int rr = warp; rr < 64; rr += 8) {
+    const int64_t row = row0 + rr;
+    if (row >= rows) break;
+    const float mu = mean[row], rs = rstd[row];
+    V8 xv[kMaxV], gv[kMaxV];
+    float a = 0.f, b = 0.f;
+#pragma unroll
+    for (int v = 0; v < kMaxV; ++v) {
+      if (v >= nv) break;
+      const int c = (v * 32 + lane) * 8;
+      xv[v] = ld8(x + row * C + c);
+      gv[v] = ld8(dy + row * C + c);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float xh = (xv[v].v[j] - mu) * rs;
+        const float dxh = gv[v].v[j] * gamma[c + j];
+        a += dxh;
+        b += dxh * xh;
+        sg[v][j] = fmaf(gv[v].v[j], xh, sg[v][j]);
+        sb[v][j] += gv[v].v[j];
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      a += __shfl_xor_sync(0xffffffffu, a, o);
+      b += __shfl_xor_sync(0xffffffffu, b, o);
+    }
+    a /= float(C);
+    b /= float(C);
+#pragma unroll
+    for (int v = 0; v < kMaxV; ++v) {
+      if (v >= nv) break;
+      const int c = (v * 32 + lane) * 8;
+      V8 o;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float xh = (xv[v].v[j] - mu) * rs;
+        const float dxh = gv[v].v[j] * gamma[c + j];
+        o.v[j] = rs * (dxh - a - xh * b);
+      }
+      if (!dx) continue;
+      if (acc) {
+        const V8 q = ld8(dx + row * C + c);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) o.v[j] += q.v[j];
+      }
+      st8(dx + row * C + c, o);
+    }
+  }
+#pragma unroll
+  for (int v = 0; v < kMaxV; ++v) {
+    if (v >= nv) break;
+    const int c = (v * 32 + lane) * 8;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      redg[warp][c + j] = sg[v][j];
+      redb[warp][c + j] = sb[v][j];
+    }
+  }
+  __syncthreads();
+  for (int c = threadIdx.x; c < C; c += blockDim.x) {
+    float tg = 0.f, tb = 0.f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      tg += redg[q][c];
+      tb += redb[q][c];
+    }
+    pg[int64_t(blockIdx.x) * C + c] = tg;
+    pb[int64_t(blockIdx.x) * C + c] = tb;
+  }
+}
+
+__global__ void finish_k(const float* __restrict__ partial, int chunks, int C, float* __restrict__ out) {
+  __shared__ float red[8][33];
+  const int cl = threadIdx.x % 32, rl = threadIdx.x / 32;
+  const int c = blockIdx.x * 32 + cl;
+  float s = 0.f;
+  if (c < C) {
+    int q = rl;
+    for (; q + 24 < chunks; q += 32) {
+      const float a0 = partial[int64_t(q) * C + c], a1 = partial[int64_t(q + 8) * C + c];
+      const float a2 = partial[int64_t(q + 16) * C + c], a3 = partial[int64_t(q + 24) * C + c];
+      s += a0;
+      s += a1;
+      s += a2;
+      s += a3;
+    }
+    for (; q < chunks; q += 8) s += partial[int64_t(q) * C + c];
+  }
+  red[rl][cl] = s;
+  __syncthreads();
+  if (rl == 0 && c < C) {
+    float t = 0.f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) t += red[q][cl];
+    out[c] = t;
+  }
+}
+
+int chunks_of(int64_t rows) { return int((rows + kChunk - 1) / kChunk); }
+
+}  // namespace
+
+bool vec8_ok(int dt, int64_t n) { return dt == kBF16 && n % 8 == 0; }
+
+void relu_bwd_x8(const void* y, const void* dy, void* dx, int64_t n, bool acc, cudaStream_t st) {
+  relu_bwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)y, (const bf16*)dy, (bf16*)dx, n / 8, acc);
+}
+void add_x8(const void* a, const void* b, void* y, int64_t n, bool relu, cudaStream_t st) {
+  add_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)a, (const bf16*)b, (bf16*)y, n / 8, relu);
+}
+void copy_acc_x8(const void* x, void* y, int64_t n, bool acc, cudaStream_t st) {
+  copy_acc_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, (bf16*)y, n / 8, acc);
+}
+void affine_fwd_x8(const void* x, const float* sc, const float* sh, void* y, int64_t n, int C, bool relu,
+                   cudaStream_t st) {
+  affine_fwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, sc, sh, (bf16*)y, n / 8, C, relu);
+}
+void gelu_fwd_x8(const void* x, void* y, int64_t n, cudaStream_t st) {
+  gelu_fwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, (bf16*)y, n / 8);
+}
+void gelu_bwd_x8(const void* x, const void* dy, void* dx, int64_t n, bool acc, cudaStream_t st) {
+  gelu_bwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, (const bf16*)dy, (bf16*)dx, n / 8, acc);
+}
+
+int64_t colsum8_partial_floats(int64_t rows, int C) { return int64_t(chunks_of(rows)) * C; }
+
+void colsum8(const void* a, int64_t rows, int C, float* partial, float* out, cudaStream_t st) {
+  dim3 grid(ceil_div(C, 256), chunks_of(rows));
+  colsum8_k<0><<<grid, 256, 0, st>>>((const bf16*)a, nullptr, nullptr, nullptr, 0, rows, C, partial, nullptr);
+  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, chunks_of(rows), C, out);
+}
+
+void affine_bwd8(const void* dy, const void* x, const float* scale, void* dx, bool acc, int64_t rows, int C,
+                 float* partial, float* dscale, float* dshift, cudaStream_t st) {
+  dim3 grid(ceil_div(C, 256), chunks_of(rows));
+  float* p1 = partial + colsum8_partial_floats(rows, C);
+  colsum8_k<1><<<grid, 256, 0, st>>>((const bf16*)dy, (const bf16*)x, scale, (bf16*)dx, acc, rows, C, partial, p1);
+  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, chunks_of(rows), C, dscale);
+  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(p1, chunks_of(rows), C, dshift);
+}
+
+bool layernorm_bwd8_ok(int dt, int C) { return dt == kBF16 && C % 256 == 0 && C <= 512; }
+
+int64_t layernorm_bwd8_partial_floats(int64_t rows, int C) { return 2 * ((rows + 63) / 64) * C; }
+
+void layernorm_bwd8(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
+                    void* dx, int64_t rows, int C, bool acc, float* partial, float* dgamma, float* dbeta,
+                    cudaStream_t st) {
+  const int blocks = int((rows + 63) / 64);
+  float* pb = partial + int64_t(blocks) * C;
+  layernorm_bwd_fused_k<<<blocks, 256, 0, st>>>((const bf16*)x, gamma, mean, rstd, (const bf16*)dy, (bf16*)dx, rows,
+                                                C, acc, partial, pb);
+  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, blocks, C, dgamma);
+  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(pb, blocks, C, dbeta);
+}
+
+}  // namespace fo
