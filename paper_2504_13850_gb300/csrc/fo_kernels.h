@@ -55,10 +55,13 @@ void layernorm_bwd_dx(const void* x, const float* gamma, const float* mean, cons
                       const void* dy, void* dx, int64_t rows, int C, int dt, bool acc,
                       cudaStream_t st);
 // out[c] = sum_r a[r][c] * f(r, c) where f = 1, b[r][c], or the layernorm xhat.
-// `partial` is scratch of at least colsum_partial_floats(rows, C) floats.
+// `partial` is scratch of at least colsum_partial_floats(rows, C) floats
+// (128-row chunks); the server passes adaptive = true (chunks sized to the
+// GPU, scratch from server_colsum_floats).
 int64_t colsum_partial_floats(int64_t rows, int C);
+int64_t server_colsum_floats(int64_t rows, int C);
 void colsum(const void* a, const void* b, int64_t rows, int C, int dt, float* partial,
-            float* out, cudaStream_t st);
+            float* out, cudaStream_t st, bool adaptive = false);
 void colsum_lnx(const void* dy, const void* x, const float* mean, const float* rstd,
                 int64_t rows, int C, int dt, float* partial, float* out, cudaStream_t st);
 void meanpool_fwd(const void* x, const int32_t* len, void* y, int B, int L, int C, int dt,
@@ -104,11 +107,12 @@ void affine_fwd_x8(const void* x, const float* sc, const float* sh, void* y, int
                    cudaStream_t st);
 void gelu_fwd_x8(const void* x, void* y, int64_t n, cudaStream_t st);
 void gelu_bwd_x8(const void* x, const void* dy, void* dx, int64_t n, bool acc, cudaStream_t st);
-// Column sums (C % 8 == 0) with a (column block, row chunk) grid.
-int64_t colsum8_partial_floats(int64_t rows, int C);
-void colsum8(const void* a, int64_t rows, int C, float* partial, float* out, cudaStream_t st);
+// Column sums (C % 8 == 0) with a (column block, row chunk) grid; chunks of
+// 128 rows, or sized to the GPU (about two blocks per SM) when `adaptive`.
+int64_t colsum8_partial_floats(int64_t rows, int C, bool adaptive);
+void colsum8(const void* a, int64_t rows, int C, float* partial, float* out, bool adaptive, cudaStream_t st);
 // Affine backward in one pass: dscale = sum dy*x, dshift = sum dy, dx (+)= dy*scale
-// (dx may be null); partial holds 2 * colsum8_partial_floats floats.
+// (dx may be null); partial holds 2 * colsum8_partial_floats(rows, C, true) floats.
 void affine_bwd8(const void* dy, const void* x, const float* scale, void* dx, bool acc, int64_t rows, int C,
                  float* partial, float* dscale, float* dshift, cudaStream_t st);
 // Layernorm backward fused with dgamma / dbeta (C % 256 == 0, C <= 512).

@@ -404,7 +404,8 @@ int build_plan(fo_server* s) {
         const double fl = 2.0 * double(s->T[o].rows()) * op.cout * double(op.kind == FO_OP_CONV ? op.k * op.k : 1) * op.cin;
         if (bias) {
           add("bias_grad", 2, 0.0, double(s->T[o].bytes()), [=](cudaStream_t st) {
-            fo::colsum(s->T[o].grad, nullptr, s->T[o].rows(), s->T[o].C, dto, s->colsum_scratch, G(s, i, 1), st);
+            fo::colsum(s->T[o].grad, nullptr, s->T[o].rows(), s->T[o].C, dto, s->colsum_scratch, G(s, i, 1), st,
+                       true);
           });
         }
         if (need_dx) {
@@ -625,9 +626,8 @@ int allocate(fo_server* s) {
   for (int i = 0; i < nops; ++i) {
     const Tensor& o = s->T[i + 1];
     const Tensor& a = s->T[s->ops[i].in0];
-    // two partial arrays (affine / layernorm backward), 64- or 128-row chunks
-    cs_floats = std::max(cs_floats, 4 * fo::colsum_partial_floats(o.rows(), o.C));
-    cs_floats = std::max(cs_floats, 4 * fo::colsum_partial_floats(a.rows(), a.C));
+    cs_floats = std::max(cs_floats, fo::server_colsum_floats(o.rows(), o.C));
+    cs_floats = std::max(cs_floats, fo::server_colsum_floats(a.rows(), a.C));
   }
   s->colsum_scratch = (float*)s->alloc(cs_floats * 4);
   s->ln_mean.assign(nops, nullptr);

@@ -4,6 +4,7 @@
 #include "fo_common.cuh"
 #include "fo_kernels.h"
 
+#include <algorithm>
 #include <cmath>
 
 namespace fo {
@@ -449,9 +450,17 @@ __global__ void colsum_finish_k(const float* partial, int chunks, int C, float* 
   }
 }
 
+// Scratch the server's column sums may use: every variant it launches.
+int64_t server_colsum_floats(int64_t rows, int C) {
+  int64_t a = colsum_partial_floats(rows, C);
+  int64_t b = 2 * colsum8_partial_floats(rows, C, true);
+  int64_t c = layernorm_bwd8_partial_floats(rows, C);
+  return std::max(a, std::max(b, c));
+}
+
 void colsum(const void* a, const void* b, int64_t rows, int C, int dt, float* partial, float* out,
-            cudaStream_t st) {
-  if (!b && dt == kBF16 && C % 8 == 0) return colsum8(a, rows, C, partial, out, st);
+            cudaStream_t st, bool adaptive) {
+  if (!b && dt == kBF16 && C % 8 == 0) return colsum8(a, rows, C, partial, out, adaptive, st);
   dim3 grid(ceil_div(C, 32), colsum_chunks(rows));
   if (b) {
     FO_DISPATCH(dt, T, colsum_partial_k<1, T><<<grid, 256, 0, st>>>((const T*)a, (const T*)b, nullptr, nullptr, rows, C, partial));

@@ -75,6 +75,9 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
                : "memory");
 }
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -250,6 +253,58 @@ __device__ __forceinline__ void cluster_reduce_rows(const TcParams& p, uint32_t 
       }
       store4(p, m, n0 + c, acc);
     }
+  }
+}
+
+// Epilogue of 16 consecutive outputs (m, n..n+15) in registers.
+__device__ __forceinline__ void store16(const TcParams& p, int m_gemm, int n, float (&v)[16]) {
+  const size_t m = out_row(p, m_gemm);
+  if (p.bias)
+#pragma unroll
+    for (int j = 0; j < 16; ++j) v[j] += p.bias[n + j];
+  if (p.relu)
+#pragma unroll
+    for (int j = 0; j < 16; ++j) v[j] = fmaxf(v[j], 0.f);
+  if (p.mask) {
+    const uint4* mk = reinterpret_cast<const uint4*>(p.mask + m * p.ldo + n);
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const uint4 u = mk[j];
+      const bf16* e = reinterpret_cast<const bf16*>(&u);
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        if (!(__bfloat162float(e[q]) > 0.f)) v[8 * j + q] = 0.f;
+    }
+  }
+  if (p.out_f32) {
+    float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + m * p.ldo + n);
+    if (p.acc)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float4 o = dst[j];
+        v[4 * j] += o.x; v[4 * j + 1] += o.y; v[4 * j + 2] += o.z; v[4 * j + 3] += o.w;
+      }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+  } else {
+    uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(p.out) + m * p.ldo + n);
+    if (p.acc)
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const uint4 o = dst[j];
+        const bf16* e = reinterpret_cast<const bf16*>(&o);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) v[8 * j + q] += __bfloat162float(e[q]);
+      }
+    uint4 pk[2];
+    uint32_t* pw = reinterpret_cast<uint32_t*>(pk);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      __nv_bfloat162 h2 = __floats2bfloat162_rn(v[2 * j], v[2 * j + 1]);
+      pw[j] = *reinterpret_cast<uint32_t*>(&h2);
+    }
+    dst[0] = pk[0];
+    dst[1] = pk[1];
   }
 }
 
@@ -504,6 +559,155 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
   }
 }
 
+
+// Persistent variant (no K split): gridDim.x CTAs loop over the output tiles
+// (n fastest).  The TMA producer runs ahead across tile boundaries and the
+// accumulator is double-buffered in TMEM, so the epilogue of one tile
+// overlaps the MMAs of the next.  Barriers: full/empty per stage (TMA <->
+// MMA), acc_full/acc_empty per accumulator (MMA <-> epilogue).
+template <int KIND, int BN, int STAGES>
+__global__ void __launch_bounds__(kThreads, 1) tc_gemm_persistent(const __grid_constant__ TcParams p) {
+  extern __shared__ __align__(1024) char smem_raw[];
+  char* smem = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  constexpr int A_BYTES = BM * BK * 2;
+  constexpr int B_BYTES = BN * BK * 2;
+  constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* acc_full = empty + STAGES;
+  uint64_t* acc_empty = acc_full + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int n_tiles = p.N / BN;
+  const int tiles = n_tiles * ((p.M + BM - 1) / BM);
+  const int KB = p.KB;
+  constexpr uint32_t kCols = 2 * BN < 32 ? 32 : 2 * BN;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 128);
+    }
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmA)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmB)) : "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(kCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint32_t g = 0;
+      for (int t = blockIdx.x; t < tiles && !*abort_flag; t += gridDim.x) {
+        const int n0 = (t % n_tiles) * BN, m0 = (t / n_tiles) * BM;
+        for (int kb = 0; kb < KB; ++kb, ++g) {
+          const int s = g % STAGES;
+          if (!mbar_wait(&empty[s], ((g / STAGES) & 1) ^ 1)) {
+            atomicExch(p.err, 4);
+            *abort_flag = 1;
+            break;
+          }
+          char* sa = smem + s * STAGE_BYTES;
+          mbar_expect_tx(&full[s], STAGE_BYTES);
+          load_kblock<KIND, BN>(p, kb, m0, n0, sa, sa + A_BYTES, &full[s]);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = instr_desc(BN, KindTraits<KIND>::a_mn, KindTraits<KIND>::b_mn);
+      uint32_t g = 0, lt = 0;
+      for (int t = blockIdx.x; t < tiles && !*abort_flag; t += gridDim.x, ++lt) {
+        const uint32_t b = lt & 1;
+        if (!mbar_wait(&acc_empty[b], ((lt >> 1) & 1) ^ 1)) {
+          atomicExch(p.err, 5);
+          *abort_flag = 1;
+          mbar_expect_tx(&acc_full[b], 0);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem + b * BN;
+        bool ok = true;
+        for (int kb = 0; kb < KB; ++kb, ++g) {
+          const int s = g % STAGES;
+          if (!mbar_wait(&full[s], (g / STAGES) & 1)) {
+            atomicExch(p.err, 6);
+            *abort_flag = 1;
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(smem + s * STAGE_BYTES);
+          const uint32_t b0 = a0 + A_BYTES;
+#pragma unroll
+          for (int k = 0; k < BK / UK; ++k) {
+            uint64_t ad, bd;
+            if (KindTraits<KIND>::a_mn) ad = smem_desc(a0 + k * UK * 128, BK * 128, 1024);
+            else ad = smem_desc(a0 + k * UK * 2, 16, 1024);
+            if (KindTraits<KIND>::b_mn) bd = smem_desc(b0 + k * UK * 128, BK * 128, 1024);
+            else bd = smem_desc(b0 + k * UK * 2, 16, 1024);
+            mma_f16(d, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+          }
+          mma_commit(&empty[s]);
+        }
+        if (ok) mma_commit(&acc_full[b]);
+        else {
+          mbar_expect_tx(&acc_full[b], 0);
+          break;
+        }
+      }
+    }
+  } else {
+    const int q = warp % 4;
+    const int row = q * 32 + lane;
+    uint32_t lt = 0;
+    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++lt) {
+      const uint32_t b = lt & 1;
+      const int n0 = (t % n_tiles) * BN, m0 = (t / n_tiles) * BM;
+      const bool ready = mbar_wait(&acc_full[b], (lt >> 1) & 1);
+      tc_fence_after();
+      if (!ready) {
+        atomicExch(p.err, 7);
+        *abort_flag = 1;
+      }
+      if (!ready || *abort_flag) break;
+      const int m = m0 + row;
+      for (int c = 0; c < BN; c += 16) {
+        uint32_t r[16];
+        tmem_ld16(tmem + b * BN + (uint32_t(q * 32) << 16) + uint32_t(c), r);
+        if (m >= p.M) continue;
+        float v[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
+        store16(p, m, n0 + c, v);
+      }
+      tc_fence_before();
+      mbar_arrive(&acc_empty[b]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kCols) : "memory");
+  }
+}
+
 template <int KIND, int BN>
 constexpr int stages_for() {
   return kSmemBudget / (BM * BK * 2 + BN * BK * 2) > 8 ? 8 : kSmemBudget / (BM * BK * 2 + BN * BK * 2);
@@ -518,7 +722,7 @@ typedef void (*KernelFn)(const TcParams);
 template <int KIND, int BN>
 KernelFn kernel_ptr(bool cluster) {
   if (cluster) return tc_gemm_kernel<KIND, BN, stages_for<KIND, BN>(), true>;
-  return tc_gemm_kernel<KIND, BN, stages_for<KIND, BN>(), false>;
+  return tc_gemm_persistent<KIND, BN, stages_for<KIND, BN>()>;
 }
 
 KernelFn pick_kernel(int kind, int bn, bool cluster, size_t* smem) {
@@ -648,11 +852,12 @@ bool window_ok(int N, int H, int W, int rows_needed, int* rows, int* imgs) {
 }
 
 
-// Tile width and K split from a small cost model.  One CTA per SM; a CTA
+// Tile width and K split from a small cost model.  One CTA per SM; a tile
 // costs its k-blocks (a 128-wide k-block runs at ~0.55 of a 256-wide one)
-// plus its epilogue, plus the cluster reduction when K is split; a split
-// cluster holds <= 8 CTAs (portable size) and clusters above 4 pay for
-// their poorer packing into GPCs.  Minimises waves x cost per CTA.
+// plus its epilogue.  Unsplit plans run persistent (epilogue overlapped,
+// paid once); a K split runs as clusters of <= 8 CTAs (portable size) that
+// pay the epilogue and the cluster reduction per CTA, and clusters above 4
+// pay for their poorer packing into GPCs.  Minimises the estimated time.
 // Candidate widths divide `ndiv` (N, or the channels of one tap for the
 // weight gradient, whose N index runs over taps x channels).
 void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv) {
@@ -670,7 +875,9 @@ void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv) {
       if (splits != sp) continue;
       const int ctas = tiles * splits;
       const double waves = double((ctas + c->num_sms - 1) / c->num_sms);
-      double cost = waves * (kper * per_kb + epi + (splits > 1 ? 2.0 : 0.0));
+      // unsplit plans run persistent: epilogues overlap the next tile's MMAs
+      double cost = splits == 1 ? waves * kper * per_kb + epi
+                                : waves * (kper * per_kb + epi + 2.0);
       if (splits > 4) cost *= 1.2;
       if (cost < best - 1e-9) {
         best = cost;
@@ -699,7 +906,12 @@ TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
     delete g;
     return nullptr;
   }
-  g->grid = dim3(N / g->bn, (M + BM - 1) / BM, g->splits);
+  if (g->splits > 1) {
+    g->grid = dim3(N / g->bn, (M + BM - 1) / BM, g->splits);
+  } else {
+    const int tiles = (N / g->bn) * ((M + BM - 1) / BM);
+    g->grid = dim3(std::min(tiles, c->num_sms), 1, 1);
+  }
   if (getenv("FO_DEBUG_PLAN"))
     fprintf(stderr, "[plan] %-16s M=%d N=%d KB=%d BN=%d splits=%d grid=(%u,%u,%u)\n", g->name, M, N, g->p.KB,
             g->bn, g->splits, g->grid.x, g->grid.y, g->grid.z);

@@ -11,7 +11,7 @@ namespace fo {
 
 namespace {
 
-constexpr int kChunk = 128;  // rows per column-sum chunk (as the scalar kernels)
+constexpr int kChunk = 128;  // rows per column-sum chunk of the public entry points
 
 struct V8 {
   float v[8];
@@ -131,19 +131,20 @@ __global__ void gelu_bwd_x8_k(const bf16* __restrict__ x, const bf16* __restrict
 template <int MODE>
 __global__ void __launch_bounds__(256) colsum8_k(const bf16* __restrict__ a, const bf16* __restrict__ x,
                                                  const float* __restrict__ scale, bf16* __restrict__ dx, int acc,
-                                                 int64_t rows, int C, float* __restrict__ p0, float* __restrict__ p1) {
+                                                 int64_t rows, int C, int chunk, float* __restrict__ p0,
+                                                 float* __restrict__ p1) {
   __shared__ float red0[8][257];
   __shared__ float red1[MODE == 1 ? 8 : 1][257];
   const int g = threadIdx.x % 32, r = threadIdx.x / 32;
   const int c = blockIdx.x * 256 + 8 * g;
-  const int64_t r0 = int64_t(blockIdx.y) * kChunk;
+  const int64_t r0 = int64_t(blockIdx.y) * chunk;
   float s0[8] = {0, 0, 0, 0, 0, 0, 0, 0}, s1[8] = {0, 0, 0, 0, 0, 0, 0, 0};
   if (c < C) {
     float sc[8];
     if (MODE == 1)
 #pragma unroll
       for (int j = 0; j < 8; ++j) sc[j] = scale[c + j];
-    for (int64_t row = r0 + r; row < r0 + kChunk && row < rows; row += 8) {
+    for (int64_t row = r0 + r; row < r0 + chunk && row < rows; row += 8) {
       const V8 d = ld8(a + row * C + c);
       if (MODE == 0) {
 #pragma unroll
@@ -189,7 +190,7 @@ __global__ void __launch_bounds__(256) colsum8_k(const bf16* __restrict__ a, con
 }
 
 // Layernorm backward fused with its parameter gradients: one warp per row
-// (dx), and per block of 8 warps x 8 rows the column partials of
+// (dx), and per block of 8 warps x 2 rows the column partials of
 // dy * xhat (gamma) and dy (beta).  C <= 512, C % 256 == 0; dx may be null
 // (a layernorm of the uploaded batch has no input gradient).
 __global__ void __launch_bounds__(256) layernorm_bwd_fused_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
@@ -207,8 +208,8 @@ __global__ void __launch_bounds__(256) layernorm_bwd_fused_k(const bf16* __restr
   for (int v = 0; v < kMaxV; ++v)
 #pragma unroll
     for (int j = 0; j < 8; ++j) sg[v][j] = sb[v][j] = 0.f;
-  const int64_t row0 = int64_t(blockIdx.x) * 64;
-  for (int rr = warp; rr < 64; rr += 8) {
+  const int64_t row0 = int64_t(blockIdx.x) * 16;
+  for (int rr = warp; rr < 16; rr += 8) {
     const int64_t row = row0 + rr;
     if (row >= rows) break;
     const float mu = mean[row], rs = rstd[row];
@@ -307,7 +308,25 @@ __global__ void finish_k(const float* __restrict__ partial, int chunks, int C, f
   }
 }
 
-int chunks_of(int64_t rows) { return int((rows + kChunk - 1) / kChunk); }
+int chunks_of(int64_t rows, int chunk) { return int((rows + chunk - 1) / chunk); }
+
+// Rows per chunk for the server's column sums: about two blocks per SM,
+// between 8 and 128 rows, a multiple of 8.
+int adaptive_chunk(int64_t rows, int C) {
+  static int sms = 0;
+  if (!sms) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (sms <= 0) sms = 148;
+  }
+  const int64_t colblocks = (C + 255) / 256;
+  int64_t ch = rows * colblocks / (2 * int64_t(sms));
+  ch = (ch + 7) / 8 * 8;
+  if (ch < 8) ch = 8;
+  if (ch > 128) ch = 128;
+  return int(ch);
+}
 
 }  // namespace
 
@@ -333,31 +352,36 @@ void gelu_bwd_x8(const void* x, const void* dy, void* dx, int64_t n, bool acc, c
   gelu_bwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, (const bf16*)dy, (bf16*)dx, n / 8, acc);
 }
 
-int64_t colsum8_partial_floats(int64_t rows, int C) { return int64_t(chunks_of(rows)) * C; }
+int64_t colsum8_partial_floats(int64_t rows, int C, bool adaptive) {
+  return int64_t(chunks_of(rows, adaptive ? adaptive_chunk(rows, C) : kChunk)) * C;
+}
 
-void colsum8(const void* a, int64_t rows, int C, float* partial, float* out, cudaStream_t st) {
-  dim3 grid(ceil_div(C, 256), chunks_of(rows));
-  colsum8_k<0><<<grid, 256, 0, st>>>((const bf16*)a, nullptr, nullptr, nullptr, 0, rows, C, partial, nullptr);
-  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, chunks_of(rows), C, out);
+void colsum8(const void* a, int64_t rows, int C, float* partial, float* out, bool adaptive, cudaStream_t st) {
+  const int ch = adaptive ? adaptive_chunk(rows, C) : kChunk;
+  dim3 grid(ceil_div(C, 256), chunks_of(rows, ch));
+  colsum8_k<0><<<grid, 256, 0, st>>>((const bf16*)a, nullptr, nullptr, nullptr, 0, rows, C, ch, partial, nullptr);
+  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, chunks_of(rows, ch), C, out);
 }
 
 void affine_bwd8(const void* dy, const void* x, const float* scale, void* dx, bool acc, int64_t rows, int C,
                  float* partial, float* dscale, float* dshift, cudaStream_t st) {
-  dim3 grid(ceil_div(C, 256), chunks_of(rows));
-  float* p1 = partial + colsum8_partial_floats(rows, C);
-  colsum8_k<1><<<grid, 256, 0, st>>>((const bf16*)dy, (const bf16*)x, scale, (bf16*)dx, acc, rows, C, partial, p1);
-  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, chunks_of(rows), C, dscale);
-  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(p1, chunks_of(rows), C, dshift);
+  const int ch = adaptive_chunk(rows, C);
+  dim3 grid(ceil_div(C, 256), chunks_of(rows, ch));
+  float* p1 = partial + colsum8_partial_floats(rows, C, true);
+  colsum8_k<1><<<grid, 256, 0, st>>>((const bf16*)dy, (const bf16*)x, scale, (bf16*)dx, acc, rows, C, ch, partial,
+                                     p1);
+  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, chunks_of(rows, ch), C, dscale);
+  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(p1, chunks_of(rows, ch), C, dshift);
 }
 
 bool layernorm_bwd8_ok(int dt, int C) { return dt == kBF16 && C % 256 == 0 && C <= 512; }
 
-int64_t layernorm_bwd8_partial_floats(int64_t rows, int C) { return 2 * ((rows + 63) / 64) * C; }
+int64_t layernorm_bwd8_partial_floats(int64_t rows, int C) { return 2 * ((rows + 15) / 16) * C; }
 
 void layernorm_bwd8(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
                     void* dx, int64_t rows, int C, bool acc, float* partial, float* dgamma, float* dbeta,
                     cudaStream_t st) {
-  const int blocks = int((rows + 63) / 64);
+  const int blocks = int((rows + 15) / 16);
   float* pb = partial + int64_t(blocks) * C;
   layernorm_bwd_fused_k<<<blocks, 256, 0, st>>>((const bf16*)x, gamma, mean, rstd, (const bf16*)dy, (bf16*)dx, rows,
                                                 C, acc, partial, pb);
