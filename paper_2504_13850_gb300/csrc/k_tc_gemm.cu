@@ -259,9 +259,14 @@ __device__ __forceinline__ void cluster_reduce_rows(const TcParams& p, uint32_t 
 // Epilogue of 16 consecutive outputs (m, n..n+15) in registers.
 __device__ __forceinline__ void store16(const TcParams& p, int m_gemm, int n, float (&v)[16]) {
   const size_t m = out_row(p, m_gemm);
-  if (p.bias)
+  if (p.bias) {
+    const float4* b4 = reinterpret_cast<const float4*>(p.bias + n);
 #pragma unroll
-    for (int j = 0; j < 16; ++j) v[j] += p.bias[n + j];
+    for (int j = 0; j < 4; ++j) {
+      const float4 b = __ldg(b4 + j);
+      v[4 * j] += b.x; v[4 * j + 1] += b.y; v[4 * j + 2] += b.z; v[4 * j + 3] += b.w;
+    }
+  }
   if (p.relu)
 #pragma unroll
     for (int j = 0; j < 16; ++j) v[j] = fmaxf(v[j], 0.f);
@@ -306,6 +311,19 @@ __device__ __forceinline__ void store16(const TcParams& p, int m_gemm, int n, fl
     dst[0] = pk[0];
     dst[1] = pk[1];
   }
+}
+
+// 32 consecutive TMEM columns of this thread's lane, one wait.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
 template <int KIND>
@@ -565,8 +583,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 // accumulator is double-buffered in TMEM, so the epilogue of one tile
 // overlaps the MMAs of the next.  Barriers: full/empty per stage (TMA <->
 // MMA), acc_full/acc_empty per accumulator (MMA <-> epilogue).
+constexpr int kPersistThreads = 320;  // TMA warp, MMA warp, 8 epilogue warps
+
 template <int KIND, int BN, int STAGES>
-__global__ void __launch_bounds__(kThreads, 1) tc_gemm_persistent(const __grid_constant__ TcParams p) {
+__global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const __grid_constant__ TcParams p) {
   extern __shared__ __align__(1024) char smem_raw[];
   char* smem = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   constexpr int A_BYTES = BM * BK * 2;
@@ -592,7 +612,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_persistent(const __grid_c
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
-      mbar_init(&acc_empty[b], 128);
+      mbar_init(&acc_empty[b], kPersistThreads - 64);
     }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -673,8 +693,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_persistent(const __grid_c
       }
     }
   } else {
-    const int q = warp % 4;
+    // Epilogue: warp w (2..9) reads TMEM lanes 32 * (w % 4) .. +31; the two
+    // warps of a lane quarter split the tile's columns.
+    const int q = warp % 4, half = (warp - 2) / 4;
     const int row = q * 32 + lane;
+    constexpr int CW = BN / 2;  // columns per epilogue warp
     uint32_t lt = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++lt) {
       const uint32_t b = lt & 1;
@@ -687,14 +710,29 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_persistent(const __grid_c
       }
       if (!ready || *abort_flag) break;
       const int m = m0 + row;
-      for (int c = 0; c < BN; c += 16) {
-        uint32_t r[16];
-        tmem_ld16(tmem + b * BN + (uint32_t(q * 32) << 16) + uint32_t(c), r);
-        if (m >= p.M) continue;
-        float v[16];
+      if (CW % 32 == 0) {
+        for (int c = half * CW; c < (half + 1) * CW; c += 32) {
+          uint32_t r[32];
+          tmem_ld32(tmem + b * BN + (uint32_t(q * 32) << 16) + uint32_t(c), r);
+          if (m >= p.M) continue;
 #pragma unroll
-        for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
-        store16(p, m, n0 + c, v);
+          for (int h = 0; h < 2; ++h) {
+            float v[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[16 * h + j]);
+            store16(p, m, n0 + c + 16 * h, v);
+          }
+        }
+      } else {
+        for (int c = half * CW; c < (half + 1) * CW; c += 16) {
+          uint32_t r[16];
+          tmem_ld16(tmem + b * BN + (uint32_t(q * 32) << 16) + uint32_t(c), r);
+          if (m >= p.M) continue;
+          float v[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
+          store16(p, m, n0 + c, v);
+        }
       }
       tc_fence_before();
       mbar_arrive(&acc_empty[b]);
@@ -1159,7 +1197,7 @@ void tc_run(TcGemm* g, const void* input, cudaStream_t st) {
   if (g->input_A) g->p.tmA = g->slot_maps[c->slot];
   if (g->input_B) g->p.tmB = g->slot_maps[c->slot];
   if (g->splits == 1) {
-    g->fn<<<g->grid, kThreads, g->smem, st>>>(g->p);
+    g->fn<<<g->grid, kPersistThreads, g->smem, st>>>(g->p);
     return;
   }
   cudaLaunchConfig_t cfg = {};
