@@ -256,63 +256,6 @@ __device__ __forceinline__ void cluster_reduce_rows(const TcParams& p, uint32_t 
   }
 }
 
-// Epilogue of 16 consecutive outputs (m, n..n+15) in registers.
-__device__ __forceinline__ void store16(const TcParams& p, int m_gemm, int n, float (&v)[16]) {
-  const size_t m = out_row(p, m_gemm);
-  if (p.bias) {
-    const float4* b4 = reinterpret_cast<const float4*>(p.bias + n);
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float4 b = __ldg(b4 + j);
-      v[4 * j] += b.x; v[4 * j + 1] += b.y; v[4 * j + 2] += b.z; v[4 * j + 3] += b.w;
-    }
-  }
-  if (p.relu)
-#pragma unroll
-    for (int j = 0; j < 16; ++j) v[j] = fmaxf(v[j], 0.f);
-  if (p.mask) {
-    const uint4* mk = reinterpret_cast<const uint4*>(p.mask + m * p.ldo + n);
-#pragma unroll
-    for (int j = 0; j < 2; ++j) {
-      const uint4 u = mk[j];
-      const bf16* e = reinterpret_cast<const bf16*>(&u);
-#pragma unroll
-      for (int q = 0; q < 8; ++q)
-        if (!(__bfloat162float(e[q]) > 0.f)) v[8 * j + q] = 0.f;
-    }
-  }
-  if (p.out_f32) {
-    float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + m * p.ldo + n);
-    if (p.acc)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const float4 o = dst[j];
-        v[4 * j] += o.x; v[4 * j + 1] += o.y; v[4 * j + 2] += o.z; v[4 * j + 3] += o.w;
-      }
-#pragma unroll
-    for (int j = 0; j < 4; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-  } else {
-    uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(p.out) + m * p.ldo + n);
-    if (p.acc)
-#pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        const uint4 o = dst[j];
-        const bf16* e = reinterpret_cast<const bf16*>(&o);
-#pragma unroll
-        for (int q = 0; q < 8; ++q) v[8 * j + q] += __bfloat162float(e[q]);
-      }
-    uint4 pk[2];
-    uint32_t* pw = reinterpret_cast<uint32_t*>(pk);
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      __nv_bfloat162 h2 = __floats2bfloat162_rn(v[2 * j], v[2 * j + 1]);
-      pw[j] = *reinterpret_cast<uint32_t*>(&h2);
-    }
-    dst[0] = pk[0];
-    dst[1] = pk[1];
-  }
-}
-
 // 32 consecutive TMEM columns of this thread's lane, one wait.
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile(
@@ -324,6 +267,113 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
         "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
       : "r"(taddr));
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Coalesced epilogue of a 32-row x 32-column accumulator chunk held one row
+// per lane (lane = row, r[j] = column j).  The warp stages the chunk in its
+// 4 KB shared-memory buffer (16-byte units XOR-swizzled by row, so both the
+// row-wise writes and the column-wise reads are free of bank conflicts), then
+// reads it back so that consecutive lanes own consecutive columns of a row:
+// bias, ReLU, ReLU mask, accumulate and the stores then touch whole 32-byte
+// sectors (bf16: 8 rows x 64 B per instruction; fp32: 4 rows x 128 B).
+// Explicit shared-space accesses: generic ones would be ordered behind the
+// warp's outstanding global stores.
+__device__ __forceinline__ void st_shared4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
+}
+__device__ __forceinline__ float4 ld_shared4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr)
+               : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void epilogue_chunk32(const TcParams& p, uint32_t stage, int lane, int m_base, int n,
+                                                 const uint32_t (&r)[32]) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j)
+    st_shared4(stage + 16u * (lane * 8 + (j ^ (lane & 7))), r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
+  __syncwarp();
+  if (p.out_f32) {
+    const int cq = lane & 7;                 // 16-byte unit: columns 4cq .. 4cq+3
+    float4 b = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (p.bias) b = __ldg(reinterpret_cast<const float4*>(p.bias + n) + cq);
+#pragma unroll 1
+    for (int it = 0; it < 8; ++it) {
+      const int rr = it * 4 + (lane >> 3);
+      const int mg = m_base + rr;
+      const float4 v = ld_shared4(stage + 16u * (rr * 8 + (cq ^ (rr & 7))));
+      if (mg < p.M) {
+        const size_t m = out_row(p, mg);
+        float e[4] = {v.x + b.x, v.y + b.y, v.z + b.z, v.w + b.w};
+        if (p.relu)
+#pragma unroll
+          for (int q = 0; q < 4; ++q) e[q] = fmaxf(e[q], 0.f);
+        if (p.mask) {
+          const uint2 u = *reinterpret_cast<const uint2*>(p.mask + m * p.ldo + n + 4 * cq);
+          const bf16* mk = reinterpret_cast<const bf16*>(&u);
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            if (!(__bfloat162float(mk[q]) > 0.f)) e[q] = 0.f;
+        }
+        float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + m * p.ldo + n) + cq;
+        if (p.acc) {
+          const float4 o = *dst;
+          e[0] += o.x; e[1] += o.y; e[2] += o.z; e[3] += o.w;
+        }
+        *dst = make_float4(e[0], e[1], e[2], e[3]);
+      }
+    }
+  } else {
+    const int co = lane & 3;                 // columns 8co .. 8co+7
+    float b[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) b[q] = 0.f;
+    if (p.bias) {
+      const float4 b0 = __ldg(reinterpret_cast<const float4*>(p.bias + n) + 2 * co);
+      const float4 b1 = __ldg(reinterpret_cast<const float4*>(p.bias + n) + 2 * co + 1);
+      b[0] = b0.x; b[1] = b0.y; b[2] = b0.z; b[3] = b0.w; b[4] = b1.x; b[5] = b1.y; b[6] = b1.z; b[7] = b1.w;
+    }
+#pragma unroll 1
+    for (int it = 0; it < 4; ++it) {
+      const int rr = it * 8 + (lane >> 2);
+      const int mg = m_base + rr;
+      const float4 v0 = ld_shared4(stage + 16u * (rr * 8 + ((2 * co) ^ (rr & 7))));
+      const float4 v1 = ld_shared4(stage + 16u * (rr * 8 + ((2 * co + 1) ^ (rr & 7))));
+      if (mg < p.M) {
+        const size_t m = out_row(p, mg);
+        float e[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+#pragma unroll
+        for (int q = 0; q < 8; ++q) e[q] += b[q];
+        if (p.relu)
+#pragma unroll
+          for (int q = 0; q < 8; ++q) e[q] = fmaxf(e[q], 0.f);
+        if (p.mask) {
+          const uint4 u = *reinterpret_cast<const uint4*>(p.mask + m * p.ldo + n + 8 * co);
+          const bf16* mk = reinterpret_cast<const bf16*>(&u);
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            if (!(__bfloat162float(mk[q]) > 0.f)) e[q] = 0.f;
+        }
+        uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(p.out) + m * p.ldo + n + 8 * co);
+        if (p.acc) {
+          const uint4 o = *dst;
+          const bf16* eo = reinterpret_cast<const bf16*>(&o);
+#pragma unroll
+          for (int q = 0; q < 8; ++q) e[q] += __bfloat162float(eo[q]);
+        }
+        uint4 pk;
+        uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          __nv_bfloat162 h2 = __floats2bfloat162_rn(e[2 * q], e[2 * q + 1]);
+          pw[q] = *reinterpret_cast<uint32_t*>(&h2);
+        }
+        *dst = pk;
+      }
+    }
+  }
+  __syncwarp();
 }
 
 template <int KIND>
@@ -584,6 +634,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 // overlaps the MMAs of the next.  Barriers: full/empty per stage (TMA <->
 // MMA), acc_full/acc_empty per accumulator (MMA <-> epilogue).
 constexpr int kPersistThreads = 320;  // TMA warp, MMA warp, 8 epilogue warps
+constexpr int kEpiStageBytes = 8 * 4096;  // one 32 x 32 fp32 staging buffer per epilogue warp
 
 template <int KIND, int BN, int STAGES>
 __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const __grid_constant__ TcParams p) {
@@ -592,7 +643,9 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
   constexpr int A_BYTES = BM * BK * 2;
   constexpr int B_BYTES = BN * BK * 2;
   constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  static_assert(STAGES * STAGE_BYTES + kEpiStageBytes + 1024 + 256 <= 232448, "shared memory per CTA");
+  float4* stage_all = reinterpret_cast<float4*>(smem + STAGES * STAGE_BYTES);   // 8 x 4 KB epilogue staging
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + kEpiStageBytes);
   uint64_t* empty = full + STAGES;
   uint64_t* acc_full = empty + STAGES;
   uint64_t* acc_empty = acc_full + 2;
@@ -696,8 +749,7 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
     // Epilogue: warp w (2..9) reads TMEM lanes 32 * (w % 4) .. +31; the two
     // warps of a lane quarter split the tile's columns.
     const int q = warp % 4, half = (warp - 2) / 4;
-    const int row = q * 32 + lane;
-    constexpr int CW = BN / 2;  // columns per epilogue warp
+    constexpr int CW = BN / 2;  // columns per epilogue warp (a multiple of 32)
     uint32_t lt = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++lt) {
       const uint32_t b = lt & 1;
@@ -709,30 +761,14 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
         *abort_flag = 1;
       }
       if (!ready || *abort_flag) break;
-      const int m = m0 + row;
-      if (CW % 32 == 0) {
-        for (int c = half * CW; c < (half + 1) * CW; c += 32) {
-          uint32_t r[32];
-          tmem_ld32(tmem + b * BN + (uint32_t(q * 32) << 16) + uint32_t(c), r);
-          if (m >= p.M) continue;
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            float v[16];
-#pragma unroll
-            for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[16 * h + j]);
-            store16(p, m, n0 + c + 16 * h, v);
-          }
-        }
-      } else {
-        for (int c = half * CW; c < (half + 1) * CW; c += 16) {
-          uint32_t r[16];
-          tmem_ld16(tmem + b * BN + (uint32_t(q * 32) << 16) + uint32_t(c), r);
-          if (m >= p.M) continue;
-          float v[16];
-#pragma unroll
-          for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
-          store16(p, m, n0 + c, v);
-        }
+      const uint32_t stage = smem_u32(stage_all) + uint32_t(warp - 2) * 4096u;
+      // Not unrolled: the epilogue runs once per tile from a cold instruction
+      // cache, so compact code matters more than loop overhead.
+#pragma unroll 1
+      for (int c = half * CW; c < (half + 1) * CW; c += 32) {
+        uint32_t r[32];
+        tmem_ld32(tmem + b * BN + (uint32_t(q * 32) << 16) + uint32_t(c), r);
+        epilogue_chunk32(p, stage, lane, m0 + q * 32, n0 + c, r);
       }
       tc_fence_before();
       mbar_arrive(&acc_empty[b]);
@@ -751,8 +787,8 @@ constexpr int stages_for() {
   return kSmemBudget / (BM * BK * 2 + BN * BK * 2) > 8 ? 8 : kSmemBudget / (BM * BK * 2 + BN * BK * 2);
 }
 template <int KIND, int BN>
-constexpr size_t smem_bytes() {
-  return size_t(stages_for<KIND, BN>()) * (BM * BK * 2 + BN * BK * 2) + 1024 + 256;
+constexpr size_t smem_bytes(bool cluster) {
+  return size_t(stages_for<KIND, BN>()) * (BM * BK * 2 + BN * BK * 2) + 1024 + 256 + (cluster ? 0 : kEpiStageBytes);
 }
 
 typedef void (*KernelFn)(const TcParams);
@@ -766,9 +802,9 @@ KernelFn kernel_ptr(bool cluster) {
 KernelFn pick_kernel(int kind, int bn, bool cluster, size_t* smem) {
 #define FO_PICK(K)                                                  \
   if (kind == K) {                                                  \
-    if (bn == 256) { *smem = smem_bytes<K, 256>(); return kernel_ptr<K, 256>(cluster); } \
-    if (bn == 128) { *smem = smem_bytes<K, 128>(); return kernel_ptr<K, 128>(cluster); } \
-    *smem = smem_bytes<K, 64>();                                    \
+    if (bn == 256) { *smem = smem_bytes<K, 256>(cluster); return kernel_ptr<K, 256>(cluster); } \
+    if (bn == 128) { *smem = smem_bytes<K, 128>(cluster); return kernel_ptr<K, 128>(cluster); } \
+    *smem = smem_bytes<K, 64>(cluster);                                    \
     return kernel_ptr<K, 64>(cluster);                              \
   }
   FO_PICK(LIN_FWD)
