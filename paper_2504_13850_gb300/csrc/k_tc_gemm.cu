@@ -23,6 +23,7 @@
 #include <cuda.h>
 #include <algorithm>
 #include <cstring>
+#include <map>
 #include <vector>
 
 namespace fo {
@@ -55,6 +56,9 @@ struct TcParams {
   // row (n*oH + ostride*i + py)*oW + ostride*j + px of `out` (identity when
   // ostride == 0)
   int ostride, py, px, Hq, Wq, oH, oW;
+  // paired CTAs: the window operand is loaded as two halves, the second at
+  // these row / image offsets (in the windowed tensor's coordinates)
+  int half_dh, half_dn;
   // epilogue
   void* out;
   int ldo;
@@ -116,6 +120,21 @@ __device__ __forceinline__ void tma_4d(void* dst, const CUtensorMap* m, uint64_t
       "l"(reinterpret_cast<uint64_t>(m)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
       : "memory");
 }
+// Multicast variant: the box lands at the same shared-memory offset in every
+// CTA of `mask` and completes bytes on the mbarrier at the same offset there.
+__device__ __forceinline__ void tma_4d_mc(void* dst, const CUtensorMap* m, uint64_t* bar, int c0, int c1, int c2,
+                                          int c3, uint16_t mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster [%0], "
+      "[%1, {%3, %4, %5, %6}], [%2], %7;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(m)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "h"(mask)
+      : "memory");
+}
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
@@ -146,6 +165,15 @@ __device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t a, uint64_t b,
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                : "memory");
+}
+// Arrive on the mbarrier at this offset in every CTA of `mask` once the
+// issuing thread's earlier MMAs are complete.
+__device__ __forceinline__ void mma_commit_mc(uint64_t* bar, uint16_t mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+          smem_u32(bar)),
+      "h"(mask)
+      : "memory");
 }
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
   asm volatile(
@@ -224,34 +252,40 @@ __device__ __forceinline__ void store4(const TcParams& p, int m_gemm, int n, flo
 
 // Sum of the S partial tiles at G elements per batch, all S*G remote loads
 // issued before the adds (fixed order over z).
-template <int BN, int S, int G>
-__device__ __forceinline__ void cluster_reduce_rows(const TcParams& p, uint32_t base, int r0, int r1, int m0,
+template <int BN>
+__device__ __forceinline__ void cluster_reduce_rows(const TcParams& p, uint32_t base, int S, int r0, int r1, int m0,
                                                     int n0, int t) {
-  constexpr int n4 = BN / 4;
+  // Rows r0..r1-1 of the tile summed over the S partials in rank order
+  // (deterministic).  Four float4 elements per thread per pass keep four
+  // remote loads in flight; the loops stay rolled to keep the code small.
+  constexpr int n4 = BN / 4, G = 4;
   const int total = (r1 - r0) * n4;
+#pragma unroll 1
   for (int e0 = t; e0 < total; e0 += 128 * G) {
-    float4 v[G][S];
+    uint32_t off[G];
+    float4 acc[G];
 #pragma unroll
     for (int g = 0; g < G; ++g) {
-      const int e = e0 + g * 128;
-      const int row = r0 + (e < total ? e : 0) / n4, c = ((e < total ? e : 0) % n4) * 4;
-      const uint32_t off = base + uint32_t((row * (BN + 4) + c) * 4);
+      const int e = min(e0 + g * 128, total - 1);
+      off[g] = base + uint32_t(((r0 + e / n4) * (BN + 4) + (e % n4) * 4) * 4);
+      acc[g] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll 1
+    for (int z = 0; z < S; ++z) {
+      float4 v[G];
 #pragma unroll
-      for (int z = 0; z < S; ++z) v[g][z] = ld_cluster_f4(map_to_cta(off, uint32_t(z)));
+      for (int g = 0; g < G; ++g) v[g] = ld_cluster_f4(map_to_cta(off[g], uint32_t(z)));
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        acc[g].x += v[g].x; acc[g].y += v[g].y; acc[g].z += v[g].z; acc[g].w += v[g].w;
+      }
     }
 #pragma unroll
     for (int g = 0; g < G; ++g) {
       const int e = e0 + g * 128;
       if (e >= total) continue;
-      const int row = r0 + e / n4, c = (e % n4) * 4;
-      const int m = m0 + row;
-      if (m >= p.M) continue;
-      float4 acc = v[g][0];
-#pragma unroll
-      for (int z = 1; z < S; ++z) {
-        acc.x += v[g][z].x; acc.y += v[g][z].y; acc.z += v[g][z].z; acc.w += v[g][z].w;
-      }
-      store4(p, m, n0 + c, acc);
+      const int m = m0 + r0 + e / n4;
+      if (m < p.M) store4(p, m, n0 + (e % n4) * 4, acc[g]);
     }
   }
 }
@@ -288,16 +322,31 @@ __device__ __forceinline__ float4 ld_shared4(uint32_t addr) {
   return v;
 }
 
+// The bias values lane `lane` applies in epilogue_chunk32 for the chunk at
+// column n: 8 columns from 8 * (lane % 4) for bf16 outputs, 4 columns from
+// 4 * (lane % 8) for fp32 outputs (zeros without a bias).
+__device__ __forceinline__ void load_bias8(const TcParams& p, int lane, int n, float (&b)[8]) {
+  float4 b0 = make_float4(0.f, 0.f, 0.f, 0.f), b1 = b0;
+  if (p.bias) {
+    const float4* src = reinterpret_cast<const float4*>(p.bias + n);
+    if (p.out_f32) {
+      b0 = __ldg(src + (lane & 7));
+    } else {
+      b0 = __ldg(src + 2 * (lane & 3));
+      b1 = __ldg(src + 2 * (lane & 3) + 1);
+    }
+  }
+  b[0] = b0.x; b[1] = b0.y; b[2] = b0.z; b[3] = b0.w; b[4] = b1.x; b[5] = b1.y; b[6] = b1.z; b[7] = b1.w;
+}
+
 __device__ __forceinline__ void epilogue_chunk32(const TcParams& p, uint32_t stage, int lane, int m_base, int n,
-                                                 const uint32_t (&r)[32]) {
+                                                 const uint32_t (&r)[32], const float (&b)[8]) {
 #pragma unroll
   for (int j = 0; j < 8; ++j)
     st_shared4(stage + 16u * (lane * 8 + (j ^ (lane & 7))), r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
   __syncwarp();
   if (p.out_f32) {
     const int cq = lane & 7;                 // 16-byte unit: columns 4cq .. 4cq+3
-    float4 b = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (p.bias) b = __ldg(reinterpret_cast<const float4*>(p.bias + n) + cq);
 #pragma unroll 1
     for (int it = 0; it < 8; ++it) {
       const int rr = it * 4 + (lane >> 3);
@@ -305,7 +354,7 @@ __device__ __forceinline__ void epilogue_chunk32(const TcParams& p, uint32_t sta
       const float4 v = ld_shared4(stage + 16u * (rr * 8 + (cq ^ (rr & 7))));
       if (mg < p.M) {
         const size_t m = out_row(p, mg);
-        float e[4] = {v.x + b.x, v.y + b.y, v.z + b.z, v.w + b.w};
+        float e[4] = {v.x + b[0], v.y + b[1], v.z + b[2], v.w + b[3]};
         if (p.relu)
 #pragma unroll
           for (int q = 0; q < 4; ++q) e[q] = fmaxf(e[q], 0.f);
@@ -326,14 +375,6 @@ __device__ __forceinline__ void epilogue_chunk32(const TcParams& p, uint32_t sta
     }
   } else {
     const int co = lane & 3;                 // columns 8co .. 8co+7
-    float b[8];
-#pragma unroll
-    for (int q = 0; q < 8; ++q) b[q] = 0.f;
-    if (p.bias) {
-      const float4 b0 = __ldg(reinterpret_cast<const float4*>(p.bias + n) + 2 * co);
-      const float4 b1 = __ldg(reinterpret_cast<const float4*>(p.bias + n) + 2 * co + 1);
-      b[0] = b0.x; b[1] = b0.y; b[2] = b0.z; b[3] = b0.w; b[4] = b1.x; b[5] = b1.y; b[6] = b1.z; b[7] = b1.w;
-    }
 #pragma unroll 1
     for (int it = 0; it < 4; ++it) {
       const int rr = it * 8 + (lane >> 2);
@@ -383,9 +424,12 @@ struct KindTraits {
 };
 
 // Issue the TMA loads of k-block `kb` for output tile (m0, n0).
-template <int KIND, int BN>
+// PAIR 1: the two CTAs of a cluster share m0 and each loads half of the
+// window operand A for both (multicast); PAIR 2: they share n0 and split the
+// window boxes of B.  `rank` is the CTA's rank in its cluster.
+template <int KIND, int BN, int PAIR = 0>
 __device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, int n0, char* sa, char* sb,
-                                            uint64_t* bar) {
+                                            uint64_t* bar, uint32_t rank = 0) {
   const int HW = p.H * p.W;
   if (KIND == LIN_FWD || KIND == LIN_DGRAD) {
     tma_2d(sa, &p.tmA, bar, kb * BK, m0);
@@ -396,11 +440,19 @@ __device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, i
     const int tap = kb / p.cblocks, c0 = (kb % p.cblocks) * 64;
     const int r = tap / p.ksz, s = tap % p.ksz;
     const int n_img = m0 / HW, h0 = (m0 % HW) / p.W;   // H, W: output grid
-    tma_4d(sa, &p.tmA, bar, c0, s - p.pad, h0 * p.stride + r - p.pad, n_img);
+    if (PAIR == 1)
+      tma_4d_mc(sa + rank * (BM * BK), &p.tmA, bar, c0, s - p.pad,
+                h0 * p.stride + r - p.pad + int(rank) * p.half_dh, n_img + int(rank) * p.half_dn, 0x3);
+    else
+      tma_4d(sa, &p.tmA, bar, c0, s - p.pad, h0 * p.stride + r - p.pad, n_img);
   } else {  // CONV_DGRAD: window over the output gradient, shifted per tap
     const int t = kb / p.cblocks, c0 = (kb % p.cblocks) * 64;
     const int n_img = m0 / HW, h0 = (m0 % HW) / p.W;   // H, W: the class grid (= gradient grid)
-    tma_4d(sa, &p.tmA, bar, c0, p.tap_dw[t], h0 + p.tap_dh[t], n_img);
+    if (PAIR == 1)
+      tma_4d_mc(sa + rank * (BM * BK), &p.tmA, bar, c0, p.tap_dw[t], h0 + p.tap_dh[t] + int(rank) * p.half_dh,
+                n_img + int(rank) * p.half_dn, 0x3);
+    else
+      tma_4d(sa, &p.tmA, bar, c0, p.tap_dw[t], h0 + p.tap_dh[t], n_img);
   }
   if (KIND == LIN_FWD) {
     tma_2d(sb, &p.tmB, bar, kb * BK, n0);
@@ -421,8 +473,14 @@ __device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, i
     const int pix0 = kb * BK;
     const int n_img = pix0 / HW, h0 = (pix0 % HW) / p.W;   // H, W: output grid
 #pragma unroll
-    for (int j = 0; j < BN / 64; ++j)
-      tma_4d(sb + j * BK * 128, &p.tmB, bar, ci0 + j * 64, s - p.pad, h0 * p.stride + r - p.pad, n_img);
+    for (int j = 0; j < BN / 64; ++j) {
+      if (PAIR == 2) {
+        if ((j & 1) == int(rank))
+          tma_4d_mc(sb + j * BK * 128, &p.tmB, bar, ci0 + j * 64, s - p.pad, h0 * p.stride + r - p.pad, n_img, 0x3);
+      } else {
+        tma_4d(sb + j * BK * 128, &p.tmB, bar, ci0 + j * 64, s - p.pad, h0 * p.stride + r - p.pad, n_img);
+      }
+    }
   }
 }
 
@@ -608,14 +666,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
       const int r0 = rank * BM / S, r1 = (rank + 1) * BM / S;
       const int t = threadIdx.x - 64;
       const uint32_t base = smem_u32(smem);
-      if (S == 2) cluster_reduce_rows<BN, 2, 8>(p, base, r0, r1, m0, n0, t);
-      else if (S == 3) cluster_reduce_rows<BN, 3, 4>(p, base, r0, r1, m0, n0, t);
-      else if (S == 4) cluster_reduce_rows<BN, 4, 4>(p, base, r0, r1, m0, n0, t);
-      else if (S <= 6) {
-        if (S == 5) cluster_reduce_rows<BN, 5, 2>(p, base, r0, r1, m0, n0, t);
-        else cluster_reduce_rows<BN, 6, 2>(p, base, r0, r1, m0, n0, t);
-      } else if (S == 7) cluster_reduce_rows<BN, 7, 2>(p, base, r0, r1, m0, n0, t);
-      else cluster_reduce_rows<BN, 8, 2>(p, base, r0, r1, m0, n0, t);
+      cluster_reduce_rows<BN>(p, base, S, r0, r1, m0, n0, t);
     }
     cluster_sync_all();
   }
@@ -636,7 +687,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 constexpr int kPersistThreads = 320;  // TMA warp, MMA warp, 8 epilogue warps
 constexpr int kEpiStageBytes = 8 * 4096;  // one 32 x 32 fp32 staging buffer per epilogue warp
 
-template <int KIND, int BN, int STAGES>
+// PAIR != 0: launched as clusters of two CTAs that run the same k-block
+// sequence on two adjacent tiles and split the TMA loads of the operand they
+// share (1: A, tiles side by side in N; 2: B, tiles stacked in M), each
+// multicasting its half to both.  A stage is then refilled only when both
+// CTAs' MMAs have released it (empty barriers count two arrivals).
+template <int KIND, int BN, int STAGES, int PAIR>
 __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const __grid_constant__ TcParams p) {
   extern __shared__ __align__(1024) char smem_raw[];
   char* smem = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -653,15 +709,21 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int n_tiles = p.N / BN;
-  const int tiles = n_tiles * ((p.M + BM - 1) / BM);
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
+  const int unit = PAIR ? int(blockIdx.x) / 2 : int(blockIdx.x);
+  const int units = PAIR ? int(gridDim.x) / 2 : int(gridDim.x);
+  const int n_tiles = p.N / BN, m_tiles = (p.M + BM - 1) / BM;
+  const int su_n = PAIR == 1 ? n_tiles / 2 : n_tiles;   // work units: tiles, or tile pairs
+  const int tiles = su_n * (PAIR == 2 ? m_tiles / 2 : m_tiles);
   const int KB = p.KB;
   constexpr uint32_t kCols = 2 * BN < 32 ? 32 : 2 * BN;
+  auto tile_n0 = [&](int t) { return (PAIR == 1 ? 2 * (t % su_n) + int(rank) : t % su_n) * BN; };
+  auto tile_m0 = [&](int t) { return (PAIR == 2 ? 2 * (t / su_n) + int(rank) : t / su_n) * BM; };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], PAIR ? 2 : 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
@@ -680,14 +742,15 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
   }
   tc_fence_before();
   __syncthreads();
+  if (PAIR) cluster_sync_all();   // the peer's barriers are initialised
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
     if (lane == 0) {
       uint32_t g = 0;
-      for (int t = blockIdx.x; t < tiles && !*abort_flag; t += gridDim.x) {
-        const int n0 = (t % n_tiles) * BN, m0 = (t / n_tiles) * BM;
+      for (int t = unit; t < tiles && !*abort_flag; t += units) {
+        const int n0 = tile_n0(t), m0 = tile_m0(t);
         for (int kb = 0; kb < KB; ++kb, ++g) {
           const int s = g % STAGES;
           if (!mbar_wait(&empty[s], ((g / STAGES) & 1) ^ 1)) {
@@ -697,7 +760,18 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
           }
           char* sa = smem + s * STAGE_BYTES;
           mbar_expect_tx(&full[s], STAGE_BYTES);
-          load_kblock<KIND, BN>(p, kb, m0, n0, sa, sa + A_BYTES, &full[s]);
+          load_kblock<KIND, BN, PAIR>(p, kb, m0, n0, sa, sa + A_BYTES, &full[s], rank);
+        }
+      }
+      if (PAIR) {
+        // Drain: every stage released by both CTAs, so no arrival from the
+        // peer is still on its way when the cluster exits.
+        for (int i = 0; i < STAGES; ++i, ++g) {
+          const int s = g % STAGES;
+          if (!mbar_wait(&empty[s], ((g / STAGES) & 1) ^ 1)) {
+            atomicExch(p.err, 8);
+            break;
+          }
         }
       }
     }
@@ -705,7 +779,7 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
     if (lane == 0) {
       constexpr uint32_t idesc = instr_desc(BN, KindTraits<KIND>::a_mn, KindTraits<KIND>::b_mn);
       uint32_t g = 0, lt = 0;
-      for (int t = blockIdx.x; t < tiles && !*abort_flag; t += gridDim.x, ++lt) {
+      for (int t = unit; t < tiles && !*abort_flag; t += units, ++lt) {
         const uint32_t b = lt & 1;
         if (!mbar_wait(&acc_empty[b], ((lt >> 1) & 1) ^ 1)) {
           atomicExch(p.err, 5);
@@ -736,7 +810,8 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
             else bd = smem_desc(b0 + k * UK * 2, 16, 1024);
             mma_f16(d, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
           }
-          mma_commit(&empty[s]);
+          if (PAIR) mma_commit_mc(&empty[s], 0x3);
+          else mma_commit(&empty[s]);
         }
         if (ok) mma_commit(&acc_full[b]);
         else {
@@ -751,9 +826,11 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
     const int q = warp % 4, half = (warp - 2) / 4;
     constexpr int CW = BN / 2;  // columns per epilogue warp (a multiple of 32)
     uint32_t lt = 0;
-    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++lt) {
+    for (int t = unit; t < tiles; t += units, ++lt) {
       const uint32_t b = lt & 1;
-      const int n0 = (t % n_tiles) * BN, m0 = (t / n_tiles) * BM;
+      const int n0 = tile_n0(t), m0 = tile_m0(t);
+      float bnext[8];
+      load_bias8(p, lane, n0 + half * CW, bnext);   // in flight during the wait
       const bool ready = mbar_wait(&acc_full[b], (lt >> 1) & 1);
       tc_fence_after();
       if (!ready) {
@@ -766,9 +843,13 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
       // cache, so compact code matters more than loop overhead.
 #pragma unroll 1
       for (int c = half * CW; c < (half + 1) * CW; c += 32) {
+        float bcur[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) bcur[j] = bnext[j];
+        if (c + 32 < (half + 1) * CW) load_bias8(p, lane, n0 + c + 32, bnext);
         uint32_t r[32];
         tmem_ld32(tmem + b * BN + (uint32_t(q * 32) << 16) + uint32_t(c), r);
-        epilogue_chunk32(p, stage, lane, m0 + q * 32, n0 + c, r);
+        epilogue_chunk32(p, stage, lane, m0 + q * 32, n0 + c, r, bcur);
       }
       tc_fence_before();
       mbar_arrive(&acc_empty[b]);
@@ -776,6 +857,7 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
   }
   tc_fence_before();
   __syncthreads();
+  if (PAIR) cluster_sync_all();
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kCols) : "memory");
@@ -794,18 +876,26 @@ constexpr size_t smem_bytes(bool cluster) {
 typedef void (*KernelFn)(const TcParams);
 
 template <int KIND, int BN>
-KernelFn kernel_ptr(bool cluster) {
-  if (cluster) return tc_gemm_kernel<KIND, BN, stages_for<KIND, BN>(), true>;
-  return tc_gemm_persistent<KIND, BN, stages_for<KIND, BN>()>;
+KernelFn kernel_ptr(bool cluster, int pair) {
+  constexpr int S = stages_for<KIND, BN>();
+  if (cluster) return pair ? nullptr : tc_gemm_kernel<KIND, BN, S, true>;
+  if constexpr ((KIND == CONV_FPROP || KIND == CONV_DGRAD) && BN >= 128) {
+    if (pair == 1) return tc_gemm_persistent<KIND, BN, S, 1>;
+  }
+  if constexpr (KIND == CONV_WGRAD && BN >= 128) {
+    if (pair == 2) return tc_gemm_persistent<KIND, BN, S, 2>;
+  }
+  if (pair) return nullptr;
+  return tc_gemm_persistent<KIND, BN, S, 0>;
 }
 
-KernelFn pick_kernel(int kind, int bn, bool cluster, size_t* smem) {
+KernelFn pick_kernel(int kind, int bn, bool cluster, int pair, size_t* smem) {
 #define FO_PICK(K)                                                  \
   if (kind == K) {                                                  \
-    if (bn == 256) { *smem = smem_bytes<K, 256>(cluster); return kernel_ptr<K, 256>(cluster); } \
-    if (bn == 128) { *smem = smem_bytes<K, 128>(cluster); return kernel_ptr<K, 128>(cluster); } \
+    if (bn == 256) { *smem = smem_bytes<K, 256>(cluster); return kernel_ptr<K, 256>(cluster, pair); } \
+    if (bn == 128) { *smem = smem_bytes<K, 128>(cluster); return kernel_ptr<K, 128>(cluster, pair); } \
     *smem = smem_bytes<K, 64>(cluster);                                    \
-    return kernel_ptr<K, 64>(cluster);                              \
+    return kernel_ptr<K, 64>(cluster, pair);                         \
   }
   FO_PICK(LIN_FWD)
   FO_PICK(LIN_DGRAD)
@@ -885,6 +975,7 @@ struct TcGemm {
   TcGemm() : p{} { p.stride = 1; }
   const char* name = nullptr;
   int kind = 0, bn = 0, splits = 1;
+  int pair = 0;            // 0, or the operand a CTA pair shares (1: A, 2: B)
   double flops = 0;
   TcParams p;
   KernelFn fn = nullptr;
@@ -898,6 +989,7 @@ struct TcGemm {
 
 struct TcContext {
   std::vector<TcGemm*> gemms;
+  std::map<int, int> cluster_fit;   // active_clusters() cache
   int num_sms = 148;
   int slot = 0;
   int* err = nullptr;
@@ -926,37 +1018,96 @@ bool window_ok(int N, int H, int W, int rows_needed, int* rows, int* imgs) {
 }
 
 
-// Tile width and K split from a small cost model.  One CTA per SM; a tile
-// costs its k-blocks (a 128-wide k-block runs at ~0.55 of a 256-wide one)
-// plus its epilogue.  Unsplit plans run persistent (epilogue overlapped,
-// paid once); a K split runs as clusters of <= 8 CTAs (portable size) that
-// pay the epilogue and the cluster reduction per CTA, and clusters above 4
-// pay for their poorer packing into GPCs.  Minimises the estimated time.
+// Clusters that fit on the GPU at once (GPC packing), from the occupancy
+// calculator; cached per context.  pair == 0: split-K clusters of S CTAs of
+// kernel (kind, bn); pair != 0: two-CTA clusters of the persistent kernel.
+int active_clusters(TcContext* c, int kind, int bn, int S, int pair) {
+  const int key = ((kind * 512 + bn) * 16 + S) * 4 + pair;
+  auto it = c->cluster_fit.find(key);
+  if (it != c->cluster_fit.end()) return it->second;
+  size_t smem = 0;
+  KernelFn fn = pick_kernel(kind, bn, pair == 0, pair, &smem);
+  int n = 0;
+  if (fn && cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem)) == cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = pair ? dim3(2, 1, 1) : dim3(1, 1, S);
+    cfg.blockDim = dim3(pair ? kPersistThreads : kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = pair ? 2 : 1;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = pair ? 1 : S;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess) n = 0;
+  }
+  cudaGetLastError();
+  if (n <= 0) {   // conservative fallback
+    const int size = pair ? 2 : S;
+    n = c->num_sms / (2 * size) > 0 ? c->num_sms / (2 * size) : 1;
+  }
+  c->cluster_fit[key] = n;
+  return n;
+}
+
+// Tile width, K split and CTA pairing from a cost model in microseconds,
+// fitted to GB300 timelines of these kernels:
+//  * a k-block stage costs at least ~0.37 us: each stage is one round of
+//    mbarrier waits (full on the MMA side, empty on the TMA side), whose
+//    dependent latency is a few hundred cycles on each side;
+//  * the TMA fills one SM's shared memory at ~128 GB/s, which bounds stages
+//    of 256-wide tiles (48 KB);
+//  * weight-gradient windows arrive as 64-row 4-D boxes costing ~0.21 us
+//    each, so a 256-wide tile (four boxes) is slow unless a CTA pair splits
+//    them;
+//  * a CTA pays a start-up ramp and the epilogue of its last tile (earlier
+//    epilogues overlap the next tile's MMAs), a K-split cluster pays the
+//    staging and distributed-shared-memory reduction of its partial tiles,
+//    and clusters run in waves of what the occupancy calculator fits at once.
 // Candidate widths divide `ndiv` (N, or the channels of one tap for the
-// weight gradient, whose N index runs over taps x channels).
-void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv) {
+// weight gradient, whose N index runs over taps x channels).  `pair_ok`: the
+// planner can split the shared operand's box in two.
+void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv, bool pair_ok) {
+  const bool win_a = g->kind == CONV_FPROP || g->kind == CONV_DGRAD;
+  const bool win_b = g->kind == CONV_WGRAD;
   double best = 1e30;
-  int best_bn = 0, best_s = 1;
+  int best_bn = 0, best_s = 1, best_pair = 0;
   for (int bn : {256, 128, 64}) {
     if (ndiv % bn || N % bn) continue;
-    const int tiles = ((M + BM - 1) / BM) * (N / bn);
-    const double per_kb = bn == 256 ? 1.0 : (bn == 128 ? 0.55 : 0.4);
-    const double epi = bn / 64.0;
-    for (int sp = 1; sp <= 8; ++sp) {
-      if (sp > 1 && KB / sp < 4) break;
-      const int kper = (KB + sp - 1) / sp;
-      const int splits = (KB + kper - 1) / kper;
-      if (splits != sp) continue;
-      const int ctas = tiles * splits;
-      const double waves = double((ctas + c->num_sms - 1) / c->num_sms);
-      // unsplit plans run persistent: epilogues overlap the next tile's MMAs
-      double cost = splits == 1 ? waves * kper * per_kb + epi
-                                : waves * (kper * per_kb + epi + 2.0);
-      if (splits > 4) cost *= 1.2;
-      if (cost < best - 1e-9) {
-        best = cost;
-        best_bn = bn;
-        best_s = splits;
+    const int n_tiles = N / bn, m_tiles = (M + BM - 1) / BM, tiles = n_tiles * m_tiles;
+    const double stage_kb = (BM + bn) * BK * 2 / 1024.0;
+    const double epi = bn == 256 ? 4.2 : (bn == 128 ? 2.2 : 1.5);
+    for (int pair = 0; pair <= 2; ++pair) {
+      if (pair == 1 && !(pair_ok && win_a && bn >= 128 && n_tiles % 2 == 0)) continue;
+      if (pair == 2 && !(pair_ok && win_b && bn >= 128 && m_tiles % 2 == 0)) continue;
+      double t_kb = std::max(0.37, stage_kb / 128.0);
+      if (win_b) t_kb = std::max(t_kb + 0.05, 0.215 * (bn / 64) / (pair ? 2 : 1));
+      if (!win_a && !win_b) t_kb = std::max(0.31, stage_kb / 128.0);
+      for (int sp = 1; sp <= (pair ? 1 : 8); ++sp) {
+        if (sp > 1 && KB / sp < 4) break;
+        const int kper = (KB + sp - 1) / sp;
+        const int splits = (KB + kper - 1) / kper;
+        if (splits != sp) continue;
+        double cost;
+        if (splits == 1) {
+          const int work = pair ? tiles / 2 : tiles;
+          const int units = std::min(work, pair ? active_clusters(c, g->kind, bn, 2, pair) : c->num_sms);
+          const int per_unit = (work + units - 1) / units;
+          const double main = kper * t_kb;
+          cost = (pair ? 2.2 : 1.7) + per_unit * main + epi + (pair ? 0.7 : 0.0) +
+                 (per_unit - 1) * std::max(0.0, epi - main);
+        } else {
+          const int fit = active_clusters(c, g->kind, bn, splits, 0);
+          const int waves = (tiles + fit - 1) / fit;
+          cost = waves * (1.0 + kper * t_kb + 3.0 + 2.5 * bn / 128.0);
+        }
+        if (cost < best - 1e-9) {
+          best = cost;
+          best_bn = bn;
+          best_s = splits;
+          best_pair = pair;
+        }
       }
     }
   }
@@ -964,6 +1115,7 @@ void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv) {
   g->p.KB = KB;
   g->p.kper = (KB + best_s - 1) / best_s;
   g->splits = best_s;
+  g->pair = best_pair;
 }
 
 TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
@@ -971,7 +1123,7 @@ TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
   g->p.N = N;
   g->flops = 2.0 * M * N * K;
   g->p.err = c->err;
-  g->fn = pick_kernel(g->kind, g->bn, g->splits > 1, &g->smem);
+  g->fn = pick_kernel(g->kind, g->bn, g->splits > 1, g->pair, &g->smem);
   if (!g->fn) {
     delete g;
     return nullptr;
@@ -982,13 +1134,16 @@ TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
   }
   if (g->splits > 1) {
     g->grid = dim3(N / g->bn, (M + BM - 1) / BM, g->splits);
+  } else if (g->pair) {
+    const int work = (N / g->bn) * ((M + BM - 1) / BM) / 2;
+    g->grid = dim3(2 * std::min(work, active_clusters(c, g->kind, g->bn, 2, g->pair)), 1, 1);
   } else {
     const int tiles = (N / g->bn) * ((M + BM - 1) / BM);
     g->grid = dim3(std::min(tiles, c->num_sms), 1, 1);
   }
   if (getenv("FO_DEBUG_PLAN"))
-    fprintf(stderr, "[plan] %-16s M=%d N=%d KB=%d BN=%d splits=%d grid=(%u,%u,%u)\n", g->name, M, N, g->p.KB,
-            g->bn, g->splits, g->grid.x, g->grid.y, g->grid.z);
+    fprintf(stderr, "[plan] %-16s M=%d N=%d KB=%d BN=%d splits=%d pair=%d grid=(%u,%u,%u)\n", g->name, M, N,
+            g->p.KB, g->bn, g->splits, g->pair, g->grid.x, g->grid.y, g->grid.z);
   g->ctx = c;
   c->gemms.push_back(g);
   return g;
@@ -1051,7 +1206,7 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i, void* out, bool relu)
     g->kind = LIN_FWD;
     g->name = "tc_linear_fwd";
     int M = int(a.rows()), KB = op.cin / 64;
-    choose_tiles(c, g, M, op.cout, KB, op.cout);
+    choose_tiles(c, g, M, op.cout, KB, op.cout, false);
     const int bn = g->bn;
     g->input_A = (op.in0 == 0);
     if (g->input_A) {
@@ -1074,14 +1229,20 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i, void* out, bool relu)
   g->p.ntap_ch = op.cin;
   g->p.win_rows = rows; g->p.win_imgs = imgs;
   int M = a.N * Ho * Wo, KB = g->p.taps * g->p.cblocks;
-  choose_tiles(c, g, M, op.cout, KB, op.cout);
+  choose_tiles(c, g, M, op.cout, KB, op.cout, imgs > 1 ? imgs % 2 == 0 : rows % 2 == 0);
   const int bn = g->bn;
+  // paired CTAs each fetch half of the window: half the images, else half the rows
+  int box_rows = rows, box_imgs = imgs;
+  if (g->pair == 1) {
+    if (imgs > 1) { box_imgs = imgs / 2; g->p.half_dn = box_imgs; }
+    else { box_rows = rows / 2; g->p.half_dh = box_rows * st; }
+  }
   g->input_A = (op.in0 == 0);
   if (g->input_A) {
     g->slot_maps.resize(s->cfg.omega);
     for (int sl = 0; sl < s->cfg.omega; ++sl)
-      if (!map_window(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, a.N, a.H, a.W, a.C, Wo, rows, imgs, st)) { delete g; return nullptr; }
-  } else if (!map_window(&g->p.tmA, tensor_act(s, op.in0), a.N, a.H, a.W, a.C, Wo, rows, imgs, st)) { delete g; return nullptr; }
+      if (!map_window(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, a.N, a.H, a.W, a.C, Wo, box_rows, box_imgs, st)) { delete g; return nullptr; }
+  } else if (!map_window(&g->p.tmA, tensor_act(s, op.in0), a.N, a.H, a.W, a.C, Wo, box_rows, box_imgs, st)) { delete g; return nullptr; }
   if (!map_2d(&g->p.tmB, w, op.cout, int64_t(g->p.taps) * op.cin, bn)) { delete g; return nullptr; }
   return finish(c, g, M, op.cout, double(g->p.taps) * op.cin);
 }
@@ -1110,7 +1271,7 @@ bool tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate, void* dx, 
     g->kind = LIN_DGRAD;
     g->name = "tc_linear_dgrad";
     int M = int(a.rows()), KB = op.cout / 64;
-    choose_tiles(c, g, M, op.cin, KB, op.cin);
+    choose_tiles(c, g, M, op.cin, KB, op.cin, false);
     if (!map_2d(&g->p.tmA, o.grad, M, op.cout, BM) || !map_2d(&g->p.tmB, w, op.cout, op.cin, BK)) { delete g; return false; }
     if (!finish(c, g, M, op.cin, double(op.cout))) return false;
     out->push_back(g);
@@ -1163,8 +1324,13 @@ bool tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate, void* dx, 
       g->p.Hq = Ho; g->p.Wq = Wo; g->p.oH = a.H; g->p.oW = a.W;
     }
     const int M = o.N * Ho * Wo, KB = cls[q].n * g->p.cblocks;
-    choose_tiles(c, g, M, op.cin, KB, op.cin);
-    if (!map_window(&g->p.tmA, o.grad, o.N, Ho, Wo, o.C, Wo, rows, imgs) ||
+    choose_tiles(c, g, M, op.cin, KB, op.cin, imgs > 1 ? imgs % 2 == 0 : rows % 2 == 0);
+    int box_rows = rows, box_imgs = imgs;
+    if (g->pair == 1) {
+      if (imgs > 1) { box_imgs = imgs / 2; g->p.half_dn = box_imgs; }
+      else { box_rows = rows / 2; g->p.half_dh = box_rows; }
+    }
+    if (!map_window(&g->p.tmA, o.grad, o.N, Ho, Wo, o.C, Wo, box_rows, box_imgs) ||
         !map_2d(&g->p.tmB, w, op.cout, int64_t(g->p.taps) * op.cin, BK)) {
       delete g;
       for (TcGemm* x : *out) (void)x;
@@ -1195,7 +1361,7 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
     g->name = "tc_linear_wgrad";
     g->p.ldo = op.cin;
     int rows = int(a.rows()), KB = (rows + BK - 1) / BK;
-    choose_tiles(c, g, op.cout, op.cin, KB, op.cin);
+    choose_tiles(c, g, op.cout, op.cin, KB, op.cin, false);
     g->input_B = (op.in0 == 0);
     if (!map_2d(&g->p.tmA, o.grad, rows, op.cout, BK)) { delete g; return nullptr; }
     if (g->input_B) {
@@ -1216,7 +1382,7 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
   g->p.ntap_ch = op.cin;
   int P = a.N * Ho * Wo, KB = P / BK;
   int N = g->p.taps * op.cin;
-  choose_tiles(c, g, op.cout, N, KB, op.cin);
+  choose_tiles(c, g, op.cout, N, KB, op.cin, true);
   g->input_B = (op.in0 == 0);
   if (!map_2d(&g->p.tmA, o.grad, P, op.cout, BK)) { delete g; return nullptr; }
   if (g->input_B) {
@@ -1232,8 +1398,24 @@ void tc_run(TcGemm* g, const void* input, cudaStream_t st) {
   TcContext* c = g->ctx;
   if (g->input_A) g->p.tmA = g->slot_maps[c->slot];
   if (g->input_B) g->p.tmB = g->slot_maps[c->slot];
-  if (g->splits == 1) {
+  if (g->splits == 1 && !g->pair) {
     g->fn<<<g->grid, kPersistThreads, g->smem, st>>>(g->p);
+    return;
+  }
+  if (g->pair) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = g->grid;
+    cfg.blockDim = dim3(kPersistThreads);
+    cfg.dynamicSmemBytes = g->smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaLaunchKernelEx(&cfg, g->fn, g->p);
     return;
   }
   cudaLaunchConfig_t cfg = {};
