@@ -223,6 +223,8 @@ int build_plan(fo_server* s) {
   const double esz = dt == fo::kF32 ? 4.0 : 2.0;
   auto& plan = s->plan;
   plan.clear();
+  for (fo::AttnTcPlan* a : s->attn_tc) fo::attention_tc_destroy(a);
+  s->attn_tc.assign(nops, nullptr);
   const Fusion fu = analyse(s);
   auto act = [s](int tid) -> const void* { return tid == 0 ? s->cur_in : s->T[tid].act; };
   auto add = [&plan](const char* name, int kernels, double flops, double bytes,
@@ -319,6 +321,17 @@ int build_plan(fo_server* s) {
         break;
       case FO_OP_ATTENTION: {
         const double Ls = ta.H, heads = op.heads, dh = double(op.cin) / op.heads;
+        fo::AttnTcPlan* tp = nullptr;
+        if (s->tc && dt == fo::kBF16 && a != 0 && !getenv("FO_NO_TC") && fo::attention_tc_ok(ta.H, op.cin, op.heads))
+          tp = fo::attention_tc_plan(s->T[a].act, s->T[o].act, s->T[o].grad, ta.N, ta.H, op.cin, op.heads,
+                                     fo::tc_error_word(s->tc));
+        s->attn_tc[i] = tp;
+        if (tp) {
+          add("tc_attention_fwd", 1, 4.0 * ta.N * heads * Ls * Ls * dh, tbytes(a) + tbytes(o), [=](cudaStream_t st) {
+            fo::attention_tc_fwd(tp, s->cur_len, s->T[o].act, s->attn_probs[i], s->T[a].N, st);
+          });
+          break;
+        }
         add("attention_fwd", 1, 4.0 * ta.N * heads * Ls * Ls * dh, tbytes(a) + tbytes(o), [=](cudaStream_t st) {
           const Tensor& x = s->T[a];
           fo::attention_fwd(act(a), s->cur_len, s->T[o].act, s->attn_probs[i], x.N, x.H, op.cin, op.heads, dt, st);
@@ -546,6 +559,13 @@ int build_plan(fo_server* s) {
           int accf = contrib(a);
           const Tensor& ta = s->T[a];
           const double Ls = ta.H, heads = op.heads, dh = double(op.cin) / op.heads;
+          if (fo::AttnTcPlan* tp = s->attn_tc[i]) {
+            add("tc_attention_bwd", 1, 10.0 * ta.N * heads * Ls * Ls * dh, (2 + accf) * tbytes(a) + 2 * csb,
+                [=](cudaStream_t st) {
+                  fo::attention_tc_bwd(tp, s->cur_len, s->attn_probs[i], s->T[a].grad, s->T[a].N, accf != 0, st);
+                });
+            break;
+          }
           add("attention_bwd", 1, 8.0 * ta.N * heads * Ls * Ls * dh, (2 + accf) * tbytes(a) + 2 * csb,
               [=](cudaStream_t st) {
                 const Tensor& x = s->T[a];
@@ -660,6 +680,8 @@ int allocate(fo_server* s) {
 void destroy_impl(fo_server* s) {
   if (!s) return;
   if (s->cs) cudaStreamSynchronize(s->cs);
+  for (fo::AttnTcPlan* a : s->attn_tc) fo::attention_tc_destroy(a);
+  s->attn_tc.clear();
   if (s->xs) cudaStreamSynchronize(s->xs);
   for (auto g : s->graphs) if (g) cudaGraphExecDestroy(g);
   for (auto g : s->prof_graphs) if (g) cudaGraphExecDestroy(g);

@@ -13,6 +13,7 @@
 
 namespace fo {
 struct TcContext;
+struct AttnTcPlan;
 }
 
 struct ParamSeg {
@@ -106,6 +107,7 @@ struct fo_server {
 
   std::vector<void*> allocs;
   fo::TcContext* tc = nullptr;
+  std::vector<fo::AttnTcPlan*> attn_tc;   // per op: tensor-core attention plan, or null
 
   void* alloc(size_t bytes) {
     void* p = nullptr;

@@ -3,6 +3,7 @@
 // shapes the tensor-core kernels do not take; the caller then uses the
 // CUDA-core kernels.
 #pragma once
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <vector>
@@ -40,5 +41,22 @@ const char* tc_name(const TcGemm* g);
 int tc_finalize(TcContext* c);
 // Device word the tensor-core kernels set on a timed-out wait (0 = none).
 int* tc_error_word(TcContext* c);
+// Tensor map of a row-major bf16 matrix [rows][cols] with 128-byte-swizzled
+// boxes of 64 columns x box_rows rows.
+bool tc_encode_2d(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int box_rows);
+
+// Tensor-core attention (k_attention_tc.cu): sequences of at most 128 tokens,
+// head width 64, bf16.  A plan holds the tensor maps of the packed q|k|v
+// input [B*L, 3C], the output O [B*L, C] and its gradient dO [B*L, C].
+struct AttnTcPlan;
+bool attention_tc_ok(int L, int C, int heads);
+AttnTcPlan* attention_tc_plan(const void* qkv, const void* out, const void* dout, int B, int L, int C, int heads,
+                              int* err);
+void attention_tc_destroy(AttnTcPlan* a);
+// O and the per-row log-sum-exp of the scaled scores (lse: [B * heads * L]).
+void attention_tc_fwd(const AttnTcPlan* a, const int32_t* len, void* out, float* lse, int B, cudaStream_t st);
+// d(q|k|v) [B*L, 3C] from dO, the saved lse and the forward output.
+void attention_tc_bwd(const AttnTcPlan* a, const int32_t* len, const float* lse, void* dqkv, int B, bool acc,
+                      cudaStream_t st);
 
 }  // namespace fo
