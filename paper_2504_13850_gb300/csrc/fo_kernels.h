@@ -1,5 +1,6 @@
 // Host launchers of the library's CUDA kernels (internal interface).
 #pragma once
+#include <vector>
 #include <cuda_runtime.h>
 #include <cstdint>
 
@@ -115,12 +116,42 @@ void colsum8(const void* a, int64_t rows, int C, float* partial, float* out, boo
 // (dx may be null); partial holds 2 * colsum8_partial_floats(rows, C, true) floats.
 void affine_bwd8(const void* dy, const void* x, const float* scale, void* dx, bool acc, int64_t rows, int C,
                  float* partial, float* dscale, float* dshift, cudaStream_t st);
+// Deferred parameter-gradient reductions, batched into one launch each (at
+// most a few dozen launches' worth of work per call; fixed summation order).
+// ColsumTask: column sums of a bf16 [rows, C] matrix (C % 8 == 0) into
+// `partial` ([colsum8_batch_chunks(rows), C] floats).  FinishTask: out[c] =
+// sum over the `chunks` rows of partial [chunks, C].
+struct ColsumTask {
+  const void* a;
+  float* partial;
+  int64_t rows;
+  int C;
+};
+struct FinishTask {
+  const float* partial;
+  float* out;
+  int chunks;
+  int C;
+};
+int colsum8_batch_chunks(int64_t rows);
+void colsum8_batched(const std::vector<ColsumTask>& tasks, cudaStream_t st);
+void finish_batched(const std::vector<FinishTask>& tasks, cudaStream_t st);
+// Affine backward pass without its finish: partials of dscale and dshift
+// ([affine_bwd8_chunks(rows, C), C] each) and dx (+)= dy * scale.
+int affine_bwd8_chunks(int64_t rows, int C);
+void affine_bwd8_pass(const void* dy, const void* x, const float* scale, void* dx, bool acc, int64_t rows, int C,
+                      float* p_scale, float* p_shift, cudaStream_t st);
 // Layernorm backward fused with dgamma / dbeta (C % 256 == 0, C <= 512).
 bool layernorm_bwd8_ok(int dt, int C);
 int64_t layernorm_bwd8_partial_floats(int64_t rows, int C);
 void layernorm_bwd8(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
                     void* dx, int64_t rows, int C, bool acc, float* partial, float* dgamma, float* dbeta,
                     cudaStream_t st);
+// The same pass without its finish: partials [layernorm_bwd8_blocks(rows), C]
+// of dgamma and dbeta.
+int layernorm_bwd8_blocks(int64_t rows);
+void layernorm_bwd8_pass(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
+                         void* dx, int64_t rows, int C, bool acc, float* p_gamma, float* p_beta, cudaStream_t st);
 
 // FedAsync update: g = fmaf(alpha, l - g, g).
 void axpby(float* g, const float* l, int64_t n, float alpha, cudaStream_t st);

@@ -367,6 +367,12 @@ int build_plan(fo_server* s) {
     written[r] = 1;
     return accf;
   };
+  // Parameter-gradient reductions deferred to two batched launches after the
+  // backward pass: column sums for the conv / linear biases, and the finish
+  // of the affine / layernorm partials.  Each has its own partial buffer.
+  std::vector<fo::ColsumTask> bias_tasks;
+  std::vector<fo::FinishTask> finish_tasks;
+  double deferred_bytes = 0.0;
   for (int i = nops - 1; i >= 0; --i) {
     const fo_op op = s->ops[i];
     if (fu.skip_bwd[i]) {
@@ -415,7 +421,15 @@ int build_plan(fo_server* s) {
         const int dto = s->T[o].dt, dta = s->T[a].dt;
         const bool bias = op.bias != 0;
         const double fl = 2.0 * double(s->T[o].rows()) * op.cout * double(op.kind == FO_OP_CONV ? op.k * op.k : 1) * op.cin;
-        if (bias) {
+        if (bias && dto == fo::kBF16 && s->T[o].C % 8 == 0) {
+          const Tensor& t = s->T[o];
+          const int chunks = fo::colsum8_batch_chunks(t.rows());
+          float* part = (float*)s->alloc(size_t(chunks) * t.C * 4);
+          if (!part) return set_err(FO_ERR_OOM, "bias-gradient partials");
+          bias_tasks.push_back({t.grad, part, t.rows(), t.C});
+          finish_tasks.push_back({part, G(s, i, 1), chunks, t.C});
+          deferred_bytes += double(t.bytes());
+        } else if (bias) {
           add("bias_grad", 2, 0.0, double(s->T[o].bytes()), [=](cudaStream_t st) {
             fo::colsum(s->T[o].grad, nullptr, s->T[o].rows(), s->T[o].C, dto, s->colsum_scratch, G(s, i, 1), st,
                        true);
@@ -456,10 +470,17 @@ int build_plan(fo_server* s) {
         if (fo::vec8_ok(dt, s->T[a0].numel()) && s->T[a0].C % 8 == 0) {
           // one pass: dscale, dshift and dx (+)= dy * scale
           const int accf = need_dx ? contrib(a) : 0;
-          add("affine_bwd", 4, 0.0, (need_dx ? 3 + accf : 2) * csb, [=](cudaStream_t st) {
+          const Tensor& x0 = s->T[a0];
+          const int chunks = fo::affine_bwd8_chunks(x0.rows(), x0.C);
+          float* ps = (float*)s->alloc(size_t(2) * chunks * x0.C * 4);
+          if (!ps) return set_err(FO_ERR_OOM, "affine partials");
+          float* ph = ps + size_t(chunks) * x0.C;
+          finish_tasks.push_back({ps, G(s, i, 0), chunks, x0.C});
+          finish_tasks.push_back({ph, G(s, i, 1), chunks, x0.C});
+          add("affine_bwd", 1, 0.0, (need_dx ? 3 + accf : 2) * csb, [=](cudaStream_t st) {
             const Tensor& x = s->T[a0];
-            fo::affine_bwd8(s->T[o].grad, act(a0), P(s, i, 0), need_dx ? s->T[a].grad : nullptr, accf != 0,
-                            x.rows(), x.C, s->colsum_scratch, G(s, i, 0), G(s, i, 1), st);
+            fo::affine_bwd8_pass(s->T[o].grad, act(a0), P(s, i, 0), need_dx ? s->T[a].grad : nullptr, accf != 0,
+                                 x.rows(), x.C, ps, ph, st);
           });
           break;
         }
@@ -523,11 +544,17 @@ int build_plan(fo_server* s) {
       case FO_OP_LAYERNORM:
         if (fo::layernorm_bwd8_ok(dt, s->T[a0].C)) {
           const int accf = need_dx ? contrib(a) : 0;
-          add("layernorm_bwd", 3, 0.0, (need_dx ? 3 + accf : 2) * csb, [=](cudaStream_t st) {
+          const Tensor& x0 = s->T[a0];
+          const int blocks = fo::layernorm_bwd8_blocks(x0.rows());
+          float* pg = (float*)s->alloc(size_t(2) * blocks * x0.C * 4);
+          if (!pg) return set_err(FO_ERR_OOM, "layernorm partials");
+          float* pb = pg + size_t(blocks) * x0.C;
+          finish_tasks.push_back({pg, G(s, i, 0), blocks, x0.C});
+          finish_tasks.push_back({pb, G(s, i, 1), blocks, x0.C});
+          add("layernorm_bwd", 1, 0.0, (need_dx ? 3 + accf : 2) * csb, [=](cudaStream_t st) {
             const Tensor& x = s->T[a0];
-            fo::layernorm_bwd8(act(a0), P(s, i, 0), s->ln_mean[i], s->ln_rstd[i], s->T[o].grad,
-                               need_dx ? s->T[a].grad : nullptr, x.rows(), x.C, accf != 0, s->colsum_scratch,
-                               G(s, i, 0), G(s, i, 1), st);
+            fo::layernorm_bwd8_pass(act(a0), P(s, i, 0), s->ln_mean[i], s->ln_rstd[i], s->T[o].grad,
+                                    need_dx ? s->T[a].grad : nullptr, x.rows(), x.C, accf != 0, pg, pb, st);
           });
           break;
         }
@@ -587,6 +614,17 @@ int build_plan(fo_server* s) {
   }
 
   // ---------------- optimizer (Algorithm 4: theta_s <- theta_s - gamma_s * update)
+  if (!bias_tasks.empty())
+    add("bias_grad", int((bias_tasks.size() + 39) / 40), 0.0, deferred_bytes, [=](cudaStream_t st) {
+      fo::colsum8_batched(bias_tasks, st);
+    });
+  if (!finish_tasks.empty()) {
+    double fb = 0.0;
+    for (const fo::FinishTask& t : finish_tasks) fb += 4.0 * double(t.chunks + 1) * t.C;
+    add("param_grad_finish", int((finish_tasks.size() + 39) / 40), 0.0, fb, [=](cudaStream_t st) {
+      fo::finish_batched(finish_tasks, st);
+    });
+  }
   add("sgd_momentum", 1, 0.0, double(s->n_padded) * (20.0 + (s->shadow ? 2.0 : 0.0)), [=](cudaStream_t st) {
     fo::sgd_momentum(s->theta, s->mom, s->grad, s->shadow, s->n_padded, s->opt.lr, s->opt.momentum, s->d_step, st);
   });

@@ -7,6 +7,9 @@
 #include "fo_common.cuh"
 #include "fo_kernels.h"
 
+#include <algorithm>
+#include <vector>
+
 namespace fo {
 
 namespace {
@@ -129,15 +132,15 @@ __global__ void gelu_bwd_x8_k(const bf16* __restrict__ x, const bf16* __restrict
 // are combined in shared memory in a fixed order.  MODE 0: sums of a;
 // MODE 1: affine backward (sums of dy * x and dy, and dx (+)= dy * scale).
 template <int MODE>
-__global__ void __launch_bounds__(256) colsum8_k(const bf16* __restrict__ a, const bf16* __restrict__ x,
-                                                 const float* __restrict__ scale, bf16* __restrict__ dx, int acc,
-                                                 int64_t rows, int C, int chunk, float* __restrict__ p0,
-                                                 float* __restrict__ p1) {
+__device__ __forceinline__ void colsum8_block(const bf16* __restrict__ a, const bf16* __restrict__ x,
+                                              const float* __restrict__ scale, bf16* __restrict__ dx, int acc,
+                                              int64_t rows, int C, int chunk, float* __restrict__ p0,
+                                              float* __restrict__ p1, int cb, int ck) {
   __shared__ float red0[8][257];
   __shared__ float red1[MODE == 1 ? 8 : 1][257];
   const int g = threadIdx.x % 32, r = threadIdx.x / 32;
-  const int c = blockIdx.x * 256 + 8 * g;
-  const int64_t r0 = int64_t(blockIdx.y) * chunk;
+  const int c = cb * 256 + 8 * g;
+  const int64_t r0 = int64_t(ck) * chunk;
   float s0[8] = {0, 0, 0, 0, 0, 0, 0, 0}, s1[8] = {0, 0, 0, 0, 0, 0, 0, 0};
   if (c < C) {
     float sc[8];
@@ -176,7 +179,7 @@ __global__ void __launch_bounds__(256) colsum8_k(const bf16* __restrict__ a, con
     if (MODE == 1) red1[r][8 * g + j] = s1[j];
   }
   __syncthreads();
-  const int cc = blockIdx.x * 256 + threadIdx.x;
+  const int cc = cb * 256 + threadIdx.x;
   if (cc < C) {
     float t0 = 0.f, t1 = 0.f;
 #pragma unroll
@@ -184,9 +187,52 @@ __global__ void __launch_bounds__(256) colsum8_k(const bf16* __restrict__ a, con
       t0 += red0[q][threadIdx.x];
       if (MODE == 1) t1 += red1[q][threadIdx.x];
     }
-    p0[int64_t(blockIdx.y) * C + cc] = t0;
-    if (MODE == 1) p1[int64_t(blockIdx.y) * C + cc] = t1;
+    p0[int64_t(ck) * C + cc] = t0;
+    if (MODE == 1) p1[int64_t(ck) * C + cc] = t1;
   }
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(256) colsum8_k(const bf16* __restrict__ a, const bf16* __restrict__ x,
+                                                 const float* __restrict__ scale, bf16* __restrict__ dx, int acc,
+                                                 int64_t rows, int C, int chunk, float* __restrict__ p0,
+                                                 float* __restrict__ p1) {
+  colsum8_block<MODE>(a, x, scale, dx, acc, rows, C, chunk, p0, p1, blockIdx.x, blockIdx.y);
+}
+
+// Several column sums in one launch: block b belongs to the task t with
+// block0[t] <= b < block0[t + 1] and covers (column block, row chunk) of it.
+constexpr int kMaxBatch = 40;
+struct ColsumBatch {
+  int n;
+  int block0[kMaxBatch + 1];
+  const bf16* a[kMaxBatch];
+  float* partial[kMaxBatch];
+  int64_t rows[kMaxBatch];
+  int C[kMaxBatch];
+  int chunk[kMaxBatch];
+};
+struct FinishBatch {
+  int n;
+  int block0[kMaxBatch + 1];
+  const float* partial[kMaxBatch];
+  float* out[kMaxBatch];
+  int chunks[kMaxBatch];
+  int C[kMaxBatch];
+};
+
+__device__ __forceinline__ int batch_task(const int* block0, int n, int b) {
+  int t = 0;
+  while (t + 1 < n && block0[t + 1] <= b) ++t;
+  return t;
+}
+
+__global__ void __launch_bounds__(256) colsum8_batch_k(const __grid_constant__ ColsumBatch p) {
+  const int t = batch_task(p.block0, p.n, blockIdx.x);
+  const int local = blockIdx.x - p.block0[t];
+  const int cbs = (p.C[t] + 255) / 256;
+  colsum8_block<0>(p.a[t], nullptr, nullptr, nullptr, 0, p.rows[t], p.C[t], p.chunk[t], p.partial[t], nullptr,
+                   local % cbs, local / cbs);
 }
 
 // Layernorm backward fused with its parameter gradients: one warp per row
@@ -308,6 +354,39 @@ __global__ void finish_k(const float* __restrict__ partial, int chunks, int C, f
   }
 }
 
+// Batched finish: block b covers 32 columns of task t (same fixed summation
+// order as finish_k).
+__global__ void __launch_bounds__(256) finish_batch_k(const __grid_constant__ FinishBatch p) {
+  const int t = batch_task(p.block0, p.n, blockIdx.x);
+  const int local = blockIdx.x - p.block0[t];
+  __shared__ float red[8][33];
+  const int cl = threadIdx.x % 32, rl = threadIdx.x / 32;
+  const int C = p.C[t], chunks = p.chunks[t];
+  const float* partial = p.partial[t];
+  const int c = local * 32 + cl;
+  float s = 0.f;
+  if (c < C) {
+    int q = rl;
+    for (; q + 24 < chunks; q += 32) {
+      const float a0 = partial[int64_t(q) * C + c], a1 = partial[int64_t(q + 8) * C + c];
+      const float a2 = partial[int64_t(q + 16) * C + c], a3 = partial[int64_t(q + 24) * C + c];
+      s += a0;
+      s += a1;
+      s += a2;
+      s += a3;
+    }
+    for (; q < chunks; q += 8) s += partial[int64_t(q) * C + c];
+  }
+  red[rl][cl] = s;
+  __syncthreads();
+  if (rl == 0 && c < C) {
+    float tot = 0.f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) tot += red[q][cl];
+    p.out[t][c] = tot;
+  }
+}
+
 int chunks_of(int64_t rows, int chunk) { return int((rows + chunk - 1) / chunk); }
 
 // Rows per chunk for the server's column sums: about two blocks per SM,
@@ -374,7 +453,67 @@ void affine_bwd8(const void* dy, const void* x, const float* scale, void* dx, bo
   finish_k<<<ceil_div(C, 32), 256, 0, st>>>(p1, chunks_of(rows, ch), C, dshift);
 }
 
+int affine_bwd8_chunks(int64_t rows, int C) { return chunks_of(rows, adaptive_chunk(rows, C)); }
+
+void affine_bwd8_pass(const void* dy, const void* x, const float* scale, void* dx, bool acc, int64_t rows, int C,
+                      float* p_scale, float* p_shift, cudaStream_t st) {
+  const int ch = adaptive_chunk(rows, C);
+  dim3 grid(ceil_div(C, 256), chunks_of(rows, ch));
+  colsum8_k<1><<<grid, 256, 0, st>>>((const bf16*)dy, (const bf16*)x, scale, (bf16*)dx, acc, rows, C, ch, p_scale,
+                                     p_shift);
+}
+
+int colsum8_batch_chunks(int64_t rows) { return chunks_of(rows, kChunk); }
+
+void colsum8_batched(const std::vector<ColsumTask>& tasks, cudaStream_t st) {
+  for (size_t t0 = 0; t0 < tasks.size(); t0 += kMaxBatch) {
+    ColsumBatch p{};
+    p.n = int(std::min(tasks.size() - t0, size_t(kMaxBatch)));
+    int blocks = 0;
+    for (int k = 0; k < p.n; ++k) {
+      const ColsumTask& t = tasks[t0 + k];
+      p.block0[k] = blocks;
+      p.a[k] = static_cast<const bf16*>(t.a);
+      p.partial[k] = t.partial;
+      p.rows[k] = t.rows;
+      p.C[k] = t.C;
+      p.chunk[k] = kChunk;
+      blocks += ceil_div(t.C, 256) * chunks_of(t.rows, kChunk);
+    }
+    p.block0[p.n] = blocks;
+    if (blocks) colsum8_batch_k<<<blocks, 256, 0, st>>>(p);
+  }
+}
+
+void finish_batched(const std::vector<FinishTask>& tasks, cudaStream_t st) {
+  for (size_t t0 = 0; t0 < tasks.size(); t0 += kMaxBatch) {
+    FinishBatch p{};
+    p.n = int(std::min(tasks.size() - t0, size_t(kMaxBatch)));
+    int blocks = 0;
+    for (int k = 0; k < p.n; ++k) {
+      const FinishTask& t = tasks[t0 + k];
+      p.block0[k] = blocks;
+      p.partial[k] = t.partial;
+      p.out[k] = t.out;
+      p.chunks[k] = t.chunks;
+      p.C[k] = t.C;
+      blocks += ceil_div(t.C, 32);
+    }
+    p.block0[p.n] = blocks;
+    if (blocks) finish_batch_k<<<blocks, 256, 0, st>>>(p);
+  }
+}
+
 bool layernorm_bwd8_ok(int dt, int C) { return dt == kBF16 && C % 256 == 0 && C <= 512; }
+
+int layernorm_bwd8_blocks(int64_t rows) { return int((rows + 15) / 16); }
+
+void layernorm_bwd8_pass(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
+                         void* dx, int64_t rows, int C, bool acc, float* p_gamma, float* p_beta, cudaStream_t st) {
+  layernorm_bwd_fused_k<<<layernorm_bwd8_blocks(rows), 256, 0, st>>>((const bf16*)x, gamma, mean, rstd,
+                                                                      (const bf16*)dy, (bf16*)dx, rows, C, acc,
+                                                                      p_gamma, p_beta);
+}
 
 int64_t layernorm_bwd8_partial_floats(int64_t rows, int C) { return 2 * ((rows + 15) / 16) * C; }
 
