@@ -171,5 +171,34 @@ __device__ __forceinline__ float4 ld_shared4(uint32_t addr) {
 }
 
 
+// Plain 16-byte store into another CTA's shared memory (shared::cluster
+// address from mapa).
+__device__ __forceinline__ void st_cluster4(uint32_t remote_addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.shared::cluster.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(remote_addr), "r"(a), "r"(b), "r"(c), "r"(d)
+               : "memory");
+}
+// Arrive on another CTA's mbarrier, releasing this thread's earlier writes at
+// cluster scope.
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t remote_bar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote_bar) : "memory");
+}
+// Wait (bounded, ~2 s) for a phase whose arrivals came from other CTAs of the
+// cluster: acquire at cluster scope.
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity) {
+  const uint64_t t0 = global_ns();
+  while (true) {
+    for (int i = 0; i < 64; ++i) {
+      uint32_t ok;
+      asm volatile(
+          "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+          : "=r"(ok)
+          : "r"(smem_u32(bar)), "r"(parity)
+          : "memory");
+      if (ok) return true;
+    }
+    if (global_ns() - t0 > 2000000000ull) return false;
+  }
+}
+
 }  // namespace
 }  // namespace fo

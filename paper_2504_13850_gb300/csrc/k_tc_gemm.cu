@@ -76,87 +76,63 @@ __device__ __forceinline__ size_t out_row(const TcParams& p, int m) {
   return (size_t(n) * p.oH + p.ostride * i + p.py) * p.oW + p.ostride * j + p.px;
 }
 
-// Epilogue of 4 consecutive outputs (m, n..n+3): bias, ReLU, ReLU mask,
-// accumulate, store as fp32 or bf16.
-__device__ __forceinline__ void store4(const TcParams& p, int m_gemm, int n, float4 a) {
+// Epilogue of 32 consecutive outputs (m, n..n+31) held by one thread: bias,
+// ReLU, ReLU mask, accumulate, store as fp32 or bf16 (16-byte accesses).
+// `sbias`: shared-memory address of the bias values for columns n..n+31.
+__device__ __forceinline__ void store_row32(const TcParams& p, int m_gemm, int n, float (&v)[32], uint32_t sbias) {
   const size_t m = out_row(p, m_gemm);
-  float v[4] = {a.x, a.y, a.z, a.w};
-  if (p.bias)
+  if (p.bias) {
 #pragma unroll
-    for (int j = 0; j < 4; ++j) v[j] += p.bias[n + j];
+    for (int j = 0; j < 8; ++j) {
+      const float4 b = ld_shared4(sbias + 16u * j);
+      v[4 * j] += b.x; v[4 * j + 1] += b.y; v[4 * j + 2] += b.z; v[4 * j + 3] += b.w;
+    }
+  }
   if (p.relu)
 #pragma unroll
-    for (int j = 0; j < 4; ++j) v[j] = fmaxf(v[j], 0.f);
+    for (int j = 0; j < 32; ++j) v[j] = fmaxf(v[j], 0.f);
   if (p.mask) {
-    uint2 u = *reinterpret_cast<const uint2*>(p.mask + size_t(m) * p.ldo + n);
-    const bf16* e = reinterpret_cast<const bf16*>(&u);
+    const uint4* mk = reinterpret_cast<const uint4*>(p.mask + m * p.ldo + n);
 #pragma unroll
-    for (int j = 0; j < 4; ++j)
-      if (!(__bfloat162float(e[j]) > 0.f)) v[j] = 0.f;
+    for (int j = 0; j < 4; ++j) {
+      const uint4 u = mk[j];
+      const bf16* e = reinterpret_cast<const bf16*>(&u);
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        if (!(__bfloat162float(e[q]) > 0.f)) v[8 * j + q] = 0.f;
+    }
   }
   if (p.out_f32) {
-    float4* d = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + size_t(m) * p.ldo + n);
-    if (p.acc) {
-      float4 o = *d;
-      v[0] += o.x; v[1] += o.y; v[2] += o.z; v[3] += o.w;
-    }
-    *d = make_float4(v[0], v[1], v[2], v[3]);
-  } else {
-    uint2* d = reinterpret_cast<uint2*>(reinterpret_cast<bf16*>(p.out) + size_t(m) * p.ldo + n);
-    if (p.acc) {
-      uint2 o = *d;
-      const bf16* e = reinterpret_cast<const bf16*>(&o);
+    float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + m * p.ldo + n);
 #pragma unroll
-      for (int j = 0; j < 4; ++j) v[j] += __bfloat162float(e[j]);
-    }
-    __nv_bfloat162 lo = __floats2bfloat162_rn(v[0], v[1]), hi = __floats2bfloat162_rn(v[2], v[3]);
-    uint2 u;
-    u.x = *reinterpret_cast<uint32_t*>(&lo);
-    u.y = *reinterpret_cast<uint32_t*>(&hi);
-    *d = u;
-  }
-}
-
-// Sum of the S partial tiles at G elements per batch, all S*G remote loads
-// issued before the adds (fixed order over z).
-template <int BN>
-__device__ __forceinline__ void cluster_reduce_rows(const TcParams& p, uint32_t base, int S, int r0, int r1, int m0,
-                                                    int n0, int t) {
-  // Rows r0..r1-1 of the tile summed over the S partials in rank order
-  // (deterministic).  Four float4 elements per thread per pass keep four
-  // remote loads in flight; the loops stay rolled to keep the code small.
-  constexpr int n4 = BN / 4, G = 4;
-  const int total = (r1 - r0) * n4;
-#pragma unroll 1
-  for (int e0 = t; e0 < total; e0 += 128 * G) {
-    uint32_t off[G];
-    float4 acc[G];
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      const int e = min(e0 + g * 128, total - 1);
-      off[g] = base + uint32_t(((r0 + e / n4) * (BN + 4) + (e % n4) * 4) * 4);
-      acc[g] = make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-#pragma unroll 1
-    for (int z = 0; z < S; ++z) {
-      float4 v[G];
-#pragma unroll
-      for (int g = 0; g < G; ++g) v[g] = ld_cluster_f4(map_to_cta(off[g], uint32_t(z)));
-#pragma unroll
-      for (int g = 0; g < G; ++g) {
-        acc[g].x += v[g].x; acc[g].y += v[g].y; acc[g].z += v[g].z; acc[g].w += v[g].w;
+    for (int j = 0; j < 8; ++j) {
+      if (p.acc) {
+        const float4 o = dst[j];
+        v[4 * j] += o.x; v[4 * j + 1] += o.y; v[4 * j + 2] += o.z; v[4 * j + 3] += o.w;
       }
+      dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
     }
+  } else {
+    uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(p.out) + m * p.ldo + n);
 #pragma unroll
-    for (int g = 0; g < G; ++g) {
-      const int e = e0 + g * 128;
-      if (e >= total) continue;
-      const int m = m0 + r0 + e / n4;
-      if (m < p.M) store4(p, m, n0 + (e % n4) * 4, acc[g]);
+    for (int j = 0; j < 4; ++j) {
+      if (p.acc) {
+        const uint4 o = dst[j];
+        const bf16* ob = reinterpret_cast<const bf16*>(&o);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[8 * j + e] += __bfloat162float(ob[e]);
+      }
+      uint4 pk;
+      uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        __nv_bfloat162 h2 = __floats2bfloat162_rn(v[8 * j + 2 * e], v[8 * j + 2 * e + 1]);
+        pw[e] = *reinterpret_cast<uint32_t*>(&h2);
+      }
+      dst[j] = pk;
     }
   }
 }
-
 
 // Coalesced epilogue of a 32-row x 32-column accumulator chunk held one row
 // per lane (lane = row, r[j] = column j).  The warp stages the chunk in its
@@ -327,27 +303,38 @@ __device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, i
   }
 }
 
-// CLUSTER: the gridDim.z CTAs of a cluster split K; each stages its fp32
-// partial tile in shared memory and reduces a slice of rows over all the
-// cluster's partials (distributed shared memory, fixed order).
-template <int KIND, int BN, int STAGES, bool CLUSTER>
+// Split-K: the gridDim.z CTAs of a (1, 1, S) cluster each run k-blocks
+// [kb0, kb0 + kper) of the same output tile.  Rank z owns rows
+// [z*BM/S, (z+1)*BM/S) of the tile.  After the MMAs every CTA pushes the
+// accumulator rows it does not own straight from TMEM into the owner's
+// shared memory (distributed-shared-memory stores, one slot per source rank)
+// and arrives, with release semantics, on the owner's receive barrier (one
+// arrival per row); the owner then adds the S partials of its rows in rank
+// order (deterministic) and runs the epilogue.
+template <int KIND, int BN, int STAGES>
 __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ TcParams p) {
   extern __shared__ __align__(1024) char smem_raw[];
   char* smem = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   constexpr int A_BYTES = BM * BK * 2;
   constexpr int B_BYTES = BN * BK * 2;
   constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  constexpr int RS = BN + 4;   // receive-buffer row stride in floats (padding against bank conflicts)
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
   uint64_t* empty = full + STAGES;
   uint64_t* accum = empty + STAGES;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+  uint64_t* rbar = accum + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rbar + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  float* sbias = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES + 256);   // bias[n0 .. n0 + BN)
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM;
-  const int kb0 = blockIdx.z * p.kper;
+  const int S = gridDim.z, me = blockIdx.z;
+  const int kb0 = me * p.kper;
   const int kb1 = min(p.KB, kb0 + p.kper);
   const int nk = kb1 - kb0;
+  const int maxr = (BM + S - 1) / S;            // rows per receive slot
+  const int r0 = me * BM / S, r1 = (me + 1) * BM / S;
   constexpr uint32_t kCols = BN < 32 ? 32 : BN;
 
   if (threadIdx.x == 0) {
@@ -356,6 +343,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
       mbar_init(&empty[s], 1);
     }
     mbar_init(accum, 1);
+    mbar_init(rbar, (S - 1) * (r1 - r0));   // one release-arrive per pushed row
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmA)) : "memory");
@@ -417,103 +405,70 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
       else mbar_expect_tx(accum, 0);  // release the epilogue without data
     }
   } else {
-    // Epilogue: warp (2..5) % 4 owns TMEM lanes 32 * q .. 32 * q + 31.
-    const int q = warp % 4;
-    const bool ready = mbar_wait(accum, 0);
+    // the tile's bias into shared memory while the MMAs run
+    for (int j = threadIdx.x - 64; j < BN; j += 128) sbias[j] = p.bias ? p.bias[n0 + j] : 0.f;
+    if (!mbar_wait(accum, 0)) atomicExch(p.err, 3);
     tc_fence_after();
-    if (!ready) atomicExch(p.err, 3);
-    const int row = q * 32 + lane;
-    const int m = m0 + row;
-    const bool valid = ready && !*abort_flag && nk > 0;
-    if (CLUSTER) {
-      // own partial tile -> shared memory (the pipeline buffers are idle now)
-      float* red = reinterpret_cast<float*>(smem);
-      for (int c = 0; c < BN; c += 16) {
-        uint32_t r[16];
-        tmem_ld16(tmem + (uint32_t(q * 32) << 16) + uint32_t(c), r);
-        float4* dst = reinterpret_cast<float4*>(red + row * (BN + 4) + c);
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-          dst[j] = valid ? make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
-                                       __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]))
-                         : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-    } else {
-    for (int c = 0; c < BN; c += 16) {
-      uint32_t r[16];
-      tmem_ld16(tmem + (uint32_t(q * 32) << 16) + uint32_t(c), r);
-      if (!valid || m >= p.M) continue;
-      float v[16];
-#pragma unroll
-      for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
-      const int n = n0 + c;
-      const size_t mo = out_row(p, m);
-      if (p.bias) {
-#pragma unroll
-        for (int j = 0; j < 16; ++j) v[j] += p.bias[n + j];
-      }
-      if (p.relu) {
-#pragma unroll
-        for (int j = 0; j < 16; ++j) v[j] = fmaxf(v[j], 0.f);
-      }
-      if (p.mask) {
-        const uint4* mk = reinterpret_cast<const uint4*>(p.mask + mo * p.ldo + n);
-#pragma unroll
-        for (int j = 0; j < 2; ++j) {
-          uint4 u = mk[j];
-          const bf16* e = reinterpret_cast<const bf16*>(&u);
-#pragma unroll
-          for (int q = 0; q < 8; ++q)
-            if (!(__bfloat162float(e[q]) > 0.f)) v[8 * j + q] = 0.f;
-        }
-      }
-      if (p.out_f32) {
-        float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + mo * p.ldo + n);
-        if (p.acc) {
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            float4 o = dst[j];
-            v[4 * j] += o.x; v[4 * j + 1] += o.y; v[4 * j + 2] += o.z; v[4 * j + 3] += o.w;
-          }
-        }
-#pragma unroll
-        for (int j = 0; j < 4; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-      } else {
-        uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(p.out) + mo * p.ldo + n);
-        if (p.acc) {
-#pragma unroll
-          for (int j = 0; j < 2; ++j) {
-            uint4 o = dst[j];
-            const bf16* ob = reinterpret_cast<const bf16*>(&o);
-#pragma unroll
-            for (int e = 0; e < 8; ++e) v[8 * j + e] += __bfloat162float(ob[e]);
-          }
-        }
-        uint4 pk[2];
-        uint32_t* pw = reinterpret_cast<uint32_t*>(pk);
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          __nv_bfloat162 h2 = __floats2bfloat162_rn(v[2 * j], v[2 * j + 1]);
-          pw[j] = *reinterpret_cast<uint32_t*>(&h2);
-        }
-        dst[0] = pk[0];
-        dst[1] = pk[1];
-      }
-    }
-    }
   }
-  if (CLUSTER) {
-    cluster_sync_all();
-    if (warp >= 2) {
-      const int S = gridDim.z, rank = blockIdx.z;
-      const int r0 = rank * BM / S, r1 = (rank + 1) * BM / S;
-      const int t = threadIdx.x - 64;
-      const uint32_t base = smem_u32(smem);
-      cluster_reduce_rows<BN>(p, base, S, r0, r1, m0, n0, t);
-    }
-    cluster_sync_all();
-  }
+  // Every CTA of the cluster is past its MMAs: its pipeline buffers (now the
+  // receive slots) are free and its receive barrier is armed.
   tc_fence_before();
+  cluster_sync_all();
+  tc_fence_after();
+  if (warp >= 2) {
+    const int q = warp % 4, row = q * 32 + lane;
+    const uint32_t trow = tmem + (uint32_t(q * 32) << 16);
+    int z = 0;                                 // owner of this row
+    while (z + 1 < S && (z + 1) * BM / S <= row) ++z;
+    const bool push = z != me;
+    const int slot = me < z ? me : me - 1;     // this rank's slot at the owner
+    const uint32_t dst = smem_u32(smem) + uint32_t(((slot * maxr + row - z * BM / S) * RS) * 4);
+    const uint32_t dst_cta = map_to_cta(dst, uint32_t(z));
+    const uint32_t bar_cta = map_to_cta(smem_u32(rbar), uint32_t(z));
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      uint32_t r[32];
+      tmem_ld32(trow + uint32_t(c), r);
+      if (push)
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          st_cluster4(dst_cta + uint32_t((c + 4 * j) * 4), r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
+    }
+    if (push) mbar_arrive_remote(bar_cta);
+    // Owner: rows r0..r1-1 of this lane quarter, summed over ranks in order.
+    if (q * 32 < r1 && q * 32 + 32 > r0) {
+      if (!mbar_wait_cluster(rbar, 0)) atomicExch(p.err, 9);
+      const bool own = row >= r0 && row < r1 && m0 + row < p.M;
+      const uint32_t rbase = smem_u32(smem) + uint32_t(((row - r0) * RS) * 4);
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 32) {
+        uint32_t r[32];
+        tmem_ld32(trow + uint32_t(c), r);
+        if (!own) continue;
+        float v[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = 0.f;
+#pragma unroll 1
+        for (int s = 0; s < S; ++s) {
+          if (s == me) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] += __uint_as_float(r[j]);
+          } else {
+            const uint32_t src = rbase + uint32_t(((s < me ? s : s - 1) * maxr * RS + c) * 4);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const float4 w = ld_shared4(src + 16u * j);
+              v[4 * j] += w.x; v[4 * j + 1] += w.y; v[4 * j + 2] += w.z; v[4 * j + 3] += w.w;
+            }
+          }
+        }
+        store_row32(p, m0 + row, n0 + c, v, smem_u32(sbias) + uint32_t(c) * 4u);
+      }
+    }
+  }
+  // No CTA leaves while a peer may still be writing into it.
+  tc_fence_before();
+  cluster_sync_all();
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
@@ -713,7 +668,8 @@ constexpr int stages_for() {
 }
 template <int KIND, int BN>
 constexpr size_t smem_bytes(bool cluster) {
-  return size_t(stages_for<KIND, BN>()) * (BM * BK * 2 + BN * BK * 2) + 1024 + 256 + (cluster ? 0 : kEpiStageBytes);
+  return size_t(stages_for<KIND, BN>()) * (BM * BK * 2 + BN * BK * 2) + 1024 + 256 +
+         (cluster ? 4 * BN : kEpiStageBytes);
 }
 
 typedef void (*KernelFn)(const TcParams);
@@ -721,7 +677,7 @@ typedef void (*KernelFn)(const TcParams);
 template <int KIND, int BN>
 KernelFn kernel_ptr(bool cluster, int pair) {
   constexpr int S = stages_for<KIND, BN>();
-  if (cluster) return pair ? nullptr : tc_gemm_kernel<KIND, BN, S, true>;
+  if (cluster) return pair ? nullptr : tc_gemm_kernel<KIND, BN, S>;
   if constexpr ((KIND == CONV_FPROP || KIND == CONV_DGRAD) && BN >= 128) {
     if (pair == 1) return tc_gemm_persistent<KIND, BN, S, 1>;
   }
