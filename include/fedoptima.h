@@ -251,6 +251,25 @@ FO_API int fo_axpby_async(float* global, const float* local, int64_t n, float al
 FO_API int fo_column_sums(const void* x, int dtype, int64_t rows, int cols, float* out, void* stream);
 
 /* ------------------------------------------------------------------------
+ * Pre-processor split selection (Sec. 3.2, "Splitting the DNN", Eqs. 4-6).
+ * Host-only; runs once at initialisation.  The model M has L layers; layer
+ * l (1-based) costs O[l-1] floating-point operations per training pass on a
+ * device and its output is S[l-1] bytes.  Device k has bandwidth b[k]
+ * (bytes/s) and compute o[k] (FLOP/s).  Splitting after layer l costs
+ * device k t_train = sum_{i<=l} O_i / o_k and t_transfer = S_l / b_k; the
+ * chosen split is
+ *     l = argmin_l  max_k  max(t_train_k(l), t_transfer_k(l))
+ * over the candidate split points: every l in 1..L when `allowed` is NULL,
+ * else the l with allowed[l-1] != 0 (split points between sequential layers,
+ * never inside a branch).  Ties go to the smallest l.  Writes l to *split and
+ * the minimised time (seconds) to *cost.
+ * Errors: FO_ERR_ARG for L < 1, K < 1, a null pointer, a negative O or S, a
+ * non-positive b or o, or no allowed candidate (the outputs are untouched).
+ * ---------------------------------------------------------------------- */
+FO_API int fo_select_split(const double* O, const double* S, int L, const double* b, const double* o, int K,
+                           const unsigned char* allowed, int* split, double* cost);
+
+/* ------------------------------------------------------------------------
  * fo_column_sums without any allocation.  The paper has no counterpart: it
  * is an interface for callers that cannot allocate device memory when they
  * need the reduction -- code running while its stream is captured into a

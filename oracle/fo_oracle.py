@@ -19,6 +19,9 @@ What it follows (arxiv 2504.13850):
     local model with staleness cut-off D and weight alpha = 1/(t - t_k + 1).
   * Layer arithmetic is the textbook definition of each layer, in fp64;
     matrix products (numpy ``@``) are used as a library primitive.
+  * The Pre-processor's split point (Sec. 3.2, Eqs. 4-6): argmin over split
+    points of the slowest device's max of training and transfer time
+    (``split_point``; ties go to the smallest l).
 
 Readings where the paper is silent (each one is listed in the design notes):
   * ties in argmin_k c_k go to the lowest k; only non-empty queues compete;
@@ -604,3 +607,29 @@ class Server:
 
     def aggregate(self, theta_d, theta_dk, t_k):
         return self.agg.aggregate(theta_d, theta_dk, t_k)
+
+
+# ---------------------------------------------------------------------------
+# Pre-processor (Sec. 3.2, "Splitting the DNN", Eqs. 4-6)
+# ---------------------------------------------------------------------------
+def split_point(O, S, b, o, allowed=None):
+    """Split point l (1-based: M_d = layers 1..l) minimising, over the
+    candidate points, the slowest device's max of its training time
+    t_train_k(l) = sum_{i<=l} O_i / o_k (Eq. 4) and its activation transfer
+    time t_transfer_k(l) = S_l / b_k (Eq. 5); Eq. 6 takes the argmin over l
+    of the max over devices.  Candidates: every l, or those with
+    allowed[l-1] true.  Ties: smallest l (the paper is silent).
+    Returns (l, cost in seconds)."""
+    L, K = len(O), len(b)
+    best_l, best_cost = None, None
+    for l in range(1, L + 1):
+        if allowed is not None and not allowed[l - 1]:
+            continue
+        worst = 0.0
+        for k in range(K):
+            t_train = sum(float(O[i]) for i in range(l)) / float(o[k])
+            t_transfer = float(S[l - 1]) / float(b[k])
+            worst = max(worst, t_train, t_transfer)
+        if best_cost is None or worst < best_cost:
+            best_l, best_cost = l, worst
+    return best_l, best_cost

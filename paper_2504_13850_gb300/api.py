@@ -92,6 +92,8 @@ _SIGS = [
     ("fo_axpby_async", C.c_int, [C.c_void_p, C.c_void_p, C.c_int64, C.c_float, C.c_void_p]),
     ("fo_column_sums", C.c_int, [C.c_void_p, C.c_int, C.c_int64, C.c_int, C.c_void_p, C.c_void_p]),
     ("fo_column_sums_noalloc", C.c_int, [C.c_void_p, C.c_int, C.c_int64, C.c_int, C.c_void_p, C.c_void_p]),
+    ("fo_select_split", C.c_int, [C.c_void_p, C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_int, C.c_void_p,
+                                  C.POINTER(C.c_int), C.POINTER(C.c_double)]),
 ]
 
 
@@ -361,3 +363,17 @@ def column_sums_noalloc(x, out, stream=None):
 def axpby_async(global_, local, alpha, stream=None):
     n = global_.numel() if hasattr(global_, "numel") else global_.size
     _check(lib().fo_axpby_async(_ptr(global_), _ptr(local), n, alpha, stream), "axpby_async")
+
+
+def select_split(O, S, b, o, allowed=None):
+    """Pre-processor split point (Eqs. 4-6) through fo_select_split: returns
+    (status, l, cost) with l 1-based (split after layer l)."""
+    O = np.ascontiguousarray(O, np.float64)
+    S = np.ascontiguousarray(S, np.float64)
+    b = np.ascontiguousarray(b, np.float64)
+    o = np.ascontiguousarray(o, np.float64)
+    al = None if allowed is None else np.ascontiguousarray(allowed, np.uint8)
+    l, cost = C.c_int(0), C.c_double(0.0)
+    rc = lib().fo_select_split(O.ctypes.data, S.ctypes.data, len(O), b.ctypes.data, o.ctypes.data, len(b),
+                               None if al is None else al.ctypes.data, C.byref(l), C.byref(cost))
+    return rc, l.value, cost.value
