@@ -386,6 +386,8 @@ def run_ours(args):
         v_cpu, dt_cpu = oracle_samples_per_s(cfg, 2, B)
         cpu = {"value": round(v_cpu, 3), "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
                "sample": f"2 oracle server steps at batch {B} ({dt_cpu:.1f} s, numpy fp64, BLAS threads = cores)"}
+    from paper_2504_13850_gb300 import study
+    sched = study.scheduler_balance("scale", uploads=6000)   # host-only: counter vs FIFO scheduling
     wsb = srv.device_bytes()
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -401,6 +403,7 @@ def run_ours(args):
         "step_tensor_frac": round(tensor_frac, 4),
         "step_gflop": round(step_flops / 1e9, 2),
         "aggregation": agg,
+        "scheduler_balance": sched,
         "cpu_baseline": cpu,
         "clocks": clk.summary(),
         "host_wall_ms_per_step": round(1e3 * wall / args.steps, 4),
