@@ -50,6 +50,8 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-agg-sweep", action="store_true")
+    p.add_argument("--no-live", action="store_true",
+                   help="skip the live pipeline (devices' networks training on the same GPU)")
     return p.parse_args()
 
 
@@ -389,6 +391,16 @@ def run_ours(args):
     from paper_2504_13850_gb300 import study
     sched = study.scheduler_balance("scale", uploads=6000)   # host-only: counter vs FIFO scheduling
     wsb = srv.device_bytes()
+    live_line = None
+    if rank == 0 and not args.no_live and args.workload == "vgg":
+        # a second workload: the VGG-style split with every device's network
+        # training on the same GPU and feeding the server (measured after the
+        # timed region, so it does not perturb `value`)
+        try:
+            from paper_2504_13850_gb300 import live
+            live_line = live.measure(events=400, warmup=40, agg_every=8)
+        except Exception as e:   # reported, not fatal: the headline above stands alone
+            live_line = {"error": f"{type(e).__name__}: {e}"}
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4), "higher_is_better": True,
@@ -404,6 +416,7 @@ def run_ours(args):
         "step_gflop": round(step_flops / 1e9, 2),
         "aggregation": agg,
         "scheduler_balance": sched,
+        "live_pipeline": live_line,
         "cpu_baseline": cpu,
         "clocks": clk.summary(),
         "host_wall_ms_per_step": round(1e3 * wall / args.steps, 4),

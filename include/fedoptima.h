@@ -133,6 +133,29 @@ FO_API int fo_server_get_params(fo_server* s, float* host, int64_t n);
 FO_API int fo_server_set_momentum(fo_server* s, const float* host, int64_t n);
 FO_API int fo_server_get_momentum(fo_server* s, float* host, int64_t n);
 
+/* Device-resident access, for running a device's network (M_dk and its
+ * auxiliary network, Alg. 1) as a second fo_server on the same GPU and
+ * feeding its split-point activations and models to the server.
+ * fo_server_tensor: device pointer, NHWC dims (dims4[0..3]) and dtype of
+ *   tensor `index` -- 1..n_ops is the output of op index-1 -- as written by
+ *   the last fo_server_step.  The pointer stays valid for the server's
+ *   lifetime; the contents change with each step, which runs on
+ *   fo_server_stream.  FO_ERR_ARG for an index outside 1..n_ops.
+ * fo_server_params_device: the fp32 master parameters on the device in the
+ *   server's padded layout (*n floats; identical for servers built from the
+ *   same op list), for device-to-device aggregation.  Read it only when the
+ *   server's stream is idle.
+ * fo_server_load_params_device: copies n (padded layout) floats from device
+ *   memory `src` into the parameters and refreshes the bf16 shadow, ordered
+ *   on the server's stream; returns after the copy is issued.
+ *   FO_ERR_ARG when n differs from the padded length. */
+FO_API int fo_server_tensor(const fo_server* s, int index, const void** data, int64_t* dims4, int* dtype);
+FO_API int fo_server_params_device(fo_server* s, float** theta, int64_t* n);
+FO_API int fo_server_load_params_device(fo_server* s, const float* src, int64_t n);
+/* The reverse copy: the parameters (padded layout, *n floats) into device
+ * memory `dst`, ordered on the server's stream. */
+FO_API int fo_server_store_params_device(fo_server* s, float* dst, int64_t n);
+
 /* Task Scheduler put() for an activation message (Algorithm 2) plus the
  * server-side flow control of Sec. 3.4.1.  `acts` (host or device) holds
  * B*H*W*C elements of the configured dtype, NHWC; `labels` (host or device)

@@ -92,6 +92,11 @@ _SIGS = [
     ("fo_axpby_async", C.c_int, [C.c_void_p, C.c_void_p, C.c_int64, C.c_float, C.c_void_p]),
     ("fo_column_sums", C.c_int, [C.c_void_p, C.c_int, C.c_int64, C.c_int, C.c_void_p, C.c_void_p]),
     ("fo_column_sums_noalloc", C.c_int, [C.c_void_p, C.c_int, C.c_int64, C.c_int, C.c_void_p, C.c_void_p]),
+    ("fo_server_tensor", C.c_int, [C.c_void_p, C.c_int, C.POINTER(C.c_void_p), C.POINTER(C.c_int64),
+                                   C.POINTER(C.c_int)]),
+    ("fo_server_params_device", C.c_int, [C.c_void_p, C.POINTER(C.c_void_p), C.POINTER(C.c_int64)]),
+    ("fo_server_load_params_device", C.c_int, [C.c_void_p, C.c_void_p, C.c_int64]),
+    ("fo_server_store_params_device", C.c_int, [C.c_void_p, C.c_void_p, C.c_int64]),
     ("fo_select_split", C.c_int, [C.c_void_p, C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_int, C.c_void_p,
                                   C.POINTER(C.c_int), C.POINTER(C.c_double)]),
 ]
@@ -300,6 +305,24 @@ class Server:
 
     def device_bytes(self):
         return lib().fo_server_device_bytes(self.h)
+
+    def tensor(self, index):
+        """(device pointer, (N, H, W, C), dtype) of the output of op index-1."""
+        ptr, dims, dt = C.c_void_p(), (C.c_int64 * 4)(), C.c_int(0)
+        _check(lib().fo_server_tensor(self.h, index, C.byref(ptr), dims, C.byref(dt)), "fo_server_tensor")
+        return ptr.value, tuple(int(v) for v in dims), dt.value
+
+    def params_device(self):
+        """(device pointer, length) of the fp32 parameters in the padded layout."""
+        ptr, n = C.c_void_p(), C.c_int64(0)
+        _check(lib().fo_server_params_device(self.h, C.byref(ptr), C.byref(n)), "fo_server_params_device")
+        return ptr.value, n.value
+
+    def load_params_device(self, src_ptr, n):
+        _check(lib().fo_server_load_params_device(self.h, C.c_void_p(src_ptr), n), "fo_server_load_params_device")
+
+    def store_params_device(self, dst_ptr, n):
+        _check(lib().fo_server_store_params_device(self.h, C.c_void_p(dst_ptr), n), "fo_server_store_params_device")
 
     def check_error(self):
         _check(lib().fo_server_error(self.h), "server_error")

@@ -21,8 +21,12 @@ void conv_fwd_simt(const ConvShape& s, const void* x, int dt_x, const void* w, i
 void conv_dgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* w, int dt_w,
                      void* dx, int dt_dx, bool accumulate, const void* mask, cudaStream_t st);
 // dw[Co][k][k][Ci] = sum over output pixels of dy (x) x-window (fp32 out).
-void conv_wgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* x,
-                     int dt_x, float* dw, cudaStream_t st);
+// Weight gradient; K is split over blocks into `scratch` (simt_wgrad_scratch_floats
+// floats, or null for one pass) and summed in split order.
+int simt_wgrad_splits(const ConvShape& s);
+int64_t simt_wgrad_scratch_floats(const ConvShape& s);
+void conv_wgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* x, int dt_x,
+                     float* dw, float* scratch, cudaStream_t st);
 
 // ---- elementwise / reductions (templated on the activation dtype) ----
 void relu_fwd(const void* x, void* y, int64_t n, int dt, cudaStream_t st);

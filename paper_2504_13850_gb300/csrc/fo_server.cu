@@ -460,8 +460,11 @@ int build_plan(fo_server* s) {
         if (tw) {
           add_tc(tw);
         } else {
-          add(op.kind == FO_OP_CONV ? "conv_wgrad_simt" : "linear_wgrad_simt", 1, fl, 0.0, [=](cudaStream_t st) {
-            fo::conv_wgrad_simt(cs, s->T[o].grad, dto, act(a0), s->T[a0].dt, G(s, i, 0), st);
+          const bool split = fo::simt_wgrad_splits(cs) > 1;
+          add(op.kind == FO_OP_CONV ? "conv_wgrad_simt" : "linear_wgrad_simt", split ? 2 : 1, fl, 0.0,
+              [=](cudaStream_t st) {
+            fo::conv_wgrad_simt(cs, s->T[o].grad, dto, act(a0), s->T[a0].dt, G(s, i, 0),
+                                split ? s->simt_scratch : nullptr, st);
           });
         }
         break;
@@ -688,6 +691,11 @@ int allocate(fo_server* s) {
     cs_floats = std::max(cs_floats, fo::server_colsum_floats(a.rows(), a.C));
   }
   s->colsum_scratch = (float*)s->alloc(cs_floats * 4);
+  int64_t simt_floats = 0;   // split-K partials of the CUDA-core weight gradient
+  for (int i = 0; i < nops; ++i)
+    if (s->ops[i].kind == FO_OP_CONV || s->ops[i].kind == FO_OP_LINEAR)
+      simt_floats = std::max(simt_floats, fo::simt_wgrad_scratch_floats(conv_shape(s, i)));
+  s->simt_scratch = simt_floats ? (float*)s->alloc(simt_floats * 4) : nullptr;
   s->ln_mean.assign(nops, nullptr);
   s->ln_rstd.assign(nops, nullptr);
   s->attn_probs.assign(nops, nullptr);
@@ -863,6 +871,41 @@ int fo_server_set_momentum(fo_server* s, const float* host, int64_t n) {
 }
 int fo_server_get_momentum(fo_server* s, float* host, int64_t n) {
   return copy_params(s, s ? s->mom : nullptr, nullptr, host, n);
+}
+
+int fo_server_tensor(const fo_server* s, int index, const void** data, int64_t* dims4, int* dtype) {
+  if (!s || !data || !dims4 || !dtype) return set_err(FO_ERR_ARG, "null argument");
+  if (index < 1 || index > int(s->ops.size())) return set_err(FO_ERR_ARG, "tensor index outside 1..n_ops");
+  const Tensor& t = s->T[index];
+  *data = t.act;
+  dims4[0] = t.N;
+  dims4[1] = t.H;
+  dims4[2] = t.W;
+  dims4[3] = t.C;
+  *dtype = t.dt;
+  return FO_OK;
+}
+
+int fo_server_params_device(fo_server* s, float** theta, int64_t* n) {
+  if (!s || !theta || !n) return set_err(FO_ERR_ARG, "null argument");
+  *theta = s->theta;
+  *n = s->n_padded;
+  return FO_OK;
+}
+
+int fo_server_load_params_device(fo_server* s, const float* src, int64_t n) {
+  if (!s || !src) return set_err(FO_ERR_ARG, "null argument");
+  if (n != s->n_padded) return set_err(FO_ERR_ARG, "parameter vector length is not the padded length");
+  FO_CUDA(cudaMemcpyAsync(s->theta, src, size_t(n) * 4, cudaMemcpyDeviceToDevice, s->cs));
+  if (s->shadow) fo::f32_to_bf16(s->theta, s->shadow, s->n_padded, s->cs);
+  return FO_OK;
+}
+
+int fo_server_store_params_device(fo_server* s, float* dst, int64_t n) {
+  if (!s || !dst) return set_err(FO_ERR_ARG, "null argument");
+  if (n != s->n_padded) return set_err(FO_ERR_ARG, "parameter vector length is not the padded length");
+  FO_CUDA(cudaMemcpyAsync(dst, s->theta, size_t(n) * 4, cudaMemcpyDeviceToDevice, s->cs));
+  return FO_OK;
 }
 
 int fo_enqueue_activations(fo_server* s, int device_id, const void* acts, const int32_t* labels,

@@ -79,6 +79,7 @@ struct fo_server {
   std::vector<Tensor> T;
   float* colsum_scratch = nullptr;
   std::vector<float*> ln_mean, ln_rstd, attn_probs;
+  float* simt_scratch = nullptr;   // K-split partials of the CUDA-core weight gradient
 
   const void* cur_in = nullptr;
   const int32_t* cur_labels = nullptr;

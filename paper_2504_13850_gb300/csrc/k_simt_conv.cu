@@ -11,6 +11,8 @@
 #include "fo_common.cuh"
 #include "fo_kernels.h"
 
+#include <algorithm>
+
 namespace fo {
 
 namespace {
@@ -22,6 +24,7 @@ constexpr int BM = 64, BN = 64, BK = 16, NT = 256;
 struct Geo {
   int N, H, W, Ci, Co, k, stride, pad, Ho, Wo;
   int64_t M, Ncol, K;
+  int64_t kper;   // k-range per blockIdx.z (K split); the output of split z starts at c + z * M * Ncol
 };
 
 template <typename T>
@@ -95,15 +98,17 @@ __global__ void __launch_bounds__(NT) simt_conv_kernel(Geo g, const TA* __restri
   const int tid = threadIdx.x;
   const int tx = tid % 16, ty = tid / 16;
   const int64_t m0 = int64_t(blockIdx.y) * BM, n0 = int64_t(blockIdx.x) * BN;
+  const int64_t kb = int64_t(blockIdx.z) * g.kper, ke = min(g.K, kb + g.kper);
+  c += int64_t(blockIdx.z) * g.M * g.Ncol;
   float accum[4][4] = {};
-  for (int64_t k0 = 0; k0 < g.K; k0 += BK) {
+  for (int64_t k0 = kb; k0 < ke; k0 += BK) {
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       int e = tid + i * NT;           // 0..1023
       int am = e / BK, ak = e % BK;   // A tile 64 x 16
-      As[ak][am] = load_a<MODE>(g, a, m0 + am, k0 + ak);
+      As[ak][am] = k0 + ak < ke ? load_a<MODE>(g, a, m0 + am, k0 + ak) : 0.f;
       int bk = e / BN, bn = e % BN;   // B tile 16 x 64
-      Bs[bk][bn] = load_b<MODE>(g, b, k0 + bk, n0 + bn);
+      Bs[bk][bn] = k0 + bk < ke ? load_b<MODE>(g, b, k0 + bk, n0 + bn) : 0.f;
     }
     __syncthreads();
 #pragma unroll
@@ -140,7 +145,7 @@ __global__ void __launch_bounds__(NT) simt_conv_kernel(Geo g, const TA* __restri
 }
 
 Geo make_geo(const ConvShape& s, int mode) {
-  Geo g{s.N, s.H, s.W, s.Ci, s.Co, s.k, s.stride, s.pad, s.Ho, s.Wo, 0, 0, 0};
+  Geo g{s.N, s.H, s.W, s.Ci, s.Co, s.k, s.stride, s.pad, s.Ho, s.Wo, 0, 0, 0, 0};
   int64_t pix_out = int64_t(s.N) * s.Ho * s.Wo, pix_in = int64_t(s.N) * s.H * s.W;
   if (mode == FWD) {
     g.M = pix_out; g.Ncol = s.Co; g.K = int64_t(s.k) * s.k * s.Ci;
@@ -149,13 +154,34 @@ Geo make_geo(const ConvShape& s, int mode) {
   } else {
     g.M = s.Co; g.Ncol = int64_t(s.k) * s.k * s.Ci; g.K = pix_out;
   }
+  g.kper = g.K;
   return g;
+}
+
+// Sums the `splits` partial outputs [splits][n] in order.
+__global__ void sum_splits_k(const float* __restrict__ part, int splits, int64_t n, float* __restrict__ out) {
+  for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < n; i += int64_t(gridDim.x) * blockDim.x) {
+    float t = 0.f;
+    for (int z = 0; z < splits; ++z) t += part[int64_t(z) * n + i];
+    out[i] = t;
+  }
+}
+
+int sm_count() {
+  static int sms = 0;
+  if (!sms) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (sms <= 0) sms = 148;
+  }
+  return sms;
 }
 
 template <int MODE, typename TA, typename TB, typename TC>
 void launch(const Geo& g, const void* a, const void* b, const float* bias, void* c, bool relu,
             bool acc, cudaStream_t st, const void* mask = nullptr) {
-  dim3 grid(ceil_div(g.Ncol, BN), ceil_div(g.M, BM));
+  dim3 grid(ceil_div(g.Ncol, BN), ceil_div(g.M, BM), unsigned(ceil_div(g.K, g.kper)));
   simt_conv_kernel<MODE, TA, TB, TC><<<grid, NT, 0, st>>>(
       g, (const TA*)a, (const TB*)b, bias, (TC*)c, relu ? 1 : 0, acc ? 1 : 0, (const TC*)mask);
 }
@@ -192,9 +218,37 @@ void conv_dgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* 
   launch_any<DGRAD>(make_geo(s, DGRAD), dy, dt_dy, w, dt_w, nullptr, dx, dt_dx, false, accumulate, st, mask);
 }
 
+// The weight gradient's K (output pixels) is long and its output small:
+// split K so the grid covers about two blocks per SM, into fp32 partials that
+// a second pass sums in split order (deterministic).
+int simt_wgrad_splits(const ConvShape& s) {
+  const Geo g = make_geo(s, WGRAD);
+  const int64_t blocks = ceil_div(g.Ncol, BN) * ceil_div(g.M, BM);
+  int64_t sp = (2 * sm_count() + blocks - 1) / blocks;
+  sp = std::min<int64_t>(sp, std::max<int64_t>(1, g.K / (8 * BK)));   // at least 8 k-tiles per split
+  return int(std::max<int64_t>(1, sp));
+}
+
+int64_t simt_wgrad_scratch_floats(const ConvShape& s) {
+  const int sp = simt_wgrad_splits(s);
+  const Geo g = make_geo(s, WGRAD);
+  return sp > 1 ? int64_t(sp) * g.M * g.Ncol : 0;
+}
+
 void conv_wgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* x, int dt_x,
-                     float* dw, cudaStream_t st) {
-  launch_any<WGRAD>(make_geo(s, WGRAD), dy, dt_dy, x, dt_x, nullptr, dw, kF32, false, false, st);
+                     float* dw, float* scratch, cudaStream_t st) {
+  Geo g = make_geo(s, WGRAD);
+  const int sp = scratch ? simt_wgrad_splits(s) : 1;
+  if (sp <= 1) {
+    launch_any<WGRAD>(g, dy, dt_dy, x, dt_x, nullptr, dw, kF32, false, false, st);
+    return;
+  }
+  g.kper = (g.K + sp - 1) / sp;
+  g.kper = (g.kper + BK - 1) / BK * BK;
+  const int real = int(ceil_div(g.K, g.kper));
+  launch_any<WGRAD>(g, dy, dt_dy, x, dt_x, nullptr, scratch, kF32, false, false, st);
+  const int64_t n = g.M * g.Ncol;
+  sum_splits_k<<<int(std::min<int64_t>(ceil_div(n, 256), 4 * sm_count())), 256, 0, st>>>(scratch, real, n, dw);
 }
 
 }  // namespace fo

@@ -87,6 +87,27 @@ def vgg_ops():
     return b.ops
 
 
+def vgg_device_ops():
+    """A device's network for the VGG-style split (Alg. 1): M_dk = conv3x3
+    3->128 + ReLU + maxpool 2 on a [32,32,3] image, whose [16,16,128] output
+    (tensor 3) is the activation uploaded to the server; then the default
+    auxiliary network (one layer of the same type as M_dk's last layer and a
+    dense classifier): conv3x3 128->128 + ReLU, global average pool,
+    FC 128 -> 10."""
+    b = _Builder()
+    t = b.add("conv", 0, cin=3, cout=128, k=3, stride=1, bias=1)
+    t = b.add("relu", t)
+    t = b.add("maxpool2", t)
+    t = b.add("conv", t, cin=128, cout=128, k=3, stride=1, bias=1)
+    t = b.add("relu", t)
+    t = b.add("avgpool", t)
+    b.add("linear", t, cin=128, cout=10, bias=1)
+    return b.ops
+
+
+VGG_DEVICE_SPLIT = 3      # tensor id of M_dk's output in vgg_device_ops()
+
+
 def _basic_block(b, x, cin, cout, stride):
     """ResNet basic block with BN folded to a trainable per-channel affine."""
     t = b.add("conv", x, cin=cin, cout=cout, k=3, stride=stride, bias=0)
@@ -186,6 +207,11 @@ CONFIGS = {
     "scale": _cfg("scale", resnet_ops(), K=100, depth=4, omega=400, batch=64,
                   in_hwc=(16, 16, 128), dtype=BF16, classes=100, seed=4,
                   steps=1000, agg_params=700_000, rates=zipf_rates(100)),
+    # one device's own trainer for the live VGG pipeline: its local data
+    # queue (K = 1) feeds M_dk + the auxiliary network
+    "vgg_device": _cfg("vgg_device", vgg_device_ops(), K=1, depth=2, omega=2, batch=64,
+                       in_hwc=(32, 32, 3), dtype=BF16, classes=10, seed=5, steps=0,
+                       agg_params=0, rates=[1.0]),
 }
 
 
