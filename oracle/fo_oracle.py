@@ -19,6 +19,12 @@ What it follows (arxiv 2504.13850):
     local model with staleness cut-off D and weight alpha = 1/(t - t_k + 1).
   * Layer arithmetic is the textbook definition of each layer, in fp64;
     matrix products (numpy ``@``) are used as a library primitive.
+  * The MobileNetV3 bottleneck pieces of the paper's testbed-B CNN
+    (Table 2): depthwise convolution, hard swish, hard sigmoid and the
+    squeeze-and-excite channel scaling (``dwconv_*``, ``hswish_*``,
+    ``hsigmoid_*``, ``chmul_*``); the derivative readings at the kinks
+    follow the usual library convention (hard swish: 0 below -3, 1 above 3;
+    hard sigmoid: 1/6 strictly inside (-3, 3)).
   * The Pre-processor's split point (Sec. 3.2, Eqs. 4-6): argmin over split
     points of the slowest device's max of training and transfer time
     (``split_point``; ties go to the smallest l).
@@ -231,6 +237,73 @@ def conv_bwd(x, w, dy, stride, pad, need_dx):
     return dx, dw, db
 
 
+def dwconv_fwd(x, w, b, stride, pad):
+    """Depthwise convolution (one k x k filter per channel, as in the
+    MobileNetV3 bottleneck): y[n,i,j,c] = b[c] +
+    sum_{r,s} xpad[n, i*stride + r, j*stride + s, c] w[c,r,s]."""
+    N, H, W, C = x.shape
+    k = w.shape[1]
+    Ho = (H + 2 * pad - k) // stride + 1
+    Wo = (W + 2 * pad - k) // stride + 1
+    xp = np.pad(x, ((0, 0), (pad, pad), (pad, pad), (0, 0)))
+    y = np.zeros((N, Ho, Wo, C))
+    for r in range(k):
+        for s in range(k):
+            y += xp[:, r:r + stride * (Ho - 1) + 1:stride, s:s + stride * (Wo - 1) + 1:stride, :] * w[:, r, s]
+    if b is not None:
+        y += b
+    return y
+
+
+def dwconv_bwd(x, w, dy, stride, pad, need_dx):
+    """Gradients of dwconv_fwd: (dx or None, dw, db)."""
+    N, H, W, C = x.shape
+    k = w.shape[1]
+    _, Ho, Wo, _ = dy.shape
+    xp = np.pad(x, ((0, 0), (pad, pad), (pad, pad), (0, 0)))
+    dxp = np.zeros_like(xp) if need_dx else None
+    dw = np.zeros_like(w)
+    for r in range(k):
+        for s in range(k):
+            sl = (slice(None), slice(r, r + stride * (Ho - 1) + 1, stride),
+                  slice(s, s + stride * (Wo - 1) + 1, stride), slice(None))
+            dw[:, r, s] = (dy * xp[sl]).sum(axis=(0, 1, 2))
+            if need_dx:
+                dxp[sl] += dy * w[:, r, s]
+    db = dy.sum(axis=(0, 1, 2))
+    dx = dxp[:, pad:pad + H, pad:pad + W, :] if need_dx else None
+    return dx, dw, db
+
+
+def hswish_fwd(x):
+    """Hard swish x * relu6(x + 3) / 6."""
+    return x * np.clip(x + 3.0, 0.0, 6.0) / 6.0
+
+
+def hswish_bwd(x, dy):
+    # derivative 0 below -3, (2x + 3) / 6 on [-3, 3], 1 above 3
+    return dy * np.where(x < -3.0, 0.0, np.where(x > 3.0, 1.0, (2.0 * x + 3.0) / 6.0))
+
+
+def hsigmoid_fwd(x):
+    """Hard sigmoid relu6(x + 3) / 6."""
+    return np.clip(x + 3.0, 0.0, 6.0) / 6.0
+
+
+def hsigmoid_bwd(x, dy):
+    # derivative 1/6 strictly inside (-3, 3), else 0
+    return dy * np.where((x > -3.0) & (x < 3.0), 1.0 / 6.0, 0.0)
+
+
+def chmul_fwd(x, s):
+    """Channel scaling of the squeeze-and-excite block: y[n,h,w,c] = x[n,h,w,c] s[n,c]."""
+    return x * s[:, None, None, :]
+
+
+def chmul_bwd(x, s, dy):
+    return dy * s[:, None, None, :], (dy * x).sum(axis=(1, 2))
+
+
 def relu_fwd(x):
     return np.maximum(x, 0.0)
 
@@ -417,6 +490,10 @@ def param_shapes(ops):
         elif kd == "layernorm":
             out.append((i, "gamma", (op["c"],)))
             out.append((i, "beta", (op["c"],)))
+        elif kd == "dwconv":
+            out.append((i, "W", (op["c"], op["k"], op["k"])))
+            if op["bias"]:
+                out.append((i, "b", (op["c"],)))
     return out
 
 
@@ -473,6 +550,14 @@ def forward(ops, params, x, lengths, storage=None):
             y, caches[i] = attention_fwd(a, lengths, op["c"], op["heads"])
         elif kd == "meanpool":
             y = meanpool_fwd(a, lengths)
+        elif kd == "dwconv":
+            y = dwconv_fwd(a, P("W"), P("b"), op["stride"], op["k"] // 2)
+        elif kd == "hswish":
+            y = hswish_fwd(a)
+        elif kd == "hsigmoid":
+            y = hsigmoid_fwd(a)
+        elif kd == "chmul":
+            y = chmul_fwd(a, T[op["in1"]])
         else:
             raise ValueError(kd)
         if storage == "bf16" and i < len(ops) - 1:
@@ -539,6 +624,20 @@ def backward(ops, params, T, caches, dlogits, lengths, storage=None):
             acc(op["in0"], attention_bwd(caches[i], dy, op["c"], op["heads"]))
         elif kd == "meanpool":
             acc(op["in0"], meanpool_bwd(a, lengths, dy))
+        elif kd == "dwconv":
+            dx, dw, db = dwconv_bwd(a, P("W"), dy, op["stride"], op["k"] // 2, need)
+            grads[(i, "W")] = dw
+            if op["bias"]:
+                grads[(i, "b")] = db
+            acc(op["in0"], dx)
+        elif kd == "hswish":
+            acc(op["in0"], hswish_bwd(a, dy))
+        elif kd == "hsigmoid":
+            acc(op["in0"], hsigmoid_bwd(a, dy))
+        elif kd == "chmul":
+            dx, ds = chmul_bwd(a, T[op["in1"]], dy)
+            acc(op["in0"], dx)
+            acc(op["in1"], ds)
         else:
             raise ValueError(kd)
     return grads

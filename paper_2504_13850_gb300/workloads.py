@@ -108,6 +108,50 @@ def vgg_device_ops():
 VGG_DEVICE_SPLIT = 3      # tensor id of M_dk's output in vgg_device_ops()
 
 
+def _bneck(b, x, cin, exp, cout, k, stride, se=True, act="hswish"):
+    """MobileNetV3 bottleneck: 1x1 expansion, k x k depthwise (stride),
+    squeeze-and-excite, 1x1 projection; batch norms folded to affines;
+    residual when the shape is kept."""
+    t = b.add("conv", x, cin=cin, cout=exp, k=1, stride=1, bias=0)
+    t = b.add("affine", t, c=exp)
+    t = b.add(act, t)
+    t = b.add("dwconv", t, c=exp, k=k, stride=stride, bias=0)
+    t = b.add("affine", t, c=exp)
+    t = b.add(act, t)
+    if se:
+        sq = b.add("avgpool", t)
+        sq = b.add("linear", sq, cin=exp, cout=exp // 4, bias=1)
+        sq = b.add("relu", sq)
+        sq = b.add("linear", sq, cin=exp // 4, cout=exp, bias=1)
+        sq = b.add("hsigmoid", sq)
+        t = b.add("chmul", t, in1=sq)
+    t = b.add("conv", t, cin=exp, cout=cout, k=1, stride=1, bias=0)
+    t = b.add("affine", t, c=cout)
+    if stride == 1 and cin == cout:
+        t = b.add("add", t, in1=x)
+    return t
+
+
+def mobilenet_ops(classes=10):
+    """Server part of MobileNetV3-Large (the paper's Table 2) after its
+    BNECK-3-112 stage: BNECK-5-160 x 3 (the first with stride 2),
+    CONV-1-960, global average pool, CONV-1-1280 (on the pooled 1 x 1 map,
+    a dense layer) and FC -> classes, with hard swish activations, on a
+    [4,4,112] input."""
+    b = _Builder()
+    t = _bneck(b, 0, 112, 672, 160, 5, 2)
+    t = _bneck(b, t, 160, 960, 160, 5, 1)
+    t = _bneck(b, t, 160, 960, 160, 5, 1)
+    t = b.add("conv", t, cin=160, cout=960, k=1, stride=1, bias=0)
+    t = b.add("affine", t, c=960)
+    t = b.add("hswish", t)
+    t = b.add("avgpool", t)
+    t = b.add("linear", t, cin=960, cout=1280, bias=1)
+    t = b.add("hswish", t)
+    b.add("linear", t, cin=1280, cout=classes, bias=1)
+    return b.ops
+
+
 def _basic_block(b, x, cin, cout, stride):
     """ResNet basic block with BN folded to a trainable per-channel affine."""
     t = b.add("conv", x, cin=cin, cout=cout, k=3, stride=stride, bias=0)
@@ -207,6 +251,9 @@ CONFIGS = {
     "scale": _cfg("scale", resnet_ops(), K=100, depth=4, omega=400, batch=64,
                   in_hwc=(16, 16, 128), dtype=BF16, classes=100, seed=4,
                   steps=1000, agg_params=700_000, rates=zipf_rates(100)),
+    "mobilenet": _cfg("mobilenet", mobilenet_ops(), K=10, depth=4, omega=40, batch=64,
+                      in_hwc=(4, 4, 112), dtype=BF16, classes=10, seed=6, steps=200,
+                      agg_params=1_000_000, rates=group_rates(10)),
     # one device's own trainer for the live VGG pipeline: its local data
     # queue (K = 1) feeds M_dk + the auxiliary network
     "vgg_device": _cfg("vgg_device", vgg_device_ops(), K=1, depth=2, omega=2, batch=64,
@@ -245,6 +292,10 @@ def param_shapes(ops):
         elif kind == "layernorm":
             shapes.append(("gamma", (op["c"],)))
             shapes.append(("beta", (op["c"],)))
+        elif kind == "dwconv":
+            shapes.append(("W", (op["c"], op["k"], op["k"])))
+            if op["bias"]:
+                shapes.append(("b", (op["c"],)))
     return shapes
 
 

@@ -59,6 +59,16 @@ def torch_loss(ops, flat, x, labels, lengths):
         elif kd == "meanpool":
             m = (torch.arange(a.shape[1])[None, :] < ln[:, None]).to(a.dtype)
             y = (a[:, :, 0, :] * m[..., None]).sum(1) / ln[:, None].to(a.dtype)
+        elif kd == "dwconv":
+            w = views[(i, "W")].unsqueeze(1)                  # [C, 1, k, k]: groups = C
+            y = F.conv2d(a.permute(0, 3, 1, 2), w, views.get((i, "b")), stride=op["stride"],
+                         padding=op["k"] // 2, groups=op["c"]).permute(0, 2, 3, 1)
+        elif kd == "hswish":
+            y = F.hardswish(a)
+        elif kd == "hsigmoid":
+            y = F.hardsigmoid(a)
+        elif kd == "chmul":
+            y = a * T[op["in1"]][:, None, None, :]
         else:
             raise ValueError(kd)
         T.append(y)
@@ -93,6 +103,15 @@ def small_resnet():
     return b.ops
 
 
+def small_mobilenet():
+    b = W._Builder()
+    t = W._bneck(b, 0, 4, 12, 6, 3, 2)
+    t = W._bneck(b, t, 6, 16, 6, 5, 1)
+    t = b.add("avgpool", t)
+    b.add("linear", t, cin=6, cout=5, bias=1)
+    return b.ops
+
+
 def small_transformer():
     return W.transformer_ops(d=8, heads=2, ffn=12, blocks=2, classes=2)
 
@@ -101,6 +120,7 @@ CASES = {
     "tiny_cnn": (W.tiny_cnn_ops(), (16, 16, 32), False, 10),
     "vgg": (small_vgg(), (8, 8, 4), False, 5),
     "resnet": (small_resnet(), (8, 8, 4), False, 5),
+    "mobilenet": (small_mobilenet(), (8, 8, 4), False, 5),
     "transformer": (small_transformer(), (6, 1, 8), True, 2),
 }
 
@@ -126,11 +146,15 @@ def test_network_matches_torch_autograd(name):
     loss, g = O.loss_and_grad(ops, theta, x, labels, lengths)
     tl, tg = torch_loss(ops, theta, x, labels, lengths)
     assert abs(loss - tl) <= 1e-12 * abs(tl)
-    # the first layer's input gradient is not part of g; every param grad is
-    assert np.linalg.norm(g - tg) <= 1e-10 * np.linalg.norm(tg)
+    # the first layer's input gradient is not part of g; every param grad is.
+    # PyTorch's hard-sigmoid backward scales by a single-precision 1/6 even in
+    # float64 (a 3e-8 relative error), so the MobileNet case agrees to ~1e-9;
+    # the finite-difference test below pins it independently.
+    tol = 1e-7 if name == "mobilenet" else 1e-10
+    assert np.linalg.norm(g - tg) <= tol * np.linalg.norm(tg)
 
 
-@pytest.mark.parametrize("name", ["vgg", "resnet", "transformer"])
+@pytest.mark.parametrize("name", ["vgg", "resnet", "transformer", "mobilenet"])
 def test_network_finite_differences(name):
     ops, theta, x, labels, lengths = make_case(name, seed=1)
     _, g = O.loss_and_grad(ops, theta, x, labels, lengths)
