@@ -37,6 +37,26 @@ WORKLOAD = "vgg"
 WORKLOAD_DESC = ("VGG-style server part: 10 devices, bf16 activations [64,128,16,16] = ReLU(N(0,1)), "
                  "2x(conv3x3 ->256, ReLU), maxpool2, 2x(conv3x3 ->512, ReLU), maxpool2, FC 8192->512->10, "
                  "softmax-CE, SGD lr 0.01 momentum 0.9; 1M-param device model aggregated each step")
+OTHER_DESC = {
+    "resnet": "ResNet-18 stages 3-4 server part: 20 devices, bf16 activations [128,128,16,16] = ReLU(N(0,1)), "
+              "basic blocks 128->256 (stride 2), 256, 256->512 (stride 2), 512 with folded batch norms, avgpool, "
+              "FC 512->100, softmax-CE, SGD lr 0.01 momentum 0.9",
+    "transformer": "Transformer encoder server part: 16 devices, bf16 activations [32,128,512] ~ N(0,1) with "
+                   "lengths 32..128, 4 pre-LN blocks (8 heads, FFN 2048, GELU), masked mean-pool, FC 512->2, "
+                   "softmax-CE, SGD lr 0.01 momentum 0.9",
+    "scale": "ResNet-18 stages 3-4 server part with 100 devices (Zipf rates), bf16 activations [64,128,16,16], "
+             "omega 400, FC 512->100, softmax-CE, SGD lr 0.01 momentum 0.9",
+    "mobilenet": "MobileNetV3-Large server part: 10 devices, bf16 activations [64,112,4,4] = ReLU(N(0,1)), "
+                 "BNECK-5-160 x3 (first stride 2; 1x1 expand, 5x5 depthwise, squeeze-and-excite, 1x1 project, "
+                 "hard swish), CONV-1-960, avgpool, FC 960->1280, hard swish, FC 1280->10, softmax-CE, "
+                 "SGD lr 0.01 momentum 0.9",
+}
+
+
+def workload_desc(name):
+    return WORKLOAD_DESC if name == WORKLOAD else OTHER_DESC.get(name, name)
+
+
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -191,7 +211,7 @@ def run_reference(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
-        "config": {"workload": WORKLOAD_DESC, "sample": f"{batch} of the 64 samples per step"},
+        "config": {"workload": workload_desc(args.workload), "sample": f"{batch} of the {cfg['batch']} samples per step"},
         "cpu_baseline": {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
                          "sample": f"{args.steps} oracle server steps at batch {batch} (numpy fp64, BLAS threads = cores)"},
         "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -405,7 +425,7 @@ def run_ours(args):
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": WORKLOAD_DESC, "global_batch": B * world, "devices": cfg["K"],
+        "config": {"workload": workload_desc(args.workload), "global_batch": B * world, "devices": cfg["K"],
                    "omega": cfg["omega"], "parallelism": f"replicas{world}",
                    "l2": f"not flushed: each step touches the server's {wsb / 1e6:.0f} MB of parameters, "
                          f"momentum, gradients, activations and scratch, above the 126 MB L2"},

@@ -69,19 +69,25 @@ enum {
   FO_OP_LAYERNORM = 9, /* over the last dim, eps 1e-5, biased variance.  params gamma[c], beta[c]               */
   FO_OP_GELU = 10,     /* exact GELU x * Phi(x)                                                                 */
   FO_OP_ATTENTION = 11,/* in0 = [B, L, 3c] packed q|k|v; `heads` heads of c/heads; keys >= length masked          */
-  FO_OP_MEANPOOL = 12  /* mean over the first length[b] tokens: [B, L, c] -> [B, c]                              */
+  FO_OP_MEANPOOL = 12, /* mean over the first length[b] tokens: [B, L, c] -> [B, c]                              */
+  /* MobileNetV3 bottleneck ops (the MobileNetV3-Large split of Table 2):                                       */
+  FO_OP_DWCONV = 13,   /* depthwise k x k (k odd, <= 7), stride 1|2, pad k/2, channels cin.  params W[cin][k][k],
+                          b[cin] if bias                                                                        */
+  FO_OP_HSWISH = 14,   /* hard swish x * relu6(x + 3) / 6; derivative 0 below -3, (2x + 3) / 6 on [-3, 3], 1 above */
+  FO_OP_HSIGMOID = 15, /* hard sigmoid relu6(x + 3) / 6; derivative 1/6 strictly inside (-3, 3), else 0          */
+  FO_OP_CHMUL = 16     /* squeeze-and-excite scaling y[b,h,w,c] = in0[b,h,w,c] * in1[b,c] (in1 is [B, 1, 1, C])    */
 };
 
 typedef struct fo_op {
   int32_t kind;    /* FO_OP_*                                                   */
   int32_t in0;     /* tensor id of the (first) input, 0 <= in0 <= op index     */
-  int32_t in1;     /* second input of FO_OP_ADD, else ignored                  */
+  int32_t in1;     /* second input of FO_OP_ADD / FO_OP_CHMUL, else ignored    */
   int32_t cin;     /* conv/linear input channels; channels c of affine,
-                      layernorm and attention                                 */
+                      layernorm, attention and the depthwise convolution      */
   int32_t cout;    /* conv/linear output channels                             */
-  int32_t k;       /* conv kernel size                                         */
-  int32_t stride;  /* conv stride                                              */
-  int32_t bias;    /* conv/linear: 1 if the op has a bias                      */
+  int32_t k;       /* conv / depthwise conv kernel size                        */
+  int32_t stride;  /* conv / depthwise conv stride                             */
+  int32_t bias;    /* conv/linear/depthwise conv: 1 if the op has a bias       */
   int32_t heads;   /* attention heads                                           */
 } fo_op;
 

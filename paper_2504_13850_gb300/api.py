@@ -22,7 +22,7 @@ STATUS = {0: "OK", 1: "EMPTY", 2: "FULL", 3: "STALE", -1: "ERR_ARG", -2: "ERR_CU
 
 OP_KINDS = {"conv": 1, "affine": 2, "relu": 3, "maxpool2": 4, "add": 5, "avgpool": 6,
             "flatten": 7, "linear": 8, "layernorm": 9, "gelu": 10, "attention": 11,
-            "meanpool": 12}
+            "meanpool": 12, "dwconv": 13, "hswish": 14, "hsigmoid": 15, "chmul": 16}
 DTYPE_F32, DTYPE_BF16 = 0, 1
 SCHED_COUNTER, SCHED_FIFO = 0, 1
 

@@ -157,6 +157,33 @@ int layernorm_bwd8_blocks(int64_t rows);
 void layernorm_bwd8_pass(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
                          void* dx, int64_t rows, int C, bool acc, float* p_gamma, float* p_beta, cudaStream_t st);
 
+// ---- MobileNetV3 bottleneck (k_mobile.cu) ----
+// Depthwise k x k convolution, NHWC, weights [C][k][k] in the activation
+// dtype `dt`, bias fp32 or null, padding `pad`.
+struct DwShape {
+  int N, H, W, C, k, stride, pad, Ho, Wo;
+};
+void dwconv_fwd(const DwShape& d, const void* x, const void* w, const float* bias, void* y, int dt,
+                cudaStream_t st);
+// dx (+)= transposed depthwise convolution of dy.
+void dwconv_dgrad(const DwShape& d, const void* dy, const void* w, void* dx, int dt, bool acc, cudaStream_t st);
+// Per-chunk partials of dW ([chunks][C*k*k]) and, when pb is given, of the
+// bias gradient ([chunks][C]); chunks = dwconv_wgrad_chunks(d).
+int dwconv_wgrad_chunks(const DwShape& d);
+void dwconv_wgrad_pass(const DwShape& d, const void* dy, const void* x, int dt, float* pw, float* pb,
+                       cudaStream_t st);
+// Hard swish x * relu6(x + 3) / 6 and hard sigmoid relu6(x + 3) / 6; the
+// backward kernels take the forward input x: dx (+)= dy * f'(x).
+void hswish_fwd(const void* x, void* y, int64_t n, int dt, cudaStream_t st);
+void hswish_bwd(const void* x, const void* dy, void* dx, int64_t n, int dt, bool acc, cudaStream_t st);
+void hsigmoid_fwd(const void* x, void* y, int64_t n, int dt, cudaStream_t st);
+void hsigmoid_bwd(const void* x, const void* dy, void* dx, int64_t n, int dt, bool acc, cudaStream_t st);
+// Squeeze-and-excite scaling y[n,p,c] = x[n,p,c] s[n,c] (s is [N, C]);
+// backward dx (+)= dy s and ds (+)= sum_p dy x (either output may be null).
+void chmul_fwd(const void* x, const void* s, void* y, int N, int HW, int C, int dt, cudaStream_t st);
+void chmul_bwd(const void* x, const void* s, const void* dy, void* dx, bool acc_dx, void* ds, bool acc_ds, int N,
+               int HW, int C, int dt, cudaStream_t st);
+
 // FedAsync update: g = fmaf(alpha, l - g, g).
 void axpby(float* g, const float* l, int64_t n, float alpha, cudaStream_t st);
 // Number of kernels axpby launches for these arguments (vector body, tail).

@@ -133,12 +133,32 @@ int infer(fo_server* s) {
         if (a.W != 1 || !c.seq) return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": meanpool shape");
         o.H = 1;
         break;
+      case FO_OP_DWCONV: {
+        if (a.C != op.cin || op.k < 1 || op.k > 7 || op.k % 2 == 0 || (op.stride != 1 && op.stride != 2))
+          return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": bad depthwise conv");
+        int pad = op.k / 2;
+        o.H = (a.H + 2 * pad - op.k) / op.stride + 1;
+        o.W = (a.W + 2 * pad - op.k) / op.stride + 1;
+        add_seg(i, int64_t(op.cin) * op.k * op.k);
+        if (op.bias) add_seg(i, op.cin);
+        break;
+      }
+      case FO_OP_HSWISH:
+      case FO_OP_HSIGMOID:
+        break;
+      case FO_OP_CHMUL: {
+        if (op.in1 < 0 || op.in1 > i) return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": bad in1");
+        const Tensor& b = s->T[op.in1];
+        if (b.N != a.N || b.H != 1 || b.W != 1 || b.C != a.C)
+          return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": channel scale must be [B, 1, 1, C]");
+        break;
+      }
       default:
         return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": unknown kind");
     }
     s->T[i + 1] = o;
     s->T[op.in0].consumers++;
-    if (op.kind == FO_OP_ADD) s->T[op.in1].consumers++;
+    if (op.kind == FO_OP_ADD || op.kind == FO_OP_CHMUL) s->T[op.in1].consumers++;
   }
   const fo_op& last = s->ops.back();
   const Tensor& lt = s->T.back();
@@ -161,6 +181,13 @@ fo::ConvShape conv_shape(const fo_server* s, int i) {
   if (op.kind == FO_OP_LINEAR)
     return {int(a.rows()), 1, 1, op.cin, op.cout, 1, 1, 0, 1, 1};
   return {a.N, a.H, a.W, op.cin, op.cout, op.k, op.stride, op.k / 2, o.H, o.W};
+}
+
+fo::DwShape dw_shape(const fo_server* s, int i) {
+  const fo_op& op = s->ops[i];
+  const Tensor& a = s->T[op.in0];
+  const Tensor& o = s->T[i + 1];
+  return {a.N, a.H, a.W, op.cin, op.k, op.stride, op.k / 2, o.H, o.W};
 }
 
 // Which kernels absorb which neighbouring work (decided once per network).
@@ -344,6 +371,33 @@ int build_plan(fo_server* s) {
           fo::meanpool_fwd(act(a), s->cur_len, s->T[o].act, x.N, x.H, x.C, dt, st);
         });
         break;
+      case FO_OP_DWCONV: {
+        const fo::DwShape d = dw_shape(s, i);
+        add("dwconv_fwd", 1, 2.0 * double(to.numel()) * op.k * op.k, tbytes(a) + tbytes(o), [=](cudaStream_t st) {
+          // the bf16 path multiplies the bf16 copy of the weights, like the convolutions
+          const void* w = dt == fo::kBF16 ? (const void*)SH(s, i, 0) : (const void*)P(s, i, 0);
+          fo::dwconv_fwd(d, act(a), w, op.bias ? P(s, i, 1) : nullptr, s->T[o].act, dt, st);
+        });
+        break;
+      }
+      case FO_OP_HSWISH:
+        add("hswish_fwd", 1, 0.0, 2 * tbytes(a), [=](cudaStream_t st) {
+          fo::hswish_fwd(act(a), s->T[o].act, s->T[a].numel(), dt, st);
+        });
+        break;
+      case FO_OP_HSIGMOID:
+        add("hsigmoid_fwd", 1, 0.0, 2 * tbytes(a), [=](cudaStream_t st) {
+          fo::hsigmoid_fwd(act(a), s->T[o].act, s->T[a].numel(), dt, st);
+        });
+        break;
+      case FO_OP_CHMUL: {
+        const int b = op.in1;
+        add("chmul_fwd", 1, 0.0, 2 * tbytes(a) + tbytes(b), [=](cudaStream_t st) {
+          const Tensor& x = s->T[a];
+          fo::chmul_fwd(act(a), act(b), s->T[o].act, x.N, x.H * x.W, x.C, dt, st);
+        });
+        break;
+      }
     }
   }
 
@@ -613,6 +667,58 @@ int build_plan(fo_server* s) {
           });
         }
         break;
+      case FO_OP_DWCONV: {
+        const fo::DwShape d = dw_shape(s, i);
+        const int kk = op.k * op.k;
+        const double fl = 2.0 * double(s->T[o].numel()) * kk;
+        if (need_dx) {
+          int accf = contrib(a);
+          add("dwconv_dgrad", 1, fl, (1 + accf) * tbytes(a) + csb, [=](cudaStream_t st) {
+            const void* w = dt == fo::kBF16 ? (const void*)SH(s, i, 0) : (const void*)P(s, i, 0);
+            fo::dwconv_dgrad(d, s->T[o].grad, w, s->T[a].grad, dt, accf != 0, st);
+          });
+        }
+        // weight (and bias) gradient partials, summed by the batched finish
+        const int chunks = fo::dwconv_wgrad_chunks(d);
+        float* pw = (float*)s->alloc(size_t(chunks) * op.cin * (kk + (op.bias ? 1 : 0)) * 4);
+        if (!pw) return set_err(FO_ERR_OOM, "depthwise weight-gradient partials");
+        float* pb = op.bias ? pw + size_t(chunks) * op.cin * kk : nullptr;
+        finish_tasks.push_back({pw, G(s, i, 0), chunks, op.cin * kk});
+        if (pb) finish_tasks.push_back({pb, G(s, i, 1), chunks, op.cin});
+        add("dwconv_wgrad", 1, fl, tbytes(a0) + csb, [=](cudaStream_t st) {
+          fo::dwconv_wgrad_pass(d, s->T[o].grad, act(a0), dt, pw, pb, st);
+        });
+        break;
+      }
+      case FO_OP_HSWISH:
+        if (need_dx) {
+          int accf = contrib(a);
+          add("hswish_bwd", 1, 0.0, (3 + accf) * csb, [=](cudaStream_t st) {
+            fo::hswish_bwd(act(a0), s->T[o].grad, s->T[a].grad, s->T[a].numel(), dt, accf != 0, st);
+          });
+        }
+        break;
+      case FO_OP_HSIGMOID:
+        if (need_dx) {
+          int accf = contrib(a);
+          add("hsigmoid_bwd", 1, 0.0, (3 + accf) * csb, [=](cudaStream_t st) {
+            fo::hsigmoid_bwd(act(a0), s->T[o].grad, s->T[a].grad, s->T[a].numel(), dt, accf != 0, st);
+          });
+        }
+        break;
+      case FO_OP_CHMUL: {
+        const int b = op.in1;
+        const int acc_dx = need_dx ? contrib(a0) : 0;
+        const bool need_ds = b != 0;
+        const int acc_ds = need_ds ? contrib(b) : 0;
+        add("chmul_bwd", 1, 0.0, (2 + (need_dx ? 1 + acc_dx : 0)) * csb + (1 + acc_ds) * tbytes(b),
+            [=](cudaStream_t st) {
+              const Tensor& x = s->T[a0];
+              fo::chmul_bwd(act(a0), act(b), s->T[o].grad, need_dx ? s->T[a0].grad : nullptr, acc_dx != 0,
+                            need_ds ? s->T[b].grad : nullptr, acc_ds != 0, x.N, x.H * x.W, x.C, dt, st);
+            });
+        break;
+      }
     }
   }
 

@@ -79,8 +79,11 @@ __device__ __forceinline__ size_t out_row(const TcParams& p, int m) {
 // Epilogue of 32 consecutive outputs (m, n..n+31) held by one thread: bias,
 // ReLU, ReLU mask, accumulate, store as fp32 or bf16 (16-byte accesses).
 // `sbias`: shared-memory address of the bias values for columns n..n+31.
+// Columns >= N (the ragged last tile; N is a multiple of 8) are not touched.
 __device__ __forceinline__ void store_row32(const TcParams& p, int m_gemm, int n, float (&v)[32], uint32_t sbias) {
   const size_t m = out_row(p, m_gemm);
+  const int nv = p.N - n;   // valid columns from n
+  if (nv <= 0) return;
   if (p.bias) {
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
@@ -95,6 +98,7 @@ __device__ __forceinline__ void store_row32(const TcParams& p, int m_gemm, int n
     const uint4* mk = reinterpret_cast<const uint4*>(p.mask + m * p.ldo + n);
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
+      if (8 * j >= nv) break;
       const uint4 u = mk[j];
       const bf16* e = reinterpret_cast<const bf16*>(&u);
 #pragma unroll
@@ -106,6 +110,7 @@ __device__ __forceinline__ void store_row32(const TcParams& p, int m_gemm, int n
     float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + m * p.ldo + n);
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
+      if (4 * j >= nv) break;
       if (p.acc) {
         const float4 o = dst[j];
         v[4 * j] += o.x; v[4 * j + 1] += o.y; v[4 * j + 2] += o.z; v[4 * j + 3] += o.w;
@@ -116,6 +121,7 @@ __device__ __forceinline__ void store_row32(const TcParams& p, int m_gemm, int n
     uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(p.out) + m * p.ldo + n);
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
+      if (8 * j >= nv) break;
       if (p.acc) {
         const uint4 o = dst[j];
         const bf16* ob = reinterpret_cast<const bf16*>(&o);
@@ -146,7 +152,7 @@ __device__ __forceinline__ void store_row32(const TcParams& p, int m_gemm, int n
 // 4 * (lane % 8) for fp32 outputs (zeros without a bias).
 __device__ __forceinline__ void load_bias8(const TcParams& p, int lane, int n, float (&b)[8]) {
   float4 b0 = make_float4(0.f, 0.f, 0.f, 0.f), b1 = b0;
-  if (p.bias) {
+  if (p.bias && n + (p.out_f32 ? 4 * (lane & 7) : 8 * (lane & 3)) < p.N) {
     const float4* src = reinterpret_cast<const float4*>(p.bias + n);
     if (p.out_f32) {
       b0 = __ldg(src + (lane & 7));
@@ -171,7 +177,7 @@ __device__ __forceinline__ void epilogue_chunk32(const TcParams& p, uint32_t sta
       const int rr = it * 4 + (lane >> 3);
       const int mg = m_base + rr;
       const float4 v = ld_shared4(stage + 16u * (rr * 8 + (cq ^ (rr & 7))));
-      if (mg < p.M) {
+      if (mg < p.M && n + 4 * cq < p.N) {
         const size_t m = out_row(p, mg);
         float e[4] = {v.x + b[0], v.y + b[1], v.z + b[2], v.w + b[3]};
         if (p.relu)
@@ -200,7 +206,7 @@ __device__ __forceinline__ void epilogue_chunk32(const TcParams& p, uint32_t sta
       const int mg = m_base + rr;
       const float4 v0 = ld_shared4(stage + 16u * (rr * 8 + ((2 * co) ^ (rr & 7))));
       const float4 v1 = ld_shared4(stage + 16u * (rr * 8 + ((2 * co + 1) ^ (rr & 7))));
-      if (mg < p.M) {
+      if (mg < p.M && n + 8 * co < p.N) {
         const size_t m = out_row(p, mg);
         float e[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
 #pragma unroll
@@ -406,7 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     }
   } else {
     // the tile's bias into shared memory while the MMAs run
-    for (int j = threadIdx.x - 64; j < BN; j += 128) sbias[j] = p.bias ? p.bias[n0 + j] : 0.f;
+    for (int j = threadIdx.x - 64; j < BN; j += 128) sbias[j] = p.bias && n0 + j < p.N ? p.bias[n0 + j] : 0.f;
     if (!mbar_wait(accum, 0)) atomicExch(p.err, 3);
     tc_fence_after();
   }
@@ -510,7 +516,7 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
   const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
   const int unit = PAIR ? int(blockIdx.x) / 2 : int(blockIdx.x);
   const int units = PAIR ? int(gridDim.x) / 2 : int(gridDim.x);
-  const int n_tiles = p.N / BN, m_tiles = (p.M + BM - 1) / BM;
+  const int n_tiles = (p.N + BN - 1) / BN, m_tiles = (p.M + BM - 1) / BM;
   const int su_n = PAIR == 1 ? n_tiles / 2 : n_tiles;   // work units: tiles, or tile pairs
   const int tiles = su_n * (PAIR == 2 ? m_tiles / 2 : m_tiles);
   const int KB = p.KB;
@@ -873,8 +879,9 @@ void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv, bool 
   double best = 1e30;
   int best_bn = 0, best_s = 1, best_pair = 0;
   for (int bn : {256, 128, 64}) {
-    if (ndiv % bn || N % bn) continue;
-    const int n_tiles = N / bn, m_tiles = (M + BM - 1) / BM, tiles = n_tiles * m_tiles;
+    // window kinds tile whole taps; the plain GEMMs take a ragged last tile
+    if ((win_a || win_b) && (ndiv % bn || N % bn)) continue;
+    const int n_tiles = (N + bn - 1) / bn, m_tiles = (M + BM - 1) / BM, tiles = n_tiles * m_tiles;
     const double stage_kb = (BM + bn) * BK * 2 / 1024.0;
     const double epi = bn == 256 ? 4.2 : (bn == 128 ? 2.2 : 1.5);
     for (int pair = 0; pair <= 2; ++pair) {
@@ -931,13 +938,14 @@ TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
     delete g;
     return nullptr;
   }
+  const int n_tiles = (N + g->bn - 1) / g->bn;
   if (g->splits > 1) {
-    g->grid = dim3(N / g->bn, (M + BM - 1) / BM, g->splits);
+    g->grid = dim3(n_tiles, (M + BM - 1) / BM, g->splits);
   } else if (g->pair) {
-    const int work = (N / g->bn) * ((M + BM - 1) / BM) / 2;
+    const int work = n_tiles * ((M + BM - 1) / BM) / 2;
     g->grid = dim3(2 * std::min(work, active_clusters(c, g->kind, g->bn, 2, g->pair)), 1, 1);
   } else {
-    const int tiles = (N / g->bn) * ((M + BM - 1) / BM);
+    const int tiles = n_tiles * ((M + BM - 1) / BM);
     g->grid = dim3(std::min(tiles, c->num_sms), 1, 1);
   }
   if (getenv("FO_DEBUG_PLAN"))
@@ -992,6 +1000,15 @@ int tc_finalize(TcContext* c) {
 
 static const void* tensor_act(fo_server* s, int tid) { return s->T[tid].act; }
 
+// Linear layers and 1x1 stride-1 convolutions are one plain GEMM over the
+// rows of an NHWC tensor.  Channel counts need only be multiples of 8 (rows
+// of 16 bytes for the tensor maps): a ragged contraction block is zero-filled
+// by the TMA, and a ragged last output tile is masked in the epilogue.
+static bool plain_gemm(const fo_op& op) {
+  return op.kind == FO_OP_LINEAR || (op.kind == FO_OP_CONV && op.k == 1 && op.stride == 1);
+}
+static bool plain_gemm_ok(const fo_op& op) { return op.cin % 8 == 0 && op.cout % 8 == 0; }
+
 TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i, void* out, bool relu) {
   if (!c || !bf16_server(s) || getenv("FO_NO_TC")) return nullptr;
   const fo_op& op = s->ops[i];
@@ -1004,11 +1021,11 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i, void* out, bool relu)
   g->p.relu = relu ? 1 : 0;
   g->p.bias = op.bias ? s->theta + s->segs[s->op_segs[i][1]].off : nullptr;
   const bf16* w = s->shadow + s->segs[s->op_segs[i][0]].off;
-  if (op.kind == FO_OP_LINEAR) {
-    if (op.cout % 64 || op.cin % 64) { delete g; return nullptr; }
+  if (plain_gemm(op)) {
+    if (!plain_gemm_ok(op)) { delete g; return nullptr; }
     g->kind = LIN_FWD;
-    g->name = "tc_linear_fwd";
-    int M = int(a.rows()), KB = op.cin / 64;
+    g->name = op.kind == FO_OP_LINEAR ? "tc_linear_fwd" : "tc_conv1x1_fwd";
+    int M = int(a.rows()), KB = (op.cin + 63) / 64;
     choose_tiles(c, g, M, op.cout, KB, op.cout, false);
     const int bn = g->bn;
     g->input_A = (op.in0 == 0);
@@ -1068,12 +1085,12 @@ bool tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate, void* dx, 
     g->p.mask = static_cast<const bf16*>(mask);
     return g;
   };
-  if (op.kind == FO_OP_LINEAR) {
-    if (op.cin % 64 || op.cout % 64) return false;
+  if (plain_gemm(op)) {
+    if (!plain_gemm_ok(op)) return false;
     TcGemm* g = base();
     g->kind = LIN_DGRAD;
-    g->name = "tc_linear_dgrad";
-    int M = int(a.rows()), KB = op.cout / 64;
+    g->name = op.kind == FO_OP_LINEAR ? "tc_linear_dgrad" : "tc_conv1x1_dgrad";
+    int M = int(a.rows()), KB = (op.cout + 63) / 64;
     choose_tiles(c, g, M, op.cin, KB, op.cin, false);
     if (!map_2d(&g->p.tmA, o.grad, M, op.cout, BM) || !map_2d(&g->p.tmB, w, op.cout, op.cin, BK)) { delete g; return false; }
     if (!finish(c, g, M, op.cin, double(op.cout))) return false;
@@ -1158,10 +1175,10 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
   TcGemm* g = new TcGemm();
   g->p.out = s->grad + s->segs[s->op_segs[i][0]].off;
   g->p.out_f32 = 1;
-  if (op.kind == FO_OP_LINEAR) {
-    if (op.cin % 64 || op.cout % 128) { delete g; return nullptr; }
+  if (plain_gemm(op)) {
+    if (!plain_gemm_ok(op)) { delete g; return nullptr; }
     g->kind = LIN_WGRAD;
-    g->name = "tc_linear_wgrad";
+    g->name = op.kind == FO_OP_LINEAR ? "tc_linear_wgrad" : "tc_conv1x1_wgrad";
     g->p.ldo = op.cin;
     int rows = int(a.rows()), KB = (rows + BK - 1) / BK;
     choose_tiles(c, g, op.cout, op.cin, KB, op.cin, false);

@@ -1,4 +1,4 @@
-"""The four bf16 workloads at their full sizes, in the launch configuration
+"""The five bf16 workloads at their full sizes, in the launch configuration
 the benchmark times (same server plan, tiles and cluster splits): scheduler
 outcomes bit-exact, and two teacher-forced steps against the oracle (loss
 1e-2, parameters 2e-2 against the exact fp64 definition; per-tensor
@@ -25,7 +25,7 @@ def events(cfg, uploaders, steps):
     return [("enq", k) for k in range(uploaders)] + [("step",)] * steps
 
 
-@pytest.mark.parametrize("name", ["vgg", "resnet", "transformer", "scale"])
+@pytest.mark.parametrize("name", ["vgg", "resnet", "transformer", "scale", "mobilenet"])
 def test_full_size_teacher_forced(name):
     cfg = W.CONFIGS[name]
     ev = events(cfg, min(cfg["K"], 3), 2)
