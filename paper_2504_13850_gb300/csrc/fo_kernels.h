@@ -141,10 +141,15 @@ int colsum8_batch_chunks(int64_t rows);
 void colsum8_batched(const std::vector<ColsumTask>& tasks, cudaStream_t st);
 void finish_batched(const std::vector<FinishTask>& tasks, cudaStream_t st);
 // Affine backward pass without its finish: partials of dscale and dshift
-// ([affine_bwd8_chunks(rows, C), C] each) and dx (+)= dy * scale.
+// ([affine_bwd8_chunks(rows, C), C] each) and dx (+)= dy * scale.  With
+// `hswish_in` (the affine output feeding a hard swish) dy is the gradient of
+// the hard swish's output and the pass applies hswish'(hswish_in) first.
 int affine_bwd8_chunks(int64_t rows, int C);
 void affine_bwd8_pass(const void* dy, const void* x, const float* scale, void* dx, bool acc, int64_t rows, int C,
-                      float* p_scale, float* p_shift, cudaStream_t st);
+                      float* p_scale, float* p_shift, cudaStream_t st, const void* hswish_in = nullptr);
+// Affine then hard swish in one pass: pre = x * scale + shift, post = hswish(pre).
+void affine_hswish_fwd_x8(const void* x, const float* sc, const float* sh, void* pre, void* post, int64_t n, int C,
+                          cudaStream_t st);
 // Layernorm backward fused with dgamma / dbeta (C % 256 == 0, C <= 512).
 bool layernorm_bwd8_ok(int dt, int C);
 int64_t layernorm_bwd8_partial_floats(int64_t rows, int C);

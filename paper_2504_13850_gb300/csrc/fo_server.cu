@@ -196,6 +196,8 @@ struct Fusion {
   std::vector<char> skip_fwd;  // relu op whose forward is done by its producer
   std::vector<int> bwd_mask;   // consumer op -> relu op whose mask it applies to its dx, or -1
   std::vector<char> skip_bwd;  // relu op whose backward is done by its consumer
+  std::vector<int> hswish_of;  // affine op -> the hard swish op it applies (both passes), or -1
+  std::vector<int> hswish_by;  // hard swish op -> the affine op that applies it, or -1
   bool head = false;           // last linear + loss handled by the head kernels
 };
 
@@ -211,6 +213,8 @@ Fusion analyse(const fo_server* s) {
   f.skip_fwd.assign(nops, 0);
   f.bwd_mask.assign(nops, -1);
   f.skip_bwd.assign(nops, 0);
+  f.hswish_of.assign(nops, -1);
+  f.hswish_by.assign(nops, -1);
   std::vector<int> sole(nops + 1, -1);  // the only consumer op of a tensor
   for (int j = 0; j < nops; ++j) {
     const fo_op& op = s->ops[j];
@@ -233,6 +237,20 @@ Fusion analyse(const fo_server* s) {
     if (j >= 0 && s->ops[j].in0 == r + 1 && (dx_takes_mask(s, j) || (f.head && j == nops - 1))) {
       f.bwd_mask[j] = r;
       f.skip_bwd[r] = 1;
+    }
+  }
+  // A batch-norm affine whose only consumer is a hard swish (the MobileNetV3
+  // bottleneck) applies it in both passes, on the vectorised bf16 path.
+  for (int h = 0; h < nops; ++h) {
+    const fo_op& op = s->ops[h];
+    if (op.kind != FO_OP_HSWISH || op.in0 == 0) continue;
+    const int p = op.in0 - 1;
+    const Tensor& t = s->T[op.in0];
+    if (s->ops[p].kind == FO_OP_AFFINE && sole[op.in0] == h && f.fwd_relu[p] < 0 && fo::vec8_ok(s->dt, t.numel()) &&
+        t.C % 8 == 0) {
+      f.hswish_of[p] = h;
+      f.hswish_by[h] = p;
+      f.skip_fwd[h] = 1;
     }
   }
   return f;
@@ -305,6 +323,14 @@ int build_plan(fo_server* s) {
         break;
       }
       case FO_OP_AFFINE:
+        if (fu.hswish_of[i] >= 0) {
+          const int h = fu.hswish_of[i] + 1;   // the hard swish's output tensor
+          add("affine_hswish_fwd", 1, 0.0, 3 * tbytes(a), [=](cudaStream_t st) {
+            fo::affine_hswish_fwd_x8(act(a), P(s, i, 0), P(s, i, 1), s->T[o].act, s->T[h].act, s->T[a].numel(),
+                                     s->T[a].C, st);
+          });
+          break;
+        }
         add("affine_fwd", 1, 0.0, 2 * tbytes(a), [=](cudaStream_t st) {
           fo::affine_fwd(act(a), P(s, i, 0), P(s, i, 1), s->T[o].act, s->T[a].rows(), s->T[a].C, dt, relu, st);
         });
@@ -433,6 +459,12 @@ int build_plan(fo_server* s) {
       written[s->T[i + 1].root] = 1;
       continue;
     }
+    if (fu.hswish_by[i] >= 0) {
+      // the affine's backward applies this hard swish: its input gradient is
+      // present exactly when the output's is
+      written[s->T[op.in0].root] = written[s->T[i + 1].root];
+      continue;
+    }
     const int a0 = op.in0, o = i + 1;
     const int ro = s->T[o].root;
     if (!written[ro]) {
@@ -525,7 +557,10 @@ int build_plan(fo_server* s) {
       }
       case FO_OP_AFFINE:
         if (fo::vec8_ok(dt, s->T[a0].numel()) && s->T[a0].C % 8 == 0) {
-          // one pass: dscale, dshift and dx (+)= dy * scale
+          // one pass: dscale, dshift and dx (+)= dy * scale; behind a fused
+          // hard swish, dy is formed from the hard swish's output gradient
+          const int hs = fu.hswish_of[i];
+          const int dyt = hs >= 0 ? hs + 1 : o;
           const int accf = need_dx ? contrib(a) : 0;
           const Tensor& x0 = s->T[a0];
           const int chunks = fo::affine_bwd8_chunks(x0.rows(), x0.C);
@@ -534,11 +569,12 @@ int build_plan(fo_server* s) {
           float* ph = ps + size_t(chunks) * x0.C;
           finish_tasks.push_back({ps, G(s, i, 0), chunks, x0.C});
           finish_tasks.push_back({ph, G(s, i, 1), chunks, x0.C});
-          add("affine_bwd", 1, 0.0, (need_dx ? 3 + accf : 2) * csb, [=](cudaStream_t st) {
-            const Tensor& x = s->T[a0];
-            fo::affine_bwd8_pass(s->T[o].grad, act(a0), P(s, i, 0), need_dx ? s->T[a].grad : nullptr, accf != 0,
-                                 x.rows(), x.C, ps, ph, st);
-          });
+          add(hs >= 0 ? "affine_hswish_bwd" : "affine_bwd", 1, 0.0, (need_dx ? 3 + accf : 2) * csb + (hs >= 0) * csb,
+              [=](cudaStream_t st) {
+                const Tensor& x = s->T[a0];
+                fo::affine_bwd8_pass(s->T[dyt].grad, act(a0), P(s, i, 0), need_dx ? s->T[a].grad : nullptr, accf != 0,
+                                     x.rows(), x.C, ps, ph, st, hs >= 0 ? s->T[o].act : nullptr);
+              });
           break;
         }
         add("affine_pgrad", 4, 0.0, 3 * csb, [=](cudaStream_t st) {

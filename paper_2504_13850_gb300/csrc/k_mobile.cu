@@ -8,6 +8,8 @@
 #include "fo_common.cuh"
 #include "fo_kernels.h"
 
+#include <algorithm>
+
 namespace fo {
 
 namespace {
@@ -33,13 +35,17 @@ __device__ __forceinline__ void store_acc(T* p, int64_t i, float v, bool acc) {
 }
 
 // --------------------------------------------------------- depthwise conv
+// KT is the kernel size when known at compile time (3 or 5: the tap loops
+// unroll, so a thread's loads are independent), or 0 for a runtime d.k.
+
 // y[n,i,j,c] = b[c] + sum_{r,s} xpad[n, i*st + r, j*st + s, c] * w[c,r,s],
 // w [C][k][k] in the activation type (the bf16 path multiplies the bf16
 // copy of the weights), zero padding `pad` on each side.
-template <typename T>
+template <typename T, int KT>
 __global__ void __launch_bounds__(256) dwconv_fwd_k(const T* __restrict__ x, const T* __restrict__ w,
                                                     const float* __restrict__ bias, T* __restrict__ y,
                                                     DwShape d) {
+  const int K = KT ? KT : d.k;
   const int64_t n_out = int64_t(d.N) * d.Ho * d.Wo * d.C;
   FO_MB_GRID_STRIDE(idx, n_out) {
     const int c = int(idx % d.C);
@@ -47,15 +53,17 @@ __global__ void __launch_bounds__(256) dwconv_fwd_k(const T* __restrict__ x, con
     const int j = int(p % d.Wo);
     const int i = int((p / d.Wo) % d.Ho);
     const int64_t n = p / (int64_t(d.Wo) * d.Ho);
-    const T* wc = w + int64_t(c) * d.k * d.k;
+    const T* wc = w + int64_t(c) * K * K;
     float acc = bias ? bias[c] : 0.f;
-    for (int r = 0; r < d.k; ++r) {
+#pragma unroll
+    for (int r = 0; r < (KT ? KT : K); ++r) {
       const int h = i * d.stride - d.pad + r;
       if (h < 0 || h >= d.H) continue;
-      for (int s = 0; s < d.k; ++s) {
+#pragma unroll
+      for (int s = 0; s < (KT ? KT : K); ++s) {
         const int ww = j * d.stride - d.pad + s;
         if (ww < 0 || ww >= d.W) continue;
-        acc = fmaf(to_f(x[((n * d.H + h) * d.W + ww) * d.C + c]), to_f(wc[r * d.k + s]), acc);
+        acc = fmaf(to_f(x[((n * d.H + h) * d.W + ww) * d.C + c]), to_f(wc[r * K + s]), acc);
       }
     }
     y[idx] = from_f<T>(acc);
@@ -65,9 +73,10 @@ __global__ void __launch_bounds__(256) dwconv_fwd_k(const T* __restrict__ x, con
 // dx[n,h,w,c] (+)= sum over the taps (r,s) whose output position
 // i = (h + pad - r) / st, j = (w + pad - s) / st is whole and in range of
 // dy[n,i,j,c] * w[c,r,s].
-template <typename T>
+template <typename T, int KT>
 __global__ void __launch_bounds__(256) dwconv_dgrad_k(const T* __restrict__ dy, const T* __restrict__ w,
                                                       T* __restrict__ dx, DwShape d, int acc_flag) {
+  const int K = KT ? KT : d.k;
   const int64_t n_in = int64_t(d.N) * d.H * d.W * d.C;
   FO_MB_GRID_STRIDE(idx, n_in) {
     const int c = int(idx % d.C);
@@ -75,19 +84,21 @@ __global__ void __launch_bounds__(256) dwconv_dgrad_k(const T* __restrict__ dy, 
     const int wx = int(p % d.W);
     const int h = int((p / d.W) % d.H);
     const int64_t n = p / (int64_t(d.W) * d.H);
-    const T* wc = w + int64_t(c) * d.k * d.k;
+    const T* wc = w + int64_t(c) * K * K;
     float acc = 0.f;
-    for (int r = 0; r < d.k; ++r) {
+#pragma unroll
+    for (int r = 0; r < (KT ? KT : K); ++r) {
       const int ti = h + d.pad - r;
       if (ti < 0 || ti % d.stride) continue;
       const int i = ti / d.stride;
       if (i >= d.Ho) continue;
-      for (int s = 0; s < d.k; ++s) {
+#pragma unroll
+      for (int s = 0; s < (KT ? KT : K); ++s) {
         const int tj = wx + d.pad - s;
         if (tj < 0 || tj % d.stride) continue;
         const int j = tj / d.stride;
         if (j >= d.Wo) continue;
-        acc = fmaf(to_f(dy[((n * d.Ho + i) * d.Wo + j) * d.C + c]), to_f(wc[r * d.k + s]), acc);
+        acc = fmaf(to_f(dy[((n * d.Ho + i) * d.Wo + j) * d.C + c]), to_f(wc[r * K + s]), acc);
       }
     }
     store_acc(dx, idx, acc, acc_flag != 0);
@@ -98,11 +109,64 @@ __global__ void __launch_bounds__(256) dwconv_dgrad_k(const T* __restrict__ dy, 
 // [q * per, min(rows, (q + 1) * per)) gives
 //   pw[q][c*k*k + r*k + s] = sum_p dy[p,c] * xpad[p's window at (r,s), c]
 //   pb[q][c]               = sum_p dy[p,c]            (when pb is given)
-// One thread per (tap, channel) and chunk; blockIdx.y is the chunk.
-template <typename T>
+// A block covers 32 channels (lane = channel) of one chunk; its 8 warps take
+// every 8th pixel of the chunk with the k*k tap sums in registers, and the
+// warps' sums are added in warp order through shared memory.
+template <typename T, int KT>
 __global__ void __launch_bounds__(256) dwconv_wgrad_k(const T* __restrict__ dy, const T* __restrict__ x,
                                                       float* __restrict__ pw, float* __restrict__ pb, DwShape d,
                                                       int per) {
+  constexpr int KK = KT * KT;
+  __shared__ float red[8][KK + 1][33];
+  const int lane = threadIdx.x % 32, warp = threadIdx.x / 32;
+  const int c = blockIdx.x * 32 + lane;
+  const int64_t rows = int64_t(d.N) * d.Ho * d.Wo;
+  const int64_t p0 = int64_t(blockIdx.y) * per;
+  const int64_t p1 = p0 + per < rows ? p0 + per : rows;
+  float acc[KK + 1];
+#pragma unroll
+  for (int t = 0; t <= KK; ++t) acc[t] = 0.f;
+  if (c < d.C) {
+    for (int64_t p = p0 + warp; p < p1; p += 8) {
+      const int j = int(p % d.Wo);
+      const int i = int((p / d.Wo) % d.Ho);
+      const int64_t n = p / (int64_t(d.Wo) * d.Ho);
+      const float g = to_f(dy[p * d.C + c]);
+      acc[KK] += g;
+#pragma unroll
+      for (int r = 0; r < KT; ++r) {
+        const int h = i * d.stride - d.pad + r;
+        if (h < 0 || h >= d.H) continue;
+#pragma unroll
+        for (int s = 0; s < KT; ++s) {
+          const int ww = j * d.stride - d.pad + s;
+          if (ww < 0 || ww >= d.W) continue;
+          acc[r * KT + s] = fmaf(g, to_f(x[((n * d.H + h) * d.W + ww) * d.C + c]), acc[r * KT + s]);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int t = 0; t <= KK; ++t) red[warp][t][lane] = acc[t];
+  __syncthreads();
+  const int c0 = blockIdx.x * 32;
+  for (int e = threadIdx.x; e < 32 * (KK + 1); e += 256) {
+    // e = (channel, tap): consecutive threads write consecutive floats of pw
+    const int cl = e / (KK + 1), t = e % (KK + 1);
+    if (c0 + cl >= d.C) continue;
+    float sum = 0.f;
+#pragma unroll
+    for (int w8 = 0; w8 < 8; ++w8) sum += red[w8][t][cl];
+    if (t < KK) pw[int64_t(blockIdx.y) * d.C * KK + int64_t(c0 + cl) * KK + t] = sum;
+    else if (pb) pb[int64_t(blockIdx.y) * d.C + c0 + cl] = sum;
+  }
+}
+
+// Any kernel size: one thread per (tap, channel) and chunk.
+template <typename T>
+__global__ void __launch_bounds__(256) dwconv_wgrad_any_k(const T* __restrict__ dy, const T* __restrict__ x,
+                                                          float* __restrict__ pw, float* __restrict__ pb, DwShape d,
+                                                          int per) {
   const int kk = d.k * d.k;
   const int taps = kk + (pb ? 1 : 0);
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
@@ -127,6 +191,17 @@ __global__ void __launch_bounds__(256) dwconv_wgrad_k(const T* __restrict__ dy, 
     for (int64_t p = p0; p < p1; ++p) acc += to_f(dy[p * d.C + c]);
     pb[int64_t(blockIdx.y) * d.C + c] = acc;
   }
+}
+
+int num_sms() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
 }
 
 // ------------------------------------------------- hard swish / sigmoid
@@ -199,21 +274,41 @@ __global__ void chmul_bwd_k(const T* __restrict__ x, const T* __restrict__ sc, c
 void dwconv_fwd(const DwShape& d, const void* x, const void* w, const float* bias, void* y, int dt,
                 cudaStream_t st) {
   const int64_t n = int64_t(d.N) * d.Ho * d.Wo * d.C;
-  FO_MB_DISPATCH(dt, T, dwconv_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (const T*)w, bias,
-                                                                                     (T*)y, d));
+  const int blocks = elementwise_blocks(n, 256);
+  FO_MB_DISPATCH(dt, T, {
+    if (d.k == 3) dwconv_fwd_k<T, 3><<<blocks, 256, 0, st>>>((const T*)x, (const T*)w, bias, (T*)y, d);
+    else if (d.k == 5) dwconv_fwd_k<T, 5><<<blocks, 256, 0, st>>>((const T*)x, (const T*)w, bias, (T*)y, d);
+    else dwconv_fwd_k<T, 0><<<blocks, 256, 0, st>>>((const T*)x, (const T*)w, bias, (T*)y, d);
+  });
 }
 
 void dwconv_dgrad(const DwShape& d, const void* dy, const void* w, void* dx, int dt, bool acc, cudaStream_t st) {
   const int64_t n = int64_t(d.N) * d.H * d.W * d.C;
-  FO_MB_DISPATCH(dt, T, dwconv_dgrad_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)dy, (const T*)w,
-                                                                                       (T*)dx, d, acc ? 1 : 0));
+  const int blocks = elementwise_blocks(n, 256);
+  const int a = acc ? 1 : 0;
+  FO_MB_DISPATCH(dt, T, {
+    if (d.k == 3) dwconv_dgrad_k<T, 3><<<blocks, 256, 0, st>>>((const T*)dy, (const T*)w, (T*)dx, d, a);
+    else if (d.k == 5) dwconv_dgrad_k<T, 5><<<blocks, 256, 0, st>>>((const T*)dy, (const T*)w, (T*)dx, d, a);
+    else dwconv_dgrad_k<T, 0><<<blocks, 256, 0, st>>>((const T*)dy, (const T*)w, (T*)dx, d, a);
+  });
 }
 
+// Pixel chunks of the weight gradient: for k = 3, 5 about two blocks of 32
+// channels per SM, at least 8 pixels (one per warp) per chunk, at most 64
+// chunks; for other k, chunks of 32 pixels.
 int dwconv_wgrad_chunks(const DwShape& d) {
   const int64_t rows = int64_t(d.N) * d.Ho * d.Wo;
-  int64_t q = (rows + 31) / 32;
-  if (q > 64) q = 64;
-  return int(q < 1 ? 1 : q);
+  int64_t q;
+  if (d.k == 3 || d.k == 5) {
+    const int64_t groups = (d.C + 31) / 32;
+    q = (2 * num_sms() + groups - 1) / groups;
+    q = std::min<int64_t>(q, (rows + 7) / 8);
+  } else {
+    q = (rows + 31) / 32;
+  }
+  q = std::max<int64_t>(1, std::min<int64_t>(q, 64));
+  const int64_t per = (rows + q - 1) / q;
+  return int((rows + per - 1) / per);
 }
 
 void dwconv_wgrad_pass(const DwShape& d, const void* dy, const void* x, int dt, float* pw, float* pb,
@@ -221,9 +316,17 @@ void dwconv_wgrad_pass(const DwShape& d, const void* dy, const void* x, int dt, 
   const int64_t rows = int64_t(d.N) * d.Ho * d.Wo;
   const int chunks = dwconv_wgrad_chunks(d);
   const int per = int((rows + chunks - 1) / chunks);
+  if (d.k == 3 || d.k == 5) {
+    dim3 grid(ceil_div(d.C, 32), chunks);
+    FO_MB_DISPATCH(dt, T, {
+      if (d.k == 3) dwconv_wgrad_k<T, 3><<<grid, 256, 0, st>>>((const T*)dy, (const T*)x, pw, pb, d, per);
+      else dwconv_wgrad_k<T, 5><<<grid, 256, 0, st>>>((const T*)dy, (const T*)x, pw, pb, d, per);
+    });
+    return;
+  }
   const int taps = d.k * d.k + (pb ? 1 : 0);
   dim3 grid(ceil_div(int64_t(taps) * d.C, 256), chunks);
-  FO_MB_DISPATCH(dt, T, dwconv_wgrad_k<T><<<grid, 256, 0, st>>>((const T*)dy, (const T*)x, pw, pb, d, per));
+  FO_MB_DISPATCH(dt, T, dwconv_wgrad_any_k<T><<<grid, 256, 0, st>>>((const T*)dy, (const T*)x, pw, pb, d, per));
 }
 
 void hswish_fwd(const void* x, void* y, int64_t n, int dt, cudaStream_t st) {

@@ -95,6 +95,30 @@ __global__ void affine_fwd_x8_k(const bf16* __restrict__ x, const float* __restr
   }
 }
 
+// Batch-norm affine followed by hard swish, both outputs stored: the affine
+// output (the hard swish's input, kept for the backward pass) and the hard
+// swish of its stored bf16 value, exactly as the two separate kernels give.
+__device__ __forceinline__ float round_bf16(float v) { return __bfloat162float(__float2bfloat16_rn(v)); }
+__device__ __forceinline__ float hswish_f(float v) { return v * fminf(fmaxf(v + 3.f, 0.f), 6.f) / 6.f; }
+__device__ __forceinline__ float hswish_d(float v) { return v < -3.f ? 0.f : (v > 3.f ? 1.f : (2.f * v + 3.f) / 6.f); }
+
+__global__ void affine_hswish_fwd_x8_k(const bf16* __restrict__ x, const float* __restrict__ sc,
+                                       const float* __restrict__ sh, bf16* __restrict__ pre, bf16* __restrict__ post,
+                                       int64_t n8, int C) {
+  GRID_STRIDE8(i, n8) {
+    const int c = int((8 * i) % C);
+    const V8 p = ld8(x + 8 * i);
+    V8 a, h;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      a.v[j] = fmaf(p.v[j], sc[c + j], sh[c + j]);
+      h.v[j] = hswish_f(round_bf16(a.v[j]));
+    }
+    st8(pre + 8 * i, a);
+    st8(post + 8 * i, h);
+  }
+}
+
 __device__ __forceinline__ float gelu_cdf(float x) { return 0.5f * (1.f + erff(x * 0.70710678118654752f)); }
 
 __global__ void gelu_fwd_x8_k(const bf16* __restrict__ x, bf16* __restrict__ y, int64_t n8) {
@@ -130,25 +154,34 @@ __global__ void gelu_bwd_x8_k(const bf16* __restrict__ x, const bf16* __restrict
 // Column partial sums over a (128-row chunk, 256-column block): thread
 // (g, r) owns columns c0 + 8g .. +7 and rows r, r + 8, ...; the 8 row lanes
 // are combined in shared memory in a fixed order.  MODE 0: sums of a;
-// MODE 1: affine backward (sums of dy * x and dy, and dx (+)= dy * scale).
+// MODE 1: affine backward (sums of dy * x and dy, and dx (+)= dy * scale);
+// MODE 2: MODE 1 behind a hard swish: `a` is the gradient of the hard
+// swish's output and `pre` its input (the affine output), and dy is the
+// bf16 value of a * hswish'(pre), as the separate hard swish backward stores.
 template <int MODE>
 __device__ __forceinline__ void colsum8_block(const bf16* __restrict__ a, const bf16* __restrict__ x,
                                               const float* __restrict__ scale, bf16* __restrict__ dx, int acc,
                                               int64_t rows, int C, int chunk, float* __restrict__ p0,
-                                              float* __restrict__ p1, int cb, int ck) {
+                                              float* __restrict__ p1, int cb, int ck,
+                                              const bf16* __restrict__ pre = nullptr) {
   __shared__ float red0[8][257];
-  __shared__ float red1[MODE == 1 ? 8 : 1][257];
+  __shared__ float red1[MODE >= 1 ? 8 : 1][257];
   const int g = threadIdx.x % 32, r = threadIdx.x / 32;
   const int c = cb * 256 + 8 * g;
   const int64_t r0 = int64_t(ck) * chunk;
   float s0[8] = {0, 0, 0, 0, 0, 0, 0, 0}, s1[8] = {0, 0, 0, 0, 0, 0, 0, 0};
   if (c < C) {
     float sc[8];
-    if (MODE == 1)
+    if (MODE >= 1)
 #pragma unroll
       for (int j = 0; j < 8; ++j) sc[j] = scale[c + j];
     for (int64_t row = r0 + r; row < r0 + chunk && row < rows; row += 8) {
-      const V8 d = ld8(a + row * C + c);
+      V8 d = ld8(a + row * C + c);
+      if (MODE == 2) {
+        const V8 h = ld8(pre + row * C + c);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) d.v[j] = round_bf16(d.v[j] * hswish_d(h.v[j]));
+      }
       if (MODE == 0) {
 #pragma unroll
         for (int j = 0; j < 8; ++j) s0[j] += d.v[j];
@@ -176,7 +209,7 @@ __device__ __forceinline__ void colsum8_block(const bf16* __restrict__ a, const 
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     red0[r][8 * g + j] = s0[j];
-    if (MODE == 1) red1[r][8 * g + j] = s1[j];
+    if (MODE >= 1) red1[r][8 * g + j] = s1[j];
   }
   __syncthreads();
   const int cc = cb * 256 + threadIdx.x;
@@ -185,10 +218,10 @@ __device__ __forceinline__ void colsum8_block(const bf16* __restrict__ a, const 
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
       t0 += red0[q][threadIdx.x];
-      if (MODE == 1) t1 += red1[q][threadIdx.x];
+      if (MODE >= 1) t1 += red1[q][threadIdx.x];
     }
     p0[int64_t(ck) * C + cc] = t0;
-    if (MODE == 1) p1[int64_t(ck) * C + cc] = t1;
+    if (MODE >= 1) p1[int64_t(ck) * C + cc] = t1;
   }
 }
 
@@ -196,8 +229,8 @@ template <int MODE>
 __global__ void __launch_bounds__(256) colsum8_k(const bf16* __restrict__ a, const bf16* __restrict__ x,
                                                  const float* __restrict__ scale, bf16* __restrict__ dx, int acc,
                                                  int64_t rows, int C, int chunk, float* __restrict__ p0,
-                                                 float* __restrict__ p1) {
-  colsum8_block<MODE>(a, x, scale, dx, acc, rows, C, chunk, p0, p1, blockIdx.x, blockIdx.y);
+                                                 float* __restrict__ p1, const bf16* __restrict__ pre = nullptr) {
+  colsum8_block<MODE>(a, x, scale, dx, acc, rows, C, chunk, p0, p1, blockIdx.x, blockIdx.y, pre);
 }
 
 // Several column sums in one launch: block b belongs to the task t with
@@ -424,6 +457,11 @@ void affine_fwd_x8(const void* x, const float* sc, const float* sh, void* y, int
                    cudaStream_t st) {
   affine_fwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, sc, sh, (bf16*)y, n / 8, C, relu);
 }
+void affine_hswish_fwd_x8(const void* x, const float* sc, const float* sh, void* pre, void* post, int64_t n, int C,
+                          cudaStream_t st) {
+  affine_hswish_fwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, sc, sh, (bf16*)pre,
+                                                                          (bf16*)post, n / 8, C);
+}
 void gelu_fwd_x8(const void* x, void* y, int64_t n, cudaStream_t st) {
   gelu_fwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, (bf16*)y, n / 8);
 }
@@ -456,11 +494,15 @@ void affine_bwd8(const void* dy, const void* x, const float* scale, void* dx, bo
 int affine_bwd8_chunks(int64_t rows, int C) { return chunks_of(rows, adaptive_chunk(rows, C)); }
 
 void affine_bwd8_pass(const void* dy, const void* x, const float* scale, void* dx, bool acc, int64_t rows, int C,
-                      float* p_scale, float* p_shift, cudaStream_t st) {
+                      float* p_scale, float* p_shift, cudaStream_t st, const void* hswish_in) {
   const int ch = adaptive_chunk(rows, C);
   dim3 grid(ceil_div(C, 256), chunks_of(rows, ch));
-  colsum8_k<1><<<grid, 256, 0, st>>>((const bf16*)dy, (const bf16*)x, scale, (bf16*)dx, acc, rows, C, ch, p_scale,
-                                     p_shift);
+  if (hswish_in)
+    colsum8_k<2><<<grid, 256, 0, st>>>((const bf16*)dy, (const bf16*)x, scale, (bf16*)dx, acc, rows, C, ch, p_scale,
+                                       p_shift, (const bf16*)hswish_in);
+  else
+    colsum8_k<1><<<grid, 256, 0, st>>>((const bf16*)dy, (const bf16*)x, scale, (bf16*)dx, acc, rows, C, ch, p_scale,
+                                       p_shift);
 }
 
 int colsum8_batch_chunks(int64_t rows) { return chunks_of(rows, kChunk); }

@@ -10,10 +10,9 @@ gates of test_gpu_train (the hard sigmoid's derivative jumps at -3 and 3
 and the SE block has a ReLU, so stored values one bf16 ulp apart may decide
 a kink the other way: the decision allowance applies).
 """
-import numpy as np
 import pytest
 
-from harness import normwise, replay_gpu, replay_oracle, teacher_forced
+from harness import teacher_forced
 from paper_2504_13850_gb300 import api, build
 from paper_2504_13850_gb300 import workloads as W
 from test_gpu_train import check_teacher_forced, compare, prefill_then_steps
@@ -71,8 +70,8 @@ def test_small_mobile_bf16_teacher_forced():
 
 def test_depthwise_gradients_reach_the_input_layer():
     """A depthwise conv reading the uploaded batch (no input gradient) and a
-    channel scale whose gate is computed from it: the fp32 trace still
-    matches, and the plan launches no input-gradient kernel for tensor 0."""
+    channel scale whose gate is computed from it (neither passes a gradient
+    to the upload): the fp32 trace still matches."""
     b = W._Builder()
     t = b.add("dwconv", 0, c=16, k=5, stride=2, bias=1)
     g = b.add("avgpool", 0)
@@ -102,3 +101,24 @@ def test_bad_mobile_shapes_are_refused():
                                                       "bias": 1}]
         with pytest.raises(RuntimeError):
             api.Server.from_config(W.shrink(base, ops=ops))
+
+
+def test_depthwise_any_kernel_size():
+    """Kernel sizes outside the unrolled 3 / 5 (k = 7 stride 1, k = 1
+    stride 2) take the generic depthwise kernels; bf16 teacher-forced."""
+    b = W._Builder()
+    t = b.add("dwconv", 0, c=16, k=7, stride=1, bias=1)
+    t = b.add("affine", t, c=16)
+    t = b.add("hswish", t)
+    t = b.add("dwconv", t, c=16, k=1, stride=2, bias=0)
+    t = b.add("hswish", t)
+    t = b.add("flatten", t)
+    b.add("linear", t, cin=4 * 4 * 16, cout=10, bias=1)
+    for dtype in (W.F32, W.BF16):
+        cfg = W.shrink(W.CONFIGS["mobilenet"], ops=b.ops, batch=6, in_hwc=(8, 8, 16), K=2, omega=4, depth=2,
+                       dtype=dtype)
+        if dtype == W.F32:
+            compare(cfg, prefill_then_steps(cfg, 4), loss_tol=1e-4, param_tol=1e-4, upd_tol=1e-4)
+        else:
+            _, _, recs = teacher_forced(cfg, prefill_then_steps(cfg, 4))
+            check_teacher_forced(recs, decisions=True)
