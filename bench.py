@@ -48,7 +48,7 @@ OTHER_DESC = {
              "omega 400, FC 512->100, softmax-CE, SGD lr 0.01 momentum 0.9",
     "mobilenet": "MobileNetV3-Large server part: 10 devices, bf16 activations [64,112,4,4] = ReLU(N(0,1)), "
                  "BNECK-5-160 x3 (first stride 2; 1x1 expand, 5x5 depthwise, squeeze-and-excite, 1x1 project, "
-                 "hard swish), CONV-1-960, avgpool, FC 960->1280, hard swish, FC 1280->10, softmax-CE, "
+                 "hard swish), CONV-1-960, avgpool, FC 960->1280, hard swish, FC 1280->200, softmax-CE, "
                  "SGD lr 0.01 momentum 0.9",
 }
 

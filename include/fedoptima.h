@@ -70,7 +70,7 @@ enum {
   FO_OP_GELU = 10,     /* exact GELU x * Phi(x)                                                                 */
   FO_OP_ATTENTION = 11,/* in0 = [B, L, 3c] packed q|k|v; `heads` heads of c/heads; keys >= length masked          */
   FO_OP_MEANPOOL = 12, /* mean over the first length[b] tokens: [B, L, c] -> [B, c]                              */
-  /* MobileNetV3 bottleneck ops (the MobileNetV3-Large split of Table 2):                                       */
+  /* MobileNetV3 bottleneck ops (the MobileNetV3-Large split of Table 4):                                       */
   FO_OP_DWCONV = 13,   /* depthwise k x k (k odd, <= 7), stride 1|2, pad k/2, channels cin.  params W[cin][k][k],
                           b[cin] if bias                                                                        */
   FO_OP_HSWISH = 14,   /* hard swish x * relu6(x + 3) / 6; derivative 0 below -3, (2x + 3) / 6 on [-3, 3], 1 above */

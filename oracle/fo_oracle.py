@@ -20,7 +20,7 @@ What it follows (arxiv 2504.13850):
   * Layer arithmetic is the textbook definition of each layer, in fp64;
     matrix products (numpy ``@``) are used as a library primitive.
   * The MobileNetV3 bottleneck pieces of the paper's testbed-B CNN
-    (Table 2): depthwise convolution, hard swish, hard sigmoid and the
+    (Table 4): depthwise convolution, hard swish, hard sigmoid and the
     squeeze-and-excite channel scaling (``dwconv_*``, ``hswish_*``,
     ``hsigmoid_*``, ``chmul_*``); the derivative readings at the kinks
     follow the usual library convention (hard swish: 0 below -3, 1 above 3;

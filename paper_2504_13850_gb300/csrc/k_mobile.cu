@@ -1,5 +1,5 @@
 // Kernels of the MobileNetV3 bottleneck (the MobileNetV3-Large server part
-// of Table 2): depthwise convolution, hard swish, hard sigmoid and the
+// of Table 4): depthwise convolution, hard swish, hard sigmoid and the
 // squeeze-and-excite channel scaling.  Activations are NHWC in fp32 or bf16
 // (template parameter T); every arithmetic step runs in fp32.  Channels are
 // the fastest index of every thread mapping, so a warp's loads and stores are

@@ -1,6 +1,6 @@
 """Workload definitions and seeded synthetic inputs.
 
-This module holds only the *inputs* of the server-side hot path: the five
+This module holds only the *inputs* of the server-side hot path: the
 server-part architectures (as op lists), their batch shapes, queue sizes and
 step counts, and seeded generators for initial weights, uploaded activation
 batches, labels, sequence lengths, device-side models and device arrival
@@ -9,7 +9,8 @@ and the CPU oracle may consume it.
 
 The architectures stand in for the paper's workloads (Sec. 5.2, Table 4:
 VGG-style CNNs on CIFAR-10-shaped data, ResNet-18 stages, transformer
-encoders on SST-2/IMDB-shaped sequences).  No dataset item is used: every
+encoders on SST-2/IMDB-shaped sequences, the MobileNetV3-Large server part
+on Tiny-ImageNet-shaped activations).  No dataset item is used: every
 activation is drawn from a PCG64 generator.
 
 Op list format (one dict per op, executed in order).  Tensor 0 is the
@@ -28,6 +29,11 @@ uploaded activation batch; op ``i`` (0-based) produces tensor ``i + 1``.
   gelu      in0                          exact (erf) GELU
   attention in0, c, heads                in0 is [B, L, 3c] = q | k | v
   meanpool  in0                          mean over the valid tokens of each row
+  dwconv    in0, c, k (odd), stride, bias  depthwise k x k, pad k // 2
+            params: W[c][k][k], then b[c] if bias
+  hswish    in0                          hard swish x * relu6(x + 3) / 6
+  hsigmoid  in0                          hard sigmoid relu6(x + 3) / 6
+  chmul     in0, in1                     y[b,h,w,c] = in0[b,h,w,c] * in1[b,c] (squeeze-and-excite)
 
 Activations are NHWC.  A sequence batch [B, L, d] is carried as H = L,
 W = 1, C = d.  The last op's output is the logits [B, classes]; the loss is
@@ -132,12 +138,12 @@ def _bneck(b, x, cin, exp, cout, k, stride, se=True, act="hswish"):
     return t
 
 
-def mobilenet_ops(classes=10):
-    """Server part of MobileNetV3-Large (the paper's Table 2) after its
+def mobilenet_ops(classes=200):
+    """Server part of MobileNetV3-Large (the paper's Table 4) after its
     BNECK-3-112 stage: BNECK-5-160 x 3 (the first with stride 2),
     CONV-1-960, global average pool, CONV-1-1280 (on the pooled 1 x 1 map,
-    a dense layer) and FC -> classes, with hard swish activations, on a
-    [4,4,112] input."""
+    a dense layer) and FC -> classes (200, Tiny ImageNet's), with hard swish
+    activations, on a [4,4,112] input."""
     b = _Builder()
     t = _bneck(b, 0, 112, 672, 160, 5, 2)
     t = _bneck(b, t, 160, 960, 160, 5, 1)
@@ -252,7 +258,7 @@ CONFIGS = {
                   in_hwc=(16, 16, 128), dtype=BF16, classes=100, seed=4,
                   steps=1000, agg_params=700_000, rates=zipf_rates(100)),
     "mobilenet": _cfg("mobilenet", mobilenet_ops(), K=10, depth=4, omega=40, batch=64,
-                      in_hwc=(4, 4, 112), dtype=BF16, classes=10, seed=6, steps=200,
+                      in_hwc=(4, 4, 112), dtype=BF16, classes=200, seed=6, steps=200,
                       agg_params=1_000_000, rates=group_rates(10)),
     # one device's own trainer for the live VGG pipeline: its local data
     # queue (K = 1) feeds M_dk + the auxiliary network
