@@ -19,6 +19,8 @@ __global__ void __launch_bounds__(256) attn_fwd_k(const T* __restrict__ qkv,
                                                   const int32_t* __restrict__ len,
                                                   T* __restrict__ out, float* __restrict__ probs,
                                                   int L, int C, int heads) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ float sm[];
   const int bh = blockIdx.x, b = bh / heads, h = bh % heads;
   const int dh = C / heads, ld = dh + 1;
@@ -102,6 +104,8 @@ __global__ void __launch_bounds__(256) attn_bwd_k(const T* __restrict__ qkv,
                                                   const int32_t* __restrict__ len,
                                                   T* __restrict__ dqkv, int L, int C, int heads,
                                                   int acc) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ float sm[];
   const int bh = blockIdx.x, b = bh / heads, h = bh % heads;
   const int dh = C / heads, ld = dh + 1, lds = L + 1;
@@ -180,9 +184,9 @@ void attention_fwd(const void* qkv, const int32_t* len, void* out, float* probs,
                    int C, int heads, int dt, cudaStream_t st) {
   size_t sm = fwd_smem(L, C / heads);
   if (dt == kF32) {
-    attn_fwd_k<float><<<B * heads, 256, sm, st>>>((const float*)qkv, len, (float*)out, probs, L, C, heads);
+    launch_k(attn_fwd_k<float>, B * heads, 256, sm, st, (const float*)qkv, len, (float*)out, probs, L, C, heads);
   } else {
-    attn_fwd_k<bf16><<<B * heads, 256, sm, st>>>((const bf16*)qkv, len, (bf16*)out, probs, L, C, heads);
+    launch_k(attn_fwd_k<bf16>, B * heads, 256, sm, st, (const bf16*)qkv, len, (bf16*)out, probs, L, C, heads);
   }
 }
 
@@ -191,11 +195,11 @@ void attention_bwd(const void* qkv, const int32_t* len, const float* probs, cons
                    cudaStream_t st) {
   size_t sm = bwd_smem(L, C / heads);
   if (dt == kF32) {
-    attn_bwd_k<float><<<B * heads, 256, sm, st>>>((const float*)qkv, probs, (const float*)out,
+    launch_k(attn_bwd_k<float>, B * heads, 256, sm, st, (const float*)qkv, probs, (const float*)out,
                                                    (const float*)dout, len, (float*)dqkv, L, C,
                                                    heads, acc ? 1 : 0);
   } else {
-    attn_bwd_k<bf16><<<B * heads, 256, sm, st>>>((const bf16*)qkv, probs, (const bf16*)out,
+    launch_k(attn_bwd_k<bf16>, B * heads, 256, sm, st, (const bf16*)qkv, probs, (const bf16*)out,
                                                   (const bf16*)dout, len, (bf16*)dqkv, L, C,
                                                   heads, acc ? 1 : 0);
   }

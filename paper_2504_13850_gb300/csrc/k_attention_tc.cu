@@ -106,6 +106,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_tc_k(const __grid_co
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tslot;          // S: columns 0..127, O: 128..191
+  pdl_trigger();   // this block holds its tensor memory
+  pdl_wait();      // the previous kernel's writes are visible from here on
 
   if (warp == 0) {
     if (lane == 0) {
@@ -230,6 +232,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_bwd_tc_k(const __grid_co
   tc_fence_after();
   // TMEM columns: S 0..127, dP 128..255, dV 256..319, dQ 320..383, dK 384..447
   const uint32_t tmem = *tslot;
+  pdl_trigger();
+  pdl_wait();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -386,7 +390,7 @@ void attention_tc_fwd(const AttnTcPlan* a, const int32_t* len, void* out, float*
   p.out = static_cast<bf16*>(out);
   p.lse = lse;
   p.acc = 0;
-  attn_fwd_tc_k<<<B * p.heads, kAttnThreads, kFwdSmem, st>>>(p);
+  launch_k(attn_fwd_tc_k, B * p.heads, kAttnThreads, kFwdSmem, st, p);
 }
 
 void attention_tc_bwd(const AttnTcPlan* a, const int32_t* len, const float* lse, void* dqkv, int B, bool acc,
@@ -396,7 +400,7 @@ void attention_tc_bwd(const AttnTcPlan* a, const int32_t* len, const float* lse,
   p.out = static_cast<bf16*>(dqkv);
   p.lse = const_cast<float*>(lse);
   p.acc = acc ? 1 : 0;
-  attn_bwd_tc_k<<<B * p.heads, kAttnThreads, kBwdSmem, st>>>(p);
+  launch_k(attn_bwd_tc_k, B * p.heads, kAttnThreads, kBwdSmem, st, p);
 }
 
 }  // namespace fo

@@ -6,6 +6,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <cstdlib>
 
 namespace fo {
 
@@ -23,6 +24,11 @@ int elementwise_blocks(int64_t n_threads_needed, int threads) {
   if (want > cap) want = cap;
   if (want < 1) want = 1;
   return int(want);
+}
+
+bool pdl_enabled() {
+  static const bool on = getenv("FO_NO_PDL") == nullptr;
+  return on;
 }
 
 #define FO_DISPATCH(dt, T, ...)   \
@@ -48,23 +54,29 @@ __device__ __forceinline__ void store(T* p, int64_t i, float v, bool acc) {
 // ------------------------------------------------------------------ relu
 template <typename T>
 __global__ void relu_fwd_k(const T* x, T* y, int64_t n) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE(i, n) y[i] = from_f<T>(fmaxf(to_f(x[i]), 0.f));
 }
 template <typename T>
 __global__ void relu_bwd_k(const T* x, const T* dy, T* dx, int64_t n, int acc) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE(i, n) store(dx, i, to_f(x[i]) > 0.f ? to_f(dy[i]) : 0.f, acc);
 }
 void relu_fwd(const void* x, void* y, int64_t n, int dt, cudaStream_t st) {
-  FO_DISPATCH(dt, T, relu_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (T*)y, n));
+  FO_DISPATCH(dt, T, launch_k(relu_fwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (T*)y, n));
 }
 void relu_bwd(const void* x, const void* dy, void* dx, int64_t n, int dt, bool acc, cudaStream_t st) {
   if (vec8_ok(dt, n)) return relu_bwd_x8(x, dy, dx, n, acc, st);
-  FO_DISPATCH(dt, T, relu_bwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (const T*)dy, (T*)dx, n, acc));
+  FO_DISPATCH(dt, T, launch_k(relu_bwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (const T*)dy, (T*)dx, n, acc));
 }
 
 // --------------------------------------------------------------- maxpool
 template <typename T>
 __global__ void maxpool2_fwd_k(const T* x, T* y, int N, int H, int W, int C) {
+  pdl_wait();
+  pdl_trigger();
   const int Ho = H / 2, Wo = W / 2;
   const int64_t n_out = int64_t(N) * Ho * Wo * C;
   GRID_STRIDE(o, n_out) {
@@ -87,6 +99,8 @@ __global__ void maxpool2_fwd_k(const T* x, T* y, int N, int H, int W, int C) {
 template <typename T>
 __global__ void maxpool2_bwd_k(const T* x, const T* dy, T* dx, int N, int H, int W, int C,
                                int acc, int relu_mask) {
+  pdl_wait();
+  pdl_trigger();
   const int Ho = H / 2, Wo = W / 2;
   const int64_t n_out = int64_t(N) * Ho * Wo * C;
   GRID_STRIDE(o, n_out) {
@@ -116,6 +130,8 @@ __global__ void maxpool2_bwd_k(const T* x, const T* dy, T* dx, int N, int H, int
 }
 // 8 channels per thread with 16-byte loads (bf16, C % 8 == 0).
 __global__ void maxpool2_fwd_x8_k(const bf16* __restrict__ x, bf16* __restrict__ y, int N, int H, int W, int C) {
+  pdl_wait();
+  pdl_trigger();
   const int Ho = H / 2, Wo = W / 2, C8 = C / 8;
   const int64_t n_out = int64_t(N) * Ho * Wo * C8;
   GRID_STRIDE(o, n_out) {
@@ -147,6 +163,8 @@ __global__ void maxpool2_fwd_x8_k(const bf16* __restrict__ x, bf16* __restrict__
 // window's gradient goes to its first maximum in row-major order.
 __global__ void maxpool2_bwd_x8_k(const bf16* __restrict__ x, const bf16* __restrict__ dy, bf16* __restrict__ dx,
                                   int N, int H, int W, int C, int acc, int relu_mask) {
+  pdl_wait();
+  pdl_trigger();
   const int Ho = H / 2, Wo = W / 2, C8 = C / 8;
   const int64_t n_out = int64_t(N) * Ho * Wo * C8;
   GRID_STRIDE(o, n_out) {
@@ -198,33 +216,35 @@ __global__ void maxpool2_bwd_x8_k(const bf16* __restrict__ x, const bf16* __rest
 void maxpool2_fwd(const void* x, void* y, int N, int H, int W, int C, int dt, cudaStream_t st) {
   int64_t n = int64_t(N) * (H / 2) * (W / 2) * C;
   if (dt == kBF16 && C % 8 == 0) {
-    maxpool2_fwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, (bf16*)y, N, H, W, C);
+    launch_k(maxpool2_fwd_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)x, (bf16*)y, N, H, W, C);
     return;
   }
-  FO_DISPATCH(dt, T, maxpool2_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (T*)y, N, H, W, C));
+  FO_DISPATCH(dt, T, launch_k(maxpool2_fwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (T*)y, N, H, W, C));
 }
 void maxpool2_bwd(const void* x, const void* dy, void* dx, int N, int H, int W, int C, int dt,
                   bool acc, cudaStream_t st) {
   int64_t n = int64_t(N) * (H / 2) * (W / 2) * C;
   if (dt == kBF16 && C % 8 == 0) {
-    maxpool2_bwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, (const bf16*)dy, (bf16*)dx, N, H, W, C, acc, 0);
+    launch_k(maxpool2_bwd_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)x, (const bf16*)dy, (bf16*)dx, N, H, W, C, acc, 0);
     return;
   }
-  FO_DISPATCH(dt, T, maxpool2_bwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (const T*)dy, (T*)dx, N, H, W, C, acc, 0));
+  FO_DISPATCH(dt, T, launch_k(maxpool2_bwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (const T*)dy, (T*)dx, N, H, W, C, acc, 0));
 }
 void relu_maxpool2_bwd(const void* x, const void* dy, void* dx, int N, int H, int W, int C,
                        int dt, bool acc, cudaStream_t st) {
   int64_t n = int64_t(N) * (H / 2) * (W / 2) * C;
   if (dt == kBF16 && C % 8 == 0) {
-    maxpool2_bwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, (const bf16*)dy, (bf16*)dx, N, H, W, C, acc, 1);
+    launch_k(maxpool2_bwd_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)x, (const bf16*)dy, (bf16*)dx, N, H, W, C, acc, 1);
     return;
   }
-  FO_DISPATCH(dt, T, maxpool2_bwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (const T*)dy, (T*)dx, N, H, W, C, acc, 1));
+  FO_DISPATCH(dt, T, launch_k(maxpool2_bwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (const T*)dy, (T*)dx, N, H, W, C, acc, 1));
 }
 
 // ---------------------------------------------------------- affine / add
 template <typename T>
 __global__ void affine_fwd_k(const T* x, const float* sc, const float* sh, T* y, int64_t n, int C, int relu) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE(i, n) {
     int c = int(i % C);
     float v = fmaf(to_f(x[i]), sc[c], sh[c]);
@@ -233,10 +253,14 @@ __global__ void affine_fwd_k(const T* x, const float* sc, const float* sh, T* y,
 }
 template <typename T>
 __global__ void affine_dx_k(const T* dy, const float* sc, T* dx, int64_t n, int C, int acc) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE(i, n) store(dx, i, to_f(dy[i]) * sc[int(i % C)], acc);
 }
 template <typename T>
 __global__ void add_fwd_k(const T* a, const T* b, T* y, int64_t n, int relu) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE(i, n) {
     float v = to_f(a[i]) + to_f(b[i]);
     y[i] = from_f<T>(relu ? fmaxf(v, 0.f) : v);
@@ -244,31 +268,35 @@ __global__ void add_fwd_k(const T* a, const T* b, T* y, int64_t n, int relu) {
 }
 template <typename T>
 __global__ void copy_acc_k(const T* x, T* y, int64_t n, int acc) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE(i, n) store(y, i, to_f(x[i]), acc);
 }
 void affine_fwd(const void* x, const float* scale, const float* shift, void* y, int64_t rows,
                 int C, int dt, bool relu, cudaStream_t st) {
   int64_t n = rows * C;
   if (vec8_ok(dt, n) && C % 8 == 0) return affine_fwd_x8(x, scale, shift, y, n, C, relu, st);
-  FO_DISPATCH(dt, T, affine_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, scale, shift, (T*)y, n, C, relu));
+  FO_DISPATCH(dt, T, launch_k(affine_fwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, scale, shift, (T*)y, n, C, relu));
 }
 void affine_dx(const void* dy, const float* scale, void* dx, int64_t rows, int C, int dt,
                bool acc, cudaStream_t st) {
   int64_t n = rows * C;
-  FO_DISPATCH(dt, T, affine_dx_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)dy, scale, (T*)dx, n, C, acc));
+  FO_DISPATCH(dt, T, launch_k(affine_dx_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)dy, scale, (T*)dx, n, C, acc));
 }
 void add_fwd(const void* a, const void* b, void* y, int64_t n, int dt, bool relu, cudaStream_t st) {
   if (vec8_ok(dt, n)) return add_x8(a, b, y, n, relu, st);
-  FO_DISPATCH(dt, T, add_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)a, (const T*)b, (T*)y, n, relu));
+  FO_DISPATCH(dt, T, launch_k(add_fwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)a, (const T*)b, (T*)y, n, relu));
 }
 void copy_or_acc(const void* x, void* y, int64_t n, int dt, bool acc, cudaStream_t st) {
   if (vec8_ok(dt, n)) return copy_acc_x8(x, y, n, acc, st);
-  FO_DISPATCH(dt, T, copy_acc_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (T*)y, n, acc));
+  FO_DISPATCH(dt, T, launch_k(copy_acc_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (T*)y, n, acc));
 }
 
 // -------------------------------------------------------------- avgpool
 template <typename T>
 __global__ void avgpool_fwd_k(const T* x, T* y, int N, int HW, int C) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE(o, int64_t(N) * C) {
     int c = int(o % C);
     int64_t n = o / C;
@@ -279,6 +307,8 @@ __global__ void avgpool_fwd_k(const T* x, T* y, int N, int HW, int C) {
 }
 template <typename T>
 __global__ void avgpool_bwd_k(const T* dy, T* dx, int N, int HW, int C, int acc) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE(i, int64_t(N) * HW * C) {
     int c = int(i % C);
     int64_t n = i / (int64_t(HW) * C);
@@ -286,16 +316,18 @@ __global__ void avgpool_bwd_k(const T* dy, T* dx, int N, int HW, int C, int acc)
   }
 }
 void avgpool_fwd(const void* x, void* y, int N, int HW, int C, int dt, cudaStream_t st) {
-  FO_DISPATCH(dt, T, avgpool_fwd_k<T><<<elementwise_blocks(int64_t(N) * C, 256), 256, 0, st>>>((const T*)x, (T*)y, N, HW, C));
+  FO_DISPATCH(dt, T, launch_k(avgpool_fwd_k<T>, elementwise_blocks(int64_t(N) * C, 256), 256, 0, st, (const T*)x, (T*)y, N, HW, C));
 }
 void avgpool_bwd(const void* dy, void* dx, int N, int HW, int C, int dt, bool acc, cudaStream_t st) {
-  FO_DISPATCH(dt, T, avgpool_bwd_k<T><<<elementwise_blocks(int64_t(N) * HW * C, 256), 256, 0, st>>>((const T*)dy, (T*)dx, N, HW, C, acc));
+  FO_DISPATCH(dt, T, launch_k(avgpool_bwd_k<T>, elementwise_blocks(int64_t(N) * HW * C, 256), 256, 0, st, (const T*)dy, (T*)dx, N, HW, C, acc));
 }
 
 // ----------------------------------------------------------------- gelu
 __device__ __forceinline__ float gelu_cdf(float x) { return 0.5f * (1.f + erff(x * 0.70710678118654752f)); }
 template <typename T>
 __global__ void gelu_fwd_k(const T* x, T* y, int64_t n) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE(i, n) {
     float v = to_f(x[i]);
     y[i] = from_f<T>(v * gelu_cdf(v));
@@ -303,6 +335,8 @@ __global__ void gelu_fwd_k(const T* x, T* y, int64_t n) {
 }
 template <typename T>
 __global__ void gelu_bwd_k(const T* x, const T* dy, T* dx, int64_t n, int acc) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE(i, n) {
     float v = to_f(x[i]);
     float pdf = 0.39894228040143268f * expf(-0.5f * v * v);
@@ -311,11 +345,11 @@ __global__ void gelu_bwd_k(const T* x, const T* dy, T* dx, int64_t n, int acc) {
 }
 void gelu_fwd(const void* x, void* y, int64_t n, int dt, cudaStream_t st) {
   if (vec8_ok(dt, n)) return gelu_fwd_x8(x, y, n, st);
-  FO_DISPATCH(dt, T, gelu_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (T*)y, n));
+  FO_DISPATCH(dt, T, launch_k(gelu_fwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (T*)y, n));
 }
 void gelu_bwd(const void* x, const void* dy, void* dx, int64_t n, int dt, bool acc, cudaStream_t st) {
   if (vec8_ok(dt, n)) return gelu_bwd_x8(x, dy, dx, n, acc, st);
-  FO_DISPATCH(dt, T, gelu_bwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (const T*)dy, (T*)dx, n, acc));
+  FO_DISPATCH(dt, T, launch_k(gelu_bwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (const T*)dy, (T*)dx, n, acc));
 }
 
 // ------------------------------------------------------------ layernorm
@@ -329,6 +363,8 @@ __device__ __forceinline__ float warp_sum(float v) {
 template <typename T>
 __global__ void layernorm_fwd_k(const T* x, const float* gamma, const float* beta, T* y,
                                 float* mean_out, float* rstd_out, int64_t rows, int C) {
+  pdl_wait();
+  pdl_trigger();
   int64_t row = int64_t(blockIdx.x) * (blockDim.x / 32) + threadIdx.x / 32;
   int lane = threadIdx.x % 32;
   if (row >= rows) return;
@@ -354,6 +390,8 @@ template <typename T>
 __global__ void layernorm_bwd_k(const T* x, const float* gamma, const float* mean,
                                 const float* rstd, const T* dy, T* dx, int64_t rows, int C,
                                 int acc) {
+  pdl_wait();
+  pdl_trigger();
   int64_t row = int64_t(blockIdx.x) * (blockDim.x / 32) + threadIdx.x / 32;
   int lane = threadIdx.x % 32;
   if (row >= rows) return;
@@ -379,13 +417,13 @@ __global__ void layernorm_bwd_k(const T* x, const float* gamma, const float* mea
 void layernorm_fwd(const void* x, const float* gamma, const float* beta, void* y, float* mean,
                    float* rstd, int64_t rows, int C, int dt, cudaStream_t st) {
   int blocks = ceil_div(rows, 8);
-  FO_DISPATCH(dt, T, layernorm_fwd_k<T><<<blocks, 256, 0, st>>>((const T*)x, gamma, beta, (T*)y, mean, rstd, rows, C));
+  FO_DISPATCH(dt, T, launch_k(layernorm_fwd_k<T>, blocks, 256, 0, st, (const T*)x, gamma, beta, (T*)y, mean, rstd, rows, C));
 }
 void layernorm_bwd_dx(const void* x, const float* gamma, const float* mean, const float* rstd,
                       const void* dy, void* dx, int64_t rows, int C, int dt, bool acc,
                       cudaStream_t st) {
   int blocks = ceil_div(rows, 8);
-  FO_DISPATCH(dt, T, layernorm_bwd_k<T><<<blocks, 256, 0, st>>>((const T*)x, gamma, mean, rstd, (const T*)dy, (T*)dx, rows, C, acc));
+  FO_DISPATCH(dt, T, launch_k(layernorm_bwd_k<T>, blocks, 256, 0, st, (const T*)x, gamma, mean, rstd, (const T*)dy, (T*)dx, rows, C, acc));
 }
 
 // ---------------------------------------------------- column reductions
@@ -399,6 +437,8 @@ int64_t colsum_partial_floats(int64_t rows, int C) { return int64_t(colsum_chunk
 template <int MODE, typename T>
 __global__ void colsum_partial_k(const T* a, const T* b, const float* mean, const float* rstd,
                                  int64_t rows, int C, float* partial) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float red[8][33];
   int cl = threadIdx.x % 32, rl = threadIdx.x / 32;
   int c = blockIdx.x * 32 + cl;
@@ -424,6 +464,8 @@ __global__ void colsum_partial_k(const T* a, const T* b, const float* mean, cons
 // Adds the per-chunk partials of each column: 8 row lanes per column sum
 // interleaved chunks, then combine in a fixed order (deterministic).
 __global__ void colsum_finish_k(const float* partial, int chunks, int C, float* out) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float red[8][33];
   const int cl = threadIdx.x % 32, rl = threadIdx.x / 32;
   const int c = blockIdx.x * 32 + cl;
@@ -463,22 +505,24 @@ void colsum(const void* a, const void* b, int64_t rows, int C, int dt, float* pa
   if (!b && dt == kBF16 && C % 8 == 0) return colsum8(a, rows, C, partial, out, adaptive, st);
   dim3 grid(ceil_div(C, 32), colsum_chunks(rows));
   if (b) {
-    FO_DISPATCH(dt, T, colsum_partial_k<1, T><<<grid, 256, 0, st>>>((const T*)a, (const T*)b, nullptr, nullptr, rows, C, partial));
+    FO_DISPATCH(dt, T, launch_k(colsum_partial_k<1, T>, grid, 256, 0, st, (const T*)a, (const T*)b, nullptr, nullptr, rows, C, partial));
   } else {
-    FO_DISPATCH(dt, T, colsum_partial_k<0, T><<<grid, 256, 0, st>>>((const T*)a, nullptr, nullptr, nullptr, rows, C, partial));
+    FO_DISPATCH(dt, T, launch_k(colsum_partial_k<0, T>, grid, 256, 0, st, (const T*)a, nullptr, nullptr, nullptr, rows, C, partial));
   }
-  colsum_finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, colsum_chunks(rows), C, out);
+  launch_k(colsum_finish_k, ceil_div(C, 32), 256, 0, st, partial, colsum_chunks(rows), C, out);
 }
 void colsum_lnx(const void* dy, const void* x, const float* mean, const float* rstd, int64_t rows,
                 int C, int dt, float* partial, float* out, cudaStream_t st) {
   dim3 grid(ceil_div(C, 32), colsum_chunks(rows));
-  FO_DISPATCH(dt, T, colsum_partial_k<2, T><<<grid, 256, 0, st>>>((const T*)dy, (const T*)x, mean, rstd, rows, C, partial));
-  colsum_finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, colsum_chunks(rows), C, out);
+  FO_DISPATCH(dt, T, launch_k(colsum_partial_k<2, T>, grid, 256, 0, st, (const T*)dy, (const T*)x, mean, rstd, rows, C, partial));
+  launch_k(colsum_finish_k, ceil_div(C, 32), 256, 0, st, partial, colsum_chunks(rows), C, out);
 }
 
 // ------------------------------------------------------------- meanpool
 template <typename T>
 __global__ void meanpool_fwd_k(const T* x, const int32_t* len, T* y, int B, int L, int C) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE(o, int64_t(B) * C) {
     int c = int(o % C);
     int b = int(o / C);
@@ -490,6 +534,8 @@ __global__ void meanpool_fwd_k(const T* x, const int32_t* len, T* y, int B, int 
 }
 template <typename T>
 __global__ void meanpool_bwd_k(const T* dy, const int32_t* len, T* dx, int B, int L, int C, int acc) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE(i, int64_t(B) * L * C) {
     int c = int(i % C);
     int64_t t = i / C;
@@ -501,11 +547,11 @@ __global__ void meanpool_bwd_k(const T* dy, const int32_t* len, T* dx, int B, in
 }
 void meanpool_fwd(const void* x, const int32_t* len, void* y, int B, int L, int C, int dt,
                   cudaStream_t st) {
-  FO_DISPATCH(dt, T, meanpool_fwd_k<T><<<elementwise_blocks(int64_t(B) * C, 256), 256, 0, st>>>((const T*)x, len, (T*)y, B, L, C));
+  FO_DISPATCH(dt, T, launch_k(meanpool_fwd_k<T>, elementwise_blocks(int64_t(B) * C, 256), 256, 0, st, (const T*)x, len, (T*)y, B, L, C));
 }
 void meanpool_bwd(const void* dy, const int32_t* len, void* dx, int B, int L, int C, int dt,
                   bool acc, cudaStream_t st) {
-  FO_DISPATCH(dt, T, meanpool_bwd_k<T><<<elementwise_blocks(int64_t(B) * L * C, 256), 256, 0, st>>>((const T*)dy, len, (T*)dx, B, L, C, acc));
+  FO_DISPATCH(dt, T, launch_k(meanpool_bwd_k<T>, elementwise_blocks(int64_t(B) * L * C, 256), 256, 0, st, (const T*)dy, len, (T*)dx, B, L, C, acc));
 }
 
 // ------------------------------------------------------ softmax + CE loss
@@ -514,6 +560,8 @@ void meanpool_bwd(const void* dy, const int32_t* len, void* dx, int B, int L, in
 template <typename T>
 __global__ void softmax_ce_k(const float* z, const int32_t* labels, int B, int C, float* losses,
                              const int64_t* step, int64_t mask, T* dz) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float row_loss[1024];
   int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   for (int b = warp; b < B; b += blockDim.x / 32) {
@@ -542,7 +590,7 @@ __global__ void softmax_ce_k(const float* z, const int32_t* labels, int B, int C
 }
 void softmax_ce(const float* logits, const int32_t* labels, int B, int C, float* losses,
                 const int64_t* step, int64_t mask, void* dlogits, int dt, cudaStream_t st) {
-  FO_DISPATCH(dt, T, softmax_ce_k<T><<<1, 256, 0, st>>>(logits, labels, B, C, losses, step, mask, (T*)dlogits));
+  FO_DISPATCH(dt, T, launch_k(softmax_ce_k<T>, 1, 256, 0, st, logits, labels, B, C, losses, step, mask, (T*)dlogits));
 }
 
 // ------------------------------------------------------ SGD with momentum
@@ -550,6 +598,8 @@ void softmax_ce(const float* logits, const int32_t* labels, int B, int C, float*
 __global__ void sgd_momentum_k(float4* __restrict__ theta, float4* __restrict__ v,
                                const float4* __restrict__ g, uint2* __restrict__ shadow,
                                int64_t n4, float lr, float mu, int64_t* step) {
+  pdl_wait();
+  pdl_trigger();
   if (step && blockIdx.x == 0 && threadIdx.x == 0) *step += 1;
   GRID_STRIDE(i, n4) {
     float4 t = theta[i], m = v[i];
@@ -576,14 +626,16 @@ __global__ void sgd_momentum_k(float4* __restrict__ theta, float4* __restrict__ 
 void sgd_momentum(float* theta, float* v, const float* g, void* shadow, int64_t n, float lr,
                   float mu, int64_t* step, cudaStream_t st) {
   int64_t n4 = n / 4;
-  sgd_momentum_k<<<elementwise_blocks(n4, 256), 256, 0, st>>>(
+  launch_k(sgd_momentum_k, elementwise_blocks(n4, 256), 256, 0, st, 
       (float4*)theta, (float4*)v, (const float4*)g, (uint2*)shadow, n4, lr, mu, step);
 }
 __global__ void f32_to_bf16_k(const float* x, bf16* y, int64_t n) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE(i, n) y[i] = __float2bfloat16_rn(x[i]);
 }
 void f32_to_bf16(const float* x, void* y, int64_t n, cudaStream_t st) {
-  f32_to_bf16_k<<<elementwise_blocks(n, 256), 256, 0, st>>>(x, (bf16*)y, n);
+  launch_k(f32_to_bf16_k, elementwise_blocks(n, 256), 256, 0, st, x, (bf16*)y, n);
 }
 
 // ------------------------------------------------------ FedAsync axpby
@@ -592,6 +644,8 @@ void f32_to_bf16(const float* x, void* y, int64_t n, cudaStream_t st) {
 // parallelism; the scalar head/tail handles n % 8 and unaligned pointers.
 __global__ void axpby_vec_k(float4* __restrict__ g, const float4* __restrict__ l, int64_t n8,
                             float alpha) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t stride = int64_t(gridDim.x) * blockDim.x;
   for (int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; i < n8; i += stride) {
     float4 a0 = g[2 * i], a1 = g[2 * i + 1];
@@ -609,6 +663,8 @@ __global__ void axpby_vec_k(float4* __restrict__ g, const float4* __restrict__ l
   }
 }
 __global__ void axpby_scalar_k(float* g, const float* l, int64_t n, float alpha) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE(i, n) g[i] = fmaf(alpha, l[i] - g[i], g[i]);
 }
 int axpby_kernels(const float* g, const float* l, int64_t n) {
@@ -622,10 +678,10 @@ void axpby(float* g, const float* l, int64_t n, float alpha, cudaStream_t st) {
   if (n <= 0) return;
   bool aligned = ((reinterpret_cast<uintptr_t>(g) | reinterpret_cast<uintptr_t>(l)) & 15) == 0;
   int64_t n8 = aligned ? n / 8 : 0;
-  if (n8 > 0) axpby_vec_k<<<elementwise_blocks(n8, 256), 256, 0, st>>>((float4*)g, (const float4*)l, n8, alpha);
+  if (n8 > 0) launch_k(axpby_vec_k, elementwise_blocks(n8, 256), 256, 0, st, (float4*)g, (const float4*)l, n8, alpha);
   int64_t done = n8 * 8;
   if (done < n)
-    axpby_scalar_k<<<elementwise_blocks(n - done, 256), 256, 0, st>>>(g + done, l + done, n - done, alpha);
+    launch_k(axpby_scalar_k, elementwise_blocks(n - done, 256), 256, 0, st, g + done, l + done, n - done, alpha);
 }
 
 }  // namespace fo

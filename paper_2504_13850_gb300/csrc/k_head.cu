@@ -31,6 +31,8 @@ __global__ void head_fwd_ce_k(const T* __restrict__ x, const float* __restrict__
                               const float* __restrict__ bias, const int32_t* __restrict__ labels, int B,
                               int K, int C, float* __restrict__ logits, float* __restrict__ dz,
                               float* __restrict__ row_loss) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ float sm[];
   float* xr = sm;
   float* z = sm + K;
@@ -71,6 +73,8 @@ template <typename T>
 __global__ void head_wgrad_k(const float* __restrict__ dz, const T* __restrict__ x, int B, int K, int C,
                              float* __restrict__ dW, float* __restrict__ db, const float* __restrict__ row_loss,
                              float* __restrict__ losses, const int64_t* __restrict__ step, int64_t mask) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float xs[64][33];
   __shared__ float ds[64][8];
   const int kk = threadIdx.x % 32, cc = threadIdx.x / 32;
@@ -109,6 +113,8 @@ __global__ void head_wgrad_k(const float* __restrict__ dz, const T* __restrict__
 template <typename T>
 __global__ void head_dgrad_k(const float* __restrict__ dz, const float* __restrict__ W, int B, int K, int C,
                              const T* __restrict__ mask, T* __restrict__ dx, int acc) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.y;
   const int k = blockIdx.x * blockDim.x + threadIdx.x;
   if (k >= K) return;
@@ -126,9 +132,9 @@ void head_forward_loss(const void* x, int dt, const float* W, const float* bias,
                        int K, int C, float* logits, float* dz, float* row_loss, cudaStream_t st) {
   size_t sm = sizeof(float) * (K + C);
   if (dt == kF32)
-    head_fwd_ce_k<float><<<B, 256, sm, st>>>((const float*)x, W, bias, labels, B, K, C, logits, dz, row_loss);
+    launch_k(head_fwd_ce_k<float>, B, 256, sm, st, (const float*)x, W, bias, labels, B, K, C, logits, dz, row_loss);
   else
-    head_fwd_ce_k<bf16><<<B, 256, sm, st>>>((const bf16*)x, W, bias, labels, B, K, C, logits, dz, row_loss);
+    launch_k(head_fwd_ce_k<bf16>, B, 256, sm, st, (const bf16*)x, W, bias, labels, B, K, C, logits, dz, row_loss);
 }
 
 void head_weight_grad(const float* dz, const void* x, int dt, int B, int K, int C, float* dW, float* db,
@@ -136,18 +142,18 @@ void head_weight_grad(const float* dz, const void* x, int dt, int B, int K, int 
                       cudaStream_t st) {
   dim3 grid(ceil_div(K, 32), ceil_div(C, 8));
   if (dt == kF32)
-    head_wgrad_k<float><<<grid, 256, 0, st>>>(dz, (const float*)x, B, K, C, dW, db, row_loss, losses, step, mask);
+    launch_k(head_wgrad_k<float>, grid, 256, 0, st, dz, (const float*)x, B, K, C, dW, db, row_loss, losses, step, mask);
   else
-    head_wgrad_k<bf16><<<grid, 256, 0, st>>>(dz, (const bf16*)x, B, K, C, dW, db, row_loss, losses, step, mask);
+    launch_k(head_wgrad_k<bf16>, grid, 256, 0, st, dz, (const bf16*)x, B, K, C, dW, db, row_loss, losses, step, mask);
 }
 
 void head_input_grad(const float* dz, const float* W, int B, int K, int C, const void* mask, void* dx, int dt,
                      bool acc, cudaStream_t st) {
   dim3 grid(ceil_div(K, 256), B);
   if (dt == kF32)
-    head_dgrad_k<float><<<grid, 256, 0, st>>>(dz, W, B, K, C, (const float*)mask, (float*)dx, acc ? 1 : 0);
+    launch_k(head_dgrad_k<float>, grid, 256, 0, st, dz, W, B, K, C, (const float*)mask, (float*)dx, acc ? 1 : 0);
   else
-    head_dgrad_k<bf16><<<grid, 256, 0, st>>>(dz, W, B, K, C, (const bf16*)mask, (bf16*)dx, acc ? 1 : 0);
+    launch_k(head_dgrad_k<bf16>, grid, 256, 0, st, dz, W, B, K, C, (const bf16*)mask, (bf16*)dx, acc ? 1 : 0);
 }
 
 }  // namespace fo

@@ -45,6 +45,8 @@ template <typename T, int KT>
 __global__ void __launch_bounds__(256) dwconv_fwd_k(const T* __restrict__ x, const T* __restrict__ w,
                                                     const float* __restrict__ bias, T* __restrict__ y,
                                                     DwShape d) {
+  pdl_wait();
+  pdl_trigger();
   const int K = KT ? KT : d.k;
   const int64_t n_out = int64_t(d.N) * d.Ho * d.Wo * d.C;
   FO_MB_GRID_STRIDE(idx, n_out) {
@@ -76,6 +78,8 @@ __global__ void __launch_bounds__(256) dwconv_fwd_k(const T* __restrict__ x, con
 template <typename T, int KT>
 __global__ void __launch_bounds__(256) dwconv_dgrad_k(const T* __restrict__ dy, const T* __restrict__ w,
                                                       T* __restrict__ dx, DwShape d, int acc_flag) {
+  pdl_wait();
+  pdl_trigger();
   const int K = KT ? KT : d.k;
   const int64_t n_in = int64_t(d.N) * d.H * d.W * d.C;
   FO_MB_GRID_STRIDE(idx, n_in) {
@@ -116,6 +120,8 @@ template <typename T, int KT>
 __global__ void __launch_bounds__(256) dwconv_wgrad_k(const T* __restrict__ dy, const T* __restrict__ x,
                                                       float* __restrict__ pw, float* __restrict__ pb, DwShape d,
                                                       int per) {
+  pdl_wait();
+  pdl_trigger();
   constexpr int KK = KT * KT;
   __shared__ float red[8][KK + 1][33];
   const int lane = threadIdx.x % 32, warp = threadIdx.x / 32;
@@ -167,6 +173,8 @@ template <typename T>
 __global__ void __launch_bounds__(256) dwconv_wgrad_any_k(const T* __restrict__ dy, const T* __restrict__ x,
                                                           float* __restrict__ pw, float* __restrict__ pb, DwShape d,
                                                           int per) {
+  pdl_wait();
+  pdl_trigger();
   const int kk = d.k * d.k;
   const int taps = kk + (pb ? 1 : 0);
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
@@ -209,6 +217,8 @@ __device__ __forceinline__ float relu6_p3(float v) { return fminf(fmaxf(v + 3.f,
 
 template <typename T>
 __global__ void hswish_fwd_k(const T* __restrict__ x, T* __restrict__ y, int64_t n) {
+  pdl_wait();
+  pdl_trigger();
   FO_MB_GRID_STRIDE(i, n) {
     const float v = to_f(x[i]);
     y[i] = from_f<T>(v * relu6_p3(v) / 6.f);
@@ -218,6 +228,8 @@ __global__ void hswish_fwd_k(const T* __restrict__ x, T* __restrict__ y, int64_t
 template <typename T>
 __global__ void hswish_bwd_k(const T* __restrict__ x, const T* __restrict__ dy, T* __restrict__ dx, int64_t n,
                              int acc) {
+  pdl_wait();
+  pdl_trigger();
   FO_MB_GRID_STRIDE(i, n) {
     const float v = to_f(x[i]);
     const float g = v < -3.f ? 0.f : (v > 3.f ? 1.f : (2.f * v + 3.f) / 6.f);
@@ -226,12 +238,16 @@ __global__ void hswish_bwd_k(const T* __restrict__ x, const T* __restrict__ dy, 
 }
 template <typename T>
 __global__ void hsigmoid_fwd_k(const T* __restrict__ x, T* __restrict__ y, int64_t n) {
+  pdl_wait();
+  pdl_trigger();
   FO_MB_GRID_STRIDE(i, n) y[i] = from_f<T>(relu6_p3(to_f(x[i])) / 6.f);
 }
 // derivative: 1/6 strictly inside (-3, 3), else 0
 template <typename T>
 __global__ void hsigmoid_bwd_k(const T* __restrict__ x, const T* __restrict__ dy, T* __restrict__ dx, int64_t n,
                                int acc) {
+  pdl_wait();
+  pdl_trigger();
   FO_MB_GRID_STRIDE(i, n) {
     const float v = to_f(x[i]);
     store_acc(dx, i, (v > -3.f && v < 3.f) ? to_f(dy[i]) / 6.f : 0.f, acc != 0);
@@ -243,6 +259,8 @@ __global__ void hsigmoid_bwd_k(const T* __restrict__ x, const T* __restrict__ dy
 template <typename T>
 __global__ void chmul_fwd_k(const T* __restrict__ x, const T* __restrict__ sc, T* __restrict__ y, int N, int HW,
                             int C) {
+  pdl_wait();
+  pdl_trigger();
   FO_MB_GRID_STRIDE(i, int64_t(N) * HW * C) {
     const int c = int(i % C);
     const int64_t n = i / (int64_t(HW) * C);
@@ -254,6 +272,8 @@ __global__ void chmul_fwd_k(const T* __restrict__ x, const T* __restrict__ sc, T
 template <typename T>
 __global__ void chmul_bwd_k(const T* __restrict__ x, const T* __restrict__ sc, const T* __restrict__ dy,
                             T* __restrict__ dx, T* __restrict__ ds, int N, int HW, int C, int acc_dx, int acc_ds) {
+  pdl_wait();
+  pdl_trigger();
   FO_MB_GRID_STRIDE(o, int64_t(N) * C) {
     const int c = int(o % C);
     const int64_t n = o / C;
@@ -276,9 +296,9 @@ void dwconv_fwd(const DwShape& d, const void* x, const void* w, const float* bia
   const int64_t n = int64_t(d.N) * d.Ho * d.Wo * d.C;
   const int blocks = elementwise_blocks(n, 256);
   FO_MB_DISPATCH(dt, T, {
-    if (d.k == 3) dwconv_fwd_k<T, 3><<<blocks, 256, 0, st>>>((const T*)x, (const T*)w, bias, (T*)y, d);
-    else if (d.k == 5) dwconv_fwd_k<T, 5><<<blocks, 256, 0, st>>>((const T*)x, (const T*)w, bias, (T*)y, d);
-    else dwconv_fwd_k<T, 0><<<blocks, 256, 0, st>>>((const T*)x, (const T*)w, bias, (T*)y, d);
+    if (d.k == 3) launch_k(dwconv_fwd_k<T, 3>, blocks, 256, 0, st, (const T*)x, (const T*)w, bias, (T*)y, d);
+    else if (d.k == 5) launch_k(dwconv_fwd_k<T, 5>, blocks, 256, 0, st, (const T*)x, (const T*)w, bias, (T*)y, d);
+    else launch_k(dwconv_fwd_k<T, 0>, blocks, 256, 0, st, (const T*)x, (const T*)w, bias, (T*)y, d);
   });
 }
 
@@ -287,9 +307,9 @@ void dwconv_dgrad(const DwShape& d, const void* dy, const void* w, void* dx, int
   const int blocks = elementwise_blocks(n, 256);
   const int a = acc ? 1 : 0;
   FO_MB_DISPATCH(dt, T, {
-    if (d.k == 3) dwconv_dgrad_k<T, 3><<<blocks, 256, 0, st>>>((const T*)dy, (const T*)w, (T*)dx, d, a);
-    else if (d.k == 5) dwconv_dgrad_k<T, 5><<<blocks, 256, 0, st>>>((const T*)dy, (const T*)w, (T*)dx, d, a);
-    else dwconv_dgrad_k<T, 0><<<blocks, 256, 0, st>>>((const T*)dy, (const T*)w, (T*)dx, d, a);
+    if (d.k == 3) launch_k(dwconv_dgrad_k<T, 3>, blocks, 256, 0, st, (const T*)dy, (const T*)w, (T*)dx, d, a);
+    else if (d.k == 5) launch_k(dwconv_dgrad_k<T, 5>, blocks, 256, 0, st, (const T*)dy, (const T*)w, (T*)dx, d, a);
+    else launch_k(dwconv_dgrad_k<T, 0>, blocks, 256, 0, st, (const T*)dy, (const T*)w, (T*)dx, d, a);
   });
 }
 
@@ -319,40 +339,40 @@ void dwconv_wgrad_pass(const DwShape& d, const void* dy, const void* x, int dt, 
   if (d.k == 3 || d.k == 5) {
     dim3 grid(ceil_div(d.C, 32), chunks);
     FO_MB_DISPATCH(dt, T, {
-      if (d.k == 3) dwconv_wgrad_k<T, 3><<<grid, 256, 0, st>>>((const T*)dy, (const T*)x, pw, pb, d, per);
-      else dwconv_wgrad_k<T, 5><<<grid, 256, 0, st>>>((const T*)dy, (const T*)x, pw, pb, d, per);
+      if (d.k == 3) launch_k(dwconv_wgrad_k<T, 3>, grid, 256, 0, st, (const T*)dy, (const T*)x, pw, pb, d, per);
+      else launch_k(dwconv_wgrad_k<T, 5>, grid, 256, 0, st, (const T*)dy, (const T*)x, pw, pb, d, per);
     });
     return;
   }
   const int taps = d.k * d.k + (pb ? 1 : 0);
   dim3 grid(ceil_div(int64_t(taps) * d.C, 256), chunks);
-  FO_MB_DISPATCH(dt, T, dwconv_wgrad_any_k<T><<<grid, 256, 0, st>>>((const T*)dy, (const T*)x, pw, pb, d, per));
+  FO_MB_DISPATCH(dt, T, launch_k(dwconv_wgrad_any_k<T>, grid, 256, 0, st, (const T*)dy, (const T*)x, pw, pb, d, per));
 }
 
 void hswish_fwd(const void* x, void* y, int64_t n, int dt, cudaStream_t st) {
-  FO_MB_DISPATCH(dt, T, hswish_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (T*)y, n));
+  FO_MB_DISPATCH(dt, T, launch_k(hswish_fwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (T*)y, n));
 }
 void hswish_bwd(const void* x, const void* dy, void* dx, int64_t n, int dt, bool acc, cudaStream_t st) {
-  FO_MB_DISPATCH(dt, T, hswish_bwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (const T*)dy,
+  FO_MB_DISPATCH(dt, T, launch_k(hswish_bwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (const T*)dy,
                                                                                       (T*)dx, n, acc ? 1 : 0));
 }
 void hsigmoid_fwd(const void* x, void* y, int64_t n, int dt, cudaStream_t st) {
-  FO_MB_DISPATCH(dt, T, hsigmoid_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (T*)y, n));
+  FO_MB_DISPATCH(dt, T, launch_k(hsigmoid_fwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (T*)y, n));
 }
 void hsigmoid_bwd(const void* x, const void* dy, void* dx, int64_t n, int dt, bool acc, cudaStream_t st) {
-  FO_MB_DISPATCH(dt, T, hsigmoid_bwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (const T*)dy,
+  FO_MB_DISPATCH(dt, T, launch_k(hsigmoid_bwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (const T*)dy,
                                                                                         (T*)dx, n, acc ? 1 : 0));
 }
 
 void chmul_fwd(const void* x, const void* s, void* y, int N, int HW, int C, int dt, cudaStream_t st) {
   const int64_t n = int64_t(N) * HW * C;
-  FO_MB_DISPATCH(dt, T, chmul_fwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (const T*)s, (T*)y,
+  FO_MB_DISPATCH(dt, T, launch_k(chmul_fwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (const T*)s, (T*)y,
                                                                                      N, HW, C));
 }
 void chmul_bwd(const void* x, const void* s, const void* dy, void* dx, bool acc_dx, void* ds, bool acc_ds, int N,
                int HW, int C, int dt, cudaStream_t st) {
   const int64_t n = int64_t(N) * C;
-  FO_MB_DISPATCH(dt, T, chmul_bwd_k<T><<<elementwise_blocks(n, 256), 256, 0, st>>>((const T*)x, (const T*)s,
+  FO_MB_DISPATCH(dt, T, launch_k(chmul_bwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (const T*)s,
                                                                                      (const T*)dy, (T*)dx, (T*)ds, N,
                                                                                      HW, C, acc_dx ? 1 : 0,
                                                                                      acc_ds ? 1 : 0));

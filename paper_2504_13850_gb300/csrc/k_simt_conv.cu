@@ -93,6 +93,8 @@ __global__ void __launch_bounds__(NT) simt_conv_kernel(Geo g, const TA* __restri
                                                        const float* __restrict__ bias,
                                                        TC* __restrict__ c, int relu, int acc,
                                                        const TC* __restrict__ mask) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float As[BK][BM + 4];
   __shared__ float Bs[BK][BN + 4];
   const int tid = threadIdx.x;
@@ -160,6 +162,8 @@ Geo make_geo(const ConvShape& s, int mode) {
 
 // Sums the `splits` partial outputs [splits][n] in order.
 __global__ void sum_splits_k(const float* __restrict__ part, int splits, int64_t n, float* __restrict__ out) {
+  pdl_wait();
+  pdl_trigger();
   for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < n; i += int64_t(gridDim.x) * blockDim.x) {
     float t = 0.f;
     for (int z = 0; z < splits; ++z) t += part[int64_t(z) * n + i];
@@ -182,7 +186,7 @@ template <int MODE, typename TA, typename TB, typename TC>
 void launch(const Geo& g, const void* a, const void* b, const float* bias, void* c, bool relu,
             bool acc, cudaStream_t st, const void* mask = nullptr) {
   dim3 grid(ceil_div(g.Ncol, BN), ceil_div(g.M, BM), unsigned(ceil_div(g.K, g.kper)));
-  simt_conv_kernel<MODE, TA, TB, TC><<<grid, NT, 0, st>>>(
+  launch_k(simt_conv_kernel<MODE, TA, TB, TC>, grid, NT, 0, st, 
       g, (const TA*)a, (const TB*)b, bias, (TC*)c, relu ? 1 : 0, acc ? 1 : 0, (const TC*)mask);
 }
 
@@ -248,7 +252,7 @@ void conv_wgrad_simt(const ConvShape& s, const void* dy, int dt_dy, const void* 
   const int real = int(ceil_div(g.K, g.kper));
   launch_any<WGRAD>(g, dy, dt_dy, x, dt_x, nullptr, scratch, kF32, false, false, st);
   const int64_t n = g.M * g.Ncol;
-  sum_splits_k<<<int(std::min<int64_t>(ceil_div(n, 256), 4 * sm_count())), 256, 0, st>>>(scratch, real, n, dw);
+  launch_k(sum_splits_k, int(std::min<int64_t>(ceil_div(n, 256), 4 * sm_count())), 256, 0, st, scratch, real, n, dw);
 }
 
 }  // namespace fo

@@ -365,6 +365,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_trigger();   // every block of this kernel is resident and holds its tensor memory
+  pdl_wait();      // the previous kernel's writes are visible from here on
 
   if (warp == 0) {
     if (lane == 0) {
@@ -549,6 +551,8 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
   if (PAIR) cluster_sync_all();   // the peer's barriers are initialised
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_trigger();
+  pdl_wait();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -1219,7 +1223,7 @@ void tc_run(TcGemm* g, const void* input, cudaStream_t st) {
   if (g->input_A) g->p.tmA = g->slot_maps[c->slot];
   if (g->input_B) g->p.tmB = g->slot_maps[c->slot];
   if (g->splits == 1 && !g->pair) {
-    g->fn<<<g->grid, kPersistThreads, g->smem, st>>>(g->p);
+    launch_k(g->fn, g->grid, kPersistThreads, g->smem, st, g->p);
     return;
   }
   if (g->pair) {
@@ -1228,13 +1232,15 @@ void tc_run(TcGemm* g, const void* input, cudaStream_t st) {
     cfg.blockDim = dim3(kPersistThreads);
     cfg.dynamicSmemBytes = g->smem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = pdl_enabled() ? 2 : 1;
     cudaLaunchKernelEx(&cfg, g->fn, g->p);
     return;
   }
@@ -1243,13 +1249,15 @@ void tc_run(TcGemm* g, const void* input, cudaStream_t st) {
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = g->smem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 1;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = g->splits;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = pdl_enabled() ? 2 : 1;
   cudaLaunchKernelEx(&cfg, g->fn, g->p);
 }
 

@@ -41,6 +41,8 @@ __device__ __forceinline__ void st8(bf16* p, const V8& r) {
 
 __global__ void relu_bwd_x8_k(const bf16* __restrict__ y, const bf16* __restrict__ dy, bf16* __restrict__ dx,
                               int64_t n8, int acc) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE8(i, n8) {
     const V8 m = ld8(y + 8 * i), g = ld8(dy + 8 * i);
     V8 o;
@@ -57,6 +59,8 @@ __global__ void relu_bwd_x8_k(const bf16* __restrict__ y, const bf16* __restrict
 
 __global__ void add_x8_k(const bf16* __restrict__ a, const bf16* __restrict__ b, bf16* __restrict__ y, int64_t n8,
                          int relu) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE8(i, n8) {
     const V8 p = ld8(a + 8 * i), q = ld8(b + 8 * i);
     V8 o;
@@ -67,6 +71,8 @@ __global__ void add_x8_k(const bf16* __restrict__ a, const bf16* __restrict__ b,
 }
 
 __global__ void copy_acc_x8_k(const bf16* __restrict__ x, bf16* __restrict__ y, int64_t n8, int acc) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE8(i, n8) {
     if (!acc) {
       *reinterpret_cast<uint4*>(y + 8 * i) = *reinterpret_cast<const uint4*>(x + 8 * i);
@@ -82,6 +88,8 @@ __global__ void copy_acc_x8_k(const bf16* __restrict__ x, bf16* __restrict__ y, 
 
 __global__ void affine_fwd_x8_k(const bf16* __restrict__ x, const float* __restrict__ sc,
                                 const float* __restrict__ sh, bf16* __restrict__ y, int64_t n8, int C, int relu) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE8(i, n8) {
     const int c = int((8 * i) % C);
     const V8 p = ld8(x + 8 * i);
@@ -105,6 +113,8 @@ __device__ __forceinline__ float hswish_d(float v) { return v < -3.f ? 0.f : (v 
 __global__ void affine_hswish_fwd_x8_k(const bf16* __restrict__ x, const float* __restrict__ sc,
                                        const float* __restrict__ sh, bf16* __restrict__ pre, bf16* __restrict__ post,
                                        int64_t n8, int C) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE8(i, n8) {
     const int c = int((8 * i) % C);
     const V8 p = ld8(x + 8 * i);
@@ -122,6 +132,8 @@ __global__ void affine_hswish_fwd_x8_k(const bf16* __restrict__ x, const float* 
 __device__ __forceinline__ float gelu_cdf(float x) { return 0.5f * (1.f + erff(x * 0.70710678118654752f)); }
 
 __global__ void gelu_fwd_x8_k(const bf16* __restrict__ x, bf16* __restrict__ y, int64_t n8) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE8(i, n8) {
     const V8 p = ld8(x + 8 * i);
     V8 o;
@@ -133,6 +145,8 @@ __global__ void gelu_fwd_x8_k(const bf16* __restrict__ x, bf16* __restrict__ y, 
 
 __global__ void gelu_bwd_x8_k(const bf16* __restrict__ x, const bf16* __restrict__ dy, bf16* __restrict__ dx,
                               int64_t n8, int acc) {
+  pdl_wait();
+  pdl_trigger();
   GRID_STRIDE8(i, n8) {
     const V8 p = ld8(x + 8 * i), g = ld8(dy + 8 * i);
     V8 o;
@@ -229,7 +243,9 @@ template <int MODE>
 __global__ void __launch_bounds__(256) colsum8_k(const bf16* __restrict__ a, const bf16* __restrict__ x,
                                                  const float* __restrict__ scale, bf16* __restrict__ dx, int acc,
                                                  int64_t rows, int C, int chunk, float* __restrict__ p0,
-                                                 float* __restrict__ p1, const bf16* __restrict__ pre = nullptr) {
+                                                 float* __restrict__ p1, const bf16* __restrict__ pre) {
+  pdl_wait();
+  pdl_trigger();
   colsum8_block<MODE>(a, x, scale, dx, acc, rows, C, chunk, p0, p1, blockIdx.x, blockIdx.y, pre);
 }
 
@@ -261,6 +277,8 @@ __device__ __forceinline__ int batch_task(const int* block0, int n, int b) {
 }
 
 __global__ void __launch_bounds__(256) colsum8_batch_k(const __grid_constant__ ColsumBatch p) {
+  pdl_wait();
+  pdl_trigger();
   const int t = batch_task(p.block0, p.n, blockIdx.x);
   const int local = blockIdx.x - p.block0[t];
   const int cbs = (p.C[t] + 255) / 256;
@@ -277,6 +295,8 @@ __global__ void __launch_bounds__(256) layernorm_bwd_fused_k(const bf16* __restr
                                                              const bf16* __restrict__ dy, bf16* __restrict__ dx,
                                                              int64_t rows, int C, int acc, float* __restrict__ pg,
                                                              float* __restrict__ pb) {
+  pdl_wait();
+  pdl_trigger();
   constexpr int kMaxV = 2;  // up to 2 x 8 x 32 = 512 columns per row
   __shared__ float redg[8][512];
   __shared__ float redb[8][512];
@@ -361,6 +381,8 @@ __global__ void __launch_bounds__(256) layernorm_bwd_fused_k(const bf16* __restr
 }
 
 __global__ void finish_k(const float* __restrict__ partial, int chunks, int C, float* __restrict__ out) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float red[8][33];
   const int cl = threadIdx.x % 32, rl = threadIdx.x / 32;
   const int c = blockIdx.x * 32 + cl;
@@ -390,6 +412,8 @@ __global__ void finish_k(const float* __restrict__ partial, int chunks, int C, f
 // Batched finish: block b covers 32 columns of task t (same fixed summation
 // order as finish_k).
 __global__ void __launch_bounds__(256) finish_batch_k(const __grid_constant__ FinishBatch p) {
+  pdl_wait();
+  pdl_trigger();
   const int t = batch_task(p.block0, p.n, blockIdx.x);
   const int local = blockIdx.x - p.block0[t];
   __shared__ float red[8][33];
@@ -445,28 +469,28 @@ int adaptive_chunk(int64_t rows, int C) {
 bool vec8_ok(int dt, int64_t n) { return dt == kBF16 && n % 8 == 0; }
 
 void relu_bwd_x8(const void* y, const void* dy, void* dx, int64_t n, bool acc, cudaStream_t st) {
-  relu_bwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)y, (const bf16*)dy, (bf16*)dx, n / 8, acc);
+  launch_k(relu_bwd_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)y, (const bf16*)dy, (bf16*)dx, n / 8, acc);
 }
 void add_x8(const void* a, const void* b, void* y, int64_t n, bool relu, cudaStream_t st) {
-  add_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)a, (const bf16*)b, (bf16*)y, n / 8, relu);
+  launch_k(add_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)a, (const bf16*)b, (bf16*)y, n / 8, relu);
 }
 void copy_acc_x8(const void* x, void* y, int64_t n, bool acc, cudaStream_t st) {
-  copy_acc_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, (bf16*)y, n / 8, acc);
+  launch_k(copy_acc_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)x, (bf16*)y, n / 8, acc);
 }
 void affine_fwd_x8(const void* x, const float* sc, const float* sh, void* y, int64_t n, int C, bool relu,
                    cudaStream_t st) {
-  affine_fwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, sc, sh, (bf16*)y, n / 8, C, relu);
+  launch_k(affine_fwd_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)x, sc, sh, (bf16*)y, n / 8, C, relu);
 }
 void affine_hswish_fwd_x8(const void* x, const float* sc, const float* sh, void* pre, void* post, int64_t n, int C,
                           cudaStream_t st) {
-  affine_hswish_fwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, sc, sh, (bf16*)pre,
+  launch_k(affine_hswish_fwd_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)x, sc, sh, (bf16*)pre,
                                                                           (bf16*)post, n / 8, C);
 }
 void gelu_fwd_x8(const void* x, void* y, int64_t n, cudaStream_t st) {
-  gelu_fwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, (bf16*)y, n / 8);
+  launch_k(gelu_fwd_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)x, (bf16*)y, n / 8);
 }
 void gelu_bwd_x8(const void* x, const void* dy, void* dx, int64_t n, bool acc, cudaStream_t st) {
-  gelu_bwd_x8_k<<<elementwise_blocks(n / 8, 256), 256, 0, st>>>((const bf16*)x, (const bf16*)dy, (bf16*)dx, n / 8, acc);
+  launch_k(gelu_bwd_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)x, (const bf16*)dy, (bf16*)dx, n / 8, acc);
 }
 
 int64_t colsum8_partial_floats(int64_t rows, int C, bool adaptive) {
@@ -476,8 +500,8 @@ int64_t colsum8_partial_floats(int64_t rows, int C, bool adaptive) {
 void colsum8(const void* a, int64_t rows, int C, float* partial, float* out, bool adaptive, cudaStream_t st) {
   const int ch = adaptive ? adaptive_chunk(rows, C) : kChunk;
   dim3 grid(ceil_div(C, 256), chunks_of(rows, ch));
-  colsum8_k<0><<<grid, 256, 0, st>>>((const bf16*)a, nullptr, nullptr, nullptr, 0, rows, C, ch, partial, nullptr);
-  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, chunks_of(rows, ch), C, out);
+  launch_k(colsum8_k<0>, grid, 256, 0, st, (const bf16*)a, nullptr, nullptr, nullptr, 0, rows, C, ch, partial, nullptr, nullptr);
+  launch_k(finish_k, ceil_div(C, 32), 256, 0, st, partial, chunks_of(rows, ch), C, out);
 }
 
 void affine_bwd8(const void* dy, const void* x, const float* scale, void* dx, bool acc, int64_t rows, int C,
@@ -485,10 +509,10 @@ void affine_bwd8(const void* dy, const void* x, const float* scale, void* dx, bo
   const int ch = adaptive_chunk(rows, C);
   dim3 grid(ceil_div(C, 256), chunks_of(rows, ch));
   float* p1 = partial + colsum8_partial_floats(rows, C, true);
-  colsum8_k<1><<<grid, 256, 0, st>>>((const bf16*)dy, (const bf16*)x, scale, (bf16*)dx, acc, rows, C, ch, partial,
-                                     p1);
-  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, chunks_of(rows, ch), C, dscale);
-  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(p1, chunks_of(rows, ch), C, dshift);
+  launch_k(colsum8_k<1>, grid, 256, 0, st, (const bf16*)dy, (const bf16*)x, scale, (bf16*)dx, acc, rows, C, ch, partial,
+                                     p1, nullptr);
+  launch_k(finish_k, ceil_div(C, 32), 256, 0, st, partial, chunks_of(rows, ch), C, dscale);
+  launch_k(finish_k, ceil_div(C, 32), 256, 0, st, p1, chunks_of(rows, ch), C, dshift);
 }
 
 int affine_bwd8_chunks(int64_t rows, int C) { return chunks_of(rows, adaptive_chunk(rows, C)); }
@@ -498,11 +522,11 @@ void affine_bwd8_pass(const void* dy, const void* x, const float* scale, void* d
   const int ch = adaptive_chunk(rows, C);
   dim3 grid(ceil_div(C, 256), chunks_of(rows, ch));
   if (hswish_in)
-    colsum8_k<2><<<grid, 256, 0, st>>>((const bf16*)dy, (const bf16*)x, scale, (bf16*)dx, acc, rows, C, ch, p_scale,
+    launch_k(colsum8_k<2>, grid, 256, 0, st, (const bf16*)dy, (const bf16*)x, scale, (bf16*)dx, acc, rows, C, ch, p_scale,
                                        p_shift, (const bf16*)hswish_in);
   else
-    colsum8_k<1><<<grid, 256, 0, st>>>((const bf16*)dy, (const bf16*)x, scale, (bf16*)dx, acc, rows, C, ch, p_scale,
-                                       p_shift);
+    launch_k(colsum8_k<1>, grid, 256, 0, st, (const bf16*)dy, (const bf16*)x, scale, (bf16*)dx, acc, rows, C, ch, p_scale,
+                                       p_shift, nullptr);
 }
 
 int colsum8_batch_chunks(int64_t rows) { return chunks_of(rows, kChunk); }
@@ -523,7 +547,7 @@ void colsum8_batched(const std::vector<ColsumTask>& tasks, cudaStream_t st) {
       blocks += ceil_div(t.C, 256) * chunks_of(t.rows, kChunk);
     }
     p.block0[p.n] = blocks;
-    if (blocks) colsum8_batch_k<<<blocks, 256, 0, st>>>(p);
+    if (blocks) launch_k(colsum8_batch_k, blocks, 256, 0, st, p);
   }
 }
 
@@ -542,7 +566,7 @@ void finish_batched(const std::vector<FinishTask>& tasks, cudaStream_t st) {
       blocks += ceil_div(t.C, 32);
     }
     p.block0[p.n] = blocks;
-    if (blocks) finish_batch_k<<<blocks, 256, 0, st>>>(p);
+    if (blocks) launch_k(finish_batch_k, blocks, 256, 0, st, p);
   }
 }
 
@@ -552,7 +576,7 @@ int layernorm_bwd8_blocks(int64_t rows) { return int((rows + 15) / 16); }
 
 void layernorm_bwd8_pass(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
                          void* dx, int64_t rows, int C, bool acc, float* p_gamma, float* p_beta, cudaStream_t st) {
-  layernorm_bwd_fused_k<<<layernorm_bwd8_blocks(rows), 256, 0, st>>>((const bf16*)x, gamma, mean, rstd,
+  launch_k(layernorm_bwd_fused_k, layernorm_bwd8_blocks(rows), 256, 0, st, (const bf16*)x, gamma, mean, rstd,
                                                                       (const bf16*)dy, (bf16*)dx, rows, C, acc,
                                                                       p_gamma, p_beta);
 }
@@ -564,10 +588,10 @@ void layernorm_bwd8(const void* x, const float* gamma, const float* mean, const 
                     cudaStream_t st) {
   const int blocks = int((rows + 15) / 16);
   float* pb = partial + int64_t(blocks) * C;
-  layernorm_bwd_fused_k<<<blocks, 256, 0, st>>>((const bf16*)x, gamma, mean, rstd, (const bf16*)dy, (bf16*)dx, rows,
+  launch_k(layernorm_bwd_fused_k, blocks, 256, 0, st, (const bf16*)x, gamma, mean, rstd, (const bf16*)dy, (bf16*)dx, rows,
                                                 C, acc, partial, pb);
-  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(partial, blocks, C, dgamma);
-  finish_k<<<ceil_div(C, 32), 256, 0, st>>>(pb, blocks, C, dbeta);
+  launch_k(finish_k, ceil_div(C, 32), 256, 0, st, partial, blocks, C, dgamma);
+  launch_k(finish_k, ceil_div(C, 32), 256, 0, st, pb, blocks, C, dbeta);
 }
 
 }  // namespace fo

@@ -52,7 +52,7 @@ def small_mobile(dtype):
     t = b.add("linear", t, cin=96, cout=64, bias=1)
     t = b.add("hswish", t)
     b.add("linear", t, cin=64, cout=10, bias=1)
-    return W.shrink(W.CONFIGS["mobilenet"], ops=b.ops, batch=10, in_hwc=(7, 7, 24), K=3, omega=6, depth=2,
+    return W.shrink(W.CONFIGS["mobilenet"], ops=b.ops, classes=10, batch=10, in_hwc=(7, 7, 24), K=3, omega=6, depth=2,
                     dtype=dtype)
 
 
@@ -83,7 +83,7 @@ def test_depthwise_gradients_reach_the_input_layer():
     t = b.add("hswish", t)
     t = b.add("flatten", t)
     b.add("linear", t, cin=4 * 4 * 16, cout=10, bias=1)
-    cfg = W.shrink(W.CONFIGS["mobilenet"], ops=b.ops, batch=6, in_hwc=(8, 8, 16), K=2, omega=4, depth=2,
+    cfg = W.shrink(W.CONFIGS["mobilenet"], ops=b.ops, classes=10, batch=6, in_hwc=(8, 8, 16), K=2, omega=4, depth=2,
                    dtype=W.F32)
     compare(cfg, prefill_then_steps(cfg, 4), loss_tol=1e-4, param_tol=1e-4, upd_tol=1e-4)
 
@@ -100,7 +100,7 @@ def test_bad_mobile_shapes_are_refused():
         ops = ops + [{"kind": "flatten", "in0": 1}, {"kind": "linear", "in0": 2, "cin": 4 * 4 * 112, "cout": 10,
                                                       "bias": 1}]
         with pytest.raises(RuntimeError):
-            api.Server.from_config(W.shrink(base, ops=ops))
+            api.Server.from_config(W.shrink(base, ops=ops, classes=10))
 
 
 def test_depthwise_any_kernel_size():
@@ -115,7 +115,7 @@ def test_depthwise_any_kernel_size():
     t = b.add("flatten", t)
     b.add("linear", t, cin=4 * 4 * 16, cout=10, bias=1)
     for dtype in (W.F32, W.BF16):
-        cfg = W.shrink(W.CONFIGS["mobilenet"], ops=b.ops, batch=6, in_hwc=(8, 8, 16), K=2, omega=4, depth=2,
+        cfg = W.shrink(W.CONFIGS["mobilenet"], ops=b.ops, classes=10, batch=6, in_hwc=(8, 8, 16), K=2, omega=4, depth=2,
                        dtype=dtype)
         if dtype == W.F32:
             compare(cfg, prefill_then_steps(cfg, 4), loss_tol=1e-4, param_tol=1e-4, upd_tol=1e-4)
