@@ -67,6 +67,9 @@ struct TcParams {
   const bf16* mask;     // ReLU mask (same layout as out): keep where mask > 0
   int relu, acc, out_f32;
   int* err;
+  // split-K: fp32 partial tiles, [tile][rank][BN/32][8][BM] float4 (tile =
+  // blockIdx.y * gridDim.x + blockIdx.x); only rows a rank does not own are written
+  float* ws;
 };
 
 __device__ __forceinline__ size_t out_row(const TcParams& p, int m) {
@@ -80,7 +83,21 @@ __device__ __forceinline__ size_t out_row(const TcParams& p, int m) {
 // ReLU, ReLU mask, accumulate, store as fp32 or bf16 (16-byte accesses).
 // `sbias`: shared-memory address of the bias values for columns n..n+31.
 // Columns >= N (the ragged last tile; N is a multiple of 8) are not touched.
-__device__ __forceinline__ void store_row32(const TcParams& p, int m_gemm, int n, float (&v)[32], uint32_t sbias) {
+// bf16 outputs take their ReLU-mask and accumulate operands preloaded by
+// load_row32 (so that a caller can fetch them ahead of time).
+__device__ __forceinline__ void load_row32(const TcParams& p, int m_gemm, int n, uint4 (&mk)[4], uint4 (&ac)[4]) {
+  const int nv = p.N - n;
+  if (p.out_f32 || nv <= 0 || m_gemm >= p.M) return;
+  const size_t m = out_row(p, m_gemm);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    if (8 * j >= nv) break;
+    if (p.mask) mk[j] = *reinterpret_cast<const uint4*>(p.mask + m * p.ldo + n + 8 * j);
+    if (p.acc) ac[j] = *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(p.out) + m * p.ldo + n + 8 * j);
+  }
+}
+__device__ __forceinline__ void store_row32(const TcParams& p, int m_gemm, int n, float (&v)[32], uint32_t sbias,
+                                            const uint4 (&mk)[4], const uint4 (&ac)[4]) {
   const size_t m = out_row(p, m_gemm);
   const int nv = p.N - n;   // valid columns from n
   if (nv <= 0) return;
@@ -94,19 +111,19 @@ __device__ __forceinline__ void store_row32(const TcParams& p, int m_gemm, int n
   if (p.relu)
 #pragma unroll
     for (int j = 0; j < 32; ++j) v[j] = fmaxf(v[j], 0.f);
-  if (p.mask) {
-    const uint4* mk = reinterpret_cast<const uint4*>(p.mask + m * p.ldo + n);
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      if (8 * j >= nv) break;
-      const uint4 u = mk[j];
-      const bf16* e = reinterpret_cast<const bf16*>(&u);
-#pragma unroll
-      for (int q = 0; q < 8; ++q)
-        if (!(__bfloat162float(e[q]) > 0.f)) v[8 * j + q] = 0.f;
-    }
-  }
   if (p.out_f32) {
+    if (p.mask) {
+      const uint4* mkp = reinterpret_cast<const uint4*>(p.mask + m * p.ldo + n);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        if (8 * j >= nv) break;
+        const uint4 u = mkp[j];
+        const bf16* e = reinterpret_cast<const bf16*>(&u);
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          if (!(__bfloat162float(e[q]) > 0.f)) v[8 * j + q] = 0.f;
+      }
+    }
     float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + m * p.ldo + n);
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
@@ -122,9 +139,14 @@ __device__ __forceinline__ void store_row32(const TcParams& p, int m_gemm, int n
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       if (8 * j >= nv) break;
+      if (p.mask) {
+        const bf16* e = reinterpret_cast<const bf16*>(&mk[j]);
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          if (!(__bfloat162float(e[q]) > 0.f)) v[8 * j + q] = 0.f;
+      }
       if (p.acc) {
-        const uint4 o = dst[j];
-        const bf16* ob = reinterpret_cast<const bf16*>(&o);
+        const bf16* ob = reinterpret_cast<const bf16*>(&ac[j]);
 #pragma unroll
         for (int e = 0; e < 8; ++e) v[8 * j + e] += __bfloat162float(ob[e]);
       }
@@ -166,6 +188,24 @@ __device__ __forceinline__ void load_bias8(const TcParams& p, int lane, int n, f
 
 __device__ __forceinline__ void epilogue_chunk32(const TcParams& p, uint32_t stage, int lane, int m_base, int n,
                                                  const uint32_t (&r)[32], const float (&b)[8]) {
+  // bf16 outputs: the chunk's ReLU-mask and accumulate operands (four rows
+  // per lane) are loaded before the staging, all at once, so that their
+  // latency overlaps the staging and each other instead of adding up row by
+  // row (the dominant cost of an input-gradient epilogue otherwise).
+  const int co = lane & 3;                   // bf16: columns 8co .. 8co+7
+  uint4 mk[4] = {}, ac[4] = {};
+  size_t off[4];
+  bool ok[4];
+  if (!p.out_f32) {
+#pragma unroll
+    for (int it = 0; it < 4; ++it) {
+      const int mg = m_base + it * 8 + (lane >> 2);
+      ok[it] = mg < p.M && n + 8 * co < p.N;
+      off[it] = ok[it] ? out_row(p, mg) * p.ldo + n + 8 * co : 0;
+      if (p.mask && ok[it]) mk[it] = *reinterpret_cast<const uint4*>(p.mask + off[it]);
+      if (p.acc && ok[it]) ac[it] = *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(p.out) + off[it]);
+    }
+  }
 #pragma unroll
   for (int j = 0; j < 8; ++j)
     st_shared4(stage + 16u * (lane * 8 + (j ^ (lane & 7))), r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
@@ -185,10 +225,10 @@ __device__ __forceinline__ void epilogue_chunk32(const TcParams& p, uint32_t sta
           for (int q = 0; q < 4; ++q) e[q] = fmaxf(e[q], 0.f);
         if (p.mask) {
           const uint2 u = *reinterpret_cast<const uint2*>(p.mask + m * p.ldo + n + 4 * cq);
-          const bf16* mk = reinterpret_cast<const bf16*>(&u);
+          const bf16* mkp = reinterpret_cast<const bf16*>(&u);
 #pragma unroll
           for (int q = 0; q < 4; ++q)
-            if (!(__bfloat162float(mk[q]) > 0.f)) e[q] = 0.f;
+            if (!(__bfloat162float(mkp[q]) > 0.f)) e[q] = 0.f;
         }
         float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + m * p.ldo + n) + cq;
         if (p.acc) {
@@ -199,15 +239,12 @@ __device__ __forceinline__ void epilogue_chunk32(const TcParams& p, uint32_t sta
       }
     }
   } else {
-    const int co = lane & 3;                 // columns 8co .. 8co+7
-#pragma unroll 1
+#pragma unroll
     for (int it = 0; it < 4; ++it) {
       const int rr = it * 8 + (lane >> 2);
-      const int mg = m_base + rr;
       const float4 v0 = ld_shared4(stage + 16u * (rr * 8 + ((2 * co) ^ (rr & 7))));
       const float4 v1 = ld_shared4(stage + 16u * (rr * 8 + ((2 * co + 1) ^ (rr & 7))));
-      if (mg < p.M && n + 8 * co < p.N) {
-        const size_t m = out_row(p, mg);
+      if (ok[it]) {
         float e[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
 #pragma unroll
         for (int q = 0; q < 8; ++q) e[q] += b[q];
@@ -215,16 +252,13 @@ __device__ __forceinline__ void epilogue_chunk32(const TcParams& p, uint32_t sta
 #pragma unroll
           for (int q = 0; q < 8; ++q) e[q] = fmaxf(e[q], 0.f);
         if (p.mask) {
-          const uint4 u = *reinterpret_cast<const uint4*>(p.mask + m * p.ldo + n + 8 * co);
-          const bf16* mk = reinterpret_cast<const bf16*>(&u);
+          const bf16* mkp = reinterpret_cast<const bf16*>(&mk[it]);
 #pragma unroll
           for (int q = 0; q < 8; ++q)
-            if (!(__bfloat162float(mk[q]) > 0.f)) e[q] = 0.f;
+            if (!(__bfloat162float(mkp[q]) > 0.f)) e[q] = 0.f;
         }
-        uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(p.out) + m * p.ldo + n + 8 * co);
         if (p.acc) {
-          const uint4 o = *dst;
-          const bf16* eo = reinterpret_cast<const bf16*>(&o);
+          const bf16* eo = reinterpret_cast<const bf16*>(&ac[it]);
 #pragma unroll
           for (int q = 0; q < 8; ++q) e[q] += __bfloat162float(eo[q]);
         }
@@ -235,7 +269,7 @@ __device__ __forceinline__ void epilogue_chunk32(const TcParams& p, uint32_t sta
           __nv_bfloat162 h2 = __floats2bfloat162_rn(e[2 * q], e[2 * q + 1]);
           pw[q] = *reinterpret_cast<uint32_t*>(&h2);
         }
-        *dst = pk;
+        *reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(p.out) + off[it]) = pk;
       }
     }
   }
@@ -310,13 +344,19 @@ __device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, i
 }
 
 // Split-K: the gridDim.z CTAs of a (1, 1, S) cluster each run k-blocks
-// [kb0, kb0 + kper) of the same output tile.  Rank z owns rows
-// [z*BM/S, (z+1)*BM/S) of the tile.  After the MMAs every CTA pushes the
-// accumulator rows it does not own straight from TMEM into the owner's
-// shared memory (distributed-shared-memory stores, one slot per source rank)
-// and arrives, with release semantics, on the owner's receive barrier (one
-// arrival per row); the owner then adds the S partials of its rows in rank
-// order (deterministic) and runs the epilogue.
+// [kb0, kb0 + kper) of the same output tile.  Rank z owns the 32-column
+// chunks [z*NC/S, (z+1)*NC/S) of the tile (NC = BN/32), all 128 rows, so all
+// four epilogue warps of every CTA take part.  After the MMAs every CTA
+// writes the chunks it does not own from TMEM to its slice of a global fp32
+// workspace (L2-resident; each warp store covers 512 contiguous bytes); the
+// cluster barrier (release / acquire) orders those writes before the owners'
+// reads; each owner pulls the other ranks' slices of its chunks into its idle
+// pipeline buffers with bulk copies, adds the S partials in rank order
+// (deterministic) and runs the epilogue, with the ReLU-mask / accumulate
+// operands of the next chunk loaded while the current one is stored.
+// (Distributed-shared-memory stores moved these partials at only ~20 GB/s
+// per SM pair, and an owner that read them chunk by chunk from L2 waited a
+// full round trip per chunk.)
 template <int KIND, int BN, int STAGES>
 __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ TcParams p) {
   extern __shared__ __align__(1024) char smem_raw[];
@@ -324,11 +364,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
   constexpr int A_BYTES = BM * BK * 2;
   constexpr int B_BYTES = BN * BK * 2;
   constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  constexpr int RS = BN + 4;   // receive-buffer row stride in floats (padding against bank conflicts)
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
   uint64_t* empty = full + STAGES;
   uint64_t* accum = empty + STAGES;
-  uint64_t* rbar = accum + 1;
+  uint64_t* rbar = accum + 1;   // the owner's bulk copies of the other ranks' partials
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rbar + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   float* sbias = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES + 256);   // bias[n0 .. n0 + BN)
@@ -339,8 +378,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
   const int kb0 = me * p.kper;
   const int kb1 = min(p.KB, kb0 + p.kper);
   const int nk = kb1 - kb0;
-  const int maxr = (BM + S - 1) / S;            // rows per receive slot
-  const int r0 = me * BM / S, r1 = (me + 1) * BM / S;
+  constexpr int NC = BN / 32;
+  const int c0 = me * NC / S, c1 = (me + 1) * NC / S;   // owned 32-column chunks
   constexpr uint32_t kCols = BN < 32 ? 32 : BN;
 
   if (threadIdx.x == 0) {
@@ -349,7 +388,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
       mbar_init(&empty[s], 1);
     }
     mbar_init(accum, 1);
-    mbar_init(rbar, (S - 1) * (r1 - r0));   // one release-arrive per pushed row
+    mbar_init(rbar, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmA)) : "memory");
@@ -418,65 +457,81 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     if (!mbar_wait(accum, 0)) atomicExch(p.err, 3);
     tc_fence_after();
   }
-  // Every CTA of the cluster is past its MMAs: its pipeline buffers (now the
-  // receive slots) are free and its receive barrier is armed.
+  // Chunks this CTA does not own go to its slice of the workspace:
+  // ws_tile[rank][chunk][j][row] (float4), one 16 KB slice per (rank, chunk).
+  constexpr int SLICE = 8 * BM;   // float4 per slice
+  const size_t tile = size_t(blockIdx.y) * gridDim.x + blockIdx.x;
+  float4* ws_tile = reinterpret_cast<float4*>(p.ws) + tile * size_t(S) * NC * SLICE;
+  const int q = warp % 4, row = q * 32 + lane;
+  const uint32_t trow = tmem + (uint32_t(q * 32) << 16);
+  if (warp >= 2) {
+    float4* dst = ws_tile + size_t(me) * NC * SLICE + row;
+#pragma unroll 1
+    for (int c = 0; c < NC; ++c) {
+      if (c >= c0 && c < c1) continue;
+      uint32_t r[32];
+      tmem_ld32(trow + uint32_t(32 * c), r);
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        __stcg(dst + (c * 8 + j) * BM,
+               make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]), __uint_as_float(r[4 * j + 2]),
+                           __uint_as_float(r[4 * j + 3])));
+    }
+  }
+  // Every CTA's partials are written (release) and visible (acquire).
   tc_fence_before();
   cluster_sync_all();
   tc_fence_after();
-  if (warp >= 2) {
-    const int q = warp % 4, row = q * 32 + lane;
-    const uint32_t trow = tmem + (uint32_t(q * 32) << 16);
-    int z = 0;                                 // owner of this row
-    while (z + 1 < S && (z + 1) * BM / S <= row) ++z;
-    const bool push = z != me;
-    const int slot = me < z ? me : me - 1;     // this rank's slot at the owner
-    const uint32_t dst = smem_u32(smem) + uint32_t(((slot * maxr + row - z * BM / S) * RS) * 4);
-    const uint32_t dst_cta = map_to_cta(dst, uint32_t(z));
-    const uint32_t bar_cta = map_to_cta(smem_u32(rbar), uint32_t(z));
-#pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
-      uint32_t r[32];
-      tmem_ld32(trow + uint32_t(c), r);
-      if (push)
-#pragma unroll
-        for (int j = 0; j < 8; ++j)
-          st_cluster4(dst_cta + uint32_t((c + 4 * j) * 4), r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
+  const int nown = c1 - c0;
+  float4* recv = reinterpret_cast<float4*>(smem);   // [(rank, chunk)][j][row]: the idle pipeline buffers
+  auto recv_slot = [&](int z, int c) { return (z < me ? z : z - 1) * nown + (c - c0); };
+  if (threadIdx.x == 64 && nown > 0) {
+    asm volatile("fence.proxy.async;" ::: "memory");   // peers' generic writes before these async-proxy reads
+    mbar_expect_tx(rbar, uint32_t((S - 1) * nown * SLICE * 16));
+    for (int z = 0; z < S; ++z) {
+      if (z == me) continue;
+      for (int c = c0; c < c1; ++c)
+        bulk_g2s(recv + size_t(recv_slot(z, c)) * SLICE, ws_tile + (size_t(z) * NC + c) * SLICE, SLICE * 16, rbar);
     }
-    if (push) mbar_arrive_remote(bar_cta);
-    // Owner: rows r0..r1-1 of this lane quarter, summed over ranks in order.
-    if (q * 32 < r1 && q * 32 + 32 > r0) {
-      if (!mbar_wait_cluster(rbar, 0)) atomicExch(p.err, 9);
-      const bool own = row >= r0 && row < r1 && m0 + row < p.M;
-      const uint32_t rbase = smem_u32(smem) + uint32_t(((row - r0) * RS) * 4);
+  }
+  if (warp >= 2 && nown > 0) {
+    const int mg = m0 + row;
+    uint4 mk[4] = {}, ac[4] = {}, mk2[4] = {}, ac2[4] = {};
+    load_row32(p, mg, n0 + 32 * c0, mk, ac);
+    if (!mbar_wait(rbar, 0)) atomicExch(p.err, 9);
 #pragma unroll 1
-      for (int c = 0; c < BN; c += 32) {
-        uint32_t r[32];
-        tmem_ld32(trow + uint32_t(c), r);
-        if (!own) continue;
+    for (int c = c0; c < c1; ++c) {
+      if (c + 1 < c1) load_row32(p, mg, n0 + 32 * (c + 1), mk2, ac2);
+      uint32_t r[32];
+      tmem_ld32(trow + uint32_t(32 * c), r);
+      if (mg < p.M) {
         float v[32];
 #pragma unroll
         for (int j = 0; j < 32; ++j) v[j] = 0.f;
 #pragma unroll 1
-        for (int s = 0; s < S; ++s) {
-          if (s == me) {
+        for (int z = 0; z < S; ++z) {
+          if (z == me) {
 #pragma unroll
             for (int j = 0; j < 32; ++j) v[j] += __uint_as_float(r[j]);
           } else {
-            const uint32_t src = rbase + uint32_t(((s < me ? s : s - 1) * maxr * RS + c) * 4);
+            const uint32_t src = smem_u32(recv + size_t(recv_slot(z, c)) * SLICE + row);
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
-              const float4 w = ld_shared4(src + 16u * j);
+              const float4 w = ld_shared4(src + uint32_t(j * BM * 16));
               v[4 * j] += w.x; v[4 * j + 1] += w.y; v[4 * j + 2] += w.z; v[4 * j + 3] += w.w;
             }
           }
         }
-        store_row32(p, m0 + row, n0 + c, v, smem_u32(sbias) + uint32_t(c) * 4u);
+        store_row32(p, mg, n0 + 32 * c, v, smem_u32(sbias) + uint32_t(32 * c) * 4u, mk, ac);
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        mk[j] = mk2[j];
+        ac[j] = ac2[j];
       }
     }
   }
-  // No CTA leaves while a peer may still be writing into it.
   tc_fence_before();
-  cluster_sync_all();
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
@@ -676,6 +731,11 @@ template <int KIND, int BN>
 constexpr int stages_for() {
   return kSmemBudget / (BM * BK * 2 + BN * BK * 2) > 8 ? 8 : kSmemBudget / (BM * BK * 2 + BN * BK * 2);
 }
+inline size_t pipeline_bytes(int bn) {
+  const int stage = BM * BK * 2 + bn * BK * 2;
+  const int stages = kSmemBudget / stage > 8 ? 8 : kSmemBudget / stage;
+  return size_t(stages) * stage;
+}
 template <int KIND, int BN>
 constexpr size_t smem_bytes(bool cluster) {
   return size_t(stages_for<KIND, BN>()) * (BM * BK * 2 + BN * BK * 2) + 1024 + 256 +
@@ -803,6 +863,8 @@ struct TcContext {
   int slot = 0;
   int* err = nullptr;
   fo_server* s = nullptr;
+  size_t ws_floats = 0;             // split-K workspace: the largest plan's need (plans run in order)
+  float* ws = nullptr;
 };
 
 namespace {
@@ -896,6 +958,8 @@ void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv, bool 
       if (!win_a && !win_b) t_kb = std::max(0.31, stage_kb / 128.0);
       for (int sp = 1; sp <= (pair ? 1 : 8); ++sp) {
         if (sp > 1 && KB / sp < 4) break;
+        // an owner's receive slices (16 KB per other rank and owned chunk) live in the pipeline buffers
+        if (sp > 1 && size_t(sp - 1) * ((bn / 32 + sp - 1) / sp) * 16384 > pipeline_bytes(bn)) continue;
         const int kper = (KB + sp - 1) / sp;
         const int splits = (KB + kper - 1) / kper;
         if (splits != sp) continue;
@@ -945,6 +1009,7 @@ TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
   const int n_tiles = (N + g->bn - 1) / g->bn;
   if (g->splits > 1) {
     g->grid = dim3(n_tiles, (M + BM - 1) / BM, g->splits);
+    c->ws_floats = std::max(c->ws_floats, size_t(g->grid.x) * g->grid.y * g->splits * BM * g->bn);
   } else if (g->pair) {
     const int work = n_tiles * ((M + BM - 1) / BM) / 2;
     g->grid = dim3(2 * std::min(work, active_clusters(c, g->kind, g->bn, 2, g->pair)), 1, 1);
@@ -996,9 +1061,14 @@ bool tc_encode_2d(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, 
 
 int* tc_error_word(TcContext* c) { return c ? c->err : nullptr; }
 
-// Allocate the split-K workspace once every plan is known.
+// Allocate the split-K workspace once every plan is known.  The GEMMs of a
+// step run one after another on one stream, so they share it.
 int tc_finalize(TcContext* c) {
-  (void)c;
+  if (!c || c->ws_floats == 0) return FO_OK;
+  c->ws = static_cast<float*>(c->s->alloc(c->ws_floats * sizeof(float)));
+  if (!c->ws) return FO_ERR_OOM;
+  for (TcGemm* g : c->gemms)
+    if (g->splits > 1) g->p.ws = c->ws;
   return FO_OK;
 }
 
