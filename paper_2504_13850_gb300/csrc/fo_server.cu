@@ -273,12 +273,13 @@ int build_plan(fo_server* s) {
   const Fusion fu = analyse(s);
   auto act = [s](int tid) -> const void* { return tid == 0 ? s->cur_in : s->T[tid].act; };
   auto add = [&plan](const char* name, int kernels, double flops, double bytes,
-                     std::function<void(cudaStream_t)> fn) {
-    plan.push_back({name, std::move(fn), kernels, flops, bytes});
+                     std::function<void(cudaStream_t)> fn, int lane = 0) {
+    plan.push_back({name, std::move(fn), kernels, flops, bytes, lane});
   };
   auto tbytes = [s](int tid) { return double(s->T[tid].bytes()); };
-  auto add_tc = [&](fo::TcGemm* g) {
-    add(fo::tc_name(g), 1, fo::tc_flops(g), 0.0, [=](cudaStream_t st) { fo::tc_run(g, nullptr, st); });
+  auto add_tc = [&](fo::TcGemm* g, int lane = 0) {
+    fo::tc_set_lane(g, lane);
+    add(fo::tc_name(g), 1, fo::tc_flops(g), 0.0, [=](cudaStream_t st) { fo::tc_run(g, nullptr, st); }, lane);
   };
   const int L = nops - 1;  // the logits layer
 
@@ -521,6 +522,19 @@ int build_plan(fo_server* s) {
                        true);
           });
         }
+        // the weight gradient only feeds the optimizer: side stream, forked
+        // before the input gradient so that the two run concurrently
+        fo::TcGemm* tw = fo::tc_plan_wgrad(s->tc, s, i);
+        if (tw) {
+          add_tc(tw, 1);
+        } else {
+          const bool split = fo::simt_wgrad_splits(cs) > 1;
+          add(op.kind == FO_OP_CONV ? "conv_wgrad_simt" : "linear_wgrad_simt", split ? 2 : 1, fl, 0.0,
+              [=](cudaStream_t st) {
+            fo::conv_wgrad_simt(cs, s->T[o].grad, dto, act(a0), s->T[a0].dt, G(s, i, 0),
+                                split ? s->simt_scratch : nullptr, st);
+          }, 1);
+        }
         if (need_dx) {
           int accf = contrib(a);
           std::vector<fo::TcGemm*> tgs;
@@ -541,17 +555,6 @@ int build_plan(fo_server* s) {
                                   accf != 0, mask, st);
             });
           }
-        }
-        fo::TcGemm* tw = fo::tc_plan_wgrad(s->tc, s, i);
-        if (tw) {
-          add_tc(tw);
-        } else {
-          const bool split = fo::simt_wgrad_splits(cs) > 1;
-          add(op.kind == FO_OP_CONV ? "conv_wgrad_simt" : "linear_wgrad_simt", split ? 2 : 1, fl, 0.0,
-              [=](cudaStream_t st) {
-            fo::conv_wgrad_simt(cs, s->T[o].grad, dto, act(a0), s->T[a0].dt, G(s, i, 0),
-                                split ? s->simt_scratch : nullptr, st);
-          });
         }
         break;
       }
@@ -759,6 +762,7 @@ int build_plan(fo_server* s) {
   }
 
   // ---------------- optimizer (Algorithm 4: theta_s <- theta_s - gamma_s * update)
+  const size_t first_opt = plan.size();   // the side stream joins before this entry
   if (!bias_tasks.empty())
     add("bias_grad", int((bias_tasks.size() + 39) / 40), 0.0, deferred_bytes, [=](cudaStream_t st) {
       fo::colsum8_batched(bias_tasks, st);
@@ -773,6 +777,7 @@ int build_plan(fo_server* s) {
   add("sgd_momentum", 1, 0.0, double(s->n_padded) * (20.0 + (s->shadow ? 2.0 : 0.0)), [=](cudaStream_t st) {
     fo::sgd_momentum(s->theta, s->mom, s->grad, s->shadow, s->n_padded, s->opt.lr, s->opt.momentum, s->d_step, st);
   });
+  plan[first_opt].join = true;
   for (int i = 0; i < nops; ++i)
     if (s->ops[i].kind == FO_OP_ATTENTION) fo::attention_prepare(s->T[s->ops[i].in0].H, s->ops[i].cin, s->ops[i].heads);
   return FO_OK;
@@ -887,8 +892,12 @@ void destroy_impl(fo_server* s) {
   }
   for (auto e : s->ev_pool) cudaEventDestroy(e);
   for (void* p : s->allocs) cudaFree(p);
+  if (s->side) cudaStreamSynchronize(s->side);
   if (s->cs) cudaStreamDestroy(s->cs);
   if (s->xs) cudaStreamDestroy(s->xs);
+  if (s->side) cudaStreamDestroy(s->side);
+  if (s->fork_ev) cudaEventDestroy(s->fork_ev);
+  if (s->join_ev) cudaEventDestroy(s->join_ev);
   delete s->sched;
   delete s;
 }
@@ -909,7 +918,27 @@ int capture_slot(fo_server* s, int slot, cudaGraphExec_t* out) {
   fo::tc_set_input(s->tc, slot);
   cudaGraph_t g = nullptr;
   FO_CUDA(cudaStreamBeginCapture(s->cs, cudaStreamCaptureModeRelaxed));
-  for (const Launch& l : s->plan) l.fn(s->cs);
+  bool forked = false;
+  for (const Launch& l : s->plan) {
+    if (l.join && forked) {
+      FO_CUDA(cudaEventRecord(s->join_ev, s->side));
+      FO_CUDA(cudaStreamWaitEvent(s->cs, s->join_ev, 0));
+      forked = false;
+    }
+    if (l.lane == 1 && s->use_side) {
+      // fork after everything the compute stream has issued so far
+      FO_CUDA(cudaEventRecord(s->fork_ev, s->cs));
+      FO_CUDA(cudaStreamWaitEvent(s->side, s->fork_ev, 0));
+      forked = true;
+      l.fn(s->side);
+    } else {
+      l.fn(s->cs);
+    }
+  }
+  if (forked) {
+    FO_CUDA(cudaEventRecord(s->join_ev, s->side));
+    FO_CUDA(cudaStreamWaitEvent(s->cs, s->join_ev, 0));
+  }
   FO_CUDA(cudaStreamEndCapture(s->cs, &g));
   cudaError_t e = cudaGraphInstantiate(out, g, 0);
   cudaGraphDestroy(g);
@@ -959,8 +988,12 @@ int fo_server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt, const
     return rc;
   }
   s->sched = new fo::TaskScheduler(c.num_devices, c.omega, c.depth, c.sched_policy);
+  s->use_side = getenv("FO_NO_SIDE") == nullptr;
   if (cudaStreamCreateWithFlags(&s->cs, cudaStreamNonBlocking) != cudaSuccess ||
-      cudaStreamCreateWithFlags(&s->xs, cudaStreamNonBlocking) != cudaSuccess) {
+      cudaStreamCreateWithFlags(&s->xs, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&s->side, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&s->fork_ev, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&s->join_ev, cudaEventDisableTiming) != cudaSuccess) {
     destroy_impl(s);
     return set_err(FO_ERR_CUDA, "stream creation");
   }

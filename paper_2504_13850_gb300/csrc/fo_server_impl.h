@@ -41,6 +41,8 @@ struct Launch {
   int kernels;     // kernel launches this entry makes
   double flops;    // algorithmic FLOPs
   double bytes;    // algorithmic HBM bytes
+  int lane = 0;    // 1: a weight gradient, which the step graph runs on the side stream
+  bool join = false;   // the step graph joins the side stream before this entry
 };
 
 struct ProfRec {
@@ -61,6 +63,13 @@ struct fo_server {
   std::vector<fo_op> ops;
   fo::TaskScheduler* sched = nullptr;
   cudaStream_t cs = nullptr, xs = nullptr;
+  // Side stream of the step graph: the weight gradients run on it, forked
+  // from the compute stream after their output gradient is ready and joined
+  // before the optimizer, so they fill the SMs the input-gradient chain
+  // leaves idle.  Events are capture-time fork / join points.
+  cudaStream_t side = nullptr;
+  cudaEvent_t fork_ev = nullptr, join_ev = nullptr;
+  bool use_side = true;
   int dt = fo::kF32;
 
   int64_t n_params = 0, n_padded = 0;

@@ -39,6 +39,10 @@ double tc_flops(const TcGemm* g);
 const char* tc_name(const TcGemm* g);
 // Allocates the split-K workspace after every plan is known.
 int tc_finalize(TcContext* c);
+// Stream lane of a plan's GEMM (0 compute stream, 1 side stream): GEMMs of
+// different lanes may run concurrently, so each lane has its own split-K
+// workspace.  Set before tc_finalize.
+void tc_set_lane(TcGemm* g, int lane);
 // Device word the tensor-core kernels set on a timed-out wait (0 = none).
 int* tc_error_word(TcContext* c);
 // Tensor map of a row-major bf16 matrix [rows][cols] with 128-byte-swizzled

@@ -850,6 +850,7 @@ struct TcGemm {
   KernelFn fn = nullptr;
   size_t smem = 0;
   dim3 grid;
+  int lane = 0;           // stream lane (split-K workspace per lane)
   bool input_A = false;   // operand fed by the uploaded batch (tensor 0)
   bool input_B = false;
   std::vector<CUtensorMap> slot_maps;  // per slot map of that operand
@@ -863,8 +864,7 @@ struct TcContext {
   int slot = 0;
   int* err = nullptr;
   fo_server* s = nullptr;
-  size_t ws_floats = 0;             // split-K workspace: the largest plan's need (plans run in order)
-  float* ws = nullptr;
+  float* ws[2] = {nullptr, nullptr};   // split-K workspace per stream lane (a lane's GEMMs run in order)
 };
 
 namespace {
@@ -1009,7 +1009,6 @@ TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
   const int n_tiles = (N + g->bn - 1) / g->bn;
   if (g->splits > 1) {
     g->grid = dim3(n_tiles, (M + BM - 1) / BM, g->splits);
-    c->ws_floats = std::max(c->ws_floats, size_t(g->grid.x) * g->grid.y * g->splits * BM * g->bn);
   } else if (g->pair) {
     const int work = n_tiles * ((M + BM - 1) / BM) / 2;
     g->grid = dim3(2 * std::min(work, active_clusters(c, g->kind, g->bn, 2, g->pair)), 1, 1);
@@ -1061,14 +1060,25 @@ bool tc_encode_2d(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, 
 
 int* tc_error_word(TcContext* c) { return c ? c->err : nullptr; }
 
-// Allocate the split-K workspace once every plan is known.  The GEMMs of a
-// step run one after another on one stream, so they share it.
+void tc_set_lane(TcGemm* g, int lane) {
+  if (g) g->lane = lane ? 1 : 0;
+}
+
+// Allocate the split-K workspaces once every plan is known: the GEMMs of one
+// stream lane run one after another, so they share that lane's workspace.
 int tc_finalize(TcContext* c) {
-  if (!c || c->ws_floats == 0) return FO_OK;
-  c->ws = static_cast<float*>(c->s->alloc(c->ws_floats * sizeof(float)));
-  if (!c->ws) return FO_ERR_OOM;
+  if (!c) return FO_OK;
+  size_t need[2] = {0, 0};
   for (TcGemm* g : c->gemms)
-    if (g->splits > 1) g->p.ws = c->ws;
+    if (g->splits > 1)
+      need[g->lane] = std::max(need[g->lane], size_t(g->grid.x) * g->grid.y * g->splits * BM * g->bn);
+  for (int l = 0; l < 2; ++l) {
+    if (!need[l]) continue;
+    c->ws[l] = static_cast<float*>(c->s->alloc(need[l] * sizeof(float)));
+    if (!c->ws[l]) return FO_ERR_OOM;
+  }
+  for (TcGemm* g : c->gemms)
+    if (g->splits > 1) g->p.ws = c->ws[g->lane];
   return FO_OK;
 }
 
