@@ -60,6 +60,9 @@ struct TcParams {
   // paired CTAs: the window operand is loaded as two halves, the second at
   // these row / image offsets (in the windowed tensor's coordinates)
   int half_dh, half_dn;
+  // MN-major operands whose 64-wide chunks one TMA box brings in at once
+  // (a chunk dimension of stride 128 bytes as the box's outermost dimension)
+  int chunk_a, chunk_b;
   // epilogue
   void* out;
   int ldo;
@@ -293,8 +296,11 @@ __device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, i
   if (KIND == LIN_FWD || KIND == LIN_DGRAD) {
     tma_2d(sa, &p.tmA, bar, kb * BK, m0);
   } else if (KIND == LIN_WGRAD || KIND == CONV_WGRAD) {
+    if (p.chunk_a)
+      tma_3d(sa, &p.tmA, bar, 0, kb * BK, m0 / 64);
+    else
 #pragma unroll
-    for (int j = 0; j < BM / 64; ++j) tma_2d(sa + j * BK * 128, &p.tmA, bar, m0 + j * 64, kb * BK);
+      for (int j = 0; j < BM / 64; ++j) tma_2d(sa + j * BK * 128, &p.tmA, bar, m0 + j * 64, kb * BK);
   } else if (KIND == CONV_FPROP) {  // windowed A over the (strided) input
     const int tap = kb / p.cblocks, c0 = (kb % p.cblocks) * 64;
     const int r = tap / p.ksz, s = tap % p.ksz;
@@ -319,13 +325,29 @@ __device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, i
     const int tap = kb / p.cblocks, c0 = (kb % p.cblocks) * 64;
     tma_2d(sb, &p.tmB, bar, tap * p.ntap_ch + c0, n0);
   } else if (KIND == LIN_DGRAD || KIND == LIN_WGRAD) {
+    if (p.chunk_b)
+      tma_3d(sb, &p.tmB, bar, 0, kb * BK, n0 / 64);
+    else
 #pragma unroll
-    for (int j = 0; j < BN / 64; ++j) tma_2d(sb + j * BK * 128, &p.tmB, bar, n0 + j * 64, kb * BK);
+      for (int j = 0; j < BN / 64; ++j) tma_2d(sb + j * BK * 128, &p.tmB, bar, n0 + j * 64, kb * BK);
   } else if (KIND == CONV_DGRAD) {
     const int t = kb / p.cblocks, co0 = (kb % p.cblocks) * 64;
     const int tap = p.tap_rs[t];
+    if (p.chunk_b)
+      tma_3d(sb, &p.tmB, bar, 0, co0, (tap * p.ntap_ch + n0) / 64);
+    else
 #pragma unroll
-    for (int j = 0; j < BN / 64; ++j) tma_2d(sb + j * BK * 128, &p.tmB, bar, tap * p.ntap_ch + n0 + j * 64, co0);
+      for (int j = 0; j < BN / 64; ++j) tma_2d(sb + j * BK * 128, &p.tmB, bar, tap * p.ntap_ch + n0 + j * 64, co0);
+  } else if (p.chunk_b) {  // CONV_WGRAD, all chunks of the tile (a pair: half each, multicast)
+    const int tap = n0 / p.ntap_ch, ci0 = n0 % p.ntap_ch;
+    const int r = tap / p.ksz, s = tap % p.ksz;
+    const int pix0 = kb * BK;
+    const int n_img = pix0 / HW, h0 = (pix0 % HW) / p.W;
+    if (PAIR == 2)
+      tma_5d_mc(sb + int(rank) * (BN / 128) * BK * 128, &p.tmB, bar, 0, s - p.pad, h0 * p.stride + r - p.pad, n_img,
+                ci0 / 64 + int(rank) * (BN / 128), 0x3);
+    else
+      tma_5d(sb, &p.tmB, bar, 0, s - p.pad, h0 * p.stride + r - p.pad, n_img, ci0 / 64);
   } else {  // CONV_WGRAD: N index = tap * Ci + ci; K = output pixel
     const int tap = n0 / p.ntap_ch, ci0 = n0 % p.ntap_ch;
     const int r = tap / p.ksz, s = tap % p.ksz;
@@ -826,6 +848,27 @@ bool map_2d(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int bo
 // 4-D NHWC window map over an N x H x W x C tensor that loads, per box,
 // 64 channels x ow columns x rows x imgs, stepping `stride` pixels in H and W
 // (the box spans ow*stride columns and rows*stride rows of the tensor).
+// [rows][cols] seen as {64, rows, cols / 64} (cols % 64 == 0): a box of
+// `chunks` 64-column chunks x box_rows rows lands chunk after chunk, each
+// box_rows x 128 bytes, the layout of an MN-major operand.
+bool map_chunked(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int box_rows, int chunks) {
+  if (cols % 64) return false;
+  uint64_t dims[3] = {64, uint64_t(rows), uint64_t(cols / 64)};
+  uint64_t strides[2] = {uint64_t(cols) * 2, 128};
+  uint32_t box[3] = {64, uint32_t(box_rows), uint32_t(chunks)};
+  return make_map(m, base, 3, dims, strides, box);
+}
+// The windowed NHWC tensor of map_window with its channels split the same
+// way: {64, W, H, N, C / 64}, `chunks` channel chunks per box (C % 64 == 0).
+bool map_window_chunked(CUtensorMap* m, const void* base, int N, int H, int W, int C, int ow, int rows, int imgs,
+                        int stride, int chunks) {
+  if (C % 64) return false;
+  uint64_t dims[5] = {64, uint64_t(W), uint64_t(H), uint64_t(N), uint64_t(C / 64)};
+  uint64_t strides[4] = {uint64_t(C) * 2, uint64_t(W) * C * 2, uint64_t(H) * W * C * 2, 128};
+  uint32_t box[5] = {64, uint32_t(ow * stride), uint32_t(rows * stride), uint32_t(imgs), uint32_t(chunks)};
+  uint32_t elem[5] = {1, uint32_t(stride), uint32_t(stride), 1, 1};
+  return make_map(m, base, 5, dims, strides, box, elem);
+}
 bool map_window(CUtensorMap* m, const void* base, int N, int H, int W, int C, int ow, int rows, int imgs,
                 int stride = 1) {
   uint64_t dims[4] = {uint64_t(C), uint64_t(W), uint64_t(H), uint64_t(N)};
@@ -1017,8 +1060,8 @@ TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
     g->grid = dim3(std::min(tiles, c->num_sms), 1, 1);
   }
   if (getenv("FO_DEBUG_PLAN"))
-    fprintf(stderr, "[plan] %-16s M=%d N=%d KB=%d BN=%d splits=%d pair=%d grid=(%u,%u,%u)\n", g->name, M, N,
-            g->p.KB, g->bn, g->splits, g->pair, g->grid.x, g->grid.y, g->grid.z);
+    fprintf(stderr, "[plan] %-16s M=%d N=%d KB=%d BN=%d splits=%d pair=%d grid=(%u,%u,%u) chunked=%d%d\n", g->name, M,
+            N, g->p.KB, g->bn, g->splits, g->pair, g->grid.x, g->grid.y, g->grid.z, g->p.chunk_a, g->p.chunk_b);
   g->ctx = c;
   c->gemms.push_back(g);
   return g;
@@ -1177,6 +1220,8 @@ bool tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate, void* dx, 
     int M = int(a.rows()), KB = (op.cout + 63) / 64;
     choose_tiles(c, g, M, op.cin, KB, op.cin, false);
     if (!map_2d(&g->p.tmA, o.grad, M, op.cout, BM) || !map_2d(&g->p.tmB, w, op.cout, op.cin, BK)) { delete g; return false; }
+    CUtensorMap cb;
+    if (map_chunked(&cb, w, op.cout, op.cin, BK, g->bn / 64)) { g->p.tmB = cb; g->p.chunk_b = 1; }
     if (!finish(c, g, M, op.cin, double(op.cout))) return false;
     out->push_back(g);
     return true;
@@ -1241,6 +1286,8 @@ bool tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate, void* dx, 
       out->clear();
       return false;
     }
+    CUtensorMap cb;
+    if (map_chunked(&cb, w, op.cout, int64_t(g->p.taps) * op.cin, BK, g->bn / 64)) { g->p.tmB = cb; g->p.chunk_b = 1; }
     if (!finish(c, g, M, op.cin, double(cls[q].n) * op.cout)) {
       out->clear();
       return false;
@@ -1268,11 +1315,24 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
     choose_tiles(c, g, op.cout, op.cin, KB, op.cin, false);
     g->input_B = (op.in0 == 0);
     if (!map_2d(&g->p.tmA, o.grad, rows, op.cout, BK)) { delete g; return nullptr; }
+    CUtensorMap ca;
+    if (map_chunked(&ca, o.grad, rows, op.cout, BK, BM / 64)) { g->p.tmA = ca; g->p.chunk_a = 1; }
+    const int nchunk = g->bn / 64;
+    g->p.chunk_b = op.cin % 64 == 0 ? 1 : 0;
+    auto map_b = [&](CUtensorMap* m, const void* base) {
+      if (g->p.chunk_b && map_chunked(m, base, rows, op.cin, BK, nchunk)) return true;
+      g->p.chunk_b = 0;
+      return map_2d(m, base, rows, op.cin, BK);
+    };
     if (g->input_B) {
       g->slot_maps.resize(s->cfg.omega);
-      for (int sl = 0; sl < s->cfg.omega; ++sl)
-        if (!map_2d(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, rows, op.cin, BK)) { delete g; return nullptr; }
-    } else if (!map_2d(&g->p.tmB, tensor_act(s, op.in0), rows, op.cin, BK)) { delete g; return nullptr; }
+      for (int pass = 0; pass < 2; ++pass) {   // a second pass if chunked maps fell back midway
+        const int chunked = g->p.chunk_b;
+        for (int sl = 0; sl < s->cfg.omega; ++sl)
+          if (!map_b(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride)) { delete g; return nullptr; }
+        if (chunked == g->p.chunk_b) break;
+      }
+    } else if (!map_b(&g->p.tmB, tensor_act(s, op.in0))) { delete g; return nullptr; }
     return finish(c, g, op.cout, op.cin, double(rows));
   }
   const int st = op.stride, Ho = o.H, Wo = o.W;
@@ -1289,11 +1349,24 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
   choose_tiles(c, g, op.cout, N, KB, op.cin, true);
   g->input_B = (op.in0 == 0);
   if (!map_2d(&g->p.tmA, o.grad, P, op.cout, BK)) { delete g; return nullptr; }
+  CUtensorMap ca;
+  if (map_chunked(&ca, o.grad, P, op.cout, BK, BM / 64)) { g->p.tmA = ca; g->p.chunk_a = 1; }
+  const int nchunk = g->pair == 2 ? g->bn / 128 : g->bn / 64;
+  g->p.chunk_b = 1;
+  auto map_b = [&](CUtensorMap* m, const void* base) {
+    if (g->p.chunk_b && map_window_chunked(m, base, a.N, a.H, a.W, a.C, Wo, rows, imgs, st, nchunk)) return true;
+    g->p.chunk_b = 0;
+    return map_window(m, base, a.N, a.H, a.W, a.C, Wo, rows, imgs, st);
+  };
   if (g->input_B) {
     g->slot_maps.resize(s->cfg.omega);
-    for (int sl = 0; sl < s->cfg.omega; ++sl)
-      if (!map_window(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride, a.N, a.H, a.W, a.C, Wo, rows, imgs, st)) { delete g; return nullptr; }
-  } else if (!map_window(&g->p.tmB, tensor_act(s, op.in0), a.N, a.H, a.W, a.C, Wo, rows, imgs, st)) { delete g; return nullptr; }
+    for (int pass = 0; pass < 2; ++pass) {   // a second pass if chunked maps fell back midway
+      const int chunked = g->p.chunk_b;
+      for (int sl = 0; sl < s->cfg.omega; ++sl)
+        if (!map_b(&g->slot_maps[sl], s->slab + size_t(sl) * s->slot_stride)) { delete g; return nullptr; }
+      if (chunked == g->p.chunk_b) break;
+    }
+  } else if (!map_b(&g->p.tmB, tensor_act(s, op.in0))) { delete g; return nullptr; }
   return finish(c, g, op.cout, N, double(P));
 }
 
