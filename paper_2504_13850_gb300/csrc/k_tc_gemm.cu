@@ -393,6 +393,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rbar + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   float* sbias = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES + 256);   // bias[n0 .. n0 + BN)
+  static_assert(STAGES * STAGE_BYTES + 1024 + 256 + 4 * BN <= 232448, "shared memory per CTA");
+  static_assert(2 * STAGES * 8 + 8 + 8 + 4 + 4 <= 256, "barrier area");
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM;
@@ -749,18 +751,26 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
   }
 }
 
-template <int KIND, int BN>
-constexpr int stages_for() {
-  return kSmemBudget / (BM * BK * 2 + BN * BK * 2) > 8 ? 8 : kSmemBudget / (BM * BK * 2 + BN * BK * 2);
-}
-inline size_t pipeline_bytes(int bn) {
+// Pipeline depth.  A stage's round trip (TMA load, MMAs, release) takes
+// ~1.5-2.5 us, so the main loop of a narrow tile runs at stages / round trip
+// and every stage that fits counts.  The persistent kernel keeps 32 KB of
+// epilogue staging; the split-K kernel takes all the rest of the 227 KB.
+constexpr int kSmemMax = 232448;
+constexpr int stages_of(int bn, bool cluster) {
   const int stage = BM * BK * 2 + bn * BK * 2;
-  const int stages = kSmemBudget / stage > 8 ? 8 : kSmemBudget / stage;
-  return size_t(stages) * stage;
+  const int budget = cluster ? kSmemMax - 1024 - 256 - 4 * bn : kSmemBudget;
+  return budget / stage > 8 ? 8 : budget / stage;
+}
+template <int KIND, int BN, bool CLUSTER>
+constexpr int stages_for() {
+  return stages_of(BN, CLUSTER);
+}
+inline size_t pipeline_bytes(int bn) {   // the split-K kernel's pipeline buffers
+  return size_t(stages_of(bn, true)) * (BM * BK * 2 + bn * BK * 2);
 }
 template <int KIND, int BN>
 constexpr size_t smem_bytes(bool cluster) {
-  return size_t(stages_for<KIND, BN>()) * (BM * BK * 2 + BN * BK * 2) + 1024 + 256 +
+  return size_t(stages_of(BN, cluster)) * (BM * BK * 2 + BN * BK * 2) + 1024 + 256 +
          (cluster ? 4 * BN : kEpiStageBytes);
 }
 
@@ -768,8 +778,8 @@ typedef void (*KernelFn)(const TcParams);
 
 template <int KIND, int BN>
 KernelFn kernel_ptr(bool cluster, int pair) {
-  constexpr int S = stages_for<KIND, BN>();
-  if (cluster) return pair ? nullptr : tc_gemm_kernel<KIND, BN, S>;
+  constexpr int S = stages_for<KIND, BN, false>();
+  if (cluster) return pair ? nullptr : tc_gemm_kernel<KIND, BN, stages_for<KIND, BN, true>()>;
   if constexpr ((KIND == CONV_FPROP || KIND == CONV_DGRAD) && BN >= 128) {
     if (pair == 1) return tc_gemm_persistent<KIND, BN, S, 1>;
   }
@@ -972,9 +982,11 @@ int active_clusters(TcContext* c, int kind, int bn, int S, int pair) {
 //    dependent latency is a few hundred cycles on each side;
 //  * the TMA fills one SM's shared memory at ~128 GB/s, which bounds stages
 //    of 256-wide tiles (48 KB);
-//  * weight-gradient windows arrive as 64-row 4-D boxes costing ~0.21 us
-//    each, so a 256-wide tile (four boxes) is slow unless a CTA pair splits
-//    them;
+//  * a stage issues four 128 x BN x 16 MMAs, and each takes ~190 cycles
+//    whatever BN <= 256 (measured: 128- and 256-wide weight-gradient stages
+//    both ~0.38-0.40 us once all chunks of an operand come in one TMA box),
+//    so 256-wide tiles run at ~3/4 of the MMA peak and 128-wide ones at
+//    ~3/8: the floor above;
 //  * a CTA pays a start-up ramp and the epilogue of its last tile (earlier
 //    epilogues overlap the next tile's MMAs), a K-split cluster pays the
 //    staging and distributed-shared-memory reduction of its partial tiles,
@@ -997,7 +1009,7 @@ void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv, bool 
       if (pair == 1 && !(pair_ok && win_a && bn >= 128 && n_tiles % 2 == 0)) continue;
       if (pair == 2 && !(pair_ok && win_b && bn >= 128 && m_tiles % 2 == 0)) continue;
       double t_kb = std::max(0.37, stage_kb / 128.0);
-      if (win_b) t_kb = std::max(t_kb + 0.05, 0.215 * (bn / 64) / (pair ? 2 : 1));
+      if (win_b) t_kb = std::max(t_kb, 0.39);
       if (!win_a && !win_b) t_kb = std::max(0.31, stage_kb / 128.0);
       for (int sp = 1; sp <= (pair ? 1 : 8); ++sp) {
         if (sp > 1 && KB / sp < 4) break;
