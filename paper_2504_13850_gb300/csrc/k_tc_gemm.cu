@@ -1010,7 +1010,6 @@ void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv, bool 
       if (pair == 2 && !(pair_ok && win_b && bn >= 128 && m_tiles % 2 == 0)) continue;
       double t_kb = std::max(0.37, stage_kb / 128.0);
       if (win_b) t_kb = std::max(t_kb, 0.39);
-      if (!win_a && !win_b) t_kb = std::max(0.31, stage_kb / 128.0);
       for (int sp = 1; sp <= (pair ? 1 : 8); ++sp) {
         if (sp > 1 && KB / sp < 4) break;
         // an owner's receive slices (16 KB per other rank and owned chunk) live in the pipeline buffers
