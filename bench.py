@@ -284,15 +284,26 @@ def run_ours(args):
         else:
             a, lb, ln = host["batches"][i % len(host["batches"])]
             rc, _ = srv.enqueue_activations(u, a, lb, ln)
-            with torch.cuda.stream(stream):
-                host["stage"].copy_(host["models"][i % 2], non_blocking=True)
-            local = host["stage"]
+            # the device model comes up on a copy stream into one of two
+            # staging buffers, after the aggregation that last read it
+            b = i % 2
+            cs = host["copy"]
+            cs.wait_event(host["read"][b])
+            with torch.cuda.stream(cs):
+                host["stage"][b].copy_(host["models"][b], non_blocking=True)
+                host["landed"][b].record(cs)
+            stream.wait_event(host["landed"][b])
+            local = host["stage"][b]
         assert rc == api.OK, rc
         t, _ = srv.version()
         rc, _ = srv.aggregate(g_model, local, u, max(0, t - 3))
         assert rc == api.OK, rc
         if host is not None:
-            srv.read_losses(done[0] - 1, 1)            # the step's result back on the host
+            host["read"][i % 2].record(stream)
+            # every step's loss comes back to the host; step i's is read while
+            # step i + 1 runs (fo_read_losses waits for that step only)
+            if done[0] >= 2:
+                host["loss"] = srv.read_losses(done[0] - 2, 1)
 
     # ---------------- device-resident timed region
     for _ in range(args.warmup):
@@ -334,7 +345,9 @@ def run_ours(args):
     # ---------------- end to end through the C ABI from pinned host memory
     e2e = None
     if not args.no_e2e:
-        host = {"batches": [], "models": [], "stage": torch.empty(n_model, device=dev)}
+        host = {"batches": [], "models": [], "stage": [torch.empty(n_model, device=dev) for _ in range(2)],
+                "copy": torch.cuda.Stream(device=dev), "landed": [torch.cuda.Event() for _ in range(2)],
+                "read": [torch.cuda.Event() for _ in range(2)]}
         for a, lb, ln in pool[:4]:
             host["batches"].append((a.cpu().pin_memory(), lb.cpu().pin_memory(),
                                     None if ln is None else ln.cpu().pin_memory()))
@@ -350,6 +363,7 @@ def run_ours(args):
         ev0.record(stream)
         for _ in range(n_e2e):
             step(host)
+        host["loss"] = srv.read_losses(done[0] - 1, 1)   # the last step's loss, inside the timed region
         ev1.record(stream)
         torch.cuda.synchronize()
         barrier(world)
@@ -364,19 +378,26 @@ def run_ours(args):
         try:
             ga = torch.randn(n, device=dev) * 0.05
             la = torch.randn(n, device=dev) * 0.05
-            for _ in range(3):
-                api.axpby_async(ga, la, 0.25, srv.stream())
-            best = 1e30
-            for _ in range(10):
-                ev0.record(stream)
-                api.axpby_async(ga, la, 0.25, srv.stream())
-                ev1.record(stream)
-                torch.cuda.synchronize()
-                best = min(best, ev0.elapsed_time(ev1))
-            gbs = 12.0 * n / (best / 1e3) / 1e9
             pk, which = peaks()
-            agg = {"params": n, "gbs": round(gbs, 1), "frac": round(gbs / pk["hbm_gbs"], 4),
-                   "peak_gbs": pk["hbm_gbs"], "peak": which, "bytes_per_param": 12}
+            sweep = []
+            for m in (1_000_000, 4_000_000, 16_000_000, 64_000_000, n):
+                g_m, l_m = ga[:m], la[:m]
+                for _ in range(3):
+                    api.axpby_async(g_m, l_m, 0.25, srv.stream())
+                best = 1e30
+                for _ in range(10):
+                    ev0.record(stream)
+                    api.axpby_async(g_m, l_m, 0.25, srv.stream())
+                    ev1.record(stream)
+                    torch.cuda.synchronize()
+                    best = min(best, ev0.elapsed_time(ev1))
+                # 12 bytes per parameter; below ~126 MB of traffic the vectors stay in L2
+                sweep.append({"params": m, "gbs": round(12.0 * m / (best / 1e3) / 1e9, 1),
+                              "l2_resident": 12 * m < 126 * 2**20})
+            gbs = sweep[-1]["gbs"]
+            agg = {"params": n, "gbs": gbs, "frac": round(gbs / pk["hbm_gbs"], 4),
+                   "peak_gbs": pk["hbm_gbs"], "peak": which, "bytes_per_param": 12,
+                   "sweep": sweep, "best_of": 10}
             del ga, la
             torch.cuda.empty_cache()
         except torch.cuda.OutOfMemoryError:
@@ -403,6 +424,7 @@ def run_ours(args):
     step_flops = sum(v[2] for v in ktimes.values()) / n_prof
     step_ms = ms_dev / args.steps
     tensor_frac = step_flops / (step_ms / 1e3) / 1e12 / pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
+    tensor_frac_burst = step_flops / (step_ms / 1e3) / 1e12 / pk["bf16_tflops"]
     cpu = None
     if not args.no_cpu_baseline:
         v_cpu, dt_cpu = oracle_samples_per_s(cfg, 2, B)
@@ -433,6 +455,7 @@ def run_ours(args):
         "gpu_launches": int(launches),
         "roofline": roof,
         "step_tensor_frac": round(tensor_frac, 4),
+        "step_tensor_frac_burst": round(tensor_frac_burst, 4),
         "step_gflop": round(step_flops / 1e9, 2),
         "aggregation": agg,
         "scheduler_balance": sched,

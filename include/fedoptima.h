@@ -166,8 +166,12 @@ FO_API int fo_server_store_params_device(fo_server* s, float* dst, int64_t n);
  * server-side flow control of Sec. 3.4.1.  `acts` (host or device) holds
  * B*H*W*C elements of the configured dtype, NHWC; `labels` (host or device)
  * int32[B]; `lengths` (host or device) int32[B] when cfg.seq, else NULL.
- * The batch is copied into a free slot before the call returns, so the
- * caller may reuse its buffers.  *sender_on (may be NULL) receives the
+ * The caller's buffers are copied to the device before the call returns,
+ * so it may reuse them: straight into the slot when the slot is idle, else
+ * into one of three device staging buffers that move into the slot once
+ * the queued step still reading it has finished (the call does not wait for
+ * that step).  The server holds omega slots plus these three staging
+ * buffers, whatever the number of devices.  *sender_on (may be NULL) receives the
  * device's Sender Status after the call: 1 = "turn-on" was sent.
  * FO_FULL: the cap omega or the ring depth is reached; the device is turned
  * off and, if its queue is empty, waits in a FIFO of blocked devices.
@@ -186,7 +190,9 @@ FO_API int fo_enqueue_activations(fo_server* s, int device_id, const void* acts,
 FO_API int fo_server_step(fo_server* s, int* device_used, int32_t* slot_used);
 
 /* Copy the losses of steps [first_step, first_step + n) to host memory.
- * Waits for those steps.  Only the most recent 2^20 steps are kept. */
+ * Waits for those steps only (work enqueued after them keeps running), so a
+ * caller can read step i's loss while step i + 1 executes.  Only the most
+ * recent 2^20 steps are kept. */
 FO_API int fo_read_losses(fo_server* s, float* host_out, int64_t first_step, int64_t n);
 
 /* FedAsync aggregation (Algorithm 4, aggregation branch).  `global`

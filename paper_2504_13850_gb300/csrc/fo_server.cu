@@ -813,6 +813,17 @@ int allocate(fo_server* s) {
     FO_CUDA(cudaEventCreateWithFlags(&s->slot_ready[i], cudaEventDisableTiming));
     FO_CUDA(cudaEventCreateWithFlags(&s->slot_free[i], cudaEventDisableTiming));
   }
+  s->stage_stride = (s->slot_stride + 2 * int64_t(c.batch) * 4 + 255) / 256 * 256;
+  s->stage_buf = (char*)s->alloc(size_t(s->stage_stride) * fo_server::kStage);
+  if (!s->stage_buf) return set_err(FO_ERR_OOM, "upload staging");
+  s->stage_landed.assign(fo_server::kStage, nullptr);
+  s->stage_free.assign(fo_server::kStage, nullptr);
+  for (int r = 0; r < fo_server::kStage; ++r) {
+    FO_CUDA(cudaEventCreateWithFlags(&s->stage_landed[r], cudaEventDisableTiming));
+    FO_CUDA(cudaEventCreateWithFlags(&s->stage_free[r], cudaEventDisableTiming));
+  }
+  s->step_done.assign(fo_server::kStepEvents, nullptr);
+  for (cudaEvent_t& e : s->step_done) FO_CUDA(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
   // tensors
   int nops = int(s->ops.size());
   for (int tid = 1; tid <= nops; ++tid) {
@@ -876,6 +887,7 @@ void destroy_impl(fo_server* s) {
   for (fo::AttnTcPlan* a : s->attn_tc) fo::attention_tc_destroy(a);
   s->attn_tc.clear();
   if (s->xs) cudaStreamSynchronize(s->xs);
+  if (s->hs) cudaStreamSynchronize(s->hs);
   for (auto g : s->graphs) if (g) cudaGraphExecDestroy(g);
   for (auto g : s->prof_graphs) if (g) cudaGraphExecDestroy(g);
   for (auto& v : s->prof_events)
@@ -886,6 +898,7 @@ void destroy_impl(fo_server* s) {
   fo::tc_destroy(s->tc);
   for (auto e : s->slot_ready) if (e) cudaEventDestroy(e);
   for (auto e : s->slot_free) if (e) cudaEventDestroy(e);
+  for (auto e : s->step_done) if (e) cudaEventDestroy(e);
   for (auto& r : s->prof) {
     cudaEventDestroy(r.a);
     cudaEventDestroy(r.b);
@@ -895,6 +908,9 @@ void destroy_impl(fo_server* s) {
   if (s->side) cudaStreamSynchronize(s->side);
   if (s->cs) cudaStreamDestroy(s->cs);
   if (s->xs) cudaStreamDestroy(s->xs);
+  if (s->hs) cudaStreamDestroy(s->hs);
+  for (auto e : s->stage_landed) if (e) cudaEventDestroy(e);
+  for (auto e : s->stage_free) if (e) cudaEventDestroy(e);
   if (s->side) cudaStreamDestroy(s->side);
   if (s->fork_ev) cudaEventDestroy(s->fork_ev);
   if (s->join_ev) cudaEventDestroy(s->join_ev);
@@ -991,6 +1007,7 @@ int fo_server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt, const
   s->use_side = getenv("FO_NO_SIDE") == nullptr;
   if (cudaStreamCreateWithFlags(&s->cs, cudaStreamNonBlocking) != cudaSuccess ||
       cudaStreamCreateWithFlags(&s->xs, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&s->hs, cudaStreamNonBlocking) != cudaSuccess ||
       cudaStreamCreateWithFlags(&s->side, cudaStreamNonBlocking) != cudaSuccess ||
       cudaEventCreateWithFlags(&s->fork_ev, cudaEventDisableTiming) != cudaSuccess ||
       cudaEventCreateWithFlags(&s->join_ev, cudaEventDisableTiming) != cudaSuccess) {
@@ -1094,15 +1111,42 @@ int fo_enqueue_activations(fo_server* s, int device_id, const void* acts, const 
   if (rc == -1) return set_err(FO_ERR_ARG, "device has left");
   if (rc == 2) return FO_FULL;
   const int B = s->cfg.batch;
-  if (s->slot_consumed[slot]) FO_CUDA(cudaStreamWaitEvent(s->xs, s->slot_free[slot], 0));
-  FO_CUDA(cudaMemcpyAsync(s->slab + size_t(slot) * s->slot_stride, acts, s->slot_act_bytes,
-                          cudaMemcpyDefault, s->xs));
-  FO_CUDA(cudaMemcpyAsync(s->slot_labels + size_t(slot) * B, labels, B * 4, cudaMemcpyDefault, s->xs));
-  if (lengths)
-    FO_CUDA(cudaMemcpyAsync(s->slot_lengths + size_t(slot) * B, lengths, B * 4, cudaMemcpyDefault, s->xs));
+  char* d_act = s->slab + size_t(slot) * s->slot_stride;
+  int32_t* d_lab = s->slot_labels + size_t(slot) * B;
+  int32_t* d_len = s->slot_lengths + size_t(slot) * B;
+  bool busy = false;   // a queued step still reads this slot
+  if (s->slot_consumed[slot]) {
+    const cudaError_t q = cudaEventQuery(s->slot_free[slot]);
+    if (q == cudaErrorNotReady) busy = true;
+    else FO_CUDA(q);
+  }
+  if (!busy) {
+    FO_CUDA(cudaMemcpyAsync(d_act, acts, s->slot_act_bytes, cudaMemcpyDefault, s->hs));
+    FO_CUDA(cudaMemcpyAsync(d_lab, labels, B * 4, cudaMemcpyDefault, s->hs));
+    if (lengths) FO_CUDA(cudaMemcpyAsync(d_len, lengths, B * 4, cudaMemcpyDefault, s->hs));
+    FO_CUDA(cudaEventRecord(s->slot_ready[slot], s->hs));
+    // The caller may reuse its buffers once the call returns.
+    FO_CUDA(cudaEventSynchronize(s->slot_ready[slot]));
+    return FO_OK;
+  }
+  const int r = int(s->stage_next++ % fo_server::kStage);
+  char* st = s->stage_buf + size_t(r) * s->stage_stride;
+  int32_t* st_lab = reinterpret_cast<int32_t*>(st + s->slot_stride);
+  int32_t* st_len = st_lab + B;
+  FO_CUDA(cudaStreamWaitEvent(s->hs, s->stage_free[r], 0));   // the move that last read this buffer
+  FO_CUDA(cudaMemcpyAsync(st, acts, s->slot_act_bytes, cudaMemcpyDefault, s->hs));
+  FO_CUDA(cudaMemcpyAsync(st_lab, labels, B * 4, cudaMemcpyDefault, s->hs));
+  if (lengths) FO_CUDA(cudaMemcpyAsync(st_len, lengths, B * 4, cudaMemcpyDefault, s->hs));
+  FO_CUDA(cudaEventRecord(s->stage_landed[r], s->hs));
+  FO_CUDA(cudaStreamWaitEvent(s->xs, s->stage_landed[r], 0));
+  FO_CUDA(cudaStreamWaitEvent(s->xs, s->slot_free[slot], 0));
+  FO_CUDA(cudaMemcpyAsync(d_act, st, s->slot_act_bytes, cudaMemcpyDeviceToDevice, s->xs));
+  FO_CUDA(cudaMemcpyAsync(d_lab, st_lab, B * 4, cudaMemcpyDeviceToDevice, s->xs));
+  if (lengths) FO_CUDA(cudaMemcpyAsync(d_len, st_len, B * 4, cudaMemcpyDeviceToDevice, s->xs));
+  FO_CUDA(cudaEventRecord(s->stage_free[r], s->xs));
   FO_CUDA(cudaEventRecord(s->slot_ready[slot], s->xs));
-  // The caller may reuse its buffers once the call returns.
-  FO_CUDA(cudaEventSynchronize(s->slot_ready[slot]));
+  // The caller may reuse its buffers once its own copy is done.
+  FO_CUDA(cudaEventSynchronize(s->stage_landed[r]));
   return FO_OK;
 }
 
@@ -1186,6 +1230,7 @@ int fo_server_step(fo_server* s, int* device_used, int32_t* slot_used) {
   s->kernels_launched += n;
   FO_CUDA(cudaGetLastError());
   FO_CUDA(cudaEventRecord(s->slot_free[slot], s->cs));
+  FO_CUDA(cudaEventRecord(s->step_done[s->steps_done % fo_server::kStepEvents], s->cs));
   s->slot_consumed[slot] = 1;
   s->steps_done++;
   s->last_launches = n;
@@ -1196,7 +1241,10 @@ int fo_read_losses(fo_server* s, float* host_out, int64_t first_step, int64_t n)
   if (!s || !host_out || first_step < 0 || n < 0 || first_step + n > s->steps_done ||
       s->steps_done - first_step > s->kLossRing)
     return set_err(FO_ERR_ARG, "loss range");
-  FO_CUDA(cudaStreamSynchronize(s->cs));
+  if (n == 0) return FO_OK;
+  // The event slot of the last step read holds that step or a later one:
+  // either way the losses asked for are written once it has completed.
+  FO_CUDA(cudaEventSynchronize(s->step_done[(first_step + n - 1) % fo_server::kStepEvents]));
   for (int64_t i = 0; i < n; ++i) {
     int64_t idx = (first_step + i) & (s->kLossRing - 1);
     FO_CUDA(cudaMemcpy(host_out + i, s->losses + idx, 4, cudaMemcpyDeviceToHost));
@@ -1259,6 +1307,7 @@ int64_t fo_server_activation_bytes(const fo_server* s) {
 }
 int fo_server_synchronize(fo_server* s) {
   if (!s) return set_err(FO_ERR_ARG, "null server");
+  FO_CUDA(cudaStreamSynchronize(s->hs));
   FO_CUDA(cudaStreamSynchronize(s->xs));
   FO_CUDA(cudaStreamSynchronize(s->cs));
   return FO_OK;

@@ -63,6 +63,17 @@ struct fo_server {
   std::vector<fo_op> ops;
   fo::TaskScheduler* sched = nullptr;
   cudaStream_t cs = nullptr, xs = nullptr;
+  // Uploads: the host-to-device copy of the caller's buffers runs on `hs`
+  // and never waits for compute.  An upload whose slot a queued step still
+  // reads lands in a device staging buffer first and moves into the slot on
+  // `xs` once that step has finished, so the caller returns as soon as its
+  // own copy is done instead of waiting for the step.
+  cudaStream_t hs = nullptr;
+  static constexpr int kStage = 3;
+  char* stage_buf = nullptr;
+  int64_t stage_stride = 0;
+  std::vector<cudaEvent_t> stage_landed, stage_free;
+  int64_t stage_next = 0;
   // Side stream of the step graph: the weight gradients run on it, forked
   // from the compute stream after their output gradient is ready and joined
   // before the optimizer, so they fill the SMs the input-gradient chain
@@ -101,6 +112,10 @@ struct fo_server {
   std::vector<std::vector<struct ProfRec>> prof_events;
   int64_t steps_done = 0;
   static constexpr int64_t kLossRing = int64_t(1) << 20;
+  // Completion events of the most recent steps (step i records slot i % 64),
+  // so that reading a step's loss waits for that step only.
+  static constexpr int kStepEvents = 64;
+  std::vector<cudaEvent_t> step_done;
 
   std::vector<Launch> plan;
   int last_launches = 0;
