@@ -98,9 +98,10 @@ void softmax_ce(const float* logits, const int32_t* labels, int B, int C, float*
 
 // SGD with momentum over a flat vector (n a multiple of 4, 16-byte aligned):
 // v = mu v + g; theta -= lr v; shadow (bf16, may be null) = bf16(theta).
-// The step counter (may be null) is incremented once, after the update.
+// The step counter (may be null) is incremented once.  skip64 (device, may
+// be null): one flag per 64 elements; flagged blocks are not touched.
 void sgd_momentum(float* theta, float* v, const float* g, void* shadow, int64_t n, float lr,
-                  float mu, int64_t* step, cudaStream_t st);
+                  float mu, int64_t* step, cudaStream_t st, const uint8_t* skip64 = nullptr);
 void f32_to_bf16(const float* x, void* y, int64_t n, cudaStream_t st);
 
 // ---- vectorised bf16 kernels (k_vec.cu): 8 elements per 16-byte access ----

@@ -454,6 +454,11 @@ int build_plan(fo_server* s) {
   std::vector<fo::ColsumTask> bias_tasks;
   std::vector<fo::FinishTask> finish_tasks;
   double deferred_bytes = 0.0;
+  // Weight tensors whose optimizer update runs on the side stream as soon as
+  // their gradient is complete and no kernel of the step reads them any more
+  // (their layer's input gradient has run): the update's HBM traffic then
+  // overlaps the rest of the backward pass.  Flags per 64 parameters.
+  std::vector<uint8_t> early(size_t(s->n_padded / 64), 0);
   for (int i = nops - 1; i >= 0; --i) {
     const fo_op op = s->ops[i];
     if (fu.skip_bwd[i]) {
@@ -555,6 +560,17 @@ int build_plan(fo_server* s) {
                                   accf != 0, mask, st);
             });
           }
+        }
+        {
+          // the weights' update, forked after the input gradient that read them
+          const ParamSeg seg = s->segs[s->op_segs[i][0]];
+          const int64_t len = pad64(seg.n);
+          add("sgd_momentum", 1, 0.0, double(len) * (20.0 + (s->shadow ? 2.0 : 0.0)), [=](cudaStream_t st) {
+            fo::sgd_momentum(s->theta + seg.off, s->mom + seg.off, s->grad + seg.off,
+                             s->shadow ? (void*)(s->shadow + seg.off) : nullptr, len, s->opt.lr, s->opt.momentum,
+                             nullptr, st);
+          }, 2);
+          for (int64_t b = seg.off / 64; b < (seg.off + len) / 64; ++b) early[size_t(b)] = 1;
         }
         break;
       }
@@ -774,8 +790,17 @@ int build_plan(fo_server* s) {
       fo::finish_batched(finish_tasks, st);
     });
   }
-  add("sgd_momentum", 1, 0.0, double(s->n_padded) * (20.0 + (s->shadow ? 2.0 : 0.0)), [=](cudaStream_t st) {
-    fo::sgd_momentum(s->theta, s->mom, s->grad, s->shadow, s->n_padded, s->opt.lr, s->opt.momentum, s->d_step, st);
+  int64_t late = 0;   // parameters the final update still covers
+  for (uint8_t e : early) late += e ? 0 : 64;
+  uint8_t* skip = nullptr;
+  if (late < s->n_padded) {
+    skip = (uint8_t*)s->alloc(early.size());
+    if (!skip) return set_err(FO_ERR_OOM, "optimizer flags");
+    FO_CUDA(cudaMemcpy(skip, early.data(), early.size(), cudaMemcpyHostToDevice));
+  }
+  add("sgd_momentum", 1, 0.0, double(late) * (20.0 + (s->shadow ? 2.0 : 0.0)), [=](cudaStream_t st) {
+    fo::sgd_momentum(s->theta, s->mom, s->grad, s->shadow, s->n_padded, s->opt.lr, s->opt.momentum, s->d_step, st,
+                     skip);
   });
   plan[first_opt].join = true;
   for (int i = 0; i < nops; ++i)
@@ -906,12 +931,16 @@ void destroy_impl(fo_server* s) {
   for (auto e : s->ev_pool) cudaEventDestroy(e);
   for (void* p : s->allocs) cudaFree(p);
   if (s->side) cudaStreamSynchronize(s->side);
+  if (s->opt_st) cudaStreamSynchronize(s->opt_st);
   if (s->cs) cudaStreamDestroy(s->cs);
   if (s->xs) cudaStreamDestroy(s->xs);
   if (s->hs) cudaStreamDestroy(s->hs);
   for (auto e : s->stage_landed) if (e) cudaEventDestroy(e);
   for (auto e : s->stage_free) if (e) cudaEventDestroy(e);
   if (s->side) cudaStreamDestroy(s->side);
+  if (s->opt_st) cudaStreamDestroy(s->opt_st);
+  if (s->fork2_ev) cudaEventDestroy(s->fork2_ev);
+  if (s->join2_ev) cudaEventDestroy(s->join2_ev);
   if (s->fork_ev) cudaEventDestroy(s->fork_ev);
   if (s->join_ev) cudaEventDestroy(s->join_ev);
   delete s->sched;
@@ -934,12 +963,29 @@ int capture_slot(fo_server* s, int slot, cudaGraphExec_t* out) {
   fo::tc_set_input(s->tc, slot);
   cudaGraph_t g = nullptr;
   FO_CUDA(cudaStreamBeginCapture(s->cs, cudaStreamCaptureModeRelaxed));
-  bool forked = false;
+  bool forked = false, forked2 = false;
   for (const Launch& l : s->plan) {
     if (l.join && forked) {
       FO_CUDA(cudaEventRecord(s->join_ev, s->side));
       FO_CUDA(cudaStreamWaitEvent(s->cs, s->join_ev, 0));
       forked = false;
+    }
+    if (l.join && forked2) {
+      FO_CUDA(cudaEventRecord(s->join2_ev, s->opt_st));
+      FO_CUDA(cudaStreamWaitEvent(s->cs, s->join2_ev, 0));
+      forked2 = false;
+    }
+    if (l.lane == 2 && s->use_side) {
+      // after the compute stream's work so far and the side stream's
+      FO_CUDA(cudaEventRecord(s->fork_ev, s->cs));
+      FO_CUDA(cudaStreamWaitEvent(s->opt_st, s->fork_ev, 0));
+      if (forked) {
+        FO_CUDA(cudaEventRecord(s->fork2_ev, s->side));
+        FO_CUDA(cudaStreamWaitEvent(s->opt_st, s->fork2_ev, 0));
+      }
+      forked2 = true;
+      l.fn(s->opt_st);
+      continue;
     }
     if (l.lane == 1 && s->use_side) {
       // fork after everything the compute stream has issued so far
@@ -954,6 +1000,10 @@ int capture_slot(fo_server* s, int slot, cudaGraphExec_t* out) {
   if (forked) {
     FO_CUDA(cudaEventRecord(s->join_ev, s->side));
     FO_CUDA(cudaStreamWaitEvent(s->cs, s->join_ev, 0));
+  }
+  if (forked2) {
+    FO_CUDA(cudaEventRecord(s->join2_ev, s->opt_st));
+    FO_CUDA(cudaStreamWaitEvent(s->cs, s->join2_ev, 0));
   }
   FO_CUDA(cudaStreamEndCapture(s->cs, &g));
   cudaError_t e = cudaGraphInstantiate(out, g, 0);
@@ -1009,6 +1059,9 @@ int fo_server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt, const
       cudaStreamCreateWithFlags(&s->xs, cudaStreamNonBlocking) != cudaSuccess ||
       cudaStreamCreateWithFlags(&s->hs, cudaStreamNonBlocking) != cudaSuccess ||
       cudaStreamCreateWithFlags(&s->side, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&s->opt_st, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&s->fork2_ev, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&s->join2_ev, cudaEventDisableTiming) != cudaSuccess ||
       cudaEventCreateWithFlags(&s->fork_ev, cudaEventDisableTiming) != cudaSuccess ||
       cudaEventCreateWithFlags(&s->join_ev, cudaEventDisableTiming) != cudaSuccess) {
     destroy_impl(s);

@@ -41,7 +41,8 @@ struct Launch {
   int kernels;     // kernel launches this entry makes
   double flops;    // algorithmic FLOPs
   double bytes;    // algorithmic HBM bytes
-  int lane = 0;    // 1: a weight gradient, which the step graph runs on the side stream
+  int lane = 0;    // 1: a weight gradient, which the step graph runs on the side stream;
+                   // 2: an early weight update, on the optimizer stream
   bool join = false;   // the step graph joins the side stream before this entry
 };
 
@@ -80,6 +81,11 @@ struct fo_server {
   // leaves idle.  Events are capture-time fork / join points.
   cudaStream_t side = nullptr;
   cudaEvent_t fork_ev = nullptr, join_ev = nullptr;
+  // Optimizer stream: the update of a weight tensor, forked once both its
+  // gradient (side stream) and its layer's input gradient (compute stream)
+  // are done, so the HBM-bound update overlaps the GEMMs that follow.
+  cudaStream_t opt_st = nullptr;
+  cudaEvent_t fork2_ev = nullptr, join2_ev = nullptr;
   bool use_side = true;
   int dt = fo::kF32;
 

@@ -594,14 +594,16 @@ void softmax_ce(const float* logits, const int32_t* labels, int B, int C, float*
 }
 
 // ------------------------------------------------------ SGD with momentum
-// 16-byte vector loads/stores; n is a multiple of 4.
+// 16-byte vector loads/stores; n is a multiple of 4.  skip64 (may be null)
+// marks 64-element blocks updated earlier in the step, which are left alone.
 __global__ void sgd_momentum_k(float4* __restrict__ theta, float4* __restrict__ v,
                                const float4* __restrict__ g, uint2* __restrict__ shadow,
-                               int64_t n4, float lr, float mu, int64_t* step) {
+                               int64_t n4, float lr, float mu, int64_t* step, const uint8_t* __restrict__ skip64) {
   pdl_wait();
   pdl_trigger();
   if (step && blockIdx.x == 0 && threadIdx.x == 0) *step += 1;
   GRID_STRIDE(i, n4) {
+    if (skip64 && skip64[i / 16]) continue;
     float4 t = theta[i], m = v[i];
     const float4 gr = g[i];
     m.x = fmaf(mu, m.x, gr.x);
@@ -624,10 +626,10 @@ __global__ void sgd_momentum_k(float4* __restrict__ theta, float4* __restrict__ 
   }
 }
 void sgd_momentum(float* theta, float* v, const float* g, void* shadow, int64_t n, float lr,
-                  float mu, int64_t* step, cudaStream_t st) {
+                  float mu, int64_t* step, cudaStream_t st, const uint8_t* skip64) {
   int64_t n4 = n / 4;
-  launch_k(sgd_momentum_k, elementwise_blocks(n4, 256), 256, 0, st, 
-      (float4*)theta, (float4*)v, (const float4*)g, (uint2*)shadow, n4, lr, mu, step);
+  launch_k(sgd_momentum_k, elementwise_blocks(n4, 256), 256, 0, st,
+      (float4*)theta, (float4*)v, (const float4*)g, (uint2*)shadow, n4, lr, mu, step, skip64);
 }
 __global__ void f32_to_bf16_k(const float* x, bf16* y, int64_t n) {
   pdl_wait();
