@@ -102,6 +102,10 @@ void softmax_ce(const float* logits, const int32_t* labels, int B, int C, float*
 // be null): one flag per 64 elements; flagged blocks are not touched.
 void sgd_momentum(float* theta, float* v, const float* g, void* shadow, int64_t n, float lr,
                   float mu, int64_t* step, cudaStream_t st, const uint8_t* skip64 = nullptr);
+// The update restricted to the 64-element blocks listed in blocks64 (device,
+// nb entries: block b covers elements 64b .. 64b + 63).
+void sgd_momentum_blocks(float* theta, float* v, const float* g, void* shadow, const int64_t* blocks64, int64_t nb,
+                         float lr, float mu, int64_t* step, cudaStream_t st);
 void f32_to_bf16(const float* x, void* y, int64_t n, cudaStream_t st);
 
 // ---- vectorised bf16 kernels (k_vec.cu): 8 elements per 16-byte access ----

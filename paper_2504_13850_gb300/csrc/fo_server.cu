@@ -790,18 +790,35 @@ int build_plan(fo_server* s) {
       fo::finish_batched(finish_tasks, st);
     });
   }
-  int64_t late = 0;   // parameters the final update still covers
-  for (uint8_t e : early) late += e ? 0 : 64;
-  uint8_t* skip = nullptr;
-  if (late < s->n_padded) {
-    skip = (uint8_t*)s->alloc(early.size());
+  // the final update covers the parameters not updated early: the whole
+  // vector, a list of 64-element blocks when that list is short, or the
+  // whole vector minus flagged blocks
+  std::vector<int64_t> late;
+  for (size_t b = 0; b < early.size(); ++b)
+    if (!early[b]) late.push_back(int64_t(b));
+  const double late_bytes = double(late.size()) * 64.0 * (20.0 + (s->shadow ? 2.0 : 0.0));
+  if (late.size() == early.size()) {
+    add("sgd_momentum", 1, 0.0, late_bytes, [=](cudaStream_t st) {
+      fo::sgd_momentum(s->theta, s->mom, s->grad, s->shadow, s->n_padded, s->opt.lr, s->opt.momentum, s->d_step, st);
+    });
+  } else if (late.size() * 8 < early.size()) {
+    int64_t* blk = (int64_t*)s->alloc(std::max<size_t>(late.size(), 1) * sizeof(int64_t));
+    if (!blk) return set_err(FO_ERR_OOM, "optimizer block list");
+    if (!late.empty()) FO_CUDA(cudaMemcpy(blk, late.data(), late.size() * sizeof(int64_t), cudaMemcpyHostToDevice));
+    const int64_t nb = int64_t(late.size());
+    add("sgd_momentum", 1, 0.0, late_bytes, [=](cudaStream_t st) {
+      fo::sgd_momentum_blocks(s->theta, s->mom, s->grad, s->shadow, blk, nb, s->opt.lr, s->opt.momentum, s->d_step,
+                              st);
+    });
+  } else {
+    uint8_t* skip = (uint8_t*)s->alloc(early.size());
     if (!skip) return set_err(FO_ERR_OOM, "optimizer flags");
     FO_CUDA(cudaMemcpy(skip, early.data(), early.size(), cudaMemcpyHostToDevice));
+    add("sgd_momentum", 1, 0.0, late_bytes, [=](cudaStream_t st) {
+      fo::sgd_momentum(s->theta, s->mom, s->grad, s->shadow, s->n_padded, s->opt.lr, s->opt.momentum, s->d_step,
+                       st, skip);
+    });
   }
-  add("sgd_momentum", 1, 0.0, double(late) * (20.0 + (s->shadow ? 2.0 : 0.0)), [=](cudaStream_t st) {
-    fo::sgd_momentum(s->theta, s->mom, s->grad, s->shadow, s->n_padded, s->opt.lr, s->opt.momentum, s->d_step, st,
-                     skip);
-  });
   plan[first_opt].join = true;
   for (int i = 0; i < nops; ++i)
     if (s->ops[i].kind == FO_OP_ATTENTION) fo::attention_prepare(s->T[s->ops[i].in0].H, s->ops[i].cin, s->ops[i].heads);

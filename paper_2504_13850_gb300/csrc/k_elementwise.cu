@@ -631,6 +631,43 @@ void sgd_momentum(float* theta, float* v, const float* g, void* shadow, int64_t 
   launch_k(sgd_momentum_k, elementwise_blocks(n4, 256), 256, 0, st,
       (float4*)theta, (float4*)v, (const float4*)g, (uint2*)shadow, n4, lr, mu, step, skip64);
 }
+// The same update over a list of 64-element blocks (the parameters an
+// earlier partial update left): 16 float4 per block.
+__global__ void sgd_momentum_blocks_k(float4* __restrict__ theta, float4* __restrict__ v,
+                                      const float4* __restrict__ g, uint2* __restrict__ shadow,
+                                      const int64_t* __restrict__ blocks, int64_t nb, float lr, float mu,
+                                      int64_t* step) {
+  pdl_wait();
+  pdl_trigger();
+  if (step && blockIdx.x == 0 && threadIdx.x == 0) *step += 1;
+  GRID_STRIDE(j, nb * 16) {
+    const int64_t i = blocks[j / 16] * 16 + j % 16;
+    float4 t = theta[i], m = v[i];
+    const float4 gr = g[i];
+    m.x = fmaf(mu, m.x, gr.x);
+    m.y = fmaf(mu, m.y, gr.y);
+    m.z = fmaf(mu, m.z, gr.z);
+    m.w = fmaf(mu, m.w, gr.w);
+    t.x = fmaf(-lr, m.x, t.x);
+    t.y = fmaf(-lr, m.y, t.y);
+    t.z = fmaf(-lr, m.z, t.z);
+    t.w = fmaf(-lr, m.w, t.w);
+    v[i] = m;
+    theta[i] = t;
+    if (shadow) {
+      __nv_bfloat162 lo = __floats2bfloat162_rn(t.x, t.y), hi = __floats2bfloat162_rn(t.z, t.w);
+      uint2 u;
+      u.x = *reinterpret_cast<uint32_t*>(&lo);
+      u.y = *reinterpret_cast<uint32_t*>(&hi);
+      shadow[i] = u;
+    }
+  }
+}
+void sgd_momentum_blocks(float* theta, float* v, const float* g, void* shadow, const int64_t* blocks64, int64_t nb,
+                         float lr, float mu, int64_t* step, cudaStream_t st) {
+  launch_k(sgd_momentum_blocks_k, elementwise_blocks(nb * 16, 256), 256, 0, st, (float4*)theta, (float4*)v,
+           (const float4*)g, (uint2*)shadow, blocks64, nb, lr, mu, step);
+}
 __global__ void f32_to_bf16_k(const float* x, bf16* y, int64_t n) {
   pdl_wait();
   pdl_trigger();
