@@ -496,7 +496,7 @@ int build_plan(fo_server* s) {
         fo::head_weight_grad((const float*)s->T[o].grad, act(a0), s->T[a0].dt, B, K, C, G(s, i, 0),
                              op.bias ? G(s, i, 1) : nullptr, s->row_loss, s->losses, s->d_step,
                              s->kLossRing - 1, st);
-      });
+      }, 1);
       if (need_dx) {
         int accf = contrib(a);
         add("head_dgrad", 1, 2.0 * B * K * C, (2 + accf) * tbytes(a), [=](cudaStream_t st) {
@@ -778,7 +778,6 @@ int build_plan(fo_server* s) {
   }
 
   // ---------------- optimizer (Algorithm 4: theta_s <- theta_s - gamma_s * update)
-  const size_t first_opt = plan.size();   // the side stream joins before this entry
   if (!bias_tasks.empty())
     add("bias_grad", int((bias_tasks.size() + 39) / 40), 0.0, deferred_bytes, [=](cudaStream_t st) {
       fo::colsum8_batched(bias_tasks, st);
@@ -819,7 +818,7 @@ int build_plan(fo_server* s) {
                        st, skip);
     });
   }
-  plan[first_opt].join = true;
+  plan.back().join = true;   // the side and optimizer streams join before the final update
   for (int i = 0; i < nops; ++i)
     if (s->ops[i].kind == FO_OP_ATTENTION) fo::attention_prepare(s->T[s->ops[i].in0].H, s->ops[i].cin, s->ops[i].heads);
   return FO_OK;
