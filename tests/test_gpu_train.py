@@ -230,3 +230,24 @@ def test_empty_and_bad_calls():
     assert s.enqueue_activations(7, x, labels)[0] == api.ERR_ARG
     s.set_device_active(2, False)
     assert s.enqueue_activations(2, x, labels)[0] == api.ERR_ARG
+
+
+@pytest.mark.parametrize("name", ["tiny", "vgg"])
+def test_uploads_into_slots_still_being_read(name):
+    """Backlogged queues: after every step the next upload goes into the slot
+    that step has just freed while its kernels may still be running, so the
+    upload is staged on the device and moved in after the step.  Outcomes
+    bit-exact, losses and parameters at the path's tolerances."""
+    cfg = W.CONFIGS[name]
+    if name == "vgg":
+        cfg = W.shrink(cfg, K=3, omega=3, depth=1)
+    ev = [("enq", k) for k in range(cfg["K"])]
+    for j in range(8):
+        ev += [("step",), ("enq", j % cfg["K"])]
+    if cfg["dtype"] == W.F32:
+        s, _ = compare(cfg, ev, loss_tol=1e-4, param_tol=1e-4, upd_tol=1e-4)
+        assert s.read_losses(0, 8).shape == (8,)
+    else:
+        _, _, recs = teacher_forced(cfg, ev)
+        assert len(recs) == 8
+        check_teacher_forced(recs)
