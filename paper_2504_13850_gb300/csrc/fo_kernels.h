@@ -155,6 +155,10 @@ void affine_bwd8_pass(const void* dy, const void* x, const float* scale, void* d
 // Affine then hard swish in one pass: pre = x * scale + shift, post = hswish(pre).
 void affine_hswish_fwd_x8(const void* x, const float* sc, const float* sh, void* pre, void* post, int64_t n, int C,
                           cudaStream_t st);
+// Layernorm forward with the row in registers (bf16, C % 256 == 0, C <= 1024).
+bool layernorm_fwd8_ok(int dt, int C);
+void layernorm_fwd_x8(const void* x, const float* gamma, const float* beta, void* y, float* mean, float* rstd,
+                      int64_t rows, int C, cudaStream_t st);
 // Layernorm backward fused with dgamma / dbeta (C % 256 == 0, C <= 512).
 bool layernorm_bwd8_ok(int dt, int C);
 int64_t layernorm_bwd8_partial_floats(int64_t rows, int C);

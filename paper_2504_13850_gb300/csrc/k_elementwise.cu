@@ -416,6 +416,7 @@ __global__ void layernorm_bwd_k(const T* x, const float* gamma, const float* mea
 }
 void layernorm_fwd(const void* x, const float* gamma, const float* beta, void* y, float* mean,
                    float* rstd, int64_t rows, int C, int dt, cudaStream_t st) {
+  if (layernorm_fwd8_ok(dt, C)) return layernorm_fwd_x8(x, gamma, beta, y, mean, rstd, rows, C, st);
   int blocks = ceil_div(rows, 8);
   FO_DISPATCH(dt, T, launch_k(layernorm_fwd_k<T>, blocks, 256, 0, st, (const T*)x, gamma, beta, (T*)y, mean, rstd, rows, C));
 }

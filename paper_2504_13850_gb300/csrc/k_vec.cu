@@ -286,6 +286,61 @@ __global__ void __launch_bounds__(256) colsum8_batch_k(const __grid_constant__ C
                    local % cbs, local / cbs);
 }
 
+// Layernorm forward, one warp per row held in registers (C % 256 == 0,
+// C <= 1024): one read of x, mean then biased variance from the registers
+// (eps 1e-5), one write of y; the row mean and 1/std are kept for the
+// backward pass.
+__global__ void __launch_bounds__(256) layernorm_fwd_x8_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
+                                                          const float* __restrict__ beta, bf16* __restrict__ y,
+                                                          float* __restrict__ mean_out, float* __restrict__ rstd_out,
+                                                          int64_t rows, int C) {
+  pdl_wait();
+  pdl_trigger();
+  constexpr int kMaxV = 4;
+  const int lane = threadIdx.x % 32;
+  const int64_t row = int64_t(blockIdx.x) * (blockDim.x / 32) + threadIdx.x / 32;
+  if (row >= rows) return;
+  const int nv = C / 256;
+  V8 xv[kMaxV];
+  float sum = 0.f;
+#pragma unroll
+  for (int v = 0; v < kMaxV; ++v) {
+    if (v >= nv) break;
+    xv[v] = ld8(x + row * C + (v * 32 + lane) * 8);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) sum += xv[v].v[j];
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+  const float mu = sum / float(C);
+  float q = 0.f;
+#pragma unroll
+  for (int v = 0; v < kMaxV; ++v) {
+    if (v >= nv) break;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float d = xv[v].v[j] - mu;
+      q = fmaf(d, d, q);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+  const float rs = rsqrtf(q / float(C) + 1e-5f);
+#pragma unroll
+  for (int v = 0; v < kMaxV; ++v) {
+    if (v >= nv) break;
+    const int c = (v * 32 + lane) * 8;
+    V8 o;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) o.v[j] = (xv[v].v[j] - mu) * rs * gamma[c + j] + beta[c + j];
+    st8(y + row * C + c, o);
+  }
+  if (lane == 0) {
+    mean_out[row] = mu;
+    rstd_out[row] = rs;
+  }
+}
+
 // Layernorm backward fused with its parameter gradients: one warp per row
 // (dx), and per block of 8 warps x 2 rows the column partials of
 // dy * xhat (gamma) and dy (beta).  C <= 512, C % 256 == 0; dx may be null
@@ -573,6 +628,13 @@ void finish_batched(const std::vector<FinishTask>& tasks, cudaStream_t st) {
 bool layernorm_bwd8_ok(int dt, int C) { return dt == kBF16 && C % 256 == 0 && C <= 512; }
 
 int layernorm_bwd8_blocks(int64_t rows) { return int((rows + 15) / 16); }
+
+bool layernorm_fwd8_ok(int dt, int C) { return dt == kBF16 && C % 256 == 0 && C <= 1024; }
+void layernorm_fwd_x8(const void* x, const float* gamma, const float* beta, void* y, float* mean, float* rstd,
+                      int64_t rows, int C, cudaStream_t st) {
+  launch_k(layernorm_fwd_x8_k, ceil_div(rows, 8), 256, 0, st, (const bf16*)x, gamma, beta, (bf16*)y, mean, rstd, rows,
+           C);
+}
 
 void layernorm_bwd8_pass(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
                          void* dx, int64_t rows, int C, bool acc, float* p_gamma, float* p_beta, cudaStream_t st) {
