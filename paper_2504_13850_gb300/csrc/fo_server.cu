@@ -43,6 +43,11 @@ namespace {
 
 int64_t pad64(int64_t n) { return (n + 63) / 64 * 64; }
 
+// Weight tensors of at least this many parameters get their own update as
+// soon as their gradient is final; smaller ones (where a launch costs more
+// than the traffic it moves) are left to the step's final update.
+constexpr int64_t kEarlyUpdateMin = 128 * 1024;
+
 // Shape inference and parameter layout.  Returns FO_OK or an error.
 int infer(fo_server* s) {
   const fo_server_cfg& c = s->cfg;
@@ -561,7 +566,7 @@ int build_plan(fo_server* s) {
             });
           }
         }
-        {
+        if (s->segs[s->op_segs[i][0]].n >= kEarlyUpdateMin) {
           // the weights' update, forked after the input gradient that read them
           const ParamSeg seg = s->segs[s->op_segs[i][0]];
           const int64_t len = pad64(seg.n);
