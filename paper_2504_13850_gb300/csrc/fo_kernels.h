@@ -83,8 +83,11 @@ void attention_bwd(const void* qkv, const int32_t* len, const float* probs, cons
                    cudaStream_t st);
 
 // Classifier head (last linear layer + softmax cross-entropy), fp32 weights.
+// With dx given, also the input gradient dx (+)= dz W (times mask > 0 when
+// mask is given), formed by the same blocks (no second launch).
 void head_forward_loss(const void* x, int dt, const float* W, const float* bias, const int32_t* labels,
-                       int B, int K, int C, float* logits, float* dz, float* row_loss, cudaStream_t st);
+                       int B, int K, int C, float* logits, float* dz, float* row_loss, cudaStream_t st,
+                       const void* mask = nullptr, void* dx = nullptr, bool acc = false);
 // The batch loss goes to losses[*step & mask].
 void head_weight_grad(const float* dz, const void* x, int dt, int B, int K, int C, float* dW, float* db,
                       const float* row_loss, float* losses, const int64_t* step, int64_t mask,

@@ -299,10 +299,18 @@ int build_plan(fo_server* s) {
     const Tensor& ta = s->T[a];
     const Tensor& to = s->T[i + 1];
     if (fu.head && i == L) {
+      // logits, loss, dz and (when the input needs one) the input gradient:
+      // the classifier is the first op of the backward pass, so that
+      // gradient is its destination's first contribution
       const int B = s->cfg.batch, K = op.cin, C = op.cout;
-      add("head_fwd_ce", 1, 2.0 * B * K * C, tbytes(a), [=](cudaStream_t st) {
+      const int mr = fu.bwd_mask[i];
+      const int da = mr >= 0 ? s->ops[mr].in0 : a;
+      const void* mask = mr >= 0 ? s->T[mr + 1].act : nullptr;
+      const bool dx = a != 0;
+      add("head_fwd_ce", 1, 2.0 * B * K * C * (dx ? 2.0 : 1.0), tbytes(a) * (dx ? 3.0 : 1.0), [=](cudaStream_t st) {
         fo::head_forward_loss(act(a), s->T[a].dt, P(s, i, 0), op.bias ? P(s, i, 1) : nullptr, s->cur_labels, B,
-                              K, C, (float*)s->T[i + 1].act, (float*)s->T[i + 1].grad, s->row_loss, st);
+                              K, C, (float*)s->T[i + 1].act, (float*)s->T[i + 1].grad, s->row_loss, st, mask,
+                              dx ? s->T[da].grad : nullptr, false);
       });
       continue;
     }
@@ -502,13 +510,8 @@ int build_plan(fo_server* s) {
                              op.bias ? G(s, i, 1) : nullptr, s->row_loss, s->losses, s->d_step,
                              s->kLossRing - 1, st);
       }, 1);
-      if (need_dx) {
-        int accf = contrib(a);
-        add("head_dgrad", 1, 2.0 * B * K * C, (2 + accf) * tbytes(a), [=](cudaStream_t st) {
-          fo::head_input_grad((const float*)s->T[o].grad, P(s, i, 0), B, K, C, mask, s->T[a].grad, s->T[a].dt,
-                              accf != 0, st);
-        });
-      }
+      if (need_dx && contrib(a) != 0)   // formed in the forward launch as the first contribution
+        return set_err(FO_ERR_ARG, "classifier input gradient is not the first contribution");
       continue;
     }
     switch (op.kind) {

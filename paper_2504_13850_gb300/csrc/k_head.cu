@@ -26,16 +26,21 @@ __device__ __forceinline__ float warp_max(float v) {
 
 // One block per batch row; warps split the classes.  smem: x row (K floats)
 // and the logits (C floats).
+// With `dx` given, the same block then forms its row's input gradient
+// dx[b][k] (+)= (sum_c dz[b][c] W[c][k]) * (mask[b][k] > 0): a row's input
+// gradient needs only that row's dz, so the backward needs no second launch.
 template <typename T>
 __global__ void head_fwd_ce_k(const T* __restrict__ x, const float* __restrict__ W,
                               const float* __restrict__ bias, const int32_t* __restrict__ labels, int B,
                               int K, int C, float* __restrict__ logits, float* __restrict__ dz,
-                              float* __restrict__ row_loss) {
+                              float* __restrict__ row_loss, const T* __restrict__ mask, T* __restrict__ dx,
+                              int acc) {
   pdl_wait();
   pdl_trigger();
   extern __shared__ float sm[];
   float* xr = sm;
   float* z = sm + K;
+  float* zd = z + C;
   const int b = blockIdx.x;
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32, nw = blockDim.x / 32;
   for (int k = threadIdx.x; k < K; k += blockDim.x) xr[k] = to_f(x[int64_t(b) * K + k]);
@@ -58,10 +63,22 @@ __global__ void head_fwd_ce_k(const T* __restrict__ x, const float* __restrict__
     const int y = labels[b];
     for (int c = lane; c < C; c += 32) {
       const float p = expf(z[c] - m) / se;
-      dz[int64_t(b) * C + c] = (p - (c == y ? 1.f : 0.f)) / float(B);
+      const float d = (p - (c == y ? 1.f : 0.f)) / float(B);
+      dz[int64_t(b) * C + c] = d;
+      zd[c] = d;
       logits[int64_t(b) * C + c] = z[c];
     }
     if (lane == 0) row_loss[b] = m + logf(se) - z[y];
+  }
+  if (!dx) return;
+  __syncthreads();
+  for (int k = threadIdx.x; k < K; k += blockDim.x) {
+    float s = 0.f;
+    for (int c = 0; c < C; ++c) s = fmaf(zd[c], W[int64_t(c) * K + k], s);
+    const int64_t i = int64_t(b) * K + k;
+    if (mask && !(to_f(mask[i]) > 0.f)) s = 0.f;
+    if (acc) s += to_f(dx[i]);
+    dx[i] = from_f<T>(s);
   }
 }
 
@@ -129,12 +146,15 @@ __global__ void head_dgrad_k(const float* __restrict__ dz, const float* __restri
 }  // namespace
 
 void head_forward_loss(const void* x, int dt, const float* W, const float* bias, const int32_t* labels, int B,
-                       int K, int C, float* logits, float* dz, float* row_loss, cudaStream_t st) {
-  size_t sm = sizeof(float) * (K + C);
+                       int K, int C, float* logits, float* dz, float* row_loss, cudaStream_t st, const void* mask,
+                       void* dx, bool acc) {
+  size_t sm = sizeof(float) * (K + 2 * C);
   if (dt == kF32)
-    launch_k(head_fwd_ce_k<float>, B, 256, sm, st, (const float*)x, W, bias, labels, B, K, C, logits, dz, row_loss);
+    launch_k(head_fwd_ce_k<float>, B, 256, sm, st, (const float*)x, W, bias, labels, B, K, C, logits, dz, row_loss,
+             (const float*)mask, (float*)dx, acc ? 1 : 0);
   else
-    launch_k(head_fwd_ce_k<bf16>, B, 256, sm, st, (const bf16*)x, W, bias, labels, B, K, C, logits, dz, row_loss);
+    launch_k(head_fwd_ce_k<bf16>, B, 256, sm, st, (const bf16*)x, W, bias, labels, B, K, C, logits, dz, row_loss,
+             (const bf16*)mask, (bf16*)dx, acc ? 1 : 0);
 }
 
 void head_weight_grad(const float* dz, const void* x, int dt, int B, int K, int C, float* dW, float* db,
