@@ -1,10 +1,12 @@
 // Classifier head of the server network: the last linear layer (few
 // outputs) fused with the server loss f_s (softmax cross-entropy averaged
 // over the batch) and its backward pass.
-//   head_fwd_ce : logits z = x W^T + b, per-row CE, dz = (softmax(z) - onehot)/B
+//   head_fwd_ce : logits z = x W^T + b, per-row CE, dz = (softmax(z) - onehot)/B,
+//                 and (optionally, in the same blocks) dx (+)= dz W, times a
+//                 ReLU mask (mask > 0) when one is given
 //   head_wgrad  : dW = dz^T x, db = sum_b dz, loss = mean of the row losses
 //                 (summed in row order, deterministic)
-//   head_dgrad  : dx (+)= dz W, optionally times a ReLU mask (mask > 0)
+//   head_dgrad  : dx (+)= dz W as a launch of its own (the same arithmetic)
 // W and b are the fp32 master weights; dz and the gradients are fp32.
 #include "fo_common.cuh"
 #include "fo_kernels.h"
