@@ -47,6 +47,10 @@ void affine_dx(const void* dy, const float* scale, void* dx, int64_t rows, int C
 void add_fwd(const void* a, const void* b, void* y, int64_t n, int dt, bool relu, cudaStream_t st);
 // y (+)= x
 void copy_or_acc(const void* x, void* y, int64_t n, int dt, bool acc, cudaStream_t st);
+// Backward of a residual add, optionally through the ReLU after it:
+// g = dy * (mask > 0) (mask may be null); d0 (+)= g; d1 (+)= g (d1 may be null).
+void grad_split(const void* dy, const void* mask, void* d0, bool acc0, void* d1, bool acc1, int64_t n, int dt,
+                cudaStream_t st);
 void avgpool_fwd(const void* x, void* y, int N, int HW, int C, int dt, cudaStream_t st);
 void avgpool_bwd(const void* dy, void* dx, int N, int HW, int C, int dt, bool acc,
                  cudaStream_t st);
@@ -116,6 +120,8 @@ bool vec8_ok(int dt, int64_t n);
 void relu_bwd_x8(const void* y, const void* dy, void* dx, int64_t n, bool acc, cudaStream_t st);
 void add_x8(const void* a, const void* b, void* y, int64_t n, bool relu, cudaStream_t st);
 void copy_acc_x8(const void* x, void* y, int64_t n, bool acc, cudaStream_t st);
+void grad_split_x8(const void* dy, const void* mask, void* d0, bool acc0, void* d1, bool acc1, int64_t n,
+                   cudaStream_t st);
 void affine_fwd_x8(const void* x, const float* sc, const float* sh, void* y, int64_t n, int C, bool relu,
                    cudaStream_t st);
 void gelu_fwd_x8(const void* x, void* y, int64_t n, cudaStream_t st);

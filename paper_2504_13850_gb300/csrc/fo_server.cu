@@ -203,6 +203,8 @@ struct Fusion {
   std::vector<char> skip_bwd;  // relu op whose backward is done by its consumer
   std::vector<int> hswish_of;  // affine op -> the hard swish op it applies (both passes), or -1
   std::vector<int> hswish_by;  // hard swish op -> the affine op that applies it, or -1
+  std::vector<int> add_relu;   // residual add op -> the relu after it, whose backward the add's applies, or -1
+  std::vector<int> relu_into_add;  // that relu op -> the add op, or -1
   bool head = false;           // last linear + loss handled by the head kernels
 };
 
@@ -220,6 +222,8 @@ Fusion analyse(const fo_server* s) {
   f.skip_bwd.assign(nops, 0);
   f.hswish_of.assign(nops, -1);
   f.hswish_by.assign(nops, -1);
+  f.add_relu.assign(nops, -1);
+  f.relu_into_add.assign(nops, -1);
   std::vector<int> sole(nops + 1, -1);  // the only consumer op of a tensor
   for (int j = 0; j < nops; ++j) {
     const fo_op& op = s->ops[j];
@@ -242,6 +246,18 @@ Fusion analyse(const fo_server* s) {
     if (j >= 0 && s->ops[j].in0 == r + 1 && (dx_takes_mask(s, j) || (f.head && j == nops - 1))) {
       f.bwd_mask[j] = r;
       f.skip_bwd[r] = 1;
+    }
+  }
+  // A relu whose input is a residual add's output (and that add's only
+  // consumer), not already applied by its own consumer: the add's backward
+  // masks the relu output's gradient on the fly and writes both inputs.
+  for (int r = 0; r < nops; ++r) {
+    const fo_op& op = s->ops[r];
+    if (op.kind != FO_OP_RELU || op.in0 == 0 || f.skip_bwd[r]) continue;
+    const int p = op.in0 - 1;
+    if (s->ops[p].kind == FO_OP_ADD && sole[op.in0] == r) {
+      f.add_relu[p] = r;
+      f.relu_into_add[r] = p;
     }
   }
   // A batch-norm affine whose only consumer is a hard swish (the MobileNetV3
@@ -478,9 +494,9 @@ int build_plan(fo_server* s) {
       written[s->T[i + 1].root] = 1;
       continue;
     }
-    if (fu.hswish_by[i] >= 0) {
-      // the affine's backward applies this hard swish: its input gradient is
-      // present exactly when the output's is
+    if (fu.hswish_by[i] >= 0 || fu.relu_into_add[i] >= 0) {
+      // the producer's backward applies this hard swish / relu: its input
+      // gradient is present exactly when the output's is
       written[s->T[op.in0].root] = written[s->T[i + 1].root];
       continue;
     }
@@ -640,14 +656,35 @@ int build_plan(fo_server* s) {
         }
         break;
       case FO_OP_ADD: {
+        // one pass over the output gradient (masked by the relu after the
+        // add when that relu's backward is folded in) into both inputs
         const int b = op.in1;
+        const int rr = fu.add_relu[i];
+        const int dyt = rr >= 0 ? rr + 1 : o;
+        const void* msk = rr >= 0 ? s->T[rr + 1].act : nullptr;
+        int srcs[2], accs[2], ns = 0;
         for (int src : {a0, b}) {
           if (src == 0) continue;
-          int accf = contrib(src);
-          add("add_bwd", 1, 0.0, (2 + accf) * csb, [=](cudaStream_t st) {
-            fo::copy_or_acc(s->T[o].grad, s->T[src].grad, s->T[o].numel(), dt, accf != 0, st);
-          });
+          srcs[ns] = src;
+          accs[ns] = contrib(src);
+          ++ns;
         }
+        if (ns == 0) break;
+        const int64_t n = s->T[o].numel();
+        if (ns == 2 && s->T[srcs[0]].root == s->T[srcs[1]].root) {   // x + x: two passes into one buffer
+          for (int q = 0; q < 2; ++q) {
+            const int src = srcs[q], accf = accs[q];
+            add("add_bwd", 1, 0.0, (2 + accf + (msk ? 1 : 0)) * csb, [=](cudaStream_t st) {
+              fo::grad_split(s->T[dyt].grad, msk, s->T[src].grad, accf != 0, nullptr, false, n, dt, st);
+            });
+          }
+          break;
+        }
+        const int s0 = srcs[0], s1 = ns == 2 ? srcs[1] : -1, acc0 = accs[0], acc1 = ns == 2 ? accs[1] : 0;
+        add("add_bwd", 1, 0.0, (1 + (msk ? 1 : 0) + ns + acc0 + acc1) * csb, [=](cudaStream_t st) {
+          fo::grad_split(s->T[dyt].grad, msk, s->T[s0].grad, acc0 != 0, s1 >= 0 ? s->T[s1].grad : nullptr,
+                         acc1 != 0, n, dt, st);
+        });
         break;
       }
       case FO_OP_AVGPOOL:

@@ -267,6 +267,23 @@ __global__ void add_fwd_k(const T* a, const T* b, T* y, int64_t n, int relu) {
   }
 }
 template <typename T>
+__global__ void grad_split_k(const T* __restrict__ dy, const T* __restrict__ mask, T* __restrict__ d0, int acc0,
+                             T* __restrict__ d1, int acc1, int64_t n) {
+  pdl_wait();
+  pdl_trigger();
+  GRID_STRIDE(i, n) {
+    const float g = (mask && !(to_f(mask[i]) > 0.f)) ? 0.f : to_f(dy[i]);
+    store(d0, i, g, acc0);
+    if (d1) store(d1, i, g, acc1);
+  }
+}
+void grad_split(const void* dy, const void* mask, void* d0, bool acc0, void* d1, bool acc1, int64_t n, int dt,
+                cudaStream_t st) {
+  if (vec8_ok(dt, n)) return grad_split_x8(dy, mask, d0, acc0, d1, acc1, n, st);
+  FO_DISPATCH(dt, T, launch_k(grad_split_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)dy, (const T*)mask,
+                              (T*)d0, acc0 ? 1 : 0, (T*)d1, acc1 ? 1 : 0, n));
+}
+template <typename T>
 __global__ void copy_acc_k(const T* x, T* y, int64_t n, int acc) {
   pdl_wait();
   pdl_trigger();

@@ -70,6 +70,43 @@ __global__ void add_x8_k(const bf16* __restrict__ a, const bf16* __restrict__ b,
   }
 }
 
+// Backward of a residual add (optionally with the ReLU that follows it):
+// g = dy (times mask > 0 when mask is given) goes to both inputs' gradients,
+// d0 (+)= g and d1 (+)= g (d1 may be null), in one pass over dy.
+__global__ void grad_split_x8_k(const bf16* __restrict__ dy, const bf16* __restrict__ mask, bf16* __restrict__ d0,
+                                int acc0, bf16* __restrict__ d1, int acc1, int64_t n8) {
+  pdl_wait();
+  pdl_trigger();
+  GRID_STRIDE8(i, n8) {
+    V8 g = ld8(dy + 8 * i);
+    if (mask) {
+      const V8 m = ld8(mask + 8 * i);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) g.v[j] = m.v[j] > 0.f ? g.v[j] : 0.f;
+    }
+    if (acc0) {
+      const V8 q = ld8(d0 + 8 * i);
+      V8 o;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) o.v[j] = g.v[j] + q.v[j];
+      st8(d0 + 8 * i, o);
+    } else {
+      st8(d0 + 8 * i, g);
+    }
+    if (d1) {
+      if (acc1) {
+        const V8 q = ld8(d1 + 8 * i);
+        V8 o;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) o.v[j] = g.v[j] + q.v[j];
+        st8(d1 + 8 * i, o);
+      } else {
+        st8(d1 + 8 * i, g);
+      }
+    }
+  }
+}
+
 __global__ void copy_acc_x8_k(const bf16* __restrict__ x, bf16* __restrict__ y, int64_t n8, int acc) {
   pdl_wait();
   pdl_trigger();
@@ -528,6 +565,11 @@ void relu_bwd_x8(const void* y, const void* dy, void* dx, int64_t n, bool acc, c
 }
 void add_x8(const void* a, const void* b, void* y, int64_t n, bool relu, cudaStream_t st) {
   launch_k(add_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)a, (const bf16*)b, (bf16*)y, n / 8, relu);
+}
+void grad_split_x8(const void* dy, const void* mask, void* d0, bool acc0, void* d1, bool acc1, int64_t n,
+                   cudaStream_t st) {
+  launch_k(grad_split_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)dy, (const bf16*)mask, (bf16*)d0,
+           acc0 ? 1 : 0, (bf16*)d1, acc1 ? 1 : 0, n / 8);
 }
 void copy_acc_x8(const void* x, void* y, int64_t n, bool acc, cudaStream_t st) {
   launch_k(copy_acc_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)x, (bf16*)y, n / 8, acc);
