@@ -50,6 +50,11 @@ extern "C" {
 #define FO_ERR_TIMEOUT (-4)  /* a bounded device-side wait gave up                 */
 #define FO_ERR_UNSUPPORTED (-5) /* a layer shape this build has no kernel for      */
 
+/* Size limits of the Task Scheduler (both fo_server_create and
+ * fo_sched_create return FO_ERR_ARG beyond them). */
+#define FO_MAX_DEVICES (1 << 20)  /* K     */
+#define FO_MAX_OMEGA (1 << 24)    /* omega */
+
 /* ------------------------------------------------------------ layer spec */
 /* Op kinds of the server-side network M_s (Sec. 3.2: M is split at a layer,
  * M_s holds the remaining layers).  Tensor 0 is the uploaded activation
@@ -121,7 +126,9 @@ typedef struct fo_server fo_server;
  * memory is mu_model + omega * mu_act, independent of K) and all
  * intermediate tensors for one batch.  Parameters start at zero: load them
  * with fo_server_set_params.  Returns FO_ERR_UNSUPPORTED for layer shapes
- * without a kernel (e.g. bf16 conv channels not a multiple of 64). */
+ * without a kernel (e.g. bf16 conv channels not a multiple of 64), FO_ERR_ARG
+ * for K or omega above FO_MAX_DEVICES / FO_MAX_OMEGA, FO_ERR_OOM when a
+ * device or host allocation fails. */
 FO_API int fo_server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt,
                      const fo_server_cfg* cfg, fo_server** out);
 FO_API int fo_server_destroy(fo_server* s);
@@ -252,6 +259,9 @@ FO_API const char* fo_last_error(void);
  * Host-only Task Scheduler (Algorithms 2-3 and the flow control of Sec.
  * 3.4.1) without any GPU state: the same logic fo_server uses, for trace
  * replay and tests.  put returns the slot the batch would occupy.
+ * 1 <= K <= FO_MAX_DEVICES, 1 <= omega <= FO_MAX_OMEGA, depth >= 1 (a depth
+ * above omega acts as omega: the cap is reached first).  Create returns
+ * FO_ERR_OOM when the host allocation fails.
  * ---------------------------------------------------------------------- */
 typedef struct fo_sched fo_sched;
 FO_API int fo_sched_create(int K, int omega, int depth, int policy, fo_sched** out);

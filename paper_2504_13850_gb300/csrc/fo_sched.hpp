@@ -20,9 +20,11 @@ enum SchedPolicy { kCounter = 0, kFifo = 1 };
 
 class TaskScheduler {
  public:
+  // A depth above omega never binds (sum_k |Q_k| <= omega is reached
+  // first), so the rings hold min(depth, omega) entries per device.
   TaskScheduler(int K, int omega, int depth, int policy)
-      : K_(K), omega_(omega), depth_(depth), policy_(policy),
-        ring_(size_t(K) * depth), head_(K, 0), len_(K, 0), c_(K, 0),
+      : K_(K), omega_(omega), depth_(depth < omega ? depth : omega), policy_(policy),
+        ring_(size_t(K) * depth_), head_(K, 0), len_(K, 0), c_(K, 0),
         on_(K, 1), active_(K, 1), free_(omega), blocked_flag_(K, 0) {
     for (int i = 0; i < omega; ++i) free_[i] = i;
     free_head_ = 0;

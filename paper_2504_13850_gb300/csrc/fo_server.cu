@@ -990,9 +990,9 @@ void destroy_impl(fo_server* s) {
     cudaEventDestroy(r.b);
   }
   for (auto e : s->ev_pool) cudaEventDestroy(e);
-  for (void* p : s->allocs) cudaFree(p);
   if (s->side) cudaStreamSynchronize(s->side);
   if (s->opt_st) cudaStreamSynchronize(s->opt_st);
+  for (void* p : s->allocs) cudaFree(p);
   if (s->cs) cudaStreamDestroy(s->cs);
   if (s->xs) cudaStreamDestroy(s->xs);
   if (s->hs) cudaStreamDestroy(s->hs);
@@ -1092,19 +1092,40 @@ extern "C" {
 
 const char* fo_last_error(void) { return g_err.c_str(); }
 
+static int server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt, const fo_server_cfg* cfg,
+                         fo_server** out, fo_server** held);
+
+// No C++ exception crosses the C ABI: a host allocation that fails inside
+// (std::bad_alloc) releases the half-built server and returns FO_ERR_OOM.
 int fo_server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt, const fo_server_cfg* cfg,
                      fo_server** out) {
+  fo_server* held = nullptr;
+  try {
+    return server_create(ops, n_ops, opt, cfg, out, &held);
+  } catch (const std::bad_alloc&) {
+    destroy_impl(held);
+    return set_err(FO_ERR_OOM, "host allocation");
+  } catch (const std::exception& e) {
+    destroy_impl(held);
+    return set_err(FO_ERR_ARG, e.what());
+  }
+}
+
+static int server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt, const fo_server_cfg* cfg,
+                         fo_server** out, fo_server** held) {
   g_err.clear();
   if (!ops || n_ops <= 0 || !opt || !cfg || !out) return set_err(FO_ERR_ARG, "null argument");
   *out = nullptr;
   const fo_server_cfg& c = *cfg;
-  if (c.num_devices <= 0 || c.omega <= 0 || c.depth <= 0 || c.batch <= 0 || c.batch > 1024 ||
+  if (c.num_devices <= 0 || c.num_devices > FO_MAX_DEVICES || c.omega <= 0 || c.omega > FO_MAX_OMEGA ||
+      c.depth <= 0 || c.batch <= 0 || c.batch > 1024 ||
       c.in_h <= 0 || c.in_w <= 0 || c.in_c <= 0 || c.num_classes <= 0 ||
       (c.dtype != FO_DTYPE_F32 && c.dtype != FO_DTYPE_BF16) || c.max_delay < 0 ||
       (c.sched_policy != FO_SCHED_COUNTER && c.sched_policy != FO_SCHED_FIFO))
     return set_err(FO_ERR_ARG, "bad server configuration");
   fo_server* s = new (std::nothrow) fo_server();
   if (!s) return set_err(FO_ERR_OOM, "host allocation");
+  *held = s;
   s->cfg = c;
   s->opt = *opt;
   s->dt = c.dtype == FO_DTYPE_F32 ? fo::kF32 : fo::kBF16;
@@ -1519,9 +1540,18 @@ struct fo_sched {
 };
 
 int fo_sched_create(int K, int omega, int depth, int policy, fo_sched** out) {
-  if (!out || K <= 0 || omega <= 0 || depth <= 0 || (policy != FO_SCHED_COUNTER && policy != FO_SCHED_FIFO))
+  if (!out || K <= 0 || K > FO_MAX_DEVICES || omega <= 0 || omega > FO_MAX_OMEGA || depth <= 0 ||
+      (policy != FO_SCHED_COUNTER && policy != FO_SCHED_FIFO))
     return set_err(FO_ERR_ARG, "bad scheduler configuration");
-  *out = new fo_sched{new fo::TaskScheduler(K, omega, depth, policy)};
+  *out = nullptr;
+  fo::TaskScheduler* t = nullptr;
+  try {
+    t = new fo::TaskScheduler(K, omega, depth, policy);
+    *out = new fo_sched{t};
+  } catch (const std::bad_alloc&) {
+    delete t;
+    return set_err(FO_ERR_OOM, "host allocation");
+  }
   return FO_OK;
 }
 int fo_sched_destroy(fo_sched* s) {

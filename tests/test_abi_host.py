@@ -113,3 +113,28 @@ def test_scheduler_matches_oracle_on_zipf_trace_of_100_devices():
     served = [c for c in o.c if c > 0]
     fifo_served = [c for c in f.c if c > 0]
     assert max(o.c) - min(served) <= max(fifo_served) - min(fifo_served)
+
+
+def test_scheduler_size_limits_and_depth_above_omega():
+    """K and omega beyond FO_MAX_DEVICES / FO_MAX_OMEGA are refused before
+    anything is allocated; a ring depth far above omega never binds (the
+    global cap is met first), so the trace equals the oracle's with that
+    depth, without rings of that depth being allocated."""
+    import ctypes
+    L = api.lib()
+    h = ctypes.c_void_p()
+    assert L.fo_sched_create((1 << 20) + 1, 4, 2, api.SCHED_COUNTER, ctypes.byref(h)) == api.ERR_ARG
+    assert L.fo_sched_create(4, (1 << 24) + 1, 2, api.SCHED_COUNTER, ctypes.byref(h)) == api.ERR_ARG
+    assert L.fo_sched_create(4, 4, 0, api.SCHED_COUNTER, ctypes.byref(h)) == api.ERR_ARG
+    r = np.random.default_rng(7)
+    K, omega, depth = 5, 7, 1 << 30
+    a = api.Scheduler(K, omega, depth)
+    o = O.TaskScheduler(K, omega, depth)
+    for _ in range(400):
+        if r.random() < 0.55:
+            k = int(r.integers(K))
+            rc, slot, on = a.put(k)
+            assert (rc, slot, on) == (*o.put(k), int(o.on[k]))
+        else:
+            assert a.get() == o.get()
+        assert a.counters() == o.c
