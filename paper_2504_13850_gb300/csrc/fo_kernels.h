@@ -45,8 +45,6 @@ void affine_fwd(const void* x, const float* scale, const float* shift, void* y, 
 void affine_dx(const void* dy, const float* scale, void* dx, int64_t rows, int C, int dt,
                bool acc, cudaStream_t st);
 void add_fwd(const void* a, const void* b, void* y, int64_t n, int dt, bool relu, cudaStream_t st);
-// y (+)= x
-void copy_or_acc(const void* x, void* y, int64_t n, int dt, bool acc, cudaStream_t st);
 // Backward of a residual add, optionally through the ReLU after it:
 // g = dy * (mask > 0) (mask may be null); d0 (+)= g; d1 (+)= g (d1 may be null).
 void grad_split(const void* dy, const void* mask, void* d0, bool acc0, void* d1, bool acc1, int64_t n, int dt,
@@ -96,8 +94,6 @@ void head_forward_loss(const void* x, int dt, const float* W, const float* bias,
 void head_weight_grad(const float* dz, const void* x, int dt, int B, int K, int C, float* dW, float* db,
                       const float* row_loss, float* losses, const int64_t* step, int64_t mask,
                       cudaStream_t st);
-void head_input_grad(const float* dz, const float* W, int B, int K, int C, const void* mask, void* dx,
-                     int dt, bool acc, cudaStream_t st);
 
 // Softmax cross-entropy: losses[*step & mask] <- mean_b CE; dlogits = (softmax - onehot)/B.
 void softmax_ce(const float* logits, const int32_t* labels, int B, int C, float* losses,
@@ -119,7 +115,6 @@ void f32_to_bf16(const float* x, void* y, int64_t n, cudaStream_t st);
 bool vec8_ok(int dt, int64_t n);
 void relu_bwd_x8(const void* y, const void* dy, void* dx, int64_t n, bool acc, cudaStream_t st);
 void add_x8(const void* a, const void* b, void* y, int64_t n, bool relu, cudaStream_t st);
-void copy_acc_x8(const void* x, void* y, int64_t n, bool acc, cudaStream_t st);
 void grad_split_x8(const void* dy, const void* mask, void* d0, bool acc0, void* d1, bool acc1, int64_t n,
                    cudaStream_t st);
 void affine_fwd_x8(const void* x, const float* sc, const float* sh, void* y, int64_t n, int C, bool relu,
@@ -130,10 +125,6 @@ void gelu_bwd_x8(const void* x, const void* dy, void* dx, int64_t n, bool acc, c
 // 128 rows, or sized to the GPU (about two blocks per SM) when `adaptive`.
 int64_t colsum8_partial_floats(int64_t rows, int C, bool adaptive);
 void colsum8(const void* a, int64_t rows, int C, float* partial, float* out, bool adaptive, cudaStream_t st);
-// Affine backward in one pass: dscale = sum dy*x, dshift = sum dy, dx (+)= dy*scale
-// (dx may be null); partial holds 2 * colsum8_partial_floats(rows, C, true) floats.
-void affine_bwd8(const void* dy, const void* x, const float* scale, void* dx, bool acc, int64_t rows, int C,
-                 float* partial, float* dscale, float* dshift, cudaStream_t st);
 // Deferred parameter-gradient reductions, batched into one launch each (at
 // most a few dozen launches' worth of work per call; fixed summation order).
 // ColsumTask: column sums of a bf16 [rows, C] matrix (C % 8 == 0) into
@@ -171,9 +162,6 @@ void layernorm_fwd_x8(const void* x, const float* gamma, const float* beta, void
 // Layernorm backward fused with dgamma / dbeta (C % 256 == 0, C <= 512).
 bool layernorm_bwd8_ok(int dt, int C);
 int64_t layernorm_bwd8_partial_floats(int64_t rows, int C);
-void layernorm_bwd8(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
-                    void* dx, int64_t rows, int C, bool acc, float* partial, float* dgamma, float* dbeta,
-                    cudaStream_t st);
 // The same pass without its finish: partials [layernorm_bwd8_blocks(rows), C]
 // of dgamma and dbeta.
 int layernorm_bwd8_blocks(int64_t rows);

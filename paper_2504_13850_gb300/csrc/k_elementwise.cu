@@ -283,12 +283,6 @@ void grad_split(const void* dy, const void* mask, void* d0, bool acc0, void* d1,
   FO_DISPATCH(dt, T, launch_k(grad_split_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)dy, (const T*)mask,
                               (T*)d0, acc0 ? 1 : 0, (T*)d1, acc1 ? 1 : 0, n));
 }
-template <typename T>
-__global__ void copy_acc_k(const T* x, T* y, int64_t n, int acc) {
-  pdl_wait();
-  pdl_trigger();
-  GRID_STRIDE(i, n) store(y, i, to_f(x[i]), acc);
-}
 void affine_fwd(const void* x, const float* scale, const float* shift, void* y, int64_t rows,
                 int C, int dt, bool relu, cudaStream_t st) {
   int64_t n = rows * C;
@@ -303,10 +297,6 @@ void affine_dx(const void* dy, const float* scale, void* dx, int64_t rows, int C
 void add_fwd(const void* a, const void* b, void* y, int64_t n, int dt, bool relu, cudaStream_t st) {
   if (vec8_ok(dt, n)) return add_x8(a, b, y, n, relu, st);
   FO_DISPATCH(dt, T, launch_k(add_fwd_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)a, (const T*)b, (T*)y, n, relu));
-}
-void copy_or_acc(const void* x, void* y, int64_t n, int dt, bool acc, cudaStream_t st) {
-  if (vec8_ok(dt, n)) return copy_acc_x8(x, y, n, acc, st);
-  FO_DISPATCH(dt, T, launch_k(copy_acc_k<T>, elementwise_blocks(n, 256), 256, 0, st, (const T*)x, (T*)y, n, acc));
 }
 
 // -------------------------------------------------------------- avgpool

@@ -6,7 +6,6 @@
 //                 ReLU mask (mask > 0) when one is given
 //   head_wgrad  : dW = dz^T x, db = sum_b dz, loss = mean of the row losses
 //                 (summed in row order, deterministic)
-//   head_dgrad  : dx (+)= dz W as a launch of its own (the same arithmetic)
 // W and b are the fp32 master weights; dz and the gradients are fp32.
 #include "fo_common.cuh"
 #include "fo_kernels.h"
@@ -128,23 +127,6 @@ __global__ void head_wgrad_k(const float* __restrict__ dz, const T* __restrict__
   }
 }
 
-// dx[b][k] (+)= (sum_c dz[b][c] W[c][k]) * (mask[b][k] > 0); grid (ceil(K/256), B).
-template <typename T>
-__global__ void head_dgrad_k(const float* __restrict__ dz, const float* __restrict__ W, int B, int K, int C,
-                             const T* __restrict__ mask, T* __restrict__ dx, int acc) {
-  pdl_wait();
-  pdl_trigger();
-  const int b = blockIdx.y;
-  const int k = blockIdx.x * blockDim.x + threadIdx.x;
-  if (k >= K) return;
-  float s = 0.f;
-  for (int c = 0; c < C; ++c) s = fmaf(dz[int64_t(b) * C + c], W[int64_t(c) * K + k], s);
-  const int64_t i = int64_t(b) * K + k;
-  if (mask && !(to_f(mask[i]) > 0.f)) s = 0.f;
-  if (acc) s += to_f(dx[i]);
-  dx[i] = from_f<T>(s);
-}
-
 }  // namespace
 
 void head_forward_loss(const void* x, int dt, const float* W, const float* bias, const int32_t* labels, int B,
@@ -167,15 +149,6 @@ void head_weight_grad(const float* dz, const void* x, int dt, int B, int K, int 
     launch_k(head_wgrad_k<float>, grid, 256, 0, st, dz, (const float*)x, B, K, C, dW, db, row_loss, losses, step, mask);
   else
     launch_k(head_wgrad_k<bf16>, grid, 256, 0, st, dz, (const bf16*)x, B, K, C, dW, db, row_loss, losses, step, mask);
-}
-
-void head_input_grad(const float* dz, const float* W, int B, int K, int C, const void* mask, void* dx, int dt,
-                     bool acc, cudaStream_t st) {
-  dim3 grid(ceil_div(K, 256), B);
-  if (dt == kF32)
-    launch_k(head_dgrad_k<float>, grid, 256, 0, st, dz, W, B, K, C, (const float*)mask, (float*)dx, acc ? 1 : 0);
-  else
-    launch_k(head_dgrad_k<bf16>, grid, 256, 0, st, dz, W, B, K, C, (const bf16*)mask, (bf16*)dx, acc ? 1 : 0);
 }
 
 }  // namespace fo

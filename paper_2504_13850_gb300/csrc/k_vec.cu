@@ -107,22 +107,6 @@ __global__ void grad_split_x8_k(const bf16* __restrict__ dy, const bf16* __restr
   }
 }
 
-__global__ void copy_acc_x8_k(const bf16* __restrict__ x, bf16* __restrict__ y, int64_t n8, int acc) {
-  pdl_wait();
-  pdl_trigger();
-  GRID_STRIDE8(i, n8) {
-    if (!acc) {
-      *reinterpret_cast<uint4*>(y + 8 * i) = *reinterpret_cast<const uint4*>(x + 8 * i);
-    } else {
-      const V8 p = ld8(x + 8 * i), q = ld8(y + 8 * i);
-      V8 o;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) o.v[j] = p.v[j] + q.v[j];
-      st8(y + 8 * i, o);
-    }
-  }
-}
-
 __global__ void affine_fwd_x8_k(const bf16* __restrict__ x, const float* __restrict__ sc,
                                 const float* __restrict__ sh, bf16* __restrict__ y, int64_t n8, int C, int relu) {
   pdl_wait();
@@ -571,9 +555,6 @@ void grad_split_x8(const void* dy, const void* mask, void* d0, bool acc0, void* 
   launch_k(grad_split_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)dy, (const bf16*)mask, (bf16*)d0,
            acc0 ? 1 : 0, (bf16*)d1, acc1 ? 1 : 0, n / 8);
 }
-void copy_acc_x8(const void* x, void* y, int64_t n, bool acc, cudaStream_t st) {
-  launch_k(copy_acc_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)x, (bf16*)y, n / 8, acc);
-}
 void affine_fwd_x8(const void* x, const float* sc, const float* sh, void* y, int64_t n, int C, bool relu,
                    cudaStream_t st) {
   launch_k(affine_fwd_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)x, sc, sh, (bf16*)y, n / 8, C, relu);
@@ -599,17 +580,6 @@ void colsum8(const void* a, int64_t rows, int C, float* partial, float* out, boo
   dim3 grid(ceil_div(C, 256), chunks_of(rows, ch));
   launch_k(colsum8_k<0>, grid, 256, 0, st, (const bf16*)a, nullptr, nullptr, nullptr, 0, rows, C, ch, partial, nullptr, nullptr);
   launch_k(finish_k, ceil_div(C, 32), 256, 0, st, partial, chunks_of(rows, ch), C, out);
-}
-
-void affine_bwd8(const void* dy, const void* x, const float* scale, void* dx, bool acc, int64_t rows, int C,
-                 float* partial, float* dscale, float* dshift, cudaStream_t st) {
-  const int ch = adaptive_chunk(rows, C);
-  dim3 grid(ceil_div(C, 256), chunks_of(rows, ch));
-  float* p1 = partial + colsum8_partial_floats(rows, C, true);
-  launch_k(colsum8_k<1>, grid, 256, 0, st, (const bf16*)dy, (const bf16*)x, scale, (bf16*)dx, acc, rows, C, ch, partial,
-                                     p1, nullptr);
-  launch_k(finish_k, ceil_div(C, 32), 256, 0, st, partial, chunks_of(rows, ch), C, dscale);
-  launch_k(finish_k, ceil_div(C, 32), 256, 0, st, p1, chunks_of(rows, ch), C, dshift);
 }
 
 int affine_bwd8_chunks(int64_t rows, int C) { return chunks_of(rows, adaptive_chunk(rows, C)); }
@@ -686,16 +656,5 @@ void layernorm_bwd8_pass(const void* x, const float* gamma, const float* mean, c
 }
 
 int64_t layernorm_bwd8_partial_floats(int64_t rows, int C) { return 2 * ((rows + 15) / 16) * C; }
-
-void layernorm_bwd8(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
-                    void* dx, int64_t rows, int C, bool acc, float* partial, float* dgamma, float* dbeta,
-                    cudaStream_t st) {
-  const int blocks = int((rows + 15) / 16);
-  float* pb = partial + int64_t(blocks) * C;
-  launch_k(layernorm_bwd_fused_k, blocks, 256, 0, st, (const bf16*)x, gamma, mean, rstd, (const bf16*)dy, (bf16*)dx, rows,
-                                                C, acc, partial, pb);
-  launch_k(finish_k, ceil_div(C, 32), 256, 0, st, partial, blocks, C, dgamma);
-  launch_k(finish_k, ceil_div(C, 32), 256, 0, st, pb, blocks, C, dbeta);
-}
 
 }  // namespace fo
