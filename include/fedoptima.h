@@ -127,7 +127,9 @@ typedef struct fo_server fo_server;
  * intermediate tensors for one batch.  Parameters start at zero: load them
  * with fo_server_set_params.  Returns FO_ERR_UNSUPPORTED for layer shapes
  * without a kernel (e.g. bf16 conv channels not a multiple of 64), FO_ERR_ARG
- * for K or omega above FO_MAX_DEVICES / FO_MAX_OMEGA, FO_ERR_OOM when a
+ * for K or omega above FO_MAX_DEVICES / FO_MAX_OMEGA, for an op list whose
+ * shapes do not chain, or for any tensor of more than 2^31 - 1 elements per
+ * sample (all checked on the host before any CUDA call), FO_ERR_OOM when a
  * device or host allocation fails. */
 FO_API int fo_server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt,
                      const fo_server_cfg* cfg, fo_server** out);

@@ -161,6 +161,8 @@ int infer(fo_server* s) {
       default:
         return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": unknown kind");
     }
+    if (int64_t(o.H) * o.W * o.C > INT32_MAX)
+      return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": more than 2^31 - 1 elements per sample");
     s->T[i + 1] = o;
     s->T[op.in0].consumers++;
     if (op.kind == FO_OP_ADD || op.kind == FO_OP_CHMUL) s->T[op.in1].consumers++;
@@ -1123,6 +1125,8 @@ static int server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt, c
       (c.dtype != FO_DTYPE_F32 && c.dtype != FO_DTYPE_BF16) || c.max_delay < 0 ||
       (c.sched_policy != FO_SCHED_COUNTER && c.sched_policy != FO_SCHED_FIFO))
     return set_err(FO_ERR_ARG, "bad server configuration");
+  if (int64_t(c.in_h) * c.in_w * c.in_c > INT32_MAX)
+    return set_err(FO_ERR_ARG, "more than 2^31 - 1 activation elements per sample");
   fo_server* s = new (std::nothrow) fo_server();
   if (!s) return set_err(FO_ERR_OOM, "host allocation");
   *held = s;
