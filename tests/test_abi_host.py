@@ -53,6 +53,12 @@ def test_scheduler_matches_golden_trace():
                 assert s.counters() == [int(v) for v in p[5:9]]
 
 
+def test_scheduler_matches_slot_reuse_golden():
+    from test_oracle_sched_agg import replay_slot_reuse_golden
+    s = api.Scheduler(3, 3, 2)
+    replay_slot_reuse_golden(lambda k: s.put(k)[:2], s.get, s.counters, s.sender_status)
+
+
 @pytest.mark.parametrize("policy", ["counter", "fifo"])
 @pytest.mark.parametrize("seed", range(12))
 def test_scheduler_matches_oracle_on_random_traces(seed, policy):

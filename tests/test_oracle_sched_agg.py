@@ -39,6 +39,29 @@ def test_tiny_schedule_matches_hand_derived_golden():
             assert s.c == [int(v) for v in f[5:9]]
 
 
+def replay_slot_reuse_golden(put, get, counters, sender_on):
+    """Replays tests/golden/sched_slot_reuse.txt (3 devices, depth 2, omega 3)
+    through the given put / get and state readers."""
+    for f in golden_lines("sched_slot_reuse.txt"):
+        if f[0] == "enqueue":
+            k = int(f[1])
+            st, slot = put(k)
+            assert (st, slot, int(sender_on()[k])) == (NAMES[f[3]], int(f[4]), int(f[5])), f
+        else:
+            st, k, slot = get()
+            assert (st, k, slot) == (NAMES[f[2]], int(f[3]), int(f[4])), f
+            assert list(counters()) == [int(v) for v in f[5:8]], f
+            assert [int(v) for v in sender_on()] == [int(v) for v in f[9:12]], f
+
+
+def test_slot_reuse_matches_hand_derived_golden():
+    """Freed slots are reused in the order they were freed, a device refused
+    with an empty queue is turned on by the next dequeue, and one refused
+    with a non-empty queue only by a dequeue of its own."""
+    s = O.TaskScheduler(K=3, omega=3, depth=2)
+    replay_slot_reuse_golden(s.put, s.get, lambda: s.c, lambda: s.on)
+
+
 def test_backlogged_queues_are_served_round_robin():
     K = 7
     s = O.TaskScheduler(K, omega=K * 3, depth=3)
