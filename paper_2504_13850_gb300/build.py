@@ -1,8 +1,14 @@
 """Build the C-ABI shared library libfedoptima.so in-tree with nvcc for
-sm_103a (GB300).  Sources compile in parallel; objects go to _build/."""
+sm_103a (GB300).  Sources compile in parallel; objects go to _build/.
+
+Several processes may call build() at once (one per rank under torchrun):
+an exclusive file lock serialises them, and every object and the library
+are written under a temporary name and renamed into place, so a process
+never loads a half-written library."""
 from __future__ import annotations
 
 import concurrent.futures as cf
+import fcntl
 import os
 import shutil
 import subprocess
@@ -33,28 +39,38 @@ def _compile(src, extra):
     deps.append(os.path.join(HERE, "..", "include", "fedoptima.h"))
     if os.path.exists(obj) and all(os.path.getmtime(obj) >= os.path.getmtime(d) for d in deps):
         return obj, ""
-    cmd = [nvcc(), *ARCH, *FLAGS, *extra, "-c", srcp, "-o", obj]
+    tmp = f"{obj}.{os.getpid()}.tmp"
+    cmd = [nvcc(), *ARCH, *FLAGS, *extra, "-c", srcp, "-o", tmp]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
+        if os.path.exists(tmp):
+            os.remove(tmp)
         raise RuntimeError(f"nvcc failed for {src}:\n{r.stdout}\n{r.stderr}")
+    os.replace(tmp, obj)
     return obj, r.stderr
 
 
 def build(verbose=False, extra=()):
     os.makedirs(BUILD, exist_ok=True)
-    with cf.ThreadPoolExecutor(max_workers=min(len(SOURCES), os.cpu_count() or 4)) as ex:
-        results = list(ex.map(lambda s: _compile(s, list(extra)), SOURCES))
-    objs = [o for o, _ in results]
-    if verbose:
-        for _, log in results:
-            if log:
-                sys.stderr.write(log)
-    newest = max(os.path.getmtime(o) for o in objs)
-    if not os.path.exists(OUT) or os.path.getmtime(OUT) < newest:
-        cmd = [nvcc(), *ARCH, "-shared", "-o", OUT, *objs]
-        r = subprocess.run(cmd, capture_output=True, text=True)
-        if r.returncode != 0:
-            raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
+    with open(os.path.join(BUILD, ".lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)      # released when the file closes
+        with cf.ThreadPoolExecutor(max_workers=min(len(SOURCES), os.cpu_count() or 4)) as ex:
+            results = list(ex.map(lambda s: _compile(s, list(extra)), SOURCES))
+        objs = [o for o, _ in results]
+        if verbose:
+            for _, log in results:
+                if log:
+                    sys.stderr.write(log)
+        newest = max(os.path.getmtime(o) for o in objs)
+        if not os.path.exists(OUT) or os.path.getmtime(OUT) < newest:
+            tmp = f"{OUT}.{os.getpid()}.tmp"
+            cmd = [nvcc(), *ARCH, "-shared", "-o", tmp, *objs]
+            r = subprocess.run(cmd, capture_output=True, text=True)
+            if r.returncode != 0:
+                if os.path.exists(tmp):
+                    os.remove(tmp)
+                raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
+            os.replace(tmp, OUT)
     return OUT
 
 
