@@ -191,6 +191,25 @@ def oracle_samples_per_s(cfg, n_steps, batch):
     return n_steps * batch / dt, dt
 
 
+def oracle_sample(cfg, batch, seconds=12.0, min_steps=2, max_steps=50):
+    """The oracle timed over whole server steps at `batch` samples each,
+    until about `seconds` of CPU work have run (at least `min_steps`).
+    Returns (samples/s, steps, elapsed seconds)."""
+    import numpy as np
+    from oracle import fo_oracle as O
+    from paper_2504_13850_gb300 import workloads as W
+    theta = W.init_params(cfg).astype(np.float64)
+    v = np.zeros_like(theta)
+    dt, j = 0.0, 0
+    while j < max_steps and (j < min_steps or dt < seconds):
+        x, _, y, ln = W.device_batch(cfg, j % cfg["K"], j, batch=batch)
+        t0 = time.perf_counter()
+        _, theta, v, _ = O.server_step(cfg["ops"], theta, v, x, y, ln, cfg["lr"], cfg["momentum"])
+        dt += time.perf_counter() - t0
+        j += 1
+    return j * batch / dt, j, dt
+
+
 def run_reference(args):
     world, rank, _ = dist_setup(0)
     if rank != 0:
@@ -426,10 +445,10 @@ def run_ours(args):
     tensor_frac = step_flops / (step_ms / 1e3) / 1e12 / pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
     tensor_frac_burst = step_flops / (step_ms / 1e3) / 1e12 / pk["bf16_tflops"]
     cpu = None
-    if not args.no_cpu_baseline:
-        v_cpu, dt_cpu = oracle_samples_per_s(cfg, 2, B)
+    if not args.no_cpu_baseline and world == 1:
+        v_cpu, n_cpu, dt_cpu = oracle_sample(cfg, B)
         cpu = {"value": round(v_cpu, 3), "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-               "sample": f"2 oracle server steps at batch {B} ({dt_cpu:.1f} s, numpy fp64, BLAS threads = cores)"}
+               "sample": f"{n_cpu} oracle server steps at batch {B} ({dt_cpu:.1f} s, numpy fp64, BLAS threads = cores)"}
     from paper_2504_13850_gb300 import study
     sched = study.scheduler_balance("scale", uploads=6000)   # host-only: counter vs FIFO scheduling
     wsb = srv.device_bytes()

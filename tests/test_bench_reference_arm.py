@@ -66,3 +66,18 @@ def test_reference_arm_under_two_ranks_prints_once():
     lines = json_lines(r.stdout)
     assert len(lines) == 1
     check_line(lines[0], 2)
+
+
+def test_cpu_baseline_sample_runs_until_its_time_budget():
+    """The GPU arm's `cpu_baseline` times whole oracle steps until about the
+    requested seconds of CPU work have run (at least two steps)."""
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2504_13850_gb300 import workloads as W
+    cfg = W.CONFIGS["tiny"]
+    v, n, dt = bench.oracle_sample(cfg, cfg["batch"], seconds=0.3)
+    assert n >= 2 and dt >= 0.3 and v == pytest.approx(n * cfg["batch"] / dt)
+    v, n, dt = bench.oracle_sample(cfg, 4, seconds=0.0)
+    assert n == 2 and v > 0
+    v, n, dt = bench.oracle_sample(cfg, 4, seconds=1e9, max_steps=3)
+    assert n == 3
