@@ -53,7 +53,10 @@ def _compile(src, extra):
 def build(verbose=False, extra=()):
     os.makedirs(BUILD, exist_ok=True)
     with open(os.path.join(BUILD, ".lock"), "w") as lock:
-        fcntl.flock(lock, fcntl.LOCK_EX)      # released when the file closes
+        try:
+            fcntl.flock(lock, fcntl.LOCK_EX)  # released when the file closes
+        except OSError:                       # a filesystem without locks: build unserialised
+            pass
         with cf.ThreadPoolExecutor(max_workers=min(len(SOURCES), os.cpu_count() or 4)) as ex:
             results = list(ex.map(lambda s: _compile(s, list(extra)), SOURCES))
         objs = [o for o, _ in results]
