@@ -14,6 +14,7 @@ import pytest
 from oracle import fo_oracle as O
 
 import test_oracle_layers as TL          # noqa: E402  (tests/ is on sys.path under pytest)
+import test_oracle_network as TN         # noqa: E402
 import test_oracle_mobile as TM          # noqa: E402
 import test_oracle_sched_agg as TS       # noqa: E402
 import test_preproc as TP                # noqa: E402
@@ -293,6 +294,24 @@ def split_fastest_device(Oflop, S, b, o, allowed=None):
     return best_l, best_cost
 
 
+def source_mutant(fn, old, new):
+    """`fn` with one expression of its source replaced, compiled against
+    the oracle's own globals (for mistakes inside the network wiring)."""
+    import inspect
+    import textwrap
+    src = textwrap.dedent(inspect.getsource(fn))
+    assert src.count(old) == 1, old
+    scope = dict(vars(O))
+    exec(compile(src.replace(old, new), f"<mutant of {fn.__name__}>", "exec"), scope)
+    return scope[fn.__name__]
+
+
+backward_residual_dropped = source_mutant(O.backward, 'acc(op["in1"], dy)', "None")
+backward_overwrites = source_mutant(O.backward, "G[tid] = rnd(G[tid] + g) if tid in G else rnd(g)", "G[tid] = rnd(g)")
+forward_flatten_nchw = source_mutant(O.forward, "y = a.reshape(a.shape[0], -1)",
+                                     "y = a.transpose(0, 3, 1, 2).reshape(a.shape[0], -1)")
+
+
 # --------------------------------------------------------------------------
 # the table: mistake -> (patches, pins expected to catch it)
 # --------------------------------------------------------------------------
@@ -381,6 +400,14 @@ MUTATIONS = {
         {"TaskScheduler.put": put_cap_off_by_one},
         [(TS.test_tiny_schedule_matches_hand_derived_golden, ())]
         + [(TS.test_random_traces_keep_invariants_and_pick_min_counter, (s,)) for s in range(4)]),
+    "network backward: the residual branch gets no gradient": (
+        {"backward": backward_residual_dropped},
+        [(TN.test_network_matches_torch_autograd, ("resnet",)), (TN.test_network_finite_differences, ("resnet",))]),
+    "network backward: a second gradient contribution overwrites the first": (
+        {"backward": backward_overwrites},
+        [(TN.test_network_matches_torch_autograd, ("resnet",)), (TN.test_network_matches_torch_autograd, ("mobilenet",))]),
+    "network forward: flatten in channel-first order": (
+        {"forward": forward_flatten_nchw}, [(TN.test_network_matches_torch_autograd, ("vgg",))]),
     "split selection: training and transfer added, not overlapped": (
         {"split_point": split_sum_not_max}, golden_split_cases()),
     "split selection: the fastest device decides": (
