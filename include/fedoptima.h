@@ -135,14 +135,18 @@ FO_API int fo_server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt
                      const fo_server_cfg* cfg, fo_server** out);
 FO_API int fo_server_destroy(fo_server* s);
 
-/* Number of parameters of M_s (length of the flat vector below). */
+/* Number of parameters of M_s, the server-side model of Sec. 3.2 (length of
+ * the flat vector below); -1 for a NULL handle. */
 FO_API int64_t fo_server_num_params(const fo_server* s);
 
-/* Flat parameter / momentum vectors, fp32, in op order: conv W[cout][k][k][cin]
- * then b; linear W[cout][cin] then b; affine scale then shift; layernorm gamma
- * then beta.  `host` is host memory of n floats; n must equal
- * fo_server_num_params.  set_* also refreshes the bf16 shadow; get_* waits
- * for pending steps. */
+/* theta_s, the single server model that every training iteration of
+ * Algorithm 4 updates whichever device's activations it takes (Sec. 3.3.2),
+ * and its SGD momentum.
+ * Flat fp32 vectors in op order: conv W[cout][k][k][cin] then b; linear
+ * W[cout][cin] then b; affine scale then shift; layernorm gamma then beta.
+ * `host` is host memory of n floats owned by the caller; n must equal
+ * fo_server_num_params, else FO_ERR_ARG.  set_* also refreshes the bf16
+ * shadow; every call waits for pending steps first. */
 FO_API int fo_server_set_params(fo_server* s, const float* host, int64_t n);
 FO_API int fo_server_get_params(fo_server* s, float* host, int64_t n);
 FO_API int fo_server_set_momentum(fo_server* s, const float* host, int64_t n);
@@ -167,8 +171,10 @@ FO_API int fo_server_get_momentum(fo_server* s, float* host, int64_t n);
 FO_API int fo_server_tensor(const fo_server* s, int index, const void** data, int64_t* dims4, int* dtype);
 FO_API int fo_server_params_device(fo_server* s, float** theta, int64_t* n);
 FO_API int fo_server_load_params_device(fo_server* s, const float* src, int64_t n);
-/* The reverse copy: the parameters (padded layout, *n floats) into device
- * memory `dst`, ordered on the server's stream. */
+/* The reverse copy (Alg. 1: a device pulls the global model): the
+ * parameters (padded layout, n floats) into caller-owned device memory
+ * `dst`, ordered on the server's stream.  FO_ERR_ARG when n differs from
+ * the padded length. */
 FO_API int fo_server_store_params_device(fo_server* s, float* dst, int64_t n);
 
 /* Task Scheduler put() for an activation message (Algorithm 2) plus the
@@ -198,10 +204,12 @@ FO_API int fo_enqueue_activations(fo_server* s, int device_id, const void* acts,
  * FO_EMPTY when every queue is empty (nothing changes). */
 FO_API int fo_server_step(fo_server* s, int* device_used, int32_t* slot_used);
 
-/* Copy the losses of steps [first_step, first_step + n) to host memory.
- * Waits for those steps only (work enqueued after them keeps running), so a
- * caller can read step i's loss while step i + 1 executes.  Only the most
- * recent 2^20 steps are kept. */
+/* The server loss f_s of training iterations [first_step, first_step + n)
+ * of Algorithm 4 (softmax cross-entropy, batch mean), copied to caller-owned
+ * host memory of n floats.  Waits for those steps only (work enqueued after
+ * them keeps running), so a caller can read step i's loss while step i + 1
+ * executes.  Only the most recent 2^20 steps are kept: FO_ERR_ARG for a
+ * range not yet run or older than that. */
 FO_API int fo_read_losses(fo_server* s, float* host_out, int64_t first_step, int64_t n);
 
 /* FedAsync aggregation (Algorithm 4, aggregation branch).  `global`
@@ -216,35 +224,50 @@ FO_API int fo_read_losses(fo_server* s, float* host_out, int64_t first_step, int
 FO_API int fo_aggregate(fo_server* s, float* global, const float* local, int64_t n,
                  int device_id, int32_t version, int32_t* new_version);
 
-/* Scheduler state. */
-FO_API int fo_get_counters(const fo_server* s, uint64_t* c_host /* K */);
-FO_API int fo_get_sender_status(const fo_server* s, uint8_t* on_host /* K */);
-FO_API int fo_get_version(const fo_server* s, int32_t* t, int32_t* round /* t / K */);
+/* Scheduler state, copied to caller-owned host arrays of K entries: the
+ * consumption counters c_k of Algorithm 3, and the Sender Status of each
+ * device (1 = on, Sec. 3.4.1).  fo_get_version: the global device-model
+ * version t of Algorithm 4 and the completed rounds t / K (either pointer
+ * may be NULL).  FO_ERR_ARG for a NULL handle or array. */
+FO_API int fo_get_counters(const fo_server* s, uint64_t* c_host);
+FO_API int fo_get_sender_status(const fo_server* s, uint8_t* on_host);
+FO_API int fo_get_version(const fo_server* s, int32_t* t, int32_t* round);
 /* Device leaving (active = 0: further uploads are refused, its queued
  * batches are still consumed) or (re)joining (active = 1: c_k becomes
  * max(c_k, min over the other active devices), Sender on) — Sec. 3.4.2. */
 FO_API int fo_set_device_active(fo_server* s, int device_id, int active);
 
-/* Bytes of the activation slab (omega slots, acts + labels + lengths). */
+/* Bytes of the activation slab, omega slots of acts + labels + lengths: the
+ * omega * mu_act term of Eq. 3, independent of K.  -1 for a NULL handle.
+ * The helpers from here to fo_server_kernel_times have no counterpart in
+ * the paper: they expose memory, streams and timing to the caller. */
 FO_API int64_t fo_server_activation_bytes(const fo_server* s);
-/* Wait for all work the server has enqueued. */
+/* Wait for all work the server has enqueued (uploads, steps,
+ * aggregations); no counterpart in the paper.  FO_ERR_CUDA if any of it
+ * failed. */
 FO_API int fo_server_synchronize(fo_server* s);
 /* The compute stream (a cudaStream_t) the step and aggregation kernels run
- * on, for callers that time them with CUDA events. */
+ * on, for callers that time them with CUDA events; no counterpart in the
+ * paper.  NULL for a NULL handle. */
 FO_API void* fo_server_stream(const fo_server* s);
 /* Kernel launches the last fo_server_step enqueued, and all kernels the
- * server has launched since creation (steps and aggregations). */
+ * server has launched since creation (steps and aggregations); no
+ * counterpart in the paper.  -1 for a NULL handle. */
 FO_API int fo_server_last_step_launches(const fo_server* s);
 FO_API int64_t fo_server_kernels_launched(const fo_server* s);
 /* Device bytes the server allocated (parameters, momentum, gradient, bf16
- * shadow, activation slab, intermediate tensors, scratch). */
+ * shadow, activation slab, intermediate tensors, scratch): the whole of Eq.
+ * 3's mu_model + omega * mu_act plus this implementation's buffers.  -1 for
+ * a NULL handle. */
 FO_API int64_t fo_server_device_bytes(const fo_server* s);
 /* Waits for the compute stream and reports FO_ERR_TIMEOUT if a tensor-core
- * kernel gave up a bounded wait since creation (FO_OK otherwise). */
+ * kernel gave up a bounded wait since creation (FO_OK otherwise); no
+ * counterpart in the paper. */
 FO_API int fo_server_error(fo_server* s);
 
-/* Optional per-kernel timing of fo_server_step and fo_aggregate: when
- * enabled, each launch is bracketed by CUDA events on the compute stream.
+/* Optional per-kernel timing of fo_server_step and fo_aggregate (no
+ * counterpart in the paper): when enabled, each launch is bracketed by CUDA
+ * events on the compute stream.
  * fo_server_kernel_times fills up to `cap` entries (any output array may be
  * NULL) with the name (static string), kernel launches, summed milliseconds
  * and summed algorithmic FLOPs and HBM bytes of every kernel class seen since
@@ -255,6 +278,9 @@ FO_API int fo_server_profile_reset(fo_server* s);
 FO_API int fo_server_kernel_times(fo_server* s, const char** names, int64_t* launches,
                            double* ms, double* flops, double* bytes, int cap, int* n_out);
 
+/* The message of the last error returned on the calling thread (empty
+ * when there is none; no counterpart in the paper); a buffer valid until the
+ * thread's next call into the library. */
 FO_API const char* fo_last_error(void);
 
 /* ------------------------------------------------------------------------
@@ -276,18 +302,21 @@ FO_API int fo_sched_sender_status(const fo_sched* s, uint8_t* on_host);
 FO_API int fo_sched_queued(const fo_sched* s, int k); /* |Q_k|, or the total when k < 0 */
 
 /* ------------------------------------------------------------------------
- * Standalone FedAsync update on caller buffers, for bandwidth sweeps:
- * global <- fmaf(alpha, local - global, global) over n fp32 elements on
- * `stream` (a cudaStream_t, NULL = default).  global and local are device
- * pointers; alpha in (0, 1].  No version bookkeeping.
+ * Standalone FedAsync update on caller buffers (the arithmetic of Algorithm
+ * 4's aggregation branch without its version bookkeeping), for bandwidth
+ * sweeps: global <- fmaf(alpha, local - global, global) over n fp32 elements
+ * on `stream` (a cudaStream_t, NULL = default).  global (updated in place)
+ * and local (read only) are caller-owned device pointers; alpha in (0, 1].
+ * FO_ERR_ARG for a NULL pointer, n < 0 or alpha outside (0, 1].
  * ---------------------------------------------------------------------- */
 FO_API int fo_axpby_async(float* global, const float* local, int64_t n, float alpha,
                    void* stream);
 
 /* ------------------------------------------------------------------------
  * Deterministic column sums out[c] = sum_r x[r][c] of a row-major
- * [rows][cols] matrix: the reduction the server uses for bias gradients
- * (the sum over all positions of a layer's output gradient).  x is a device
+ * [rows][cols] matrix: the reduction the server uses for bias gradients in
+ * the backward pass of Algorithm 4 (the sum over all positions of a layer's
+ * output gradient).  x is a device
  * pointer to fp32 (dtype FO_DTYPE_F32) or bf16 (FO_DTYPE_BF16) values, out a
  * device pointer to `cols` floats; partial sums over 128-row chunks are added
  * in a fixed order, so results are bitwise reproducible.  The partial sums
