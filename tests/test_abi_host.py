@@ -144,3 +144,28 @@ def test_scheduler_size_limits_and_depth_above_omega():
         else:
             assert a.get() == o.get()
         assert a.counters() == o.c
+
+
+def test_every_entry_point_cites_its_passage_or_says_it_has_none():
+    """Each FO_API declaration follows a comment block that cites the
+    paper's section, algorithm, equation or table defining the operation,
+    or states that the paper has no counterpart."""
+    with open(os.path.join(ROOT, "include", "fedoptima.h")) as f:
+        lines = f.read().split("\n")
+    blocks, cur = [], None
+    for i, line in enumerate(lines):
+        if "/*" in line:
+            cur = [line]
+        elif cur is not None:
+            cur.append(line)
+        if cur is not None and "*/" in line:
+            blocks.append((i, "\n".join(cur)))
+            cur = None
+    cite = re.compile(r"Sec\.|Alg|Eqs?\.|Table|no\s+(\*\s+)?counterpart|paper has no")
+    missing = []
+    for i, line in enumerate(lines):
+        if line.startswith("FO_API"):
+            before = [b for b in blocks if b[0] < i]
+            if not before or not cite.search(before[-1][1]):
+                missing.append(re.search(r"(fo_\w+)\s*\(", line).group(1))
+    assert not missing, missing
