@@ -308,6 +308,15 @@ def source_mutant(fn, old, new):
 
 backward_residual_dropped = source_mutant(O.backward, 'acc(op["in1"], dy)', "None")
 backward_overwrites = source_mutant(O.backward, "G[tid] = rnd(G[tid] + g) if tid in G else rnd(g)", "G[tid] = rnd(g)")
+param_shapes_bias_first = source_mutant(
+    O.param_shapes,
+    """            out.append((i, "W", (op["cout"], op["k"], op["k"], op["cin"])))
+            if op["bias"]:
+                out.append((i, "b", (op["cout"],)))""",
+    """            if op["bias"]:
+                out.append((i, "b", (op["cout"],)))
+            out.append((i, "W", (op["cout"], op["k"], op["k"], op["cin"])))""")
+server_trains_highest_slot = source_mutant(O.Server.step, "self.slots.pop(slot)", "self.slots.pop(max(self.slots))")
 forward_flatten_nchw = source_mutant(O.forward, "y = a.reshape(a.shape[0], -1)",
                                      "y = a.transpose(0, 3, 1, 2).reshape(a.shape[0], -1)")
 
@@ -408,6 +417,10 @@ MUTATIONS = {
         [(TN.test_network_matches_torch_autograd, ("resnet",)), (TN.test_network_matches_torch_autograd, ("mobilenet",))]),
     "network forward: flatten in channel-first order": (
         {"forward": forward_flatten_nchw}, [(TN.test_network_matches_torch_autograd, ("vgg",))]),
+    "flat layout: conv bias before its weights": (
+        {"param_shapes": param_shapes_bias_first}, [(TN.test_flat_layout_is_the_documented_order, ())]),
+    "event replay: a step trains on the highest-numbered slot, not the served one": (
+        {"Server.step": server_trains_highest_slot}, [(TN.test_server_trains_on_the_batch_the_scheduler_served, ())]),
     "split selection: training and transfer added, not overlapped": (
         {"split_point": split_sum_not_max}, golden_split_cases()),
     "split selection: the fastest device decides": (

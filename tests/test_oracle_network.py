@@ -188,3 +188,66 @@ def test_param_layout_matches_workload_counts():
     assert W.num_params(W.CONFIGS["resnet"]["ops"]) == 10_544_740
     assert W.num_params(W.CONFIGS["transformer"]["ops"]) == 12_611_586
     assert W.num_params(W.CONFIGS["tiny"]["ops"]) == 59_466
+
+
+def test_flat_layout_is_the_documented_order():
+    """The flat parameter order the C header documents, written out by hand
+    for one op of every parameterised kind: conv W[cout][k][k][cin] then b;
+    affine scale then shift; depthwise W[c][k][k] then b; layernorm gamma
+    then beta; linear W[cout][cin] then b; ops without a bias have none."""
+    ops = [{"kind": "conv", "in0": 0, "cin": 2, "cout": 3, "k": 3, "stride": 1, "bias": 1},
+           {"kind": "affine", "in0": 1, "c": 3},
+           {"kind": "dwconv", "in0": 2, "c": 3, "k": 5, "stride": 1, "bias": 1},
+           {"kind": "conv", "in0": 3, "cin": 3, "cout": 4, "k": 1, "stride": 1, "bias": 0},
+           {"kind": "relu", "in0": 4},
+           {"kind": "layernorm", "in0": 5, "c": 4},
+           {"kind": "flatten", "in0": 6},
+           {"kind": "linear", "in0": 7, "cin": 4, "cout": 2, "bias": 1}]
+    assert O.param_shapes(ops) == [
+        (0, "W", (3, 3, 3, 2)), (0, "b", (3,)),
+        (1, "scale", (3,)), (1, "shift", (3,)),
+        (2, "W", (3, 5, 5)), (2, "b", (3,)),
+        (3, "W", (4, 1, 1, 3)),
+        (5, "gamma", (4,)), (5, "beta", (4,)),
+        (7, "W", (2, 4)), (7, "b", (2,))]
+    flat = np.arange(54 + 3 + 6 + 75 + 3 + 12 + 8 + 8 + 2, dtype=np.float64)
+    p = O.unflatten(ops, flat)
+    assert p[(0, "b")].tolist() == [54.0, 55.0, 56.0]
+    assert p[(0, "W")][1, 0, 2, 1] == 1 * 18 + 0 * 6 + 2 * 2 + 1
+    assert np.array_equal(O.flatten(ops, p), flat)
+
+
+def test_server_trains_on_the_batch_the_scheduler_served():
+    """The event-replay server trains each step on the oldest queued batch
+    of the device the scheduler picked (FIFO within a device), from the
+    parameters the previous step left."""
+    ops = small_vgg()
+    r = np.random.default_rng(11)
+    theta0 = O.flatten(ops, {k: 0.3 * r.standard_normal(s) for k, s in
+                             (((i, n), s) for i, n, s in O.param_shapes(ops))})
+    K, lr, mu = 3, 0.01, 0.9
+    srv = O.Server(ops, K, omega=5, depth=2, theta0=theta0, lr=lr, mu=mu)
+    sent = {k: [] for k in range(K)}
+
+    def upload(k):
+        x = np.maximum(r.standard_normal((2, 8, 8, 4)), 0.0)
+        y = r.integers(0, 5, 2)
+        st, _ = srv.enqueue(k, x, y)
+        if st == O.OK:
+            sent[k].append((x, y))
+
+    for k in (0, 1, 0, 2, 1):
+        upload(k)
+    theta, v = theta0.copy(), np.zeros_like(theta0)
+    for step in range(8):
+        if step == 3:
+            upload(2)
+            upload(0)
+        st, k, _ = srv.step()
+        if st != O.OK:
+            break
+        x, y = sent[k].pop(0)
+        loss, theta, v, _ = O.server_step(ops, theta, v, x, y, None, lr, mu)
+        assert srv.losses[-1] == loss
+        assert np.array_equal(srv.theta, theta) and np.array_equal(srv.v, v)
+    assert all(not q for q in sent.values())
