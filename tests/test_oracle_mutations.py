@@ -317,6 +317,10 @@ param_shapes_bias_first = source_mutant(
                 out.append((i, "b", (op["cout"],)))
             out.append((i, "W", (op["cout"], op["k"], op["k"], op["cin"])))""")
 server_trains_highest_slot = source_mutant(O.Server.step, "self.slots.pop(slot)", "self.slots.pop(max(self.slots))")
+rejoin_keeps_counter = source_mutant(O.TaskScheduler.set_active, "self.c[k] = max(self.c[k], min(others))", "pass")
+fifo_serves_newest = source_mutant(O.TaskScheduler.get, "k = self.arrivals.popleft()", "k = self.arrivals.pop()")
+refused_never_blocked = source_mutant(O.TaskScheduler.put, "self.blocked.append(k)", "pass")
+sender_on_at_cap = source_mutant(O.TaskScheduler.put, "(total + 1 < self.omega)", "(total + 1 <= self.omega)")
 forward_flatten_nchw = source_mutant(O.forward, "y = a.reshape(a.shape[0], -1)",
                                      "y = a.transpose(0, 3, 1, 2).reshape(a.shape[0], -1)")
 
@@ -417,6 +421,17 @@ MUTATIONS = {
         [(TN.test_network_matches_torch_autograd, ("resnet",)), (TN.test_network_matches_torch_autograd, ("mobilenet",))]),
     "network forward: flatten in channel-first order": (
         {"forward": forward_flatten_nchw}, [(TN.test_network_matches_torch_autograd, ("vgg",))]),
+    "join: a rejoining device keeps its stale counter": (
+        {"TaskScheduler.set_active": rejoin_keeps_counter},
+        [(TS.test_leave_drains_queue_and_join_does_not_monopolise, ())]),
+    "FIFO policy: newest upload served first": (
+        {"TaskScheduler.get": fifo_serves_newest}, [(TS.test_fifo_policy_serves_in_arrival_order, ())]),
+    "flow control: a device refused with an empty queue is never turned on again": (
+        {"TaskScheduler.put": refused_never_blocked},
+        [(TS.test_blocked_device_is_turned_on_by_next_dequeue, ()), (TS.test_slot_reuse_matches_hand_derived_golden, ())]),
+    "flow control: Sender left on when the upload reaches the cap": (
+        {"TaskScheduler.put": sender_on_at_cap},
+        [(TS.test_tiny_schedule_matches_hand_derived_golden, ()), (TS.test_slot_reuse_matches_hand_derived_golden, ())]),
     "flat layout: conv bias before its weights": (
         {"param_shapes": param_shapes_bias_first}, [(TN.test_flat_layout_is_the_documented_order, ())]),
     "event replay: a step trains on the highest-numbered slot, not the served one": (
