@@ -321,6 +321,9 @@ rejoin_keeps_counter = source_mutant(O.TaskScheduler.set_active, "self.c[k] = ma
 fifo_serves_newest = source_mutant(O.TaskScheduler.get, "k = self.arrivals.popleft()", "k = self.arrivals.pop()")
 refused_never_blocked = source_mutant(O.TaskScheduler.put, "self.blocked.append(k)", "pass")
 sender_on_at_cap = source_mutant(O.TaskScheduler.put, "(total + 1 < self.omega)", "(total + 1 <= self.omega)")
+split_ignores_allowed = source_mutant(O.split_point, "if allowed is not None and not allowed[l - 1]:", "if False:")
+split_ties_to_largest = source_mutant(O.split_point, "if best_cost is None or worst < best_cost:",
+                                      "if best_cost is None or worst <= best_cost:")
 forward_flatten_nchw = source_mutant(O.forward, "y = a.reshape(a.shape[0], -1)",
                                      "y = a.transpose(0, 3, 1, 2).reshape(a.shape[0], -1)")
 
@@ -438,6 +441,11 @@ MUTATIONS = {
         {"Server.step": server_trains_highest_slot}, [(TN.test_server_trains_on_the_batch_the_scheduler_served, ())]),
     "split selection: training and transfer added, not overlapped": (
         {"split_point": split_sum_not_max}, golden_split_cases()),
+    "split selection: the allowed split points ignored": (
+        {"split_point": split_ignores_allowed}, golden_split_cases()),
+    "split selection: ties to the largest l": (
+        {"split_point": split_ties_to_largest},
+        golden_split_cases() + [(TP.test_ties_go_to_the_smallest_split, ())]),
     "split selection: the fastest device decides": (
         {"split_point": split_fastest_device}, golden_split_cases() + [(TP.test_slowest_device_decides, ())]),
 }

@@ -81,3 +81,18 @@ def test_bad_arguments():
     assert api.select_split(ok[0], ok[1], ok[2], [-1.0])[0] == api.ERR_ARG
     assert api.select_split(*ok, allowed=[0, 0])[0] == api.ERR_ARG
     assert api.select_split(*ok)[0] == api.OK
+
+
+def test_ties_go_to_the_smallest_split():
+    """Every split point costs exactly the same (compute far faster than the
+    link, every layer's output the same size): the reading takes the
+    smallest l, or the smallest allowed one when a mask is given."""
+    Oflop, S = [1.0, 1.0, 1.0, 1.0], [4096.0] * 4
+    b, o = [1e6, 2e6], [1e30, 1e30]
+    l, cost = O.split_point(Oflop, S, b, o)
+    assert (l, cost) == (1, 4096.0 / 1e6)
+    assert O.split_point(Oflop, S, b, o, [0, 0, 1, 1]) == (3, 4096.0 / 1e6)
+    rc, l2, c2 = api.select_split(Oflop, S, b, o, None)
+    assert (rc, l2, c2) == (api.OK, 1, 4096.0 / 1e6)
+    rc, l2, c2 = api.select_split(Oflop, S, b, o, [0, 0, 1, 1])
+    assert (rc, l2) == (api.OK, 3)
