@@ -22,9 +22,11 @@ What it follows (arxiv 2504.13850):
   * The MobileNetV3 bottleneck pieces of the paper's testbed-B CNN
     (Table 4): depthwise convolution, hard swish, hard sigmoid and the
     squeeze-and-excite channel scaling (``dwconv_*``, ``hswish_*``,
-    ``hsigmoid_*``, ``chmul_*``); the derivative readings at the kinks
-    follow the usual library convention (hard swish: 0 below -3, 1 above 3;
-    hard sigmoid: 1/6 strictly inside (-3, 3)).
+    ``hsigmoid_*``, ``chmul_*``).  The derivatives at the kinks are a
+    convention (the paper is silent): hard swish takes (2x + 3)/6 on the
+    closed interval [-3, 3], 0 below and 1 above; hard sigmoid takes 1/6
+    only strictly inside (-3, 3).  PyTorch 2.11 agrees on hard sigmoid but
+    gives hard swish the open interval.
   * The Pre-processor's split point (Sec. 3.2, Eqs. 4-6): argmin over split
     points of the slowest device's max of training and transfer time
     (``split_point``; ties go to the smallest l).

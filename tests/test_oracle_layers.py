@@ -326,3 +326,27 @@ def test_bf16_storage_rounds_every_stored_tensor():
     T64, _ = O.forward(ops, params, O.to_bf16(x), lengths)
     rel = np.linalg.norm(T[-1] - T64[-1]) / np.linalg.norm(T64[-1])
     assert 1e-5 < rel < 3e-2
+
+
+def test_bf16_reading_keeps_the_classifier_weights_fp32():
+    """In the bf16-storage reading every stored tensor and every hidden
+    conv / linear weight is rounded, but the logits layer reads the fp32
+    master weights (the classifier kernel does), so its output equals the
+    fp64 product of the rounded input with the unrounded weights."""
+    ops = [{"kind": "flatten", "in0": 0},
+           {"kind": "linear", "in0": 1, "cin": 6, "cout": 3, "bias": 1}]
+    r = rng(30)
+    w = r.standard_normal((3, 6))
+    w[0, 0] = 1.0 + 2.0 ** -12                    # not a bf16 value
+    b = r.standard_normal(3)
+    x = r.standard_normal((2, 1, 2, 3))
+    params = {(1, "W"): w, (1, "b"): b}
+    T, _ = O.forward(ops, params, x, None, storage="bf16")
+    assert np.array_equal(T[-1], O.to_bf16(x).reshape(2, 6) @ w.T + b)
+    hidden = [{"kind": "flatten", "in0": 0},
+              {"kind": "linear", "in0": 1, "cin": 6, "cout": 3, "bias": 0},
+              {"kind": "linear", "in0": 2, "cin": 3, "cout": 2, "bias": 0}]
+    w2 = r.standard_normal((2, 3))
+    T, _ = O.forward(hidden, {(1, "W"): w, (2, "W"): w2}, x, None, storage="bf16")
+    h = O.to_bf16(O.to_bf16(x).reshape(2, 6) @ O.to_bf16(w).T)
+    assert np.array_equal(T[2], h) and np.array_equal(T[3], h @ w2.T)

@@ -63,3 +63,28 @@ def test_channel_scaling_gradients():
         e = np.zeros_like(s)
         e[idx] = h
         assert ds[idx] == pytest.approx((f(x, s + e) - f(x, s - e)) / (2 * h), rel=1e-6)
+
+
+
+def test_kink_derivatives_are_the_stated_one_sided_limits():
+    """At exactly -3 and 3 the derivative is a convention (any value between
+    the one-sided derivatives is a subgradient).  The one taken here, by the
+    oracle and the kernels alike, is checked against one-sided finite
+    differences: hard swish uses its interior formula on the closed interval
+    [-3, 3] (the right derivative at -3, the left one at 3); hard sigmoid
+    uses 1/6 only strictly inside, so at both kinks it takes the outer
+    one-sided derivative, 0.  PyTorch 2.11 agrees on hard sigmoid but gives
+    hard swish the open interval (0 at -3, 1 at 3)."""
+    h = 1e-7
+    one = np.ones(1)
+
+    def right(f, x):
+        return float((f(np.array([x + h])) - f(np.array([x])))[0] / h)
+
+    def left(f, x):
+        return float((f(np.array([x])) - f(np.array([x - h])))[0] / h)
+
+    assert O.hswish_bwd(np.array([-3.0]), one)[0] == pytest.approx(right(O.hswish_fwd, -3.0), abs=1e-6)
+    assert O.hswish_bwd(np.array([3.0]), one)[0] == pytest.approx(left(O.hswish_fwd, 3.0), abs=1e-6)
+    assert O.hsigmoid_bwd(np.array([-3.0]), one)[0] == pytest.approx(left(O.hsigmoid_fwd, -3.0), abs=1e-6)
+    assert O.hsigmoid_bwd(np.array([3.0]), one)[0] == pytest.approx(right(O.hsigmoid_fwd, 3.0), abs=1e-6)

@@ -324,6 +324,25 @@ sender_on_at_cap = source_mutant(O.TaskScheduler.put, "(total + 1 < self.omega)"
 split_ignores_allowed = source_mutant(O.split_point, "if allowed is not None and not allowed[l - 1]:", "if False:")
 split_ties_to_largest = source_mutant(O.split_point, "if best_cost is None or worst < best_cost:",
                                       "if best_cost is None or worst <= best_cost:")
+head_weights_rounded = source_mutant(O._weights, 'if storage == "bf16" and i < len(ops) - 1:', 'if storage == "bf16":')
+hswish_bwd_open_interval = source_mutant(O.hswish_bwd, "np.where(x < -3.0, 0.0, np.where(x > 3.0, 1.0,",
+                                         "np.where(x <= -3.0, 0.0, np.where(x >= 3.0, 1.0,")
+hsigmoid_bwd_closed_interval = source_mutant(O.hsigmoid_bwd, "(x > -3.0) & (x < 3.0)", "(x >= -3.0) & (x <= 3.0)")
+depth_off_by_one = source_mutant(O.TaskScheduler.put, "len(self.q[k]) >= self.depth", "len(self.q[k]) > self.depth")
+future_version_accepted = source_mutant(O.Aggregator.aggregate, "if t_k < 0 or t_k > self.t:", "if t_k < 0:")
+
+
+def get_empty_argmin_serves_nothing(self):
+    """The argmin taken over every device, empty queues included: when the
+    least-served device has nothing queued the step does nothing."""
+    if self.policy != "counter":
+        return ORIG_GET(self)
+    k = min(range(self.K), key=lambda j: (self.c[j], j))
+    if not self.q[k]:
+        return O.EMPTY, -1, -1
+    return ORIG_GET(self)
+
+
 forward_flatten_nchw = source_mutant(O.forward, "y = a.reshape(a.shape[0], -1)",
                                      "y = a.transpose(0, 3, 1, 2).reshape(a.shape[0], -1)")
 
@@ -435,6 +454,20 @@ MUTATIONS = {
     "flow control: Sender left on when the upload reaches the cap": (
         {"TaskScheduler.put": sender_on_at_cap},
         [(TS.test_tiny_schedule_matches_hand_derived_golden, ()), (TS.test_slot_reuse_matches_hand_derived_golden, ())]),
+    "bf16 reading: the classifier's weights rounded too": (
+        {"_weights": head_weights_rounded}, [(TL.test_bf16_reading_keeps_the_classifier_weights_fp32, ())]),
+    "hard swish derivative on the open interval at the kinks": (
+        {"hswish_bwd": hswish_bwd_open_interval}, [(TM.test_kink_derivatives_are_the_stated_one_sided_limits, ())]),
+    "hard sigmoid derivative 1/6 at the kinks too": (
+        {"hsigmoid_bwd": hsigmoid_bwd_closed_interval},
+        [(TM.test_kink_derivatives_are_the_stated_one_sided_limits, ())]),
+    "flow control: ring depth off by one": (
+        {"TaskScheduler.put": depth_off_by_one}, [(TS.test_slot_reuse_matches_hand_derived_golden, ())]),
+    "scheduler: empty queues compete in the argmin": (
+        {"TaskScheduler.get": get_empty_argmin_serves_nothing},
+        [(TS.test_random_traces_keep_invariants_and_pick_min_counter, (s,)) for s in range(4)]),
+    "FedAsync: a version from the future accepted": (
+        {"Aggregator.aggregate": future_version_accepted}, [(TS.test_stale_and_invalid_versions, ())]),
     "flat layout: conv bias before its weights": (
         {"param_shapes": param_shapes_bias_first}, [(TN.test_flat_layout_is_the_documented_order, ())]),
     "event replay: a step trains on the highest-numbered slot, not the served one": (
@@ -471,7 +504,7 @@ def test_planted_mistake_fails_a_pin(name, monkeypatch):
     for fn, args in pins:
         try:
             fn(*args)
-        except AssertionError:
+        except Exception:           # a failed assertion, or a pin the mistake crashes
             caught.append(fn.__name__)
     assert caught, f"no pin caught the planted mistake: {name}"
 
