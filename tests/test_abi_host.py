@@ -169,3 +169,17 @@ def test_every_entry_point_cites_its_passage_or_says_it_has_none():
             if not before or not cite.search(before[-1][1]):
                 missing.append(re.search(r"(fo_\w+)\s*\(", line).group(1))
     assert not missing, missing
+
+
+def test_missing_library_fails_loudly(monkeypatch):
+    """Without the built library every entry point raises: there is no
+    fallback path (CPU or otherwise) behind the binding."""
+    monkeypatch.setattr(api, "_lib", None)
+    monkeypatch.setattr(api, "LIB_PATH", os.path.join(ROOT, "_no_such_dir", "libfedoptima.so"))
+    with pytest.raises(api.FedOptimaError, match="missing"):
+        api.lib()
+    with pytest.raises(api.FedOptimaError):
+        api.Scheduler(2, 2, 1)
+    from paper_2504_13850_gb300 import workloads as W
+    with pytest.raises(api.FedOptimaError):
+        api.Server.from_config(W.CONFIGS["tiny"])
