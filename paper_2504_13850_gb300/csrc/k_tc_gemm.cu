@@ -57,9 +57,6 @@ struct TcParams {
   // row (n*oH + ostride*i + py)*oW + ostride*j + px of `out` (identity when
   // ostride == 0)
   int ostride, py, px, Hq, Wq, oH, oW;
-  // paired CTAs: the window operand is loaded as two halves, the second at
-  // these row / image offsets (in the windowed tensor's coordinates)
-  int half_dh, half_dn;
   // MN-major operands whose 64-wide chunks one TMA box brings in at once
   // (a chunk dimension of stride 128 bytes as the box's outermost dimension)
   int chunk_a, chunk_b;
@@ -286,12 +283,9 @@ struct KindTraits {
 };
 
 // Issue the TMA loads of k-block `kb` for output tile (m0, n0).
-// PAIR 1: the two CTAs of a cluster share m0 and each loads half of the
-// window operand A for both (multicast); PAIR 2: they share n0 and split the
-// window boxes of B.  `rank` is the CTA's rank in its cluster.
-template <int KIND, int BN, int PAIR = 0>
+template <int KIND, int BN>
 __device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, int n0, char* sa, char* sb,
-                                            uint64_t* bar, uint32_t rank = 0) {
+                                            uint64_t* bar) {
   const int HW = p.H * p.W;
   if (KIND == LIN_FWD || KIND == LIN_DGRAD) {
     tma_2d(sa, &p.tmA, bar, kb * BK, m0);
@@ -305,19 +299,11 @@ __device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, i
     const int tap = kb / p.cblocks, c0 = (kb % p.cblocks) * 64;
     const int r = tap / p.ksz, s = tap % p.ksz;
     const int n_img = m0 / HW, h0 = (m0 % HW) / p.W;   // H, W: output grid
-    if (PAIR == 1)
-      tma_4d_mc(sa + rank * (BM * BK), &p.tmA, bar, c0, s - p.pad,
-                h0 * p.stride + r - p.pad + int(rank) * p.half_dh, n_img + int(rank) * p.half_dn, 0x3);
-    else
-      tma_4d(sa, &p.tmA, bar, c0, s - p.pad, h0 * p.stride + r - p.pad, n_img);
+    tma_4d(sa, &p.tmA, bar, c0, s - p.pad, h0 * p.stride + r - p.pad, n_img);
   } else {  // CONV_DGRAD: window over the output gradient, shifted per tap
     const int t = kb / p.cblocks, c0 = (kb % p.cblocks) * 64;
     const int n_img = m0 / HW, h0 = (m0 % HW) / p.W;   // H, W: the class grid (= gradient grid)
-    if (PAIR == 1)
-      tma_4d_mc(sa + rank * (BM * BK), &p.tmA, bar, c0, p.tap_dw[t], h0 + p.tap_dh[t] + int(rank) * p.half_dh,
-                n_img + int(rank) * p.half_dn, 0x3);
-    else
-      tma_4d(sa, &p.tmA, bar, c0, p.tap_dw[t], h0 + p.tap_dh[t], n_img);
+    tma_4d(sa, &p.tmA, bar, c0, p.tap_dw[t], h0 + p.tap_dh[t], n_img);
   }
   if (KIND == LIN_FWD) {
     tma_2d(sb, &p.tmB, bar, kb * BK, n0);
@@ -338,30 +324,20 @@ __device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, i
     else
 #pragma unroll
       for (int j = 0; j < BN / 64; ++j) tma_2d(sb + j * BK * 128, &p.tmB, bar, tap * p.ntap_ch + n0 + j * 64, co0);
-  } else if (p.chunk_b) {  // CONV_WGRAD, all chunks of the tile (a pair: half each, multicast)
+  } else if (p.chunk_b) {  // CONV_WGRAD, all chunks of the tile in one box
     const int tap = n0 / p.ntap_ch, ci0 = n0 % p.ntap_ch;
     const int r = tap / p.ksz, s = tap % p.ksz;
     const int pix0 = kb * BK;
     const int n_img = pix0 / HW, h0 = (pix0 % HW) / p.W;
-    if (PAIR == 2)
-      tma_5d_mc(sb + int(rank) * (BN / 128) * BK * 128, &p.tmB, bar, 0, s - p.pad, h0 * p.stride + r - p.pad, n_img,
-                ci0 / 64 + int(rank) * (BN / 128), 0x3);
-    else
-      tma_5d(sb, &p.tmB, bar, 0, s - p.pad, h0 * p.stride + r - p.pad, n_img, ci0 / 64);
+    tma_5d(sb, &p.tmB, bar, 0, s - p.pad, h0 * p.stride + r - p.pad, n_img, ci0 / 64);
   } else {  // CONV_WGRAD: N index = tap * Ci + ci; K = output pixel
     const int tap = n0 / p.ntap_ch, ci0 = n0 % p.ntap_ch;
     const int r = tap / p.ksz, s = tap % p.ksz;
     const int pix0 = kb * BK;
     const int n_img = pix0 / HW, h0 = (pix0 % HW) / p.W;   // H, W: output grid
 #pragma unroll
-    for (int j = 0; j < BN / 64; ++j) {
-      if (PAIR == 2) {
-        if ((j & 1) == int(rank))
-          tma_4d_mc(sb + j * BK * 128, &p.tmB, bar, ci0 + j * 64, s - p.pad, h0 * p.stride + r - p.pad, n_img, 0x3);
-      } else {
-        tma_4d(sb + j * BK * 128, &p.tmB, bar, ci0 + j * 64, s - p.pad, h0 * p.stride + r - p.pad, n_img);
-      }
-    }
+    for (int j = 0; j < BN / 64; ++j)
+      tma_4d(sb + j * BK * 128, &p.tmB, bar, ci0 + j * 64, s - p.pad, h0 * p.stride + r - p.pad, n_img);
   }
 }
 
@@ -571,13 +547,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 // MMA), acc_full/acc_empty per accumulator (MMA <-> epilogue).
 constexpr int kPersistThreads = 320;  // TMA warp, MMA warp, 8 epilogue warps
 constexpr int kEpiStageBytes = 8 * 4096;  // one 32 x 32 fp32 staging buffer per epilogue warp
-
-// PAIR != 0: launched as clusters of two CTAs that run the same k-block
-// sequence on two adjacent tiles and split the TMA loads of the operand they
-// share (1: A, tiles side by side in N; 2: B, tiles stacked in M), each
-// multicasting its half to both.  A stage is then refilled only when both
-// CTAs' MMAs have released it (empty barriers count two arrivals).
-template <int KIND, int BN, int STAGES, int PAIR>
+template <int KIND, int BN, int STAGES>
 __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const __grid_constant__ TcParams p) {
   extern __shared__ __align__(1024) char smem_raw[];
   char* smem = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -594,21 +564,19 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
-  const int unit = PAIR ? int(blockIdx.x) / 2 : int(blockIdx.x);
-  const int units = PAIR ? int(gridDim.x) / 2 : int(gridDim.x);
+  const int unit = int(blockIdx.x);
+  const int units = int(gridDim.x);
   const int n_tiles = (p.N + BN - 1) / BN, m_tiles = (p.M + BM - 1) / BM;
-  const int su_n = PAIR == 1 ? n_tiles / 2 : n_tiles;   // work units: tiles, or tile pairs
-  const int tiles = su_n * (PAIR == 2 ? m_tiles / 2 : m_tiles);
+  const int tiles = n_tiles * m_tiles;
   const int KB = p.KB;
   constexpr uint32_t kCols = 2 * BN < 32 ? 32 : 2 * BN;
-  auto tile_n0 = [&](int t) { return (PAIR == 1 ? 2 * (t % su_n) + int(rank) : t % su_n) * BN; };
-  auto tile_m0 = [&](int t) { return (PAIR == 2 ? 2 * (t / su_n) + int(rank) : t / su_n) * BM; };
+  auto tile_n0 = [&](int t) { return (t % n_tiles) * BN; };
+  auto tile_m0 = [&](int t) { return (t / n_tiles) * BM; };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], PAIR ? 2 : 1);
+      mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
@@ -627,7 +595,6 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
   }
   tc_fence_before();
   __syncthreads();
-  if (PAIR) cluster_sync_all();   // the peer's barriers are initialised
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   pdl_trigger();
@@ -647,18 +614,7 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
           }
           char* sa = smem + s * STAGE_BYTES;
           mbar_expect_tx(&full[s], STAGE_BYTES);
-          load_kblock<KIND, BN, PAIR>(p, kb, m0, n0, sa, sa + A_BYTES, &full[s], rank);
-        }
-      }
-      if (PAIR) {
-        // Drain: every stage released by both CTAs, so no arrival from the
-        // peer is still on its way when the cluster exits.
-        for (int i = 0; i < STAGES; ++i, ++g) {
-          const int s = g % STAGES;
-          if (!mbar_wait(&empty[s], ((g / STAGES) & 1) ^ 1)) {
-            atomicExch(p.err, 8);
-            break;
-          }
+          load_kblock<KIND, BN>(p, kb, m0, n0, sa, sa + A_BYTES, &full[s]);
         }
       }
     }
@@ -697,8 +653,7 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
             else bd = smem_desc(b0 + k * UK * 2, 16, 1024);
             mma_f16(d, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
           }
-          if (PAIR) mma_commit_mc(&empty[s], 0x3);
-          else mma_commit(&empty[s]);
+          mma_commit(&empty[s]);
         }
         if (ok) mma_commit(&acc_full[b]);
         else {
@@ -744,7 +699,6 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
   }
   tc_fence_before();
   __syncthreads();
-  if (PAIR) cluster_sync_all();
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kCols) : "memory");
@@ -777,26 +731,18 @@ constexpr size_t smem_bytes(bool cluster) {
 typedef void (*KernelFn)(const TcParams);
 
 template <int KIND, int BN>
-KernelFn kernel_ptr(bool cluster, int pair) {
-  constexpr int S = stages_for<KIND, BN, false>();
-  if (cluster) return pair ? nullptr : tc_gemm_kernel<KIND, BN, stages_for<KIND, BN, true>()>;
-  if constexpr ((KIND == CONV_FPROP || KIND == CONV_DGRAD) && BN >= 128) {
-    if (pair == 1) return tc_gemm_persistent<KIND, BN, S, 1>;
-  }
-  if constexpr (KIND == CONV_WGRAD && BN >= 128) {
-    if (pair == 2) return tc_gemm_persistent<KIND, BN, S, 2>;
-  }
-  if (pair) return nullptr;
-  return tc_gemm_persistent<KIND, BN, S, 0>;
+KernelFn kernel_ptr(bool cluster) {
+  if (cluster) return tc_gemm_kernel<KIND, BN, stages_for<KIND, BN, true>()>;
+  return tc_gemm_persistent<KIND, BN, stages_for<KIND, BN, false>()>;
 }
 
-KernelFn pick_kernel(int kind, int bn, bool cluster, int pair, size_t* smem) {
+KernelFn pick_kernel(int kind, int bn, bool cluster, size_t* smem) {
 #define FO_PICK(K)                                                  \
   if (kind == K) {                                                  \
-    if (bn == 256) { *smem = smem_bytes<K, 256>(cluster); return kernel_ptr<K, 256>(cluster, pair); } \
-    if (bn == 128) { *smem = smem_bytes<K, 128>(cluster); return kernel_ptr<K, 128>(cluster, pair); } \
+    if (bn == 256) { *smem = smem_bytes<K, 256>(cluster); return kernel_ptr<K, 256>(cluster); } \
+    if (bn == 128) { *smem = smem_bytes<K, 128>(cluster); return kernel_ptr<K, 128>(cluster); } \
     *smem = smem_bytes<K, 64>(cluster);                                    \
-    return kernel_ptr<K, 64>(cluster, pair);                         \
+    return kernel_ptr<K, 64>(cluster);                               \
   }
   FO_PICK(LIN_FWD)
   FO_PICK(LIN_DGRAD)
@@ -897,7 +843,6 @@ struct TcGemm {
   TcGemm() : p{} { p.stride = 1; }
   const char* name = nullptr;
   int kind = 0, bn = 0, splits = 1;
-  int pair = 0;            // 0, or the operand a CTA pair shares (1: A, 2: B)
   double flops = 0;
   TcParams p;
   KernelFn fn = nullptr;
@@ -942,40 +887,37 @@ bool window_ok(int N, int H, int W, int rows_needed, int* rows, int* imgs) {
 }
 
 
-// Clusters that fit on the GPU at once (GPC packing), from the occupancy
-// calculator; cached per context.  pair == 0: split-K clusters of S CTAs of
-// kernel (kind, bn); pair != 0: two-CTA clusters of the persistent kernel.
-int active_clusters(TcContext* c, int kind, int bn, int S, int pair) {
-  const int key = ((kind * 512 + bn) * 16 + S) * 4 + pair;
+// Split-K clusters of S CTAs of kernel (kind, bn) that fit on the GPU at
+// once (GPC packing), from the occupancy calculator; cached per context.
+int active_clusters(TcContext* c, int kind, int bn, int S) {
+  const int key = (kind * 512 + bn) * 16 + S;
   auto it = c->cluster_fit.find(key);
   if (it != c->cluster_fit.end()) return it->second;
   size_t smem = 0;
-  KernelFn fn = pick_kernel(kind, bn, pair == 0, pair, &smem);
+  KernelFn fn = pick_kernel(kind, bn, true, &smem);
   int n = 0;
   if (fn && cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem)) == cudaSuccess) {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = pair ? dim3(2, 1, 1) : dim3(1, 1, S);
-    cfg.blockDim = dim3(pair ? kPersistThreads : kThreads);
+    cfg.gridDim = dim3(1, 1, S);
+    cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem;
     cudaLaunchAttribute attr;
     attr.id = cudaLaunchAttributeClusterDimension;
-    attr.val.clusterDim.x = pair ? 2 : 1;
+    attr.val.clusterDim.x = 1;
     attr.val.clusterDim.y = 1;
-    attr.val.clusterDim.z = pair ? 1 : S;
+    attr.val.clusterDim.z = S;
     cfg.attrs = &attr;
     cfg.numAttrs = 1;
     if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess) n = 0;
   }
   cudaGetLastError();
-  if (n <= 0) {   // conservative fallback
-    const int size = pair ? 2 : S;
-    n = c->num_sms / (2 * size) > 0 ? c->num_sms / (2 * size) : 1;
-  }
+  if (n <= 0)   // conservative fallback
+    n = c->num_sms / (2 * S) > 0 ? c->num_sms / (2 * S) : 1;
   c->cluster_fit[key] = n;
   return n;
 }
 
-// Tile width, K split and CTA pairing from a cost model in microseconds,
+// Tile width and K split from a cost model in microseconds,
 // fitted to GB300 timelines of these kernels:
 //  * a k-block stage costs at least ~0.37 us: each stage is one round of
 //    mbarrier waits (full on the MMA side, empty on the TMA side), whose
@@ -992,50 +934,42 @@ int active_clusters(TcContext* c, int kind, int bn, int S, int pair) {
 //    staging and distributed-shared-memory reduction of its partial tiles,
 //    and clusters run in waves of what the occupancy calculator fits at once.
 // Candidate widths divide `ndiv` (N, or the channels of one tap for the
-// weight gradient, whose N index runs over taps x channels).  `pair_ok`: the
-// planner can split the shared operand's box in two.
-void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv, bool pair_ok) {
+// weight gradient, whose N index runs over taps x channels).
+void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv) {
   const bool win_a = g->kind == CONV_FPROP || g->kind == CONV_DGRAD;
   const bool win_b = g->kind == CONV_WGRAD;
   double best = 1e30;
-  int best_bn = 0, best_s = 1, best_pair = 0;
+  int best_bn = 0, best_s = 1;
   for (int bn : {256, 128, 64}) {
     // window kinds tile whole taps; the plain GEMMs take a ragged last tile
     if ((win_a || win_b) && (ndiv % bn || N % bn)) continue;
     const int n_tiles = (N + bn - 1) / bn, m_tiles = (M + BM - 1) / BM, tiles = n_tiles * m_tiles;
     const double stage_kb = (BM + bn) * BK * 2 / 1024.0;
     const double epi = bn == 256 ? 4.2 : (bn == 128 ? 2.2 : 1.5);
-    for (int pair = 0; pair <= 2; ++pair) {
-      if (pair == 1 && !(pair_ok && win_a && bn >= 128 && n_tiles % 2 == 0)) continue;
-      if (pair == 2 && !(pair_ok && win_b && bn >= 128 && m_tiles % 2 == 0)) continue;
-      double t_kb = std::max(0.37, stage_kb / 128.0);
-      if (win_b) t_kb = std::max(t_kb, 0.39);
-      for (int sp = 1; sp <= (pair ? 1 : 8); ++sp) {
-        if (sp > 1 && KB / sp < 4) break;
-        // an owner's receive slices (16 KB per other rank and owned chunk) live in the pipeline buffers
-        if (sp > 1 && size_t(sp - 1) * ((bn / 32 + sp - 1) / sp) * 16384 > pipeline_bytes(bn)) continue;
-        const int kper = (KB + sp - 1) / sp;
-        const int splits = (KB + kper - 1) / kper;
-        if (splits != sp) continue;
-        double cost;
-        if (splits == 1) {
-          const int work = pair ? tiles / 2 : tiles;
-          const int units = std::min(work, pair ? active_clusters(c, g->kind, bn, 2, pair) : c->num_sms);
-          const int per_unit = (work + units - 1) / units;
-          const double main = kper * t_kb;
-          cost = (pair ? 2.2 : 1.7) + per_unit * main + epi + (pair ? 0.7 : 0.0) +
-                 (per_unit - 1) * std::max(0.0, epi - main);
-        } else {
-          const int fit = active_clusters(c, g->kind, bn, splits, 0);
-          const int waves = (tiles + fit - 1) / fit;
-          cost = waves * (1.0 + kper * t_kb + 3.0 + 2.5 * bn / 128.0);
-        }
-        if (cost < best - 1e-9) {
-          best = cost;
-          best_bn = bn;
-          best_s = splits;
-          best_pair = pair;
-        }
+    double t_kb = std::max(0.37, stage_kb / 128.0);
+    if (win_b) t_kb = std::max(t_kb, 0.39);
+    for (int sp = 1; sp <= 8; ++sp) {
+      if (sp > 1 && KB / sp < 4) break;
+      // an owner's receive slices (16 KB per other rank and owned chunk) live in the pipeline buffers
+      if (sp > 1 && size_t(sp - 1) * ((bn / 32 + sp - 1) / sp) * 16384 > pipeline_bytes(bn)) continue;
+      const int kper = (KB + sp - 1) / sp;
+      const int splits = (KB + kper - 1) / kper;
+      if (splits != sp) continue;
+      double cost;
+      if (splits == 1) {
+        const int units = std::min(tiles, c->num_sms);
+        const int per_unit = (tiles + units - 1) / units;
+        const double main = kper * t_kb;
+        cost = 1.7 + per_unit * main + epi + (per_unit - 1) * std::max(0.0, epi - main);
+      } else {
+        const int fit = active_clusters(c, g->kind, bn, splits);
+        const int waves = (tiles + fit - 1) / fit;
+        cost = waves * (1.0 + kper * t_kb + 3.0 + 2.5 * bn / 128.0);
+      }
+      if (cost < best - 1e-9) {
+        best = cost;
+        best_bn = bn;
+        best_s = splits;
       }
     }
   }
@@ -1043,7 +977,6 @@ void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv, bool 
   g->p.KB = KB;
   g->p.kper = (KB + best_s - 1) / best_s;
   g->splits = best_s;
-  g->pair = best_pair;
 }
 
 TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
@@ -1051,7 +984,7 @@ TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
   g->p.N = N;
   g->flops = 2.0 * M * N * K;
   g->p.err = c->err;
-  g->fn = pick_kernel(g->kind, g->bn, g->splits > 1, g->pair, &g->smem);
+  g->fn = pick_kernel(g->kind, g->bn, g->splits > 1, &g->smem);
   if (!g->fn) {
     delete g;
     return nullptr;
@@ -1063,16 +996,13 @@ TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
   const int n_tiles = (N + g->bn - 1) / g->bn;
   if (g->splits > 1) {
     g->grid = dim3(n_tiles, (M + BM - 1) / BM, g->splits);
-  } else if (g->pair) {
-    const int work = n_tiles * ((M + BM - 1) / BM) / 2;
-    g->grid = dim3(2 * std::min(work, active_clusters(c, g->kind, g->bn, 2, g->pair)), 1, 1);
   } else {
     const int tiles = n_tiles * ((M + BM - 1) / BM);
     g->grid = dim3(std::min(tiles, c->num_sms), 1, 1);
   }
   if (getenv("FO_DEBUG_PLAN"))
-    fprintf(stderr, "[plan] %-16s M=%d N=%d KB=%d BN=%d splits=%d pair=%d grid=(%u,%u,%u) chunked=%d%d\n", g->name, M,
-            N, g->p.KB, g->bn, g->splits, g->pair, g->grid.x, g->grid.y, g->grid.z, g->p.chunk_a, g->p.chunk_b);
+    fprintf(stderr, "[plan] %-16s M=%d N=%d KB=%d BN=%d splits=%d grid=(%u,%u,%u) chunked=%d%d\n", g->name, M, N,
+            g->p.KB, g->bn, g->splits, g->grid.x, g->grid.y, g->grid.z, g->p.chunk_a, g->p.chunk_b);
   g->ctx = c;
   c->gemms.push_back(g);
   return g;
@@ -1164,7 +1094,7 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i, void* out, bool relu)
     g->kind = LIN_FWD;
     g->name = op.kind == FO_OP_LINEAR ? "tc_linear_fwd" : "tc_conv1x1_fwd";
     int M = int(a.rows()), KB = (op.cin + 63) / 64;
-    choose_tiles(c, g, M, op.cout, KB, op.cout, false);
+    choose_tiles(c, g, M, op.cout, KB, op.cout);
     const int bn = g->bn;
     g->input_A = (op.in0 == 0);
     if (g->input_A) {
@@ -1187,14 +1117,9 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i, void* out, bool relu)
   g->p.ntap_ch = op.cin;
   g->p.win_rows = rows; g->p.win_imgs = imgs;
   int M = a.N * Ho * Wo, KB = g->p.taps * g->p.cblocks;
-  choose_tiles(c, g, M, op.cout, KB, op.cout, imgs > 1 ? imgs % 2 == 0 : rows % 2 == 0);
+  choose_tiles(c, g, M, op.cout, KB, op.cout);
   const int bn = g->bn;
-  // paired CTAs each fetch half of the window: half the images, else half the rows
-  int box_rows = rows, box_imgs = imgs;
-  if (g->pair == 1) {
-    if (imgs > 1) { box_imgs = imgs / 2; g->p.half_dn = box_imgs; }
-    else { box_rows = rows / 2; g->p.half_dh = box_rows * st; }
-  }
+  const int box_rows = rows, box_imgs = imgs;
   g->input_A = (op.in0 == 0);
   if (g->input_A) {
     g->slot_maps.resize(s->cfg.omega);
@@ -1229,7 +1154,7 @@ bool tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate, void* dx, 
     g->kind = LIN_DGRAD;
     g->name = op.kind == FO_OP_LINEAR ? "tc_linear_dgrad" : "tc_conv1x1_dgrad";
     int M = int(a.rows()), KB = (op.cout + 63) / 64;
-    choose_tiles(c, g, M, op.cin, KB, op.cin, false);
+    choose_tiles(c, g, M, op.cin, KB, op.cin);
     if (!map_2d(&g->p.tmA, o.grad, M, op.cout, BM) || !map_2d(&g->p.tmB, w, op.cout, op.cin, BK)) { delete g; return false; }
     CUtensorMap cb;
     if (map_chunked(&cb, w, op.cout, op.cin, BK, g->bn / 64)) { g->p.tmB = cb; g->p.chunk_b = 1; }
@@ -1284,13 +1209,8 @@ bool tc_plan_dgrad(TcContext* c, fo_server* s, int i, int accumulate, void* dx, 
       g->p.Hq = Ho; g->p.Wq = Wo; g->p.oH = a.H; g->p.oW = a.W;
     }
     const int M = o.N * Ho * Wo, KB = cls[q].n * g->p.cblocks;
-    choose_tiles(c, g, M, op.cin, KB, op.cin, imgs > 1 ? imgs % 2 == 0 : rows % 2 == 0);
-    int box_rows = rows, box_imgs = imgs;
-    if (g->pair == 1) {
-      if (imgs > 1) { box_imgs = imgs / 2; g->p.half_dn = box_imgs; }
-      else { box_rows = rows / 2; g->p.half_dh = box_rows; }
-    }
-    if (!map_window(&g->p.tmA, o.grad, o.N, Ho, Wo, o.C, Wo, box_rows, box_imgs) ||
+    choose_tiles(c, g, M, op.cin, KB, op.cin);
+    if (!map_window(&g->p.tmA, o.grad, o.N, Ho, Wo, o.C, Wo, rows, imgs) ||
         !map_2d(&g->p.tmB, w, op.cout, int64_t(g->p.taps) * op.cin, BK)) {
       delete g;
       for (TcGemm* x : *out) (void)x;
@@ -1323,7 +1243,7 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
     g->name = op.kind == FO_OP_LINEAR ? "tc_linear_wgrad" : "tc_conv1x1_wgrad";
     g->p.ldo = op.cin;
     int rows = int(a.rows()), KB = (rows + BK - 1) / BK;
-    choose_tiles(c, g, op.cout, op.cin, KB, op.cin, false);
+    choose_tiles(c, g, op.cout, op.cin, KB, op.cin);
     g->input_B = (op.in0 == 0);
     if (!map_2d(&g->p.tmA, o.grad, rows, op.cout, BK)) { delete g; return nullptr; }
     CUtensorMap ca;
@@ -1357,12 +1277,12 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
   g->p.ntap_ch = op.cin;
   int P = a.N * Ho * Wo, KB = P / BK;
   int N = g->p.taps * op.cin;
-  choose_tiles(c, g, op.cout, N, KB, op.cin, true);
+  choose_tiles(c, g, op.cout, N, KB, op.cin);
   g->input_B = (op.in0 == 0);
   if (!map_2d(&g->p.tmA, o.grad, P, op.cout, BK)) { delete g; return nullptr; }
   CUtensorMap ca;
   if (map_chunked(&ca, o.grad, P, op.cout, BK, BM / 64)) { g->p.tmA = ca; g->p.chunk_a = 1; }
-  const int nchunk = g->pair == 2 ? g->bn / 128 : g->bn / 64;
+  const int nchunk = g->bn / 64;
   g->p.chunk_b = 1;
   auto map_b = [&](CUtensorMap* m, const void* base) {
     if (g->p.chunk_b && map_window_chunked(m, base, a.N, a.H, a.W, a.C, Wo, rows, imgs, st, nchunk)) return true;
@@ -1386,26 +1306,8 @@ void tc_run(TcGemm* g, const void* input, cudaStream_t st) {
   TcContext* c = g->ctx;
   if (g->input_A) g->p.tmA = g->slot_maps[c->slot];
   if (g->input_B) g->p.tmB = g->slot_maps[c->slot];
-  if (g->splits == 1 && !g->pair) {
+  if (g->splits == 1) {
     launch_k(g->fn, g->grid, kPersistThreads, g->smem, st, g->p);
-    return;
-  }
-  if (g->pair) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = g->grid;
-    cfg.blockDim = dim3(kPersistThreads);
-    cfg.dynamicSmemBytes = g->smem;
-    cfg.stream = st;
-    cudaLaunchAttribute attr[2];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 2;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[1].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = pdl_enabled() ? 2 : 1;
-    cudaLaunchKernelEx(&cfg, g->fn, g->p);
     return;
   }
   cudaLaunchConfig_t cfg = {};

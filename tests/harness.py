@@ -126,17 +126,32 @@ def teacher_forced(cfg, events, max_steps=None):
         loss = float(s.read_losses(steps, 1)[0])
         th1 = s.get_params().astype(np.float64)
         v1 = s.get_momentum().astype(np.float64)
-        g_gpu = v1 - mu * v0
-        rec = {"step": steps, "loss": loss}
-        for tag, srv in (("exact", o), ("stored", ob)):
-            g_ref = srv.v - mu * v0
-            rec[tag] = {
-                "loss": srv.losses[-1],
-                "param_err": normwise(th1, srv.theta),
-                "update_err": normwise(th1 - th0, srv.theta - th0),
-                "grad_err": normwise(g_gpu, g_ref),
-                "tensor_grad_err": {n: normwise(g_gpu[sl], g_ref[sl]) for n, sl in slices},
-            }
-        recs.append(rec)
+        recs.append(step_record(steps, loss, th0, v0, th1, v1, o, ob, mu, slices))
         steps += 1
     return s, o, recs
+
+
+def step_record(step, loss, th0, v0, th1, v1, o, ob, mu, slices):
+    """One teacher-forced step's errors.  `th1, v1, loss` are the path under
+    test, `o` the exact oracle and `ob` its bf16-storage reading, both
+    stepped from (th0, v0).  The gradient is recovered exactly from the
+    momentum, g = v1 - mu v0.  "reading" records how far the bf16-storage
+    reading's own gradient lies from the exact one (per tensor and whole):
+    the distance that storing the path's tensors in bf16 moves the
+    definition by, which sets the allowance for decision flips."""
+    g_gpu = v1 - mu * v0
+    g_ex = o.v - mu * v0
+    g_rd = ob.v - mu * v0
+    rec = {"step": step, "loss": loss,
+           "g_norm": float(np.linalg.norm(g_ex)), "v_norm": float(np.linalg.norm(o.v)),
+           "reading": {"whole": normwise(g_rd, g_ex),
+                       "tensor": {n: normwise(g_rd[sl], g_ex[sl]) for n, sl in slices}}}
+    for tag, srv, g_ref in (("exact", o, g_ex), ("stored", ob, g_rd)):
+        rec[tag] = {
+            "loss": srv.losses[-1],
+            "param_err": normwise(th1, srv.theta),
+            "update_err": normwise(th1 - th0, srv.theta - th0),
+            "grad_err": normwise(g_gpu, g_ref),
+            "tensor_grad_err": {n: normwise(g_gpu[sl], g_ref[sl]) for n, sl in slices},
+        }
+    return rec
