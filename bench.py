@@ -9,9 +9,12 @@ turned on uploads its next batch into the freed HBM slot (Algorithm 2 with
 the flow control of Sec. 3.4.1), and one device-side model is aggregated
 FedAsync-style (Algorithm 4, aggregation branch).
 
-Workload: the VGG-style server part (10 devices, bf16 activations
-[64,128,16,16], 8,625,162 parameters; device model 1,000,000 fp32
-parameters), with synthetic seeded inputs.  Prints one JSON line.
+Headline workload: the transformer server part (16 devices, bf16 hidden
+states [32,128,512] with lengths 32..128, 4 pre-LN encoder blocks, 12,611,586
+parameters; device model 21,932,032 fp32 parameters), the largest of the
+workloads in FLOPs per step.  The same run also measures the VGG-style,
+ResNet-18-style, 100-device scale and MobileNetV3 server parts
+("workloads").  All inputs are synthetic and seeded.  Prints one JSON line.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -33,17 +36,18 @@ sys.path.insert(0, ROOT)
 
 METRIC = "server-side train samples/s at 1 GB300; % bf16 tensor peak; aggregation HBM GB/s"
 UNIT = "samples/s"
-WORKLOAD = "vgg"
-WORKLOAD_DESC = ("VGG-style server part: 10 devices, bf16 activations [64,128,16,16] = ReLU(N(0,1)), "
-                 "2x(conv3x3 ->256, ReLU), maxpool2, 2x(conv3x3 ->512, ReLU), maxpool2, FC 8192->512->10, "
-                 "softmax-CE, SGD lr 0.01 momentum 0.9; 1M-param device model aggregated each step")
+WORKLOAD = "transformer"
+WORKLOAD_DESC = ("Transformer encoder server part: 16 devices, bf16 activations [32,128,512] ~ N(0,1) with "
+                 "lengths 32..128, 4 pre-LN blocks (8 heads, FFN 2048, GELU), masked mean-pool, FC 512->2, "
+                 "softmax-CE, SGD lr 0.01 momentum 0.9; 21.9M-param device model aggregated each step")
+OTHER_WORKLOADS = ("vgg", "resnet", "scale", "mobilenet")
 OTHER_DESC = {
+    "vgg": "VGG-style server part: 10 devices, bf16 activations [64,128,16,16] = ReLU(N(0,1)), "
+           "2x(conv3x3 ->256, ReLU), maxpool2, 2x(conv3x3 ->512, ReLU), maxpool2, FC 8192->512->10, "
+           "softmax-CE, SGD lr 0.01 momentum 0.9; 1M-param device model aggregated each step",
     "resnet": "ResNet-18 stages 3-4 server part: 20 devices, bf16 activations [128,128,16,16] = ReLU(N(0,1)), "
               "basic blocks 128->256 (stride 2), 256, 256->512 (stride 2), 512 with folded batch norms, avgpool, "
               "FC 512->100, softmax-CE, SGD lr 0.01 momentum 0.9",
-    "transformer": "Transformer encoder server part: 16 devices, bf16 activations [32,128,512] ~ N(0,1) with "
-                   "lengths 32..128, 4 pre-LN blocks (8 heads, FFN 2048, GELU), masked mean-pool, FC 512->2, "
-                   "softmax-CE, SGD lr 0.01 momentum 0.9",
     "scale": "ResNet-18 stages 3-4 server part with 100 devices (Zipf rates), bf16 activations [64,128,16,16], "
              "omega 400, FC 512->100, softmax-CE, SGD lr 0.01 momentum 0.9",
     "mobilenet": "MobileNetV3-Large server part: 10 devices, bf16 activations [64,112,4,4] = ReLU(N(0,1)), "
@@ -72,6 +76,7 @@ def parse():
     p.add_argument("--no-agg-sweep", action="store_true")
     p.add_argument("--no-live", action="store_true",
                    help="skip the live pipeline (devices' networks training on the same GPU)")
+    p.add_argument("--no-workloads", action="store_true", help="measure the headline workload only")
     return p.parse_args()
 
 
@@ -238,157 +243,252 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+class Harness:
+    """One server of workload `name` fed like a loaded FedOptima server: every
+    device's ring backlogged, then per step one scheduled training iteration,
+    one upload by a device whose sender is on (Poisson arrival order), and
+    one FedAsync aggregation of a device model."""
+
+    def __init__(self, name, dev, rank=0):
+        import numpy as np
+        import torch
+        from paper_2504_13850_gb300 import api
+        from paper_2504_13850_gb300 import workloads as W
+        self.np, self.torch, self.api = np, torch, api
+        self.cfg = cfg = W.CONFIGS[name]
+        self.dev = dev
+        self.B = cfg["batch"]
+        self.srv = api.Server.from_config(cfg)
+        self.srv.set_params(W.init_params(cfg))
+        self.stream = torch.cuda.ExternalStream(self.srv.stream(), device=dev)
+        P = 8   # resident uploaded batches
+        self.pool = []
+        for j in range(P):
+            x, bits, labels, lengths = W.device_batch(cfg, j % cfg["K"], 10_000 + j)
+            up = bits.view(np.int16) if bits is not None else x
+            self.pool.append((torch.from_numpy(np.ascontiguousarray(up)).to(dev),
+                              torch.from_numpy(labels).to(dev),
+                              None if lengths is None else torch.from_numpy(lengths).to(dev)))
+        self.n_model = cfg["agg_params"]
+        self.g_model = torch.from_numpy(W.global_model(self.n_model, cfg["seed"])).to(dev)
+        self.locals = [torch.from_numpy(W.device_model(self.n_model, cfg["seed"], j, 0)).to(dev) for j in range(2)]
+        self.order = W.arrival_order(cfg["rates"], 200_000, cfg["seed"] + rank)
+        self.pos = 0
+        self.it = 0
+        self.done = 0
+        for r in range(cfg["depth"]):
+            for k in range(cfg["K"]):
+                a, lb, ln = self.pool[(r * cfg["K"] + k) % P]
+                self.srv.enqueue_activations(k, a, lb, ln)
+        self.host = None
+
+    def next_uploader(self):
+        on = self.srv.sender_status()
+        for _ in range(100_000):
+            k = self.order[self.pos % len(self.order)]
+            self.pos += 1
+            if on[k]:
+                return k
+        return int(self.np.argmax(on))
+
+    def use_host_buffers(self):
+        """Pinned host copies of the uploads and device models (end to end)."""
+        self.host = {"batches": [(a.cpu().pin_memory(), lb.cpu().pin_memory(),
+                                  None if ln is None else ln.cpu().pin_memory()) for a, lb, ln in self.pool[:4]],
+                     "models": [m.cpu().pin_memory() for m in self.locals]}
+        b0 = self.host["batches"][0]
+        return (b0[0].numel() * b0[0].element_size() + 4 * self.B + (4 * self.B if self.cfg["seq"] else 0)
+                + 4 * self.n_model)
+
+    def step(self, host=False):
+        api = self.api
+        i = self.it
+        self.it += 1
+        rc, k, slot = self.srv.server_step()
+        assert rc == api.OK, rc
+        self.done += 1
+        u = self.next_uploader()
+        if host:
+            a, lb, ln = self.host["batches"][i % len(self.host["batches"])]
+            local = self.host["models"][i % 2]
+        else:
+            a, lb, ln = self.pool[i % len(self.pool)]
+            local = self.locals[i % 2]
+        rc, _ = self.srv.enqueue_activations(u, a, lb, ln)
+        assert rc == api.OK, rc
+        t, _ = self.srv.version()
+        rc, _ = self.srv.aggregate(self.g_model, local, u, max(0, t - 3))
+        assert rc == api.OK, rc
+        if host and self.done >= 2:
+            # every step's loss comes back to the host; step i's is read
+            # while step i + 1 runs (fo_read_losses waits for that step only)
+            self.last_loss = self.srv.read_losses(self.done - 2, 1)
+
+    def timed(self, steps, warmup, world=1, clocks=None):
+        """Device time (ms) of `steps` steps after `warmup`, CUDA events on
+        the compute stream, barrier + synchronize on both sides."""
+        torch = self.torch
+        for _ in range(warmup):
+            self.step()
+        self.srv.synchronize()
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier(world)
+        torch.cuda.synchronize()
+        k0 = self.srv.kernels_launched()
+        ev0.record(self.stream)
+        w0 = time.perf_counter()
+        for _ in range(steps):
+            self.step()
+        ev1.record(self.stream)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - w0
+        barrier(world)
+        self.srv.check_error()
+        return ev0.elapsed_time(ev1), wall, self.srv.kernels_launched() - k0
+
+    def busy(self, steps):
+        """GPU busy fraction of the step loop: the summed device time from
+        each step's first kernel to its aggregation, over the device time of
+        the whole loop (the rest is the server idling on the host)."""
+        torch = self.torch
+        self.srv.synchronize()
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        for a, b in evs:
+            a.record(self.stream)
+            self.step()
+            b.record(self.stream)
+        torch.cuda.synchronize()
+        busy = sum(a.elapsed_time(b) for a, b in evs)
+        span = evs[0][0].elapsed_time(evs[-1][1])
+        return {"busy_frac": round(busy / span, 4), "idle_ms_per_step": round((span - busy) / steps, 4),
+                "steps": steps}
+
+    def kernel_profile(self, steps):
+        """Per-kernel-class times: the same steps again with CUDA events
+        around every plan entry inside a profiled copy of the step graph (a
+        separate pass, so that the events do not perturb the timed value)."""
+        self.srv.profile(True)
+        self.srv.profile_reset()
+        self.torch.cuda.synchronize()
+        for _ in range(steps):
+            self.step()
+        kt = self.srv.kernel_times()
+        self.srv.profile(False)
+        self.srv.check_error()
+        return kt
+
+    def e2e(self, steps, warmup, world=1):
+        """The same loop through the C ABI from pinned host memory: every
+        step uploads its activations, labels (and lengths) and the device
+        model from the host, and the last step's loss is read back inside
+        the timed region."""
+        torch = self.torch
+        h2d = self.use_host_buffers()
+        self.srv.synchronize()
+        for _ in range(max(1, warmup)):
+            self.step(host=True)
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier(world)
+        torch.cuda.synchronize()
+        ev0.record(self.stream)
+        for _ in range(steps):
+            self.step(host=True)
+        self.last_loss = self.srv.read_losses(self.done - 1, 1)
+        ev1.record(self.stream)
+        torch.cuda.synchronize()
+        barrier(world)
+        return ev0.elapsed_time(ev1), h2d
+
+    def close(self):
+        self.srv.close()
+
+
+def roofline_of(ktimes, pk, which):
+    """The dominant kernel class of a step (largest total time in the
+    profiled pass): achieved = algorithmic FLOPs (bytes) / its event time."""
+    name, (nl, ms_k, fl_k, by_k) = max(ktimes.items(), key=lambda kv: kv[1][1])
+    if fl_k > 0:
+        achieved = fl_k / (ms_k / 1e3) / 1e12
+        sus = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
+        return {"kernel": name, "bound": "tensor", "achieved": round(achieved, 2), "peak": pk["bf16_tflops"],
+                "unit": "TFLOP/s", "frac": round(achieved / pk["bf16_tflops"], 4),
+                "frac_sustained": round(achieved / sus, 4), "traffic": traffic_for(name),
+                "peak_kind": f"{which} burst bf16 (sustained {sus})", "launches": nl, "ms_total": round(ms_k, 3)}
+    achieved = by_k / (ms_k / 1e3) / 1e9
+    return {"kernel": name, "bound": "hbm", "achieved": round(achieved, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
+            "frac": round(achieved / pk["hbm_gbs"], 4), "traffic": traffic_for(name), "peak_kind": f"{which} copy",
+            "launches": nl, "ms_total": round(ms_k, 3)}
+
+
+def kernels_table(ktimes):
+    return {k: {"launches": v[0], "ms": round(v[1], 3),
+                "tflops": round(v[2] / (v[1] / 1e3) / 1e12, 1) if v[2] and v[1] else None,
+                "gbs": round(v[3] / (v[1] / 1e3) / 1e9, 1) if v[3] and v[1] else None}
+            for k, v in sorted(ktimes.items(), key=lambda kv: -kv[1][1])}
+
+
+def step_fracs(ktimes, n_prof, step_ms, pk):
+    step_flops = sum(v[2] for v in ktimes.values()) / n_prof
+    tf = step_flops / (step_ms / 1e3) / 1e12
+    return step_flops, tf / pk["bf16_tflops"], tf / pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
+
+
 def run_ours(args):
-    import numpy as np
     import torch
 
     from paper_2504_13850_gb300 import api, build
-    from paper_2504_13850_gb300 import workloads as W
 
     world, rank, local = dist_setup(args.gpus)
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     build.build()
     api.lib()
-    cfg = W.CONFIGS[args.workload]
-    B, (H, Wd, C) = cfg["batch"], cfg["in_hwc"]
-    srv = api.Server.from_config(cfg)
-    srv.set_params(W.init_params(cfg))
-    stream = torch.cuda.ExternalStream(srv.stream(), device=dev)
-
-    # Resident inputs: a pool of uploaded batches and device models in HBM.
-    P = 8
-    pool = []
-    for j in range(P):
-        x, bits, labels, lengths = W.device_batch(cfg, j % cfg["K"], 10_000 + j)
-        up = bits.view(np.int16) if bits is not None else x
-        pool.append((torch.from_numpy(np.ascontiguousarray(up)).to(dev),
-                     torch.from_numpy(labels).to(dev),
-                     None if lengths is None else torch.from_numpy(lengths).to(dev)))
-    n_model = cfg["agg_params"]
-    g_model = torch.from_numpy(W.global_model(n_model, cfg["seed"])).to(dev)
-    locals_ = [torch.from_numpy(W.device_model(n_model, cfg["seed"], j, 0)).to(dev) for j in range(2)]
-    order = W.arrival_order(cfg["rates"], 200_000, cfg["seed"] + rank)
-    pos = [0]
-
-    def next_uploader():
-        on = srv.sender_status()
-        for _ in range(100_000):
-            k = order[pos[0] % len(order)]
-            pos[0] += 1
-            if on[k]:
-                return k
-        return int(np.argmax(on))
-
-    # Backlog: every device fills its ring (the steady state of a loaded server).
-    for r in range(cfg["depth"]):
-        for k in range(cfg["K"]):
-            a, lb, ln = pool[(r * cfg["K"] + k) % P]
-            srv.enqueue_activations(k, a, lb, ln)
-
-    it = [0]
-    done = [0]                      # server steps run so far (loss ring index)
-
-    def step(host=None):
-        i = it[0]
-        it[0] += 1
-        rc, k, slot = srv.server_step()
-        assert rc == api.OK, rc
-        done[0] += 1
-        u = next_uploader()
-        if host is None:
-            a, lb, ln = pool[i % P]
-            rc, _ = srv.enqueue_activations(u, a, lb, ln)
-            local = locals_[i % 2]
-        else:
-            a, lb, ln = host["batches"][i % len(host["batches"])]
-            rc, _ = srv.enqueue_activations(u, a, lb, ln)
-            # the device model comes up on a copy stream into one of two
-            # staging buffers, after the aggregation that last read it
-            b = i % 2
-            cs = host["copy"]
-            cs.wait_event(host["read"][b])
-            with torch.cuda.stream(cs):
-                host["stage"][b].copy_(host["models"][b], non_blocking=True)
-                host["landed"][b].record(cs)
-            stream.wait_event(host["landed"][b])
-            local = host["stage"][b]
-        assert rc == api.OK, rc
-        t, _ = srv.version()
-        rc, _ = srv.aggregate(g_model, local, u, max(0, t - 3))
-        assert rc == api.OK, rc
-        if host is not None:
-            host["read"][i % 2].record(stream)
-            # every step's loss comes back to the host; step i's is read while
-            # step i + 1 runs (fo_read_losses waits for that step only)
-            if done[0] >= 2:
-                host["loss"] = srv.read_losses(done[0] - 2, 1)
+    pk, which = peaks()
+    h = Harness(args.workload, dev, rank)
+    cfg, B = h.cfg, h.B
 
     # ---------------- device-resident timed region
-    for _ in range(args.warmup):
-        step()
-    srv.synchronize()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clk:
-        barrier(world)
-        torch.cuda.synchronize()
-        k0 = srv.kernels_launched()
-        ev0.record(stream)
-        w0 = time.perf_counter()
-        for _ in range(args.steps):
-            step()
-        ev1.record(stream)
-        torch.cuda.synchronize()
-        wall = time.perf_counter() - w0
-        barrier(world)
-    srv.check_error()
-    ms_dev = ev0.elapsed_time(ev1)
-    launches = srv.kernels_launched() - k0
+        ms_dev, wall, launches = h.timed(args.steps, args.warmup, world)
     ms_max = max_over_ranks(world, ms_dev, dev)
     samples = sum_over_ranks(world, float(args.steps * B), dev)
     value = samples / (ms_max / 1e3)
 
-    # ---------------- per-kernel times: the same steps again, each launch
-    # bracketed by CUDA events on the compute stream (a separate timed region,
-    # so the events do not perturb the value above)
     n_prof = min(args.steps, 200)
-    srv.profile(True)
-    srv.profile_reset()
-    torch.cuda.synchronize()
-    for _ in range(n_prof):
-        step()
-    ktimes = srv.kernel_times()
-    srv.profile(False)
-    srv.check_error()
+    ktimes = h.kernel_profile(n_prof)
+    busy = h.busy(min(args.steps, 200))
 
     # ---------------- end to end through the C ABI from pinned host memory
     e2e = None
     if not args.no_e2e:
-        host = {"batches": [], "models": [], "stage": [torch.empty(n_model, device=dev) for _ in range(2)],
-                "copy": torch.cuda.Stream(device=dev), "landed": [torch.cuda.Event() for _ in range(2)],
-                "read": [torch.cuda.Event() for _ in range(2)]}
-        for a, lb, ln in pool[:4]:
-            host["batches"].append((a.cpu().pin_memory(), lb.cpu().pin_memory(),
-                                    None if ln is None else ln.cpu().pin_memory()))
-        host["models"] = [m.cpu().pin_memory() for m in locals_]
-        h2d = (host["batches"][0][0].numel() * host["batches"][0][0].element_size() + 4 * B
-               + (4 * B if cfg["seq"] else 0) + 4 * n_model)
-        srv.synchronize()
-        for _ in range(max(1, args.warmup)):
-            step(host)
         n_e2e = min(args.steps, 100)
-        barrier(world)
-        torch.cuda.synchronize()
-        ev0.record(stream)
-        for _ in range(n_e2e):
-            step(host)
-        host["loss"] = srv.read_losses(done[0] - 1, 1)   # the last step's loss, inside the timed region
-        ev1.record(stream)
-        torch.cuda.synchronize()
-        barrier(world)
-        ms_e = max_over_ranks(world, ev0.elapsed_time(ev1), dev)
+        ms_e, h2d = h.e2e(n_e2e, args.warmup, world)
+        ms_e = max_over_ranks(world, ms_e, dev)
         e2e = {"value": sum_over_ranks(world, float(n_e2e * B), dev) / (ms_e / 1e3), "unit": UNIT,
-               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": 4}
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": 4, "steps": n_e2e}
+    wsb = h.srv.device_bytes()
+    h.close()
+    del h
+    torch.cuda.empty_cache()
+
+    # ---------------- the other workloads, same loop, one after another
+    others = {}
+    if not args.no_workloads and args.workload == WORKLOAD:
+        n_w = min(args.steps, 300)
+        for name in OTHER_WORKLOADS:
+            hw = Harness(name, dev, rank)
+            ms_w, _, _ = hw.timed(n_w, args.warmup, world)
+            ms_w = max_over_ranks(world, ms_w, dev)
+            kt = hw.kernel_profile(min(n_w, 50))
+            fl, fb, fs = step_fracs(kt, min(n_w, 50), ms_w / n_w, pk)
+            others[name] = {"workload": workload_desc(name), "value": round(sum_over_ranks(world, float(n_w * hw.B), dev)
+                                                                             / (ms_w / 1e3), 1),
+                            "unit": UNIT, "steps": n_w, "ms_per_step": round(ms_w / n_w, 4),
+                            "step_gflop": round(fl / 1e9, 2), "step_tensor_frac_burst": round(fb, 4),
+                            "step_tensor_frac_sustained": round(fs, 4), "roofline": roofline_of(kt, pk, which)}
+            hw.close()
+            del hw
+            torch.cuda.empty_cache()
 
     # ---------------- aggregation bandwidth sweep (standalone FedAsync update)
     agg = None
@@ -397,17 +497,18 @@ def run_ours(args):
         try:
             ga = torch.randn(n, device=dev) * 0.05
             la = torch.randn(n, device=dev) * 0.05
-            pk, which = peaks()
+            st = torch.cuda.Stream(device=dev)
+            ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             sweep = []
             for m in (1_000_000, 4_000_000, 16_000_000, 64_000_000, n):
                 g_m, l_m = ga[:m], la[:m]
                 for _ in range(3):
-                    api.axpby_async(g_m, l_m, 0.25, srv.stream())
+                    api.axpby_async(g_m, l_m, 0.25, st.cuda_stream)
                 best = 1e30
                 for _ in range(10):
-                    ev0.record(stream)
-                    api.axpby_async(g_m, l_m, 0.25, srv.stream())
-                    ev1.record(stream)
+                    ev0.record(st)
+                    api.axpby_async(g_m, l_m, 0.25, st.cuda_stream)
+                    ev1.record(st)
                     torch.cuda.synchronize()
                     best = min(best, ev0.elapsed_time(ev1))
                 # 12 bytes per parameter; below ~126 MB of traffic the vectors stay in L2
@@ -424,26 +525,8 @@ def run_ours(args):
 
     if rank != 0:
         return
-    pk, which = peaks()
-    # dominant kernel class of the step, by total time
-    dom = max(ktimes.items(), key=lambda kv: kv[1][1])
-    name, (nl, ms_k, fl_k, by_k) = dom
-    if fl_k > 0:
-        peak = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
-        achieved = fl_k / (ms_k / 1e3) / 1e12
-        roof = {"kernel": name, "bound": "tensor", "achieved": round(achieved, 2), "peak": peak,
-                "unit": "TFLOP/s", "frac": round(achieved / peak, 4), "traffic": traffic_for(name),
-                "peak_kind": f"{which} sustained bf16", "launches": nl, "ms_total": round(ms_k, 3)}
-    else:
-        peak = pk["hbm_gbs"]
-        achieved = by_k / (ms_k / 1e3) / 1e9
-        roof = {"kernel": name, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
-                "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": traffic_for(name),
-                "peak_kind": f"{which} copy", "launches": nl, "ms_total": round(ms_k, 3)}
-    step_flops = sum(v[2] for v in ktimes.values()) / n_prof
-    step_ms = ms_dev / args.steps
-    tensor_frac = step_flops / (step_ms / 1e3) / 1e12 / pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
-    tensor_frac_burst = step_flops / (step_ms / 1e3) / 1e12 / pk["bf16_tflops"]
+    roof = roofline_of(ktimes, pk, which)
+    step_flops, tensor_frac_burst, tensor_frac = step_fracs(ktimes, n_prof, ms_dev / args.steps, pk)
     cpu = None
     if not args.no_cpu_baseline and world == 1:
         v_cpu, n_cpu, dt_cpu = oracle_sample(cfg, B)
@@ -451,10 +534,9 @@ def run_ours(args):
                "sample": f"{n_cpu} oracle server steps at batch {B} ({dt_cpu:.1f} s, numpy fp64, BLAS threads = cores)"}
     from paper_2504_13850_gb300 import study
     sched = study.scheduler_balance("scale", uploads=6000)   # host-only: counter vs FIFO scheduling
-    wsb = srv.device_bytes()
     live_line = None
-    if rank == 0 and not args.no_live and args.workload == "vgg":
-        # a second workload: the VGG-style split with every device's network
+    if rank == 0 and not args.no_live:
+        # a second pipeline: the VGG-style split with every device's network
         # training on the same GPU and feeding the server (measured after the
         # timed region, so it does not perturb `value`)
         try:
@@ -469,13 +551,16 @@ def run_ours(args):
         "config": {"workload": workload_desc(args.workload), "global_batch": B * world, "devices": cfg["K"],
                    "omega": cfg["omega"], "parallelism": f"replicas{world}",
                    "l2": f"not flushed: each step touches the server's {wsb / 1e6:.0f} MB of parameters, "
-                         f"momentum, gradients, activations and scratch, above the 126 MB L2"},
+                         f"momentum, gradients, activations and scratch, above the 126 MB L2",
+                   "switches": {k: os.environ.get(k) for k in ("FO_NO_TC", "FO_NO_GRAPH", "FO_NO_SIDE", "FO_NO_PDL")}},
         "e2e": e2e,
         "gpu_launches": int(launches),
         "roofline": roof,
         "step_tensor_frac": round(tensor_frac, 4),
         "step_tensor_frac_burst": round(tensor_frac_burst, 4),
         "step_gflop": round(step_flops / 1e9, 2),
+        "server_busy": busy,
+        "workloads": others or None,
         "aggregation": agg,
         "scheduler_balance": sched,
         "live_pipeline": live_line,
@@ -483,10 +568,7 @@ def run_ours(args):
         "clocks": clk.summary(),
         "host_wall_ms_per_step": round(1e3 * wall / args.steps, 4),
         "kernels_profiled_steps": n_prof,
-        "kernels": {k: {"launches": v[0], "ms": round(v[1], 3),
-                        "tflops": round(v[2] / (v[1] / 1e3) / 1e12, 1) if v[2] and v[1] else None,
-                        "gbs": round(v[3] / (v[1] / 1e3) / 1e9, 1) if v[3] and v[1] else None}
-                    for k, v in sorted(ktimes.items(), key=lambda kv: -kv[1][1])},
+        "kernels": kernels_table(ktimes),
     }
     print(json.dumps(line), flush=True)
 

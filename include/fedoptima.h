@@ -220,7 +220,12 @@ FO_API int fo_read_losses(fo_server* s, float* host_out, int64_t first_step, int
  * n floats, read only) is theta_dk || theta~_dk trained from version t_k =
  * `version`.  FO_STALE when t - version > D (global and t unchanged).
  * FO_ERR_ARG when version < 0 or version > t.  Runs on the server's compute
- * stream, ordered after earlier steps. */
+ * stream, ordered after earlier steps.  `local` may also be host memory
+ * (page-locked for an asynchronous copy): it is then copied into one of two
+ * server-owned device buffers on the upload stream, overlapping the steps
+ * already queued, and the call returns once that copy has landed, so the
+ * caller may reuse its buffer at once; the buffers grow to the largest n
+ * seen (FO_ERR_OOM if that fails). */
 FO_API int fo_aggregate(fo_server* s, float* global, const float* local, int64_t n,
                  int device_id, int32_t version, int32_t* new_version);
 
@@ -322,7 +327,8 @@ FO_API int fo_axpby_async(float* global, const float* local, int64_t n, float al
  * in a fixed order, so results are bitwise reproducible.  The partial sums
  * live in scratch this call allocates and frees stream-ordered on `stream`
  * (a cudaStream_t, NULL = default stream).  FO_ERR_ARG for rows < 1,
- * cols < 1 or an unknown dtype.
+ * cols < 1, an unknown dtype, or more than 65,535 chunks of 128 rows
+ * (rows > 8,388,480: the chunks are one grid dimension).
  * ---------------------------------------------------------------------- */
 FO_API int fo_column_sums(const void* x, int dtype, int64_t rows, int cols, float* out, void* stream);
 
@@ -356,8 +362,9 @@ FO_API int fo_select_split(const double* O, const double* S, int L, const double
  * Same arguments, result and determinism as fo_column_sums; the partial
  * sums go to one fixed device array of 262,144 floats (1 MiB) that the
  * library holds on every GPU it is loaded on until the process exits.
- * Limit: ceil(rows / 128) * cols <= 262,144 (e.g. 65,536 rows x 512 columns);
- * larger inputs return FO_ERR_ARG with the reason in fo_last_error().
+ * Limits: ceil(rows / 128) * cols <= 262,144 (e.g. 65,536 rows x 512
+ * columns) and ceil(rows / 128) <= 65,535 (as for fo_column_sums); larger
+ * inputs return FO_ERR_ARG with the reason in fo_last_error().
  * The first call on a device looks up the array's device address (once per
  * device, with that device current); make that first call before any stream
  * capture.  All calls share the array, and it keeps the last call's

@@ -240,7 +240,8 @@ class Server:
         return out
 
     def aggregate(self, global_, local, device_id, version):
-        """Returns (status, new_version); global_/local are device buffers."""
+        """Returns (status, new_version); global_ is a device buffer, local a
+        device or host buffer (a host model is copied in by the library)."""
         nv = C.c_int32(-1)
         n = global_.numel() if hasattr(global_, "numel") else global_.size
         rc = lib().fo_aggregate(self.h, _ptr(global_), _ptr(local), n, device_id, version,

@@ -19,7 +19,7 @@ CSRC = os.path.join(HERE, "csrc")
 OUT = os.path.join(HERE, "libfedoptima.so")
 BUILD = os.path.join(HERE, "_build")
 
-SOURCES = ["fo_server.cu", "k_elementwise.cu", "k_simt_conv.cu", "k_attention.cu", "k_tc_gemm.cu", "k_head.cu", "k_vec.cu", "fo_noalloc.cu", "k_attention_tc.cu", "fo_preproc.cu", "k_mobile.cu"]
+SOURCES = ["fo_server.cu", "k_elementwise.cu", "k_simt_conv.cu", "k_attention.cu", "k_tc_gemm.cu", "k_tc_gemm_fwd.cu", "k_tc_gemm_dgrad.cu", "k_tc_gemm_wgrad.cu", "k_head.cu", "k_vec.cu", "fo_noalloc.cu", "k_attention_tc.cu", "fo_preproc.cu", "k_mobile.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
          "-Xcompiler", "-fvisibility=hidden"]

@@ -66,6 +66,9 @@ void layernorm_bwd_dx(const void* x, const float* gamma, const float* mean, cons
 // (128-row chunks); the server passes adaptive = true (chunks sized to the
 // GPU, scratch from server_colsum_floats).
 int64_t colsum_partial_floats(int64_t rows, int C);
+// Most rows the public column sums take: their row chunks (128 rows each)
+// are one grid dimension, at most 65,535 blocks.
+constexpr int64_t kColsumMaxRows = int64_t(65535) * 128;
 int64_t server_colsum_floats(int64_t rows, int C);
 void colsum(const void* a, const void* b, int64_t rows, int C, int dt, float* partial,
             float* out, cudaStream_t st, bool adaptive = false);
@@ -160,13 +163,19 @@ bool layernorm_fwd8_ok(int dt, int C);
 void layernorm_fwd_x8(const void* x, const float* gamma, const float* beta, void* y, float* mean, float* rstd,
                       int64_t rows, int C, cudaStream_t st);
 // Layernorm backward fused with dgamma / dbeta (C % 256 == 0, C <= 512).
+// Masked mean-pool over tokens and its gradient, 8 bf16 columns per access.
+bool meanpool8_ok(int dt, int C);
+void meanpool_fwd_x8(const void* x, const int32_t* len, void* y, int B, int L, int C, cudaStream_t st);
+void meanpool_bwd_x8(const void* dy, const int32_t* len, void* dx, int B, int L, int C, bool acc, cudaStream_t st);
 bool layernorm_bwd8_ok(int dt, int C);
 int64_t layernorm_bwd8_partial_floats(int64_t rows, int C);
 // The same pass without its finish: partials [layernorm_bwd8_blocks(rows), C]
 // of dgamma and dbeta.
 int layernorm_bwd8_blocks(int64_t rows);
+// dx = (dx if acc) + input gradient + (addend if given, dx's layout).
 void layernorm_bwd8_pass(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
-                         void* dx, int64_t rows, int C, bool acc, float* p_gamma, float* p_beta, cudaStream_t st);
+                         void* dx, int64_t rows, int C, bool acc, float* p_gamma, float* p_beta, cudaStream_t st,
+                         const void* addend = nullptr);
 
 // ---- MobileNetV3 bottleneck (k_mobile.cu) ----
 // Depthwise k x k convolution, NHWC, weights [C][k][k] in the activation

@@ -55,6 +55,9 @@ int scratch_address(float** out) {
 extern "C" int fo_column_sums_noalloc(const void* x, int dtype, int64_t rows, int cols, float* out, void* stream) {
   if (!x || !out || rows < 1 || cols < 1 || (dtype != FO_DTYPE_F32 && dtype != FO_DTYPE_BF16))
     return fo::report_error(FO_ERR_ARG, "bad column-sum arguments");
+  if (rows > fo::kColsumMaxRows)
+    return fo::report_error(FO_ERR_ARG, "fo_column_sums_noalloc: " + std::to_string(rows) + " rows exceed " +
+                                            std::to_string(fo::kColsumMaxRows) + " (65,535 chunks of 128 rows)");
   const int64_t need = fo::colsum_partial_floats(rows, cols);
   if (need > kScratchFloats)
     return fo::report_error(FO_ERR_ARG, "fo_column_sums_noalloc: ceil(rows / 128) * cols = " + std::to_string(need) +

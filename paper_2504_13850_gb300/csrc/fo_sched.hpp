@@ -39,6 +39,16 @@ class TaskScheduler {
   const std::vector<uint8_t>& sender_on() const { return on_; }
   bool active(int k) const { return active_[k] != 0; }
 
+  // What put(k) would do, without changing any state: 0 = it would accept
+  // (slot set to the slot it would hand out), 2 = it would refuse, -1 = bad
+  // argument.  Lets a caller fill the slot before committing the upload.
+  int peek(int k, int32_t* slot) const {
+    if (k < 0 || k >= K_ || !active_[k]) return -1;
+    if (total_ >= omega_ || len_[k] >= depth_) return 2;
+    *slot = free_[free_head_];
+    return 0;
+  }
+
   // put(): returns 0 = accepted (slot set), 2 = refused (cap/depth), -1 bad arg.
   int put(int k, int32_t* slot) {
     if (k < 0 || k >= K_ || !active_[k]) return -1;

@@ -207,6 +207,13 @@ struct Fusion {
   std::vector<int> hswish_by;  // hard swish op -> the affine op that applies it, or -1
   std::vector<int> add_relu;   // residual add op -> the relu after it, whose backward the add's applies, or -1
   std::vector<int> relu_into_add;  // that relu op -> the add op, or -1
+  // Residual add whose branch ends in a plain tensor-core GEMM: the GEMM's
+  // epilogue writes branch + residual straight into the add's output, the
+  // branch's gradient is the add's output gradient itself (one buffer), and
+  // the residual's gradient joins its next contribution as an addend.
+  std::vector<int> add_into;   // producer op -> the add op whose output it writes, or -1
+  std::vector<int> add_other;  // that add op -> its residual operand tensor
+  std::vector<int> branch_of;  // that add op -> its branch tensor, or -1
   bool head = false;           // last linear + loss handled by the head kernels
 };
 
@@ -226,6 +233,9 @@ Fusion analyse(const fo_server* s) {
   f.hswish_by.assign(nops, -1);
   f.add_relu.assign(nops, -1);
   f.relu_into_add.assign(nops, -1);
+  f.add_into.assign(nops, -1);
+  f.add_other.assign(nops, -1);
+  f.branch_of.assign(nops, -1);
   std::vector<int> sole(nops + 1, -1);  // the only consumer op of a tensor
   for (int j = 0; j < nops; ++j) {
     const fo_op& op = s->ops[j];
@@ -276,6 +286,23 @@ Fusion analyse(const fo_server* s) {
       f.skip_fwd[h] = 1;
     }
   }
+  const int L = nops - 1;
+  auto plain = [&](int j) { return fo::tc_plain_ok(s->tc, s, j) && !(f.head && j == L); };
+  for (int a = 0; a < nops; ++a) {
+    const fo_op& op = s->ops[a];
+    if (op.kind != FO_OP_ADD || f.fwd_relu[a] >= 0 || f.add_relu[a] >= 0) continue;
+    for (int t : {op.in1, op.in0}) {
+      const int other = t == op.in1 ? op.in0 : op.in1;
+      if (t == 0 || s->T[t].root != t || s->T[t].root == s->T[other].root || sole[t] != a) continue;
+      const int p = t - 1;
+      if (!plain(p) || f.fwd_relu[p] >= 0) continue;
+      f.add_into[p] = a;
+      f.add_other[a] = other;
+      f.branch_of[a] = t;
+      f.skip_fwd[a] = 1;
+      break;
+    }
+  }
   return f;
 }
 
@@ -294,6 +321,8 @@ int build_plan(fo_server* s) {
   for (fo::AttnTcPlan* a : s->attn_tc) fo::attention_tc_destroy(a);
   s->attn_tc.assign(nops, nullptr);
   const Fusion fu = analyse(s);
+  for (int i = 0; i < nops; ++i)   // a fused residual's branch shares the add's output gradient
+    if (fu.branch_of[i] >= 0) s->T[fu.branch_of[i]].grad = s->T[i + 1].grad;
   auto act = [s](int tid) -> const void* { return tid == 0 ? s->cur_in : s->T[tid].act; };
   auto add = [&plan](const char* name, int kernels, double flops, double bytes,
                      std::function<void(cudaStream_t)> fn, int lane = 0) {
@@ -311,8 +340,9 @@ int build_plan(fo_server* s) {
     const fo_op op = s->ops[i];
     if (fu.skip_fwd[i]) continue;
     const int a = op.in0;
-    // output buffer: a fused relu writes the relu's output tensor
-    const int o = fu.fwd_relu[i] >= 0 ? fu.fwd_relu[i] + 1 : i + 1;
+    // output buffer: a fused relu writes the relu's output tensor, a fused
+    // residual add the add's output
+    const int o = fu.fwd_relu[i] >= 0 ? fu.fwd_relu[i] + 1 : (fu.add_into[i] >= 0 ? fu.add_into[i] + 1 : i + 1);
     const bool relu = fu.fwd_relu[i] >= 0;
     const Tensor& ta = s->T[a];
     const Tensor& to = s->T[i + 1];
@@ -338,7 +368,15 @@ int build_plan(fo_server* s) {
         fo::ConvShape cs = conv_shape(s, i);
         const bool bias = op.bias != 0;
         const double fl = 2.0 * double(to.rows()) * op.cout * double(op.kind == FO_OP_CONV ? op.k * op.k : 1) * op.cin;
-        fo::TcGemm* tg = fo::tc_plan_forward(s->tc, s, i, s->T[o].act, relu);
+        fo::TcEpilogue ex;
+        const bool fused = fu.add_into[i] >= 0;
+        if (fused) {
+          const int r = fu.add_other[fu.add_into[i]];
+          if (r == 0) ex.addend_is_input = true;
+          else ex.addend = s->T[r].act;
+        }
+        fo::TcGemm* tg = fo::tc_plan_forward(s->tc, s, i, s->T[o].act, relu, fused ? &ex : nullptr);
+        if (fused && !tg) return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": fused epilogue not planned");
         if (tg) {
           add_tc(tg);
         } else {
@@ -473,11 +511,39 @@ int build_plan(fo_server* s) {
   written[nops] = 1;  // dlogits
   // Contribution to tensor `tid`'s gradient: returns the accumulate flag
   // and marks the root written; tensor 0 receives none.
+  // A fused residual add leaves the residual operand's first contribution
+  // (the add's output gradient) pending: root -> tensor whose gradient is
+  // still to be added.  The next contributor that can add it in its own
+  // epilogue takes it as an addend; any other contributor, and any kernel
+  // that reads the gradient, first has it copied in.
+  std::vector<int> pending(nops + 1, -1);
+  auto materialize = [&](int tid) {
+    const int r = s->T[tid].root;
+    if (pending[r] < 0) return;
+    const int src = pending[r];
+    pending[r] = -1;
+    const int64_t n = s->T[r].numel();
+    add("add_bwd", 1, 0.0, 2 * tbytes(r), [=](cudaStream_t st) {
+      fo::grad_split(s->T[src].grad, nullptr, s->T[r].grad, false, nullptr, false, n, dt, st);
+    });
+  };
   auto contrib = [&](int tid) -> int {
+    materialize(tid);
     int r = s->T[tid].root;
     int accf = written[r] ? 1 : 0;
     written[r] = 1;
     return accf;
+  };
+  // A contribution whose kernel adds `*addend` (a pending gradient) itself.
+  auto contrib_addend = [&](int tid, const void** addend) -> int {
+    const int r = s->T[tid].root;
+    *addend = nullptr;
+    if (pending[r] >= 0) {
+      *addend = s->T[pending[r]].grad;
+      pending[r] = -1;
+      return 0;
+    }
+    return contrib(tid);
   };
   // Parameter-gradient reductions deferred to two batched launches after the
   // backward pass: column sums for the conv / linear biases, and the finish
@@ -499,11 +565,13 @@ int build_plan(fo_server* s) {
     if (fu.hswish_by[i] >= 0 || fu.relu_into_add[i] >= 0) {
       // the producer's backward applies this hard swish / relu: its input
       // gradient is present exactly when the output's is
+      materialize(i + 1);   // the producer's backward reads this op's output gradient
       written[s->T[op.in0].root] = written[s->T[i + 1].root];
       continue;
     }
     const int a0 = op.in0, o = i + 1;
     const int ro = s->T[o].root;
+    materialize(o);   // this op's backward reads its output gradient
     if (!written[ro]) {
       // Nothing downstream produced a gradient: zero this op's parameter grads.
       for (int si : s->op_segs[i]) {
@@ -567,10 +635,19 @@ int build_plan(fo_server* s) {
           }, 1);
         }
         if (need_dx) {
-          int accf = contrib(a);
+          const void* addend = nullptr;
+          const bool plain = fo::tc_plain_ok(s->tc, s, i);
+          int accf = plain ? contrib_addend(a, &addend) : contrib(a);
+          fo::TcEpilogue ex;
+          ex.addend = addend;
+          const bool fused = addend != nullptr;
           std::vector<fo::TcGemm*> tgs;
           bool zero_first = false;
-          if (fo::tc_plan_dgrad(s->tc, s, i, accf, s->T[a].grad, mask, &tgs, &zero_first)) {
+          const bool planned = fo::tc_plan_dgrad(s->tc, s, i, accf, s->T[a].grad, mask, &tgs, &zero_first,
+                                                 fused ? &ex : nullptr);
+          if (fused && !planned)
+            return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": fused input gradient not planned");
+          if (planned) {
             if (zero_first) {
               const int ta = a;
               add("memset_dx", 1, 0.0, tbytes(ta), [=](cudaStream_t st) {
@@ -658,6 +735,25 @@ int build_plan(fo_server* s) {
         }
         break;
       case FO_OP_ADD: {
+        if (fu.branch_of[i] >= 0) {
+          // the branch's gradient is this gradient (the same buffer); the
+          // residual's is left pending for its next contributor
+          written[s->T[fu.branch_of[i]].root] = 1;
+          const int x = fu.add_other[i];
+          if (x == 0) break;
+          const int rx = s->T[x].root;
+          if (!written[rx]) {
+            pending[rx] = o;
+            written[rx] = 1;
+          } else {
+            materialize(x);
+            const int64_t n = s->T[o].numel();
+            add("add_bwd", 1, 0.0, 3 * csb, [=](cudaStream_t st) {
+              fo::grad_split(s->T[o].grad, nullptr, s->T[x].grad, true, nullptr, false, n, dt, st);
+            });
+          }
+          break;
+        }
         // one pass over the output gradient (masked by the relu after the
         // add when that relu's backward is folded in) into both inputs
         const int b = op.in1;
@@ -702,7 +798,8 @@ int build_plan(fo_server* s) {
         break;  // shares the input's gradient buffer
       case FO_OP_LAYERNORM:
         if (fo::layernorm_bwd8_ok(dt, s->T[a0].C)) {
-          const int accf = need_dx ? contrib(a) : 0;
+          const void* addend = nullptr;
+          const int accf = need_dx ? contrib_addend(a, &addend) : 0;
           const Tensor& x0 = s->T[a0];
           const int blocks = fo::layernorm_bwd8_blocks(x0.rows());
           float* pg = (float*)s->alloc(size_t(2) * blocks * x0.C * 4);
@@ -710,10 +807,10 @@ int build_plan(fo_server* s) {
           float* pb = pg + size_t(blocks) * x0.C;
           finish_tasks.push_back({pg, G(s, i, 0), blocks, x0.C});
           finish_tasks.push_back({pb, G(s, i, 1), blocks, x0.C});
-          add("layernorm_bwd", 1, 0.0, (need_dx ? 3 + accf : 2) * csb, [=](cudaStream_t st) {
+          add("layernorm_bwd", 1, 0.0, (need_dx ? 3 + accf + (addend ? 1 : 0) : 2) * csb, [=](cudaStream_t st) {
             const Tensor& x = s->T[a0];
             fo::layernorm_bwd8_pass(act(a0), P(s, i, 0), s->ln_mean[i], s->ln_rstd[i], s->T[o].grad,
-                                    need_dx ? s->T[a].grad : nullptr, x.rows(), x.C, accf != 0, pg, pb, st);
+                                    need_dx ? s->T[a].grad : nullptr, x.rows(), x.C, accf != 0, pg, pb, st, addend);
           });
           break;
         }
@@ -823,6 +920,8 @@ int build_plan(fo_server* s) {
       }
     }
   }
+
+  for (int r = 0; r <= nops; ++r) materialize(r);
 
   // ---------------- optimizer (Algorithm 4: theta_s <- theta_s - gamma_s * update)
   if (!bias_tasks.empty())
@@ -995,6 +1094,11 @@ void destroy_impl(fo_server* s) {
   if (s->side) cudaStreamSynchronize(s->side);
   if (s->opt_st) cudaStreamSynchronize(s->opt_st);
   for (void* p : s->allocs) cudaFree(p);
+  for (int b = 0; b < 2; ++b) {
+    if (s->agg_stage[b]) cudaFree(s->agg_stage[b]);
+    if (s->agg_landed[b]) cudaEventDestroy(s->agg_landed[b]);
+    if (s->agg_read[b]) cudaEventDestroy(s->agg_read[b]);
+  }
   if (s->cs) cudaStreamDestroy(s->cs);
   if (s->xs) cudaStreamDestroy(s->xs);
   if (s->hs) cudaStreamDestroy(s->hs);
@@ -1239,16 +1343,10 @@ int fo_server_store_params_device(fo_server* s, float* dst, int64_t n) {
   return FO_OK;
 }
 
-int fo_enqueue_activations(fo_server* s, int device_id, const void* acts, const int32_t* labels,
-                           const int32_t* lengths, int* sender_on) {
-  if (!s || !acts || !labels) return set_err(FO_ERR_ARG, "null argument");
-  if (s->cfg.seq && !lengths) return set_err(FO_ERR_ARG, "lengths required for sequence batches");
-  if (device_id < 0 || device_id >= s->cfg.num_devices) return set_err(FO_ERR_ARG, "bad device id");
-  int32_t slot = -1;
-  int rc = s->sched->put(device_id, &slot);
-  if (sender_on) *sender_on = s->sched->sender_on()[device_id];
-  if (rc == -1) return set_err(FO_ERR_ARG, "device has left");
-  if (rc == 2) return FO_FULL;
+// The copies of an accepted upload into batch slot `slot` (before the
+// scheduler commits it).
+static int upload_copies(fo_server* s, int32_t slot, const void* acts, const int32_t* labels,
+                         const int32_t* lengths) {
   const int B = s->cfg.batch;
   char* d_act = s->slab + size_t(slot) * s->slot_stride;
   int32_t* d_lab = s->slot_labels + size_t(slot) * B;
@@ -1286,6 +1384,31 @@ int fo_enqueue_activations(fo_server* s, int device_id, const void* acts, const 
   FO_CUDA(cudaEventRecord(s->slot_ready[slot], s->xs));
   // The caller may reuse its buffers once its own copy is done.
   FO_CUDA(cudaEventSynchronize(s->stage_landed[r]));
+  return FO_OK;
+}
+
+int fo_enqueue_activations(fo_server* s, int device_id, const void* acts, const int32_t* labels,
+                           const int32_t* lengths, int* sender_on) {
+  if (!s || !acts || !labels) return set_err(FO_ERR_ARG, "null argument");
+  if (s->cfg.seq && !lengths) return set_err(FO_ERR_ARG, "lengths required for sequence batches");
+  if (device_id < 0 || device_id >= s->cfg.num_devices) return set_err(FO_ERR_ARG, "bad device id");
+  // The slot is filled first and the upload committed to Q^act_k only once
+  // its copies are issued: a failed copy leaves the scheduler as it was.
+  int32_t slot = -1;
+  const int peek = s->sched->peek(device_id, &slot);
+  if (peek == 0) {
+    const int rc = upload_copies(s, slot, acts, labels, lengths);
+    if (rc != FO_OK) {
+      if (sender_on) *sender_on = s->sched->sender_on()[device_id];
+      return rc;
+    }
+  }
+  int32_t committed = -1;
+  const int rc = s->sched->put(device_id, &committed);
+  if (sender_on) *sender_on = s->sched->sender_on()[device_id];
+  if (rc == -1) return set_err(FO_ERR_ARG, "device has left");
+  if (rc == 2) return FO_FULL;
+  if (committed != slot) return set_err(FO_ERR_ARG, "scheduler slot changed between peek and put");
   return FO_OK;
 }
 
@@ -1401,6 +1524,41 @@ int fo_aggregate(fo_server* s, float* global, const float* local, int64_t n, int
     return FO_STALE;
   }
   float alpha = 1.0f / float(s->t - version + 1);
+  cudaPointerAttributes pa{};
+  FO_CUDA(cudaPointerGetAttributes(&pa, local));
+  int stage_buf = -1;
+  if (n > 0 && pa.type != cudaMemoryTypeDevice && pa.type != cudaMemoryTypeManaged) {
+    // a host-resident local model: copied to a device buffer first
+    if (n > s->agg_stage_n) {
+      FO_CUDA(cudaStreamSynchronize(s->cs));
+      for (int b = 0; b < 2; ++b) {
+        if (s->agg_stage[b]) {
+          cudaFree(s->agg_stage[b]);
+          s->device_bytes -= s->agg_stage_n * 4;
+          s->agg_stage[b] = nullptr;
+        }
+        if (cudaMalloc(&s->agg_stage[b], size_t(n) * 4) != cudaSuccess) {
+          cudaGetLastError();
+          s->agg_stage_n = 0;
+          return set_err(FO_ERR_OOM, "aggregation staging");
+        }
+        s->device_bytes += n * 4;
+        if (!s->agg_landed[b]) {
+          FO_CUDA(cudaEventCreateWithFlags(&s->agg_landed[b], cudaEventDisableTiming));
+          FO_CUDA(cudaEventCreateWithFlags(&s->agg_read[b], cudaEventDisableTiming));
+        }
+      }
+      s->agg_stage_n = n;
+    }
+    stage_buf = int(s->agg_next++ & 1);
+    float* dst = s->agg_stage[stage_buf];
+    FO_CUDA(cudaStreamWaitEvent(s->hs, s->agg_read[stage_buf], 0));   // the aggregation that last read it
+    FO_CUDA(cudaMemcpyAsync(dst, local, size_t(n) * 4, cudaMemcpyHostToDevice, s->hs));
+    FO_CUDA(cudaEventRecord(s->agg_landed[stage_buf], s->hs));
+    FO_CUDA(cudaStreamWaitEvent(s->cs, s->agg_landed[stage_buf], 0));
+    FO_CUDA(cudaEventSynchronize(s->agg_landed[stage_buf]));   // the caller may reuse `local`
+    local = dst;
+  }
   const int nk = fo::axpby_kernels(global, local, n);
   if (s->profiling) {
     ProfRec r{prof_id(s, "fedasync_axpby"), pool_event(s), pool_event(s), nk, 0.0, 12.0 * double(n)};
@@ -1413,6 +1571,7 @@ int fo_aggregate(fo_server* s, float* global, const float* local, int64_t n, int
   }
   s->kernels_launched += nk;
   FO_CUDA(cudaGetLastError());
+  if (stage_buf >= 0) FO_CUDA(cudaEventRecord(s->agg_read[stage_buf], s->cs));
   s->t += 1;
   if (new_version) *new_version = s->t;
   return FO_OK;
@@ -1520,6 +1679,9 @@ int fo_server_error(fo_server* s) {
 int fo_column_sums(const void* x, int dtype, int64_t rows, int cols, float* out, void* stream) {
   if (!x || !out || rows < 1 || cols < 1 || (dtype != FO_DTYPE_F32 && dtype != FO_DTYPE_BF16))
     return set_err(FO_ERR_ARG, "bad column-sum arguments");
+  if (rows > fo::kColsumMaxRows)
+    return set_err(FO_ERR_ARG, "fo_column_sums: " + std::to_string(rows) + " rows exceed " +
+                                   std::to_string(fo::kColsumMaxRows) + " (65,535 chunks of 128 rows)");
   cudaStream_t st = (cudaStream_t)stream;
   float* ws = nullptr;
   FO_CUDA(cudaMallocAsync((void**)&ws, fo::colsum_partial_floats(rows, cols) * sizeof(float), st));

@@ -122,6 +122,13 @@ struct fo_server {
   // so that reading a step's loss waits for that step only.
   static constexpr int kStepEvents = 64;
   std::vector<cudaEvent_t> step_done;
+  // Device copies of host-resident local models for fo_aggregate: two
+  // buffers, so that the upload of one model overlaps the aggregation of the
+  // previous one (landed: copy done; read: the aggregation that used it).
+  float* agg_stage[2] = {nullptr, nullptr};
+  int64_t agg_stage_n = 0;
+  cudaEvent_t agg_landed[2] = {nullptr, nullptr}, agg_read[2] = {nullptr, nullptr};
+  int64_t agg_next = 0;
 
   std::vector<Launch> plan;
   int last_launches = 0;

@@ -19,17 +19,31 @@ int tc_create(TcContext** out, fo_server* s);
 void tc_destroy(TcContext* c);
 // Selects the tensor maps of batch slot `slot` for the first layer.
 void tc_set_input(TcContext* c, int slot);
+// Extra epilogue work of a GEMM with a bf16 output (all fields optional).
+struct TcEpilogue {
+  // out = result + addend: a residual add in the forward pass, or the
+  // gradient a residual connection passes around a layer in the backward
+  // pass (bf16, out's layout)
+  const void* addend = nullptr;
+  bool addend_is_input = false;   // the addend is the uploaded batch of the step's slot
+};
 // Forward of conv/linear op `op` into `out` (bf16, the op's output layout),
 // applying a ReLU when `relu`.
-TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int op, void* out, bool relu);
+TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int op, void* out, bool relu, const TcEpilogue* ex = nullptr);
 // Input gradient of op `op` into `dx` (accumulating when `accumulate`),
 // multiplied by (mask > 0) when `mask` (same layout as dx) is given.  A
 // strided convolution gives one GEMM per output-parity class; when some
 // class has no taps and this is the first contribution, *zero_first asks
 // the caller to clear dx before the GEMMs (which then accumulate).
 // Returns false when the tensor cores do not take the shape.
+// An `ex` (plain GEMMs only: linear layers and 1x1 convolutions) adds an
+// addend (then `accumulate` must be 0).
 bool tc_plan_dgrad(TcContext* c, fo_server* s, int op, int accumulate, void* dx, const void* mask,
-                   std::vector<TcGemm*>* out, bool* zero_first);
+                   std::vector<TcGemm*>* out, bool* zero_first, const TcEpilogue* ex = nullptr);
+// True when the tensor cores take op `op` as one plain GEMM (a linear layer
+// or a 1x1 stride-1 convolution on the bf16 path), so that its forward and
+// input-gradient epilogues can take a TcEpilogue.
+bool tc_plain_ok(TcContext* c, const fo_server* s, int op);
 TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int op);
 // Launches the GEMM kernel; a split-K plan runs as clusters of tc_splits(g)
 // CTAs that reduce their partial tiles through distributed shared memory.

@@ -156,7 +156,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_tc_k(const __grid_co
       tmem_ld32(trow + 32 * c, r);
 #pragma unroll
       for (int e = 0; e < 32; ++e)
-        if (32 * c + e < n) sum += expf(__uint_as_float(r[e]) * kScale - m);
+        if (32 * c + e < n) sum += __expf(__uint_as_float(r[e]) * kScale - m);
     }
     const float inv = sum > 0.f ? 1.f / sum : 0.f;
     const uint32_t p_base = smem_u32(sP);
@@ -169,7 +169,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_tc_k(const __grid_co
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
           const int j = 32 * c + 8 * g + e;
-          v[e] = j < n ? expf(__uint_as_float(r[8 * g + e]) * kScale - m) * inv : 0.f;
+          v[e] = j < n ? __expf(__uint_as_float(r[8 * g + e]) * kScale - m) * inv : 0.f;
         }
         st_shared4(p_base + (c >> 1) * kTile + sw_off(i, (c & 1) * 4 + g), pack_bf16x2(v[0], v[1]),
                    pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
@@ -309,7 +309,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_bwd_tc_k(const __grid_co
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
           const int j = 32 * c + 8 * g + e;
-          const float pj = (live && j < n) ? expf(__uint_as_float(rs[8 * g + e]) * kScale - lse) : 0.f;
+          const float pj = (live && j < n) ? __expf(__uint_as_float(rs[8 * g + e]) * kScale - lse) : 0.f;
           pv[e] = pj;
           dv[e] = pj * (__uint_as_float(rp[8 * g + e]) - D) * kScale;
         }

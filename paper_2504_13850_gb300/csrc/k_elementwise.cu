@@ -555,10 +555,12 @@ __global__ void meanpool_bwd_k(const T* dy, const int32_t* len, T* dx, int B, in
 }
 void meanpool_fwd(const void* x, const int32_t* len, void* y, int B, int L, int C, int dt,
                   cudaStream_t st) {
+  if (meanpool8_ok(dt, C)) return meanpool_fwd_x8(x, len, y, B, L, C, st);
   FO_DISPATCH(dt, T, launch_k(meanpool_fwd_k<T>, elementwise_blocks(int64_t(B) * C, 256), 256, 0, st, (const T*)x, len, (T*)y, B, L, C));
 }
 void meanpool_bwd(const void* dy, const int32_t* len, void* dx, int B, int L, int C, int dt,
                   bool acc, cudaStream_t st) {
+  if (meanpool8_ok(dt, C)) return meanpool_bwd_x8(dy, len, dx, B, L, C, acc, st);
   FO_DISPATCH(dt, T, launch_k(meanpool_bwd_k<T>, elementwise_blocks(int64_t(B) * L * C, 256), 256, 0, st, (const T*)dy, len, (T*)dx, B, L, C, acc));
 }
 

@@ -174,7 +174,7 @@ __global__ void gelu_bwd_x8_k(const bf16* __restrict__ x, const bf16* __restrict
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const float v = p.v[j];
-      const float pdf = 0.39894228040143268f * expf(-0.5f * v * v);
+      const float pdf = 0.39894228040143268f * __expf(-0.5f * v * v);   // result stored as bf16
       o.v[j] = g.v[j] * (gelu_cdf(v) + v * pdf);
     }
     if (acc) {
@@ -310,7 +310,8 @@ __global__ void __launch_bounds__(256) colsum8_batch_k(const __grid_constant__ C
 // Layernorm forward, one warp per row held in registers (C % 256 == 0,
 // C <= 1024): one read of x, mean then biased variance from the registers
 // (eps 1e-5), one write of y; the row mean and 1/std are kept for the
-// backward pass.
+// backward pass.  gamma and beta are read as float4 alongside x, so that
+// the row's only dependent global access is x itself.
 __global__ void __launch_bounds__(256) layernorm_fwd_x8_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
                                                           const float* __restrict__ beta, bf16* __restrict__ y,
                                                           float* __restrict__ mean_out, float* __restrict__ rstd_out,
@@ -323,11 +324,21 @@ __global__ void __launch_bounds__(256) layernorm_fwd_x8_k(const bf16* __restrict
   if (row >= rows) return;
   const int nv = C / 256;
   V8 xv[kMaxV];
+  float4 g4[kMaxV][2], b4[kMaxV][2];
+#pragma unroll
+  for (int v = 0; v < kMaxV; ++v) {
+    if (v >= nv) break;
+    const int c = (v * 32 + lane) * 8;
+    xv[v] = ld8(x + row * C + c);
+    g4[v][0] = __ldg(reinterpret_cast<const float4*>(gamma + c));
+    g4[v][1] = __ldg(reinterpret_cast<const float4*>(gamma + c) + 1);
+    b4[v][0] = __ldg(reinterpret_cast<const float4*>(beta + c));
+    b4[v][1] = __ldg(reinterpret_cast<const float4*>(beta + c) + 1);
+  }
   float sum = 0.f;
 #pragma unroll
   for (int v = 0; v < kMaxV; ++v) {
     if (v >= nv) break;
-    xv[v] = ld8(x + row * C + (v * 32 + lane) * 8);
 #pragma unroll
     for (int j = 0; j < 8; ++j) sum += xv[v].v[j];
   }
@@ -351,9 +362,11 @@ __global__ void __launch_bounds__(256) layernorm_fwd_x8_k(const bf16* __restrict
   for (int v = 0; v < kMaxV; ++v) {
     if (v >= nv) break;
     const int c = (v * 32 + lane) * 8;
+    const float gm[8] = {g4[v][0].x, g4[v][0].y, g4[v][0].z, g4[v][0].w, g4[v][1].x, g4[v][1].y, g4[v][1].z, g4[v][1].w};
+    const float bt[8] = {b4[v][0].x, b4[v][0].y, b4[v][0].z, b4[v][0].w, b4[v][1].x, b4[v][1].y, b4[v][1].z, b4[v][1].w};
     V8 o;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) o.v[j] = (xv[v].v[j] - mu) * rs * gamma[c + j] + beta[c + j];
+    for (int j = 0; j < 8; ++j) o.v[j] = (xv[v].v[j] - mu) * rs * gm[j] + bt[j];
     st8(y + row * C + c, o);
   }
   if (lane == 0) {
@@ -363,14 +376,18 @@ __global__ void __launch_bounds__(256) layernorm_fwd_x8_k(const bf16* __restrict
 }
 
 // Layernorm backward fused with its parameter gradients: one warp per row
-// (dx), and per block of 8 warps x 2 rows the column partials of
-// dy * xhat (gamma) and dy (beta).  C <= 512, C % 256 == 0; dx may be null
-// (a layernorm of the uploaded batch has no input gradient).
+// (8 rows per block), with the row's x, dy, addend, mean and 1/std loads
+// all issued before any arithmetic, and the block's column partials of
+// dy * xhat (gamma) and dy (beta) added in warp order.  C <= 512,
+// C % 256 == 0; dx may be null (a layernorm of the uploaded batch has no
+// input gradient).  dx receives the layernorm's input gradient, plus its old
+// value when `acc`, plus `addend` (same layout) when given: the gradient a
+// residual connection passes around the layernorm.
 __global__ void __launch_bounds__(256) layernorm_bwd_fused_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
                                                              const float* __restrict__ mean, const float* __restrict__ rstd,
                                                              const bf16* __restrict__ dy, bf16* __restrict__ dx,
                                                              int64_t rows, int C, int acc, float* __restrict__ pg,
-                                                             float* __restrict__ pb) {
+                                                             float* __restrict__ pb, const bf16* __restrict__ addend) {
   pdl_wait();
   pdl_trigger();
   constexpr int kMaxV = 2;  // up to 2 x 8 x 32 = 512 columns per row
@@ -378,69 +395,68 @@ __global__ void __launch_bounds__(256) layernorm_bwd_fused_k(const bf16* __restr
   __shared__ float redb[8][512];
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int nv = C / 256;  // 8-wide vectors per lane
-  float sg[kMaxV][8], sb[kMaxV][8];
+  const int64_t row = int64_t(blockIdx.x) * 8 + warp;
+  const bool live = row < rows;
+  float gm[kMaxV][8];
+  V8 xv[kMaxV], gv[kMaxV], av[kMaxV], ov[kMaxV];
+  float mu = 0.f, rs = 0.f;
 #pragma unroll
-  for (int v = 0; v < kMaxV; ++v)
+  for (int v = 0; v < kMaxV; ++v) {
 #pragma unroll
-    for (int j = 0; j < 8; ++j) sg[v][j] = sb[v][j] = 0.f;
-  const int64_t row0 = int64_t(blockIdx.x) * 16;
-  for (int rr = warp; rr < 16; rr += 8) {
-    const int64_t row = row0 + rr;
-    if (row >= rows) break;
-    const float mu = mean[row], rs = rstd[row];
-    V8 xv[kMaxV], gv[kMaxV];
-    float a = 0.f, b = 0.f;
+    for (int j = 0; j < 8; ++j) xv[v].v[j] = gv[v].v[j] = av[v].v[j] = ov[v].v[j] = gm[v][j] = 0.f;
+    if (v >= nv) continue;
+    const int c = (v * 32 + lane) * 8;
+    const float4 ga = __ldg(reinterpret_cast<const float4*>(gamma + c));
+    const float4 gb = __ldg(reinterpret_cast<const float4*>(gamma + c) + 1);
+    gm[v][0] = ga.x; gm[v][1] = ga.y; gm[v][2] = ga.z; gm[v][3] = ga.w;
+    gm[v][4] = gb.x; gm[v][5] = gb.y; gm[v][6] = gb.z; gm[v][7] = gb.w;
+    if (!live) continue;
+    xv[v] = ld8(x + row * C + c);
+    gv[v] = ld8(dy + row * C + c);
+    if (dx && addend) av[v] = ld8(addend + row * C + c);
+    if (dx && acc) ov[v] = ld8(dx + row * C + c);
+  }
+  if (live) {
+    mu = mean[row];
+    rs = rstd[row];
+  }
+  float a = 0.f, b = 0.f;
 #pragma unroll
-    for (int v = 0; v < kMaxV; ++v) {
-      if (v >= nv) break;
-      const int c = (v * 32 + lane) * 8;
-      xv[v] = ld8(x + row * C + c);
-      gv[v] = ld8(dy + row * C + c);
+  for (int v = 0; v < kMaxV; ++v) {
+    if (v >= nv) break;
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const float xh = (xv[v].v[j] - mu) * rs;
-        const float dxh = gv[v].v[j] * gamma[c + j];
-        a += dxh;
-        b += dxh * xh;
-        sg[v][j] = fmaf(gv[v].v[j], xh, sg[v][j]);
-        sb[v][j] += gv[v].v[j];
-      }
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      a += __shfl_xor_sync(0xffffffffu, a, o);
-      b += __shfl_xor_sync(0xffffffffu, b, o);
-    }
-    a /= float(C);
-    b /= float(C);
-#pragma unroll
-    for (int v = 0; v < kMaxV; ++v) {
-      if (v >= nv) break;
-      const int c = (v * 32 + lane) * 8;
-      V8 o;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const float xh = (xv[v].v[j] - mu) * rs;
-        const float dxh = gv[v].v[j] * gamma[c + j];
-        o.v[j] = rs * (dxh - a - xh * b);
-      }
-      if (!dx) continue;
-      if (acc) {
-        const V8 q = ld8(dx + row * C + c);
-#pragma unroll
-        for (int j = 0; j < 8; ++j) o.v[j] += q.v[j];
-      }
-      st8(dx + row * C + c, o);
+    for (int j = 0; j < 8; ++j) {
+      const float xh = (xv[v].v[j] - mu) * rs;
+      const float dxh = gv[v].v[j] * gm[v][j];
+      a += dxh;
+      b += dxh * xh;
     }
   }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    a += __shfl_xor_sync(0xffffffffu, a, o);
+    b += __shfl_xor_sync(0xffffffffu, b, o);
+  }
+  a /= float(C);
+  b /= float(C);
 #pragma unroll
   for (int v = 0; v < kMaxV; ++v) {
     if (v >= nv) break;
     const int c = (v * 32 + lane) * 8;
+    if (live && dx) {
+      V8 o;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      redg[warp][c + j] = sg[v][j];
-      redb[warp][c + j] = sb[v][j];
+      for (int j = 0; j < 8; ++j) {
+        const float xh = (xv[v].v[j] - mu) * rs;
+        const float dxh = gv[v].v[j] * gm[v][j];
+        o.v[j] = rs * (dxh - a - xh * b) + ov[v].v[j] + av[v].v[j];
+      }
+      st8(dx + row * C + c, o);
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {   // zeros for a row past the end
+      redg[warp][c + j] = gv[v].v[j] * ((xv[v].v[j] - mu) * rs);
+      redb[warp][c + j] = gv[v].v[j];
     }
   }
   __syncthreads();
@@ -453,6 +469,76 @@ __global__ void __launch_bounds__(256) layernorm_bwd_fused_k(const bf16* __restr
     }
     pg[int64_t(blockIdx.x) * C + c] = tg;
     pb[int64_t(blockIdx.x) * C + c] = tb;
+  }
+}
+
+// Masked mean over the valid tokens of each sequence: block (b, 256-column
+// block), warp w sums tokens w, w + 8, ... of its 8 columns per lane (four
+// independent loads in flight), then the 8 warp sums are added in warp order.
+__global__ void __launch_bounds__(256) meanpool_fwd_x8_k(const bf16* __restrict__ x, const int32_t* __restrict__ len,
+                                                         bf16* __restrict__ y, int L, int C) {
+  pdl_wait();
+  pdl_trigger();
+  __shared__ float red[8][257];
+  const int b = blockIdx.x, warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int c = blockIdx.y * 256 + lane * 8;
+  const int n = len[b];
+  float s[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  if (c < C) {
+    const bf16* base = x + int64_t(b) * L * C + c;
+    int i = warp;
+    for (; i + 24 < n; i += 32) {
+      const V8 a0 = ld8(base + int64_t(i) * C), a1 = ld8(base + int64_t(i + 8) * C);
+      const V8 a2 = ld8(base + int64_t(i + 16) * C), a3 = ld8(base + int64_t(i + 24) * C);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) s[j] += ((a0.v[j] + a1.v[j]) + (a2.v[j] + a3.v[j]));
+    }
+    for (; i < n; i += 8) {
+      const V8 a = ld8(base + int64_t(i) * C);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) s[j] += a.v[j];
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 8; ++j) red[warp][lane * 8 + j] = s[j];
+  __syncthreads();
+  const int cc = blockIdx.y * 256 + threadIdx.x;
+  if (cc < C) {
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) t += red[w][threadIdx.x];
+    y[int64_t(b) * C + cc] = __float2bfloat16_rn(t / float(n));
+  }
+}
+
+// Its gradient: dx[b, t, :] = dy[b, :] / len[b] for the valid tokens, 0 for
+// the padding, 8 columns per thread (plus dx's old value when `acc`).
+__global__ void meanpool_bwd_x8_k(const bf16* __restrict__ dy, const int32_t* __restrict__ len,
+                                  bf16* __restrict__ dx, int L, int C, int64_t n8, int acc) {
+  pdl_wait();
+  pdl_trigger();
+  const int c8 = C / 8;
+  GRID_STRIDE8(i, n8) {
+    const int c = int(i % c8) * 8;
+    const int64_t bt = i / c8;
+    const int b = int(bt / L), t = int(bt % L);
+    const int n = len[b];
+    V8 o;
+    if (t < n) {
+      o = ld8(dy + int64_t(b) * C + c);
+      const float inv = 1.f / float(n);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) o.v[j] *= inv;
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) o.v[j] = 0.f;
+    }
+    if (acc) {
+      const V8 q = ld8(dx + 8 * i);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) o.v[j] += q.v[j];
+    }
+    st8(dx + 8 * i, o);
   }
 }
 
@@ -639,7 +725,7 @@ void finish_batched(const std::vector<FinishTask>& tasks, cudaStream_t st) {
 
 bool layernorm_bwd8_ok(int dt, int C) { return dt == kBF16 && C % 256 == 0 && C <= 512; }
 
-int layernorm_bwd8_blocks(int64_t rows) { return int((rows + 15) / 16); }
+int layernorm_bwd8_blocks(int64_t rows) { return int((rows + 7) / 8); }
 
 bool layernorm_fwd8_ok(int dt, int C) { return dt == kBF16 && C % 256 == 0 && C <= 1024; }
 void layernorm_fwd_x8(const void* x, const float* gamma, const float* beta, void* y, float* mean, float* rstd,
@@ -649,12 +735,22 @@ void layernorm_fwd_x8(const void* x, const float* gamma, const float* beta, void
 }
 
 void layernorm_bwd8_pass(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
-                         void* dx, int64_t rows, int C, bool acc, float* p_gamma, float* p_beta, cudaStream_t st) {
+                         void* dx, int64_t rows, int C, bool acc, float* p_gamma, float* p_beta, cudaStream_t st,
+                         const void* addend) {
   launch_k(layernorm_bwd_fused_k, layernorm_bwd8_blocks(rows), 256, 0, st, (const bf16*)x, gamma, mean, rstd,
-                                                                      (const bf16*)dy, (bf16*)dx, rows, C, acc,
-                                                                      p_gamma, p_beta);
+           (const bf16*)dy, (bf16*)dx, rows, C, acc ? 1 : 0, p_gamma, p_beta, (const bf16*)addend);
 }
 
-int64_t layernorm_bwd8_partial_floats(int64_t rows, int C) { return 2 * ((rows + 15) / 16) * C; }
+int64_t layernorm_bwd8_partial_floats(int64_t rows, int C) { return 2 * ((rows + 7) / 8) * C; }
+
+bool meanpool8_ok(int dt, int C) { return dt == kBF16 && C % 8 == 0; }
+void meanpool_fwd_x8(const void* x, const int32_t* len, void* y, int B, int L, int C, cudaStream_t st) {
+  launch_k(meanpool_fwd_x8_k, dim3(B, ceil_div(C, 256)), 256, 0, st, (const bf16*)x, len, (bf16*)y, L, C);
+}
+void meanpool_bwd_x8(const void* dy, const int32_t* len, void* dx, int B, int L, int C, bool acc, cudaStream_t st) {
+  const int64_t n8 = int64_t(B) * L * C / 8;
+  launch_k(meanpool_bwd_x8_k, elementwise_blocks(n8, 256), 256, 0, st, (const bf16*)dy, len, (bf16*)dx, L, C, n8,
+           acc ? 1 : 0);
+}
 
 }  // namespace fo

@@ -357,10 +357,18 @@ def device_batch(cfg, k, j, batch=None):
     x = rng.standard_normal((B, H, W, C), dtype=np.float32)
     if not cfg["seq"]:
         x = np.maximum(x, 0.0, dtype=np.float32)
+    if cfg.get("kink_values"):
+        # edge cases: about a quarter of the elements set exactly to the given
+        # values (e.g. the hard-swish kinks -3 and 3)
+        kv = np.asarray(cfg["kink_values"], np.float32)
+        pick = rng.random(x.shape) < 0.25
+        x = np.where(pick, kv[rng.integers(0, len(kv), size=x.shape)], x).astype(np.float32)
     if cfg["seq"]:
         labels = rng.integers(0, 2, size=B).astype(np.int32)
         lengths = rng.integers(32, 129, size=B).astype(np.int32)
         lengths = np.minimum(lengths, H).astype(np.int32)
+        if cfg.get("fixed_len") is not None:   # edge cases: every sequence of one length
+            lengths = np.full(B, cfg["fixed_len"], np.int32)
     else:
         labels = rng.integers(0, cfg["classes"], size=B).astype(np.int32)
         lengths = None

@@ -16,6 +16,10 @@ int shim_put(void* s, int k, int32_t* slot) {
   *slot = -1;
   return static_cast<fo::TaskScheduler*>(s)->put(k, slot);
 }
+int shim_peek(void* s, int k, int32_t* slot) {
+  *slot = -1;
+  return static_cast<const fo::TaskScheduler*>(s)->peek(k, slot);
+}
 int shim_get(void* s, int* k, int32_t* slot) {
   *k = -1;
   *slot = -1;

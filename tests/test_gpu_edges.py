@@ -1,0 +1,121 @@
+"""Edge cases and long runs of the server step on the GPU against the oracle.
+
+* one device, one batch slot (omega = 1), batch 1, on both precisions: the
+  scheduler serves the only queue, every upload goes into the slot the
+  previous step has just freed;
+* sequences that are all of length 1 (a single valid key per query, the
+  mean-pool over one token) and all of length 128 (no padding);
+* hard swish and hard sigmoid at exactly -3 and 3 (a quarter of the inputs
+  sit on the kinks), where the derivative convention of reading r24 decides
+  the gradients of the layer in front;
+* long runs: 200 steps of the VGG-style workload and 300 of the transformer
+  on the GPU alone, with the step at the middle and the last step
+  teacher-forced against the exact oracle.
+
+fp32 workloads run whole traces at 1e-4; bf16 ones are gated step by step
+with harness.gate_failures."""
+import numpy as np
+import pytest
+
+from harness import check_teacher_forced, teacher_forced
+from paper_2504_13850_gb300 import api, build
+from paper_2504_13850_gb300 import workloads as W
+from test_gpu_train import compare
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    build.build()
+    api.lib()
+
+
+def one_slot_events(steps):
+    ev = []
+    for _ in range(steps):
+        ev += [("enq", 0), ("step",)]
+    return ev + [("step",)]          # and one on the empty queue
+
+
+def small_vgg_ops(cin=64):
+    b = W._Builder()
+    t = b.add("conv", 0, cin=cin, cout=128, k=3, stride=1, bias=1)
+    t = b.add("relu", t)
+    t = b.add("maxpool2", t)
+    t = b.add("flatten", t)
+    t = b.add("linear", t, cin=8 * 8 * 128, cout=64, bias=1)
+    t = b.add("relu", t)
+    b.add("linear", t, cin=64, cout=10, bias=1)
+    return b.ops
+
+
+@pytest.mark.parametrize("dtype", [W.F32, W.BF16])
+def test_batch_one_one_device_one_slot(dtype):
+    cfg = W.shrink(W.CONFIGS["vgg"], ops=small_vgg_ops(), batch=1, in_hwc=(16, 16, 64), K=1, omega=1, depth=1,
+                   dtype=dtype, lr=1e-3)
+    ev = one_slot_events(4)
+    if dtype == W.F32:
+        s, o = compare(cfg, ev, loss_tol=1e-4, param_tol=1e-4, upd_tol=1e-4)
+        assert [int(c) for c in s.counters()] == o.sched.c == [4]
+    else:
+        _, o, recs = teacher_forced(cfg, ev)
+        assert len(recs) == 4 and o.sched.c == [4]
+        check_teacher_forced(recs)
+
+
+@pytest.mark.parametrize("length", [1, 128])
+def test_sequences_all_of_one_length(length):
+    cfg = W.shrink(W.CONFIGS["transformer"], ops=W.transformer_ops(d=128, heads=2, ffn=256, blocks=2),
+                   batch=6, in_hwc=(128, 1, 128), K=2, omega=4, depth=2, fixed_len=length, lr=1e-3)
+    ev = [("enq", k) for _ in range(2) for k in range(2)] + [("step",)] * 4
+    _, _, recs = teacher_forced(cfg, ev)
+    assert len(recs) == 4
+    check_teacher_forced(recs)
+
+
+def kink_ops():
+    """Two affines of the upload (scale 1, shift 0 at the start: their
+    outputs are the upload itself), one into a hard swish and one into a
+    hard sigmoid, summed, then a dense classifier: the affines' gradients
+    see both derivatives at the kinks."""
+    b = W._Builder()
+    h = b.add("affine", 0, c=16)
+    h = b.add("hswish", h)
+    g = b.add("affine", 0, c=16)
+    g = b.add("hsigmoid", g)
+    t = b.add("add", h, in1=g)
+    t = b.add("flatten", t)
+    b.add("linear", t, cin=4 * 4 * 16, cout=10, bias=1)
+    return b.ops
+
+
+@pytest.mark.parametrize("dtype", [W.F32, W.BF16])
+def test_hard_swish_and_sigmoid_exactly_at_the_kinks(dtype):
+    cfg = W.shrink(W.CONFIGS["mobilenet"], ops=kink_ops(), classes=10, batch=8, in_hwc=(4, 4, 16), K=2, omega=4,
+                   depth=2, dtype=dtype, kink_values=(-3.0, 3.0), lr=1e-3)
+    x, _, _, _ = W.device_batch(cfg, 0, 0)
+    assert np.mean(np.abs(np.abs(x) - 3.0) == 0) > 0.2          # the inputs do sit on the kinks
+    ev = [("enq", k) for _ in range(2) for k in range(2)] + [("step",)] * 4
+    if dtype == W.F32:
+        compare(cfg, ev, loss_tol=1e-4, param_tol=1e-4, upd_tol=1e-4)
+    else:
+        _, _, recs = teacher_forced(cfg, ev)
+        assert len(recs) == 4
+        check_teacher_forced(recs)
+
+
+@pytest.mark.parametrize("name,steps", [("vgg", 200), ("transformer", 300)])
+def test_long_run_teacher_forced_at_the_middle_and_the_end(name, steps):
+    """The full-size workload for `steps` steps (its step count in the
+    workload table) from the backlogged queues, every device re-uploading
+    as its batches are served; the GPU alone runs all but the middle and the
+    last step, which are compared with one exact oracle step each."""
+    cfg = W.CONFIGS[name]
+    K, depth = cfg["K"], cfg["depth"]
+    ev = [("enq", k) for _ in range(depth) for k in range(K)]
+    for j in range(steps):
+        ev += [("step",), ("enq", j % K)]
+    _, _, recs = teacher_forced(cfg, ev, compare={steps // 2, steps - 1})
+    assert [r["step"] for r in recs] == [steps // 2, steps - 1]
+    check_teacher_forced(recs)

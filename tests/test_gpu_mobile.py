@@ -5,17 +5,17 @@ that still span several tiles and ragged channel tails, on both precisions.
 
 fp32 path: the full trace (scheduler outcomes bit-exact, loss 1e-4,
 parameters, update and momentum 1e-4 normwise: fp32 roundings over sums of
-at most a few thousand terms).  bf16 path: teacher-forced steps with the
-gates of test_gpu_train (the hard sigmoid's derivative jumps at -3 and 3
-and the SE block has a ReLU, so stored values one bf16 ulp apart may decide
-a kink the other way: the decision allowance applies).
+at most a few thousand terms).  bf16 path: teacher-forced steps against the
+exact oracle with the gates of harness.gate_failures (the hard sigmoid's
+derivative jumps at -3 and 3 and the SE block has a ReLU, so decisions at
+those kinks can flip: the allowance of harness.grad_bound applies).
 """
 import pytest
 
-from harness import teacher_forced
+from harness import check_teacher_forced, teacher_forced
 from paper_2504_13850_gb300 import api, build
 from paper_2504_13850_gb300 import workloads as W
-from test_gpu_train import check_teacher_forced, compare, prefill_then_steps
+from test_gpu_train import compare, prefill_then_steps
 
 pytestmark = pytest.mark.gpu
 
@@ -65,7 +65,7 @@ def test_small_mobile_bf16_teacher_forced():
     cfg = small_mobile(W.BF16)
     _, _, recs = teacher_forced(cfg, prefill_then_steps(cfg, 6))
     assert len(recs) == 6
-    check_teacher_forced(recs, decisions=True)
+    check_teacher_forced(recs)
 
 
 def test_depthwise_gradients_reach_the_input_layer():
@@ -121,4 +121,4 @@ def test_depthwise_any_kernel_size():
             compare(cfg, prefill_then_steps(cfg, 4), loss_tol=1e-4, param_tol=1e-4, upd_tol=1e-4)
         else:
             _, _, recs = teacher_forced(cfg, prefill_then_steps(cfg, 4))
-            check_teacher_forced(recs, decisions=True)
+            check_teacher_forced(recs)

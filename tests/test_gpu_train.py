@@ -8,13 +8,14 @@ derived below.
 Update tolerance (fp32 path).  Each gradient is formed from a chain of a
 few fp32 roundings (2^-24) over sums of <= 4096 terms, < 1e-5 normwise;
 1e-4 is used.  The bf16 path is checked step by step (teacher forced)
-against both the exact oracle and its bf16-storage reading, see
-check_teacher_forced.
+against the exact oracle: loss, parameters, the gradient of every
+parameter tensor and the update, with the bound derived in
+harness.grad_bound.
 """
 import numpy as np
 import pytest
 
-from harness import normwise, replay_gpu, replay_oracle, teacher_forced
+from harness import check_teacher_forced, normwise, replay_gpu, replay_oracle, teacher_forced
 from paper_2504_13850_gb300 import api, build
 from paper_2504_13850_gb300 import workloads as W
 
@@ -90,51 +91,17 @@ def test_tiny_config_fp32_full_trace():
     assert [int(c) for c in s.counters()] == o.sched.c == [2, 2, 2, 2]
 
 
-def check_teacher_forced(recs, loss_tol=1e-2, param_tol=2e-2, kernel_loss_tol=2e-3, clean_tol=3e-2,
-                         flip_tol=8e-2, decisions=True, free_tol=1e-2):
-    """Gates of each step.
-
-    Against the exact oracle (the stated tolerances): loss within 1e-2
-    relative, parameters within 2e-2 normwise.
-
-    Against the bf16-storage reading (same stored values, so ReLU / max-pool
-    decisions are taken on the same bf16 numbers): loss within 2e-3 and the
-    gradient of every parameter tensor normwise.  Without decisions (conv /
-    linear / layernorm / attention / GELU chains) what is left is fp32
-    accumulation order (~1e-6) and one-ulp bf16 rounding differences of rare
-    elements, a few 1e-3 over a backward chain of ~10 stored tensors: every
-    tensor within free_tol = 1e-2 on every step (the noise grows like the
-    square root of the chain length, so a chain four times longer gets
-    2e-2).  With decisions, a stored value that lands one bf16 ulp
-    apart can still decide a ReLU at 0 or a max-pool tie (ties are common in
-    bf16) the other way; each such flip re-routes one gradient element and
-    moves the weight gradient of its layer, and everything upstream, by
-    about 1/sqrt(#gradient elements of that layer) -- up to 3.6% for the
-    small FC layer here, ~0.6% per max-pool flip with a few flips per step.
-    So there every tensor stays within 8e-2 on every step and within 3e-2
-    on at least half of the steps."""
-    clean = 0
-    for r in recs:
-        ex, st = r["exact"], r["stored"]
-        assert abs(r["loss"] - ex["loss"]) <= loss_tol * abs(ex["loss"]), r
-        assert ex["param_err"] <= param_tol, r
-        assert abs(r["loss"] - st["loss"]) <= kernel_loss_tol * abs(st["loss"]), r
-        worst = max(st["tensor_grad_err"].values())
-        if not decisions:
-            assert worst <= free_tol, (r["step"], st["tensor_grad_err"])
-        assert worst <= flip_tol, (r["step"], st["tensor_grad_err"])
-        clean += worst <= clean_tol
-    assert 2 * clean >= len(recs), [max(r["stored"]["tensor_grad_err"].values()) for r in recs]
-
-
 @pytest.mark.parametrize("kind", ["vgg", "resnet", "transformer"])
 def test_small_bf16_configs_teacher_forced(kind):
-    """Every step from the GPU's own state: loss, parameters and the gradient
-    of every parameter tensor against one oracle step."""
-    cfg = small(kind)
+    """Every step from the GPU's own state: loss, parameters, update and the
+    gradient of every parameter tensor against one exact oracle step.  At
+    lr 1e-3 the loss stays near ln C over the six steps (at lr 0.01 the
+    small VGG-style network reaches a loss of 11 by its fourth step, where
+    the softmax is saturated and the gradient ill-conditioned)."""
+    cfg = W.shrink(small(kind), lr=1e-3)
     _, _, recs = teacher_forced(cfg, prefill_then_steps(cfg, 6))
     assert len(recs) == 6
-    check_teacher_forced(recs, decisions=kind != "transformer")
+    check_teacher_forced(recs)
 
 
 def decision_free(kind):
@@ -188,7 +155,9 @@ def test_decision_free_teacher_forced(kind):
     cfg = decision_free(kind)
     _, _, recs = teacher_forced(cfg, prefill_then_steps(cfg, 4))
     assert len(recs) == 4
-    check_teacher_forced(recs, decisions=False)
+    check_teacher_forced(recs)
+    for r in recs:   # no decisions: every tensor within the stated 2e-2 itself
+        assert max(r["exact"]["tensor_grad_err"].values()) <= 2e-2, r["exact"]["tensor_grad_err"]
 
 
 @pytest.mark.parametrize("kind", ["vgg", "resnet", "transformer"])

@@ -54,6 +54,7 @@ def build(name, source):
     L.shim_destroy.argtypes = [C.c_void_p]
     L.shim_put.argtypes = [C.c_void_p, C.c_int, C.POINTER(C.c_int32)]
     L.shim_get.argtypes = [C.c_void_p, C.POINTER(C.c_int), C.POINTER(C.c_int32)]
+    L.shim_peek.argtypes = [C.c_void_p, C.c_int, C.POINTER(C.c_int32)]
     L.shim_set_active.argtypes = [C.c_void_p, C.c_int, C.c_int]
     L.shim_counters.argtypes = [C.c_void_p, C.c_void_p]
     L.shim_sender.argtypes = [C.c_void_p, C.c_void_p]
@@ -75,6 +76,11 @@ class Shim:
         slot = C.c_int32(-1)
         rc = self.L.shim_put(self.h, k, C.byref(slot)) if 0 <= k < self.K else -1
         return rc, slot.value, (int(self.sender_status()[k]) if 0 <= k < self.K else -1)
+
+    def peek(self, k):
+        slot = C.c_int32(-1)
+        rc = self.L.shim_peek(self.h, k, C.byref(slot))
+        return rc, slot.value
 
     def get(self):
         k, slot = C.c_int(-1), C.c_int32(-1)
@@ -144,7 +150,33 @@ def check_random_traces(L):
                 assert a.queued() == o.queued()
 
 
-CHECKS = (check_tiny_golden, check_slot_reuse_golden, check_random_traces)
+def check_peek_predicts_put(L):
+    """An upload's slot is filled before the scheduler commits it: peek(k)
+    must give put(k)'s outcome and slot exactly, and change nothing."""
+    for policy in ("counter", "fifo"):
+        for seed in range(4):
+            r = np.random.default_rng(100 + seed)
+            K, depth = int(r.integers(1, 7)), int(r.integers(1, 4))
+            omega = int(r.integers(1, K * depth + 2))
+            a = Shim(L, K, omega, depth, policy)
+            for _ in range(300):
+                u = r.random()
+                if u < 0.5:
+                    k = int(r.integers(K))
+                    state = (a.counters(), a.sender_status(), a.queued())
+                    prc, pslot = a.peek(k)
+                    assert (a.counters(), a.sender_status(), a.queued()) == state
+                    rc, slot, _ = a.put(k)
+                    assert prc == {0: 0, 2: 2, -1: -1}.get(rc, rc)
+                    if rc == 0:
+                        assert slot == pslot
+                elif u < 0.9:
+                    a.get()
+                else:
+                    a.set_active(int(r.integers(K)), bool(r.integers(2)))
+
+
+CHECKS = (check_tiny_golden, check_slot_reuse_golden, check_random_traces, check_peek_predicts_put)
 
 
 def source():
