@@ -339,6 +339,7 @@ class Harness:
         w0 = time.perf_counter()
         for _ in range(steps):
             self.step()
+        self.srv.join_aggregations()     # the aggregations (their own stream) inside the timed region
         ev1.record(self.stream)
         torch.cuda.synchronize()
         wall = time.perf_counter() - w0
@@ -347,9 +348,10 @@ class Harness:
         return ev0.elapsed_time(ev1), wall, self.srv.kernels_launched() - k0
 
     def busy(self, steps):
-        """GPU busy fraction of the step loop: the summed device time from
-        each step's first kernel to its aggregation, over the device time of
-        the whole loop (the rest is the server idling on the host)."""
+        """GPU busy fraction of the step loop: the summed device time of the
+        steps on the compute stream, over the device time of the whole loop
+        (the rest is the compute stream idling, waiting for the host; the
+        aggregations run on their own stream alongside)."""
         torch = self.torch
         self.srv.synchronize()
         evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
@@ -394,6 +396,7 @@ class Harness:
         for _ in range(steps):
             self.step(host=True)
         self.last_loss = self.srv.read_losses(self.done - 1, 1)
+        self.srv.join_aggregations()
         ev1.record(self.stream)
         torch.cuda.synchronize()
         barrier(world)

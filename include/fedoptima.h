@@ -219,8 +219,12 @@ FO_API int fo_read_losses(fo_server* s, float* host_out, int64_t first_step, int
  * global) in fp32; then t <- t + 1 and *new_version = t.  `local` (device,
  * n floats, read only) is theta_dk || theta~_dk trained from version t_k =
  * `version`.  FO_STALE when t - version > D (global and t unchanged).
- * FO_ERR_ARG when version < 0 or version > t.  Runs on the server's compute
- * stream, ordered after earlier steps.  `local` may also be host memory
+ * FO_ERR_ARG when version < 0 or version > t.  Runs on the server's
+ * aggregation stream (fo_server_agg_stream), ordered after earlier
+ * aggregations but not after the training steps: the two touch disjoint data
+ * and overlap on the GPU (fo_server_synchronize waits for both;
+ * fo_server_join_aggregations orders the compute stream after the
+ * aggregations enqueued so far).  `local` may also be host memory
  * (page-locked for an asynchronous copy): it is then copied into one of two
  * server-owned device buffers on the upload stream, overlapping the steps
  * already queued, and the call returns once that copy has landed, so the
@@ -255,6 +259,15 @@ FO_API int fo_server_synchronize(fo_server* s);
  * on, for callers that time them with CUDA events; no counterpart in the
  * paper.  NULL for a NULL handle. */
 FO_API void* fo_server_stream(const fo_server* s);
+/* The aggregation stream (a cudaStream_t) fo_aggregate runs on, for callers
+ * that order their work after aggregations; no counterpart in the paper.
+ * NULL for a NULL handle. */
+FO_API void* fo_server_agg_stream(const fo_server* s);
+/* Makes the compute stream wait for every aggregation enqueued so far
+ * (asynchronous; an event on the aggregation stream), e.g. before the caller
+ * records a timing event on fo_server_stream; no counterpart in the paper.
+ * FO_ERR_ARG for a NULL handle. */
+FO_API int fo_server_join_aggregations(fo_server* s);
 /* Kernel launches the last fo_server_step enqueued, and all kernels the
  * server has launched since creation (steps and aggregations); no
  * counterpart in the paper.  -1 for a NULL handle. */

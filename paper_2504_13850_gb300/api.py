@@ -71,6 +71,8 @@ _SIGS = [
     ("fo_server_activation_bytes", C.c_int64, [C.c_void_p]),
     ("fo_server_synchronize", C.c_int, [C.c_void_p]),
     ("fo_server_stream", C.c_void_p, [C.c_void_p]),
+    ("fo_server_agg_stream", C.c_void_p, [C.c_void_p]),
+    ("fo_server_join_aggregations", C.c_int, [C.c_void_p]),
     ("fo_server_last_step_launches", C.c_int, [C.c_void_p]),
     ("fo_server_profile", C.c_int, [C.c_void_p, C.c_int]),
     ("fo_server_kernel_times", C.c_int, [C.c_void_p, C.POINTER(C.c_char_p), C.POINTER(C.c_int64),
@@ -277,6 +279,12 @@ class Server:
 
     def stream(self):
         return lib().fo_server_stream(self.h)
+
+    def agg_stream(self):
+        return lib().fo_server_agg_stream(self.h)
+
+    def join_aggregations(self):
+        _check(lib().fo_server_join_aggregations(self.h), "join_aggregations")
 
     def last_step_launches(self):
         return lib().fo_server_last_step_launches(self.h)

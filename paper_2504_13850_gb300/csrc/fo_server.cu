@@ -1071,6 +1071,7 @@ int allocate(fo_server* s) {
 void destroy_impl(fo_server* s) {
   if (!s) return;
   if (s->cs) cudaStreamSynchronize(s->cs);
+  if (s->as) cudaStreamSynchronize(s->as);
   for (fo::AttnTcPlan* a : s->attn_tc) fo::attention_tc_destroy(a);
   s->attn_tc.clear();
   if (s->xs) cudaStreamSynchronize(s->xs);
@@ -1100,6 +1101,8 @@ void destroy_impl(fo_server* s) {
     if (s->agg_read[b]) cudaEventDestroy(s->agg_read[b]);
   }
   if (s->cs) cudaStreamDestroy(s->cs);
+  if (s->as) cudaStreamDestroy(s->as);
+  if (s->agg_ev) cudaEventDestroy(s->agg_ev);
   if (s->xs) cudaStreamDestroy(s->xs);
   if (s->hs) cudaStreamDestroy(s->hs);
   for (auto e : s->stage_landed) if (e) cudaEventDestroy(e);
@@ -1250,6 +1253,8 @@ static int server_create(const fo_op* ops, int n_ops, const fo_optimizer* opt, c
       cudaStreamCreateWithFlags(&s->hs, cudaStreamNonBlocking) != cudaSuccess ||
       cudaStreamCreateWithFlags(&s->side, cudaStreamNonBlocking) != cudaSuccess ||
       cudaStreamCreateWithFlags(&s->opt_st, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&s->as, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&s->agg_ev, cudaEventDisableTiming) != cudaSuccess ||
       cudaEventCreateWithFlags(&s->fork2_ev, cudaEventDisableTiming) != cudaSuccess ||
       cudaEventCreateWithFlags(&s->join2_ev, cudaEventDisableTiming) != cudaSuccess ||
       cudaEventCreateWithFlags(&s->fork_ev, cudaEventDisableTiming) != cudaSuccess ||
@@ -1555,23 +1560,23 @@ int fo_aggregate(fo_server* s, float* global, const float* local, int64_t n, int
     FO_CUDA(cudaStreamWaitEvent(s->hs, s->agg_read[stage_buf], 0));   // the aggregation that last read it
     FO_CUDA(cudaMemcpyAsync(dst, local, size_t(n) * 4, cudaMemcpyHostToDevice, s->hs));
     FO_CUDA(cudaEventRecord(s->agg_landed[stage_buf], s->hs));
-    FO_CUDA(cudaStreamWaitEvent(s->cs, s->agg_landed[stage_buf], 0));
+    FO_CUDA(cudaStreamWaitEvent(s->as, s->agg_landed[stage_buf], 0));
     FO_CUDA(cudaEventSynchronize(s->agg_landed[stage_buf]));   // the caller may reuse `local`
     local = dst;
   }
   const int nk = fo::axpby_kernels(global, local, n);
   if (s->profiling) {
     ProfRec r{prof_id(s, "fedasync_axpby"), pool_event(s), pool_event(s), nk, 0.0, 12.0 * double(n)};
-    cudaEventRecord(r.a, s->cs);
-    fo::axpby(global, local, n, alpha, s->cs);
-    cudaEventRecord(r.b, s->cs);
+    cudaEventRecord(r.a, s->as);
+    fo::axpby(global, local, n, alpha, s->as);
+    cudaEventRecord(r.b, s->as);
     s->prof.push_back(r);
   } else {
-    fo::axpby(global, local, n, alpha, s->cs);
+    fo::axpby(global, local, n, alpha, s->as);
   }
   s->kernels_launched += nk;
   FO_CUDA(cudaGetLastError());
-  if (stage_buf >= 0) FO_CUDA(cudaEventRecord(s->agg_read[stage_buf], s->cs));
+  if (stage_buf >= 0) FO_CUDA(cudaEventRecord(s->agg_read[stage_buf], s->as));
   s->t += 1;
   if (new_version) *new_version = s->t;
   return FO_OK;
@@ -1608,9 +1613,17 @@ int fo_server_synchronize(fo_server* s) {
   FO_CUDA(cudaStreamSynchronize(s->hs));
   FO_CUDA(cudaStreamSynchronize(s->xs));
   FO_CUDA(cudaStreamSynchronize(s->cs));
+  FO_CUDA(cudaStreamSynchronize(s->as));
   return FO_OK;
 }
 void* fo_server_stream(const fo_server* s) { return s ? (void*)s->cs : nullptr; }
+void* fo_server_agg_stream(const fo_server* s) { return s ? (void*)s->as : nullptr; }
+int fo_server_join_aggregations(fo_server* s) {
+  if (!s) return set_err(FO_ERR_ARG, "null server");
+  FO_CUDA(cudaEventRecord(s->agg_ev, s->as));
+  FO_CUDA(cudaStreamWaitEvent(s->cs, s->agg_ev, 0));
+  return FO_OK;
+}
 int fo_server_last_step_launches(const fo_server* s) { return s ? s->last_launches : -1; }
 
 int fo_server_profile(fo_server* s, int enable) {

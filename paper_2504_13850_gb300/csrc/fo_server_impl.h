@@ -86,6 +86,11 @@ struct fo_server {
   // are done, so the HBM-bound update overlaps the GEMMs that follow.
   cudaStream_t opt_st = nullptr;
   cudaEvent_t fork2_ev = nullptr, join2_ev = nullptr;
+  // Aggregation stream: FedAsync updates of device models touch no data of
+  // the training step, so they run here and overlap the steps; agg_ev lets
+  // the compute stream join them (fo_server_join_aggregations).
+  cudaStream_t as = nullptr;
+  cudaEvent_t agg_ev = nullptr;
   bool use_side = true;
   int dt = fo::kF32;
 

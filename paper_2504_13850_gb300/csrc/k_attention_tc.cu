@@ -14,8 +14,11 @@
 // two 64-column sub-tiles, which serves both as a K-major operand (P V,
 // dS K) and as an MN-major one (P^T dO, dS^T Q).
 // Warp roles: warp 0 issues the TMA loads, warp 1 owns TMEM and issues the
-// MMAs (one thread each), warps 2..5 own one TMEM lane quarter (= 32 rows)
-// for the softmax and the stores.  Waits are bounded (error word 11..16).
+// MMAs (one thread each), warps 2..9 do the softmax and the stores: warp w
+// reads TMEM lane quarter w % 4 (32 rows) and takes keys 64 * ((w - 2) / 4)
+// .. +63 of them, so every row is shared by two threads (the forward pass
+// combines their partial maxima and sums through shared memory).  Waits are
+// bounded (error word 11..16).
 #include "fo_common.cuh"
 #include "fo_kernels.h"
 #include "fo_ptx.cuh"
@@ -25,7 +28,8 @@ namespace fo {
 
 namespace {
 
-constexpr int kAttnThreads = 192;
+constexpr int kAttnThreads = 320;
+constexpr int kSoftmaxThreads = 256;      // warps 2..9
 constexpr int kTile = 16384;              // 128 rows x 64 bf16
 constexpr float kScale = 0.125f;          // 1 / sqrt(64)
 
@@ -84,6 +88,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_tc_k(const __grid_co
   char* sP = sm + 3 * kTile;                       // two sub-tiles (keys 0..63, 64..127)
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + 5 * kTile);   // ld, s, p, o
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 4);
+  float2* xch = reinterpret_cast<float2*>(sm + 5 * kTile + 64);   // [half][row]: partial (max, sum)
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int bh = blockIdx.x, b = bh / p.heads, h = bh % p.heads;
@@ -91,7 +96,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_tc_k(const __grid_co
   if (threadIdx.x == 0) {
     mbar_init(&bars[0], 1);
     mbar_init(&bars[1], 1);
-    mbar_init(&bars[2], 128);
+    mbar_init(&bars[2], kSoftmaxThreads);
     mbar_init(&bars[3], 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_qkv)) : "memory");
@@ -136,56 +141,67 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_tc_k(const __grid_co
       mma_commit(&bars[3]);
     }
   } else {
-    const int q = warp % 4, i = q * 32 + lane;
-    const uint32_t trow = tmem + (uint32_t(q * 32) << 16);
+    const int q = warp % 4, i = q * 32 + lane, hf = (warp - 2) / 4;
+    const uint32_t trow = tmem + (uint32_t(q * 32) << 16) + uint32_t(64 * hf);   // this thread's 64 keys
     const int n = min(p.len[b], p.L);
     if (!mbar_wait(&bars[1], 0)) atomicExch(p.err, 13);
     tc_fence_after();
+    // one pass: running maximum and rescaled sum over this thread's keys
     uint32_t r[32];
-    float m = -INFINITY;
+    float m = -INFINITY, sum = 0.f;
 #pragma unroll 1
-    for (int c = 0; c < 4; ++c) {
+    for (int c = 0; c < 2; ++c) {
       tmem_ld32(trow + 32 * c, r);
+      const int j0 = 64 * hf + 32 * c;
+      float cm = -INFINITY;
 #pragma unroll
       for (int e = 0; e < 32; ++e)
-        if (32 * c + e < n) m = fmaxf(m, __uint_as_float(r[e]) * kScale);
-    }
-    float sum = 0.f;
-#pragma unroll 1
-    for (int c = 0; c < 4; ++c) {
-      tmem_ld32(trow + 32 * c, r);
+        if (j0 + e < n) cm = fmaxf(cm, __uint_as_float(r[e]) * kScale);
+      const float mn = fmaxf(m, cm);
+      if (mn > -INFINITY) {
+        sum = m > -INFINITY ? sum * __expf(m - mn) : 0.f;
 #pragma unroll
-      for (int e = 0; e < 32; ++e)
-        if (32 * c + e < n) sum += __expf(__uint_as_float(r[e]) * kScale - m);
+        for (int e = 0; e < 32; ++e)
+          if (j0 + e < n) sum += __expf(__uint_as_float(r[e]) * kScale - mn);
+        m = mn;
+      }
     }
-    const float inv = sum > 0.f ? 1.f / sum : 0.f;
-    const uint32_t p_base = smem_u32(sP);
+    // combine with the other half of the row
+    xch[hf * 128 + i] = make_float2(m, sum);
+    asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
+    const float2 o2 = xch[(1 - hf) * 128 + i];
+    const float M = fmaxf(m, o2.x);
+    float S = 0.f;
+    if (M > -INFINITY) {
+      if (m > -INFINITY) S += sum * __expf(m - M);
+      if (o2.x > -INFINITY) S += o2.y * __expf(o2.x - M);
+    }
+    const float inv = S > 0.f ? 1.f / S : 0.f;
+    const uint32_t p_base = smem_u32(sP) + uint32_t(hf) * kTile;
 #pragma unroll 1
-    for (int c = 0; c < 4; ++c) {
+    for (int c = 0; c < 2; ++c) {
       tmem_ld32(trow + 32 * c, r);
 #pragma unroll
       for (int g = 0; g < 4; ++g) {
         float v[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          const int j = 32 * c + 8 * g + e;
-          v[e] = j < n ? __expf(__uint_as_float(r[8 * g + e]) * kScale - m) * inv : 0.f;
+          const int j = 64 * hf + 32 * c + 8 * g + e;
+          v[e] = j < n ? __expf(__uint_as_float(r[8 * g + e]) * kScale - M) * inv : 0.f;
         }
-        st_shared4(p_base + (c >> 1) * kTile + sw_off(i, (c & 1) * 4 + g), pack_bf16x2(v[0], v[1]),
-                   pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
+        st_shared4(p_base + sw_off(i, c * 4 + g), pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
+                   pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
       }
     }
-    if (i < p.L) p.lse[size_t(bh) * p.L + i] = m + logf(sum);
+    if (hf == 0 && i < p.L) p.lse[size_t(bh) * p.L + i] = M + logf(S);
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // P visible to the tensor cores
     tc_fence_before();
     mbar_arrive(&bars[2]);
     if (!mbar_wait(&bars[3], 0)) atomicExch(p.err, 14);
     tc_fence_after();
-#pragma unroll 1
-    for (int c = 0; c < 2; ++c) {
-      tmem_ld32(trow + 128 + 32 * c, r);
-      if (i < p.L) store_row32(p.out + size_t(row0 + i) * p.C + h * 64 + 32 * c, r, false);
-    }
+    // O: 64 columns at TMEM column 128; each half of the pair stores 32
+    tmem_ld32(tmem + (uint32_t(q * 32) << 16) + 128 + 32 * hf, r);
+    if (i < p.L) store_row32(p.out + size_t(row0 + i) * p.C + h * 64 + 32 * hf, r, false);
   }
   tc_fence_before();
   __syncthreads();
@@ -214,7 +230,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_bwd_tc_k(const __grid_co
   if (threadIdx.x == 0) {
     mbar_init(&bars[0], 1);
     mbar_init(&bars[1], 1);
-    mbar_init(&bars[2], 128);
+    mbar_init(&bars[2], kSoftmaxThreads);
     mbar_init(&bars[3], 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_qkv)) : "memory");
@@ -277,7 +293,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_bwd_tc_k(const __grid_co
       mma_commit(&bars[3]);
     }
   } else {
-    const int q = warp % 4, i = q * 32 + lane;
+    const int q = warp % 4, i = q * 32 + lane, hf = (warp - 2) / 4;   // keys 64 hf .. +63
     const uint32_t trow = tmem + (uint32_t(q * 32) << 16);
     const int n = min(p.len[b], p.L);
     const bool live = i < p.L;          // rows past the sequence get P = dS = 0
@@ -299,7 +315,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_bwd_tc_k(const __grid_co
     tc_fence_after();
     const uint32_t p_base = smem_u32(sP), ds_base = smem_u32(sdS);
 #pragma unroll 1
-    for (int c = 0; c < 4; ++c) {
+    for (int c = 2 * hf; c < 2 * hf + 2; ++c) {
       uint32_t rs[32], rp[32];
       tmem_ld32(trow + 32 * c, rs);
       tmem_ld32(trow + 128 + 32 * c, rp);
@@ -325,17 +341,15 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_bwd_tc_k(const __grid_co
     mbar_arrive(&bars[2]);
     if (!mbar_wait(&bars[3], 0)) atomicExch(p.err, 14);
     tc_fence_after();
-    // TMEM row i holds dQ row i and dK / dV row j = i
+    // TMEM row i holds dQ row i and dK / dV row j = i; each half of the
+    // pair stores 32 of the 64 columns of each
     bf16* drow = p.out + size_t(row0 + i) * 3 * p.C;
 #pragma unroll 1
     for (int t = 0; t < 3; ++t) {
       const uint32_t col = t == 0 ? 320u : (t == 1 ? 384u : 256u);     // dQ, dK, dV
-#pragma unroll 1
-      for (int c = 0; c < 2; ++c) {
-        uint32_t r[32];
-        tmem_ld32(trow + col + 32 * c, r);
-        if (live) store_row32(drow + t * p.C + h * 64 + 32 * c, r, p.acc != 0);
-      }
+      uint32_t r[32];
+      tmem_ld32(trow + col + 32 * hf, r);
+      if (live) store_row32(drow + t * p.C + h * 64 + 32 * hf, r, p.acc != 0);
     }
   }
   tc_fence_before();
@@ -346,7 +360,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_bwd_tc_k(const __grid_co
   }
 }
 
-constexpr size_t kFwdSmem = 5 * kTile + 1024 + 64;
+constexpr size_t kFwdSmem = 5 * kTile + 1024 + 64 + 2 * 128 * sizeof(float2);
 constexpr size_t kBwdSmem = 9 * kTile + 1024 + 64;
 
 }  // namespace

@@ -376,61 +376,75 @@ __global__ void __launch_bounds__(256) layernorm_fwd_x8_k(const bf16* __restrict
 }
 
 // Layernorm backward fused with its parameter gradients: one warp per row
-// (8 rows per block), with the row's x, dy, addend, mean and 1/std loads
-// all issued before any arithmetic, and the block's column partials of
-// dy * xhat (gamma) and dy (beta) added in warp order.  C <= 512,
+// (8 rows per block).  The row's x, dy, addend and old dx are all loaded
+// before any arithmetic and kept as packed bf16 (so that four blocks fit on
+// an SM and the whole grid is resident at once); the block's column partials
+// of dy * xhat (gamma) and dy (beta) are added in warp order.  C <= 512,
 // C % 256 == 0; dx may be null (a layernorm of the uploaded batch has no
 // input gradient).  dx receives the layernorm's input gradient, plus its old
 // value when `acc`, plus `addend` (same layout) when given: the gradient a
 // residual connection passes around the layernorm.
-__global__ void __launch_bounds__(256) layernorm_bwd_fused_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
-                                                             const float* __restrict__ mean, const float* __restrict__ rstd,
-                                                             const bf16* __restrict__ dy, bf16* __restrict__ dx,
-                                                             int64_t rows, int C, int acc, float* __restrict__ pg,
-                                                             float* __restrict__ pb, const bf16* __restrict__ addend) {
+__device__ __forceinline__ float bf_at(const uint4& u, int j) {
+  return __bfloat162float(reinterpret_cast<const bf16*>(&u)[j]);
+}
+__device__ __forceinline__ void gamma8(const float* gamma, int c, float (&g)[8]) {
+  const float4 a = __ldg(reinterpret_cast<const float4*>(gamma + c));
+  const float4 b = __ldg(reinterpret_cast<const float4*>(gamma + c) + 1);
+  g[0] = a.x; g[1] = a.y; g[2] = a.z; g[3] = a.w; g[4] = b.x; g[5] = b.y; g[6] = b.z; g[7] = b.w;
+}
+__global__ void __launch_bounds__(256, 4) layernorm_bwd_fused_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
+                                                                const float* __restrict__ mean, const float* __restrict__ rstd,
+                                                                const bf16* __restrict__ dy, bf16* __restrict__ dx,
+                                                                int64_t rows, int C, int acc, float* __restrict__ pg,
+                                                                float* __restrict__ pb, const bf16* __restrict__ addend) {
   pdl_wait();
   pdl_trigger();
   constexpr int kMaxV = 2;  // up to 2 x 8 x 32 = 512 columns per row
-  __shared__ float redg[8][512];
-  __shared__ float redb[8][512];
+  __shared__ __align__(16) float redg[8][512];
+  __shared__ __align__(16) float redb[8][512];
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int nv = C / 256;  // 8-wide vectors per lane
   const int64_t row = int64_t(blockIdx.x) * 8 + warp;
   const bool live = row < rows;
-  float gm[kMaxV][8];
-  V8 xv[kMaxV], gv[kMaxV], av[kMaxV], ov[kMaxV];
-  float mu = 0.f, rs = 0.f;
-#pragma unroll
-  for (int v = 0; v < kMaxV; ++v) {
-#pragma unroll
-    for (int j = 0; j < 8; ++j) xv[v].v[j] = gv[v].v[j] = av[v].v[j] = ov[v].v[j] = gm[v][j] = 0.f;
-    if (v >= nv) continue;
-    const int c = (v * 32 + lane) * 8;
-    const float4 ga = __ldg(reinterpret_cast<const float4*>(gamma + c));
-    const float4 gb = __ldg(reinterpret_cast<const float4*>(gamma + c) + 1);
-    gm[v][0] = ga.x; gm[v][1] = ga.y; gm[v][2] = ga.z; gm[v][3] = ga.w;
-    gm[v][4] = gb.x; gm[v][5] = gb.y; gm[v][6] = gb.z; gm[v][7] = gb.w;
-    if (!live) continue;
-    xv[v] = ld8(x + row * C + c);
-    gv[v] = ld8(dy + row * C + c);
-    if (dx && addend) av[v] = ld8(addend + row * C + c);
-    if (dx && acc) ov[v] = ld8(dx + row * C + c);
-  }
+  const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+  uint4 xr[kMaxV] = {z, z}, gr[kMaxV] = {z, z}, ar[kMaxV] = {z, z}, orr[kMaxV] = {z, z};
   if (live) {
-    mu = mean[row];
-    rs = rstd[row];
+#pragma unroll
+    for (int v = 0; v < kMaxV; ++v) {
+      if (v >= nv) break;
+      const int64_t off = row * C + (v * 32 + lane) * 8;
+      xr[v] = *reinterpret_cast<const uint4*>(x + off);
+      gr[v] = *reinterpret_cast<const uint4*>(dy + off);
+      if (dx && addend) ar[v] = *reinterpret_cast<const uint4*>(addend + off);
+      if (dx && acc) orr[v] = *reinterpret_cast<const uint4*>(dx + off);
+    }
   }
+  const float mu = live ? mean[row] : 0.f, rs = live ? rstd[row] : 0.f;
   float a = 0.f, b = 0.f;
 #pragma unroll
   for (int v = 0; v < kMaxV; ++v) {
     if (v >= nv) break;
+    const int c = (v * 32 + lane) * 8;
+    float gm[8];
+    gamma8(gamma, c, gm);
+    float pgv[8], pbv[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      const float xh = (xv[v].v[j] - mu) * rs;
-      const float dxh = gv[v].v[j] * gm[v][j];
+      const float xh = (bf_at(xr[v], j) - mu) * rs;
+      const float g = bf_at(gr[v], j);
+      const float dxh = g * gm[j];
       a += dxh;
       b += dxh * xh;
+      pgv[j] = g * xh;
+      pbv[j] = g;
     }
+    // this row's contributions to the column partials (zeros past the end)
+    float4* rg = reinterpret_cast<float4*>(&redg[warp][c]);
+    float4* rb = reinterpret_cast<float4*>(&redb[warp][c]);
+    rg[0] = make_float4(pgv[0], pgv[1], pgv[2], pgv[3]);
+    rg[1] = make_float4(pgv[4], pgv[5], pgv[6], pgv[7]);
+    rb[0] = make_float4(pbv[0], pbv[1], pbv[2], pbv[3]);
+    rb[1] = make_float4(pbv[4], pbv[5], pbv[6], pbv[7]);
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -439,24 +453,20 @@ __global__ void __launch_bounds__(256) layernorm_bwd_fused_k(const bf16* __restr
   }
   a /= float(C);
   b /= float(C);
+  if (live && dx) {
 #pragma unroll
-  for (int v = 0; v < kMaxV; ++v) {
-    if (v >= nv) break;
-    const int c = (v * 32 + lane) * 8;
-    if (live && dx) {
+    for (int v = 0; v < kMaxV; ++v) {
+      if (v >= nv) break;
+      const int c = (v * 32 + lane) * 8;
+      float gm[8];
+      gamma8(gamma, c, gm);
       V8 o;
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
-        const float xh = (xv[v].v[j] - mu) * rs;
-        const float dxh = gv[v].v[j] * gm[v][j];
-        o.v[j] = rs * (dxh - a - xh * b) + ov[v].v[j] + av[v].v[j];
+        const float xh = (bf_at(xr[v], j) - mu) * rs;
+        o.v[j] = rs * (bf_at(gr[v], j) * gm[j] - a - xh * b) + bf_at(orr[v], j) + bf_at(ar[v], j);
       }
       st8(dx + row * C + c, o);
-    }
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {   // zeros for a row past the end
-      redg[warp][c + j] = gv[v].v[j] * ((xv[v].v[j] - mu) * rs);
-      redb[warp][c + j] = gv[v].v[j];
     }
   }
   __syncthreads();

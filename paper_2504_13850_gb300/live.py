@@ -55,7 +55,7 @@ class LivePipeline:
         self.local_steps = [0] * self.K
         self.order = W.arrival_order(self.scfg["rates"], 1_000_000, self.scfg["seed"] + seed)
         self.pos = 0
-        self.s_stream = torch.cuda.ExternalStream(self.server.stream(), device=dev)
+        self.a_stream = torch.cuda.ExternalStream(self.server.agg_stream(), device=dev)
         self.stats = {"device_iterations": 0, "uploads": 0, "refused": 0, "skipped_off": 0, "server_steps": 0,
                       "aggregations": 0, "stale": 0}
 
@@ -89,7 +89,7 @@ class LivePipeline:
                 self.version[k], _ = self.server.version()
                 # the device continues from the global model once the update is done
                 ev = self.torch.cuda.Event()
-                ev.record(self.s_stream)
+                ev.record(self.a_stream)
                 ev.synchronize()
                 d.load_params_device(self.global_model.data_ptr(), self.n_dev_params)
         else:

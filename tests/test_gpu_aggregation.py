@@ -20,6 +20,16 @@ def lib():
     api.lib()
 
 
+def agg(s, g, l, k, version):
+    """fo_aggregate ordered after the caller's torch work on its inputs and
+    completed before the caller reads the result (the aggregation runs on the
+    server's own stream)."""
+    torch.cuda.synchronize()
+    out = s.aggregate(g, l, k, version)
+    s.synchronize()
+    return out
+
+
 def tiny_server(max_delay=2**31 - 1):
     return api.Server.from_config(W.CONFIGS["tiny"], max_delay=max_delay)
 
@@ -51,7 +61,7 @@ def test_tiny_config_each_device_once_is_running_mean():
         step = O.Aggregator(cfg["K"], 2**31 - 1)
         step.t = k
         _, ref = step.aggregate(g_before, l, 0)
-        rc, t = s.aggregate(gd, torch.tensor(l, device="cuda"), k, 0)
+        rc, t = agg(s, gd, torch.tensor(l, device="cuda"), k, 0)
         assert rc == api.OK and t == k + 1
         check(gd.cpu().numpy(), ref, g_before, l)
         _, g_chain = chain.aggregate(g_chain, l, 0)
@@ -70,9 +80,9 @@ def test_ragged_sizes_and_unaligned_pointers(n, offset):
     s = tiny_server()
     # advance t so that alpha is not 1: three identity aggregations first
     for _ in range(3):
-        s.aggregate(gd[offset:], gd[offset:].clone(), 0, s.version()[0])
+        agg(s, gd[offset:], gd[offset:].clone(), 0, s.version()[0])
     g_mid = gd.cpu().numpy()[offset:].astype(np.float64)
-    rc, t = s.aggregate(gd[offset:], ld[offset:], 1, 1)        # t = 3, t_k = 1 -> alpha = 1/3
+    rc, t = agg(s, gd[offset:], ld[offset:], 1, 1)        # t = 3, t_k = 1 -> alpha = 1/3
     assert rc == api.OK and t == 4
     ref = (1 / 3) * l[offset:].astype(np.float64) + (1 - 1 / 3) * g_mid
     check(gd.cpu().numpy()[offset:], ref, g_mid, l[offset:])
@@ -85,7 +95,7 @@ def test_identity_is_bit_exact():
     before = g.clone()
     s = tiny_server()
     for v in range(5):
-        s.aggregate(g, g.clone(), 0, max(0, s.version()[0] - v % 3))
+        agg(s, g, g.clone(), 0, max(0, s.version()[0] - v % 3))
     assert torch.equal(g, before)
 
 
@@ -94,16 +104,16 @@ def test_stale_and_invalid_versions():
     g = torch.zeros(1000, device="cuda")
     l = torch.ones(1000, device="cuda")
     for _ in range(4):
-        s.aggregate(g, l, 0, s.version()[0])
+        agg(s, g, l, 0, s.version()[0])
     t = s.version()[0]
     before = g.clone()
-    rc, nv = s.aggregate(g, l * 5, 1, t - 3)
+    rc, nv = agg(s, g, l * 5, 1, t - 3)
     assert rc == api.STALE and nv == t and s.version()[0] == t
     torch.cuda.synchronize()
     assert torch.equal(g, before)
-    assert s.aggregate(g, l, 1, t + 1)[0] == api.ERR_ARG
-    assert s.aggregate(g, l, 1, -1)[0] == api.ERR_ARG
-    assert s.aggregate(g, l, 99, t)[0] == api.ERR_ARG
+    assert agg(s, g, l, 1, t + 1)[0] == api.ERR_ARG
+    assert agg(s, g, l, 1, -1)[0] == api.ERR_ARG
+    assert agg(s, g, l, 99, t)[0] == api.ERR_ARG
 
 
 @pytest.mark.parametrize("n", [16_000_000, 200_000_000])
