@@ -555,7 +555,8 @@ def run_ours(args):
                    "omega": cfg["omega"], "parallelism": f"replicas{world}",
                    "l2": f"not flushed: each step touches the server's {wsb / 1e6:.0f} MB of parameters, "
                          f"momentum, gradients, activations and scratch, above the 126 MB L2",
-                   "switches": {k: os.environ.get(k) for k in ("FO_NO_TC", "FO_NO_GRAPH", "FO_NO_SIDE", "FO_NO_PDL")}},
+                   "switches": {k: os.environ.get(k) for k in ("FO_NO_TC", "FO_NO_GRAPH", "FO_NO_SIDE", "FO_NO_PDL",
+                                                                "FO_NO_POOL_EPILOGUE")}},
         "e2e": e2e,
         "gpu_launches": int(launches),
         "roofline": roof,

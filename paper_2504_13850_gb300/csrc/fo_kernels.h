@@ -37,6 +37,11 @@ void maxpool2_fwd(const void* x, void* y, int N, int H, int W, int C, int dt, cu
 void maxpool2_bwd(const void* x, const void* dy, void* dx, int N, int H, int W, int C,
                   int dt, bool acc, cudaStream_t st);
 // Fused backward of relu(x) followed by maxpool2: dx (+)= route(dy) * (x > 0)
+// ReLU + 2x2 max-pool backward from the pooled values y and the window codes
+// (first-maximum position 0..3 per pooled element) that a GEMM epilogue
+// stored in the forward pass (bf16, C % 8 == 0).
+void relu_maxpool2_bwd_codes(const void* y, const uint8_t* code, const void* dy, void* dx, int N, int H, int W,
+                             int C, bool acc, cudaStream_t st);
 void relu_maxpool2_bwd(const void* x, const void* dy, void* dx, int N, int H, int W, int C,
                        int dt, bool acc, cudaStream_t st);
 void affine_fwd(const void* x, const float* scale, const float* shift, void* y, int64_t rows,
@@ -110,6 +115,16 @@ void sgd_momentum(float* theta, float* v, const float* g, void* shadow, int64_t 
                   float mu, int64_t* step, cudaStream_t st, const uint8_t* skip64 = nullptr);
 // The update restricted to the 64-element blocks listed in blocks64 (device,
 // nb entries: block b covers elements 64b .. 64b + 63).
+// Contiguous segments of the parameter vector updated by one launch:
+// segment k is float4 elements [off4[k], off4[k] + pre4[k+1] - pre4[k]).
+constexpr int kSgdMaxSegs = 32;
+struct SgdSegments {
+  int n;
+  int64_t off4[kSgdMaxSegs];
+  int64_t pre4[kSgdMaxSegs + 1];
+};
+void sgd_momentum_segments(float* theta, float* v, const float* g, void* shadow, const SgdSegments& sg, float lr,
+                           float mu, cudaStream_t st);
 void sgd_momentum_blocks(float* theta, float* v, const float* g, void* shadow, const int64_t* blocks64, int64_t nb,
                          float lr, float mu, int64_t* step, cudaStream_t st);
 void f32_to_bf16(const float* x, void* y, int64_t n, cudaStream_t st);

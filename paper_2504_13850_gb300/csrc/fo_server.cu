@@ -47,6 +47,9 @@ int64_t pad64(int64_t n) { return (n + 63) / 64 * 64; }
 // soon as their gradient is final; smaller ones (where a launch costs more
 // than the traffic it moves) are left to the step's final update.
 constexpr int64_t kEarlyUpdateMin = 128 * 1024;
+// Early updates are batched: consecutive weight tensors share one launch once
+// they add up to this many parameters (or the segment table is full).
+constexpr int64_t kEarlyGroupMin = 1024 * 1024;
 
 // Shape inference and parameter layout.  Returns FO_OK or an error.
 int infer(fo_server* s) {
@@ -335,10 +338,15 @@ int build_plan(fo_server* s) {
   };
   const int L = nops - 1;  // the logits layer
 
+  // Max-pools computed by the epilogue of the conv / linear in front of them
+  // (through its ReLU): per pool op, the window codes that epilogue stores,
+  // or null.
+  std::vector<uint8_t*> pool_codes(nops, nullptr);
+
   // ---------------- forward
   for (int i = 0; i < nops; ++i) {
     const fo_op op = s->ops[i];
-    if (fu.skip_fwd[i]) continue;
+    if (fu.skip_fwd[i] || pool_codes[i]) continue;
     const int a = op.in0;
     // output buffer: a fused relu writes the relu's output tensor, a fused
     // residual add the add's output
@@ -375,7 +383,29 @@ int build_plan(fo_server* s) {
           if (r == 0) ex.addend_is_input = true;
           else ex.addend = s->T[r].act;
         }
-        fo::TcGemm* tg = fo::tc_plan_forward(s->tc, s, i, s->T[o].act, relu, fused ? &ex : nullptr);
+        fo::TcGemm* tg = nullptr;
+        // ReLU then a 2x2 max-pool that alone reads the ReLU output and applies
+        // its mask in the backward pass: the pool goes into this epilogue
+        const int pr = fu.fwd_relu[i];
+        int pq = -1;
+        if (pr >= 0 && !fused && dt == fo::kBF16 && s->T[pr + 1].consumers == 1 && !getenv("FO_NO_POOL_EPILOGUE"))
+          for (int q = pr + 1; q < nops; ++q)
+            if (s->ops[q].in0 == pr + 1) {
+              if (s->ops[q].kind == FO_OP_MAXPOOL2 && fu.bwd_mask[q] == pr) pq = q;
+              break;
+            }
+        if (pq >= 0) {
+          const Tensor& tp = s->T[pq + 1];
+          uint8_t* codes = (uint8_t*)s->alloc(size_t(tp.numel()));
+          if (!codes) return set_err(FO_ERR_OOM, "max-pool window codes");
+          ex.pool_out = tp.act;
+          ex.pool_code = codes;
+          tg = fo::tc_plan_forward(s->tc, s, i, s->T[o].act, relu, &ex);
+          if (tg) pool_codes[pq] = codes;
+          ex.pool_out = nullptr;
+          ex.pool_code = nullptr;
+        }
+        if (!tg) tg = fo::tc_plan_forward(s->tc, s, i, s->T[o].act, relu, fused ? &ex : nullptr);
         if (fused && !tg) return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": fused epilogue not planned");
         if (tg) {
           add_tc(tg);
@@ -556,6 +586,17 @@ int build_plan(fo_server* s) {
   // (their layer's input gradient has run): the update's HBM traffic then
   // overlaps the rest of the backward pass.  Flags per 64 parameters.
   std::vector<uint8_t> early(size_t(s->n_padded / 64), 0);
+  fo::SgdSegments group{};
+  int64_t group_params = 0;
+  auto flush_group = [&]() {
+    if (group.n == 0) return;
+    const fo::SgdSegments sg = group;
+    add("sgd_momentum", 1, 0.0, double(sg.pre4[sg.n]) * 4.0 * (20.0 + (s->shadow ? 2.0 : 0.0)), [=](cudaStream_t st) {
+      fo::sgd_momentum_segments(s->theta, s->mom, s->grad, s->shadow, sg, s->opt.lr, s->opt.momentum, st);
+    }, 2);
+    group = fo::SgdSegments{};
+    group_params = 0;
+  };
   for (int i = nops - 1; i >= 0; --i) {
     const fo_op op = s->ops[i];
     if (fu.skip_bwd[i]) {
@@ -665,15 +706,16 @@ int build_plan(fo_server* s) {
           }
         }
         if (s->segs[s->op_segs[i][0]].n >= kEarlyUpdateMin) {
-          // the weights' update, forked after the input gradient that read them
+          // the weights' update, after the input gradient that read them:
+          // batched with the next weight tensors until the batch is large
           const ParamSeg seg = s->segs[s->op_segs[i][0]];
           const int64_t len = pad64(seg.n);
-          add("sgd_momentum", 1, 0.0, double(len) * (20.0 + (s->shadow ? 2.0 : 0.0)), [=](cudaStream_t st) {
-            fo::sgd_momentum(s->theta + seg.off, s->mom + seg.off, s->grad + seg.off,
-                             s->shadow ? (void*)(s->shadow + seg.off) : nullptr, len, s->opt.lr, s->opt.momentum,
-                             nullptr, st);
-          }, 2);
+          group.off4[group.n] = seg.off / 4;
+          group.pre4[group.n + 1] = group.pre4[group.n] + len / 4;
+          ++group.n;
+          group_params += len;
           for (int64_t b = seg.off / 64; b < (seg.off + len) / 64; ++b) early[size_t(b)] = 1;
+          if (group_params >= kEarlyGroupMin || group.n == fo::kSgdMaxSegs) flush_group();
         }
         break;
       }
@@ -721,6 +763,16 @@ int build_plan(fo_server* s) {
         }
         break;
       case FO_OP_MAXPOOL2:
+        if (need_dx && pool_codes[i]) {   // forward ran in the producing GEMM's epilogue
+          int accf = contrib(a);
+          const uint8_t* codes = pool_codes[i];
+          add("relu_maxpool2_bwd", 1, 0.0, (2 + accf) * tbytes(a0) + 2.5 * csb, [=](cudaStream_t st) {
+            const Tensor& x = s->T[a0];
+            fo::relu_maxpool2_bwd_codes(s->T[o].act, codes, s->T[o].grad, s->T[a].grad, x.N, x.H, x.W, x.C,
+                                        accf != 0, st);
+          });
+          break;
+        }
         if (need_dx) {
           int accf = contrib(a);
           const bool masked = mr >= 0;
@@ -922,6 +974,7 @@ int build_plan(fo_server* s) {
   }
 
   for (int r = 0; r <= nops; ++r) materialize(r);
+  flush_group();
 
   // ---------------- optimizer (Algorithm 4: theta_s <- theta_s - gamma_s * update)
   if (!bias_tasks.empty())

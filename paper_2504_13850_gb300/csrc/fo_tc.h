@@ -26,6 +26,11 @@ struct TcEpilogue {
   // pass (bf16, out's layout)
   const void* addend = nullptr;
   bool addend_is_input = false;   // the addend is the uploaded batch of the step's slot
+  // forward with ReLU: a 2x2 max-pool of the output (output width <= 16):
+  // the pooled values [N][H/2][W/2][C] and the window code of each pooled
+  // element (first maximum, 0..3 row-major) instead of the full output
+  void* pool_out = nullptr;
+  uint8_t* pool_code = nullptr;
 };
 // Forward of conv/linear op `op` into `out` (bf16, the op's output layout),
 // applying a ReLU when `relu`.

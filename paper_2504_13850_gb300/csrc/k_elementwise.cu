@@ -213,6 +213,64 @@ __global__ void maxpool2_bwd_x8_k(const bf16* __restrict__ x, const bf16* __rest
   }
 }
 
+// Backward of a 2x2 max-pool (after a ReLU) whose forward ran in the
+// producing GEMM's epilogue: that epilogue stored the pooled values and, per
+// pooled element and channel, the window position of the first maximum
+// (code 0..3, row-major).  The window's gradient goes to that position if the
+// pooled value is > 0 (the ReLU mask there), the other three get zero.
+__global__ void maxpool2_bwd_codes_x8_k(const bf16* __restrict__ y, const uint8_t* __restrict__ code,
+                                        const bf16* __restrict__ dy, bf16* __restrict__ dx, int N, int H, int W,
+                                        int C, int acc) {
+  pdl_wait();
+  pdl_trigger();
+  const int Ho = H / 2, Wo = W / 2, C8 = C / 8;
+  const int64_t n_out = int64_t(N) * Ho * Wo * C8;
+  GRID_STRIDE(o, n_out) {
+    const int c8 = int(o % C8);
+    int64_t t = o / C8;
+    const int j = int(t % Wo);
+    t /= Wo;
+    const int i = int(t % Ho);
+    const int n = int(t / Ho);
+    const int64_t b0 = ((int64_t(n) * H + 2 * i) * W + 2 * j) * C + 8 * c8;
+    const int64_t offs[4] = {b0, b0 + C, b0 + int64_t(W) * C, b0 + int64_t(W) * C + C};
+    const uint4 y4 = *reinterpret_cast<const uint4*>(y + o * 8);
+    const uint4 g4 = *reinterpret_cast<const uint4*>(dy + o * 8);
+    const uint2 c2 = *reinterpret_cast<const uint2*>(code + o * 8);
+    const bf16* yb = reinterpret_cast<const bf16*>(&y4);
+    const bf16* gb = reinterpret_cast<const bf16*>(&g4);
+    const uint8_t* cb = reinterpret_cast<const uint8_t*>(&c2);
+    float out[4][8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const float g = __bfloat162float(yb[e]) > 0.f ? __bfloat162float(gb[e]) : 0.f;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) out[q][e] = q == int(cb[e]) ? g : 0.f;
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      uint4* d = reinterpret_cast<uint4*>(dx + offs[q]);
+      if (acc) {
+        const uint4 old = *d;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) out[q][e] += __bfloat162float(reinterpret_cast<const bf16*>(&old)[e]);
+      }
+      uint4 r;
+      bf16* rb = reinterpret_cast<bf16*>(&r);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) rb[e] = __float2bfloat16_rn(out[q][e]);
+      *d = r;
+    }
+  }
+}
+
+void relu_maxpool2_bwd_codes(const void* y, const uint8_t* code, const void* dy, void* dx, int N, int H, int W,
+                             int C, bool acc, cudaStream_t st) {
+  const int64_t n = int64_t(N) * (H / 2) * (W / 2) * C;
+  launch_k(maxpool2_bwd_codes_x8_k, elementwise_blocks(n / 8, 256), 256, 0, st, (const bf16*)y, code,
+           (const bf16*)dy, (bf16*)dx, N, H, W, C, acc ? 1 : 0);
+}
+
 void maxpool2_fwd(const void* x, void* y, int N, int H, int W, int C, int dt, cudaStream_t st) {
   int64_t n = int64_t(N) * (H / 2) * (W / 2) * C;
   if (dt == kBF16 && C % 8 == 0) {
@@ -677,6 +735,46 @@ void sgd_momentum_blocks(float* theta, float* v, const float* g, void* shadow, c
                          float lr, float mu, int64_t* step, cudaStream_t st) {
   launch_k(sgd_momentum_blocks_k, elementwise_blocks(nb * 16, 256), 256, 0, st, (float4*)theta, (float4*)v,
            (const float4*)g, (uint2*)shadow, blocks64, nb, lr, mu, step);
+}
+// The same update over up to kSgdMaxSegs contiguous segments of the
+// parameter vector in one launch (weight tensors whose gradients are final),
+// so that several small tensors share the launch and its ramp: thread j of the
+// concatenated float4 range finds its segment in the prefix table.
+__global__ void sgd_momentum_segs_k(float4* __restrict__ theta, float4* __restrict__ v,
+                                    const float4* __restrict__ g, uint2* __restrict__ shadow,
+                                    const __grid_constant__ SgdSegments sg, float lr, float mu) {
+  pdl_wait();
+  pdl_trigger();
+  GRID_STRIDE(j, sg.pre4[sg.n]) {
+    int k = 0;
+    while (k + 1 < sg.n && sg.pre4[k + 1] <= j) ++k;
+    const int64_t i = sg.off4[k] + (j - sg.pre4[k]);
+    float4 t = theta[i], m = v[i];
+    const float4 gr = g[i];
+    m.x = fmaf(mu, m.x, gr.x);
+    m.y = fmaf(mu, m.y, gr.y);
+    m.z = fmaf(mu, m.z, gr.z);
+    m.w = fmaf(mu, m.w, gr.w);
+    t.x = fmaf(-lr, m.x, t.x);
+    t.y = fmaf(-lr, m.y, t.y);
+    t.z = fmaf(-lr, m.z, t.z);
+    t.w = fmaf(-lr, m.w, t.w);
+    v[i] = m;
+    theta[i] = t;
+    if (shadow) {
+      __nv_bfloat162 lo = __floats2bfloat162_rn(t.x, t.y), hi = __floats2bfloat162_rn(t.z, t.w);
+      uint2 u;
+      u.x = *reinterpret_cast<uint32_t*>(&lo);
+      u.y = *reinterpret_cast<uint32_t*>(&hi);
+      shadow[i] = u;
+    }
+  }
+}
+void sgd_momentum_segments(float* theta, float* v, const float* g, void* shadow, const SgdSegments& sg, float lr,
+                           float mu, cudaStream_t st) {
+  if (sg.n <= 0) return;
+  launch_k(sgd_momentum_segs_k, elementwise_blocks(sg.pre4[sg.n], 256), 256, 0, st, (float4*)theta, (float4*)v,
+           (const float4*)g, (uint2*)shadow, sg, lr, mu);
 }
 __global__ void f32_to_bf16_k(const float* x, bf16* y, int64_t n) {
   pdl_wait();

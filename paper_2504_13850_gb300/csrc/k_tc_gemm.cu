@@ -19,7 +19,8 @@ namespace {
 
 // The epilogue variant a plan's parameters ask for.
 int epi_of(const TcParams& p) {
-  return (p.out_f32 ? E_F32 : 0) | (p.relu ? E_RELU : 0) | (p.mask ? E_MASK : 0) | (p.acc ? E_ACC : 0);
+  return (p.out_f32 ? E_F32 : 0) | (p.relu ? E_RELU : 0) | (p.mask ? E_MASK : 0) | (p.acc ? E_ACC : 0) |
+         (p.pool_out ? E_POOL : 0);
 }
 
 KernelFn pick_kernel(int kind, int bn, bool cluster, int epi, size_t* smem) {
@@ -370,6 +371,8 @@ bool tc_plain_ok(TcContext* c, const fo_server* s, int i) {
 
 static void apply_epilogue(TcGemm* g, const TcEpilogue* ex) {
   if (!ex) return;
+  g->p.pool_out = static_cast<bf16*>(ex->pool_out);
+  g->p.pool_code = ex->pool_code;
   if (ex->addend || ex->addend_is_input) {
     g->p.acc = 1;
     g->p.accsrc = static_cast<const bf16*>(ex->addend);
@@ -383,11 +386,16 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i, void* out, bool relu,
   const Tensor& a = s->T[op.in0];
   const Tensor& o = s->T[i + 1];
   if (o.dt != kBF16) return nullptr;  // fp32 logits: CUDA-core path
-  if (ex && (relu || !plain_gemm(op))) return nullptr;
+  if (ex && (ex->addend || ex->addend_is_input) && (relu || !plain_gemm(op))) return nullptr;
+  if (ex && ex->pool_out) {   // whole 2 x 2 windows inside each warp's 32 rows
+    const bool w_ok = o.W == 2 || o.W == 4 || o.W == 8 || o.W == 16;
+    if (!relu || !w_ok || o.H % 2 || o.C % 8 || o.rows() % BM) return nullptr;
+  }
   TcGemm* g = new TcGemm();
   g->p.out = out;
   g->p.ldo = o.C;
   g->p.relu = relu ? 1 : 0;
+  g->p.pool_w = o.W;
   apply_epilogue(g, ex);
   g->p.bias = op.bias ? s->theta + s->segs[s->op_segs[i][1]].off : nullptr;
   const bf16* w = s->shadow + s->segs[s->op_segs[i][0]].off;

@@ -307,29 +307,28 @@ __global__ void __launch_bounds__(256) colsum8_batch_k(const __grid_constant__ C
                    local % cbs, local / cbs);
 }
 
-// Layernorm forward, one warp per row held in registers (C % 256 == 0,
-// C <= 1024): one read of x, mean then biased variance from the registers
-// (eps 1e-5), one write of y; the row mean and 1/std are kept for the
-// backward pass.  gamma and beta are read as float4 alongside x, so that
-// the row's only dependent global access is x itself.
-__global__ void __launch_bounds__(256) layernorm_fwd_x8_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
+// Layernorm forward, one warp per row held in registers (C = 256 NV,
+// NV <= 4, a template parameter so that a 512-column row takes only the
+// registers it needs and four blocks fit per SM): one read of x, mean then
+// biased variance from the registers (eps 1e-5), one write of y; the row
+// mean and 1/std are kept for the backward pass.  gamma and beta are read as
+// float4 alongside x, so that the row's only dependent global access is x.
+template <int NV>
+__global__ void __launch_bounds__(256, NV <= 2 ? 4 : 2) layernorm_fwd_x8_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
                                                           const float* __restrict__ beta, bf16* __restrict__ y,
                                                           float* __restrict__ mean_out, float* __restrict__ rstd_out,
                                                           int64_t rows, int C) {
   pdl_wait();
   pdl_trigger();
-  constexpr int kMaxV = 4;
   const int lane = threadIdx.x % 32;
   const int64_t row = int64_t(blockIdx.x) * (blockDim.x / 32) + threadIdx.x / 32;
   if (row >= rows) return;
-  const int nv = C / 256;
-  V8 xv[kMaxV];
-  float4 g4[kMaxV][2], b4[kMaxV][2];
+  uint4 xr[NV];
+  float4 g4[NV][2], b4[NV][2];
 #pragma unroll
-  for (int v = 0; v < kMaxV; ++v) {
-    if (v >= nv) break;
+  for (int v = 0; v < NV; ++v) {
     const int c = (v * 32 + lane) * 8;
-    xv[v] = ld8(x + row * C + c);
+    xr[v] = *reinterpret_cast<const uint4*>(x + row * C + c);
     g4[v][0] = __ldg(reinterpret_cast<const float4*>(gamma + c));
     g4[v][1] = __ldg(reinterpret_cast<const float4*>(gamma + c) + 1);
     b4[v][0] = __ldg(reinterpret_cast<const float4*>(beta + c));
@@ -337,36 +336,32 @@ __global__ void __launch_bounds__(256) layernorm_fwd_x8_k(const bf16* __restrict
   }
   float sum = 0.f;
 #pragma unroll
-  for (int v = 0; v < kMaxV; ++v) {
-    if (v >= nv) break;
+  for (int v = 0; v < NV; ++v)
 #pragma unroll
-    for (int j = 0; j < 8; ++j) sum += xv[v].v[j];
-  }
+    for (int j = 0; j < 8; ++j) sum += __bfloat162float(reinterpret_cast<const bf16*>(&xr[v])[j]);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
   const float mu = sum / float(C);
   float q = 0.f;
 #pragma unroll
-  for (int v = 0; v < kMaxV; ++v) {
-    if (v >= nv) break;
+  for (int v = 0; v < NV; ++v)
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      const float d = xv[v].v[j] - mu;
+      const float d = __bfloat162float(reinterpret_cast<const bf16*>(&xr[v])[j]) - mu;
       q = fmaf(d, d, q);
     }
-  }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
   const float rs = rsqrtf(q / float(C) + 1e-5f);
 #pragma unroll
-  for (int v = 0; v < kMaxV; ++v) {
-    if (v >= nv) break;
+  for (int v = 0; v < NV; ++v) {
     const int c = (v * 32 + lane) * 8;
     const float gm[8] = {g4[v][0].x, g4[v][0].y, g4[v][0].z, g4[v][0].w, g4[v][1].x, g4[v][1].y, g4[v][1].z, g4[v][1].w};
     const float bt[8] = {b4[v][0].x, b4[v][0].y, b4[v][0].z, b4[v][0].w, b4[v][1].x, b4[v][1].y, b4[v][1].z, b4[v][1].w};
     V8 o;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) o.v[j] = (xv[v].v[j] - mu) * rs * gm[j] + bt[j];
+    for (int j = 0; j < 8; ++j)
+      o.v[j] = (__bfloat162float(reinterpret_cast<const bf16*>(&xr[v])[j]) - mu) * rs * gm[j] + bt[j];
     st8(y + row * C + c, o);
   }
   if (lane == 0) {
@@ -740,8 +735,9 @@ int layernorm_bwd8_blocks(int64_t rows) { return int((rows + 7) / 8); }
 bool layernorm_fwd8_ok(int dt, int C) { return dt == kBF16 && C % 256 == 0 && C <= 1024; }
 void layernorm_fwd_x8(const void* x, const float* gamma, const float* beta, void* y, float* mean, float* rstd,
                       int64_t rows, int C, cudaStream_t st) {
-  launch_k(layernorm_fwd_x8_k, ceil_div(rows, 8), 256, 0, st, (const bf16*)x, gamma, beta, (bf16*)y, mean, rstd, rows,
-           C);
+  auto k = C <= 256 ? layernorm_fwd_x8_k<1> : C <= 512 ? layernorm_fwd_x8_k<2> : C <= 768 ? layernorm_fwd_x8_k<3>
+                                                                               : layernorm_fwd_x8_k<4>;
+  launch_k(k, ceil_div(rows, 8), 256, 0, st, (const bf16*)x, gamma, beta, (bf16*)y, mean, rstd, rows, C);
 }
 
 void layernorm_bwd8_pass(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,

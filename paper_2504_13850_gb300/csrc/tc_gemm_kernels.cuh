@@ -39,6 +39,10 @@ enum Epi : int {
   E_MASK = 2,   // ReLU mask of the input-gradient: y = 0 where mask <= 0
   E_ACC = 4,    // y += accsrc (accumulate, or a residual add into a new buffer)
   E_F32 = 8,    // fp32 output, nothing else (the weight gradients)
+  E_POOL = 16,  // with E_RELU: a 2x2 max-pool of the conv output (pool_w <= 16
+                // columns per image row, so a warp's 32 rows hold whole
+                // windows); writes the pooled values and the window codes
+                // instead of the full-resolution output
 };
 
 constexpr int BM = 128;      // UMMA M (cta_group::1)
@@ -81,6 +85,13 @@ struct TcParams {
   // is `out` itself unless the sum goes to a new buffer (a residual add:
   // out = result + accsrc).
   const bf16* accsrc;
+  // E_POOL: pooled output [N][H/2][W/2][ldo] and the position of each
+  // window's first maximum (0..3, row-major) per pooled element; pool_w is the
+  // output image width W (GEMM rows are (n, h, w) with h, w the image row and
+  // column)
+  bf16* pool_out;
+  uint8_t* pool_code;
+  int pool_w;
   int* err;
   // split-K: fp32 partial tiles, [tile][rank][BN/32][8][BM] float4 (tile =
   // blockIdx.y * gridDim.x + blockIdx.x); only rows a rank does not own are written
@@ -92,6 +103,16 @@ __device__ __forceinline__ size_t out_row(const TcParams& p, int m) {
   const int hw = p.Hq * p.Wq;
   const int n = m / hw, rem = m % hw, i = rem / p.Wq, j = rem % p.Wq;
   return (size_t(n) * p.oH + p.ostride * i + p.py) * p.oW + p.ostride * j + p.px;
+}
+
+// Pooled row of window `win` (0..7) of the 32 GEMM rows from m_base (m_base a
+// multiple of 2 W, so the rows are whole image rows starting at an even one),
+// and the GEMM row (offset from m_base) of the window's top-left position.
+__device__ __forceinline__ void pool_window(const TcParams& p, int m_base, int win, size_t* prow, int* r0) {
+  const int W = p.pool_w, wp = W / 2;
+  const int hp = win / wp, wq = win % wp;
+  *r0 = 2 * hp * W + 2 * wq;
+  *prow = (size_t(m_base / W) / 2 + hp) * wp + wq;
 }
 
 // Epilogue of 32 consecutive outputs (m, n..n+31) held by one thread: bias,
@@ -162,6 +183,46 @@ __device__ __forceinline__ void store_row32(const TcParams& p, int m_gemm, int n
   }
 }
 
+// E_POOL in the split-K owner: lane = GEMM row m_base + lane with its 32
+// columns v (bias and ReLU applied); the 2 x 2 windows are lanes {l, l ^ 1,
+// l ^ W, l ^ W ^ 1}, reduced with shuffles (first maximum in row-major
+// window order), and the window's top-left lane stores the pooled values and
+// codes.  Every lane of the warp must call it.
+template <int EPI>
+__device__ __forceinline__ void pool_row32(const TcParams& p, int m_base, int lane, int n, const float (&v)[32]) {
+  const int W = p.pool_w;
+  const int pos = ((lane / W) & 1) * 2 + (lane & 1);   // this lane's place in its window
+  float mx[32];
+  uint32_t cd[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    float m = fmaxf(v[j], __shfl_xor_sync(0xffffffffu, v[j], 1));
+    m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, W));
+    int c = v[j] == m ? pos : 4;
+    c = min(c, __shfl_xor_sync(0xffffffffu, c, 1));
+    c = min(c, __shfl_xor_sync(0xffffffffu, c, W));
+    mx[j] = m;
+    cd[j / 4] |= uint32_t(c) << (8 * (j % 4));
+  }
+  if (pos != 0) return;   // the window's top-left lane stores
+  const int hp = (lane / W) / 2, wq = (lane % W) / 2;
+  const size_t prow = (size_t(m_base / W) / 2 + hp) * (W / 2) + wq;
+  const int nv = p.N - n;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    if (8 * j >= nv) break;
+    uint4 pk;
+    uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      __nv_bfloat162 h2 = __floats2bfloat162_rn(mx[8 * j + 2 * q], mx[8 * j + 2 * q + 1]);
+      pw[q] = *reinterpret_cast<uint32_t*>(&h2);
+    }
+    *reinterpret_cast<uint4*>(p.pool_out + prow * p.ldo + n + 8 * j) = pk;
+    *reinterpret_cast<uint2*>(p.pool_code + prow * p.ldo + n + 8 * j) = make_uint2(cd[2 * j], cd[2 * j + 1]);
+  }
+}
+
 // Coalesced epilogue of a 32-row x 32-column accumulator chunk held one row
 // per lane (lane = row, r[j] = column j).  The warp stages the chunk in its
 // 4 KB shared-memory buffer (16-byte units XOR-swizzled by row, so both the
@@ -212,7 +273,43 @@ __device__ __forceinline__ void epilogue_chunk32(const TcParams& p, uint32_t sta
   for (int j = 0; j < 8; ++j)
     st_shared4(stage + 16u * (lane * 8 + (j ^ (lane & 7))), r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
   __syncwarp();
-  if constexpr (EPI & E_F32) {   // a weight gradient: plain fp32 store, 4 rows x 128 B per instruction
+  if constexpr (EPI & E_POOL) {   // 2 x 2 max-pool of the chunk's 32 rows: lane = (window, 8 channels)
+    const int win = lane >> 2;
+    size_t prow;
+    int r0;
+    pool_window(p, m_base, win, &prow, &r0);
+    if (n + 8 * co < p.N) {
+      float best[8];
+      int arg[8];
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        const int rr = r0 + (t >> 1) * p.pool_w + (t & 1);
+        const float4 v0 = ld_shared4(stage + 16u * (rr * 8 + ((2 * co) ^ (rr & 7))));
+        const float4 v1 = ld_shared4(stage + 16u * (rr * 8 + ((2 * co + 1) ^ (rr & 7))));
+        const float e[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const float x = fmaxf(e[q] + b[q], 0.f);   // bias and ReLU, then the window maximum
+          if (t == 0 || x > best[q]) {
+            best[q] = x;
+            arg[q] = t;
+          }
+        }
+      }
+      uint4 pk;
+      uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        __nv_bfloat162 h2 = __floats2bfloat162_rn(best[2 * q], best[2 * q + 1]);
+        pw[q] = *reinterpret_cast<uint32_t*>(&h2);
+      }
+      const size_t off = prow * p.ldo + n + 8 * co;
+      *reinterpret_cast<uint4*>(p.pool_out + off) = pk;
+      *reinterpret_cast<uint2*>(p.pool_code + off) =
+          make_uint2(uint32_t(arg[0]) | uint32_t(arg[1]) << 8 | uint32_t(arg[2]) << 16 | uint32_t(arg[3]) << 24,
+                     uint32_t(arg[4]) | uint32_t(arg[5]) << 8 | uint32_t(arg[6]) << 16 | uint32_t(arg[7]) << 24);
+    }
+  } else if constexpr (EPI & E_F32) {   // a weight gradient: plain fp32 store, 4 rows x 128 B per instruction
     const int cq = lane & 7;     // 16-byte unit: columns 4cq .. 4cq+3
 #pragma unroll 1
     for (int it = 0; it < 8; ++it) {
@@ -488,7 +585,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
       if (c + 1 < c1) load_row32<EPI>(p, mg, n0 + 32 * (c + 1), mk2, ac2);
       uint32_t r[32];
       tmem_ld32(trow + uint32_t(32 * c), r);
-      if (mg < p.M) {
+      if (mg < p.M || (EPI & E_POOL)) {   // a pooled conv has M % 128 == 0: every lane takes part
         float v[32];
 #pragma unroll
         for (int j = 0; j < 32; ++j) v[j] = 0.f;
@@ -506,7 +603,20 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             }
           }
         }
-        store_row32<EPI>(p, mg, n0 + 32 * c, v, smem_u32(sbias) + uint32_t(32 * c) * 4u, mk, ac);
+        if constexpr (EPI & E_POOL) {
+          const uint32_t sb = smem_u32(sbias) + uint32_t(32 * c) * 4u;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float4 bb = ld_shared4(sb + 16u * j);
+            v[4 * j] = fmaxf(v[4 * j] + bb.x, 0.f);
+            v[4 * j + 1] = fmaxf(v[4 * j + 1] + bb.y, 0.f);
+            v[4 * j + 2] = fmaxf(v[4 * j + 2] + bb.z, 0.f);
+            v[4 * j + 3] = fmaxf(v[4 * j + 3] + bb.w, 0.f);
+          }
+          pool_row32<EPI>(p, m0 + q * 32, lane, n0 + 32 * c, v);
+        } else {
+          store_row32<EPI>(p, mg, n0 + 32 * c, v, smem_u32(sbias) + uint32_t(32 * c) * 4u, mk, ac);
+        }
       }
 #pragma unroll
       for (int j = 0; j < 4; ++j) {

@@ -194,16 +194,20 @@ def grad_bound(reading_err):
     stored tensor the same way, shows it on the same step (`reading_err`).
     A correct path is another draw of the same rounding process, so its
     distance from the exact gradient matches the reading's up to the
-    draw-to-draw spread; measured on the GPU it stays within 1.12 times the
-    reading's on every tensor of well-conditioned steps.  The bound is twice
-    the reading's distance, and never below GRAD_FLOOR.  It does not cover
+    draw-to-draw spread.  That spread is large where only a handful of
+    elements sit near a kink (a small layer at a small batch): on one step
+    the reading may flip none of them while the path flips one, which moves
+    a 1,536-element layer's gradient by ~6%.  The flip rate itself belongs to
+    the network and its data, not to the step, so the allowance takes the
+    reading's largest distance for that tensor over the steps of the run:
+    the bound is twice that, and never below GRAD_FLOOR.  It does not cover
     steps whose softmax is saturated (loss far above ln C), where a one-ulp
     change of a logit moves the classifier's gradient by several percent;
     the tests keep their losses near ln C."""
     return max(GRAD_FLOOR, FLIP_FACTOR * reading_err)
 
 
-def gate_failures(rec, loss_tol=LOSS_TOL, param_tol=PARAM_TOL):
+def gate_failures(rec, loss_tol=LOSS_TOL, param_tol=PARAM_TOL, reading=None):
     """Every gate one teacher-forced step record fails (empty if none):
       * loss within loss_tol of the exact loss (relative);
       * parameters within param_tol of the exact step (normwise);
@@ -213,8 +217,11 @@ def gate_failures(rec, loss_tol=LOSS_TOL, param_tol=PARAM_TOL):
         |g| / |mu v0 + g| (the update is -lr (mu v0 + g) with v0 shared, so
         its error is the gradient's over that ratio), plus 1e-3 for the fp32
         rounding of theta1: a step that skips or mis-scales the update
-        fails here even when its gradient is right."""
-    ex, rd = rec["exact"], rec["reading"]
+        fails here even when its gradient is right.
+    `reading` (per-tensor and whole distances of the bf16-storage reading,
+    the run's largest) replaces this record's own."""
+    ex = rec["exact"]
+    rd = reading if reading is not None else rec["reading"]
     bad = []
     if abs(rec["loss"] - ex["loss"]) > loss_tol * abs(ex["loss"]):
         bad.append(("loss", rec["loss"], ex["loss"]))
@@ -233,9 +240,18 @@ def gate_failures(rec, loss_tol=LOSS_TOL, param_tol=PARAM_TOL):
     return bad
 
 
+def run_reading(recs):
+    """The bf16-storage reading's largest distance from the exact gradient
+    over a run's steps, per tensor and for the whole gradient."""
+    return {"whole": max(r["reading"]["whole"] for r in recs),
+            "tensor": {n: max(r["reading"]["tensor"][n] for r in recs) for n in recs[0]["reading"]["tensor"]}}
+
+
 def check_teacher_forced(recs, **kw):
-    """All gates of gate_failures on every step; the bf16-storage reading's
-    own comparison stays in the records as a diagnostic."""
+    """All gates of gate_failures on every step, with the run's largest
+    reading distances; the bf16-storage reading's own comparison stays in
+    the records as a diagnostic."""
+    reading = run_reading(recs)
     for r in recs:
-        bad = gate_failures(r, **kw)
+        bad = gate_failures(r, reading=reading, **kw)
         assert not bad, (r["step"], bad, r["stored"]["tensor_grad_err"])
