@@ -188,9 +188,13 @@ int64_t layernorm_bwd8_partial_floats(int64_t rows, int C);
 // of dgamma and dbeta.
 int layernorm_bwd8_blocks(int64_t rows);
 // dx = (dx if acc) + input gradient + (addend if given, dx's layout).
+// With p_dx, also the column partial sums of the stored dx per block
+// ([layernorm_bwd8_blocks(rows)][C]): the bias gradient of the layer whose
+// output gradient dx is.
 void layernorm_bwd8_pass(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
                          void* dx, int64_t rows, int C, bool acc, float* p_gamma, float* p_beta, cudaStream_t st,
-                         const void* addend = nullptr);
+                         const void* addend = nullptr, float* p_dx = nullptr);
+
 
 // ---- MobileNetV3 bottleneck (k_mobile.cu) ----
 // Depthwise k x k convolution, NHWC, weights [C][k][k] in the activation

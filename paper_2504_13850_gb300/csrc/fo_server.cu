@@ -7,6 +7,8 @@
 // (fo_sched.hpp); a slot's bytes live in the slab until the step that
 // consumes it has finished reading them (CUDA events order the reuse).
 #include "fo_server_impl.h"
+
+#include <memory>
 #include "fo_tc.h"
 
 #include <cstring>
@@ -49,7 +51,7 @@ int64_t pad64(int64_t n) { return (n + 63) / 64 * 64; }
 constexpr int64_t kEarlyUpdateMin = 128 * 1024;
 // Early updates are batched: consecutive weight tensors share one launch once
 // they add up to this many parameters (or the segment table is full).
-constexpr int64_t kEarlyGroupMin = 1024 * 1024;
+constexpr int64_t kEarlyGroupMin = 2 * 1024 * 1024;
 
 // Shape inference and parameter layout.  Returns FO_OK or an error.
 int infer(fo_server* s) {
@@ -547,11 +549,28 @@ int build_plan(fo_server* s) {
   // epilogue takes it as an addend; any other contributor, and any kernel
   // that reads the gradient, first has it copied in.
   std::vector<int> pending(nops + 1, -1);
+  // Bias gradients from the kernel that writes the output gradient last: a
+  // layernorm backward adds up the columns of what it stores as it goes
+  // (partial sums per row block), which saves the bias pass a read of the
+  // whole gradient.  Per gradient buffer (a fused residual's
+  // branch shares the add output's), the request slot of its last writer,
+  // or null when that writer cannot.
+  struct PartReq {
+    float* buf = nullptr;
+    int chunks = 0;
+  };
+  std::vector<int> galias(nops + 1, -1);
+  for (int i = 0; i < nops; ++i)
+    if (fu.branch_of[i] >= 0) galias[fu.branch_of[i]] = i + 1;
+  auto groot = [&](int tid) { return galias[tid] >= 0 ? s->T[galias[tid]].root : s->T[tid].root; };
+  std::vector<std::shared_ptr<PartReq>> last_part(nops + 1);
   auto materialize = [&](int tid) {
     const int r = s->T[tid].root;
     if (pending[r] < 0) return;
     const int src = pending[r];
     pending[r] = -1;
+    last_part[r] = nullptr;
+    last_part[groot(tid)] = nullptr;
     const int64_t n = s->T[r].numel();
     add("add_bwd", 1, 0.0, 2 * tbytes(r), [=](cudaStream_t st) {
       fo::grad_split(s->T[src].grad, nullptr, s->T[r].grad, false, nullptr, false, n, dt, st);
@@ -562,6 +581,7 @@ int build_plan(fo_server* s) {
     int r = s->T[tid].root;
     int accf = written[r] ? 1 : 0;
     written[r] = 1;
+    last_part[groot(tid)] = nullptr;   // callers that store partials set their request after this
     return accf;
   };
   // A contribution whose kernel adds `*addend` (a pending gradient) itself.
@@ -571,6 +591,7 @@ int build_plan(fo_server* s) {
     if (pending[r] >= 0) {
       *addend = s->T[pending[r]].grad;
       pending[r] = -1;
+      last_part[groot(tid)] = nullptr;
       return 0;
     }
     return contrib(tid);
@@ -648,7 +669,14 @@ int build_plan(fo_server* s) {
         const int dto = s->T[o].dt, dta = s->T[a].dt;
         const bool bias = op.bias != 0;
         const double fl = 2.0 * double(s->T[o].rows()) * op.cout * double(op.kind == FO_OP_CONV ? op.k * op.k : 1) * op.cin;
-        if (bias && dto == fo::kBF16 && s->T[o].C % 8 == 0) {
+        const std::shared_ptr<PartReq> lw = last_part[groot(o)];
+        if (bias && lw && !lw->buf) {
+          // the writer of this output gradient stores its column partials
+          const Tensor& t = s->T[o];
+          lw->buf = (float*)s->alloc(size_t(lw->chunks) * t.C * 4);
+          if (!lw->buf) return set_err(FO_ERR_OOM, "bias-gradient partials");
+          finish_tasks.push_back({lw->buf, G(s, i, 1), lw->chunks, t.C});
+        } else if (bias && dto == fo::kBF16 && s->T[o].C % 8 == 0) {
           const Tensor& t = s->T[o];
           const int chunks = fo::colsum8_batch_chunks(t.rows());
           float* part = (float*)s->alloc(size_t(chunks) * t.C * 4);
@@ -852,6 +880,9 @@ int build_plan(fo_server* s) {
         if (fo::layernorm_bwd8_ok(dt, s->T[a0].C)) {
           const void* addend = nullptr;
           const int accf = need_dx ? contrib_addend(a, &addend) : 0;
+          auto req = std::make_shared<PartReq>();
+          req->chunks = fo::layernorm_bwd8_blocks(s->T[a0].rows());
+          if (need_dx) last_part[groot(a)] = req;
           const Tensor& x0 = s->T[a0];
           const int blocks = fo::layernorm_bwd8_blocks(x0.rows());
           float* pg = (float*)s->alloc(size_t(2) * blocks * x0.C * 4);
@@ -862,7 +893,8 @@ int build_plan(fo_server* s) {
           add("layernorm_bwd", 1, 0.0, (need_dx ? 3 + accf + (addend ? 1 : 0) : 2) * csb, [=](cudaStream_t st) {
             const Tensor& x = s->T[a0];
             fo::layernorm_bwd8_pass(act(a0), P(s, i, 0), s->ln_mean[i], s->ln_rstd[i], s->T[o].grad,
-                                    need_dx ? s->T[a].grad : nullptr, x.rows(), x.C, accf != 0, pg, pb, st, addend);
+                                    need_dx ? s->T[a].grad : nullptr, x.rows(), x.C, accf != 0, pg, pb, st, addend,
+                                    req->buf);
           });
           break;
         }

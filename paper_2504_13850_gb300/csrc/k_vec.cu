@@ -391,12 +391,14 @@ __global__ void __launch_bounds__(256, 4) layernorm_bwd_fused_k(const bf16* __re
                                                                 const float* __restrict__ mean, const float* __restrict__ rstd,
                                                                 const bf16* __restrict__ dy, bf16* __restrict__ dx,
                                                                 int64_t rows, int C, int acc, float* __restrict__ pg,
-                                                                float* __restrict__ pb, const bf16* __restrict__ addend) {
+                                                                float* __restrict__ pb, const bf16* __restrict__ addend,
+                                                                float* __restrict__ pdx) {
   pdl_wait();
   pdl_trigger();
   constexpr int kMaxV = 2;  // up to 2 x 8 x 32 = 512 columns per row
   __shared__ __align__(16) float redg[8][512];
   __shared__ __align__(16) float redb[8][512];
+  __shared__ __align__(16) float redx[8][512];   // pdx: the written dx, for its column partials
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int nv = C / 256;  // 8-wide vectors per lane
   const int64_t row = int64_t(blockIdx.x) * 8 + warp;
@@ -448,7 +450,7 @@ __global__ void __launch_bounds__(256, 4) layernorm_bwd_fused_k(const bf16* __re
   }
   a /= float(C);
   b /= float(C);
-  if (live && dx) {
+  if (dx) {
 #pragma unroll
     for (int v = 0; v < kMaxV; ++v) {
       if (v >= nv) break;
@@ -461,7 +463,15 @@ __global__ void __launch_bounds__(256, 4) layernorm_bwd_fused_k(const bf16* __re
         const float xh = (bf_at(xr[v], j) - mu) * rs;
         o.v[j] = rs * (bf_at(gr[v], j) * gm[j] - a - xh * b) + bf_at(orr[v], j) + bf_at(ar[v], j);
       }
-      st8(dx + row * C + c, o);
+      if (live) st8(dx + row * C + c, o);
+      if (pdx) {   // the stored (bf16-rounded) values, zeros past the end
+        float4* rx = reinterpret_cast<float4*>(&redx[warp][c]);
+        float q[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) q[j] = live ? __bfloat162float(__float2bfloat16_rn(o.v[j])) : 0.f;
+        rx[0] = make_float4(q[0], q[1], q[2], q[3]);
+        rx[1] = make_float4(q[4], q[5], q[6], q[7]);
+      }
     }
   }
   __syncthreads();
@@ -474,6 +484,12 @@ __global__ void __launch_bounds__(256, 4) layernorm_bwd_fused_k(const bf16* __re
     }
     pg[int64_t(blockIdx.x) * C + c] = tg;
     pb[int64_t(blockIdx.x) * C + c] = tb;
+    if (pdx) {
+      float tx = 0.f;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) tx += redx[q][c];
+      pdx[int64_t(blockIdx.x) * C + c] = tx;
+    }
   }
 }
 
@@ -742,9 +758,9 @@ void layernorm_fwd_x8(const void* x, const float* gamma, const float* beta, void
 
 void layernorm_bwd8_pass(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
                          void* dx, int64_t rows, int C, bool acc, float* p_gamma, float* p_beta, cudaStream_t st,
-                         const void* addend) {
+                         const void* addend, float* p_dx) {
   launch_k(layernorm_bwd_fused_k, layernorm_bwd8_blocks(rows), 256, 0, st, (const bf16*)x, gamma, mean, rstd,
-           (const bf16*)dy, (bf16*)dx, rows, C, acc ? 1 : 0, p_gamma, p_beta, (const bf16*)addend);
+           (const bf16*)dy, (bf16*)dx, rows, C, acc ? 1 : 0, p_gamma, p_beta, (const bf16*)addend, p_dx);
 }
 
 int64_t layernorm_bwd8_partial_floats(int64_t rows, int C) { return 2 * ((rows + 7) / 8) * C; }
