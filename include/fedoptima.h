@@ -159,7 +159,9 @@ FO_API int fo_server_get_momentum(fo_server* s, float* host, int64_t n);
  *   tensor `index` -- 1..n_ops is the output of op index-1 -- as written by
  *   the last fo_server_step.  The pointer stays valid for the server's
  *   lifetime; the contents change with each step, which runs on
- *   fo_server_stream.  FO_ERR_ARG for an index outside 1..n_ops.
+ *   fo_server_stream.  A flatten of the uploaded batch is a view of it: its
+ *   pointer is the batch slot the last step read.  FO_ERR_ARG for an index
+ *   outside 1..n_ops.
  * fo_server_params_device: the fp32 master parameters on the device in the
  *   server's padded layout (*n floats; identical for servers built from the
  *   same op list), for device-to-device aggregation.  Read it only when the

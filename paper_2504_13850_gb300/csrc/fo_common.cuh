@@ -36,6 +36,25 @@ int elementwise_blocks(int64_t n_threads_needed, int threads);
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
+// Standard normal distribution function Phi(x) and density phi(x) for the
+// GELU, from one exponential and one reciprocal: Abramowitz & Stegun 26.2.17
+// (Hastings' rational approximation), for x >= 0
+//   1 - Phi(x) = phi(x) (b1 t + b2 t^2 + b3 t^3 + b4 t^4 + b5 t^5),
+//   t = 1 / (1 + p x),  p = 0.2316419,
+// with an absolute error below 7.5e-8; Phi(-x) = 1 - Phi(x) gives x < 0
+// without the cancellation of 1 + erf.  The density's exponential is the
+// same one, so the GELU backward gets phi(x) with no further work.
+__device__ __forceinline__ void normal_cdf_pdf(float x, float& cdf, float& pdf) {
+  float e;   // exp(-x^2 / 2) = 2^(-x^2 log2(e) / 2)
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(e) : "f"(x * x * -0.72134752044448170f));
+  pdf = 0.39894228040143268f * e;
+  const float t = __fdividef(1.f, fmaf(0.2316419f, fabsf(x), 1.f));
+  const float poly =
+      t * fmaf(t, fmaf(t, fmaf(t, fmaf(t, 1.330274429f, -1.821255978f), 1.781477937f), -0.356563782f), 0.319381530f);
+  const float q = pdf * poly;   // 1 - Phi(|x|)
+  cdf = x >= 0.f ? 1.f - q : q;
+}
+
 // False when FO_NO_PDL is set (plain stream order, for comparison).
 bool pdl_enabled();
 

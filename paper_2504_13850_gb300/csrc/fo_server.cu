@@ -251,7 +251,7 @@ Fusion analyse(const fo_server* s) {
   f.head = last.kind == FO_OP_LINEAR && s->cfg.num_classes <= 1024;
   for (int r = 0; r < nops; ++r) {
     const fo_op& op = s->ops[r];
-    if (op.kind != FO_OP_RELU || op.in0 == 0) continue;
+    if (op.kind != FO_OP_RELU || s->T[op.in0].is_input()) continue;
     const int p = op.in0 - 1;  // producer op of the relu input
     const int pk = s->ops[p].kind;
     if (sole[op.in0] == r && (pk == FO_OP_CONV || pk == FO_OP_LINEAR || pk == FO_OP_AFFINE || pk == FO_OP_ADD) &&
@@ -270,7 +270,7 @@ Fusion analyse(const fo_server* s) {
   // masks the relu output's gradient on the fly and writes both inputs.
   for (int r = 0; r < nops; ++r) {
     const fo_op& op = s->ops[r];
-    if (op.kind != FO_OP_RELU || op.in0 == 0 || f.skip_bwd[r]) continue;
+    if (op.kind != FO_OP_RELU || s->T[op.in0].is_input() || f.skip_bwd[r]) continue;
     const int p = op.in0 - 1;
     if (s->ops[p].kind == FO_OP_ADD && sole[op.in0] == r) {
       f.add_relu[p] = r;
@@ -281,7 +281,7 @@ Fusion analyse(const fo_server* s) {
   // bottleneck) applies it in both passes, on the vectorised bf16 path.
   for (int h = 0; h < nops; ++h) {
     const fo_op& op = s->ops[h];
-    if (op.kind != FO_OP_HSWISH || op.in0 == 0) continue;
+    if (op.kind != FO_OP_HSWISH || s->T[op.in0].is_input()) continue;
     const int p = op.in0 - 1;
     const Tensor& t = s->T[op.in0];
     if (s->ops[p].kind == FO_OP_AFFINE && sole[op.in0] == h && f.fwd_relu[p] < 0 && fo::vec8_ok(s->dt, t.numel()) &&
@@ -298,7 +298,7 @@ Fusion analyse(const fo_server* s) {
     if (op.kind != FO_OP_ADD || f.fwd_relu[a] >= 0 || f.add_relu[a] >= 0) continue;
     for (int t : {op.in1, op.in0}) {
       const int other = t == op.in1 ? op.in0 : op.in1;
-      if (t == 0 || s->T[t].root != t || s->T[t].root == s->T[other].root || sole[t] != a) continue;
+      if (s->T[t].is_input() || s->T[t].root != t || s->T[t].root == s->T[other].root || sole[t] != a) continue;
       const int p = t - 1;
       if (!plain(p) || f.fwd_relu[p] >= 0) continue;
       f.add_into[p] = a;
@@ -328,7 +328,7 @@ int build_plan(fo_server* s) {
   const Fusion fu = analyse(s);
   for (int i = 0; i < nops; ++i)   // a fused residual's branch shares the add's output gradient
     if (fu.branch_of[i] >= 0) s->T[fu.branch_of[i]].grad = s->T[i + 1].grad;
-  auto act = [s](int tid) -> const void* { return tid == 0 ? s->cur_in : s->T[tid].act; };
+  auto act = [s](int tid) -> const void* { return s->T[tid].is_input() ? s->cur_in : s->T[tid].act; };
   auto add = [&plan](const char* name, int kernels, double flops, double bytes,
                      std::function<void(cudaStream_t)> fn, int lane = 0) {
     plan.push_back({name, std::move(fn), kernels, flops, bytes, lane});
@@ -364,7 +364,7 @@ int build_plan(fo_server* s) {
       const int mr = fu.bwd_mask[i];
       const int da = mr >= 0 ? s->ops[mr].in0 : a;
       const void* mask = mr >= 0 ? s->T[mr + 1].act : nullptr;
-      const bool dx = a != 0;
+      const bool dx = !s->T[a].is_input();
       add("head_fwd_ce", 1, 2.0 * B * K * C * (dx ? 2.0 : 1.0), tbytes(a) * (dx ? 3.0 : 1.0), [=](cudaStream_t st) {
         fo::head_forward_loss(act(a), s->T[a].dt, P(s, i, 0), op.bias ? P(s, i, 1) : nullptr, s->cur_labels, B,
                               K, C, (float*)s->T[i + 1].act, (float*)s->T[i + 1].grad, s->row_loss, st, mask,
@@ -382,7 +382,7 @@ int build_plan(fo_server* s) {
         const bool fused = fu.add_into[i] >= 0;
         if (fused) {
           const int r = fu.add_other[fu.add_into[i]];
-          if (r == 0) ex.addend_is_input = true;
+          if (s->T[r].is_input()) ex.addend_is_input = true;
           else ex.addend = s->T[r].act;
         }
         fo::TcGemm* tg = nullptr;
@@ -477,7 +477,7 @@ int build_plan(fo_server* s) {
       case FO_OP_ATTENTION: {
         const double Ls = ta.H, heads = op.heads, dh = double(op.cin) / op.heads;
         fo::AttnTcPlan* tp = nullptr;
-        if (s->tc && dt == fo::kBF16 && a != 0 && !getenv("FO_NO_TC") && fo::attention_tc_ok(ta.H, op.cin, op.heads))
+        if (s->tc && dt == fo::kBF16 && !s->T[a].is_input() && !getenv("FO_NO_TC") && fo::attention_tc_ok(ta.H, op.cin, op.heads))
           tp = fo::attention_tc_plan(s->T[a].act, s->T[o].act, s->T[o].grad, ta.N, ta.H, op.cin, op.heads,
                                      fo::tc_error_word(s->tc));
         s->attn_tc[i] = tp;
@@ -649,7 +649,7 @@ int build_plan(fo_server* s) {
     const int mr = fu.bwd_mask[i];
     const int a = mr >= 0 ? s->ops[mr].in0 : a0;            // gradient destination
     const void* mask = mr >= 0 ? s->T[mr + 1].act : nullptr;
-    const bool need_dx = a0 != 0;
+    const bool need_dx = !s->T[a0].is_input();
     const double csb = double(s->T[o].rows()) * s->T[o].C * esz;  // one read of dy
     if (fu.head && i == L) {
       const int B = s->cfg.batch, K = op.cin, C = op.cout;
@@ -820,7 +820,7 @@ int build_plan(fo_server* s) {
           // residual's is left pending for its next contributor
           written[s->T[fu.branch_of[i]].root] = 1;
           const int x = fu.add_other[i];
-          if (x == 0) break;
+          if (s->T[x].is_input()) break;
           const int rx = s->T[x].root;
           if (!written[rx]) {
             pending[rx] = o;
@@ -842,7 +842,7 @@ int build_plan(fo_server* s) {
         const void* msk = rr >= 0 ? s->T[rr + 1].act : nullptr;
         int srcs[2], accs[2], ns = 0;
         for (int src : {a0, b}) {
-          if (src == 0) continue;
+          if (s->T[src].is_input()) continue;
           srcs[ns] = src;
           accs[ns] = contrib(src);
           ++ns;
@@ -1402,7 +1402,7 @@ int fo_server_tensor(const fo_server* s, int index, const void** data, int64_t* 
   if (!s || !data || !dims4 || !dtype) return set_err(FO_ERR_ARG, "null argument");
   if (index < 1 || index > int(s->ops.size())) return set_err(FO_ERR_ARG, "tensor index outside 1..n_ops");
   const Tensor& t = s->T[index];
-  *data = t.act;
+  *data = t.is_input() ? s->cur_in : t.act;
   dims4[0] = t.N;
   dims4[1] = t.H;
   dims4[2] = t.W;

@@ -33,6 +33,9 @@ struct Tensor {
   int64_t rows() const { return int64_t(N) * H * W; }
   int64_t numel() const { return rows() * C; }
   size_t bytes() const { return size_t(numel()) * (dt == fo::kF32 ? 4 : 2); }
+  // The uploaded batch (tensor 0) or a view of it (a flatten of the input):
+  // its data is the current batch slot, and it has no gradient.
+  bool is_input() const { return root == 0; }
 };
 
 struct Launch {

@@ -388,14 +388,15 @@ void avgpool_bwd(const void* dy, void* dx, int N, int HW, int C, int dt, bool ac
 }
 
 // ----------------------------------------------------------------- gelu
-__device__ __forceinline__ float gelu_cdf(float x) { return 0.5f * (1.f + erff(x * 0.70710678118654752f)); }
 template <typename T>
 __global__ void gelu_fwd_k(const T* x, T* y, int64_t n) {
   pdl_wait();
   pdl_trigger();
   GRID_STRIDE(i, n) {
-    float v = to_f(x[i]);
-    y[i] = from_f<T>(v * gelu_cdf(v));
+    const float v = to_f(x[i]);
+    float cdf, pdf;
+    normal_cdf_pdf(v, cdf, pdf);
+    y[i] = from_f<T>(v * cdf);
   }
 }
 template <typename T>
@@ -403,9 +404,10 @@ __global__ void gelu_bwd_k(const T* x, const T* dy, T* dx, int64_t n, int acc) {
   pdl_wait();
   pdl_trigger();
   GRID_STRIDE(i, n) {
-    float v = to_f(x[i]);
-    float pdf = 0.39894228040143268f * expf(-0.5f * v * v);
-    store(dx, i, to_f(dy[i]) * (gelu_cdf(v) + v * pdf), acc);
+    const float v = to_f(x[i]);
+    float cdf, pdf;
+    normal_cdf_pdf(v, cdf, pdf);
+    store(dx, i, to_f(dy[i]) * (cdf + v * pdf), acc);
   }
 }
 void gelu_fwd(const void* x, void* y, int64_t n, int dt, cudaStream_t st) {

@@ -133,7 +133,7 @@ struct TcGemm {
   size_t smem = 0;
   dim3 grid;
   int lane = 0;           // stream lane (split-K workspace per lane)
-  bool input_A = false;   // operand fed by the uploaded batch (tensor 0)
+  bool input_A = false;   // operand fed by the uploaded batch (tensor 0 or a view of it)
   bool input_B = false;
   bool input_acc = false; // the epilogue's addend is the uploaded batch
   std::vector<CUtensorMap> slot_maps;  // per slot map of that operand
@@ -406,7 +406,7 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i, void* out, bool relu,
     int M = int(a.rows()), KB = (op.cin + 63) / 64;
     choose_tiles(c, g, M, op.cout, KB, op.cout);
     const int bn = g->bn;
-    g->input_A = (op.in0 == 0);
+    g->input_A = s->T[op.in0].is_input();
     if (g->input_A) {
       g->slot_maps.resize(s->cfg.omega);
       for (int sl = 0; sl < s->cfg.omega; ++sl)
@@ -430,7 +430,7 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i, void* out, bool relu,
   choose_tiles(c, g, M, op.cout, KB, op.cout);
   const int bn = g->bn;
   const int box_rows = rows, box_imgs = imgs;
-  g->input_A = (op.in0 == 0);
+  g->input_A = s->T[op.in0].is_input();
   if (g->input_A) {
     g->slot_maps.resize(s->cfg.omega);
     for (int sl = 0; sl < s->cfg.omega; ++sl)
@@ -556,7 +556,7 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
     g->p.ldo = op.cin;
     int rows = int(a.rows()), KB = (rows + BK - 1) / BK;
     choose_tiles(c, g, op.cout, op.cin, KB, op.cin);
-    g->input_B = (op.in0 == 0);
+    g->input_B = s->T[op.in0].is_input();
     if (!map_2d(&g->p.tmA, o.grad, rows, op.cout, BK)) { delete g; return nullptr; }
     CUtensorMap ca;
     if (map_chunked(&ca, o.grad, rows, op.cout, BK, BM / 64)) { g->p.tmA = ca; g->p.chunk_a = 1; }
@@ -590,7 +590,7 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
   int P = a.N * Ho * Wo, KB = P / BK;
   int N = g->p.taps * op.cin;
   choose_tiles(c, g, op.cout, N, KB, op.cin);
-  g->input_B = (op.in0 == 0);
+  g->input_B = s->T[op.in0].is_input();
   if (!map_2d(&g->p.tmA, o.grad, P, op.cout, BK)) { delete g; return nullptr; }
   CUtensorMap ca;
   if (map_chunked(&ca, o.grad, P, op.cout, BK, BM / 64)) { g->p.tmA = ca; g->p.chunk_a = 1; }

@@ -150,8 +150,6 @@ __global__ void affine_hswish_fwd_x8_k(const bf16* __restrict__ x, const float* 
   }
 }
 
-__device__ __forceinline__ float gelu_cdf(float x) { return 0.5f * (1.f + erff(x * 0.70710678118654752f)); }
-
 __global__ void gelu_fwd_x8_k(const bf16* __restrict__ x, bf16* __restrict__ y, int64_t n8) {
   pdl_wait();
   pdl_trigger();
@@ -159,7 +157,11 @@ __global__ void gelu_fwd_x8_k(const bf16* __restrict__ x, bf16* __restrict__ y, 
     const V8 p = ld8(x + 8 * i);
     V8 o;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) o.v[j] = p.v[j] * gelu_cdf(p.v[j]);
+    for (int j = 0; j < 8; ++j) {
+      float cdf, pdf;
+      normal_cdf_pdf(p.v[j], cdf, pdf);
+      o.v[j] = p.v[j] * cdf;
+    }
     st8(y + 8 * i, o);
   }
 }
@@ -173,9 +175,9 @@ __global__ void gelu_bwd_x8_k(const bf16* __restrict__ x, const bf16* __restrict
     V8 o;
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      const float v = p.v[j];
-      const float pdf = 0.39894228040143268f * __expf(-0.5f * v * v);   // result stored as bf16
-      o.v[j] = g.v[j] * (gelu_cdf(v) + v * pdf);
+      float cdf, pdf;
+      normal_cdf_pdf(p.v[j], cdf, pdf);
+      o.v[j] = g.v[j] * (cdf + p.v[j] * pdf);
     }
     if (acc) {
       const V8 q = ld8(dx + 8 * i);
@@ -370,126 +372,132 @@ __global__ void __launch_bounds__(256, NV <= 2 ? 4 : 2) layernorm_fwd_x8_k(const
   }
 }
 
-// Layernorm backward fused with its parameter gradients: one warp per row
-// (8 rows per block).  The row's x, dy, addend and old dx are all loaded
-// before any arithmetic and kept as packed bf16 (so that four blocks fit on
-// an SM and the whole grid is resident at once); the block's column partials
-// of dy * xhat (gamma) and dy (beta) are added in warp order.  C <= 512,
-// C % 256 == 0; dx may be null (a layernorm of the uploaded batch has no
-// input gradient).  dx receives the layernorm's input gradient, plus its old
-// value when `acc`, plus `addend` (same layout) when given: the gradient a
-// residual connection passes around the layernorm.
+// Layernorm backward fused with its parameter gradients.  Each warp takes
+// kLnRows consecutive rows (a block 8 kLnRows), with all of their operands
+// loaded before any arithmetic.  The column partials of dy * xhat (gamma),
+// dy (beta) and, with pdx, of the stored dx accumulate in registers over the
+// warp's rows and are added over the block's 8 warps, in warp order, through
+// shared memory once per block: exchanged row by row, those partials cost
+// more than the rest of the pass.  C <= 512, C % 256 == 0; dx may be null (a
+// layernorm of the uploaded batch has no input gradient).  dx receives the
+// layernorm's input gradient plus the NX extra operands ex0, ex1 (same
+// layout): its own old value when accumulating, and the gradient a residual
+// connection passes around the layernorm.
+constexpr int kLnRows = 4;
 __device__ __forceinline__ float bf_at(const uint4& u, int j) {
   return __bfloat162float(reinterpret_cast<const bf16*>(&u)[j]);
 }
-__device__ __forceinline__ void gamma8(const float* gamma, int c, float (&g)[8]) {
-  const float4 a = __ldg(reinterpret_cast<const float4*>(gamma + c));
-  const float4 b = __ldg(reinterpret_cast<const float4*>(gamma + c) + 1);
-  g[0] = a.x; g[1] = a.y; g[2] = a.z; g[3] = a.w; g[4] = b.x; g[5] = b.y; g[6] = b.z; g[7] = b.w;
-}
-__global__ void __launch_bounds__(256, 4) layernorm_bwd_fused_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
+template <int NX, int NV>
+__global__ void __launch_bounds__(256, 1) layernorm_bwd_fused_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
                                                                 const float* __restrict__ mean, const float* __restrict__ rstd,
-                                                                const bf16* __restrict__ dy, bf16* __restrict__ dx,
-                                                                int64_t rows, int C, int acc, float* __restrict__ pg,
-                                                                float* __restrict__ pb, const bf16* __restrict__ addend,
-                                                                float* __restrict__ pdx) {
+                                                                const bf16* __restrict__ dy, bf16* dx, int64_t rows, int C,
+                                                                const bf16* ex0, const bf16* ex1, float* __restrict__ pg,
+                                                                float* __restrict__ pb, float* __restrict__ pdx) {
   pdl_wait();
   pdl_trigger();
-  constexpr int kMaxV = 2;  // up to 2 x 8 x 32 = 512 columns per row
-  __shared__ __align__(16) float redg[8][512];
-  __shared__ __align__(16) float redb[8][512];
-  __shared__ __align__(16) float redx[8][512];   // pdx: the written dx, for its column partials
+  constexpr int kMaxV = NV, nv = NV;   // 8-wide vectors per lane: C = 256 NV
+  __shared__ __align__(16) float red[3][8][256 * NV];
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int nv = C / 256;  // 8-wide vectors per lane
-  const int64_t row = int64_t(blockIdx.x) * 8 + warp;
-  const bool live = row < rows;
+  const int64_t row0 = (int64_t(blockIdx.x) * 8 + warp) * kLnRows;
   const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-  uint4 xr[kMaxV] = {z, z}, gr[kMaxV] = {z, z}, ar[kMaxV] = {z, z}, orr[kMaxV] = {z, z};
-  if (live) {
+  float gm[kMaxV][8];
+#pragma unroll
+  for (int v = 0; v < kMaxV; ++v) {
+    const int c = v < nv ? (v * 32 + lane) * 8 : 0;
+    const float4 g0 = __ldg(reinterpret_cast<const float4*>(gamma + c));
+    const float4 g1 = __ldg(reinterpret_cast<const float4*>(gamma + c) + 1);
+    gm[v][0] = g0.x; gm[v][1] = g0.y; gm[v][2] = g0.z; gm[v][3] = g0.w;
+    gm[v][4] = g1.x; gm[v][5] = g1.y; gm[v][6] = g1.z; gm[v][7] = g1.w;
+  }
+  uint4 xr[kLnRows][kMaxV], gr[kLnRows][kMaxV], er[kLnRows][kMaxV][NX > 0 ? NX : 1];
+  float mu[kLnRows], rs[kLnRows];
+#pragma unroll
+  for (int r = 0; r < kLnRows; ++r) {
+    const int64_t row = row0 + r;
+    const bool live = row < rows;
 #pragma unroll
     for (int v = 0; v < kMaxV; ++v) {
-      if (v >= nv) break;
+      const bool ok = live && v < nv;
       const int64_t off = row * C + (v * 32 + lane) * 8;
-      xr[v] = *reinterpret_cast<const uint4*>(x + off);
-      gr[v] = *reinterpret_cast<const uint4*>(dy + off);
-      if (dx && addend) ar[v] = *reinterpret_cast<const uint4*>(addend + off);
-      if (dx && acc) orr[v] = *reinterpret_cast<const uint4*>(dx + off);
+      xr[r][v] = ok ? *reinterpret_cast<const uint4*>(x + off) : z;
+      gr[r][v] = ok ? *reinterpret_cast<const uint4*>(dy + off) : z;
+      if constexpr (NX > 0) er[r][v][0] = ok ? *reinterpret_cast<const uint4*>(ex0 + off) : z;
+      if constexpr (NX > 1) er[r][v][1] = ok ? *reinterpret_cast<const uint4*>(ex1 + off) : z;
+    }
+    mu[r] = live ? mean[row] : 0.f;
+    rs[r] = live ? rstd[row] : 0.f;
+  }
+  float ag[kMaxV][8] = {}, ab[kMaxV][8] = {}, ax[kMaxV][8] = {};
+#pragma unroll
+  for (int r = 0; r < kLnRows; ++r) {
+    const int64_t row = row0 + r;
+    const bool live = row < rows;
+    float a = 0.f, b = 0.f;
+#pragma unroll
+    for (int v = 0; v < kMaxV; ++v)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {   // rows past the end and vectors past C hold zeros
+        const float xh = (bf_at(xr[r][v], j) - mu[r]) * rs[r];
+        const float g = bf_at(gr[r][v], j);
+        const float d = g * gm[v][j];
+        a += d;
+        b += d * xh;
+        ag[v][j] += g * xh;
+        ab[v][j] += g;
+      }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      a += __shfl_xor_sync(0xffffffffu, a, o);
+      b += __shfl_xor_sync(0xffffffffu, b, o);
+    }
+    a /= float(C);
+    b /= float(C);
+    if (dx) {
+#pragma unroll
+      for (int v = 0; v < kMaxV; ++v) {
+        if (v >= nv) break;
+        V8 o;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float xh = (bf_at(xr[r][v], j) - mu[r]) * rs[r];
+          float val = rs[r] * (bf_at(gr[r][v], j) * gm[v][j] - a - xh * b);
+          if constexpr (NX > 0) val += bf_at(er[r][v][0], j);
+          if constexpr (NX > 1) val += bf_at(er[r][v][1], j);
+          o.v[j] = val;
+          ax[v][j] += live ? __bfloat162float(__float2bfloat16_rn(val)) : 0.f;   // the stored value
+        }
+        if (live) st8(dx + row * C + (v * 32 + lane) * 8, o);
+      }
     }
   }
-  const float mu = live ? mean[row] : 0.f, rs = live ? rstd[row] : 0.f;
-  float a = 0.f, b = 0.f;
 #pragma unroll
   for (int v = 0; v < kMaxV; ++v) {
     if (v >= nv) break;
     const int c = (v * 32 + lane) * 8;
-    float gm[8];
-    gamma8(gamma, c, gm);
-    float pgv[8], pbv[8];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const float xh = (bf_at(xr[v], j) - mu) * rs;
-      const float g = bf_at(gr[v], j);
-      const float dxh = g * gm[j];
-      a += dxh;
-      b += dxh * xh;
-      pgv[j] = g * xh;
-      pbv[j] = g;
-    }
-    // this row's contributions to the column partials (zeros past the end)
-    float4* rg = reinterpret_cast<float4*>(&redg[warp][c]);
-    float4* rb = reinterpret_cast<float4*>(&redb[warp][c]);
-    rg[0] = make_float4(pgv[0], pgv[1], pgv[2], pgv[3]);
-    rg[1] = make_float4(pgv[4], pgv[5], pgv[6], pgv[7]);
-    rb[0] = make_float4(pbv[0], pbv[1], pbv[2], pbv[3]);
-    rb[1] = make_float4(pbv[4], pbv[5], pbv[6], pbv[7]);
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    a += __shfl_xor_sync(0xffffffffu, a, o);
-    b += __shfl_xor_sync(0xffffffffu, b, o);
-  }
-  a /= float(C);
-  b /= float(C);
-  if (dx) {
-#pragma unroll
-    for (int v = 0; v < kMaxV; ++v) {
-      if (v >= nv) break;
-      const int c = (v * 32 + lane) * 8;
-      float gm[8];
-      gamma8(gamma, c, gm);
-      V8 o;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const float xh = (bf_at(xr[v], j) - mu) * rs;
-        o.v[j] = rs * (bf_at(gr[v], j) * gm[j] - a - xh * b) + bf_at(orr[v], j) + bf_at(ar[v], j);
-      }
-      if (live) st8(dx + row * C + c, o);
-      if (pdx) {   // the stored (bf16-rounded) values, zeros past the end
-        float4* rx = reinterpret_cast<float4*>(&redx[warp][c]);
-        float q[8];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) q[j] = live ? __bfloat162float(__float2bfloat16_rn(o.v[j])) : 0.f;
-        rx[0] = make_float4(q[0], q[1], q[2], q[3]);
-        rx[1] = make_float4(q[4], q[5], q[6], q[7]);
-      }
+    float4* p0 = reinterpret_cast<float4*>(&red[0][warp][c]);
+    float4* p1 = reinterpret_cast<float4*>(&red[1][warp][c]);
+    float4* p2 = reinterpret_cast<float4*>(&red[2][warp][c]);
+    p0[0] = make_float4(ag[v][0], ag[v][1], ag[v][2], ag[v][3]);
+    p0[1] = make_float4(ag[v][4], ag[v][5], ag[v][6], ag[v][7]);
+    p1[0] = make_float4(ab[v][0], ab[v][1], ab[v][2], ab[v][3]);
+    p1[1] = make_float4(ab[v][4], ab[v][5], ab[v][6], ab[v][7]);
+    if (pdx) {
+      p2[0] = make_float4(ax[v][0], ax[v][1], ax[v][2], ax[v][3]);
+      p2[1] = make_float4(ax[v][4], ax[v][5], ax[v][6], ax[v][7]);
     }
   }
   __syncthreads();
   for (int c = threadIdx.x; c < C; c += blockDim.x) {
-    float tg = 0.f, tb = 0.f;
+    float tg = 0.f, tb = 0.f, tx = 0.f;
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
-      tg += redg[q][c];
-      tb += redb[q][c];
+      tg += red[0][q][c];
+      tb += red[1][q][c];
+      if (pdx) tx += red[2][q][c];
     }
     pg[int64_t(blockIdx.x) * C + c] = tg;
     pb[int64_t(blockIdx.x) * C + c] = tb;
-    if (pdx) {
-      float tx = 0.f;
-#pragma unroll
-      for (int q = 0; q < 8; ++q) tx += redx[q][c];
-      pdx[int64_t(blockIdx.x) * C + c] = tx;
-    }
+    if (pdx) pdx[int64_t(blockIdx.x) * C + c] = tx;
   }
 }
 
@@ -746,7 +754,7 @@ void finish_batched(const std::vector<FinishTask>& tasks, cudaStream_t st) {
 
 bool layernorm_bwd8_ok(int dt, int C) { return dt == kBF16 && C % 256 == 0 && C <= 512; }
 
-int layernorm_bwd8_blocks(int64_t rows) { return int((rows + 7) / 8); }
+int layernorm_bwd8_blocks(int64_t rows) { return int((rows + 8 * kLnRows - 1) / (8 * kLnRows)); }
 
 bool layernorm_fwd8_ok(int dt, int C) { return dt == kBF16 && C % 256 == 0 && C <= 1024; }
 void layernorm_fwd_x8(const void* x, const float* gamma, const float* beta, void* y, float* mean, float* rstd,
@@ -759,11 +767,17 @@ void layernorm_fwd_x8(const void* x, const float* gamma, const float* beta, void
 void layernorm_bwd8_pass(const void* x, const float* gamma, const float* mean, const float* rstd, const void* dy,
                          void* dx, int64_t rows, int C, bool acc, float* p_gamma, float* p_beta, cudaStream_t st,
                          const void* addend, float* p_dx) {
-  launch_k(layernorm_bwd_fused_k, layernorm_bwd8_blocks(rows), 256, 0, st, (const bf16*)x, gamma, mean, rstd,
-           (const bf16*)dy, (bf16*)dx, rows, C, acc ? 1 : 0, p_gamma, p_beta, (const bf16*)addend, p_dx);
+  const bf16* ex[2] = {nullptr, nullptr};
+  int nx = 0;
+  if (dx && acc) ex[nx++] = static_cast<const bf16*>(dx);
+  if (dx && addend) ex[nx++] = static_cast<const bf16*>(addend);
+  auto k = C <= 256 ? (nx == 0 ? layernorm_bwd_fused_k<0, 1> : nx == 1 ? layernorm_bwd_fused_k<1, 1> : layernorm_bwd_fused_k<2, 1>)
+                    : (nx == 0 ? layernorm_bwd_fused_k<0, 2> : nx == 1 ? layernorm_bwd_fused_k<1, 2> : layernorm_bwd_fused_k<2, 2>);
+  launch_k(k, layernorm_bwd8_blocks(rows), 256, 0, st, (const bf16*)x, gamma, mean, rstd, (const bf16*)dy, (bf16*)dx,
+           rows, C, ex[0], ex[1], p_gamma, p_beta, dx ? p_dx : nullptr);
 }
 
-int64_t layernorm_bwd8_partial_floats(int64_t rows, int C) { return 2 * ((rows + 7) / 8) * C; }
+int64_t layernorm_bwd8_partial_floats(int64_t rows, int C) { return 2 * int64_t(layernorm_bwd8_blocks(rows)) * C; }
 
 bool meanpool8_ok(int dt, int C) { return dt == kBF16 && C % 8 == 0; }
 void meanpool_fwd_x8(const void* x, const int32_t* len, void* y, int B, int L, int C, cudaStream_t st) {

@@ -81,7 +81,7 @@ def param_slices(ops):
     return out
 
 
-def teacher_forced(cfg, events, max_steps=None, compare=None):
+def teacher_forced(cfg, events, max_steps=None, compare=None, theta0=None):
     """GPU and oracle in lockstep: before every step the oracle takes the
     GPU's theta and momentum, then both run the same scheduled batch.  Two
     oracle readings run side by side: the exact fp64 definition, and the
@@ -90,10 +90,11 @@ def teacher_forced(cfg, events, max_steps=None, compare=None):
     with the loss, parameter and per-tensor gradient errors against each
     (gradient recovered exactly as g = v_new - mu v_old).  With `compare` (a
     set of step indices) only those steps are compared; the others run on
-    the GPU alone while the oracles' schedulers follow them (long runs)."""
+    the GPU alone while the oracles' schedulers follow them (long runs).
+    `theta0` replaces the workload's initial parameters."""
     from paper_2504_13850_gb300 import api
     s = api.Server.from_config(cfg)
-    theta0 = W.init_params(cfg)
+    theta0 = W.init_params(cfg) if theta0 is None else theta0
     s.set_params(theta0)
     storage = "bf16" if cfg["dtype"] == W.BF16 else None
     mk = lambda st: O.Server(cfg["ops"], cfg["K"], cfg["omega"], cfg["depth"], theta0, cfg["lr"],

@@ -67,16 +67,16 @@ def prefill_then_steps(cfg, steps):
     return ev + [("step",)] * steps
 
 
-def compare(cfg, events, loss_tol, param_tol, upd_tol=None):
-    s, glog = replay_gpu(cfg, events)
-    o, olog = replay_oracle(cfg, events)
+def compare(cfg, events, loss_tol, param_tol, upd_tol=None, theta0=None):
+    s, glog = replay_gpu(cfg, events, theta0)
+    o, olog = replay_oracle(cfg, events, theta0)
     assert glog == olog                           # scheduler outcomes, slots: bit-exact
     nsteps = sum(1 for e in glog if e[0] == "step" and e[1] == api.OK)
     losses = s.read_losses(0, nsteps)
     ol = np.array(o.losses)
     assert np.all(np.abs(losses - ol) <= loss_tol * np.abs(ol)), (losses, ol)
     theta = s.get_params()
-    theta0 = W.init_params(cfg).astype(np.float64)
+    theta0 = (W.init_params(cfg) if theta0 is None else theta0).astype(np.float64)
     assert normwise(theta, o.theta) <= param_tol
     if upd_tol is not None:
         assert normwise(theta - theta0, o.theta - theta0) <= upd_tol
