@@ -20,7 +20,7 @@ namespace {
 // The epilogue variant a plan's parameters ask for.
 int epi_of(const TcParams& p) {
   return (p.out_f32 ? E_F32 : 0) | (p.relu ? E_RELU : 0) | (p.mask ? E_MASK : 0) | (p.acc ? E_ACC : 0) |
-         (p.pool_out ? E_POOL : 0);
+         (p.pool_out ? E_POOL : 0) | (p.tma_out ? E_TMA : 0);
 }
 
 KernelFn pick_kernel(int kind, int bn, bool cluster, int epi, size_t* smem) {
@@ -60,7 +60,8 @@ EncodeTiledFn encode_fn() {
 // elem (may be null): traversal step per dimension (the box then spans
 // box[i] elements and loads box[i] / elem[i] of them).
 bool make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, const uint64_t* strides,
-              const uint32_t* box, const uint32_t* elem = nullptr) {
+              const uint32_t* box, const uint32_t* elem = nullptr,
+              CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t d[5], st[4];
@@ -72,7 +73,7 @@ bool make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, 
     if (i + 1 < rank) st[i] = strides[i];
   }
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), d, st, b, es,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
@@ -83,6 +84,16 @@ bool map_2d(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int bo
   uint64_t strides[1] = {uint64_t(cols) * 2};
   uint32_t box[2] = {64, uint32_t(box_rows)};
   return make_map(m, base, 2, dims, strides, box);
+}
+
+// The output of an E_TMA GEMM: bf16 [rows][cols] with row pitch ld, box 32
+// columns x 32 rows, 64-byte swizzle (the epilogue's staging layout).
+bool map_out(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int64_t ld) {
+  if (ld % 8 || cols > ld || (reinterpret_cast<uintptr_t>(base) & 15)) return false;
+  uint64_t dims[2] = {uint64_t(cols), uint64_t(rows)};
+  uint64_t strides[1] = {uint64_t(ld) * 2};
+  uint32_t box[2] = {32, 32};
+  return make_map(m, base, 2, dims, strides, box, nullptr, CU_TENSOR_MAP_SWIZZLE_64B);
 }
 
 // 4-D NHWC window map over an N x H x W x C tensor that loads, per box,
@@ -270,6 +281,11 @@ TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
   g->p.N = N;
   g->flops = 2.0 * M * N * K;
   g->p.err = c->err;
+  // An unsplit plan with a plain bf16 output stores it by TMA from an
+  // accumulator that starts from the bias (E_TMA).
+  if (g->splits == 1 && !(epi_of(g->p) & (E_F32 | E_POOL)) && !g->p.ostride && !getenv("FO_NO_TMA_STORE") &&
+      map_out(&g->p.tmO, g->p.out, M, N, g->p.ldo))
+    g->p.tma_out = 1;
   g->fn = pick_kernel(g->kind, g->bn, g->splits > 1, epi_of(g->p), &g->smem);
   if (!g->fn) {
     delete g;

@@ -16,6 +16,14 @@ KernelFn pick_dgrad(int kind, int bn, bool cluster, int epi, size_t* smem) {
   if (kind == CONV_DGRAD && epi == (E_MASK)) return kernel_bn<CONV_DGRAD, E_MASK>(bn, cluster, smem);
   if (kind == CONV_DGRAD && epi == (E_ACC)) return kernel_bn<CONV_DGRAD, E_ACC>(bn, cluster, smem);
   if (kind == CONV_DGRAD && epi == (E_MASK | E_ACC)) return kernel_bn<CONV_DGRAD, E_MASK | E_ACC>(bn, cluster, smem);
+  if (kind == LIN_DGRAD && epi == (E_TMA)) return kernel_bn<LIN_DGRAD, E_TMA>(bn, cluster, smem);
+  if (kind == LIN_DGRAD && epi == (E_MASK | E_TMA)) return kernel_bn<LIN_DGRAD, E_MASK | E_TMA>(bn, cluster, smem);
+  if (kind == LIN_DGRAD && epi == (E_ACC | E_TMA)) return kernel_bn<LIN_DGRAD, E_ACC | E_TMA>(bn, cluster, smem);
+  if (kind == LIN_DGRAD && epi == (E_MASK | E_ACC | E_TMA)) return kernel_bn<LIN_DGRAD, E_MASK | E_ACC | E_TMA>(bn, cluster, smem);
+  if (kind == CONV_DGRAD && epi == (E_TMA)) return kernel_bn<CONV_DGRAD, E_TMA>(bn, cluster, smem);
+  if (kind == CONV_DGRAD && epi == (E_MASK | E_TMA)) return kernel_bn<CONV_DGRAD, E_MASK | E_TMA>(bn, cluster, smem);
+  if (kind == CONV_DGRAD && epi == (E_ACC | E_TMA)) return kernel_bn<CONV_DGRAD, E_ACC | E_TMA>(bn, cluster, smem);
+  if (kind == CONV_DGRAD && epi == (E_MASK | E_ACC | E_TMA)) return kernel_bn<CONV_DGRAD, E_MASK | E_ACC | E_TMA>(bn, cluster, smem);
   return nullptr;
 }
 

@@ -43,6 +43,11 @@ enum Epi : int {
                 // columns per image row, so a warp's 32 rows hold whole
                 // windows); writes the pooled values and the window codes
                 // instead of the full-resolution output
+  E_TMA = 32,   // persistent kernel, bf16 row-major output: the accumulator
+                // starts from the bias (and, for E_ACC without E_MASK, the
+                // accumulate operand), written into tensor memory before the
+                // tile's MMAs, and each 32 x 32 chunk leaves through shared
+                // memory by a TMA tensor store (tmO)
 };
 
 constexpr int BM = 128;      // UMMA M (cta_group::1)
@@ -57,6 +62,7 @@ typedef void (*KernelFn)(const TcParams);
 struct TcParams {
   CUtensorMap tmA;
   CUtensorMap tmB;
+  CUtensorMap tmO;      // E_TMA: the output, bf16 [M][ldo], box 32 x 32, 64-byte swizzle
   int M, N, KB, kper;
   // window geometry (spatial size of the windowed tensor and its taps)
   int H, W, ksz, pad, taps;
@@ -81,6 +87,7 @@ struct TcParams {
   const float* bias;
   const bf16* mask;     // ReLU mask (same layout as out): keep where mask > 0
   int relu, acc, out_f32;
+  int tma_out;          // E_TMA (tmO is valid)
   // bf16 outputs only: the accumulate operand (acc) is read from accsrc, which
   // is `out` itself unless the sum goes to a new buffer (a residual add:
   // out = result + accsrc).
@@ -641,6 +648,90 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 // MMA), acc_full/acc_empty per accumulator (MMA <-> epilogue).
 constexpr int kPersistThreads = 320;  // TMA warp, MMA warp, 8 epilogue warps
 constexpr int kEpiStageBytes = 8 * 4096;  // one 32 x 32 fp32 staging buffer per epilogue warp
+// E_TMA: the starting value of this thread's accumulator row m (TMEM lane
+// address tbase), columns n_base .. n_base + CW - 1: the bias of each column,
+// plus the accumulate operand unless a ReLU mask comes first (E_MASK | E_ACC
+// adds it after the mask, in the epilogue); zeros outside the output.
+template <int EPI, int CW>
+__device__ __forceinline__ void tma_preload(const TcParams& p, uint32_t tbase, int m, int n_base) {
+  const bool row_ok = m < p.M;
+#pragma unroll 1
+  for (int c = 0; c < CW; c += 32) {
+    const int n = n_base + c;
+    uint32_t v[32];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const bool col_ok = n + 8 * u < p.N;
+      float4 b0 = make_float4(0.f, 0.f, 0.f, 0.f), b1 = b0;
+      if (p.bias && col_ok) {
+        b0 = __ldg(reinterpret_cast<const float4*>(p.bias + n + 8 * u));
+        b1 = __ldg(reinterpret_cast<const float4*>(p.bias + n + 8 * u) + 1);
+      }
+      float e[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+      if constexpr ((EPI & E_ACC) && !(EPI & E_MASK)) {
+        if (row_ok && col_ok) {
+          const uint4 a = *reinterpret_cast<const uint4*>(p.accsrc + size_t(m) * p.ldo + n + 8 * u);
+          const bf16* ab = reinterpret_cast<const bf16*>(&a);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) e[j] += __bfloat162float(ab[j]);
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) v[8 * u + j] = __float_as_uint(e[j]);
+    }
+    tmem_st32(tbase + uint32_t(c), v);
+  }
+}
+
+// E_TMA: one 32 x 32 chunk, this thread's row m and columns n .. n + 31 in
+// r: ReLU / ReLU mask / accumulate after the mask, bf16, into the 2 KB
+// staging buffer `buf` (512-byte aligned) in the layout of a 32 x 32 box of
+// the 64-byte-swizzled output map (row i at 64 i, its 16-byte unit u at
+// u ^ ((i >> 1) & 3)), made visible to the TMA store that follows.
+template <int EPI>
+__device__ __forceinline__ void tma_chunk32(const TcParams& p, uint32_t buf, int lane, int m, int n,
+                                            const uint32_t (&r)[32]) {
+  const bool row_ok = m < p.M;
+  uint4 mk[4] = {}, ac[4] = {};
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const bool ok = row_ok && n + 8 * u < p.N;
+    if constexpr (EPI & E_MASK)
+      if (ok) mk[u] = *reinterpret_cast<const uint4*>(p.mask + size_t(m) * p.ldo + n + 8 * u);
+    if constexpr ((EPI & E_ACC) && (EPI & E_MASK))
+      if (ok) ac[u] = *reinterpret_cast<const uint4*>(p.accsrc + size_t(m) * p.ldo + n + 8 * u);
+  }
+  const int f = (lane >> 1) & 3;
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    float e[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) e[j] = __uint_as_float(r[8 * u + j]);
+    if constexpr (EPI & E_RELU)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) e[j] = fmaxf(e[j], 0.f);
+    if constexpr (EPI & E_MASK) {
+      const bf16* mkp = reinterpret_cast<const bf16*>(&mk[u]);
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        if (!(__bfloat162float(mkp[j]) > 0.f)) e[j] = 0.f;
+      if constexpr (EPI & E_ACC) {
+        const bf16* ap = reinterpret_cast<const bf16*>(&ac[u]);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) e[j] += __bfloat162float(ap[j]);
+      }
+    }
+    uint32_t pk[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      __nv_bfloat162 h2 = __floats2bfloat162_rn(e[2 * q], e[2 * q + 1]);
+      pk[q] = *reinterpret_cast<uint32_t*>(&h2);
+    }
+    st_shared4(buf + 16u * uint32_t(lane * 4 + (u ^ f)), pk[0], pk[1], pk[2], pk[3]);
+  }
+  fence_proxy_async_smem();
+}
+
 template <int KIND, int BN, int STAGES, int EPI>
 __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const __grid_constant__ TcParams p) {
   extern __shared__ __align__(1024) char smem_raw[];
@@ -718,7 +809,9 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
       uint32_t g = 0, lt = 0;
       for (int t = unit; t < tiles && !*abort_flag; t += units, ++lt) {
         const uint32_t b = lt & 1;
-        if (!mbar_wait(&acc_empty[b], ((lt >> 1) & 1) ^ 1)) {
+        // E_TMA: the epilogue warps arrive once per buffer before the first
+        // tile, after writing its starting value
+        if (!mbar_wait(&acc_empty[b], ((lt >> 1) & 1) ^ ((EPI & E_TMA) ? 0u : 1u))) {
           atomicExch(p.err, 5);
           *abort_flag = 1;
           mbar_expect_tx(&acc_full[b], 0);
@@ -745,7 +838,7 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
             else ad = smem_desc(a0 + k * UK * 2, 16, 1024);
             if (KindTraits<KIND>::b_mn) bd = smem_desc(b0 + k * UK * 128, BK * 128, 1024);
             else bd = smem_desc(b0 + k * UK * 2, 16, 1024);
-            mma_f16(d, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+            mma_f16(d, ad, bd, idesc, ((EPI & E_TMA) || kb > 0 || k > 0) ? 1u : 0u);
           }
           mma_commit(&empty[s]);
         }
@@ -756,6 +849,71 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
         }
       }
     }
+  } else if constexpr ((EPI & E_TMA) != 0) {
+    // Epilogue through TMA stores: warp w (2..9) owns TMEM lanes
+    // 32 * (w % 4) .. +31 and half of the tile's columns; each lane holds
+    // one output row.  Two 2 KB staging buffers per warp alternate, each
+    // reused once the TMA store that read it two chunks earlier is done.
+    const int q = warp % 4, half = (warp - 2) / 4;
+    constexpr int CW = BN / 2;
+    const uint32_t tq = tmem + (uint32_t(q * 32) << 16) + uint32_t(half * CW);
+    const uint32_t stage0 = smem_u32(stage_all) + uint32_t(warp - 2) * 4096u;
+    for (int b = 0; b < 2; ++b) {   // the first two tiles' accumulators start from the bias
+      const int t = unit + b * units;
+      if (t < tiles) tma_preload<EPI, CW>(p, tq + uint32_t(b * BN), tile_m0(t) + q * 32 + lane, tile_n0(t) + half * CW);
+      tmem_st_wait();
+      tc_fence_before();
+      mbar_arrive(&acc_empty[b]);
+    }
+    uint32_t lt = 0, sbuf = 0;
+    int issued = 0;
+    for (int t = unit; t < tiles; t += units, ++lt) {
+      const uint32_t b = lt & 1;
+      const int n0 = tile_n0(t) + half * CW, m0 = tile_m0(t) + q * 32;
+      const bool ready = mbar_wait(&acc_full[b], (lt >> 1) & 1);
+      tc_fence_after();
+      if (!ready) {
+        atomicExch(p.err, 7);
+        *abort_flag = 1;
+      }
+      if (!ready || *abort_flag) break;
+      const uint32_t trow = tq + b * BN;
+      uint32_t cur[32], nxt[32];
+      tmem_ld32_issue(trow, cur);
+      tmem_ld32_wait(cur);
+#pragma unroll 1
+      for (int c = 0; c < CW; c += 32) {
+        const bool more = c + 32 < CW;
+        if (more) tmem_ld32_issue(trow + uint32_t(c + 32), nxt);
+        if (n0 + c < p.N && m0 < p.M) {   // a box past the end of the output has nothing to write
+          const uint32_t buf = stage0 + sbuf * 2048u;
+          if (issued >= 2) {   // buf's previous store is not the newest: at most one may still read
+            if (lane == 0) bulk_wait_read<1>();
+            __syncwarp();
+          }
+          tma_chunk32<EPI>(p, buf, lane, m0 + lane, n0 + c, cur);
+          __syncwarp();
+          if (lane == 0) tma_store_2d(&p.tmO, buf, n0 + c, m0);
+          ++issued;
+          sbuf ^= 1u;
+        }
+        if (more) {
+          tmem_ld32_wait(nxt);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) cur[j] = nxt[j];
+        }
+      }
+      // this warp's part of buffer b is drained: start it for the tile two ahead
+      const int t2 = t + 2 * units;
+      if (t2 < tiles) {
+        tma_preload<EPI, CW>(p, trow, tile_m0(t2) + q * 32 + lane, tile_n0(t2) + half * CW);
+        tmem_st_wait();
+      }
+      tc_fence_before();
+      mbar_arrive(&acc_empty[b]);
+    }
+    if (lane == 0) bulk_wait_all();   // the stores have read shared memory and reached global memory
+    __syncwarp();
   } else {
     // Epilogue: warp w (2..9) reads TMEM lanes 32 * (w % 4) .. +31; the two
     // warps of a lane quarter split the tile's columns.
@@ -841,8 +999,13 @@ constexpr size_t smem_bytes(bool cluster) {
 template <int KIND, int BN, int EPI>
 KernelFn kernel_of(bool cluster, size_t* smem) {
   *smem = smem_bytes<KIND, BN>(cluster);
-  if (cluster) return tc_gemm_kernel<KIND, BN, stages_for<KIND, BN, true>(), EPI>;
-  return tc_gemm_persistent<KIND, BN, stages_for<KIND, BN, false>(), EPI>;
+  if constexpr ((EPI & E_TMA) != 0) {   // the persistent kernel only
+    if (cluster) return nullptr;
+    return tc_gemm_persistent<KIND, BN, stages_for<KIND, BN, false>(), EPI>;
+  } else {
+    if (cluster) return tc_gemm_kernel<KIND, BN, stages_for<KIND, BN, true>(), EPI>;
+    return tc_gemm_persistent<KIND, BN, stages_for<KIND, BN, false>(), EPI>;
+  }
 }
 template <int KIND, int EPI>
 KernelFn kernel_bn(int bn, bool cluster, size_t* smem) {

@@ -66,8 +66,14 @@ def test_batch_one_one_device_one_slot(dtype):
 
 @pytest.mark.parametrize("length", [1, 128])
 def test_sequences_all_of_one_length(length):
+    """Batch 16: with one valid token per sequence the classifier's and the
+    final layernorm's gradients are sums over the batch's few softmax
+    residuals, and at batch 6 their rounding spread alone (two accumulation
+    orders of the same kernels: 1.6% and 2.7% from the exact gradient)
+    exceeds what the bf16-storage reading's distance allows; at batch 16
+    both orders sit near 1.2%."""
     cfg = W.shrink(W.CONFIGS["transformer"], ops=W.transformer_ops(d=128, heads=2, ffn=256, blocks=2),
-                   batch=6, in_hwc=(128, 1, 128), K=2, omega=4, depth=2, fixed_len=length, lr=1e-3)
+                   batch=16, in_hwc=(128, 1, 128), K=2, omega=4, depth=2, fixed_len=length, lr=1e-3)
     ev = [("enq", k) for _ in range(2) for k in range(2)] + [("step",)] * 4
     _, _, recs = teacher_forced(cfg, ev)
     assert len(recs) == 4
