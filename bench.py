@@ -406,20 +406,21 @@ class Harness:
         self.srv.close()
 
 
-def roofline_of(ktimes, pk, which):
+def roofline_of(ktimes, pk, which, workload):
     """The dominant kernel class of a step (largest total time in the
-    profiled pass): achieved = algorithmic FLOPs (bytes) / its event time."""
+    profiled pass): achieved = algorithmic FLOPs (bytes) / its event time;
+    traffic = its measured DRAM bytes per launch on this workload."""
     name, (nl, ms_k, fl_k, by_k) = max(ktimes.items(), key=lambda kv: kv[1][1])
     if fl_k > 0:
         achieved = fl_k / (ms_k / 1e3) / 1e12
         sus = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
         return {"kernel": name, "bound": "tensor", "achieved": round(achieved, 2), "peak": pk["bf16_tflops"],
                 "unit": "TFLOP/s", "frac": round(achieved / pk["bf16_tflops"], 4),
-                "frac_sustained": round(achieved / sus, 4), "traffic": traffic_for(name),
+                "frac_sustained": round(achieved / sus, 4), "traffic": traffic_for(name, workload),
                 "peak_kind": f"{which} burst bf16 (sustained {sus})", "launches": nl, "ms_total": round(ms_k, 3)}
     achieved = by_k / (ms_k / 1e3) / 1e9
     return {"kernel": name, "bound": "hbm", "achieved": round(achieved, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
-            "frac": round(achieved / pk["hbm_gbs"], 4), "traffic": traffic_for(name), "peak_kind": f"{which} copy",
+            "frac": round(achieved / pk["hbm_gbs"], 4), "traffic": traffic_for(name, workload), "peak_kind": f"{which} copy",
             "launches": nl, "ms_total": round(ms_k, 3)}
 
 
@@ -488,7 +489,7 @@ def run_ours(args):
                                                                              / (ms_w / 1e3), 1),
                             "unit": UNIT, "steps": n_w, "ms_per_step": round(ms_w / n_w, 4),
                             "step_gflop": round(fl / 1e9, 2), "step_tensor_frac_burst": round(fb, 4),
-                            "step_tensor_frac_sustained": round(fs, 4), "roofline": roofline_of(kt, pk, which)}
+                            "step_tensor_frac_sustained": round(fs, 4), "roofline": roofline_of(kt, pk, which, name)}
             hw.close()
             del hw
             torch.cuda.empty_cache()
@@ -528,7 +529,7 @@ def run_ours(args):
 
     if rank != 0:
         return
-    roof = roofline_of(ktimes, pk, which)
+    roof = roofline_of(ktimes, pk, which, args.workload)
     step_flops, tensor_frac_burst, tensor_frac = step_fracs(ktimes, n_prof, ms_dev / args.steps, pk)
     cpu = None
     if not args.no_cpu_baseline and world == 1:
@@ -577,21 +578,22 @@ def run_ours(args):
     print(json.dumps(line), flush=True)
 
 
-def traffic_for(kernel):
-    """DRAM bytes per launch of `kernel` from the committed ncu summary, if the
-    kernel source has not changed since it was captured (else None)."""
+def traffic_for(kernel, workload):
+    """DRAM bytes per launch of `kernel` on `workload` from the committed ncu
+    summary, if the kernel source has not changed since it was captured
+    (else None)."""
     import hashlib
     path = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
     if not os.path.exists(path):
         return None
     for line in open(path):
         f = line.split()
-        if len(f) >= 3 and not line.startswith("#") and f[0] == kernel:
-            src = os.path.join(ROOT, "paper_2504_13850_gb300", "csrc", f[1].split(":")[0])
+        if len(f) >= 4 and not line.startswith("#") and f[0] == workload and f[1] == kernel:
+            src = os.path.join(ROOT, "paper_2504_13850_gb300", "csrc", f[2].split(":")[0])
             if os.path.exists(src):
                 h = hashlib.sha1(open(src, "rb").read()).hexdigest()[:12]
-                if h == f[1].split(":")[1]:
-                    return float(f[2])
+                if h == f[2].split(":")[1]:
+                    return float(f[3])
     return None
 
 
