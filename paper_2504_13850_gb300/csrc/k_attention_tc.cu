@@ -9,7 +9,8 @@
 //             dS = P (dP - rowsum(dO * O)) / 8 (bf16, shared memory) ->
 //             dV = P^T dO, dQ = dS K, dK = dS^T Q (TMEM) -> d(q|k|v).
 // Operand tiles are 128 rows x 64 bf16 (128-byte rows, 128-byte swizzle),
-// loaded by TMA from the packed q|k|v [B*L, 3C], O [B*L, C] and dO [B*L, C];
+// loaded by TMA from the packed q|k|v [B*L, 3C] and dO [B*L, C] (the
+// backward reads O's rows directly for rowsum(dO * O));
 // P and dS are written by the softmax threads in the same swizzled layout as
 // two 64-column sub-tiles, which serves both as a K-major operand (P V,
 // dS K) and as an MN-major one (P^T dO, dS^T Q).
@@ -35,9 +36,9 @@ constexpr float kScale = 0.125f;          // 1 / sqrt(64)
 
 struct AttnParams {
   CUtensorMap tm_qkv;     // [B*L, 3C], box 64 x 128
-  CUtensorMap tm_o;       // [B*L, C],  box 64 x 128 (backward)
   CUtensorMap tm_do;      // [B*L, C],  box 64 x 128 (backward)
   const int32_t* len;     // [B]
+  const bf16* o;          // backward: the forward output O [B*L, C] (for rowsum(dO * O))
   bf16* out;              // forward: O [B*L, C]; backward: d(q|k|v) [B*L, 3C]
   float* lse;             // [B * heads * L]
   int L, C, heads, acc;
@@ -211,17 +212,24 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_tc_k(const __grid_co
   }
 }
 
-__global__ void __launch_bounds__(kAttnThreads, 1) attn_bwd_tc_k(const __grid_constant__ AttnParams p) {
+// Two CTAs per SM: 7 tiles of shared memory (112 KB) and 256 TMEM columns.
+// V is read only by the first MMA phase, so P's first sub-tile takes its
+// buffer once that phase has completed; O is read from global memory (only
+// its row sums with dO are needed); dQ, dV and dK take the TMEM columns of S
+// and dP, which the softmax warps have read before the second phase starts.
+__global__ void __launch_bounds__(kAttnThreads, 2) attn_bwd_tc_k(const __grid_constant__ AttnParams p) {
   extern __shared__ __align__(1024) char smem_raw[];
   char* sm = align1024(smem_raw);
   char* sQ = sm;
   char* sK = sm + kTile;
   char* sV = sm + 2 * kTile;
-  char* sdO = sm + 3 * kTile;
-  char* sO = sm + 4 * kTile;
-  char* sP = sm + 5 * kTile;      // two sub-tiles
-  char* sdS = sm + 7 * kTile;     // two sub-tiles
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + 9 * kTile);   // ld, s, p, g
+  char* sP = sm + 2 * kTile;      // two sub-tiles: V's buffer after the first phase, then the next
+  char* sdO = sm + 4 * kTile;
+  char* sdS = sm + 5 * kTile;     // two sub-tiles
+  // barriers (ld, s, p, g) and the TMEM slot: in the alignment slack below
+  // the tiles when it has room, else after them (the request covers both)
+  const bool low = sm - smem_raw >= 64;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(low ? smem_raw : sm + 7 * kTile);
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 4);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -234,31 +242,29 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_bwd_tc_k(const __grid_co
     mbar_init(&bars[3], 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_qkv)) : "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_o)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tm_do)) : "memory");
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tslot)),
-                 "r"(512)
+                 "r"(256)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  // TMEM columns: S 0..127, dP 128..255, dV 256..319, dQ 320..383, dK 384..447
+  // TMEM columns: S 0..127 and dP 128..255; then dQ 0..63, dV 128..191, dK 192..255
   const uint32_t tmem = *tslot;
   pdl_trigger();
   pdl_wait();
 
   if (warp == 0) {
     if (lane == 0) {
-      mbar_expect_tx(&bars[0], 5 * kTile);
+      mbar_expect_tx(&bars[0], 4 * kTile);
       tma_2d(sQ, &p.tm_qkv, &bars[0], h * 64, row0);
       tma_2d(sK, &p.tm_qkv, &bars[0], p.C + h * 64, row0);
       tma_2d(sV, &p.tm_qkv, &bars[0], 2 * p.C + h * 64, row0);
       tma_2d(sdO, &p.tm_do, &bars[0], h * 64, row0);
-      tma_2d(sO, &p.tm_o, &bars[0], h * 64, row0);
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -281,13 +287,13 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_bwd_tc_k(const __grid_co
       for (int k = 0; k < 8; ++k) {
         const uint32_t acc = k > 0 ? 1u : 0u;
         // dV[j][d] = sum_i P[i][j] dO[i][d]
-        mma_f16(tmem + 256, smem_desc(smem_u32(sP) + 2048 * k, kTile, 1024),
+        mma_f16(tmem + 128, smem_desc(smem_u32(sP) + 2048 * k, kTile, 1024),
                 smem_desc(smem_u32(sdO) + 2048 * k, kTile, 1024), id_tt, acc);
         // dQ[i][d] = sum_j dS[i][j] K[j][d]
-        mma_f16(tmem + 320, smem_desc(smem_u32(sdS) + (k >> 2) * kTile + 32 * (k & 3), 16, 1024),
+        mma_f16(tmem, smem_desc(smem_u32(sdS) + (k >> 2) * kTile + 32 * (k & 3), 16, 1024),
                 smem_desc(smem_u32(sK) + 2048 * k, kTile, 1024), id_nt, acc);
         // dK[j][d] = sum_i dS[i][j] Q[i][d]
-        mma_f16(tmem + 384, smem_desc(smem_u32(sdS) + 2048 * k, kTile, 1024),
+        mma_f16(tmem + 192, smem_desc(smem_u32(sdS) + 2048 * k, kTile, 1024),
                 smem_desc(smem_u32(sQ) + 2048 * k, kTile, 1024), id_tt, acc);
       }
       mma_commit(&bars[3]);
@@ -297,16 +303,24 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_bwd_tc_k(const __grid_co
     const uint32_t trow = tmem + (uint32_t(q * 32) << 16);
     const int n = min(p.len[b], p.L);
     const bool live = i < p.L;          // rows past the sequence get P = dS = 0
+    // D_i = sum_d dO[i][d] O[i][d]: O's row from global memory (in flight
+    // during the TMA wait), dO's from the swizzled tile
+    uint4 orow[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) orow[u] = make_uint4(0u, 0u, 0u, 0u);
+    if (live) {
+      const uint4* src = reinterpret_cast<const uint4*>(p.o + size_t(row0 + i) * p.C + h * 64);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) orow[u] = src[u];
+    }
     if (!mbar_wait(&bars[0], 0)) atomicExch(p.err, 15);
-    // D_i = sum_d dO[i][d] O[i][d] from the swizzled tiles
     float D = 0.f;
-    const uint32_t do_base = smem_u32(sdO), o_base = smem_u32(sO);
+    const uint32_t do_base = smem_u32(sdO);
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
       const float4 a = ld_shared4(do_base + sw_off(i, u));
-      const float4 c = ld_shared4(o_base + sw_off(i, u));
       const bf16* ab = reinterpret_cast<const bf16*>(&a);
-      const bf16* cb = reinterpret_cast<const bf16*>(&c);
+      const bf16* cb = reinterpret_cast<const bf16*>(&orow[u]);
 #pragma unroll
       for (int e = 0; e < 8; ++e) D = fmaf(__bfloat162float(ab[e]), __bfloat162float(cb[e]), D);
     }
@@ -346,7 +360,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_bwd_tc_k(const __grid_co
     bf16* drow = p.out + size_t(row0 + i) * 3 * p.C;
 #pragma unroll 1
     for (int t = 0; t < 3; ++t) {
-      const uint32_t col = t == 0 ? 320u : (t == 1 ? 384u : 256u);     // dQ, dK, dV
+      const uint32_t col = t == 0 ? 0u : (t == 1 ? 192u : 128u);     // dQ, dK, dV
       uint32_t r[32];
       tmem_ld32(trow + col + 32 * hf, r);
       if (live) store_row32(drow + t * p.C + h * 64 + 32 * hf, r, p.acc != 0);
@@ -356,12 +370,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_bwd_tc_k(const __grid_co
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512) : "memory");
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(256) : "memory");
   }
 }
 
 constexpr size_t kFwdSmem = 5 * kTile + 1024 + 64 + 2 * 128 * sizeof(float2);
-constexpr size_t kBwdSmem = 9 * kTile + 1024 + 64;
+constexpr size_t kBwdSmem = 7 * kTile + 1024;   // 115,712 B: two CTAs in an SM's 228 KB
 
 }  // namespace
 
@@ -380,16 +394,23 @@ AttnTcPlan* attention_tc_plan(const void* qkv, const void* out, const void* dout
   a->p.C = C;
   a->p.heads = heads;
   a->p.err = err;
+  a->p.o = static_cast<const bf16*>(out);
   const int64_t rows = int64_t(B) * L;
-  if (!tc_encode_2d(&a->p.tm_qkv, qkv, rows, 3 * C, 128) || !tc_encode_2d(&a->p.tm_o, out, rows, C, 128) ||
+  if (!tc_encode_2d(&a->p.tm_qkv, qkv, rows, 3 * C, 128) ||
       (dout && !tc_encode_2d(&a->p.tm_do, dout, rows, C, 128))) {
     delete a;
     return nullptr;
   }
+  // Both kernels are sized for two CTAs per SM, which needs the largest
+  // shared-memory carveout (the default sizes the carveout for one block).
   if (cudaFuncSetAttribute(attn_fwd_tc_k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kFwdSmem)) !=
           cudaSuccess ||
       cudaFuncSetAttribute(attn_bwd_tc_k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kBwdSmem)) !=
-          cudaSuccess) {
+          cudaSuccess ||
+      cudaFuncSetAttribute(attn_fwd_tc_k, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           int(cudaSharedmemCarveoutMaxShared)) != cudaSuccess ||
+      cudaFuncSetAttribute(attn_bwd_tc_k, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           int(cudaSharedmemCarveoutMaxShared)) != cudaSuccess) {
     delete a;
     return nullptr;
   }
