@@ -219,6 +219,9 @@ struct Fusion {
   std::vector<int> add_into;   // producer op -> the add op whose output it writes, or -1
   std::vector<int> add_other;  // that add op -> its residual operand tensor
   std::vector<int> branch_of;  // that add op -> its branch tensor, or -1
+  // A linear layer whose output feeds only a GELU: its epilogue may store
+  // the GELU too (the plan decides; the GELU op runs alone otherwise).
+  std::vector<int> gelu_of;    // producer op -> the GELU op, or -1
   bool head = false;           // last linear + loss handled by the head kernels
 };
 
@@ -234,6 +237,7 @@ Fusion analyse(const fo_server* s) {
   f.skip_fwd.assign(nops, 0);
   f.bwd_mask.assign(nops, -1);
   f.skip_bwd.assign(nops, 0);
+  f.gelu_of.assign(nops, -1);
   f.hswish_of.assign(nops, -1);
   f.hswish_by.assign(nops, -1);
   f.add_relu.assign(nops, -1);
@@ -308,6 +312,13 @@ Fusion analyse(const fo_server* s) {
       break;
     }
   }
+  for (int g = 0; g < nops && !getenv("FO_NO_GELU_EPILOGUE"); ++g) {
+    const fo_op& op = s->ops[g];
+    if (op.kind != FO_OP_GELU || s->T[op.in0].is_input()) continue;
+    const int p = op.in0 - 1;
+    if (s->ops[p].kind == FO_OP_LINEAR && sole[op.in0] == g && plain(p) && f.fwd_relu[p] < 0 && f.add_into[p] < 0)
+      f.gelu_of[p] = g;
+  }
   return f;
 }
 
@@ -344,6 +355,7 @@ int build_plan(fo_server* s) {
   // (through its ReLU): per pool op, the window codes that epilogue stores,
   // or null.
   std::vector<uint8_t*> pool_codes(nops, nullptr);
+  std::vector<char> gelu_done(nops, 0);   // GELU ops stored by the producing GEMM's epilogue
 
   // ---------------- forward
   for (int i = 0; i < nops; ++i) {
@@ -406,6 +418,12 @@ int build_plan(fo_server* s) {
           if (tg) pool_codes[pq] = codes;
           ex.pool_out = nullptr;
           ex.pool_code = nullptr;
+        }
+        if (!tg && fu.gelu_of[i] >= 0) {
+          ex.gelu_out = s->T[fu.gelu_of[i] + 1].act;
+          tg = fo::tc_plan_forward(s->tc, s, i, s->T[o].act, relu, &ex);
+          if (tg) gelu_done[fu.gelu_of[i]] = 1;
+          ex.gelu_out = nullptr;
         }
         if (!tg) tg = fo::tc_plan_forward(s->tc, s, i, s->T[o].act, relu, fused ? &ex : nullptr);
         if (fused && !tg) return set_err(FO_ERR_ARG, "op " + std::to_string(i) + ": fused epilogue not planned");
@@ -470,6 +488,7 @@ int build_plan(fo_server* s) {
         });
         break;
       case FO_OP_GELU:
+        if (gelu_done[i]) break;   // stored by the producing GEMM's epilogue
         add("gelu_fwd", 1, 0.0, 2 * tbytes(a), [=](cudaStream_t st) {
           fo::gelu_fwd(act(a), s->T[o].act, s->T[a].numel(), dt, st);
         });

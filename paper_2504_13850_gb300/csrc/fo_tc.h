@@ -31,6 +31,9 @@ struct TcEpilogue {
   // element (first maximum, 0..3 row-major) instead of the full output
   void* pool_out = nullptr;
   uint8_t* pool_code = nullptr;
+  // forward of a linear layer whose output feeds only a GELU: `out` gets the
+  // bias-added result and gelu_out the GELU of it (bf16, the same layout)
+  void* gelu_out = nullptr;
 };
 // Forward of conv/linear op `op` into `out` (bf16, the op's output layout),
 // applying a ReLU when `relu`.
@@ -51,7 +54,7 @@ bool tc_plan_dgrad(TcContext* c, fo_server* s, int op, int accumulate, void* dx,
 bool tc_plain_ok(TcContext* c, const fo_server* s, int op);
 TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int op);
 // Launches the GEMM kernel; a split-K plan runs as clusters of tc_splits(g)
-// CTAs that reduce their partial tiles through distributed shared memory.
+// CTAs that reduce their partial tiles through an L2-resident workspace.
 void tc_run(TcGemm* g, const void* input, cudaStream_t st);
 int tc_splits(const TcGemm* g);
 double tc_flops(const TcGemm* g);
@@ -70,7 +73,8 @@ bool tc_encode_2d(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, 
 
 // Tensor-core attention (k_attention_tc.cu): sequences of at most 128 tokens,
 // head width 64, bf16.  A plan holds the tensor maps of the packed q|k|v
-// input [B*L, 3C], the output O [B*L, C] and its gradient dO [B*L, C].
+// input [B*L, 3C] and of dO [B*L, C], and the address of the output O
+// [B*L, C] (the backward reads its rows directly).
 struct AttnTcPlan;
 bool attention_tc_ok(int L, int C, int heads);
 AttnTcPlan* attention_tc_plan(const void* qkv, const void* out, const void* dout, int B, int L, int C, int heads,

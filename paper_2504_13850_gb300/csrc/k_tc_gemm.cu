@@ -20,7 +20,7 @@ namespace {
 // The epilogue variant a plan's parameters ask for.
 int epi_of(const TcParams& p) {
   return (p.out_f32 ? E_F32 : 0) | (p.relu ? E_RELU : 0) | (p.mask ? E_MASK : 0) | (p.acc ? E_ACC : 0) |
-         (p.pool_out ? E_POOL : 0) | (p.tma_out ? E_TMA : 0);
+         (p.pool_out ? E_POOL : 0) | (p.tma_out ? E_TMA : 0) | (p.gelu_out ? E_GELU : 0);
 }
 
 KernelFn pick_kernel(int kind, int bn, bool cluster, int epi, size_t* smem) {
@@ -286,6 +286,12 @@ TcGemm* finish(TcContext* c, TcGemm* g, int M, int N, double K) {
   if (g->splits == 1 && !(epi_of(g->p) & (E_F32 | E_POOL)) && !g->p.ostride && !getenv("FO_NO_TMA_STORE") &&
       map_out(&g->p.tmO, g->p.out, M, N, g->p.ldo))
     g->p.tma_out = 1;
+  // The GELU epilogue exists only in that form (a split plan runs the GELU
+  // as its own kernel: the caller plans again without it).
+  if (g->p.gelu_out && (!g->p.tma_out || !map_out(&g->p.tmG, g->p.gelu_out, M, N, g->p.ldo))) {
+    delete g;
+    return nullptr;
+  }
   g->fn = pick_kernel(g->kind, g->bn, g->splits > 1, epi_of(g->p), &g->smem);
   if (!g->fn) {
     delete g;
@@ -389,6 +395,7 @@ static void apply_epilogue(TcGemm* g, const TcEpilogue* ex) {
   if (!ex) return;
   g->p.pool_out = static_cast<bf16*>(ex->pool_out);
   g->p.pool_code = ex->pool_code;
+  g->p.gelu_out = static_cast<bf16*>(ex->gelu_out);
   if (ex->addend || ex->addend_is_input) {
     g->p.acc = 1;
     g->p.accsrc = static_cast<const bf16*>(ex->addend);
@@ -403,6 +410,8 @@ TcGemm* tc_plan_forward(TcContext* c, fo_server* s, int i, void* out, bool relu,
   const Tensor& o = s->T[i + 1];
   if (o.dt != kBF16) return nullptr;  // fp32 logits: CUDA-core path
   if (ex && (ex->addend || ex->addend_is_input) && (relu || !plain_gemm(op))) return nullptr;
+  if (ex && ex->gelu_out && (relu || !plain_gemm(op) || ex->pool_out || ex->addend || ex->addend_is_input))
+    return nullptr;
   if (ex && ex->pool_out) {   // whole 2 x 2 windows inside each warp's 32 rows
     const bool w_ok = o.W == 2 || o.W == 4 || o.W == 8 || o.W == 16;
     if (!relu || !w_ok || o.H % 2 || o.C % 8 || o.rows() % BM) return nullptr;

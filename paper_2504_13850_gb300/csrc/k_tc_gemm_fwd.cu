@@ -15,6 +15,7 @@ KernelFn pick_fwd(int kind, int bn, bool cluster, int epi, size_t* smem) {
   if (kind == LIN_FWD && epi == (E_TMA)) return kernel_bn<LIN_FWD, E_TMA>(bn, cluster, smem);
   if (kind == LIN_FWD && epi == (E_RELU | E_TMA)) return kernel_bn<LIN_FWD, E_RELU | E_TMA>(bn, cluster, smem);
   if (kind == LIN_FWD && epi == (E_ACC | E_TMA)) return kernel_bn<LIN_FWD, E_ACC | E_TMA>(bn, cluster, smem);
+  if (kind == LIN_FWD && epi == (E_GELU | E_TMA)) return kernel_bn<LIN_FWD, E_GELU | E_TMA>(bn, cluster, smem);
   if (kind == CONV_FPROP && epi == (0)) return kernel_bn<CONV_FPROP, 0>(bn, cluster, smem);
   if (kind == CONV_FPROP && epi == (E_RELU)) return kernel_bn<CONV_FPROP, E_RELU>(bn, cluster, smem);
   if (kind == CONV_FPROP && epi == (E_ACC)) return kernel_bn<CONV_FPROP, E_ACC>(bn, cluster, smem);

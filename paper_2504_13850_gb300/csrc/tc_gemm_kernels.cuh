@@ -43,6 +43,8 @@ enum Epi : int {
                 // columns per image row, so a warp's 32 rows hold whole
                 // windows); writes the pooled values and the window codes
                 // instead of the full-resolution output
+  E_GELU = 64,  // with E_TMA: out = the bias-added result (bf16), and
+                // gelu_out = GELU of that stored value (the FFN's activation)
   E_TMA = 32,   // persistent kernel, bf16 row-major output: the accumulator
                 // starts from the bias (and, for E_ACC without E_MASK, the
                 // accumulate operand), written into tensor memory before the
@@ -63,6 +65,7 @@ struct TcParams {
   CUtensorMap tmA;
   CUtensorMap tmB;
   CUtensorMap tmO;      // E_TMA: the output, bf16 [M][ldo], box 32 x 32, 64-byte swizzle
+  CUtensorMap tmG;      // E_GELU: gelu_out, the same layout
   int M, N, KB, kper;
   // window geometry (spatial size of the windowed tensor and its taps)
   int H, W, ksz, pad, taps;
@@ -88,6 +91,7 @@ struct TcParams {
   const bf16* mask;     // ReLU mask (same layout as out): keep where mask > 0
   int relu, acc, out_f32;
   int tma_out;          // E_TMA (tmO is valid)
+  bf16* gelu_out;       // E_GELU
   // bf16 outputs only: the accumulate operand (acc) is read from accsrc, which
   // is `out` itself unless the sum goes to a new buffer (a residual add:
   // out = result + accsrc).
@@ -683,6 +687,33 @@ __device__ __forceinline__ void tma_preload(const TcParams& p, uint32_t tbase, i
   }
 }
 
+// This thread's row (32 bf16, 16 packed words) into the 2 KB staging buffer
+// `buf` in the layout of a 32 x 32 box of a 64-byte-swizzled map (row i at
+// 64 i, its 16-byte unit u at u ^ ((i >> 1) & 3)).
+__device__ __forceinline__ void stage_row64(uint32_t buf, int lane, const uint32_t (&pk)[16]) {
+  const int f = (lane >> 1) & 3;
+#pragma unroll
+  for (int u = 0; u < 4; ++u)
+    st_shared4(buf + 16u * uint32_t(lane * 4 + (u ^ f)), pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+}
+
+// E_GELU: this thread's 32 accumulator values (bias included) as bf16 (the
+// pre-activation, kept for the backward pass) and the GELU of each stored
+// bf16 value, as the separate GELU kernel computes it.
+__device__ __forceinline__ void gelu_pack32(const uint32_t (&r)[32], uint32_t (&hk)[16], uint32_t (&gk)[16]) {
+#pragma unroll
+  for (int q = 0; q < 16; ++q) {
+    __nv_bfloat162 h2 = __floats2bfloat162_rn(__uint_as_float(r[2 * q]), __uint_as_float(r[2 * q + 1]));
+    hk[q] = *reinterpret_cast<uint32_t*>(&h2);
+    const float x0 = __low2float(h2), x1 = __high2float(h2);
+    float c0, d0, c1, d1;
+    normal_cdf_pdf(x0, c0, d0);
+    normal_cdf_pdf(x1, c1, d1);
+    __nv_bfloat162 g2 = __floats2bfloat162_rn(x0 * c0, x1 * c1);
+    gk[q] = *reinterpret_cast<uint32_t*>(&g2);
+  }
+}
+
 // E_TMA: one 32 x 32 chunk, this thread's row m and columns n .. n + 31 in
 // r: ReLU / ReLU mask / accumulate after the mask, bf16, into the 2 KB
 // staging buffer `buf` (512-byte aligned) in the layout of a 32 x 32 box of
@@ -886,16 +917,36 @@ __global__ void __launch_bounds__(kPersistThreads, 1) tc_gemm_persistent(const _
         const bool more = c + 32 < CW;
         if (more) tmem_ld32_issue(trow + uint32_t(c + 32), nxt);
         if (n0 + c < p.N && m0 < p.M) {   // a box past the end of the output has nothing to write
-          const uint32_t buf = stage0 + sbuf * 2048u;
-          if (issued >= 2) {   // buf's previous store is not the newest: at most one may still read
-            if (lane == 0) bulk_wait_read<1>();
+          if constexpr ((EPI & E_GELU) != 0) {
+            // both buffers per chunk (pre-activation, GELU); the GELU is
+            // computed while the previous chunk's stores read shared memory
+            uint32_t hk[16], gk[16];
+            gelu_pack32(cur, hk, gk);
+            if (issued > 0) {
+              if (lane == 0) bulk_wait_read<0>();
+              __syncwarp();
+            }
+            stage_row64(stage0, lane, hk);
+            stage_row64(stage0 + 2048u, lane, gk);
+            fence_proxy_async_smem();
             __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(&p.tmO, stage0, n0 + c, m0);
+              tma_store_2d(&p.tmG, stage0 + 2048u, n0 + c, m0);
+            }
+            ++issued;
+          } else {
+            const uint32_t buf = stage0 + sbuf * 2048u;
+            if (issued >= 2) {   // buf's previous store is not the newest: at most one may still read
+              if (lane == 0) bulk_wait_read<1>();
+              __syncwarp();
+            }
+            tma_chunk32<EPI>(p, buf, lane, m0 + lane, n0 + c, cur);
+            __syncwarp();
+            if (lane == 0) tma_store_2d(&p.tmO, buf, n0 + c, m0);
+            ++issued;
+            sbuf ^= 1u;
           }
-          tma_chunk32<EPI>(p, buf, lane, m0 + lane, n0 + c, cur);
-          __syncwarp();
-          if (lane == 0) tma_store_2d(&p.tmO, buf, n0 + c, m0);
-          ++issued;
-          sbuf ^= 1u;
         }
         if (more) {
           tmem_ld32_wait(nxt);
