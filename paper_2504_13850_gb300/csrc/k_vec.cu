@@ -387,7 +387,7 @@ constexpr int kLnRows = 4;
 __device__ __forceinline__ float bf_at(const uint4& u, int j) {
   return __bfloat162float(reinterpret_cast<const bf16*>(&u)[j]);
 }
-template <int NX, int NV>
+template <int NX, int NV, int DXP>   // DXP: 0 no dx, 1 dx, 2 dx and its column partials (pdx)
 __global__ void __launch_bounds__(256, 1) layernorm_bwd_fused_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
                                                                 const float* __restrict__ mean, const float* __restrict__ rstd,
                                                                 const bf16* __restrict__ dy, bf16* dx, int64_t rows, int C,
@@ -395,7 +395,7 @@ __global__ void __launch_bounds__(256, 1) layernorm_bwd_fused_k(const bf16* __re
                                                                 float* __restrict__ pb, float* __restrict__ pdx) {
   pdl_wait();
   pdl_trigger();
-  constexpr int kMaxV = NV, nv = NV;   // 8-wide vectors per lane: C = 256 NV
+  constexpr int kMaxV = NV, nv = NV, CC = 256 * NV;   // 8-wide vectors per lane: C = 256 NV
   __shared__ __align__(16) float red[3][8][256 * NV];
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int64_t row0 = (int64_t(blockIdx.x) * 8 + warp) * kLnRows;
@@ -418,7 +418,7 @@ __global__ void __launch_bounds__(256, 1) layernorm_bwd_fused_k(const bf16* __re
 #pragma unroll
     for (int v = 0; v < kMaxV; ++v) {
       const bool ok = live && v < nv;
-      const int64_t off = row * C + (v * 32 + lane) * 8;
+      const int64_t off = row * CC + (v * 32 + lane) * 8;
       xr[r][v] = ok ? *reinterpret_cast<const uint4*>(x + off) : z;
       gr[r][v] = ok ? *reinterpret_cast<const uint4*>(dy + off) : z;
       if constexpr (NX > 0) er[r][v][0] = ok ? *reinterpret_cast<const uint4*>(ex0 + off) : z;
@@ -450,23 +450,24 @@ __global__ void __launch_bounds__(256, 1) layernorm_bwd_fused_k(const bf16* __re
       a += __shfl_xor_sync(0xffffffffu, a, o);
       b += __shfl_xor_sync(0xffffffffu, b, o);
     }
-    a /= float(C);
-    b /= float(C);
-    if (dx) {
+    a *= 1.f / float(CC);
+    b *= 1.f / float(CC);
+    if constexpr (DXP > 0) {
 #pragma unroll
       for (int v = 0; v < kMaxV; ++v) {
         if (v >= nv) break;
-        V8 o;
+        uint4 o;
+        bf16* ob = reinterpret_cast<bf16*>(&o);
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
           const float xh = (bf_at(xr[r][v], j) - mu[r]) * rs[r];
           float val = rs[r] * (bf_at(gr[r][v], j) * gm[v][j] - a - xh * b);
           if constexpr (NX > 0) val += bf_at(er[r][v][0], j);
           if constexpr (NX > 1) val += bf_at(er[r][v][1], j);
-          o.v[j] = val;
-          ax[v][j] += live ? __bfloat162float(__float2bfloat16_rn(val)) : 0.f;   // the stored value
+          ob[j] = __float2bfloat16_rn(val);
+          if constexpr (DXP == 2) ax[v][j] += live ? __bfloat162float(ob[j]) : 0.f;   // the stored value
         }
-        if (live) st8(dx + row * C + (v * 32 + lane) * 8, o);
+        if (live) *reinterpret_cast<uint4*>(dx + row * CC + (v * 32 + lane) * 8) = o;
       }
     }
   }
@@ -481,7 +482,7 @@ __global__ void __launch_bounds__(256, 1) layernorm_bwd_fused_k(const bf16* __re
     p0[1] = make_float4(ag[v][4], ag[v][5], ag[v][6], ag[v][7]);
     p1[0] = make_float4(ab[v][0], ab[v][1], ab[v][2], ab[v][3]);
     p1[1] = make_float4(ab[v][4], ab[v][5], ab[v][6], ab[v][7]);
-    if (pdx) {
+    if constexpr (DXP == 2) {
       p2[0] = make_float4(ax[v][0], ax[v][1], ax[v][2], ax[v][3]);
       p2[1] = make_float4(ax[v][4], ax[v][5], ax[v][6], ax[v][7]);
     }
@@ -493,11 +494,11 @@ __global__ void __launch_bounds__(256, 1) layernorm_bwd_fused_k(const bf16* __re
     for (int q = 0; q < 8; ++q) {
       tg += red[0][q][c];
       tb += red[1][q][c];
-      if (pdx) tx += red[2][q][c];
+      if constexpr (DXP == 2) tx += red[2][q][c];
     }
     pg[int64_t(blockIdx.x) * C + c] = tg;
     pb[int64_t(blockIdx.x) * C + c] = tb;
-    if (pdx) pdx[int64_t(blockIdx.x) * C + c] = tx;
+    if constexpr (DXP == 2) pdx[int64_t(blockIdx.x) * C + c] = tx;
   }
 }
 
@@ -771,8 +772,16 @@ void layernorm_bwd8_pass(const void* x, const float* gamma, const float* mean, c
   int nx = 0;
   if (dx && acc) ex[nx++] = static_cast<const bf16*>(dx);
   if (dx && addend) ex[nx++] = static_cast<const bf16*>(addend);
-  auto k = C <= 256 ? (nx == 0 ? layernorm_bwd_fused_k<0, 1> : nx == 1 ? layernorm_bwd_fused_k<1, 1> : layernorm_bwd_fused_k<2, 1>)
-                    : (nx == 0 ? layernorm_bwd_fused_k<0, 2> : nx == 1 ? layernorm_bwd_fused_k<1, 2> : layernorm_bwd_fused_k<2, 2>);
+  using K = decltype(&layernorm_bwd_fused_k<0, 1, 0>);
+  static const K table[2][3][3] = {   // [NV - 1][NX][DXP]; NX > 0 comes with a dx
+      {{layernorm_bwd_fused_k<0, 1, 0>, layernorm_bwd_fused_k<0, 1, 1>, layernorm_bwd_fused_k<0, 1, 2>},
+       {nullptr, layernorm_bwd_fused_k<1, 1, 1>, layernorm_bwd_fused_k<1, 1, 2>},
+       {nullptr, layernorm_bwd_fused_k<2, 1, 1>, layernorm_bwd_fused_k<2, 1, 2>}},
+      {{layernorm_bwd_fused_k<0, 2, 0>, layernorm_bwd_fused_k<0, 2, 1>, layernorm_bwd_fused_k<0, 2, 2>},
+       {nullptr, layernorm_bwd_fused_k<1, 2, 1>, layernorm_bwd_fused_k<1, 2, 2>},
+       {nullptr, layernorm_bwd_fused_k<2, 2, 1>, layernorm_bwd_fused_k<2, 2, 2>}}};
+  const int dxp = dx ? (p_dx ? 2 : 1) : 0;
+  auto k = table[C <= 256 ? 0 : 1][nx][dxp];
   launch_k(k, layernorm_bwd8_blocks(rows), 256, 0, st, (const bf16*)x, gamma, mean, rstd, (const bf16*)dy, (bf16*)dx,
            rows, C, ex[0], ex[1], p_gamma, p_beta, dx ? p_dx : nullptr);
 }
