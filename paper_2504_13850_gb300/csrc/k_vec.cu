@@ -311,12 +311,12 @@ __global__ void __launch_bounds__(256) colsum8_batch_k(const __grid_constant__ C
 
 // Layernorm forward, one warp per row held in registers (C = 256 NV,
 // NV <= 4, a template parameter so that a 512-column row takes only the
-// registers it needs and four blocks fit per SM): one read of x, mean then
+// registers it needs and three blocks fit per SM without spilling): one read of x, mean then
 // biased variance from the registers (eps 1e-5), one write of y; the row
 // mean and 1/std are kept for the backward pass.  gamma and beta are read as
 // float4 alongside x, so that the row's only dependent global access is x.
 template <int NV>
-__global__ void __launch_bounds__(256, NV <= 2 ? 4 : 2) layernorm_fwd_x8_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
+__global__ void __launch_bounds__(256, NV <= 2 ? 3 : 2) layernorm_fwd_x8_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
                                                           const float* __restrict__ beta, bf16* __restrict__ y,
                                                           float* __restrict__ mean_out, float* __restrict__ rstd_out,
                                                           int64_t rows, int C) {
