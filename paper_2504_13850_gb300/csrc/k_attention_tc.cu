@@ -89,7 +89,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_tc_k(const __grid_co
   char* sP = sm + 3 * kTile;                       // two sub-tiles (keys 0..63, 64..127)
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + 5 * kTile);   // ld, s, p, o
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 4);
-  float2* xch = reinterpret_cast<float2*>(sm + 5 * kTile + 64);   // [half][row]: partial (max, sum)
+  float2* xch = reinterpret_cast<float2*>(sm + 5 * kTile + 64);   // [half][row]: partial maxima, then sums
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int bh = blockIdx.x, b = bh / p.heads, h = bh % p.heads;
@@ -147,37 +147,23 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_tc_k(const __grid_co
     const int n = min(p.len[b], p.L);
     if (!mbar_wait(&bars[1], 0)) atomicExch(p.err, 13);
     tc_fence_after();
-    // one pass: running maximum and rescaled sum over this thread's keys
+    // the row maximum over this thread's keys, combined with the other half
     uint32_t r[32];
-    float m = -INFINITY, sum = 0.f;
+    float m = -INFINITY;
 #pragma unroll 1
     for (int c = 0; c < 2; ++c) {
       tmem_ld32(trow + 32 * c, r);
       const int j0 = 64 * hf + 32 * c;
-      float cm = -INFINITY;
 #pragma unroll
       for (int e = 0; e < 32; ++e)
-        if (j0 + e < n) cm = fmaxf(cm, __uint_as_float(r[e]) * kScale);
-      const float mn = fmaxf(m, cm);
-      if (mn > -INFINITY) {
-        sum = m > -INFINITY ? sum * __expf(m - mn) : 0.f;
-#pragma unroll
-        for (int e = 0; e < 32; ++e)
-          if (j0 + e < n) sum += __expf(__uint_as_float(r[e]) * kScale - mn);
-        m = mn;
-      }
+        if (j0 + e < n) m = fmaxf(m, __uint_as_float(r[e]) * kScale);
     }
-    // combine with the other half of the row
-    xch[hf * 128 + i] = make_float2(m, sum);
+    xch[hf * 128 + i] = make_float2(m, 0.f);
     asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
-    const float2 o2 = xch[(1 - hf) * 128 + i];
-    const float M = fmaxf(m, o2.x);
-    float S = 0.f;
-    if (M > -INFINITY) {
-      if (m > -INFINITY) S += sum * __expf(m - M);
-      if (o2.x > -INFINITY) S += o2.y * __expf(o2.x - M);
-    }
-    const float inv = S > 0.f ? 1.f / S : 0.f;
+    const float M = fmaxf(m, xch[(1 - hf) * 128 + i].x);
+    // P~ = exp(s / 8 - M) (bf16, unnormalised: one exponential per score) and
+    // its row sum; O = P~ V is normalised by the sum in the store below
+    float sum = 0.f;
     const uint32_t p_base = smem_u32(sP) + uint32_t(hf) * kTile;
 #pragma unroll 1
     for (int c = 0; c < 2; ++c) {
@@ -188,20 +174,28 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_tc_k(const __grid_co
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
           const int j = 64 * hf + 32 * c + 8 * g + e;
-          v[e] = j < n ? __expf(__uint_as_float(r[8 * g + e]) * kScale - M) * inv : 0.f;
+          v[e] = j < n ? __expf(__uint_as_float(r[8 * g + e]) * kScale - M) : 0.f;
+          sum += v[e];
         }
         st_shared4(p_base + sw_off(i, c * 4 + g), pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
                    pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
       }
     }
-    if (hf == 0 && i < p.L) p.lse[size_t(bh) * p.L + i] = M + logf(S);
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // P visible to the tensor cores
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // P~ visible to the tensor cores
     tc_fence_before();
     mbar_arrive(&bars[2]);
+    // the row sum over both halves, while the tensor cores form O
+    xch[256 + hf * 128 + i] = make_float2(sum, 0.f);
+    asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
+    const float S = sum + xch[256 + (1 - hf) * 128 + i].x;
+    const float inv = S > 0.f ? 1.f / S : 0.f;
+    if (hf == 0 && i < p.L) p.lse[size_t(bh) * p.L + i] = M + logf(S);
     if (!mbar_wait(&bars[3], 0)) atomicExch(p.err, 14);
     tc_fence_after();
     // O: 64 columns at TMEM column 128; each half of the pair stores 32
     tmem_ld32(tmem + (uint32_t(q * 32) << 16) + 128 + 32 * hf, r);
+#pragma unroll
+    for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * inv);
     if (i < p.L) store_row32(p.out + size_t(row0 + i) * p.C + h * 64 + 32 * hf, r, false);
   }
   tc_fence_before();
@@ -374,7 +368,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_bwd_tc_k(const __grid_co
   }
 }
 
-constexpr size_t kFwdSmem = 5 * kTile + 1024 + 64 + 2 * 128 * sizeof(float2);
+constexpr size_t kFwdSmem = 5 * kTile + 1024 + 64 + 4 * 128 * sizeof(float2);
 constexpr size_t kBwdSmem = 7 * kTile + 1024;   // 115,712 B: two CTAs in an SM's 228 KB
 
 }  // namespace
