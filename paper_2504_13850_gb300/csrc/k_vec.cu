@@ -309,66 +309,78 @@ __global__ void __launch_bounds__(256) colsum8_batch_k(const __grid_constant__ C
                    local % cbs, local / cbs);
 }
 
-// Layernorm forward, one warp per row held in registers (C = 256 NV,
-// NV <= 4, a template parameter so that a 512-column row takes only the
-// registers it needs and three blocks fit per SM without spilling): one read of x, mean then
-// biased variance from the registers (eps 1e-5), one write of y; the row
-// mean and 1/std are kept for the backward pass.  gamma and beta are read as
-// float4 alongside x, so that the row's only dependent global access is x.
-template <int NV>
-__global__ void __launch_bounds__(256, NV <= 2 ? 3 : 2) layernorm_fwd_x8_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
+// Layernorm forward, rows held in registers (C = 256 NV, NV <= 4, a
+// template parameter so that a row takes only the registers it needs): each
+// warp takes R consecutive rows and loads all of them before any
+// arithmetic; one read of x, mean then biased variance from the registers
+// (eps 1e-5), one write of y; the row mean and 1/std are kept for the
+// backward pass.  gamma and beta are read as float4 alongside x, so that the
+// rows' only dependent global accesses are x.  R = 2 for rows of up to 512
+// (the whole 4096-row step in one wave of two blocks per SM).
+template <int NV, int R>
+__global__ void __launch_bounds__(256, 2) layernorm_fwd_x8_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
                                                           const float* __restrict__ beta, bf16* __restrict__ y,
                                                           float* __restrict__ mean_out, float* __restrict__ rstd_out,
                                                           int64_t rows, int C) {
   pdl_wait();
   pdl_trigger();
   const int lane = threadIdx.x % 32;
-  const int64_t row = int64_t(blockIdx.x) * (blockDim.x / 32) + threadIdx.x / 32;
-  if (row >= rows) return;
-  uint4 xr[NV];
+  const int64_t row0 = (int64_t(blockIdx.x) * (blockDim.x / 32) + threadIdx.x / 32) * R;
+  if (row0 >= rows) return;
+  uint4 xr[R][NV];
   float4 g4[NV][2], b4[NV][2];
+#pragma unroll
+  for (int r = 0; r < R; ++r)
+#pragma unroll
+    for (int v = 0; v < NV; ++v)
+      xr[r][v] = row0 + r < rows ? *reinterpret_cast<const uint4*>(x + (row0 + r) * C + (v * 32 + lane) * 8)
+                                 : make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
   for (int v = 0; v < NV; ++v) {
     const int c = (v * 32 + lane) * 8;
-    xr[v] = *reinterpret_cast<const uint4*>(x + row * C + c);
     g4[v][0] = __ldg(reinterpret_cast<const float4*>(gamma + c));
     g4[v][1] = __ldg(reinterpret_cast<const float4*>(gamma + c) + 1);
     b4[v][0] = __ldg(reinterpret_cast<const float4*>(beta + c));
     b4[v][1] = __ldg(reinterpret_cast<const float4*>(beta + c) + 1);
   }
-  float sum = 0.f;
 #pragma unroll
-  for (int v = 0; v < NV; ++v)
+  for (int r = 0; r < R; ++r) {
+    const int64_t row = row0 + r;
+    if (row >= rows) break;
+    float sum = 0.f;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) sum += __bfloat162float(reinterpret_cast<const bf16*>(&xr[v])[j]);
+    for (int v = 0; v < NV; ++v)
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-  const float mu = sum / float(C);
-  float q = 0.f;
+      for (int j = 0; j < 8; ++j) sum += __bfloat162float(reinterpret_cast<const bf16*>(&xr[r][v])[j]);
 #pragma unroll
-  for (int v = 0; v < NV; ++v)
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    const float mu = sum / float(C);
+    float q = 0.f;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const float d = __bfloat162float(reinterpret_cast<const bf16*>(&xr[v])[j]) - mu;
-      q = fmaf(d, d, q);
+    for (int v = 0; v < NV; ++v)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float d = __bfloat162float(reinterpret_cast<const bf16*>(&xr[r][v])[j]) - mu;
+        q = fmaf(d, d, q);
+      }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+    const float rs = rsqrtf(q / float(C) + 1e-5f);
+#pragma unroll
+    for (int v = 0; v < NV; ++v) {
+      const int c = (v * 32 + lane) * 8;
+      const float gm[8] = {g4[v][0].x, g4[v][0].y, g4[v][0].z, g4[v][0].w, g4[v][1].x, g4[v][1].y, g4[v][1].z, g4[v][1].w};
+      const float bt[8] = {b4[v][0].x, b4[v][0].y, b4[v][0].z, b4[v][0].w, b4[v][1].x, b4[v][1].y, b4[v][1].z, b4[v][1].w};
+      V8 o;
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        o.v[j] = (__bfloat162float(reinterpret_cast<const bf16*>(&xr[r][v])[j]) - mu) * rs * gm[j] + bt[j];
+      st8(y + row * C + c, o);
     }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
-  const float rs = rsqrtf(q / float(C) + 1e-5f);
-#pragma unroll
-  for (int v = 0; v < NV; ++v) {
-    const int c = (v * 32 + lane) * 8;
-    const float gm[8] = {g4[v][0].x, g4[v][0].y, g4[v][0].z, g4[v][0].w, g4[v][1].x, g4[v][1].y, g4[v][1].z, g4[v][1].w};
-    const float bt[8] = {b4[v][0].x, b4[v][0].y, b4[v][0].z, b4[v][0].w, b4[v][1].x, b4[v][1].y, b4[v][1].z, b4[v][1].w};
-    V8 o;
-#pragma unroll
-    for (int j = 0; j < 8; ++j)
-      o.v[j] = (__bfloat162float(reinterpret_cast<const bf16*>(&xr[v])[j]) - mu) * rs * gm[j] + bt[j];
-    st8(y + row * C + c, o);
-  }
-  if (lane == 0) {
-    mean_out[row] = mu;
-    rstd_out[row] = rs;
+    if (lane == 0) {
+      mean_out[row] = mu;
+      rstd_out[row] = rs;
+    }
   }
 }
 
@@ -760,8 +772,12 @@ int layernorm_bwd8_blocks(int64_t rows) { return int((rows + 8 * kLnRows - 1) / 
 bool layernorm_fwd8_ok(int dt, int C) { return dt == kBF16 && C % 256 == 0 && C <= 1024; }
 void layernorm_fwd_x8(const void* x, const float* gamma, const float* beta, void* y, float* mean, float* rstd,
                       int64_t rows, int C, cudaStream_t st) {
-  auto k = C <= 256 ? layernorm_fwd_x8_k<1> : C <= 512 ? layernorm_fwd_x8_k<2> : C <= 768 ? layernorm_fwd_x8_k<3>
-                                                                               : layernorm_fwd_x8_k<4>;
+  if (C <= 512) {
+    auto k = C <= 256 ? layernorm_fwd_x8_k<1, 2> : layernorm_fwd_x8_k<2, 2>;
+    launch_k(k, ceil_div(rows, 16), 256, 0, st, (const bf16*)x, gamma, beta, (bf16*)y, mean, rstd, rows, C);
+    return;
+  }
+  auto k = C <= 768 ? layernorm_fwd_x8_k<3, 1> : layernorm_fwd_x8_k<4, 1>;
   launch_k(k, ceil_div(rows, 8), 256, 0, st, (const bf16*)x, gamma, beta, (bf16*)y, mean, rstd, rows, C);
 }
 
