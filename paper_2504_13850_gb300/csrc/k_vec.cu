@@ -385,10 +385,10 @@ __global__ void __launch_bounds__(256, 2) layernorm_fwd_x8_k(const bf16* __restr
 }
 
 // Layernorm backward fused with its parameter gradients.  Each warp takes
-// kLnRows consecutive rows (a block 8 kLnRows), with all of their operands
+// kLnRows consecutive rows (a block kLnWarps kLnRows), with all of their operands
 // loaded before any arithmetic.  The column partials of dy * xhat (gamma),
 // dy (beta) and, with pdx, of the stored dx accumulate in registers over the
-// warp's rows and are added over the block's 8 warps, in warp order, through
+// warp's rows and are added over the block's warps, in warp order, through
 // shared memory once per block: exchanged row by row, those partials cost
 // more than the rest of the pass.  C <= 512, C % 256 == 0; dx may be null (a
 // layernorm of the uploaded batch has no input gradient).  dx receives the
@@ -396,11 +396,12 @@ __global__ void __launch_bounds__(256, 2) layernorm_fwd_x8_k(const bf16* __restr
 // layout): its own old value when accumulating, and the gradient a residual
 // connection passes around the layernorm.
 constexpr int kLnRows = 4;
+constexpr int kLnWarps = 4;   // warps per block: the 4096-row step in 256 blocks
 __device__ __forceinline__ float bf_at(const uint4& u, int j) {
   return __bfloat162float(reinterpret_cast<const bf16*>(&u)[j]);
 }
 template <int NX, int NV, int DXP>   // DXP: 0 no dx, 1 dx, 2 dx and its column partials (pdx)
-__global__ void __launch_bounds__(256, 1) layernorm_bwd_fused_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
+__global__ void __launch_bounds__(kLnWarps * 32, 1) layernorm_bwd_fused_k(const bf16* __restrict__ x, const float* __restrict__ gamma,
                                                                 const float* __restrict__ mean, const float* __restrict__ rstd,
                                                                 const bf16* __restrict__ dy, bf16* dx, int64_t rows, int C,
                                                                 const bf16* ex0, const bf16* ex1, float* __restrict__ pg,
@@ -408,9 +409,9 @@ __global__ void __launch_bounds__(256, 1) layernorm_bwd_fused_k(const bf16* __re
   pdl_wait();
   pdl_trigger();
   constexpr int kMaxV = NV, nv = NV, CC = 256 * NV;   // 8-wide vectors per lane: C = 256 NV
-  __shared__ __align__(16) float red[3][8][256 * NV];
+  __shared__ __align__(16) float red[3][kLnWarps][256 * NV];
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int64_t row0 = (int64_t(blockIdx.x) * 8 + warp) * kLnRows;
+  const int64_t row0 = (int64_t(blockIdx.x) * kLnWarps + warp) * kLnRows;
   const uint4 z = make_uint4(0u, 0u, 0u, 0u);
   float gm[kMaxV][8];
 #pragma unroll
@@ -503,7 +504,7 @@ __global__ void __launch_bounds__(256, 1) layernorm_bwd_fused_k(const bf16* __re
   for (int c = threadIdx.x; c < C; c += blockDim.x) {
     float tg = 0.f, tb = 0.f, tx = 0.f;
 #pragma unroll
-    for (int q = 0; q < 8; ++q) {
+    for (int q = 0; q < kLnWarps; ++q) {
       tg += red[0][q][c];
       tb += red[1][q][c];
       if constexpr (DXP == 2) tx += red[2][q][c];
@@ -767,7 +768,7 @@ void finish_batched(const std::vector<FinishTask>& tasks, cudaStream_t st) {
 
 bool layernorm_bwd8_ok(int dt, int C) { return dt == kBF16 && C % 256 == 0 && C <= 512; }
 
-int layernorm_bwd8_blocks(int64_t rows) { return int((rows + 8 * kLnRows - 1) / (8 * kLnRows)); }
+int layernorm_bwd8_blocks(int64_t rows) { return int((rows + kLnWarps * kLnRows - 1) / (kLnWarps * kLnRows)); }
 
 bool layernorm_fwd8_ok(int dt, int C) { return dt == kBF16 && C % 256 == 0 && C <= 1024; }
 void layernorm_fwd_x8(const void* x, const float* gamma, const float* beta, void* y, float* mean, float* rstd,
@@ -798,7 +799,7 @@ void layernorm_bwd8_pass(const void* x, const float* gamma, const float* mean, c
        {nullptr, layernorm_bwd_fused_k<2, 2, 1>, layernorm_bwd_fused_k<2, 2, 2>}}};
   const int dxp = dx ? (p_dx ? 2 : 1) : 0;
   auto k = table[C <= 256 ? 0 : 1][nx][dxp];
-  launch_k(k, layernorm_bwd8_blocks(rows), 256, 0, st, (const bf16*)x, gamma, mean, rstd, (const bf16*)dy, (bf16*)dx,
+  launch_k(k, layernorm_bwd8_blocks(rows), kLnWarps * 32, 0, st, (const bf16*)x, gamma, mean, rstd, (const bf16*)dy, (bf16*)dx,
            rows, C, ex[0], ex[1], p_gamma, p_beta, dx ? p_dx : nullptr);
 }
 
