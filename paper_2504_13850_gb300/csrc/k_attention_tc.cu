@@ -2,8 +2,9 @@
 // head width 64 (bf16 activations): one CTA per (sequence, head), the whole
 // 128 x 128 score tile in TMEM.  Same operation as the CUDA-core kernels
 // (scaled dot-product attention with keys j >= length[b] masked out):
-//   forward   S = Q K^T (TMEM) -> row softmax of S / sqrt(64) -> P (bf16,
-//             shared memory) -> O = P V (TMEM) -> O (bf16), plus the row
+//   forward   S = Q K^T (TMEM) -> row maximum M of S / sqrt(64) -> P~ =
+//             exp(S / 8 - M) (bf16, shared memory) and its row sum ->
+//             O = P~ V (TMEM) -> O / row sum (bf16), plus the row
 //             log-sum-exp of the scaled scores for the backward pass;
 //   backward  S = Q K^T and dP = dO V^T (TMEM) -> P = exp(S / 8 - lse),
 //             dS = P (dP - rowsum(dO * O)) / 8 (bf16, shared memory) ->
@@ -11,7 +12,7 @@
 // Operand tiles are 128 rows x 64 bf16 (128-byte rows, 128-byte swizzle),
 // loaded by TMA from the packed q|k|v [B*L, 3C] and dO [B*L, C] (the
 // backward reads O's rows directly for rowsum(dO * O));
-// P and dS are written by the softmax threads in the same swizzled layout as
+// P (P~ in the forward) and dS are written by the softmax threads in the same swizzled layout as
 // two 64-column sub-tiles, which serves both as a K-major operand (P V,
 // dS K) and as an MN-major one (P^T dO, dS^T Q).
 // Warp roles: warp 0 issues the TMA loads, warp 1 owns TMEM and issues the
