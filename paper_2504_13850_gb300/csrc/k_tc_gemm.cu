@@ -230,15 +230,18 @@ int active_clusters(TcContext* c, int kind, int bn, int S, int epi) {
 //    staging and distributed-shared-memory reduction of its partial tiles,
 //    and clusters run in waves of what the occupancy calculator fits at once.
 // Candidate widths divide `ndiv` (N, or the channels of one tap for the
-// weight gradient, whose N index runs over taps x channels).
+// weight gradient, whose N index runs over taps x channels); a weight-gradient
+// tile may instead span whole taps, one TMA box per tap.
 void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv) {
   const bool win_a = g->kind == CONV_FPROP || g->kind == CONV_DGRAD;
   const bool win_b = g->kind == CONV_WGRAD;
   double best = 1e30;
   int best_bn = 0, best_s = 1;
   for (int bn : {256, 128, 64}) {
-    // window kinds tile whole taps; the plain GEMMs take a ragged last tile
-    if ((win_a || win_b) && (ndiv % bn || N % bn)) continue;
+    // window kinds tile whole taps; the plain GEMMs take a ragged last tile,
+    // and so does a weight gradient whose tiles span taps
+    if (win_a && (ndiv % bn || N % bn)) continue;
+    if (win_b && ndiv % bn && bn % ndiv) continue;
     const int n_tiles = (N + bn - 1) / bn, m_tiles = (M + BM - 1) / BM, tiles = n_tiles * m_tiles;
     const double stage_kb = (BM + bn) * BK * 2 / 1024.0;
     const double epi = bn == 256 ? 4.2 : (bn == 128 ? 2.2 : 1.5);
@@ -619,7 +622,7 @@ TcGemm* tc_plan_wgrad(TcContext* c, fo_server* s, int i) {
   if (!map_2d(&g->p.tmA, o.grad, P, op.cout, BK)) { delete g; return nullptr; }
   CUtensorMap ca;
   if (map_chunked(&ca, o.grad, P, op.cout, BK, BM / 64)) { g->p.tmA = ca; g->p.chunk_a = 1; }
-  const int nchunk = g->bn / 64;
+  const int nchunk = std::min(g->bn, op.cin) / 64;   // channel chunks per box (one box per tap)
   g->p.chunk_b = 1;
   auto map_b = [&](CUtensorMap* m, const void* base) {
     if (g->p.chunk_b && map_window_chunked(m, base, a.N, a.H, a.W, a.C, Wo, rows, imgs, st, nchunk)) return true;

@@ -416,20 +416,28 @@ __device__ __forceinline__ void load_kblock(const TcParams& p, int kb, int m0, i
     else
 #pragma unroll
       for (int j = 0; j < BN / 64; ++j) tma_2d(sb + j * BK * 128, &p.tmB, bar, tap * p.ntap_ch + n0 + j * 64, co0);
-  } else if (p.chunk_b) {  // CONV_WGRAD, all chunks of the tile in one box
-    const int tap = n0 / p.ntap_ch, ci0 = n0 % p.ntap_ch;
-    const int r = tap / p.ksz, s = tap % p.ksz;
+  } else if (p.chunk_b) {  // CONV_WGRAD: the tile's channel chunks in one box per tap
+    // (a tile wider than Ci spans BN / Ci taps; a ragged last tile's tap past
+    // the last one loads a shifted window whose columns the epilogue drops)
+    const int cw = BN < p.ntap_ch ? BN : p.ntap_ch;
     const int pix0 = kb * BK;
     const int n_img = pix0 / HW, h0 = (pix0 % HW) / p.W;
-    tma_5d(sb, &p.tmB, bar, 0, s - p.pad, h0 * p.stride + r - p.pad, n_img, ci0 / 64);
+    for (int t = 0; t * cw < BN; ++t) {
+      const int nn = n0 + t * cw;
+      const int tap = nn / p.ntap_ch, ci0 = nn % p.ntap_ch;
+      const int r = tap / p.ksz, s = tap % p.ksz;
+      tma_5d(sb + t * (cw / 64) * BK * 128, &p.tmB, bar, 0, s - p.pad, h0 * p.stride + r - p.pad, n_img, ci0 / 64);
+    }
   } else {  // CONV_WGRAD: N index = tap * Ci + ci; K = output pixel
-    const int tap = n0 / p.ntap_ch, ci0 = n0 % p.ntap_ch;
-    const int r = tap / p.ksz, s = tap % p.ksz;
     const int pix0 = kb * BK;
     const int n_img = pix0 / HW, h0 = (pix0 % HW) / p.W;   // H, W: output grid
 #pragma unroll
-    for (int j = 0; j < BN / 64; ++j)
-      tma_4d(sb + j * BK * 128, &p.tmB, bar, ci0 + j * 64, s - p.pad, h0 * p.stride + r - p.pad, n_img);
+    for (int j = 0; j < BN / 64; ++j) {
+      const int nn = n0 + j * 64;
+      const int tap = nn / p.ntap_ch, ci = nn % p.ntap_ch;
+      const int r = tap / p.ksz, s = tap % p.ksz;
+      tma_4d(sb + j * BK * 128, &p.tmB, bar, ci, s - p.pad, h0 * p.stride + r - p.pad, n_img);
+    }
   }
 }
 
