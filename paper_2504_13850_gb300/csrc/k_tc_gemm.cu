@@ -231,7 +231,7 @@ int active_clusters(TcContext* c, int kind, int bn, int S, int epi) {
 //    and clusters run in waves of what the occupancy calculator fits at once.
 // Candidate widths divide `ndiv` (N, or the channels of one tap for the
 // weight gradient, whose N index runs over taps x channels); a weight-gradient
-// tile may instead span whole taps, one TMA box per tap.
+// tile may instead span two whole taps, one TMA box per tap.
 void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv) {
   const bool win_a = g->kind == CONV_FPROP || g->kind == CONV_DGRAD;
   const bool win_b = g->kind == CONV_WGRAD;
@@ -239,9 +239,9 @@ void choose_tiles(TcContext* c, TcGemm* g, int M, int N, int KB, int ndiv) {
   int best_bn = 0, best_s = 1;
   for (int bn : {256, 128, 64}) {
     // window kinds tile whole taps; the plain GEMMs take a ragged last tile,
-    // and so does a weight gradient whose tiles span taps
+    // and so does a weight gradient whose tiles span (at most two) taps
     if (win_a && (ndiv % bn || N % bn)) continue;
-    if (win_b && ndiv % bn && bn % ndiv) continue;
+    if (win_b && ndiv % bn && (bn % ndiv || bn > 2 * ndiv)) continue;
     const int n_tiles = (N + bn - 1) / bn, m_tiles = (M + BM - 1) / BM, tiles = n_tiles * m_tiles;
     const double stage_kb = (BM + bn) * BK * 2 / 1024.0;
     const double epi = bn == 256 ? 4.2 : (bn == 128 ? 2.2 : 1.5);
