@@ -85,10 +85,14 @@ def test_gelu_forward_is_the_rounded_exact_value(width):
     check_teacher_forced(recs)
 
 
-def test_gelu_backward_teacher_forced_bf16():
-    cfg = gelu_cfg(W.BF16)
+@pytest.mark.parametrize("width", [512, 520])
+def test_gelu_backward_teacher_forced_bf16(width):
+    """520 columns: a ragged last output tile in the linear layers on both
+    sides of the GELU, and a bias gradient whose last 256-column block of
+    the column sums holds one 8-column group."""
+    cfg = gelu_cfg(W.BF16, width)
     ev = [("enq", k) for _ in range(2) for k in range(2)] + [("step",)] * 4
-    _, _, recs = teacher_forced(cfg, ev, theta0=wide_theta(cfg))
+    _, _, recs = teacher_forced(cfg, ev, theta0=wide_theta(cfg, width))
     assert len(recs) == 4
     check_teacher_forced(recs)
 
