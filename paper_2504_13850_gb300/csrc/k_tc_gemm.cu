@@ -223,12 +223,13 @@ int active_clusters(TcContext* c, int kind, int bn, int S, int epi) {
 //  * a stage issues four 128 x BN x 16 MMAs, and each takes ~190 cycles
 //    whatever BN <= 256 (measured: 128- and 256-wide weight-gradient stages
 //    both ~0.38-0.40 us once all chunks of an operand come in one TMA box),
-//    so 256-wide tiles run at ~3/4 of the MMA peak and 128-wide ones at
-//    ~3/8: the floor above;
+//    so 256-wide tiles run at the measured dense bf16 rate (about 3/4 of
+//    the nominal one) and 128-wide ones at half of it: the floor above;
 //  * a CTA pays a start-up ramp and the epilogue of its last tile (earlier
 //    epilogues overlap the next tile's MMAs), a K-split cluster pays the
-//    staging and distributed-shared-memory reduction of its partial tiles,
-//    and clusters run in waves of what the occupancy calculator fits at once.
+//    exchange of its partial tiles through the L2 workspace and their
+//    reduction, and clusters run in waves of what the occupancy calculator
+//    fits at once.
 // Candidate widths divide `ndiv` (N, or the channels of one tap for the
 // weight gradient, whose N index runs over taps x channels); a weight-gradient
 // tile may instead span two whole taps, one TMA box per tap.
