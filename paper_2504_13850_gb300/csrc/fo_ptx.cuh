@@ -1,8 +1,8 @@
 // Inline-PTX building blocks of the tcgen05 kernels (sm_103a): mbarriers with
 // bounded waits, TMA tensor copies,
 // shared-memory matrix descriptors for 128-byte-swizzled tiles, tcgen05 MMA
-// issue / commit / TMEM loads, and cluster (distributed shared memory)
-// access.  Shared by the GEMM and attention kernels.
+// issue / commit / TMEM loads and stores, TMA stores, and the cluster
+// barrier of the split-K GEMM.  Shared by the GEMM and attention kernels.
 #pragma once
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -114,31 +114,9 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                : "memory");
 }
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
 
 __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
-}
-__device__ __forceinline__ uint32_t map_to_cta(uint32_t smem_addr, uint32_t cta) {
-  uint32_t r;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr), "r"(cta));
-  return r;
-}
-// Read of another CTA's shared memory; ordered by the cluster barriers
-// around the reduction (no memory clobber, so loads can overlap).
-__device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr) {
-  float4 v;
-  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "r"(addr));
-  return v;
 }
 
 
@@ -224,36 +202,6 @@ __device__ __forceinline__ float4 ld_shared4(uint32_t addr) {
   asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr)
                : "memory");
   return v;
-}
-
-
-// Plain 16-byte store into another CTA's shared memory (shared::cluster
-// address from mapa).
-__device__ __forceinline__ void st_cluster4(uint32_t remote_addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
-  asm volatile("st.shared::cluster.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(remote_addr), "r"(a), "r"(b), "r"(c), "r"(d)
-               : "memory");
-}
-// Arrive on another CTA's mbarrier, releasing this thread's earlier writes at
-// cluster scope.
-__device__ __forceinline__ void mbar_arrive_remote(uint32_t remote_bar) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote_bar) : "memory");
-}
-// Wait (bounded, ~2 s) for a phase whose arrivals came from other CTAs of the
-// cluster: acquire at cluster scope.
-__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity) {
-  const uint64_t t0 = global_ns();
-  while (true) {
-    for (int i = 0; i < 64; ++i) {
-      uint32_t ok;
-      asm volatile(
-          "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
-          : "=r"(ok)
-          : "r"(smem_u32(bar)), "r"(parity)
-          : "memory");
-      if (ok) return true;
-    }
-    if (global_ns() - t0 > 2000000000ull) return false;
-  }
 }
 
 }  // namespace
