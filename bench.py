@@ -557,7 +557,8 @@ def run_ours(args):
                    "l2": f"not flushed: each step touches the server's {wsb / 1e6:.0f} MB of parameters, "
                          f"momentum, gradients, activations and scratch, above the 126 MB L2",
                    "switches": {k: os.environ.get(k) for k in ("FO_NO_TC", "FO_NO_GRAPH", "FO_NO_SIDE", "FO_NO_PDL",
-                                                                "FO_NO_POOL_EPILOGUE")}},
+                                                                "FO_NO_POOL_EPILOGUE", "FO_NO_TMA_STORE",
+                                                                "FO_NO_GELU_EPILOGUE")}},
         "e2e": e2e,
         "gpu_launches": int(launches),
         "roofline": roof,
