@@ -122,6 +122,54 @@ def attention_bwd_no_rowsum(cache, dout, d, heads):
     return np.concatenate([merge(dq), merge(dk), merge(dv)], -1).reshape(B, L, 1, 3 * d)
 
 
+def layernorm_eps_on_std(x, gamma, beta):
+    mu = x.mean(-1, keepdims=True)
+    var = ((x - mu) ** 2).mean(-1, keepdims=True)
+    rstd = 1.0 / (np.sqrt(var) + O.LN_EPS)
+    xhat = (x - mu) * rstd
+    return xhat * gamma + beta, (xhat, rstd)
+
+
+def gelu_bwd_no_density_term(x, dy):
+    return dy * ORIG["gelu_fwd"](x) / np.where(x == 0.0, 1.0, x)
+
+
+def attention_causal(qkv, lengths, d, heads):
+    """Each query also sees only the keys up to its own position."""
+    B, L = qkv.shape[0], qkv.shape[1]
+    dh = d // heads
+    t = qkv.reshape(B, L, 3 * d)
+    q = O._split_heads(t[..., :d], B, L, heads, dh)
+    k = O._split_heads(t[..., d:2 * d], B, L, heads, dh)
+    v = O._split_heads(t[..., 2 * d:], B, L, heads, dh)
+    s = q @ k.transpose(0, 1, 3, 2) / np.sqrt(dh)
+    valid = np.arange(L)[None, :] < np.asarray(lengths)[:, None]
+    keep = valid[:, None, None, :] & (np.arange(L)[None, None, None, :] <= np.arange(L)[None, None, :, None])
+    s = np.where(keep, s, -np.inf)
+    p = np.exp(s - s.max(-1, keepdims=True))
+    p = p / p.sum(-1, keepdims=True)
+    out = (p @ v).transpose(0, 2, 1, 3).reshape(B, L, 1, d)
+    return out, (q, k, v, p)
+
+
+def attention_interleaved_heads(qkv, lengths, d, heads):
+    """Head h takes channels h, h + heads, h + 2 heads, ... instead of a block."""
+    dh = d // heads
+    perm = np.array([j * heads + hh for hh in range(heads) for j in range(dh)])
+    full = np.concatenate([perm, perm + d, perm + 2 * d])
+    out_p, cache = ORIG["attention_fwd"](qkv[..., full], lengths, d, heads)
+    out = np.empty_like(out_p)
+    out[..., perm] = out_p
+    return out, cache
+
+
+def meanpool_bwd_not_averaged(x, lengths, dy):
+    dx = np.zeros_like(x)
+    for b in range(x.shape[0]):
+        dx[b, :lengths[b], 0, :] = dy[b]
+    return dx
+
+
 def meanpool_over_all(x, lengths):
     return x[:, :, 0, :].mean(1)
 
@@ -387,6 +435,16 @@ MUTATIONS = {
         {"attention_fwd": attention_unmasked}, [(TL.test_attention_special_cases, ())]),
     "attention backward: softmax row-sum term dropped": (
         {"attention_bwd": attention_bwd_no_rowsum}, [(TL.test_attention_fd, ())]),
+    "layernorm: eps added to the standard deviation": (
+        {"layernorm_fwd": layernorm_eps_on_std}, [(TL.test_layernorm_invariants_and_fd, ())]),
+    "GELU backward: the x phi(x) term dropped": (
+        {"gelu_bwd": gelu_bwd_no_density_term}, [(TL.test_gelu_values_and_fd, ())]),
+    "attention: a causal mask on top of the key mask": (
+        {"attention_fwd": attention_causal}, [(TL.test_attention_special_cases, ())]),
+    "attention: heads take interleaved channels": (
+        {"attention_fwd": attention_interleaved_heads}, [(TL.test_attention_brute_force_one_row, ())]),
+    "mean-pool backward: not divided by the length": (
+        {"meanpool_bwd": meanpool_bwd_not_averaged}, [(TL.test_meanpool, ())]),
     "mean-pool over padded tokens": (
         {"meanpool_fwd": meanpool_over_all}, [(TL.test_meanpool, ())]),
     "average-pool backward: 1/(H W) dropped": (
