@@ -180,6 +180,23 @@ def sum_over_ranks(world, value, device):
     return float(t.item())
 
 
+POOL = 8   # uploaded batches resident on the device, cycled through by the steps
+
+
+def valid_token_frac(cfg, pool=POOL):
+    """Share of the padded token positions that hold real tokens over the
+    resident batches the steps cycle through (sequence workloads; None for
+    the others).  The dense linear layers work on every position; only this
+    share of that work falls on tokens of the sequences."""
+    if not cfg["seq"]:
+        return None
+    import numpy as np
+
+    from paper_2504_13850_gb300 import workloads as W
+    lengths = np.concatenate([W.device_batch(cfg, j % cfg["K"], 10_000 + j)[3] for j in range(pool)])
+    return round(float(lengths.mean()) / cfg["in_hwc"][0], 4)
+
+
 def oracle_samples_per_s(cfg, n_steps, batch):
     """The oracle as it stands, timed on this host's cores: n_steps server
     steps at `batch` samples each (a bounded sample of the workload)."""
@@ -261,7 +278,7 @@ class Harness:
         self.srv = api.Server.from_config(cfg)
         self.srv.set_params(W.init_params(cfg))
         self.stream = torch.cuda.ExternalStream(self.srv.stream(), device=dev)
-        P = 8   # resident uploaded batches
+        P = POOL
         self.pool = []
         for j in range(P):
             x, bits, labels, lengths = W.device_batch(cfg, j % cfg["K"], 10_000 + j)
@@ -565,6 +582,7 @@ def run_ours(args):
         "step_tensor_frac": round(tensor_frac, 4),
         "step_tensor_frac_burst": round(tensor_frac_burst, 4),
         "step_gflop": round(step_flops / 1e9, 2),
+        "valid_token_frac": valid_token_frac(cfg),
         "server_busy": busy,
         "workloads": others or None,
         "aggregation": agg,
