@@ -275,6 +275,10 @@ def test_ce_fd_and_shift_invariance():
     labels = np.array([1, 4, 0])
     loss, dz = O.softmax_ce(z, labels)
     assert math.isclose(O.softmax_ce(z + 7.0, labels)[0], loss, rel_tol=1e-12)
+    # logits far beyond exp's range: the loss and its gradient are unchanged
+    # (a softmax that does not subtract the row maximum overflows here)
+    lz, dzz = O.softmax_ce(z + 1000.0, labels)
+    assert math.isclose(lz, loss, rel_tol=1e-9) and np.allclose(dzz, dz, rtol=1e-9, atol=1e-15)
     brute = np.mean([math.log(sum(math.exp(v) for v in z[b])) - z[b, labels[b]] for b in range(3)])
     assert math.isclose(loss, brute, rel_tol=1e-12)
     assert_fd(lambda t: O.softmax_ce(t, labels)[0], z, dz)

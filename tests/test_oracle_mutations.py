@@ -122,6 +122,37 @@ def attention_bwd_no_rowsum(cache, dout, d, heads):
     return np.concatenate([merge(dq), merge(dk), merge(dv)], -1).reshape(B, L, 1, 3 * d)
 
 
+def conv_stride2_late(x, w, b, stride, pad):
+    """Stride-2 windows start one pixel late in both directions."""
+    if stride == 2:
+        x = np.concatenate([x[:, 1:], np.zeros_like(x[:, :1])], 1)
+        x = np.concatenate([x[:, :, 1:], np.zeros_like(x[:, :, :1])], 2)
+    return ORIG["conv_fwd"](x, w, b, stride, pad)
+
+
+def maxpool_fwd_average(x):
+    return 0.25 * (x[:, 0::2, 0::2] + x[:, 0::2, 1::2] + x[:, 1::2, 0::2] + x[:, 1::2, 1::2])
+
+
+def affine_shift_first(x, scale, shift):
+    return (x + shift) * scale
+
+
+def avgpool_sum(x):
+    return x.sum(axis=(1, 2))
+
+
+def ce_unstabilised(z, labels):
+    B = z.shape[0]
+    with np.errstate(over="ignore", invalid="ignore"):
+        e = np.exp(z)
+        se = e.sum(-1, keepdims=True)
+        loss = float(np.mean(np.log(se[:, 0]) - z[np.arange(B), labels]))
+        dz = e / se
+    dz[np.arange(B), labels] -= 1.0
+    return loss, dz / B
+
+
 def layernorm_eps_on_std(x, gamma, beta):
     mu = x.mean(-1, keepdims=True)
     var = ((x - mu) ** 2).mean(-1, keepdims=True)
@@ -435,6 +466,16 @@ MUTATIONS = {
         {"attention_fwd": attention_unmasked}, [(TL.test_attention_special_cases, ())]),
     "attention backward: softmax row-sum term dropped": (
         {"attention_bwd": attention_bwd_no_rowsum}, [(TL.test_attention_fd, ())]),
+    "conv forward: stride-2 windows one pixel late": (
+        {"conv_fwd": conv_stride2_late}, [(TL.test_conv_fwd_matches_brute_force, (3, 2))]),
+    "max-pool forward: the window average instead of its maximum": (
+        {"maxpool2_fwd": maxpool_fwd_average}, [(TL.test_maxpool_brute_force_and_fd, ())]),
+    "affine forward: shift added before the scale": (
+        {"affine_fwd": affine_shift_first}, [(TL.test_affine_and_linear_fd, ())]),
+    "average pool forward: the sum, not the mean": (
+        {"avgpool_fwd": avgpool_sum}, [(TL.test_avgpool_and_flatten, ())]),
+    "cross-entropy: softmax without subtracting the row maximum": (
+        {"softmax_ce": ce_unstabilised}, [(TL.test_ce_fd_and_shift_invariance, ())]),
     "layernorm: eps added to the standard deviation": (
         {"layernorm_fwd": layernorm_eps_on_std}, [(TL.test_layernorm_invariants_and_fd, ())]),
     "GELU backward: the x phi(x) term dropped": (
