@@ -122,6 +122,24 @@ def attention_bwd_no_rowsum(cache, dout, d, heads):
     return np.concatenate([merge(dq), merge(dk), merge(dv)], -1).reshape(B, L, 1, 3 * d)
 
 
+def dwconv_stride2_late(x, w, b, stride, pad):
+    """Stride-2 depthwise windows start one pixel late in both directions."""
+    if stride == 2:
+        x = np.concatenate([x[:, 1:], np.zeros_like(x[:, :1])], 1)
+        x = np.concatenate([x[:, :, 1:], np.zeros_like(x[:, :, :1])], 2)
+    return ORIG["dwconv_fwd"](x, w, b, stride, pad)
+
+
+def hswish_bwd_half_slope(x, dy):
+    return dy * np.where(x < -3.0, 0.0, np.where(x > 3.0, 1.0, (x + 3.0) / 6.0))
+
+
+def dwconv_bwd_dx_unflipped(x, w, dy, stride, pad, need_dx):
+    """The input gradient correlates with the filter instead of its flip."""
+    dx, dw, db = ORIG["dwconv_bwd"](x, w[:, ::-1, ::-1].copy(), dy, stride, pad, need_dx)
+    return dx, ORIG["dwconv_bwd"](x, w, dy, stride, pad, False)[1], db
+
+
 def conv_stride2_late(x, w, b, stride, pad):
     """Stride-2 windows start one pixel late in both directions."""
     if stride == 2:
@@ -466,6 +484,12 @@ MUTATIONS = {
         {"attention_fwd": attention_unmasked}, [(TL.test_attention_special_cases, ())]),
     "attention backward: softmax row-sum term dropped": (
         {"attention_bwd": attention_bwd_no_rowsum}, [(TL.test_attention_fd, ())]),
+    "depthwise conv: stride-2 windows one pixel late": (
+        {"dwconv_fwd": dwconv_stride2_late}, [(TM.test_depthwise_is_a_block_diagonal_convolution, (3, 2))]),
+    "depthwise conv backward: input gradient through the unflipped filter": (
+        {"dwconv_bwd": dwconv_bwd_dx_unflipped}, [(TM.test_depthwise_is_a_block_diagonal_convolution, (3, 1))]),
+    "hard swish derivative (x + 3) / 6 between the kinks": (
+        {"hswish_bwd": hswish_bwd_half_slope}, [(TM.test_hard_swish_and_sigmoid_values, ())]),
     "conv forward: stride-2 windows one pixel late": (
         {"conv_fwd": conv_stride2_late}, [(TL.test_conv_fwd_matches_brute_force, (3, 2))]),
     "max-pool forward: the window average instead of its maximum": (
